@@ -1,0 +1,195 @@
+/*
+ * lx.h -- C ABI of the GB300 (sm_103a) LorExperts / BTExperts compressed-MoE
+ * forward (arXiv 2608.07814).
+ *
+ * The layer (Sec. 3.1 "Representation", Sec. 5 "BTExperts") is a node table:
+ *   - an ANCHOR node (parent -1, rank 0) stores full SwiGLU matrices
+ *       gate [I][H], up [I][H], down [H][I]      (nn.Linear [out][in] row-major,
+ *     the paper's W_e in R^{I x H} applied as x W^T, Sec. 2 and Sec. 5.1);
+ *   - a CORRECTION node (parent >= 0, rank r > 0) stores, per projection, the
+ *     factors of W_m ~ W_dom + B_m A_m (Sec. 3.1) as U = B_m [out][r] and
+ *     V = A_m^T [in][r]:  Ug [I][r], Vg [H][r], Uu [I][r], Vu [H][r],
+ *     Ud [H][r], Vd [I][r]   (row-major);
+ *   - expert e is the sum of the contributions on the root path of
+ *     expert_node[e]:  W_e = W_anchor + sum_{corrections n on the path} U_n V_n^T.
+ * Flat LorExperts: one anchor per cluster (the dominant maps to it, so it
+ * carries no correction) and one rank-r child per member; a protection-set
+ * singleton is an anchor without children.  BTExperts: anchors are tree roots
+ * (which need not be experts), corrections at any depth <= LX_MAX_DEPTH - 1.
+ *
+ * The forward (Sec. 5.1, "computed once per token and broadcast") routes every
+ * token top-k over all E experts with the unchanged router (Sec. 1, Fig. 1),
+ * evaluates each anchor's product once per (token, anchor) and each correction
+ * once per (token, node), applies SwiGLU per selected expert and combines
+ * y_t = sum_s g_{t,s} W_{e_s}^down act_{t,s}, using linearity so that the
+ * down-projection of shared nodes is also evaluated once per (token, node).
+ *
+ * Conventions for every call:
+ *   - All device pointers are caller-owned CUDA device memory of the current
+ *     device; host pointers are only read during the call.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).
+ *     Work is enqueued on it; no call synchronises the host except
+ *     lx_load_compressed_layer, lx_reserve (and a forward that has to grow its
+ *     workspace), lx_layer_info's row count and lx_read_profile.
+ *   - Errors are returned as lx_status; lx_last_error() gives a message for the
+ *     calling thread.  Arguments are validated on the host before any launch;
+ *     an invalid call launches nothing.  T == 0 is a valid no-op.
+ *   - A layer may be used from one host thread at a time.
+ */
+#ifndef LX_H_
+#define LX_H_
+
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define LX_API __attribute__((visibility("default")))
+#else
+#define LX_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define LX_MAX_DEPTH 4   /* nodes on a root path, anchor included */
+#define LX_MAX_K 32      /* router top-k */
+#define LX_MAX_EXPERTS 1024
+
+typedef enum {
+  LX_OK = 0,
+  LX_ERR_ARG = 1,          /* null pointer, k out of range, bad option */
+  LX_ERR_SHAPE = 2,        /* inconsistent or unsupported sizes / node table */
+  LX_ERR_CUDA = 3,         /* a CUDA runtime call failed */
+  LX_ERR_OOM = 4,          /* device allocation failed */
+  LX_ERR_TIMEOUT = 5,      /* a bounded device-side wait gave up */
+  LX_ERR_STATE = 6,        /* call out of order (e.g. buckets before a forward) */
+  LX_ERR_UNSUPPORTED = 7   /* valid request the library does not implement */
+} lx_status;
+
+typedef enum { LX_F32 = 0, LX_BF16 = 1 } lx_dtype;
+
+typedef struct lx_layer lx_layer; /* opaque, library-owned */
+
+typedef struct {
+  int32_t d_model;            /* H */
+  int32_t d_ff;               /* I */
+  int32_t n_experts;          /* E, 1..LX_MAX_EXPERTS */
+  int32_t n_nodes;            /* >= 1 */
+  int32_t dtype;              /* lx_dtype of weights, x and y */
+  const int32_t* node_parent; /* host [n_nodes]: -1 for an anchor, else parent id */
+  const int32_t* node_rank;   /* host [n_nodes]: 0 for an anchor, 1..min(I,H) else */
+  const int32_t* expert_node; /* host [n_experts]: node defining expert e */
+} lx_layer_desc;
+
+/*
+ * Load ("install", Sec. 3.2 Stage 3 iii) a compressed layer.
+ *   node_w:      host array of 6*n_nodes host pointers.  For an anchor n:
+ *                node_w[6n+0..2] = gate, up, down; node_w[6n+3..5] unused.
+ *                For a correction n: node_w[6n+0..5] = Ug, Vg, Uu, Vu, Ud, Vd.
+ *                Element type = desc->dtype (bf16 as uint16 bit patterns).
+ *   router_w:    host [E][H] (desc->dtype).
+ *   router_bias: host [E] fp32 added to the logits, or NULL.
+ * Copies (and repacks) everything to device memory owned by the layer;
+ * synchronises `stream`.  Errors: LX_ERR_ARG (null pointers), LX_ERR_SHAPE
+ * (sizes, cycles, depth > LX_MAX_DEPTH, anchor with rank != 0, correction rank
+ * outside 1..min(I,H), H or I not a multiple of 8), LX_ERR_OOM, LX_ERR_CUDA.
+ */
+LX_API lx_status lx_load_compressed_layer(const lx_layer_desc* desc, const void* const* node_w,
+                                   const void* router_w, const float* router_bias,
+                                   void* stream, lx_layer** out);
+
+/* Releases all device memory of the layer (synchronises the device first). */
+LX_API lx_status lx_free_layer(lx_layer* layer);
+
+/*
+ * Pre-sizes the layer's device workspace for up to max_tokens tokens with
+ * top-k (synchronous).  A forward with more tokens grows the workspace itself
+ * (and then synchronises its stream once).
+ */
+LX_API lx_status lx_reserve(lx_layer* layer, int32_t max_tokens, int32_t k);
+
+/*
+ * Router (Sec. 1, Fig. 1): logits l = x W_r^T (+ bias) in the canonical fp32
+ * order (H in chunks of 8; lane j = chunk mod 32 accumulates its chunks with
+ * fused multiply-adds in ascending h; the 32 partials are added pairwise at
+ * offsets 16, 8, 4, 2, 1; then the bias), top-k by (logit desc, id asc),
+ * gates = softmax over the k selected logits (fp32).
+ *   x:       device [T][H] (layer dtype)
+ *   topk_id: device [T][k] int32 out;  topk_w: device [T][k] fp32 out
+ *   logits:  device [T][E] fp32 out, or NULL
+ * Also leaves the routing in the layer for lx_bucket / lx_get_buckets.
+ * Errors: LX_ERR_ARG (k < 1, k > min(E, LX_MAX_K), T < 0, null pointers).
+ */
+LX_API lx_status lx_route(lx_layer* layer, const void* x, int32_t T, int32_t k, int32_t* topk_id,
+                   float* topk_w, float* logits, void* stream);
+
+/*
+ * Bucketing of given assignments (device [T][k] int32 expert ids, each row
+ * holding k distinct ids in [0, E)): per node the ascending list of tokens
+ * whose selected experts' root paths contain the node, per (assignment, path
+ * level) the row of that (token, node) pair, and per expert its assignments in
+ * ascending token order.  Results stay in the layer (lx_get_buckets).
+ */
+LX_API lx_status lx_bucket(lx_layer* layer, const int32_t* topk_id, int32_t T, int32_t k,
+                    void* stream);
+
+/*
+ * The compressed-MoE forward: route, bucket, shared anchor GEMMs with the
+ * low-rank corrections and SwiGLU, down-projection and weighted combine.
+ *   x: device [T][H], y: device [T][H] (layer dtype); y may not alias x.
+ */
+LX_API lx_status lx_moe_forward(lx_layer* layer, const void* x, int32_t T, int32_t k, void* y,
+                         void* stream);
+
+/*
+ * Copies the last bucketing (from lx_bucket, lx_route or lx_moe_forward) into
+ * caller device buffers (stream-ordered).  With D = info.max_depth:
+ *   node_off   [n_nodes+1]  exclusive prefix of the node bucket sizes
+ *   node_tok   [T*k*D]      capacity; first node_off[n_nodes] entries written:
+ *                           node n's tokens ascending, nodes in id order
+ *   node_row   [T*k*D]      row of (t, path(e)[l]) for assignment a = t*k+s at
+ *                           index a*D + l, -1 beyond the path's end
+ *   expert_off [E+1]        exclusive prefix of the per-expert firing counts N_e
+ *   perm       [T*k]        assignments a = t*k+s ordered by (expert, token)
+ * Any pointer may be NULL (that output is skipped).  LX_ERR_STATE if nothing
+ * has been bucketed yet.
+ */
+LX_API lx_status lx_get_buckets(lx_layer* layer, int32_t* node_off, int32_t* node_tok,
+                         int32_t* node_row, int32_t* expert_off, int32_t* perm, void* stream);
+
+typedef struct {
+  int32_t d_model, d_ff, n_experts, n_nodes, dtype;
+  int32_t n_anchors, n_corrections, max_depth, max_rank;
+  int64_t weight_bytes;       /* device bytes of the repacked weights + router */
+  int32_t last_T, last_k;     /* sizes of the last bucketing (0 if none) */
+  int32_t last_rows;          /* node_off[n_nodes] of the last bucketing (synchronises) */
+} lx_layer_info_t;
+
+LX_API lx_status lx_layer_info(lx_layer* layer, lx_layer_info_t* info);
+
+/* Execution paths.  LX_PATH_AUTO picks the fastest kernels that support the
+ * layer and batch; LX_PATH_GENERIC forces the plain CUDA-core kernels (every
+ * dtype and shape). */
+typedef enum { LX_PATH_AUTO = 0, LX_PATH_GENERIC = 1 } lx_path;
+LX_API lx_status lx_set_path(lx_layer* layer, int32_t path);
+
+/*
+ * Kernel timing.  While enabled, every kernel the layer launches is bracketed by
+ * CUDA events on its stream.  lx_read_profile synchronises on the last event,
+ * writes up to `cap` records of the launches since the previous read (oldest
+ * first) and clears the list; *n receives the number written.
+ */
+typedef struct {
+  const char* name;  /* static string */
+  float ms;          /* device time between the bracketing events */
+} lx_kernel_time;
+LX_API lx_status lx_set_profiling(lx_layer* layer, int32_t enable);
+LX_API lx_status lx_read_profile(lx_layer* layer, lx_kernel_time* out, int32_t cap, int32_t* n);
+
+/* Message of the last failed call on this thread ("" if none). */
+LX_API const char* lx_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* LX_H_ */

@@ -1,0 +1,494 @@
+// C ABI of liblx: validation, layer installation (Sec. 3.2 Stage 3 iii),
+// workspace management, profiling and the forward's orchestration.
+#include <algorithm>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "lx_internal.cuh"
+
+namespace lx {
+
+static thread_local std::string g_last_error;
+
+lx_status fail(lx_status s, const std::string& msg) {
+  g_last_error = msg;
+  return s;
+}
+
+lx_status cuda_fail(cudaError_t e, const char* what) {
+  g_last_error = std::string(what) + ": " + cudaGetErrorString(e);
+  return e == cudaErrorMemoryAllocation ? LX_ERR_OOM : LX_ERR_CUDA;
+}
+
+static size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+// ---------------------------------------------------------------------------
+// profiling
+// ---------------------------------------------------------------------------
+static cudaEvent_t take_event(lx_layer* L) {
+  if (!L->event_pool.empty()) {
+    cudaEvent_t e = L->event_pool.back();
+    L->event_pool.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+  return e;
+}
+
+ProfScope::ProfScope(lx_layer* L_, cudaStream_t s_, const char* n) : L(L_), s(s_), name(n) {
+  if (L->profiling) {
+    b = take_event(L);
+    if (b) cudaEventRecord(b, s);
+  }
+}
+
+ProfScope::~ProfScope() {
+  if (L->profiling && b) {
+    cudaEvent_t e = take_event(L);
+    if (e) {
+      cudaEventRecord(e, s);
+      L->prof.push_back(ProfRec{name, b, e});
+    } else {
+      L->event_pool.push_back(b);
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// op shapes of the generic grouped GEMMs
+// ---------------------------------------------------------------------------
+OpShape op_shape(const lx_layer* L, int op) {
+  switch (op) {
+    case OP_UP_ANCHOR: return OpShape{2 * L->I, 0, L->H, 0, 1, 1};
+    case OP_UP_V:      return OpShape{0, 2, L->H, 0, 1, 0};
+    case OP_UP_U:      return OpShape{L->I, 0, 0, 1, 2, 0};
+    case OP_DN_ANCHOR: return OpShape{L->H, 0, L->I, 0, 1, 1};
+    case OP_DN_V:      return OpShape{0, 1, L->I, 0, 1, 0};
+    default:           return OpShape{L->H, 0, 0, 1, 1, 0};  // OP_DN_U
+  }
+}
+
+int op_max_items(const lx_layer* L) { return std::max(L->n_anchor, L->n_corr); }
+
+// ---------------------------------------------------------------------------
+// workspace
+// ---------------------------------------------------------------------------
+static lx_status ensure_workspace(lx_layer* L, int T, int k, cudaStream_t s) {
+  Workspace& w = L->ws;
+  if (T <= w.cap_T && k <= w.cap_k) return LX_OK;
+  const int cT = std::max(T, w.cap_T), ck = std::max(k, w.cap_k);
+  const long Tp = align_up((size_t)cT, 16);
+  const long D = L->max_depth;
+  const long keys = (long)L->N + L->E;
+  const long Rmax = std::max<long>(1, (long)cT * std::min<long>(L->N, (long)ck * D));
+  const long rmax = std::max(1, L->max_rank);
+  struct Item { void** p; size_t bytes; };
+  std::vector<Item> items = {
+      {(void**)&w.logits, sizeof(float) * cT * L->E},
+      {(void**)&w.topk_id, sizeof(int) * cT * ck},
+      {(void**)&w.topk_w, sizeof(float) * cT * ck},
+      {(void**)&w.marks, (size_t)keys * Tp},
+      {(void**)&w.rank_in, sizeof(int) * keys * Tp},
+      {(void**)&w.key_cnt, sizeof(int) * keys},
+      {(void**)&w.key_off, sizeof(int) * (keys + 2)},
+      {(void**)&w.node_tok, sizeof(int) * cT * ck * D},
+      {(void**)&w.row_node, sizeof(int) * cT * ck * D},
+      {(void**)&w.node_row, sizeof(int) * cT * ck * D},
+      {(void**)&w.perm, sizeof(int) * cT * ck},
+      {(void**)&w.tile_off, sizeof(int) * N_OPS * (op_max_items(L) + 1)},
+      {(void**)&w.h, sizeof(float) * Rmax * 2 * L->I},
+      {(void**)&w.P, sizeof(float) * Rmax * 2 * rmax},
+      {(void**)&w.z, sizeof(float) * Rmax * L->I},
+      {(void**)&w.Q, sizeof(float) * Rmax * rmax},
+      {(void**)&w.ypart, sizeof(float) * Rmax * L->H},
+  };
+  size_t total = 0;
+  for (auto& it : items) total += align_up(it.bytes, 256);
+  if (w.base) {
+    LX_CUDA(cudaStreamSynchronize(s));
+    LX_CUDA(cudaFree(w.base));
+    w.base = nullptr;
+  }
+  void* base = nullptr;
+  cudaError_t e = cudaMalloc(&base, total);
+  if (e != cudaSuccess) {
+    w.cap_T = w.cap_k = 0;
+    return cuda_fail(e, "cudaMalloc(workspace)");
+  }
+  size_t off = 0;
+  for (auto& it : items) {
+    *it.p = (char*)base + off;
+    off += align_up(it.bytes, 256);
+  }
+  w.base = base;
+  w.bytes = total;
+  w.cap_T = cT;
+  w.cap_k = ck;
+  L->last_T = L->last_k = 0;
+  return LX_OK;
+}
+
+static lx_status check_call(lx_layer* L, int T, int k) {
+  if (!L) return fail(LX_ERR_ARG, "layer is NULL");
+  if (T < 0) return fail(LX_ERR_ARG, "T < 0");
+  if (k < 1 || k > LX_MAX_K || k > L->E)
+    return fail(LX_ERR_ARG, "k must be in 1..min(E, LX_MAX_K)");
+  if ((long)T * k * L->max_depth > (1L << 30)) return fail(LX_ERR_SHAPE, "T*k too large");
+  return LX_OK;
+}
+
+}  // namespace lx
+
+using namespace lx;
+
+// ---------------------------------------------------------------------------
+// load
+// ---------------------------------------------------------------------------
+static lx_status validate_desc(const lx_layer_desc* d, const void* const* node_w,
+                               const void* router_w) {
+  if (!d || !node_w || !router_w) return fail(LX_ERR_ARG, "NULL descriptor/weights/router");
+  if (!d->node_parent || !d->node_rank || !d->expert_node)
+    return fail(LX_ERR_ARG, "NULL node table");
+  if (d->dtype != LX_F32 && d->dtype != LX_BF16) return fail(LX_ERR_ARG, "unknown dtype");
+  const long H = d->d_model, I = d->d_ff, E = d->n_experts, N = d->n_nodes;
+  if (H < 8 || I < 8 || H % 8 || I % 8)
+    return fail(LX_ERR_SHAPE, "d_model and d_ff must be positive multiples of 8");
+  if (H > 65536 || I > 65536) return fail(LX_ERR_SHAPE, "d_model/d_ff above 65536");
+  if (E < 1 || E > LX_MAX_EXPERTS) return fail(LX_ERR_SHAPE, "n_experts outside 1..1024");
+  if (N < 1 || N > 4096) return fail(LX_ERR_SHAPE, "n_nodes outside 1..4096");
+  for (long n = 0; n < N; ++n) {
+    const int p = d->node_parent[n], r = d->node_rank[n];
+    if (p < -1 || p >= N || p == n) return fail(LX_ERR_SHAPE, "bad node_parent");
+    if (p == -1 && r != 0) return fail(LX_ERR_SHAPE, "anchor node with rank != 0");
+    if (p >= 0 && (r < 1 || r > std::min(H, I)))
+      return fail(LX_ERR_SHAPE, "correction rank outside 1..min(d_model, d_ff)");
+    const int nw = p == -1 ? 3 : 6;
+    for (int j = 0; j < nw; ++j)
+      if (!node_w[6 * n + j]) return fail(LX_ERR_ARG, "NULL node weight pointer");
+    // root path must reach an anchor within LX_MAX_DEPTH nodes (no cycles)
+    long m = n;
+    int depth = 1;
+    while (d->node_parent[m] >= 0) {
+      m = d->node_parent[m];
+      if (++depth > LX_MAX_DEPTH) return fail(LX_ERR_SHAPE, "node path deeper than LX_MAX_DEPTH or cyclic");
+    }
+  }
+  for (long e = 0; e < E; ++e)
+    if (d->expert_node[e] < 0 || d->expert_node[e] >= N)
+      return fail(LX_ERR_SHAPE, "expert_node out of range");
+  return LX_OK;
+}
+
+// dst[c][r] = src[r][c] for a [rows][cols] matrix of esz-byte elements
+static void transpose_bytes(const void* src, void* dst, long rows, long cols, int esz) {
+  const char* s = (const char*)src;
+  char* o = (char*)dst;
+  for (long r = 0; r < rows; ++r)
+    for (long c = 0; c < cols; ++c) std::memcpy(o + (c * rows + r) * esz, s + (r * cols + c) * esz, esz);
+}
+
+extern "C" lx_status lx_load_compressed_layer(const lx_layer_desc* d, const void* const* node_w,
+                                              const void* router_w, const float* router_bias,
+                                              void* stream, lx_layer** out) {
+  if (!out) return fail(LX_ERR_ARG, "out is NULL");
+  *out = nullptr;
+  LX_TRY(validate_desc(d, node_w, router_w));
+  cudaStream_t s = (cudaStream_t)stream;
+  lx_layer* L = new lx_layer();
+  L->H = d->d_model;
+  L->I = d->d_ff;
+  L->E = d->n_experts;
+  L->N = d->n_nodes;
+  L->dtype = d->dtype;
+  L->esz = d->dtype == LX_BF16 ? 2 : 4;
+  L->parent.assign(d->node_parent, d->node_parent + L->N);
+  L->rank.assign(d->node_rank, d->node_rank + L->N);
+  L->expert_node.assign(d->expert_node, d->expert_node + L->E);
+  for (int n = 0; n < L->N; ++n) {
+    if (L->parent[n] < 0) L->anchors.push_back(n);
+    else L->corrs.push_back(n);
+    L->max_rank = std::max(L->max_rank, L->rank[n]);
+  }
+  L->n_anchor = (int)L->anchors.size();
+  L->n_corr = (int)L->corrs.size();
+  std::vector<int> paths((size_t)L->E * LX_MAX_DEPTH, -1), plen(L->E, 0);
+  for (int e = 0; e < L->E; ++e) {
+    int n = L->expert_node[e], l = 0;
+    while (n >= 0) {
+      paths[(size_t)e * LX_MAX_DEPTH + l++] = n;
+      n = L->parent[n];
+    }
+    plen[e] = l;
+    L->max_depth = std::max(L->max_depth, l);
+  }
+  auto cleanup = [&](lx_status st) {
+    lx_free_layer(L);
+    return st;
+  };
+  cudaError_t ce = cudaGetDevice(&L->device);
+  if (ce != cudaSuccess) return cleanup(cuda_fail(ce, "cudaGetDevice"));
+  cudaDeviceGetAttribute(&L->num_sms, cudaDevAttrMultiProcessorCount, L->device);
+
+  // ---- weight arena layout
+  const long H = L->H, I = L->I, esz = L->esz;
+  struct Piece { int node; int slot; size_t off; size_t bytes; };
+  std::vector<Piece> pieces;
+  size_t off = 0;
+  auto add = [&](int node, int slot, size_t bytes) {
+    pieces.push_back(Piece{node, slot, off, bytes});
+    off += align_up(bytes, 256);
+  };
+  for (int n = 0; n < L->N; ++n) {
+    if (L->parent[n] < 0) {
+      add(n, 0, 2 * I * H * esz);  // [Wg;Wu]
+      add(n, 2, H * I * esz);      // Wd
+    } else {
+      const long r = L->rank[n];
+      add(n, 0, 2 * r * H * esz);  // [Vg^T;Vu^T]
+      add(n, 1, 2 * I * r * esz);  // [Ug;Uu]
+      add(n, 2, r * I * esz);      // Vd^T
+      add(n, 3, H * r * esz);      // Ud
+    }
+  }
+  const size_t router_off = off;
+  off += align_up((size_t)L->E * H * esz, 256);
+  const size_t bias_off = off;
+  if (router_bias) off += align_up((size_t)L->E * 4, 256);
+  L->arena_bytes = off;
+  ce = cudaMalloc(&L->arena, off);
+  if (ce != cudaSuccess) return cleanup(cuda_fail(ce, "cudaMalloc(weights)"));
+
+  L->h_w_up.assign(L->N, nullptr);
+  L->h_w_upU.assign(L->N, nullptr);
+  L->h_w_dn.assign(L->N, nullptr);
+  L->h_w_dnU.assign(L->N, nullptr);
+  std::vector<char> stage;
+  for (const Piece& p : pieces) {
+    char* dst = (char*)L->arena + p.off;
+    const int n = p.node;
+    const void* const* w = node_w + 6 * (size_t)n;
+    stage.resize(p.bytes);
+    if (L->parent[n] < 0) {
+      if (p.slot == 0) {
+        std::memcpy(stage.data(), w[0], I * H * esz);
+        std::memcpy(stage.data() + I * H * esz, w[1], I * H * esz);
+        L->h_w_up[n] = dst;
+      } else {
+        std::memcpy(stage.data(), w[2], H * I * esz);
+        L->h_w_dn[n] = dst;
+      }
+    } else {
+      const long r = L->rank[n];
+      if (p.slot == 0) {  // Vg [H][r] -> [r][H]; Vu likewise
+        transpose_bytes(w[1], stage.data(), H, r, esz);
+        transpose_bytes(w[3], stage.data() + r * H * esz, H, r, esz);
+        L->h_w_up[n] = dst;
+      } else if (p.slot == 1) {
+        std::memcpy(stage.data(), w[0], I * r * esz);
+        std::memcpy(stage.data() + I * r * esz, w[2], I * r * esz);
+        L->h_w_upU[n] = dst;
+      } else if (p.slot == 2) {  // Vd [I][r] -> [r][I]
+        transpose_bytes(w[5], stage.data(), I, r, esz);
+        L->h_w_dn[n] = dst;
+      } else {
+        std::memcpy(stage.data(), w[4], H * r * esz);
+        L->h_w_dnU[n] = dst;
+      }
+    }
+    ce = cudaMemcpyAsync(dst, stage.data(), p.bytes, cudaMemcpyHostToDevice, s);
+    if (ce == cudaSuccess) ce = cudaStreamSynchronize(s);
+    if (ce != cudaSuccess) return cleanup(cuda_fail(ce, "copy weights"));
+  }
+  L->router_w = (char*)L->arena + router_off;
+  ce = cudaMemcpyAsync(L->router_w, router_w, (size_t)L->E * H * esz, cudaMemcpyHostToDevice, s);
+  if (ce == cudaSuccess && router_bias) {
+    L->router_bias = (float*)((char*)L->arena + bias_off);
+    ce = cudaMemcpyAsync(L->router_bias, router_bias, (size_t)L->E * 4, cudaMemcpyHostToDevice, s);
+  }
+  if (ce != cudaSuccess) return cleanup(cuda_fail(ce, "copy router"));
+
+  // ---- small device tables
+  const size_t nptr = (size_t)L->N;
+  size_t toff = 0;
+  auto tadd = [&](size_t bytes) {
+    size_t o = toff;
+    toff += align_up(bytes, 256);
+    return o;
+  };
+  const size_t o_rank = tadd(4 * L->N), o_paths = tadd(4 * paths.size()), o_plen = tadd(4 * L->E);
+  const size_t o_anc = tadd(4 * std::max(1, L->n_anchor)), o_cor = tadd(4 * std::max(1, L->n_corr));
+  const size_t o_p0 = tadd(sizeof(void*) * nptr), o_p1 = tadd(sizeof(void*) * nptr);
+  const size_t o_p2 = tadd(sizeof(void*) * nptr), o_p3 = tadd(sizeof(void*) * nptr);
+  std::vector<char> tb(toff, 0);
+  std::memcpy(tb.data() + o_rank, L->rank.data(), 4 * L->N);
+  std::memcpy(tb.data() + o_paths, paths.data(), 4 * paths.size());
+  std::memcpy(tb.data() + o_plen, plen.data(), 4 * L->E);
+  if (L->n_anchor) std::memcpy(tb.data() + o_anc, L->anchors.data(), 4 * L->n_anchor);
+  if (L->n_corr) std::memcpy(tb.data() + o_cor, L->corrs.data(), 4 * L->n_corr);
+  std::memcpy(tb.data() + o_p0, L->h_w_up.data(), sizeof(void*) * nptr);
+  std::memcpy(tb.data() + o_p1, L->h_w_upU.data(), sizeof(void*) * nptr);
+  std::memcpy(tb.data() + o_p2, L->h_w_dn.data(), sizeof(void*) * nptr);
+  std::memcpy(tb.data() + o_p3, L->h_w_dnU.data(), sizeof(void*) * nptr);
+  ce = cudaMalloc(&L->tables, toff);
+  if (ce != cudaSuccess) return cleanup(cuda_fail(ce, "cudaMalloc(tables)"));
+  char* tbase = (char*)L->tables;
+  L->d_rank = (int*)(tbase + o_rank);
+  L->d_paths = (int*)(tbase + o_paths);
+  L->d_path_len = (int*)(tbase + o_plen);
+  L->d_anchors = (int*)(tbase + o_anc);
+  L->d_corrs = (int*)(tbase + o_cor);
+  L->d_w_up = (const void**)(tbase + o_p0);
+  L->d_w_upU = (const void**)(tbase + o_p1);
+  L->d_w_dn = (const void**)(tbase + o_p2);
+  L->d_w_dnU = (const void**)(tbase + o_p3);
+  ce = cudaMemcpyAsync(L->tables, tb.data(), toff, cudaMemcpyHostToDevice, s);
+  if (ce == cudaSuccess) ce = cudaStreamSynchronize(s);
+  if (ce != cudaSuccess) return cleanup(cuda_fail(ce, "copy tables"));
+  *out = L;
+  return LX_OK;
+}
+
+extern "C" lx_status lx_free_layer(lx_layer* L) {
+  if (!L) return fail(LX_ERR_ARG, "layer is NULL");
+  cudaDeviceSynchronize();
+  for (auto& r : L->prof) {
+    cudaEventDestroy(r.a);
+    cudaEventDestroy(r.b);
+  }
+  for (auto e : L->event_pool) cudaEventDestroy(e);
+  if (L->ws.base) cudaFree(L->ws.base);
+  if (L->arena) cudaFree(L->arena);
+  if (L->tables) cudaFree(L->tables);
+  delete L;
+  return LX_OK;
+}
+
+extern "C" lx_status lx_reserve(lx_layer* L, int32_t max_tokens, int32_t k) {
+  LX_TRY(check_call(L, max_tokens, k));
+  LX_TRY(ensure_workspace(L, std::max(1, max_tokens), k, nullptr));
+  LX_CUDA(cudaDeviceSynchronize());
+  return LX_OK;
+}
+
+extern "C" lx_status lx_route(lx_layer* L, const void* x, int32_t T, int32_t k, int32_t* topk_id,
+                              float* topk_w, float* logits, void* stream) {
+  LX_TRY(check_call(L, T, k));
+  if (T == 0) return LX_OK;
+  if (!x || !topk_id || !topk_w) return fail(LX_ERR_ARG, "NULL x/topk_id/topk_w");
+  cudaStream_t s = (cudaStream_t)stream;
+  LX_TRY(ensure_workspace(L, T, k, s));
+  LX_TRY(launch_router(L, x, T, k, topk_id, topk_w, logits, s));
+  LX_TRY(launch_bucket(L, topk_id, T, k, s));
+  L->last_T = T;
+  L->last_k = k;
+  return LX_OK;
+}
+
+extern "C" lx_status lx_bucket(lx_layer* L, const int32_t* topk_id, int32_t T, int32_t k,
+                               void* stream) {
+  LX_TRY(check_call(L, T, k));
+  if (T == 0) return LX_OK;
+  if (!topk_id) return fail(LX_ERR_ARG, "NULL topk_id");
+  cudaStream_t s = (cudaStream_t)stream;
+  LX_TRY(ensure_workspace(L, T, k, s));
+  LX_TRY(launch_bucket(L, topk_id, T, k, s));
+  L->last_T = T;
+  L->last_k = k;
+  return LX_OK;
+}
+
+extern "C" lx_status lx_moe_forward(lx_layer* L, const void* x, int32_t T, int32_t k, void* y,
+                                    void* stream) {
+  LX_TRY(check_call(L, T, k));
+  if (T == 0) return LX_OK;
+  if (!x || !y) return fail(LX_ERR_ARG, "NULL x/y");
+  if (x == y) return fail(LX_ERR_ARG, "y may not alias x");
+  cudaStream_t s = (cudaStream_t)stream;
+  LX_TRY(ensure_workspace(L, T, k, s));
+  Workspace& w = L->ws;
+  LX_TRY(launch_router(L, x, T, k, w.topk_id, w.topk_w, nullptr, s));
+  LX_TRY(launch_bucket(L, w.topk_id, T, k, s));
+  L->last_T = T;
+  L->last_k = k;
+  LX_TRY(launch_generic_experts(L, x, T, k, y, s));
+  return LX_OK;
+}
+
+extern "C" lx_status lx_get_buckets(lx_layer* L, int32_t* node_off, int32_t* node_tok,
+                                    int32_t* node_row, int32_t* expert_off, int32_t* perm,
+                                    void* stream) {
+  if (!L) return fail(LX_ERR_ARG, "layer is NULL");
+  if (L->last_T == 0) return fail(LX_ERR_STATE, "nothing bucketed yet");
+  cudaStream_t s = (cudaStream_t)stream;
+  const Workspace& w = L->ws;
+  const long T = L->last_T, k = L->last_k, D = L->max_depth;
+  if (node_off)
+    LX_CUDA(cudaMemcpyAsync(node_off, w.key_off, 4 * (L->N + 1), cudaMemcpyDeviceToDevice, s));
+  if (expert_off)
+    LX_CUDA(cudaMemcpyAsync(expert_off, w.key_off + L->N + 1, 4 * (L->E + 1),
+                            cudaMemcpyDeviceToDevice, s));
+  if (node_tok)
+    LX_CUDA(cudaMemcpyAsync(node_tok, w.node_tok, 4 * T * k * D, cudaMemcpyDeviceToDevice, s));
+  if (node_row)
+    LX_CUDA(cudaMemcpyAsync(node_row, w.node_row, 4 * T * k * D, cudaMemcpyDeviceToDevice, s));
+  if (perm) LX_CUDA(cudaMemcpyAsync(perm, w.perm, 4 * T * k, cudaMemcpyDeviceToDevice, s));
+  return LX_OK;
+}
+
+extern "C" lx_status lx_layer_info(lx_layer* L, lx_layer_info_t* info) {
+  if (!L || !info) return fail(LX_ERR_ARG, "NULL argument");
+  info->d_model = L->H;
+  info->d_ff = L->I;
+  info->n_experts = L->E;
+  info->n_nodes = L->N;
+  info->dtype = L->dtype;
+  info->n_anchors = L->n_anchor;
+  info->n_corrections = L->n_corr;
+  info->max_depth = L->max_depth;
+  info->max_rank = L->max_rank;
+  info->weight_bytes = (int64_t)L->arena_bytes;
+  info->last_T = L->last_T;
+  info->last_k = L->last_k;
+  info->last_rows = 0;
+  if (L->last_T > 0) {
+    int rows = 0;
+    LX_CUDA(cudaDeviceSynchronize());
+    LX_CUDA(cudaMemcpy(&rows, L->ws.key_off + L->N, 4, cudaMemcpyDeviceToHost));
+    info->last_rows = rows;
+  }
+  return LX_OK;
+}
+
+extern "C" lx_status lx_set_path(lx_layer* L, int32_t path) {
+  if (!L) return fail(LX_ERR_ARG, "layer is NULL");
+  if (path != LX_PATH_AUTO && path != LX_PATH_GENERIC) return fail(LX_ERR_ARG, "unknown path");
+  L->path_mode = path;
+  return LX_OK;
+}
+
+extern "C" lx_status lx_set_profiling(lx_layer* L, int32_t enable) {
+  if (!L) return fail(LX_ERR_ARG, "layer is NULL");
+  L->profiling = enable != 0;
+  return LX_OK;
+}
+
+extern "C" lx_status lx_read_profile(lx_layer* L, lx_kernel_time* out, int32_t cap, int32_t* n) {
+  if (!L || !n || (cap > 0 && !out)) return fail(LX_ERR_ARG, "NULL argument");
+  *n = 0;
+  if (!L->prof.empty()) LX_CUDA(cudaEventSynchronize(L->prof.back().b));
+  int w = 0;
+  for (auto& r : L->prof) {
+    float ms = 0.f;
+    cudaEventElapsedTime(&ms, r.a, r.b);
+    if (w < cap) out[w++] = lx_kernel_time{r.name, ms};
+    L->event_pool.push_back(r.a);
+    L->event_pool.push_back(r.b);
+  }
+  L->prof.clear();
+  *n = w;
+  return LX_OK;
+}
+
+extern "C" const char* lx_last_error(void) { return g_last_error.c_str(); }

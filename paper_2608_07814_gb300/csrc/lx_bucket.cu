@@ -1,0 +1,231 @@
+// Bucketing: per node the ascending list of tokens whose selected experts' root
+// paths contain the node (the (token, node) pairs whose products the amortised
+// forward computes once, Sec. 5.1), per assignment and path level the row of
+// that pair, and per expert its assignments in token order.
+//
+// Keys are the N nodes followed by the E experts.  A byte matrix marks[key][t]
+// records which (key, token) pairs occur; one CTA per key turns its row into
+// exclusive ranks with a block scan (so the order inside a bucket is the token
+// order, with no atomics); a single CTA scans the per-key counts into offsets
+// and builds the tile plans of the grouped GEMMs; a last pass scatters.
+// Everything is deterministic.
+#include "lx_internal.cuh"
+
+namespace lx {
+
+namespace {
+
+constexpr int SCAN_THREADS = 512;
+
+__global__ void k_mark(const int* __restrict__ topk_id, int T, int k, int N, int E, long Tp,
+                       const int* __restrict__ paths, const int* __restrict__ path_len,
+                       uint8_t* __restrict__ marks) {
+  const int t = blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= T) return;
+  for (int s = 0; s < k; ++s) {
+    const int e = topk_id[(size_t)t * k + s];
+    if (e < 0 || e >= E) continue;  // invalid ids are ignored
+    marks[(size_t)(N + e) * Tp + t] = 1;
+    const int len = path_len[e];
+    for (int l = 0; l < len; ++l) marks[(size_t)paths[e * LX_MAX_DEPTH + l] * Tp + t] = 1;
+  }
+}
+
+// block-wide exclusive scan of one int per thread; returns the block total
+__device__ int block_excl_scan(int v, int* total) {
+  __shared__ int warp_sums[32];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  int incl = v;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const int o = __shfl_up_sync(0xffffffffu, incl, off);
+    if (lane >= off) incl += o;
+  }
+  if (lane == 31) warp_sums[warp] = incl;
+  __syncthreads();
+  if (warp == 0) {
+    int ws = lane < nw ? warp_sums[lane] : 0;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const int o = __shfl_up_sync(0xffffffffu, ws, off);
+      if (lane >= off) ws += o;
+    }
+    if (lane < nw) warp_sums[lane] = ws;  // inclusive
+  }
+  __syncthreads();
+  const int warp_base = warp > 0 ? warp_sums[warp - 1] : 0;
+  *total = warp_sums[nw - 1];
+  __syncthreads();
+  return warp_base + incl - v;
+}
+
+__global__ void __launch_bounds__(SCAN_THREADS)
+k_key_scan(const uint8_t* __restrict__ marks, int T, long Tp, int* __restrict__ rank_in,
+           int* __restrict__ key_cnt) {
+  const int key = blockIdx.x;
+  const uint8_t* m = marks + (size_t)key * Tp;
+  int* r = rank_in + (size_t)key * Tp;
+  int running = 0;
+  for (int base = 0; base < T; base += blockDim.x * 4) {
+    const int i0 = base + threadIdx.x * 4;
+    int v[4], c = 0;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      v[j] = (i0 + j < T) ? m[i0 + j] : 0;
+      c += v[j];
+    }
+    int total;
+    int run = running + block_excl_scan(c, &total);
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      if (v[j]) r[i0 + j] = run++;
+    running += total;
+  }
+  if (threadIdx.x == 0) key_cnt[key] = running;
+}
+
+struct PlanArgs {
+  const int* items[N_OPS];
+  int n_items[N_OPS];
+  OpShape shape[N_OPS];
+};
+
+// one CTA: node/expert offsets and the tile prefix of every grouped-GEMM op
+__global__ void k_offsets_plan(const int* __restrict__ key_cnt, int N, int E,
+                               int* __restrict__ key_off, const int* __restrict__ rank,
+                               int* __restrict__ tile_off, int max_items, PlanArgs pa) {
+  __shared__ int total_s;
+  // node offsets then expert offsets
+  for (int part = 0; part < 2; ++part) {
+    const int n0 = part == 0 ? 0 : N, cnt = part == 0 ? N : E;
+    int* out = key_off + (part == 0 ? 0 : N + 1);
+    int carry = 0;
+    for (int base = 0; base < cnt; base += blockDim.x) {
+      const int i = base + threadIdx.x;
+      const int v = i < cnt ? key_cnt[n0 + i] : 0;
+      int total;
+      const int ex = block_excl_scan(v, &total);
+      if (i < cnt) out[i] = carry + ex;
+      carry += total;
+    }
+    if (threadIdx.x == 0) out[cnt] = carry;
+    __syncthreads();
+  }
+  (void)total_s;
+  for (int op = 0; op < N_OPS; ++op) {
+    const OpShape sh = pa.shape[op];
+    int* to = tile_off + op * (max_items + 1);
+    int carry = 0;
+    for (int base = 0; base < pa.n_items[op]; base += blockDim.x) {
+      const int i = base + threadIdx.x;
+      int v = 0;
+      if (i < pa.n_items[op]) {
+        const int n = pa.items[op][i];
+        const int r = rank[n];
+        const int Ng = sh.n_const + sh.n_rank * r;
+        const int rows = key_cnt[n];
+        v = ((rows + G_BM - 1) / G_BM) * sh.groups * ((Ng + G_BN - 1) / G_BN);
+      }
+      int total;
+      const int ex = block_excl_scan(v, &total);
+      if (i < pa.n_items[op]) to[i] = carry + ex;
+      carry += total;
+    }
+    if (threadIdx.x == 0) to[pa.n_items[op]] = carry;
+    __syncthreads();
+  }
+}
+
+__global__ void k_scatter(const uint8_t* __restrict__ marks, const int* __restrict__ rank_in,
+                          const int* __restrict__ key_off, const int* __restrict__ topk_id, int T,
+                          int k, int N, long Tp, int* __restrict__ node_tok,
+                          int* __restrict__ row_node, int* __restrict__ perm) {
+  const int key = blockIdx.y;
+  const int t = blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= T) return;
+  const size_t idx = (size_t)key * Tp + t;
+  if (!marks[idx]) return;
+  const int rk = rank_in[idx];
+  if (key < N) {
+    const int row = key_off[key] + rk;
+    node_tok[row] = t;
+    row_node[row] = key;
+  } else {
+    const int e = key - N;
+    const int pos = key_off[N + 1 + e] + rk;
+    for (int s = 0; s < k; ++s)
+      if (topk_id[(size_t)t * k + s] == e) {
+        perm[pos] = t * k + s;
+        break;
+      }
+  }
+}
+
+__global__ void k_node_row(const int* __restrict__ topk_id, int T, int k, int E, int D, long Tp,
+                           const int* __restrict__ paths, const int* __restrict__ path_len,
+                           const int* __restrict__ key_off, const int* __restrict__ rank_in,
+                           int* __restrict__ node_row) {
+  const long a = (long)blockIdx.x * blockDim.x + threadIdx.x;
+  if (a >= (long)T * k) return;
+  const int t = (int)(a / k);
+  const int e = topk_id[a];
+  const int len = (e >= 0 && e < E) ? path_len[e] : 0;
+  for (int l = 0; l < D; ++l) {
+    int row = -1;
+    if (l < len) {
+      const int n = paths[e * LX_MAX_DEPTH + l];
+      row = key_off[n] + rank_in[(size_t)n * Tp + t];
+    }
+    node_row[a * D + l] = row;
+  }
+}
+
+}  // namespace
+
+lx_status launch_bucket(lx_layer* L, const int* topk_id, int T, int k, cudaStream_t s) {
+  Workspace& w = L->ws;
+  const long Tp = (w.cap_T + 15) / 16 * 16;
+  const int keys = L->N + L->E;
+  {
+    ProfScope ps(L, s, "bucket_clear");
+    LX_CUDA(cudaMemsetAsync(w.marks, 0, (size_t)keys * Tp, s));
+  }
+  {
+    ProfScope ps(L, s, "bucket_mark");
+    k_mark<<<(T + 255) / 256, 256, 0, s>>>(topk_id, T, k, L->N, L->E, Tp, L->d_paths,
+                                           L->d_path_len, w.marks);
+    LX_CUDA(cudaGetLastError());
+  }
+  {
+    ProfScope ps(L, s, "bucket_scan");
+    k_key_scan<<<keys, SCAN_THREADS, 0, s>>>(w.marks, T, Tp, w.rank_in, w.key_cnt);
+    LX_CUDA(cudaGetLastError());
+  }
+  {
+    PlanArgs pa;
+    for (int op = 0; op < N_OPS; ++op) {
+      pa.shape[op] = op_shape(L, op);
+      pa.items[op] = pa.shape[op].on_anchors ? L->d_anchors : L->d_corrs;
+      pa.n_items[op] = pa.shape[op].on_anchors ? L->n_anchor : L->n_corr;
+    }
+    ProfScope ps(L, s, "bucket_offsets");
+    k_offsets_plan<<<1, 1024, 0, s>>>(w.key_cnt, L->N, L->E, w.key_off, L->d_rank, w.tile_off,
+                                      op_max_items(L), pa);
+    LX_CUDA(cudaGetLastError());
+  }
+  {
+    ProfScope ps(L, s, "bucket_scatter");
+    const dim3 grid((T + 255) / 256, keys);
+    k_scatter<<<grid, 256, 0, s>>>(w.marks, w.rank_in, w.key_off, topk_id, T, k, L->N, Tp,
+                                   w.node_tok, w.row_node, w.perm);
+    LX_CUDA(cudaGetLastError());
+    const long A = (long)T * k;
+    k_node_row<<<(unsigned)((A + 255) / 256), 256, 0, s>>>(topk_id, T, k, L->E, L->max_depth, Tp,
+                                                           L->d_paths, L->d_path_len, w.key_off,
+                                                           w.rank_in, w.node_row);
+    LX_CUDA(cudaGetLastError());
+  }
+  return LX_OK;
+}
+
+}  // namespace lx

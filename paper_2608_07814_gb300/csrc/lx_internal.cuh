@@ -1,0 +1,171 @@
+// Internal declarations shared by the CUDA translation units of liblx.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+#include <string>
+#include <vector>
+
+#include "../../include/lx.h"
+
+namespace lx {
+
+// ---------------------------------------------------------------------------
+// error handling
+// ---------------------------------------------------------------------------
+lx_status fail(lx_status s, const std::string& msg);
+lx_status cuda_fail(cudaError_t e, const char* what);
+
+#define LX_CUDA(call)                                              \
+  do {                                                             \
+    cudaError_t e_ = (call);                                       \
+    if (e_ != cudaSuccess) return ::lx::cuda_fail(e_, #call);      \
+  } while (0)
+
+#define LX_TRY(call)                                               \
+  do {                                                             \
+    lx_status s_ = (call);                                         \
+    if (s_ != LX_OK) return s_;                                    \
+  } while (0)
+
+// ---------------------------------------------------------------------------
+// element helpers
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ float to_f32(float v) { return v; }
+__device__ __forceinline__ float to_f32(__nv_bfloat16 v) { return __bfloat162float(v); }
+template <typename T> __device__ __forceinline__ T from_f32(float v);
+template <> __device__ __forceinline__ float from_f32<float>(float v) { return v; }
+template <> __device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(float v) {
+  return __float2bfloat16_rn(v);
+}
+
+// ---------------------------------------------------------------------------
+// grouped GEMM over node buckets (the generic CUDA-core path)
+// ---------------------------------------------------------------------------
+// Op kinds, indexing the per-op tile plans.
+enum OpKind {
+  OP_UP_ANCHOR = 0,  // h[row, 0:2I]   = x[tok] . [Wg;Wu]^T          (anchors)
+  OP_UP_V = 1,       // P[row, 0:2r]   = x[tok] . [Vg|Vu]            (corrections)
+  OP_UP_U = 2,       // h[row, gI:(g+1)I] = P[row, g r:(g+1) r] . U_g^T, g in {gate, up}
+  OP_DN_ANCHOR = 3,  // ypart[row, 0:H] = z[row] . Wd^T              (anchors)
+  OP_DN_V = 4,       // Q[row, 0:r]    = z[row] . Vd
+  OP_DN_U = 5,       // ypart[row, 0:H] = Q[row] . Ud^T
+  N_OPS = 6
+};
+
+// Per-op shape rule: for node n with rank r, each group has
+//   N_g = n_const + n_rank * r output columns and K = k_const + k_rank * r.
+struct OpShape {
+  int n_const, n_rank, k_const, k_rank, groups;
+  int on_anchors;  // 1: items are anchors; 0: corrections
+};
+
+// Generic tile sizes
+constexpr int G_BM = 32, G_BN = 64, G_BK = 32;
+
+struct GemmArgs {
+  const int* items;        // node ids [n_items]
+  int n_items;
+  const int* tile_off;     // [n_items+1] tile prefix (device, from the plan)
+  const int* node_off;     // [n_nodes+1]
+  const int* gather;       // row -> A row index (e.g. node_tok), or null = identity
+  const void* A;           // activations (f32 or layer dtype)
+  long lda;                // elements
+  const void* const* W;    // per node id: weight [groups*N_g][K] row-major
+  const int* rank;         // per node
+  OpShape shape;
+  float* out;
+  long ldo;
+};
+
+// ---------------------------------------------------------------------------
+// device workspace of one forward
+// ---------------------------------------------------------------------------
+struct Workspace {
+  int cap_T = 0, cap_k = 0;
+  void* base = nullptr;
+  size_t bytes = 0;
+  // routing
+  float* logits = nullptr;   // [T][E]
+  int* topk_id = nullptr;    // [T][k]
+  float* topk_w = nullptr;   // [T][k]
+  // bucketing
+  uint8_t* marks = nullptr;  // [(N+E)][Tp]
+  int* rank_in = nullptr;    // [(N+E)][Tp]
+  int* key_cnt = nullptr;    // [N+E]
+  int* key_off = nullptr;    // [N+1 + E+1]: node_off then expert_off
+  int* node_tok = nullptr;   // [T*k*D]
+  int* row_node = nullptr;   // [T*k*D]
+  int* node_row = nullptr;   // [T*k*D]
+  int* perm = nullptr;       // [T*k]
+  int* tile_off = nullptr;   // [N_OPS][max_items+1]
+  // generic path intermediates (fp32)
+  float* h = nullptr;        // [Rmax][2I]
+  float* P = nullptr;        // [Rmax][2 rmax]
+  float* z = nullptr;        // [Rmax][I]
+  float* Q = nullptr;        // [Rmax][rmax]
+  float* ypart = nullptr;    // [Rmax][H]
+};
+
+struct ProfRec {
+  const char* name;
+  cudaEvent_t a, b;
+};
+
+}  // namespace lx
+
+struct lx_layer {
+  int H = 0, I = 0, E = 0, N = 0, dtype = 0, esz = 0;
+  int n_anchor = 0, n_corr = 0, max_depth = 0, max_rank = 0;
+  int path_mode = LX_PATH_AUTO;
+  int device = 0, num_sms = 0;
+  std::vector<int> parent, rank, expert_node;
+  std::vector<int> anchors, corrs;  // node ids
+  // device copies of the tables
+  int* d_rank = nullptr;
+  int* d_paths = nullptr;           // [E][LX_MAX_DEPTH] node ids, -1 padded
+  int* d_path_len = nullptr;        // [E]
+  int* d_anchors = nullptr;
+  int* d_corrs = nullptr;
+  const void** d_w_up = nullptr;    // per node: anchor [Wg;Wu] [2I][H] | corr [Vg^T;Vu^T] [2r][H]
+  const void** d_w_upU = nullptr;   // per node: corr [Ug;Uu] [2I][r] (null for anchors)
+  const void** d_w_dn = nullptr;    // per node: anchor Wd [H][I] | corr Vd^T [r][I]
+  const void** d_w_dnU = nullptr;   // per node: corr Ud [H][r] (null for anchors)
+  std::vector<const void*> h_w_up, h_w_upU, h_w_dn, h_w_dnU;  // same, host copies
+  void* router_w = nullptr;         // [E][H]
+  float* router_bias = nullptr;     // [E] or null
+  void* arena = nullptr;            // weights
+  size_t arena_bytes = 0;
+  void* tables = nullptr;           // small device tables
+  lx::Workspace ws;
+  int last_T = 0, last_k = 0;       // last bucketing
+  bool profiling = false;
+  std::vector<lx::ProfRec> prof;
+  std::vector<cudaEvent_t> event_pool;
+};
+
+namespace lx {
+
+// Launch-time timing helper: records events around a launch when profiling.
+struct ProfScope {
+  lx_layer* L;
+  cudaStream_t s;
+  cudaEvent_t b = nullptr;
+  const char* name;
+  ProfScope(lx_layer* L_, cudaStream_t s_, const char* n);
+  ~ProfScope();
+};
+
+// kernels / launchers (defined in the .cu files)
+lx_status launch_router(lx_layer* L, const void* x, int T, int k, int* topk_id, float* topk_w,
+                        float* logits, cudaStream_t s);
+lx_status launch_bucket(lx_layer* L, const int* topk_id, int T, int k, cudaStream_t s);
+lx_status launch_generic_experts(lx_layer* L, const void* x, int T, int k, void* y,
+                                 cudaStream_t s);
+
+OpShape op_shape(const lx_layer* L, int op);
+int op_max_items(const lx_layer* L);
+
+}  // namespace lx

@@ -1,0 +1,221 @@
+"""GPU parity of liblx against the CPU oracle, through the C ABI.
+
+Bar (per output tensor): routing ids, bucketing and permutation bit-exact;
+router logits bit-exact (same canonical fp32 order on both sides); gates within
+1e-6; y within max|y - y_ref| / max|y_ref| <= 2e-2 for bf16 layers and 1e-5 for
+fp32 layers.  Sizes span several GEMM tiles with ragged tails; the full-size
+workloads are checked on sampled tokens (the oracle is per token) plus bit-exact
+routing and bucketing of every token.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+from paper_2608_07814_gb300 import lx
+
+pytestmark = pytest.mark.gpu
+
+TOL = {"bf16": 2e-2, "f32": 1e-5}
+
+
+def _dev(a, dtype):
+    return lx.host_to_torch(a, dtype).cuda()
+
+
+def _rel(y, ref):
+    return float(np.max(np.abs(y - ref)) / max(np.max(np.abs(ref)), 1e-30))
+
+
+def _y_host(y):
+    return y.float().cpu().numpy().astype(np.float64)
+
+
+_cache = {}
+
+
+def installed(key, make):
+    """(synth layer, lx.Layer) cached per test session."""
+    if key not in _cache:
+        src = make()
+        _cache[key] = (src, lx.Layer(src))
+    return _cache[key]
+
+
+def check_route(src, L, x, k):
+    xd = _dev(x, src.dtype)
+    ids, w, logits = L.route(xd, k, want_logits=True)
+    torch.cuda.synchronize()
+    o_ids, o_g, o_l = oracle.route(src, x, k)
+    assert np.array_equal(logits.cpu().numpy(), o_l), "logits not bit-exact"
+    assert np.array_equal(ids.cpu().numpy(), o_ids), "top-k ids not bit-exact"
+    assert np.max(np.abs(w.cpu().numpy() - o_g)) < 1e-6
+    return o_ids, o_g
+
+
+def check_buckets(src, L, ids_host):
+    L.bucket(torch.from_numpy(ids_host).cuda())
+    b = L.get_buckets()
+    torch.cuda.synchronize()
+    ref = oracle.buckets(src, ids_host)
+    for key in ("node_off", "node_tok", "node_row", "expert_off", "perm"):
+        got = b[key].cpu().numpy()
+        assert np.array_equal(got, ref[key]), key
+
+
+def check_forward(src, L, x, k, sample=None, path=lx.LX_PATH_AUTO, tol=None):
+    L.set_path(path)
+    xd = _dev(x, src.dtype)
+    y = L.moe_forward(xd, k)
+    torch.cuda.synchronize()
+    yh = _y_host(y)
+    toks = np.arange(x.shape[0]) if sample is None else np.asarray(sample)
+    ref = oracle.moe_forward(src, x, k, token_subset=toks)
+    err = _rel(yh[toks], ref)
+    assert np.all(np.isfinite(yh))
+    assert err <= (tol or TOL[src.dtype]), f"rel err {err}"
+    return err
+
+
+# ----------------------------------------------------------------------------
+# small layers: every output element
+# ----------------------------------------------------------------------------
+SMALL = {
+    "tiny_fp32": lambda: synth.tiny_layer(seed=0),
+    "tiny_fp32_fullrank": lambda: synth.tiny_layer(seed=1, rank=64),
+    "flat_bf16_visible": lambda: synth.flat_layer(512, 384, [4] * 8, 32, 8, "bf16", seed=3,
+                                                  factor_std="visible", skew=synth.QWEN_SKEW),
+    "flat_bf16_zero_dom": lambda: synth.flat_layer(512, 384, [4] * 8, 32, 8, "bf16", seed=3,
+                                                   factor_std="visible", zero_dominants=True,
+                                                   skew=synth.QWEN_SKEW),
+    "flat_bf16_zero_fac": lambda: synth.flat_layer(512, 384, [4] * 8, 32, 8, "bf16", seed=3,
+                                                   zero_factors=True, skew=synth.QWEN_SKEW),
+    "flat_fp32_singletons": lambda: synth.flat_layer(136, 72, [1, 3, 1, 5, 1, 2, 1], 24, 3,
+                                                     "f32", seed=5, factor_std="visible"),
+    "flat_fp32_mixed_rank": lambda: synth.flat_layer(64, 96, [4, 4, 4], [8, 16, 24, 40, 8, 64,
+                                                                         1, 2, 3], 4, "f32",
+                                                     seed=6, factor_std="visible"),
+    "tree_bf16": lambda: synth.tree_layer(256, 192, 2, 4, 3, 48, 16, 8, "bf16", seed=7,
+                                          factor_std="visible", skew=synth.TREE_SKEW),
+    "tree_fp32": lambda: synth.tree_layer(128, 64, 2, 2, 3, 24, 8, 4, "f32", seed=8,
+                                          factor_std="visible", skew=synth.TREE_SKEW),
+}
+
+
+@pytest.mark.parametrize("name", sorted(SMALL))
+@pytest.mark.parametrize("T", [1, 37, 200])
+def test_small_route_bucket_forward(name, T):
+    src, L = installed(name, SMALL[name])
+    x = synth.tokens(src, T, seed=T)
+    ids, _ = check_route(src, L, x, src.top_k)
+    check_buckets(src, L, ids)
+    check_forward(src, L, x, src.top_k)
+    check_forward(src, L, x, src.top_k, path=lx.LX_PATH_GENERIC)
+
+
+def test_tiny_fp32_config_full():
+    """The tiny fp32 workload: 256 tokens, top-2, rank-8 SVD members."""
+    src, L = installed("tiny_fp32", SMALL["tiny_fp32"])
+    x = synth.tokens(src, 256, seed=0)
+    check_route(src, L, x, 2)
+    check_forward(src, L, x, 2)
+
+
+@pytest.mark.parametrize("k", [1, 3, 8])
+def test_other_k(k):
+    src, L = installed("flat_bf16_visible", SMALL["flat_bf16_visible"])
+    x = synth.tokens(src, 64, seed=100 + k)
+    check_route(src, L, x, k)
+    check_forward(src, L, x, k)
+
+
+def test_ties_go_to_lower_id():
+    src = synth.flat_layer(64, 32, [4, 4], 8, 3, "f32", seed=9)
+    src.router_w[5] = src.router_w[2]      # experts 2 and 5 tie on every token
+    src.router_w[7] = src.router_w[2]
+    L = lx.Layer(src)
+    x = synth.tokens(src, 50, seed=1)
+    ids, _ = check_route(src, L, x, 3)
+    for row in ids:
+        if 2 in row or 5 in row or 7 in row:
+            pos = {e: list(row).index(e) for e in (2, 5, 7) if e in row}
+            assert sorted(pos, key=pos.get) == sorted(pos)
+
+
+def test_all_tokens_on_one_cluster():
+    src = synth.flat_layer(256, 128, [4] * 4, 16, 4, "bf16", seed=10, factor_std="visible")
+    src.router_bias = np.zeros(16, np.float32)
+    src.router_bias[src.meta["clusters"][2]] = 50.0
+    L = lx.Layer(src)
+    x = synth.tokens(src, 70, seed=2)
+    ids, _ = check_route(src, L, x, 4)
+    assert set(np.unique(ids)) == set(src.meta["clusters"][2])
+    check_buckets(src, L, ids)
+    check_forward(src, L, x, 4)
+
+
+def test_zero_tokens_is_noop():
+    src, L = installed("tiny_fp32", SMALL["tiny_fp32"])
+    x = torch.empty((0, src.d_model), dtype=torch.float32, device="cuda")
+    y = L.moe_forward(x, 2)
+    assert y.shape == (0, src.d_model)
+
+
+def test_call_errors():
+    src, L = installed("tiny_fp32", SMALL["tiny_fp32"])
+    x = _dev(synth.tokens(src, 4), "f32")
+    with pytest.raises(lx.LxError) as e:
+        L.moe_forward(x, src.n_experts + 1)
+    assert e.value.status == lx.LX_ERR_ARG
+    with pytest.raises(lx.LxError) as e:
+        L.moe_forward(x, 0)
+    assert e.value.status == lx.LX_ERR_ARG
+    big = torch.zeros(4 * 64 + 1, dtype=torch.float32, device="cuda")
+    with pytest.raises(lx.LxError) as e:
+        L.moe_forward(big[1:].view(4, 64), 2)      # misaligned x
+    assert e.value.status == lx.LX_ERR_ARG
+    with pytest.raises(lx.LxError) as e:
+        L.moe_forward(x, 2, y=x)                   # aliasing
+    assert e.value.status == lx.LX_ERR_ARG
+
+
+# ----------------------------------------------------------------------------
+# full-size workloads
+# ----------------------------------------------------------------------------
+FULL = {
+    "qwen": lambda: synth.qwen_decode_layer(),
+    "qwen_visible": lambda: synth.qwen_decode_layer(factor_std="visible"),
+    "high_e": lambda: synth.high_e_layer(),
+    "tree": lambda: synth.btexperts_tree_layer(factor_std="visible"),
+}
+
+
+@pytest.mark.parametrize("T", [1, 8, 32, 64])
+def test_qwen_decode_batches(T):
+    src, L = installed("qwen", FULL["qwen"])
+    x = synth.tokens(src, T, seed=T)
+    ids, _ = check_route(src, L, x, 8)
+    check_buckets(src, L, ids)
+    check_forward(src, L, x, 8)
+
+
+def test_qwen_decode_correction_visible():
+    src, L = installed("qwen_visible", FULL["qwen_visible"])
+    x = synth.tokens(src, 64, seed=3)
+    check_route(src, L, x, 8)
+    check_forward(src, L, x, 8)
+
+
+def _sample(T, n=24, seed=0):
+    rng = np.random.default_rng(seed)
+    return np.unique(np.concatenate([[0, T - 1], rng.choice(T, n, replace=False)]))
+
+
+@pytest.mark.parametrize("name,T", [("qwen", 8192), ("high_e", 4096), ("tree", 2048)])
+def test_full_size_sampled(name, T):
+    src, L = installed(name, FULL[name])
+    x = synth.tokens(src, T, seed=11)
+    ids, _ = check_route(src, L, x, 8)
+    check_buckets(src, L, ids)
+    check_forward(src, L, x, 8, sample=_sample(T))
