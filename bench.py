@@ -1,0 +1,431 @@
+"""Benchmark of the compressed-MoE forward (LorExperts / BTExperts) on GB300.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl lx|reference]
+
+A step is one full forward (route, bucket, shared anchor and correction
+products with SwiGLU, down projection, combine) over one batch of synthetic
+tokens, inputs already resident in HBM.  The default workload is the
+Qwen3-30B-A3B-shaped layer (H=2048, I=768, E=128 top-8, 32 clusters of 4,
+rank-128 members, bf16) at a decode batch of 64 tokens.  Four device copies of
+the layer (2 GB) rotate between steps and every step takes a fresh token batch,
+so weights come from HBM, not L2.
+
+Prints one JSON line (rank 0).  `--impl reference` times the CPU oracle (the
+plain definition of the method) on the host cores instead, on a bounded sample.
+Under torchrun every rank runs its own replica on its own batches (no
+collective on the data path); the timing is the max over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import shutil
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "compressed-MoE layer tokens/s (1 GB300); % HBM roofline decode, % bf16 peak prefill"
+
+WORKLOADS = {
+    # name: (layer maker, T, description)
+    "decode64": ("qwen", 64, "Qwen3-30B-A3B-shaped compressed MoE layer, decode batch of 64 tokens"),
+    "decode32": ("qwen", 32, "Qwen3-30B-A3B-shaped compressed MoE layer, decode batch of 32 tokens"),
+    "decode8": ("qwen", 8, "Qwen3-30B-A3B-shaped compressed MoE layer, decode batch of 8 tokens"),
+    "decode1": ("qwen", 1, "Qwen3-30B-A3B-shaped compressed MoE layer, decode batch of 1 token"),
+    "prefill": ("qwen", 8192, "Qwen3-30B-A3B-shaped compressed MoE layer, prefill of 8192 tokens"),
+    "high_e": ("high_e", 4096, "E=256 (32 clusters of 8, rank 64), H=2560, I=1536, 4096 tokens"),
+    "tree": ("tree", 2048, "BTExperts depth-2 tree (8 roots, 32 rank-192 subs, 96 rank-64 leaves), 2048 tokens"),
+}
+
+
+def make_layer(kind):
+    import synth
+    return {"qwen": synth.qwen_decode_layer, "high_e": synth.high_e_layer,
+            "tree": synth.btexperts_tree_layer}[kind]()
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return d, "measured"
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}, "fallback"
+
+
+# ----------------------------------------------------------------------------
+# clocks sampler (nvidia-smi during the timed region)
+# ----------------------------------------------------------------------------
+class Clocks:
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap,"
+             "utilization.gpu")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.path = None
+        self.windows = []
+
+    def start(self):
+        if not shutil.which("nvidia-smi"):
+            return
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        self.f = open(self.path, "w")
+        self.proc = subprocess.Popen(
+            ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.QUERY}",
+             "--format=csv,noheader,nounits", "-lms", "50"], stdout=self.f,
+            stderr=subprocess.DEVNULL)
+
+    def mark(self, t0, t1):
+        self.windows.append((t0, t1))
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.f.close()
+        rows = []
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 10:
+                continue
+            try:
+                util = float(parts[9])
+                rows.append((float(parts[1]), float(parts[2]), parts[4:9], util))
+            except ValueError:
+                continue
+        os.unlink(self.path)
+        if not rows:
+            return None
+        names = ["active", "hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown",
+                 "sw_power_cap"]
+        loaded = [r for r in rows if r[3] >= 50] or rows
+        reasons = set()
+        for _, _, flags, _ in loaded:
+            for n, v in zip(names[1:], flags[1:]):
+                if v.strip().lower() in ("active", "1", "yes"):
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(r[0] for r in loaded),
+                "sm_max_mhz": max(r[1] for r in rows), "reasons": sorted(reasons),
+                "samples": len(rows), "samples_under_load": len(loaded),
+                "window": "warm-up + timed loops (50 ms sampling, utilization >= 50%)"}
+
+
+# ----------------------------------------------------------------------------
+# algorithmic bytes per kernel launch, from the realised routing
+# ----------------------------------------------------------------------------
+def routing_stats(src, node_off, T, k):
+    cnt = np.diff(node_off.astype(np.int64))
+    anchor = np.asarray(src.node_parent) < 0
+    rank = np.asarray(src.node_rank, np.int64)
+    return dict(cnt=cnt, anchor=anchor, rank=rank, T=T, k=k,
+                touched_anchor=int(np.sum((cnt > 0) & anchor)),
+                touched_corr=int(np.sum((cnt > 0) & ~anchor)),
+                R_anchor=int(cnt[anchor].sum()), R_corr=int(cnt[~anchor].sum()),
+                corr_r_touched=int(rank[(cnt > 0) & ~anchor].sum()),
+                corr_r_rows=int((rank * cnt)[~anchor].sum()))
+
+
+def kernel_bytes(name, st, src, esz):
+    """Bytes a kernel must move per launch (its inputs read once, outputs written
+    once), for the kernels whose traffic is dominated by weight streaming."""
+    H, I, E = src.d_model, src.d_ff, src.n_experts
+    Ra, Rc, ta = st["R_anchor"], st["R_corr"], st["touched_anchor"]
+    rt, rr = st["corr_r_touched"], st["corr_r_rows"]
+    T, k = st["T"], st["k"]
+    table = {
+        "router": E * H * esz + T * H * esz + T * k * 8,
+        "generic_up_anchor": ta * 2 * I * H * esz + Ra * H * esz + Ra * 2 * I * 4,
+        "generic_up_V": rt * 2 * H * esz + Rc * H * esz + rr * 2 * 4,
+        "generic_up_U": rt * 2 * I * esz + rr * 2 * 4 + Rc * 2 * I * 4,
+        "generic_dn_anchor": ta * H * I * esz + Ra * I * 4 + Ra * H * 4,
+        "generic_dn_V": rt * I * esz + Rc * I * 4 + rr * 4,
+        "generic_dn_U": rt * H * esz + rr * 4 + Rc * H * 4,
+    }
+    return table.get(name)
+
+
+def step_bytes(st, src, esz):
+    from paper_2608_07814_gb300 import cost
+    c = cost.step_counts(src.d_model, src.d_ff, src.n_experts, src.node_parent, src.node_rank,
+                         st["cnt"], st["T"], esz, esz)
+    return c
+
+
+def traffic_for(kernel):
+    """dram bytes per launch from the committed ncu summary, if the kernel's
+    source is unchanged since the capture; else None."""
+    p = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(p):
+        return None
+    d = json.load(open(p)).get(kernel)
+    if not d:
+        return None
+    src = os.path.join(ROOT, d["source"])
+    if not os.path.exists(src):
+        return None
+    if hashlib.sha256(open(src, "rb").read()).hexdigest() != d["sha256"]:
+        return None
+    return d["bytes_per_launch"]
+
+
+# ----------------------------------------------------------------------------
+# the CUDA arm
+# ----------------------------------------------------------------------------
+def run_lx(args, rank, world, local_rank):
+    import torch
+    import synth
+    from paper_2608_07814_gb300 import lx
+
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    kind, T, desc = WORKLOADS[args.workload]
+    src = make_layer(kind)
+    k = src.top_k
+    esz = 2 if src.dtype == "bf16" else 4
+    wbytes = src.weight_bytes()
+    n_copies = args.copies if args.copies else (4 if T <= 512 else 1)
+    layers = [lx.Layer(src) for _ in range(n_copies)]
+    for L in layers:
+        L.reserve(T, k)
+    n_batches = 8
+    xs_host = [synth.tokens(src, T, seed=1000 * rank + b) for b in range(n_batches)]
+    xs = [lx.host_to_torch(x, src.dtype).to(dev) for x in xs_host]
+    ys = [torch.empty_like(x) for x in xs]
+    stream = torch.cuda.current_stream()
+
+    # routing statistics of every batch (outside the timed region)
+    stats = []
+    for b in range(n_batches):
+        layers[0].moe_forward(xs[b], k, ys[b])
+        bk = layers[0].get_buckets()
+        torch.cuda.synchronize()
+        stats.append(routing_stats(src, bk["node_off"].cpu().numpy(), T, k))
+
+    clocks = Clocks(local_rank)
+    clocks.start()
+    for i in range(args.warmup):
+        layers[i % n_copies].moe_forward(xs[i % n_batches], k, ys[i % n_batches])
+    torch.cuda.synchronize()
+
+    for L in layers:
+        L.read_profile()
+        L.set_profiling(True)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t_wall0 = time.time()
+    ev0.record(stream)
+    for i in range(args.steps):
+        layers[i % n_copies].moe_forward(xs[i % n_batches], k, ys[i % n_batches])
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    t_wall1 = time.time()
+    clocks.mark(t_wall0, t_wall1)
+    ms = ev0.elapsed_time(ev1)
+    for L in layers:
+        L.set_profiling(False)
+
+    # per-kernel device times of the timed launches (in launch order per copy)
+    per_copy = [L.read_profile(cap=1 << 20) for L in layers]
+    totals, counts = {}, {}
+    launches = 0
+    kbytes = {}
+    for c, recs in enumerate(per_copy):
+        steps_of_copy = [i for i in range(args.steps) if i % n_copies == c]
+        per_step = len(recs) // max(1, len(steps_of_copy))
+        for j, (name, kms) in enumerate(recs):
+            totals[name] = totals.get(name, 0.0) + kms
+            counts[name] = counts.get(name, 0) + 1
+            if name != "bucket_clear":
+                launches += 1
+            step_i = steps_of_copy[j // per_step] if per_step else 0
+            b = kernel_bytes(name, stats[step_i % n_batches], src, esz)
+            if b is not None:
+                kbytes[name] = kbytes.get(name, 0.0) + b
+
+    # e2e: host buffers, copies inside the timed region, a read of every result
+    xh = [lx.host_to_torch(x, src.dtype).pin_memory() for x in xs_host]
+    yh = [torch.empty_like(x).pin_memory() for x in xh]
+    xd, yd = torch.empty_like(xs[0]), torch.empty_like(xs[0])
+    k_e2e = max(3, min(args.steps, 200))
+    for i in range(3):
+        xd.copy_(xh[i % n_batches], non_blocking=True)
+        layers[i % n_copies].moe_forward(xd, k, yd)
+        yh[i % n_batches].copy_(yd, non_blocking=True)
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t_e2e0 = time.time()
+    e0.record(stream)
+    for i in range(k_e2e):
+        xd.copy_(xh[i % n_batches], non_blocking=True)
+        layers[i % n_copies].moe_forward(xd, k, yd)
+        yh[i % n_batches].copy_(yd, non_blocking=True)
+        stream.synchronize()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    clocks.mark(t_e2e0, time.time())
+    ms_e2e = e0.elapsed_time(e1)
+    clk = clocks.stop()
+
+    # max over ranks
+    if world > 1:
+        t = torch.tensor([ms, ms_e2e], dtype=torch.float64, device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        ms, ms_e2e = float(t[0]), float(t[1])
+    if rank != 0:
+        return None
+
+    peaks, peak_kind = load_peaks()
+    hbm = float(peaks["hbm_gbs"])
+    dom = max(totals, key=totals.get)
+    avg_ms = totals[dom] / counts[dom]
+    roof = None
+    if dom in kbytes:
+        bytes_per_launch = kbytes[dom] / counts[dom]
+        ach = bytes_per_launch / (avg_ms * 1e-3) / 1e9
+        roof = {"kernel": dom, "bound": "hbm", "achieved": round(ach, 1), "peak": hbm,
+                "unit": "GB/s", "frac": round(ach / hbm, 4), "traffic": traffic_for(dom),
+                "algorithmic_bytes_per_launch": round(bytes_per_launch),
+                "avg_launch_us": round(avg_ms * 1e3, 2), "peak_source": f"{peak_kind} hbm_gbs"}
+    sb = [step_bytes(stats[i % n_batches], src, esz)["bytes"] for i in range(args.steps)]
+    step_gbs = sum(sb) / (ms * 1e-3) / 1e9
+    tokens = T * args.steps * world
+    amort = np.mean([st["T"] * st["k"] / max(1, st["R_anchor"]) for st in stats])
+    line = {
+        "metric": METRIC, "value": round(tokens / (ms * 1e-3), 1), "unit": "tokens/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(ms / args.steps, 5), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16" if src.dtype == "bf16" else "f32",
+        "data": "synthetic (seeded Gaussian weights and tokens, Zipf-skewed cluster-correlated router)",
+        "config": {"workload": desc, "d_model": src.d_model, "d_ff": src.d_ff,
+                   "n_experts": src.n_experts, "top_k": k, "n_nodes": src.n_nodes,
+                   "tokens_per_step": T, "layer_bytes": wbytes, "layer_copies": n_copies,
+                   "l2": f"{n_copies} rotating device copies of the layer and 8 token batches "
+                         "(inputs larger than L2)",
+                   "parallelism": f"replica per GPU x{world}"},
+        "roofline": roof,
+        "kernels": {n: {"launches": counts[n], "avg_us": round(totals[n] / counts[n] * 1e3, 2),
+                        "share": round(totals[n] / sum(totals.values()), 4)} for n in totals},
+        "step_roofline": {"algorithmic_bytes_per_step": round(float(np.mean(sb))),
+                          "achieved_gbs": round(step_gbs, 1), "frac": round(step_gbs / hbm, 4)},
+        "amortisation": round(float(amort), 3),
+        "e2e": {"value": round(T * k_e2e * world / (ms_e2e * 1e-3), 1), "unit": "tokens/s",
+                "steps": k_e2e, "h2d_bytes_per_step": int(xs[0].numel() * xs[0].element_size()),
+                "d2h_bytes_per_step": int(ys[0].numel() * ys[0].element_size())},
+        "gpu_launches": launches,
+        "clocks": clk,
+        "impl": "lx",
+    }
+    if world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(src, xs_host, T, args.cpu_seconds)
+    return line
+
+
+def cpu_baseline(src, xs_host, T, budget_s):
+    """The oracle, as it stands, on a bounded sample of the same workload."""
+    import oracle
+    done, t0 = 0, time.time()
+    b = 0
+    n = min(T, 64)
+    while True:
+        oracle.moe_forward(src, xs_host[b % len(xs_host)][:n])
+        done += n
+        b += 1
+        if time.time() - t0 > budget_s or b >= 4 * len(xs_host):
+            break
+    el = time.time() - t0
+    return {"value": round(done / el, 3), "unit": "tokens/s", "cores": os.cpu_count(),
+            "kind": "oracle", "seconds": round(el, 2),
+            "sample": f"{b} batch(es) of {n} tokens of the same workload (routing, fp64 "
+                      "reconstruction of every selected expert, standard MoE forward)"}
+
+
+# ----------------------------------------------------------------------------
+# the reference arm: the CPU oracle
+# ----------------------------------------------------------------------------
+def run_reference(args, rank, world):
+    if rank != 0:
+        return None
+    import synth
+    kind, T, desc = WORKLOADS[args.workload]
+    src = make_layer(kind)
+    n = min(T, args.ref_tokens)
+    xs = [synth.tokens(src, T, seed=b)[:n] for b in range(4)]
+    import oracle
+    for i in range(args.warmup):
+        oracle.moe_forward(src, xs[i % 4])
+    t0 = time.time()
+    for i in range(args.steps):
+        oracle.moe_forward(src, xs[i % 4])
+    el = time.time() - t0
+    v = n * args.steps / el
+    sample = f"{n} of the {T} tokens of each step's batch"
+    return {"metric": METRIC, "value": round(v, 3), "unit": "tokens/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(el / args.steps * 1e3, 3), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": desc, "tokens_per_step": T},
+            "impl": "reference",
+            "cpu_baseline": {"value": round(v, 3), "unit": "tokens/s", "cores": os.cpu_count(),
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": round(v, 3), "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=400)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--workload", default="decode64", choices=sorted(WORKLOADS))
+    ap.add_argument("--impl", default="lx", choices=["lx", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--ref-tokens", type=int, default=8)
+    ap.add_argument("--copies", type=int, default=None,
+                    help="device copies of the layer rotated between steps (default 4 for decode)")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1 and args.impl == "lx":
+        import torch
+        torch.cuda.set_device(local_rank)
+        torch.distributed.init_process_group("nccl")
+    if args.impl == "reference":
+        line = run_reference(args, rank, world)
+    else:
+        line = run_lx(args, rank, world, local_rank)
+    if line is not None:
+        print(json.dumps(line), flush=True)
+    if world > 1 and args.impl == "lx":
+        import torch
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -219,6 +219,9 @@ lx_status launch_bucket(lx_layer* L, const int* topk_id, int T, int k, cudaStrea
     k_scatter<<<grid, 256, 0, s>>>(w.marks, w.rank_in, w.key_off, topk_id, T, k, L->N, Tp,
                                    w.node_tok, w.row_node, w.perm);
     LX_CUDA(cudaGetLastError());
+  }
+  {
+    ProfScope ps(L, s, "bucket_node_row");
     const long A = (long)T * k;
     k_node_row<<<(unsigned)((A + 255) / 256), 256, 0, s>>>(topk_id, T, k, L->E, L->max_depth, Tp,
                                                            L->d_paths, L->d_path_len, w.key_off,

@@ -20,7 +20,8 @@ namespace {
 
 constexpr int GG_THREADS = 256;
 
-template <typename TA, typename TW>
+// OPK only names the instantiation (one kernel symbol per op in profiles)
+template <typename TA, typename TW, int OPK>
 __global__ void __launch_bounds__(GG_THREADS)
 k_grouped_gemm(GemmArgs g) {
   __shared__ float As[G_BK][G_BM + 1];
@@ -169,8 +170,8 @@ __global__ void k_combine(const int* __restrict__ node_row, int k, int D,
   }
 }
 
-template <typename TA, typename TW>
-lx_status run_gemm(lx_layer* L, int op, const void* A, long lda, const int* gather,
+template <typename TA, typename TW, int op>
+lx_status run_gemm(lx_layer* L, const void* A, long lda, const int* gather,
                    const void* const* W, float* out, long ldo, cudaStream_t s, const char* name) {
   const OpShape sh = op_shape(L, op);
   GemmArgs g;
@@ -188,7 +189,7 @@ lx_status run_gemm(lx_layer* L, int op, const void* A, long lda, const int* gath
   g.out = out;
   g.ldo = ldo;
   ProfScope ps(L, s, name);
-  k_grouped_gemm<TA, TW><<<L->num_sms * 4, GG_THREADS, 0, s>>>(g);
+  k_grouped_gemm<TA, TW, op><<<L->num_sms * 4, GG_THREADS, 0, s>>>(g);
   LX_CUDA(cudaGetLastError());
   return LX_OK;
 }
@@ -199,11 +200,11 @@ lx_status generic_impl(lx_layer* L, const void* x, int T, int k, void* y, cudaSt
   const long H = L->H, I = L->I, rmax = std::max(1, L->max_rank);
   const int D = L->max_depth;
   // x-side products
-  LX_TRY((run_gemm<TX, TX>(L, OP_UP_ANCHOR, x, H, w.node_tok, (const void* const*)L->d_w_up,
+  LX_TRY((run_gemm<TX, TX, OP_UP_ANCHOR>(L, x, H, w.node_tok, (const void* const*)L->d_w_up,
                            w.h, 2 * I, s, "generic_up_anchor")));
-  LX_TRY((run_gemm<TX, TX>(L, OP_UP_V, x, H, w.node_tok, (const void* const*)L->d_w_up, w.P,
+  LX_TRY((run_gemm<TX, TX, OP_UP_V>(L, x, H, w.node_tok, (const void* const*)L->d_w_up, w.P,
                            2 * rmax, s, "generic_up_V")));
-  LX_TRY((run_gemm<float, TX>(L, OP_UP_U, w.P, 2 * rmax, nullptr,
+  LX_TRY((run_gemm<float, TX, OP_UP_U>(L, w.P, 2 * rmax, nullptr,
                               (const void* const*)L->d_w_upU, w.h, 2 * I, s, "generic_up_U")));
   {
     ProfScope ps(L, s, "generic_swiglu");
@@ -213,11 +214,11 @@ lx_status generic_impl(lx_layer* L, const void* x, int T, int k, void* y, cudaSt
     LX_CUDA(cudaGetLastError());
   }
   // z-side products
-  LX_TRY((run_gemm<float, TX>(L, OP_DN_ANCHOR, w.z, I, nullptr, (const void* const*)L->d_w_dn,
+  LX_TRY((run_gemm<float, TX, OP_DN_ANCHOR>(L, w.z, I, nullptr, (const void* const*)L->d_w_dn,
                               w.ypart, H, s, "generic_dn_anchor")));
-  LX_TRY((run_gemm<float, TX>(L, OP_DN_V, w.z, I, nullptr, (const void* const*)L->d_w_dn, w.Q,
+  LX_TRY((run_gemm<float, TX, OP_DN_V>(L, w.z, I, nullptr, (const void* const*)L->d_w_dn, w.Q,
                               rmax, s, "generic_dn_V")));
-  LX_TRY((run_gemm<float, TX>(L, OP_DN_U, w.Q, rmax, nullptr, (const void* const*)L->d_w_dnU,
+  LX_TRY((run_gemm<float, TX, OP_DN_U>(L, w.Q, rmax, nullptr, (const void* const*)L->d_w_dnU,
                               w.ypart, H, s, "generic_dn_U")));
   {
     ProfScope ps(L, s, "generic_combine");
