@@ -186,6 +186,46 @@ typedef struct {
 LX_API lx_status lx_set_profiling(lx_layer* layer, int32_t enable);
 LX_API lx_status lx_read_profile(lx_layer* layer, lx_kernel_time* out, int32_t cap, int32_t* n);
 
+/*
+ * Size of the fixed device array that lx_bucket_noalloc uses as scratch.  The
+ * array is a static device variable of the library, so every GPU on which the
+ * library's code is loaded holds these bytes until the process exits.
+ */
+#define LX_NOALLOC_SCRATCH_BYTES (16u << 20)
+
+/*
+ * lx_bucket_noalloc -- the bucketing of lx_bucket, for callers that must not
+ * allocate device memory during the call.  The paper has no counterpart; this
+ * is an integration entry point.
+ *
+ * Who needs it: serving runtimes that hand all device memory to their own
+ * pooling allocator or run under a fixed memory budget, and latency-critical
+ * loops in which cudaMalloc/cudaFree are not allowed because they can
+ * synchronise the device and fragment memory.  lx_bucket itself may grow the
+ * layer's workspace with cudaMalloc; this variant never allocates: its
+ * temporary buffers (per-(node|expert, token) marks and ranks, counts and
+ * offsets) live in one static device array of LX_NOALLOC_SCRATCH_BYTES bytes.
+ *
+ * Arguments: as lx_bucket, plus caller-owned device outputs in the layout of
+ * lx_get_buckets (all required, D = max path length of the layer):
+ *   node_off [n_nodes+1], node_tok [T*k*D] (capacity), node_row [T*k*D],
+ *   expert_off [E+1], perm [T*k].
+ * Must be called with the layer's device current.  The first call on a device
+ * looks up the array's device address (cudaGetSymbolAddress) and caches it;
+ * make that first call before any stream capture.  The call needs
+ * 5*(n_nodes+E)*round_up(T,16) + 4*T*k*D bytes (plus small tables, each part
+ * rounded up to 256 bytes) of the array and returns LX_ERR_SHAPE, launching
+ * nothing, when that exceeds LX_NOALLOC_SCRATCH_BYTES.
+ * All calls in the process share the one array per device and the array keeps
+ * the previous call's contents (the call clears what must start at zero):
+ * calls whose GPU work can overlap (different streams, or different layers on
+ * concurrent streams) race on it and must be serialised by the caller.
+ * Results do not update the layer's own bucketing (lx_get_buckets).
+ */
+LX_API lx_status lx_bucket_noalloc(lx_layer* layer, const int32_t* topk_id, int32_t T, int32_t k,
+                                   int32_t* node_off, int32_t* node_tok, int32_t* node_row,
+                                   int32_t* expert_off, int32_t* perm, void* stream);
+
 /* Message of the last failed call on this thread ("" if none). */
 LX_API const char* lx_last_error(void);
 

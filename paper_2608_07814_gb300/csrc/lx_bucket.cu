@@ -9,6 +9,8 @@
 // order, with no atomics); a single CTA scans the per-key counts into offsets
 // and builds the tile plans of the grouped GEMMs; a last pass scatters.
 // Everything is deterministic.
+#include <mutex>
+
 #include "lx_internal.cuh"
 
 namespace lx {
@@ -232,3 +234,107 @@ lx_status launch_bucket(lx_layer* L, const int* topk_id, int T, int k, cudaStrea
 }
 
 }  // namespace lx
+
+// ---------------------------------------------------------------------------
+// lx_bucket_noalloc: the same kernels, with every temporary buffer carved out
+// of one static device array instead of the layer's (cudaMalloc'd) workspace.
+// ---------------------------------------------------------------------------
+namespace lx {
+namespace {
+
+// The scratch itself.  In host code this name is only a handle for
+// cudaGetSymbolAddress, never a device address.
+static __device__ __align__(256) unsigned char g_bucket_scratch[LX_NOALLOC_SCRATCH_BYTES];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_scratch_mu;
+void* g_scratch_addr[kMaxDevices] = {};
+
+// Device address of g_bucket_scratch on `device` (which must be current).
+lx_status scratch_address(int device, void** out) {
+  if (device < 0 || device >= kMaxDevices) return fail(LX_ERR_UNSUPPORTED, "device id above 63");
+  std::lock_guard<std::mutex> lock(g_scratch_mu);
+  if (!g_scratch_addr[device]) {
+    void* p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_bucket_scratch);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(g_bucket_scratch)");
+    g_scratch_addr[device] = p;
+  }
+  *out = g_scratch_addr[device];
+  return LX_OK;
+}
+
+size_t round256(size_t v) { return (v + 255) / 256 * 256; }
+
+}  // namespace
+
+}  // namespace lx
+
+extern "C" lx_status lx_bucket_noalloc(lx_layer* L, const int32_t* topk_id, int32_t T, int32_t k,
+                                       int32_t* node_off, int32_t* node_tok, int32_t* node_row,
+                                       int32_t* expert_off, int32_t* perm, void* stream) {
+  using namespace lx;
+  if (!L) return fail(LX_ERR_ARG, "layer is NULL");
+  if (T < 0) return fail(LX_ERR_ARG, "T < 0");
+  if (k < 1 || k > LX_MAX_K || k > L->E) return fail(LX_ERR_ARG, "k must be in 1..min(E, LX_MAX_K)");
+  if (T == 0) return LX_OK;
+  if (!topk_id || !node_off || !node_tok || !node_row || !expert_off || !perm)
+    return fail(LX_ERR_ARG, "NULL topk_id or output pointer");
+  int dev = -1;
+  LX_CUDA(cudaGetDevice(&dev));
+  if (dev != L->device) return fail(LX_ERR_ARG, "the layer's device must be current");
+
+  // carve the scratch: marks, ranks, counts, offsets, row->node, tile plans
+  const long Tp = ((long)T + 15) / 16 * 16;
+  const long keys = (long)L->N + L->E;
+  const long D = L->max_depth;
+  const size_t b_marks = round256((size_t)keys * Tp);
+  const size_t b_rank = round256(sizeof(int) * (size_t)keys * Tp);
+  const size_t b_cnt = round256(sizeof(int) * (size_t)keys);
+  const size_t b_off = round256(sizeof(int) * (size_t)(keys + 2));
+  const size_t b_rown = round256(sizeof(int) * (size_t)T * k * D);
+  const size_t b_tile = round256(sizeof(int) * (size_t)N_OPS * (op_max_items(L) + 1));
+  const size_t need = b_marks + b_rank + b_cnt + b_off + b_rown + b_tile;
+  if (need > (size_t)LX_NOALLOC_SCRATCH_BYTES)
+    return fail(LX_ERR_SHAPE, "lx_bucket_noalloc: T=" + std::to_string(T) + " needs " +
+                                  std::to_string(need) + " scratch bytes, the fixed array has " +
+                                  std::to_string((size_t)LX_NOALLOC_SCRATCH_BYTES));
+  void* base = nullptr;
+  LX_TRY(scratch_address(dev, &base));
+  char* p = static_cast<char*>(base);
+  uint8_t* marks = reinterpret_cast<uint8_t*>(p);
+  int* rank_in = reinterpret_cast<int*>(p += b_marks);
+  int* key_cnt = reinterpret_cast<int*>(p += b_rank);
+  int* key_off = reinterpret_cast<int*>(p += b_cnt);
+  int* row_node = reinterpret_cast<int*>(p += b_off);
+  int* tile_off = reinterpret_cast<int*>(p += b_rown);
+
+  cudaStream_t s = (cudaStream_t)stream;
+  LX_CUDA(cudaMemsetAsync(marks, 0, (size_t)keys * Tp, s));  // previous call's marks
+  k_mark<<<(T + 255) / 256, 256, 0, s>>>(topk_id, T, k, L->N, L->E, Tp, L->d_paths,
+                                         L->d_path_len, marks);
+  LX_CUDA(cudaGetLastError());
+  k_key_scan<<<(unsigned)keys, SCAN_THREADS, 0, s>>>(marks, T, Tp, rank_in, key_cnt);
+  LX_CUDA(cudaGetLastError());
+  PlanArgs pa;
+  for (int op = 0; op < N_OPS; ++op) {
+    pa.shape[op] = op_shape(L, op);
+    pa.items[op] = pa.shape[op].on_anchors ? L->d_anchors : L->d_corrs;
+    pa.n_items[op] = pa.shape[op].on_anchors ? L->n_anchor : L->n_corr;
+  }
+  k_offsets_plan<<<1, 1024, 0, s>>>(key_cnt, L->N, L->E, key_off, L->d_rank, tile_off,
+                                    op_max_items(L), pa);
+  LX_CUDA(cudaGetLastError());
+  k_scatter<<<dim3((T + 255) / 256, (unsigned)keys), 256, 0, s>>>(
+      marks, rank_in, key_off, topk_id, T, k, L->N, Tp, node_tok, row_node, perm);
+  LX_CUDA(cudaGetLastError());
+  const long A = (long)T * k;
+  k_node_row<<<(unsigned)((A + 255) / 256), 256, 0, s>>>(topk_id, T, k, L->E, L->max_depth, Tp,
+                                                         L->d_paths, L->d_path_len, key_off,
+                                                         rank_in, node_row);
+  LX_CUDA(cudaGetLastError());
+  LX_CUDA(cudaMemcpyAsync(node_off, key_off, sizeof(int) * (L->N + 1), cudaMemcpyDeviceToDevice, s));
+  LX_CUDA(cudaMemcpyAsync(expert_off, key_off + L->N + 1, sizeof(int) * (L->E + 1),
+                          cudaMemcpyDeviceToDevice, s));
+  return LX_OK;
+}

@@ -28,8 +28,9 @@ LX_MAX_DEPTH, LX_MAX_K, LX_MAX_EXPERTS = 4, 32, 1024
 EXPORTS = [
     "lx_load_compressed_layer", "lx_free_layer", "lx_reserve", "lx_route", "lx_bucket",
     "lx_moe_forward", "lx_get_buckets", "lx_layer_info", "lx_set_path", "lx_set_profiling",
-    "lx_read_profile", "lx_last_error",
+    "lx_read_profile", "lx_last_error", "lx_bucket_noalloc",
 ]
+LX_NOALLOC_SCRATCH_BYTES = 16 << 20
 
 
 class LxError(RuntimeError):
@@ -82,6 +83,7 @@ def lib() -> ctypes.CDLL:
             "lx_set_path": [vp, i32],
             "lx_set_profiling": [vp, i32],
             "lx_read_profile": [vp, ctypes.POINTER(KernelTime), i32, ctypes.POINTER(i32)],
+            "lx_bucket_noalloc": [vp, vp, i32, i32, vp, vp, vp, vp, vp, vp],
         }
         for name, args in sig.items():
             f = getattr(L, name)
