@@ -163,6 +163,9 @@ typedef struct {
   int64_t weight_bytes;       /* device bytes of the repacked weights + router */
   int32_t last_T, last_k;     /* sizes of the last bucketing (0 if none) */
   int32_t last_rows;          /* node_off[n_nodes] of the last bucketing (synchronises) */
+  int32_t device_error;       /* lx_status recorded by a kernel (e.g. LX_ERR_TIMEOUT when a
+                                 bounded device-side wait gave up), 0 if none (synchronises) */
+  int32_t stream_path;        /* 1 if the weight-streaming (TMA) decode kernels serve the layer */
 } lx_layer_info_t;
 
 LX_API lx_status lx_layer_info(lx_layer* layer, lx_layer_info_t* info);

@@ -1,5 +1,7 @@
 // C ABI of liblx: validation, layer installation (Sec. 3.2 Stage 3 iii),
 // workspace management, profiling and the forward's orchestration.
+#include <cudaTypedefs.h>
+
 #include <algorithm>
 #include <cstring>
 #include <string>
@@ -97,12 +99,16 @@ static lx_status ensure_workspace(lx_layer* L, int T, int k, cudaStream_t s) {
       {(void**)&w.row_node, sizeof(int) * cT * ck * D},
       {(void**)&w.node_row, sizeof(int) * cT * ck * D},
       {(void**)&w.perm, sizeof(int) * cT * ck},
-      {(void**)&w.tile_off, sizeof(int) * N_OPS * (op_max_items(L) + 1)},
+      {(void**)&w.tile_off, sizeof(int) * N_PLANS * (op_max_items(L) + 1)},
       {(void**)&w.h, sizeof(float) * Rmax * 2 * L->I},
       {(void**)&w.P, sizeof(float) * Rmax * 2 * rmax},
       {(void**)&w.z, sizeof(float) * Rmax * L->I},
       {(void**)&w.Q, sizeof(float) * Rmax * rmax},
       {(void**)&w.ypart, sizeof(float) * Rmax * L->H},
+      {(void**)&w.Pb, 2 * Rmax * 2 * rmax},
+      {(void**)&w.zb, 2 * Rmax * L->I},
+      {(void**)&w.Qb, 2 * Rmax * rmax},
+      {(void**)&w.err, 256},
   };
   size_t total = 0;
   for (auto& it : items) total += align_up(it.bytes, 256);
@@ -124,6 +130,9 @@ static lx_status ensure_workspace(lx_layer* L, int T, int k, cudaStream_t s) {
   }
   w.base = base;
   w.bytes = total;
+  e = cudaMemsetAsync(w.err, 0, sizeof(int), s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return cuda_fail(e, "clear workspace error word");
   w.cap_T = cT;
   w.cap_k = ck;
   L->last_T = L->last_k = 0;
@@ -136,6 +145,81 @@ static lx_status check_call(lx_layer* L, int T, int k) {
   if (k < 1 || k > LX_MAX_K || k > L->E)
     return fail(LX_ERR_ARG, "k must be in 1..min(E, LX_MAX_K)");
   if ((long)T * k * L->max_depth > (1L << 30)) return fail(LX_ERR_SHAPE, "T*k too large");
+  return LX_OK;
+}
+
+// Logits, top-k and bucketing of T tokens (single-CTA bucketing for small T).
+static lx_status route_and_bucket(lx_layer* L, const void* x, int T, int k, int* ids, float* w,
+                                  float* logits_user, cudaStream_t s) {
+  float* logits = logits_user ? logits_user : L->ws.logits;
+  LX_TRY(launch_router_logits(L, x, T, logits, s));
+  if (bucket_small_fits(L, T, k)) {
+    LX_TRY(launch_bucket_small(L, logits, nullptr, T, k, ids, w, s));
+  } else {
+    LX_TRY(launch_topk(L, logits, T, k, ids, w, s));
+    LX_TRY(launch_bucket(L, ids, T, k, s));
+  }
+  return LX_OK;
+}
+
+static lx_status bucket_ids(lx_layer* L, const int* ids, int T, int k, cudaStream_t s) {
+  if (bucket_small_fits(L, T, k)) return launch_bucket_small(L, nullptr, ids, T, k, nullptr, nullptr, s);
+  return launch_bucket(L, ids, T, k, s);
+}
+
+// Largest batch the weight-streaming (decode) kernels take; beyond it every
+// weight would be re-streamed per 64-token block.
+constexpr int kStreamMaxT = 256;
+
+static bool use_stream(const lx_layer* L, int T) {
+  return L->path_mode == LX_PATH_AUTO && L->stream_ok && T <= kStreamMaxT;
+}
+
+// TMA descriptors of every weight matrix the streaming kernels read.
+static lx_status encode_tensor_maps(lx_layer* L, cudaStream_t s) {
+  L->stream_ok = false;
+  if (L->dtype != LX_BF16) return LX_OK;
+  if (L->H % 64 || L->I % 64) return LX_OK;
+  for (int n = 0; n < L->N; ++n)
+    if (L->parent[n] >= 0 && L->rank[n] % 64) return LX_OK;
+  void* fn = nullptr;
+  cudaDriverEntryPointQueryResult q;
+  cudaError_t ce = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000,
+                                                    cudaEnableDefault, &q);
+  if (ce != cudaSuccess || q != cudaDriverEntryPointSuccess || !fn) return LX_OK;
+  auto encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  std::vector<CUtensorMap> maps((size_t)N_OPS * L->N);
+  std::memset(maps.data(), 0, maps.size() * sizeof(CUtensorMap));
+  for (int op = 0; op < N_OPS; ++op) {
+    const OpShape sh = op_shape(L, op);
+    for (int n = 0; n < L->N; ++n) {
+      const bool anchor = L->parent[n] < 0;
+      if ((sh.on_anchors != 0) != anchor) continue;
+      const int r = L->rank[n];
+      const cuuint64_t K = sh.k_const + sh.k_rank * r;
+      const cuuint64_t rows = (cuuint64_t)sh.groups * (sh.n_const + sh.n_rank * r);
+      const void* base = op == OP_UP_ANCHOR || op == OP_UP_V ? L->h_w_up[n]
+                         : op == OP_UP_U                     ? L->h_w_upU[n]
+                         : op == OP_DN_U                     ? L->h_w_dnU[n]
+                                                             : L->h_w_dn[n];
+      const cuuint64_t dims[2] = {K, rows};
+      const cuuint64_t strides[1] = {K * 2};
+      const cuuint32_t box[2] = {(cuuint32_t)stream_box(), (cuuint32_t)stream_tile_rows()};
+      const cuuint32_t estr[2] = {1, 1};
+      CUresult cr = encode(&maps[(size_t)op * L->N + n], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+                           const_cast<void*>(base), dims, strides, box, estr,
+                           CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+      if (cr != CUDA_SUCCESS) return LX_OK;  // streaming path stays off
+    }
+  }
+  void* d = nullptr;
+  LX_CUDA(cudaMalloc(&d, maps.size() * sizeof(CUtensorMap)));
+  L->d_tmaps = static_cast<CUtensorMap*>(d);
+  LX_CUDA(cudaMemcpyAsync(d, maps.data(), maps.size() * sizeof(CUtensorMap),
+                          cudaMemcpyHostToDevice, s));
+  LX_CUDA(cudaStreamSynchronize(s));
+  L->stream_ok = true;
   return LX_OK;
 }
 
@@ -346,6 +430,8 @@ extern "C" lx_status lx_load_compressed_layer(const lx_layer_desc* d, const void
   ce = cudaMemcpyAsync(L->tables, tb.data(), toff, cudaMemcpyHostToDevice, s);
   if (ce == cudaSuccess) ce = cudaStreamSynchronize(s);
   if (ce != cudaSuccess) return cleanup(cuda_fail(ce, "copy tables"));
+  const lx_status st = encode_tensor_maps(L, s);
+  if (st != LX_OK) return cleanup(st);
   *out = L;
   return LX_OK;
 }
@@ -361,6 +447,7 @@ extern "C" lx_status lx_free_layer(lx_layer* L) {
   if (L->ws.base) cudaFree(L->ws.base);
   if (L->arena) cudaFree(L->arena);
   if (L->tables) cudaFree(L->tables);
+  if (L->d_tmaps) cudaFree(L->d_tmaps);
   delete L;
   return LX_OK;
 }
@@ -379,8 +466,7 @@ extern "C" lx_status lx_route(lx_layer* L, const void* x, int32_t T, int32_t k, 
   if (!x || !topk_id || !topk_w) return fail(LX_ERR_ARG, "NULL x/topk_id/topk_w");
   cudaStream_t s = (cudaStream_t)stream;
   LX_TRY(ensure_workspace(L, T, k, s));
-  LX_TRY(launch_router(L, x, T, k, topk_id, topk_w, logits, s));
-  LX_TRY(launch_bucket(L, topk_id, T, k, s));
+  LX_TRY(route_and_bucket(L, x, T, k, topk_id, topk_w, logits, s));
   L->last_T = T;
   L->last_k = k;
   return LX_OK;
@@ -393,7 +479,7 @@ extern "C" lx_status lx_bucket(lx_layer* L, const int32_t* topk_id, int32_t T, i
   if (!topk_id) return fail(LX_ERR_ARG, "NULL topk_id");
   cudaStream_t s = (cudaStream_t)stream;
   LX_TRY(ensure_workspace(L, T, k, s));
-  LX_TRY(launch_bucket(L, topk_id, T, k, s));
+  LX_TRY(bucket_ids(L, topk_id, T, k, s));
   L->last_T = T;
   L->last_k = k;
   return LX_OK;
@@ -408,11 +494,14 @@ extern "C" lx_status lx_moe_forward(lx_layer* L, const void* x, int32_t T, int32
   cudaStream_t s = (cudaStream_t)stream;
   LX_TRY(ensure_workspace(L, T, k, s));
   Workspace& w = L->ws;
-  LX_TRY(launch_router(L, x, T, k, w.topk_id, w.topk_w, nullptr, s));
-  LX_TRY(launch_bucket(L, w.topk_id, T, k, s));
+  LX_TRY(route_and_bucket(L, x, T, k, w.topk_id, w.topk_w, nullptr, s));
   L->last_T = T;
   L->last_k = k;
-  LX_TRY(launch_generic_experts(L, x, T, k, y, s));
+  if (use_stream(L, T)) {
+    LX_TRY(launch_fast_experts(L, x, T, k, y, s));
+  } else {
+    LX_TRY(launch_generic_experts(L, x, T, k, y, s));
+  }
   return LX_OK;
 }
 
@@ -452,11 +541,18 @@ extern "C" lx_status lx_layer_info(lx_layer* L, lx_layer_info_t* info) {
   info->last_T = L->last_T;
   info->last_k = L->last_k;
   info->last_rows = 0;
-  if (L->last_T > 0) {
-    int rows = 0;
+  info->device_error = 0;
+  info->stream_path = L->stream_ok ? 1 : 0;
+  if (L->ws.base) {
     LX_CUDA(cudaDeviceSynchronize());
-    LX_CUDA(cudaMemcpy(&rows, L->ws.key_off + L->N, 4, cudaMemcpyDeviceToHost));
-    info->last_rows = rows;
+    int err = 0;
+    LX_CUDA(cudaMemcpy(&err, L->ws.err, 4, cudaMemcpyDeviceToHost));
+    info->device_error = err;
+    if (L->last_T > 0) {
+      int rows = 0;
+      LX_CUDA(cudaMemcpy(&rows, L->ws.key_off + L->N, 4, cudaMemcpyDeviceToHost));
+      info->last_rows = rows;
+    }
   }
   return LX_OK;
 }

@@ -87,16 +87,24 @@ k_key_scan(const uint8_t* __restrict__ marks, int T, long Tp, int* __restrict__ 
 }
 
 struct PlanArgs {
-  const int* items[N_OPS];
-  int n_items[N_OPS];
-  OpShape shape[N_OPS];
+  const int* items[N_PLANS];
+  int n_items[N_PLANS];
+  OpShape shape[N_PLANS];
+  int bm[N_PLANS], bn[N_PLANS];  // token rows and output columns per tile
+  int n_plans;
 };
 
-// one CTA: node/expert offsets and the tile prefix of every grouped-GEMM op
+// tiles of one node in one plan
+__device__ __forceinline__ int plan_tiles(const PlanArgs& pa, int p, int r, int rows) {
+  const OpShape sh = pa.shape[p];
+  const int Ng = sh.n_const + sh.n_rank * r;
+  return ((rows + pa.bm[p] - 1) / pa.bm[p]) * sh.groups * ((Ng + pa.bn[p] - 1) / pa.bn[p]);
+}
+
+// one CTA: node/expert offsets and the tile prefix of every plan
 __global__ void k_offsets_plan(const int* __restrict__ key_cnt, int N, int E,
                                int* __restrict__ key_off, const int* __restrict__ rank,
                                int* __restrict__ tile_off, int max_items, PlanArgs pa) {
-  __shared__ int total_s;
   // node offsets then expert offsets
   for (int part = 0; part < 2; ++part) {
     const int n0 = part == 0 ? 0 : N, cnt = part == 0 ? N : E;
@@ -113,27 +121,22 @@ __global__ void k_offsets_plan(const int* __restrict__ key_cnt, int N, int E,
     if (threadIdx.x == 0) out[cnt] = carry;
     __syncthreads();
   }
-  (void)total_s;
-  for (int op = 0; op < N_OPS; ++op) {
-    const OpShape sh = pa.shape[op];
-    int* to = tile_off + op * (max_items + 1);
+  for (int p = 0; p < pa.n_plans; ++p) {
+    int* to = tile_off + p * (max_items + 1);
     int carry = 0;
-    for (int base = 0; base < pa.n_items[op]; base += blockDim.x) {
+    for (int base = 0; base < pa.n_items[p]; base += blockDim.x) {
       const int i = base + threadIdx.x;
       int v = 0;
-      if (i < pa.n_items[op]) {
-        const int n = pa.items[op][i];
-        const int r = rank[n];
-        const int Ng = sh.n_const + sh.n_rank * r;
-        const int rows = key_cnt[n];
-        v = ((rows + G_BM - 1) / G_BM) * sh.groups * ((Ng + G_BN - 1) / G_BN);
+      if (i < pa.n_items[p]) {
+        const int n = pa.items[p][i];
+        v = plan_tiles(pa, p, rank[n], key_cnt[n]);
       }
       int total;
       const int ex = block_excl_scan(v, &total);
-      if (i < pa.n_items[op]) to[i] = carry + ex;
+      if (i < pa.n_items[p]) to[i] = carry + ex;
       carry += total;
     }
-    if (threadIdx.x == 0) to[pa.n_items[op]] = carry;
+    if (threadIdx.x == 0) to[pa.n_items[p]] = carry;
     __syncthreads();
   }
 }
@@ -182,7 +185,179 @@ __global__ void k_node_row(const int* __restrict__ topk_id, int T, int k, int E,
   }
 }
 
+
+// ---------------------------------------------------------------------------
+// Small batches (decode): top-k and the whole bucketing in one CTA, with the
+// marks and ranks in shared memory (ranks fit a byte since T <= 256).  Same
+// outputs, same order, as the multi-kernel path above.
+// ---------------------------------------------------------------------------
+constexpr int SB_THREADS = 1024;
+constexpr int SB_MAX_T = 256;
+constexpr size_t SB_SMEM_LIMIT = 160 * 1024;
+
+__host__ __device__ inline size_t sb_smem(int T, int k, int keys) {
+  const size_t Tp = ((size_t)T + 15) / 16 * 16;
+  return (size_t)T * k * 4 + 2 * (size_t)keys * Tp + (size_t)keys * 4 + ((size_t)keys + 2) * 4 + 64;
+}
+
+__global__ void __launch_bounds__(SB_THREADS)
+k_bucket_small(const float* __restrict__ logits, const int* __restrict__ ids_in, int T, int k,
+               int E, int N, int D, const int* __restrict__ paths,
+               const int* __restrict__ path_len, const int* __restrict__ rank,
+               int* __restrict__ topk_id, float* __restrict__ topk_w, int* __restrict__ key_off_g,
+               int* __restrict__ node_tok, int* __restrict__ row_node, int* __restrict__ node_row,
+               int* __restrict__ perm, int* __restrict__ tile_off, int max_items, PlanArgs pa) {
+  extern __shared__ __align__(16) unsigned char sm[];
+  const int keys = N + E;
+  const int Tp = (T + 15) & ~15;
+  int* ids = reinterpret_cast<int*>(sm);
+  uint8_t* marks = reinterpret_cast<uint8_t*>(ids + T * k);
+  uint8_t* rk = marks + (size_t)keys * Tp;
+  int* cnt = reinterpret_cast<int*>(rk + (((size_t)keys * Tp + 3) & ~(size_t)3));
+  int* off = cnt + keys;
+  const int tid = threadIdx.x, nth = blockDim.x;
+  const int warp = tid >> 5, lane = tid & 31, nw = nth >> 5;
+
+  // 1. routing (or the given ids)
+  if (logits) {
+    for (int t = warp; t < T; t += nw) {
+      int id;
+      float w;
+      warp_topk(logits + (size_t)t * E, E, k, id, w);
+      if (lane < k) {
+        ids[t * k + lane] = id;
+        topk_id[(size_t)t * k + lane] = id;
+        topk_w[(size_t)t * k + lane] = w;
+      }
+    }
+  } else {
+    for (int i = tid; i < T * k; i += nth) ids[i] = ids_in[i];
+  }
+  for (int i = tid; i < keys * Tp; i += nth) marks[i] = 0;
+  __syncthreads();
+  // 2. marks
+  for (int a = tid; a < T * k; a += nth) {
+    const int t = a / k, e = ids[a];
+    if (e < 0 || e >= E) continue;
+    marks[(N + e) * Tp + t] = 1;
+    const int len = path_len[e];
+    for (int l = 0; l < len; ++l) marks[paths[e * LX_MAX_DEPTH + l] * Tp + t] = 1;
+  }
+  __syncthreads();
+  // 3. per-key ranks in token order
+  for (int key = tid; key < keys; key += nth) {
+    int c = 0;
+    for (int t = 0; t < T; ++t)
+      if (marks[key * Tp + t]) rk[key * Tp + t] = (uint8_t)c++;
+    cnt[key] = c;
+  }
+  __syncthreads();
+  // 4. node offsets then expert offsets
+  for (int part = 0; part < 2; ++part) {
+    const int n0 = part == 0 ? 0 : N, n = part == 0 ? N : E;
+    const int o0 = part == 0 ? 0 : N + 1;
+    int carry = 0;
+    for (int base = 0; base < n; base += nth) {
+      const int i = base + tid;
+      const int v = i < n ? cnt[n0 + i] : 0;
+      int total;
+      const int ex = block_excl_scan(v, &total);
+      if (i < n) off[o0 + i] = carry + ex;
+      carry += total;
+    }
+    if (tid == 0) off[o0 + n] = carry;
+    __syncthreads();
+  }
+  for (int i = tid; i < keys + 2; i += nth) key_off_g[i] = off[i];
+  // 5. scatter
+  for (int idx = tid; idx < keys * T; idx += nth) {
+    const int key = idx / T, t = idx % T;
+    if (!marks[key * Tp + t]) continue;
+    const int r = rk[key * Tp + t];
+    if (key < N) {
+      const int row = off[key] + r;
+      node_tok[row] = t;
+      row_node[row] = key;
+    } else {
+      const int e = key - N;
+      const int pos = off[N + 1 + e] + r;
+      for (int s = 0; s < k; ++s)
+        if (ids[t * k + s] == e) {
+          perm[pos] = t * k + s;
+          break;
+        }
+    }
+  }
+  // 6. rows of every (assignment, path level)
+  for (int a = tid; a < T * k; a += nth) {
+    const int t = a / k, e = ids[a];
+    const int len = (e >= 0 && e < E) ? path_len[e] : 0;
+    for (int l = 0; l < D; ++l) {
+      int row = -1;
+      if (l < len) {
+        const int n = paths[e * LX_MAX_DEPTH + l];
+        row = off[n] + rk[n * Tp + t];
+      }
+      node_row[(size_t)a * D + l] = row;
+    }
+  }
+  // 7. tile plans
+  for (int p = 0; p < pa.n_plans; ++p) {
+    int* to = tile_off + p * (max_items + 1);
+    int carry = 0;
+    for (int base = 0; base < pa.n_items[p]; base += nth) {
+      const int i = base + tid;
+      int v = 0;
+      if (i < pa.n_items[p]) {
+        const int n = pa.items[p][i];
+        v = plan_tiles(pa, p, rank[n], cnt[n]);
+      }
+      int total;
+      const int ex = block_excl_scan(v, &total);
+      if (i < pa.n_items[p]) to[i] = carry + ex;
+      carry += total;
+    }
+    if (tid == 0) to[pa.n_items[p]] = carry;
+    __syncthreads();
+  }
+}
+
 }  // namespace
+
+// plans 0..N_OPS-1: generic tiles; N_OPS..2*N_OPS-1: streaming tiles
+static PlanArgs make_plans(const lx_layer* L, int n_plans) {
+  PlanArgs pa;
+  pa.n_plans = n_plans;
+  for (int p = 0; p < n_plans; ++p) {
+    const int op = p % N_OPS;
+    pa.shape[p] = op_shape(L, op);
+    pa.items[p] = pa.shape[p].on_anchors ? L->d_anchors : L->d_corrs;
+    pa.n_items[p] = pa.shape[p].on_anchors ? L->n_anchor : L->n_corr;
+    pa.bm[p] = p < N_OPS ? G_BM : stream_tile_tokens();
+    pa.bn[p] = p < N_OPS ? G_BN : stream_tile_rows();
+  }
+  return pa;
+}
+
+bool bucket_small_fits(const lx_layer* L, int T, int k) {
+  return T <= SB_MAX_T && sb_smem(T, k, L->N + L->E) <= SB_SMEM_LIMIT;
+}
+
+lx_status launch_bucket_small(lx_layer* L, const float* logits, const int* ids_in, int T, int k,
+                              int* topk_id, float* topk_w, cudaStream_t s) {
+  Workspace& w = L->ws;
+  const size_t smem = sb_smem(T, k, L->N + L->E);
+  const PlanArgs pa = make_plans(L, N_PLANS);
+  LX_CUDA(cudaFuncSetAttribute(k_bucket_small, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               (int)smem));
+  ProfScope ps(L, s, logits ? "topk_bucket_small" : "bucket_small");
+  k_bucket_small<<<1, SB_THREADS, smem, s>>>(logits, ids_in, T, k, L->E, L->N, L->max_depth,
+                                             L->d_paths, L->d_path_len, L->d_rank, topk_id, topk_w,
+                                             w.key_off, w.node_tok, w.row_node, w.node_row, w.perm,
+                                             w.tile_off, op_max_items(L), pa);
+  LX_CUDA(cudaGetLastError());
+  return LX_OK;
+}
 
 lx_status launch_bucket(lx_layer* L, const int* topk_id, int T, int k, cudaStream_t s) {
   Workspace& w = L->ws;
@@ -204,12 +379,7 @@ lx_status launch_bucket(lx_layer* L, const int* topk_id, int T, int k, cudaStrea
     LX_CUDA(cudaGetLastError());
   }
   {
-    PlanArgs pa;
-    for (int op = 0; op < N_OPS; ++op) {
-      pa.shape[op] = op_shape(L, op);
-      pa.items[op] = pa.shape[op].on_anchors ? L->d_anchors : L->d_corrs;
-      pa.n_items[op] = pa.shape[op].on_anchors ? L->n_anchor : L->n_corr;
-    }
+    const PlanArgs pa = make_plans(L, N_PLANS);
     ProfScope ps(L, s, "bucket_offsets");
     k_offsets_plan<<<1, 1024, 0, s>>>(w.key_cnt, L->N, L->E, w.key_off, L->d_rank, w.tile_off,
                                       op_max_items(L), pa);
@@ -316,12 +486,7 @@ extern "C" lx_status lx_bucket_noalloc(lx_layer* L, const int32_t* topk_id, int3
   LX_CUDA(cudaGetLastError());
   k_key_scan<<<(unsigned)keys, SCAN_THREADS, 0, s>>>(marks, T, Tp, rank_in, key_cnt);
   LX_CUDA(cudaGetLastError());
-  PlanArgs pa;
-  for (int op = 0; op < N_OPS; ++op) {
-    pa.shape[op] = op_shape(L, op);
-    pa.items[op] = pa.shape[op].on_anchors ? L->d_anchors : L->d_corrs;
-    pa.n_items[op] = pa.shape[op].on_anchors ? L->n_anchor : L->n_corr;
-  }
+  const PlanArgs pa = make_plans(L, N_OPS);
   k_offsets_plan<<<1, 1024, 0, s>>>(key_cnt, L->N, L->E, key_off, L->d_rank, tile_off,
                                     op_max_items(L), pa);
   LX_CUDA(cudaGetLastError());

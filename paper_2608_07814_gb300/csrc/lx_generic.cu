@@ -102,6 +102,7 @@ k_grouped_gemm(GemmArgs g) {
 __device__ __forceinline__ float silu_f(float v) { return v / (1.f + expf(-v)); }
 
 // z[row] for every (token, node) row
+template <typename TZ>
 __global__ void k_swiglu_aggregate(const int* __restrict__ key_off, int N,
                                    const int* __restrict__ node_tok,
                                    const int* __restrict__ row_node,
@@ -109,7 +110,7 @@ __global__ void k_swiglu_aggregate(const int* __restrict__ key_off, int N,
                                    const float* __restrict__ topk_w,
                                    const int* __restrict__ node_row, int k, int D, int E,
                                    const int* __restrict__ paths, const int* __restrict__ path_len,
-                                   const float* __restrict__ h, int I, float* __restrict__ z) {
+                                   const float* __restrict__ h, int I, TZ* __restrict__ z) {
   const int R = key_off[N];
   for (int row = blockIdx.x; row < R; row += gridDim.x) {
     const int t = node_tok[row];
@@ -133,7 +134,7 @@ __global__ void k_swiglu_aggregate(const int* __restrict__ key_off, int N,
         }
         acc = fmaf(topk_w[a], silu_f(pg) * pu, acc);
       }
-      z[(size_t)row * I + i] = acc;
+      z[(size_t)row * I + i] = from_f32<TZ>(acc);
     }
   }
 }
@@ -169,6 +170,39 @@ __global__ void k_combine(const int* __restrict__ node_row, int k, int D,
     __syncthreads();
   }
 }
+
+}  // namespace
+
+lx_status launch_swiglu(lx_layer* L, int k, void* z, bool z_bf16, cudaStream_t s) {
+  Workspace& w = L->ws;
+  ProfScope ps(L, s, z_bf16 ? "swiglu" : "generic_swiglu");
+  const dim3 grid(L->num_sms * 8);
+  if (z_bf16)
+    k_swiglu_aggregate<__nv_bfloat16><<<grid, 256, 0, s>>>(
+        w.key_off, L->N, w.node_tok, w.row_node, w.topk_id, w.topk_w, w.node_row, k,
+        L->max_depth, L->E, L->d_paths, L->d_path_len, w.h, L->I, (__nv_bfloat16*)z);
+  else
+    k_swiglu_aggregate<float><<<grid, 256, 0, s>>>(
+        w.key_off, L->N, w.node_tok, w.row_node, w.topk_id, w.topk_w, w.node_row, k,
+        L->max_depth, L->E, L->d_paths, L->d_path_len, w.h, L->I, (float*)z);
+  LX_CUDA(cudaGetLastError());
+  return LX_OK;
+}
+
+lx_status launch_combine(lx_layer* L, int T, int k, void* y, cudaStream_t s) {
+  Workspace& w = L->ws;
+  ProfScope ps(L, s, "combine");
+  const int grid = std::min(T, L->num_sms * 8);
+  if (L->dtype == LX_BF16)
+    k_combine<__nv_bfloat16><<<grid, 256, 0, s>>>(w.node_row, k, L->max_depth, w.ypart, L->H,
+                                                  (__nv_bfloat16*)y, T);
+  else
+    k_combine<float><<<grid, 256, 0, s>>>(w.node_row, k, L->max_depth, w.ypart, L->H, (float*)y, T);
+  LX_CUDA(cudaGetLastError());
+  return LX_OK;
+}
+
+namespace {
 
 template <typename TA, typename TW, int op>
 lx_status run_gemm(lx_layer* L, const void* A, long lda, const int* gather,
@@ -206,13 +240,7 @@ lx_status generic_impl(lx_layer* L, const void* x, int T, int k, void* y, cudaSt
                            2 * rmax, s, "generic_up_V")));
   LX_TRY((run_gemm<float, TX, OP_UP_U>(L, w.P, 2 * rmax, nullptr,
                               (const void* const*)L->d_w_upU, w.h, 2 * I, s, "generic_up_U")));
-  {
-    ProfScope ps(L, s, "generic_swiglu");
-    k_swiglu_aggregate<<<L->num_sms * 8, 256, 0, s>>>(
-        w.key_off, L->N, w.node_tok, w.row_node, w.topk_id, w.topk_w, w.node_row, k, D, L->E,
-        L->d_paths, L->d_path_len, w.h, (int)I, w.z);
-    LX_CUDA(cudaGetLastError());
-  }
+  LX_TRY(launch_swiglu(L, k, w.z, false, s));
   // z-side products
   LX_TRY((run_gemm<float, TX, OP_DN_ANCHOR>(L, w.z, I, nullptr, (const void* const*)L->d_w_dn,
                               w.ypart, H, s, "generic_dn_anchor")));
@@ -220,12 +248,7 @@ lx_status generic_impl(lx_layer* L, const void* x, int T, int k, void* y, cudaSt
                               rmax, s, "generic_dn_V")));
   LX_TRY((run_gemm<float, TX, OP_DN_U>(L, w.Q, rmax, nullptr, (const void* const*)L->d_w_dnU,
                               w.ypart, H, s, "generic_dn_U")));
-  {
-    ProfScope ps(L, s, "generic_combine");
-    const int grid = std::min(T, L->num_sms * 8);
-    k_combine<TX><<<grid, 256, 0, s>>>(w.node_row, k, D, w.ypart, (int)H, (TX*)y, T);
-    LX_CUDA(cudaGetLastError());
-  }
+  LX_TRY(launch_combine(L, T, k, y, s));
   return LX_OK;
 }
 

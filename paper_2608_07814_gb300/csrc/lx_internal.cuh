@@ -1,6 +1,7 @@
 // Internal declarations shared by the CUDA translation units of liblx.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <cuda_bf16.h>
 #include <stdint.h>
@@ -42,6 +43,53 @@ template <> __device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(flo
 }
 
 // ---------------------------------------------------------------------------
+// top-k of one token's logits by one warp: k rounds of a warp arg-max with
+// the order (logit descending, expert id ascending); softmax over the k
+// selected logits.  Lane j ends with slot j's id and gate (j < k).  A NaN
+// logit is never preferred; if only NaNs remain the lowest free id is taken,
+// so ids always stay in [0, E).
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ bool topk_better(float v, int i, float bv, int bi) {
+  return v > bv || (v == bv && i < bi);
+}
+
+__device__ __forceinline__ void warp_topk(const float* lt, int E, int k, int& sel_id,
+                                          float& sel_w) {
+  const int lane = threadIdx.x & 31;
+  uint32_t taken = 0;  // bit i <-> expert lane + 32 i
+  float m = 0.f, denom = 0.f, selv = 0.f;
+  int seli = 0;
+  for (int j = 0; j < k; ++j) {
+    float bv = -INFINITY;
+    int bi = 0x7fffffff;
+    for (int i = 0, e = lane; e < E; ++i, e += 32)
+      if (!((taken >> i) & 1u) && topk_better(lt[e], e, bv, bi)) { bv = lt[e]; bi = e; }
+#pragma unroll
+    for (int off = 16; off >= 1; off >>= 1) {
+      const float ov = __shfl_xor_sync(0xffffffffu, bv, off);
+      const int oi = __shfl_xor_sync(0xffffffffu, bi, off);
+      if (topk_better(ov, oi, bv, bi)) { bv = ov; bi = oi; }
+    }
+    if (bi == 0x7fffffff) {
+      int fi = 0x7fffffff;
+      for (int i = 0, e = lane; e < E; ++i, e += 32)
+        if (!((taken >> i) & 1u)) { fi = e; break; }
+#pragma unroll
+      for (int off = 16; off >= 1; off >>= 1) fi = min(fi, __shfl_xor_sync(0xffffffffu, fi, off));
+      bi = fi;
+      bv = lt[bi];
+    }
+    if ((bi & 31) == lane) taken |= 1u << (bi >> 5);
+    if (j == 0) m = bv;
+    const float ex = expf(bv - m);
+    denom += ex;
+    if (lane == j) { selv = ex; seli = bi; }
+  }
+  sel_id = seli;
+  sel_w = selv / denom;
+}
+
+// ---------------------------------------------------------------------------
 // grouped GEMM over node buckets (the generic CUDA-core path)
 // ---------------------------------------------------------------------------
 // Op kinds, indexing the per-op tile plans.
@@ -54,6 +102,12 @@ enum OpKind {
   OP_DN_U = 5,       // ypart[row, 0:H] = Q[row] . Ud^T
   N_OPS = 6
 };
+
+// Tile plans: plan p < N_OPS is op p for the generic kernel (32-token x
+// 64-column tiles); plan N_OPS + p is op p for the streaming kernel (64-token
+// x 64-weight-row tiles).
+constexpr int N_PLANS = 2 * N_OPS;
+constexpr int PLAN_STREAM = N_OPS;
 
 // Per-op shape rule: for node n with rank r, each group has
 //   N_g = n_const + n_rank * r output columns and K = k_const + k_rank * r.
@@ -80,6 +134,29 @@ struct GemmArgs {
   long ldo;
 };
 
+// Streaming (decode) grouped GEMM: one op of a launch
+struct StreamOp {
+  const CUtensorMap* tmaps;  // [n_nodes] weight tensor maps of this op
+  const int* items;          // node ids
+  int n_items;
+  const int* tile_off;       // [n_items+1] stream plan
+  const int* node_off;
+  const int* gather;         // row -> X row (token ids), or null = identity
+  const __nv_bfloat16* X;    // activations, bf16
+  long ldx;
+  void* out;                 // fp32 or bf16
+  long ldo;
+  int out_f32;
+  OpShape shape;
+  const int* rank;
+};
+
+struct StreamLaunch {
+  StreamOp op[2];
+  int n_ops;
+  int* err;                  // device error word (LX_ERR_TIMEOUT on a bounded wait)
+};
+
 // ---------------------------------------------------------------------------
 // device workspace of one forward
 // ---------------------------------------------------------------------------
@@ -100,13 +177,18 @@ struct Workspace {
   int* row_node = nullptr;   // [T*k*D]
   int* node_row = nullptr;   // [T*k*D]
   int* perm = nullptr;       // [T*k]
-  int* tile_off = nullptr;   // [N_OPS][max_items+1]
+  int* tile_off = nullptr;   // [N_PLANS][max_items+1]
   // generic path intermediates (fp32)
   float* h = nullptr;        // [Rmax][2I]
   float* P = nullptr;        // [Rmax][2 rmax]
   float* z = nullptr;        // [Rmax][I]
   float* Q = nullptr;        // [Rmax][rmax]
   float* ypart = nullptr;    // [Rmax][H]
+  // streaming path intermediates (bf16 operands of the next product)
+  __nv_bfloat16* Pb = nullptr;  // [Rmax][2 rmax]
+  __nv_bfloat16* zb = nullptr;  // [Rmax][I]
+  __nv_bfloat16* Qb = nullptr;  // [Rmax][rmax]
+  int* err = nullptr;           // device error word
 };
 
 struct ProfRec {
@@ -133,6 +215,8 @@ struct lx_layer {
   const void** d_w_upU = nullptr;   // per node: corr [Ug;Uu] [2I][r] (null for anchors)
   const void** d_w_dn = nullptr;    // per node: anchor Wd [H][I] | corr Vd^T [r][I]
   const void** d_w_dnU = nullptr;   // per node: corr Ud [H][r] (null for anchors)
+  CUtensorMap* d_tmaps = nullptr;   // [N_OPS][N] TMA descriptors (bf16 layers)
+  bool stream_ok = false;           // the streaming kernels support this layer
   std::vector<const void*> h_w_up, h_w_upU, h_w_dn, h_w_dnU;  // same, host copies
   void* router_w = nullptr;         // [E][H]
   float* router_bias = nullptr;     // [E] or null
@@ -159,11 +243,22 @@ struct ProfScope {
 };
 
 // kernels / launchers (defined in the .cu files)
-lx_status launch_router(lx_layer* L, const void* x, int T, int k, int* topk_id, float* topk_w,
-                        float* logits, cudaStream_t s);
+lx_status launch_router_logits(lx_layer* L, const void* x, int T, float* logits, cudaStream_t s);
 lx_status launch_bucket(lx_layer* L, const int* topk_id, int T, int k, cudaStream_t s);
 lx_status launch_generic_experts(lx_layer* L, const void* x, int T, int k, void* y,
                                  cudaStream_t s);
+lx_status launch_swiglu(lx_layer* L, int k, void* z, bool z_bf16, cudaStream_t s);
+lx_status launch_combine(lx_layer* L, int T, int k, void* y, cudaStream_t s);
+lx_status launch_fast_experts(lx_layer* L, const void* x, int T, int k, void* y, cudaStream_t s);
+lx_status launch_stream(lx_layer* L, const StreamLaunch& P, cudaStream_t s, const char* name);
+lx_status launch_topk(lx_layer* L, const float* logits, int T, int k, int* topk_id,
+                      float* topk_w, cudaStream_t s);
+lx_status launch_bucket_small(lx_layer* L, const float* logits, const int* ids_in, int T, int k,
+                              int* topk_id, float* topk_w, cudaStream_t s);
+bool bucket_small_fits(const lx_layer* L, int T, int k);
+int stream_tile_rows();
+int stream_tile_tokens();
+int stream_box();
 
 OpShape op_shape(const lx_layer* L, int op);
 int op_max_items(const lx_layer* L);

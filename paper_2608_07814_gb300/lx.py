@@ -51,7 +51,8 @@ class LayerInfo(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in (
         "d_model", "d_ff", "n_experts", "n_nodes", "dtype", "n_anchors", "n_corrections",
         "max_depth", "max_rank")] + [("weight_bytes", ctypes.c_int64)] + [
-        (n, ctypes.c_int32) for n in ("last_T", "last_k", "last_rows")]
+        (n, ctypes.c_int32) for n in ("last_T", "last_k", "last_rows", "device_error",
+                                      "stream_path")]
 
 
 class KernelTime(ctypes.Structure):

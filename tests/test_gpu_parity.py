@@ -73,6 +73,7 @@ def check_forward(src, L, x, k, sample=None, path=lx.LX_PATH_AUTO, tol=None):
     toks = np.arange(x.shape[0]) if sample is None else np.asarray(sample)
     ref = oracle.moe_forward(src, x, k, token_subset=toks)
     err = _rel(yh[toks], ref)
+    assert L.info()["device_error"] == 0
     assert np.all(np.isfinite(yh))
     assert err <= (tol or TOL[src.dtype]), f"rel err {err}"
     return err
@@ -100,7 +101,22 @@ SMALL = {
                                           factor_std="visible", skew=synth.TREE_SKEW),
     "tree_fp32": lambda: synth.tree_layer(128, 64, 2, 2, 3, 24, 8, 4, "f32", seed=8,
                                           factor_std="visible", skew=synth.TREE_SKEW),
+    # served by the weight-streaming (TMA) kernels: dims and ranks multiples of 64
+    "stream_flat": lambda: synth.flat_layer(512, 384, [4] * 8, 64, 8, "bf16", seed=13,
+                                            factor_std="visible", skew=synth.QWEN_SKEW),
+    "stream_flat_zero_dom": lambda: synth.flat_layer(512, 384, [4] * 8, 64, 8, "bf16", seed=13,
+                                                     factor_std="visible", zero_dominants=True,
+                                                     skew=synth.QWEN_SKEW),
+    "stream_flat_zero_fac": lambda: synth.flat_layer(512, 384, [4] * 8, 64, 8, "bf16", seed=13,
+                                                     zero_factors=True, skew=synth.QWEN_SKEW),
+    "stream_singletons_mixed": lambda: synth.flat_layer(320, 448, [1, 3, 1, 5, 2], [64, 128, 192,
+                                                        64, 64, 128, 192], 3, "bf16",
+                                                        seed=14, factor_std="visible"),
+    "stream_tree": lambda: synth.tree_layer(256, 192, 2, 4, 3, 128, 64, 8, "bf16", seed=15,
+                                            factor_std="visible", skew=synth.TREE_SKEW),
 }
+
+STREAM = [n for n in SMALL if n.startswith("stream")]
 
 
 @pytest.mark.parametrize("name", sorted(SMALL))
@@ -114,6 +130,21 @@ def test_small_route_bucket_forward(name, T):
     check_forward(src, L, x, src.top_k, path=lx.LX_PATH_GENERIC)
 
 
+@pytest.mark.parametrize("name", STREAM)
+def test_stream_path_serves_layer(name):
+    src, L = installed(name, SMALL[name])
+    assert L.info()["stream_path"] == 1
+
+
+@pytest.mark.parametrize("T", [64, 256, 257])
+def test_stream_generic_boundary(T):
+    src, L = installed("stream_flat", SMALL["stream_flat"])
+    x = synth.tokens(src, T, seed=300 + T)
+    ids, _ = check_route(src, L, x, src.top_k)
+    check_buckets(src, L, ids)
+    check_forward(src, L, x, src.top_k)
+
+
 def test_tiny_fp32_config_full():
     """The tiny fp32 workload: 256 tokens, top-2, rank-8 SVD members."""
     src, L = installed("tiny_fp32", SMALL["tiny_fp32"])
@@ -122,9 +153,10 @@ def test_tiny_fp32_config_full():
     check_forward(src, L, x, 2)
 
 
+@pytest.mark.parametrize("name", ["flat_bf16_visible", "stream_flat"])
 @pytest.mark.parametrize("k", [1, 3, 8])
-def test_other_k(k):
-    src, L = installed("flat_bf16_visible", SMALL["flat_bf16_visible"])
+def test_other_k(name, k):
+    src, L = installed(name, SMALL[name])
     x = synth.tokens(src, 64, seed=100 + k)
     check_route(src, L, x, k)
     check_forward(src, L, x, k)
@@ -144,7 +176,7 @@ def test_ties_go_to_lower_id():
 
 
 def test_all_tokens_on_one_cluster():
-    src = synth.flat_layer(256, 128, [4] * 4, 16, 4, "bf16", seed=10, factor_std="visible")
+    src = synth.flat_layer(256, 128, [4] * 4, 64, 4, "bf16", seed=10, factor_std="visible")
     src.router_bias = np.zeros(16, np.float32)
     src.router_bias[src.meta["clusters"][2]] = 50.0
     L = lx.Layer(src)
