@@ -148,14 +148,21 @@ def kernel_bytes(name, st, src, esz):
     Ra, Rc, ta = st["R_anchor"], st["R_corr"], st["touched_anchor"]
     rt, rr = st["corr_r_touched"], st["corr_r_rows"]
     T, k = st["T"], st["k"]
+    Ra_c = Ra + Rc
     table = {
-        "router": E * H * esz + T * H * esz + T * k * 8,
+        "router": E * H * esz + T * H * esz + T * E * 4,
         "generic_up_anchor": ta * 2 * I * H * esz + Ra * H * esz + Ra * 2 * I * 4,
         "generic_up_V": rt * 2 * H * esz + Rc * H * esz + rr * 2 * 4,
         "generic_up_U": rt * 2 * I * esz + rr * 2 * 4 + Rc * 2 * I * 4,
         "generic_dn_anchor": ta * H * I * esz + Ra * I * 4 + Ra * H * 4,
         "generic_dn_V": rt * I * esz + Rc * I * 4 + rr * 4,
         "generic_dn_U": rt * H * esz + rr * 4 + Rc * H * 4,
+        # streaming kernels: weights once, activations in, results out
+        "stream_up_anchor_V": (ta * 2 * I * H + rt * 2 * H) * esz + Ra_c * H * esz
+                              + Ra * 2 * I * 4 + rr * 2 * 2,
+        "stream_up_U": rt * 2 * I * esz + rr * 2 * 2 + Rc * 2 * I * 4,
+        "stream_dn_anchor_V": (ta * H * I + rt * I) * esz + Ra_c * I * 2 + Ra * H * 4 + rr * 2,
+        "stream_dn_U": rt * H * esz + rr * 2 + Rc * H * 4,
     }
     return table.get(name)
 
@@ -223,17 +230,37 @@ def run_lx(args, rank, world, local_rank):
         layers[i % n_copies].moe_forward(xs[i % n_batches], k, ys[i % n_batches])
     torch.cuda.synchronize()
 
+    def steps(n):
+        for i in range(n):
+            layers[i % n_copies].moe_forward(xs[i % n_batches], k, ys[i % n_batches])
+
+    # One profiled pass of the same steps fills each layer's event pool, so the
+    # capture below creates no events.
     for L in layers:
         L.read_profile()
         L.set_profiling(True)
+    steps(args.steps)
+    torch.cuda.synchronize()
+    for L in layers:
+        L.read_profile(cap=1 << 20)
+    graph = None
+    if not args.no_graph:
+        # The timed region is one CUDA graph of the K forwards: the GPU runs the
+        # launches back to back, with the library's per-kernel events as
+        # external event nodes stamped by the replay.
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            steps(args.steps)
     if world > 1:
         torch.distributed.barrier()
     torch.cuda.synchronize()
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     t_wall0 = time.time()
     ev0.record(stream)
-    for i in range(args.steps):
-        layers[i % n_copies].moe_forward(xs[i % n_batches], k, ys[i % n_batches])
+    if graph is not None:
+        graph.replay()
+    else:
+        steps(args.steps)
     ev1.record(stream)
     torch.cuda.synchronize()
     if world > 1:
@@ -323,7 +350,9 @@ def run_lx(args, rank, world, local_rank):
                    "tokens_per_step": T, "layer_bytes": wbytes, "layer_copies": n_copies,
                    "l2": f"{n_copies} rotating device copies of the layer and 8 token batches "
                          "(inputs larger than L2)",
-                   "parallelism": f"replica per GPU x{world}"},
+                   "parallelism": f"replica per GPU x{world}",
+                   "timing": "one CUDA graph of the K forwards" if graph is not None
+                             else "K forwards launched one by one"},
         "roofline": roof,
         "kernels": {n: {"launches": counts[n], "avg_us": round(totals[n] / counts[n] * 1e3, 2),
                         "share": round(totals[n] / sum(totals.values()), 4)} for n in totals},
@@ -403,6 +432,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--ref-tokens", type=int, default=8)
+    ap.add_argument("--no-graph", action="store_true",
+                    help="launch the timed steps one by one instead of as one CUDA graph")
     ap.add_argument("--copies", type=int, default=None,
                     help="device copies of the layer rotated between steps (default 4 for decode)")
     args = ap.parse_args()

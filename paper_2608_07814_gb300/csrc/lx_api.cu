@@ -39,10 +39,19 @@ static cudaEvent_t take_event(lx_layer* L) {
   return e;
 }
 
+// Under stream capture the events become external record nodes of the graph,
+// so every replay stamps them.
+static void record(cudaEvent_t e, cudaStream_t s) {
+  cudaStreamCaptureStatus st = cudaStreamCaptureStatusNone;
+  cudaStreamIsCapturing(s, &st);
+  if (st == cudaStreamCaptureStatusActive) cudaEventRecordWithFlags(e, s, cudaEventRecordExternal);
+  else cudaEventRecord(e, s);
+}
+
 ProfScope::ProfScope(lx_layer* L_, cudaStream_t s_, const char* n) : L(L_), s(s_), name(n) {
   if (L->profiling) {
     b = take_event(L);
-    if (b) cudaEventRecord(b, s);
+    if (b) record(b, s);
   }
 }
 
@@ -50,7 +59,7 @@ ProfScope::~ProfScope() {
   if (L->profiling && b) {
     cudaEvent_t e = take_event(L);
     if (e) {
-      cudaEventRecord(e, s);
+      record(e, s);
       L->prof.push_back(ProfRec{name, b, e});
     } else {
       L->event_pool.push_back(b);
@@ -86,6 +95,25 @@ static lx_status ensure_workspace(lx_layer* L, int T, int k, cudaStream_t s) {
   const long keys = (long)L->N + L->E;
   const long Rmax = std::max<long>(1, (long)cT * std::min<long>(L->N, (long)ck * D));
   const long rmax = std::max(1, L->max_rank);
+  // streaming tile descriptors: per launch group, at most ceil(T/64) token
+  // blocks of every node's column tiles
+  long scap = 0;
+  if (L->stream_ok) {
+    const long tb = (cT + stream_tile_tokens() - 1) / stream_tile_tokens();
+    for (int g = 0; g < N_STREAM_GROUPS; ++g) {
+      long tot = 0;
+      for (int j = 0; j < 2; ++j) {
+        const int op = stream_group_op(g, j);
+        if (op < 0) continue;
+        const OpShape sh = op_shape(L, op);
+        for (int n : (sh.on_anchors ? L->anchors : L->corrs)) {
+          const long Ng = sh.n_const + (long)sh.n_rank * L->rank[n];
+          tot += tb * sh.groups * ((Ng + stream_tile_rows() - 1) / stream_tile_rows());
+        }
+      }
+      scap = std::max(scap, tot);
+    }
+  }
   struct Item { void** p; size_t bytes; };
   std::vector<Item> items = {
       {(void**)&w.logits, sizeof(float) * cT * L->E},
@@ -108,6 +136,8 @@ static lx_status ensure_workspace(lx_layer* L, int T, int k, cudaStream_t s) {
       {(void**)&w.Pb, 2 * Rmax * 2 * rmax},
       {(void**)&w.zb, 2 * Rmax * L->I},
       {(void**)&w.Qb, 2 * Rmax * rmax},
+      {(void**)&w.stiles, sizeof(int4) * 2 * N_STREAM_GROUPS * std::max<long>(1, scap)},
+      {(void**)&w.stile_cnt, sizeof(int) * N_STREAM_GROUPS},
       {(void**)&w.err, 256},
   };
   size_t total = 0;
@@ -135,6 +165,7 @@ static lx_status ensure_workspace(lx_layer* L, int T, int k, cudaStream_t s) {
   if (e != cudaSuccess) return cuda_fail(e, "clear workspace error word");
   w.cap_T = cT;
   w.cap_k = ck;
+  w.stile_cap = (int)scap;
   L->last_T = L->last_k = 0;
   return LX_OK;
 }
@@ -175,13 +206,12 @@ static bool use_stream(const lx_layer* L, int T) {
   return L->path_mode == LX_PATH_AUTO && L->stream_ok && T <= kStreamMaxT;
 }
 
-// TMA descriptors of every weight matrix the streaming kernels read.
+// TMA descriptors of every weight matrix the streaming kernels read: each
+// matrix is a 4-D tensor {64 K, 64 rows, K/64 tiles, rows/64 tiles} over the
+// tiled layout, read one 64x64 box (8 KiB, contiguous) at a time.
 static lx_status encode_tensor_maps(lx_layer* L, cudaStream_t s) {
   L->stream_ok = false;
-  if (L->dtype != LX_BF16) return LX_OK;
-  if (L->H % 64 || L->I % 64) return LX_OK;
-  for (int n = 0; n < L->N; ++n)
-    if (L->parent[n] >= 0 && L->rank[n] % 64) return LX_OK;
+  if (!L->tiled) return LX_OK;
   void* fn = nullptr;
   cudaDriverEntryPointQueryResult q;
   cudaError_t ce = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000,
@@ -202,11 +232,11 @@ static lx_status encode_tensor_maps(lx_layer* L, cudaStream_t s) {
                          : op == OP_UP_U                     ? L->h_w_upU[n]
                          : op == OP_DN_U                     ? L->h_w_dnU[n]
                                                              : L->h_w_dn[n];
-      const cuuint64_t dims[2] = {K, rows};
-      const cuuint64_t strides[1] = {K * 2};
-      const cuuint32_t box[2] = {(cuuint32_t)stream_box(), (cuuint32_t)stream_tile_rows()};
-      const cuuint32_t estr[2] = {1, 1};
-      CUresult cr = encode(&maps[(size_t)op * L->N + n], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+      const cuuint64_t dims[4] = {64, 64, K / 64, rows / 64};
+      const cuuint64_t strides[3] = {128, 8192, (K / 64) * 8192};
+      const cuuint32_t box[4] = {64, 64, 1, 1};
+      const cuuint32_t estr[4] = {1, 1, 1, 1};
+      CUresult cr = encode(&maps[(size_t)op * L->N + n], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4,
                            const_cast<void*>(base), dims, strides, box, estr,
                            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
@@ -315,7 +345,13 @@ extern "C" lx_status lx_load_compressed_layer(const lx_layer_desc* d, const void
   if (ce != cudaSuccess) return cleanup(cuda_fail(ce, "cudaGetDevice"));
   cudaDeviceGetAttribute(&L->num_sms, cudaDevAttrMultiProcessorCount, L->device);
 
-  // ---- weight arena layout
+  // ---- weight arena layout.  Layers the streaming kernels serve (bf16, every
+  // dimension and rank a multiple of 64) store each weight matrix [rows][K] as
+  // 64x64 tiles [rows/64][K/64][64][64]: one TMA box is then one contiguous
+  // 8 KiB run, and a 64-row block's whole K extent is sequential in memory.
+  L->tiled = L->dtype == LX_BF16 && L->H % 64 == 0 && L->I % 64 == 0;
+  for (int n = 0; n < L->N; ++n)
+    if (L->parent[n] >= 0 && L->rank[n] % 64) L->tiled = false;
   const long H = L->H, I = L->I, esz = L->esz;
   struct Piece { int node; int slot; size_t off; size_t bytes; };
   std::vector<Piece> pieces;
@@ -348,7 +384,7 @@ extern "C" lx_status lx_load_compressed_layer(const lx_layer_desc* d, const void
   L->h_w_upU.assign(L->N, nullptr);
   L->h_w_dn.assign(L->N, nullptr);
   L->h_w_dnU.assign(L->N, nullptr);
-  std::vector<char> stage;
+  std::vector<char> stage, tiled;
   for (const Piece& p : pieces) {
     char* dst = (char*)L->arena + p.off;
     const int n = p.node;
@@ -381,7 +417,24 @@ extern "C" lx_status lx_load_compressed_layer(const lx_layer_desc* d, const void
         L->h_w_dnU[n] = dst;
       }
     }
-    ce = cudaMemcpyAsync(dst, stage.data(), p.bytes, cudaMemcpyHostToDevice, s);
+    const char* src = stage.data();
+    if (L->tiled) {
+      const long r = L->parent[n] < 0 ? 0 : L->rank[n];
+      long rows, K;
+      if (L->parent[n] < 0) { rows = p.slot == 0 ? 2 * I : H; K = p.slot == 0 ? H : I; }
+      else if (p.slot == 0) { rows = 2 * r; K = H; }
+      else if (p.slot == 1) { rows = 2 * I; K = r; }
+      else if (p.slot == 2) { rows = r; K = I; }
+      else { rows = H; K = r; }
+      tiled.resize(p.bytes);
+      const long nkt = K / 64;
+      for (long row = 0; row < rows; ++row)
+        for (long kt = 0; kt < nkt; ++kt)
+          std::memcpy(tiled.data() + ((((row / 64) * nkt + kt) * 64 + row % 64) * 64) * esz,
+                      stage.data() + (row * K + kt * 64) * esz, 64 * esz);
+      src = tiled.data();
+    }
+    ce = cudaMemcpyAsync(dst, src, p.bytes, cudaMemcpyHostToDevice, s);
     if (ce == cudaSuccess) ce = cudaStreamSynchronize(s);
     if (ce != cudaSuccess) return cleanup(cuda_fail(ce, "copy weights"));
   }

@@ -98,13 +98,67 @@ struct PlanArgs {
 __device__ __forceinline__ int plan_tiles(const PlanArgs& pa, int p, int r, int rows) {
   const OpShape sh = pa.shape[p];
   const int Ng = sh.n_const + sh.n_rank * r;
-  return ((rows + pa.bm[p] - 1) / pa.bm[p]) * sh.groups * ((Ng + pa.bn[p] - 1) / pa.bn[p]);
+  int ncol = (Ng + pa.bn[p] - 1) / pa.bn[p];
+  if (p >= PLAN_STREAM) {
+    const int ncb = stream_col_blocks(sh.k_const + sh.k_rank * r, ncol);
+    ncol = (ncol + ncb - 1) / ncb;
+  }
+  return ((rows + pa.bm[p] - 1) / pa.bm[p]) * sh.groups * ncol;
+}
+
+
+// Expands the streaming plans (plans PLAN_STREAM + op) into one flat list of
+// tile descriptors per launch group (see StreamLaunch).  Called by one CTA
+// after the plans are written; node_off and rank may live in shared memory.
+__device__ void expand_stream_tiles(const PlanArgs& pa, const int* tile_off, int toff_stride,
+                                    const int* const* items, const int* node_off, const int* rank,
+                                    int4* tiles, int* cnt, int cap) {
+  for (int g = 0; g < N_STREAM_GROUPS; ++g) {
+    int tot[2] = {0, 0};
+    for (int j = 0; j < 2; ++j) {
+      const int op = stream_group_op(g, j);
+      if (op >= 0) tot[j] = tile_off[op * toff_stride + pa.n_items[PLAN_STREAM + op]];
+    }
+    const int total = min(tot[0] + tot[1], cap);
+    if (threadIdx.x == 0) cnt[g] = total;
+    int4* out = tiles + (size_t)g * cap * 2;
+    for (int idx = threadIdx.x; idx < total; idx += blockDim.x) {
+      const int j = idx < tot[0] ? 0 : 1;
+      const int op = stream_group_op(g, j);
+      const int p = PLAN_STREAM + op;
+      const int local0 = idx - (j ? tot[0] : 0);
+      const int* to = tile_off + op * toff_stride;
+      int lo = 0, hi = pa.n_items[p];
+      while (hi - lo > 1) {
+        const int mid = (lo + hi) >> 1;
+        if (to[mid] <= local0) lo = mid; else hi = mid;
+      }
+      const int n = items[op][lo];
+      const int local = local0 - to[lo];
+      const OpShape sh = pa.shape[p];
+      const int r = rank[n];
+      const int Ng = sh.n_const + sh.n_rank * r, K = sh.k_const + sh.k_rank * r;
+      const int ncol = (Ng + pa.bn[p] - 1) / pa.bn[p];
+      const int ncb = stream_col_blocks(K, ncol);
+      const int nct = (ncol + ncb - 1) / ncb;
+      const int per_tb = nct * sh.groups;
+      const int tb = local / per_tb, rem = local % per_tb;
+      const int ct = rem % nct;
+      const int tok0 = node_off[n] + tb * pa.bm[p];
+      const int M = min(pa.bm[p], node_off[n + 1] - tok0);
+      const int cbs = min(ncb, ncol - ct * ncb);
+      out[2 * idx] = make_int4(op, n, ct * ncb * pa.bn[p], tok0);
+      out[2 * idx + 1] = make_int4(M, K, Ng, (rem / nct) | (cbs << 4));
+    }
+  }
 }
 
 // one CTA: node/expert offsets and the tile prefix of every plan
 __global__ void k_offsets_plan(const int* __restrict__ key_cnt, int N, int E,
                                int* __restrict__ key_off, const int* __restrict__ rank,
-                               int* __restrict__ tile_off, int max_items, PlanArgs pa) {
+                               int* __restrict__ tile_off, int max_items, PlanArgs pa,
+                               int4* __restrict__ stiles, int* __restrict__ stile_cnt,
+                               int stile_cap) {
   // node offsets then expert offsets
   for (int part = 0; part < 2; ++part) {
     const int n0 = part == 0 ? 0 : N, cnt = part == 0 ? N : E;
@@ -138,6 +192,12 @@ __global__ void k_offsets_plan(const int* __restrict__ key_cnt, int N, int E,
     }
     if (threadIdx.x == 0) to[pa.n_items[p]] = carry;
     __syncthreads();
+  }
+  if (stiles) {
+    const int* its[N_OPS];
+    for (int op = 0; op < N_OPS; ++op) its[op] = pa.items[PLAN_STREAM + op];
+    expand_stream_tiles(pa, tile_off + PLAN_STREAM * (max_items + 1), max_items + 1, its, key_off,
+                        rank, stiles, stile_cnt, stile_cap);
   }
 }
 
@@ -195,9 +255,11 @@ constexpr int SB_THREADS = 1024;
 constexpr int SB_MAX_T = 256;
 constexpr size_t SB_SMEM_LIMIT = 160 * 1024;
 
-__host__ __device__ inline size_t sb_smem(int T, int k, int keys) {
+__host__ __device__ inline size_t sb_smem(int T, int k, int keys, int E, int N, int max_items) {
   const size_t Tp = ((size_t)T + 15) / 16 * 16;
-  return (size_t)T * k * 4 + 2 * (size_t)keys * Tp + (size_t)keys * 4 + ((size_t)keys + 2) * 4 + 64;
+  return (size_t)T * k * 4 + 2 * (size_t)keys * Tp + (size_t)keys * 4 + ((size_t)keys + 2) * 4 +
+         (size_t)E * (LX_MAX_DEPTH + 1) * 4 + (size_t)N * 4 +
+         (size_t)N_OPS * (max_items + 1) * 4 + (size_t)N * 4 + 64;
 }
 
 __global__ void __launch_bounds__(SB_THREADS)
@@ -206,7 +268,8 @@ k_bucket_small(const float* __restrict__ logits, const int* __restrict__ ids_in,
                const int* __restrict__ path_len, const int* __restrict__ rank,
                int* __restrict__ topk_id, float* __restrict__ topk_w, int* __restrict__ key_off_g,
                int* __restrict__ node_tok, int* __restrict__ row_node, int* __restrict__ node_row,
-               int* __restrict__ perm, int* __restrict__ tile_off, int max_items, PlanArgs pa) {
+               int* __restrict__ perm, int* __restrict__ tile_off, int max_items, PlanArgs pa,
+               int4* __restrict__ stiles, int* __restrict__ stile_cnt, int stile_cap) {
   extern __shared__ __align__(16) unsigned char sm[];
   const int keys = N + E;
   const int Tp = (T + 15) & ~15;
@@ -215,9 +278,23 @@ k_bucket_small(const float* __restrict__ logits, const int* __restrict__ ids_in,
   uint8_t* rk = marks + (size_t)keys * Tp;
   int* cnt = reinterpret_cast<int*>(rk + (((size_t)keys * Tp + 3) & ~(size_t)3));
   int* off = cnt + keys;
+  int* spaths = off + keys + 2;                 // [E][LX_MAX_DEPTH]
+  int* splen = spaths + E * LX_MAX_DEPTH;       // [E]
+  int* srank = splen + E;                       // [N]
+  int* stoff = srank + N;                       // [N_OPS][max_items+1] streaming plans
+  int* sitems = stoff + N_OPS * (max_items + 1); // anchors then corrections
   const int tid = threadIdx.x, nth = blockDim.x;
   const int warp = tid >> 5, lane = tid & 31, nw = nth >> 5;
-
+  for (int i = tid; i < E * LX_MAX_DEPTH; i += nth) spaths[i] = paths[i];
+  for (int i = tid; i < E; i += nth) splen[i] = path_len[i];
+  for (int i = tid; i < N; i += nth) srank[i] = rank[i];
+  const int n_anc = pa.n_items[PLAN_STREAM + OP_UP_ANCHOR], n_cor = pa.n_items[PLAN_STREAM + OP_UP_V];
+  for (int i = tid; i < n_anc; i += nth) sitems[i] = pa.items[PLAN_STREAM + OP_UP_ANCHOR][i];
+  for (int i = tid; i < n_cor; i += nth) sitems[n_anc + i] = pa.items[PLAN_STREAM + OP_UP_V][i];
+  {
+    uint32_t* m32 = reinterpret_cast<uint32_t*>(marks);  // keys*Tp is a multiple of 16
+    for (int i = tid; i < keys * Tp / 4; i += nth) m32[i] = 0;
+  }
   // 1. routing (or the given ids)
   if (logits) {
     for (int t = warp; t < T; t += nw) {
@@ -233,23 +310,27 @@ k_bucket_small(const float* __restrict__ logits, const int* __restrict__ ids_in,
   } else {
     for (int i = tid; i < T * k; i += nth) ids[i] = ids_in[i];
   }
-  for (int i = tid; i < keys * Tp; i += nth) marks[i] = 0;
   __syncthreads();
   // 2. marks
   for (int a = tid; a < T * k; a += nth) {
     const int t = a / k, e = ids[a];
     if (e < 0 || e >= E) continue;
     marks[(N + e) * Tp + t] = 1;
-    const int len = path_len[e];
-    for (int l = 0; l < len; ++l) marks[paths[e * LX_MAX_DEPTH + l] * Tp + t] = 1;
+    const int len = splen[e];
+    for (int l = 0; l < len; ++l) marks[spaths[e * LX_MAX_DEPTH + l] * Tp + t] = 1;
   }
   __syncthreads();
-  // 3. per-key ranks in token order
-  for (int key = tid; key < keys; key += nth) {
-    int c = 0;
-    for (int t = 0; t < T; ++t)
-      if (marks[key * Tp + t]) rk[key * Tp + t] = (uint8_t)c++;
-    cnt[key] = c;
+  // 3. per-key ranks in token order (warp ballots)
+  for (int key = warp; key < keys; key += nw) {
+    int running = 0;
+    for (int t0 = 0; t0 < T; t0 += 32) {
+      const int t = t0 + lane;
+      const bool m = t < T && marks[key * Tp + t];
+      const uint32_t b = __ballot_sync(0xffffffffu, m);
+      if (m) rk[key * Tp + t] = (uint8_t)(running + __popc(b & ((1u << lane) - 1u)));
+      running += __popc(b);
+    }
+    if (lane == 0) cnt[key] = running;
   }
   __syncthreads();
   // 4. node offsets then expert offsets
@@ -269,56 +350,58 @@ k_bucket_small(const float* __restrict__ logits, const int* __restrict__ ids_in,
     __syncthreads();
   }
   for (int i = tid; i < keys + 2; i += nth) key_off_g[i] = off[i];
-  // 5. scatter
-  for (int idx = tid; idx < keys * T; idx += nth) {
-    const int key = idx / T, t = idx % T;
-    if (!marks[key * Tp + t]) continue;
-    const int r = rk[key * Tp + t];
-    if (key < N) {
-      const int row = off[key] + r;
-      node_tok[row] = t;
-      row_node[row] = key;
-    } else {
-      const int e = key - N;
-      const int pos = off[N + 1 + e] + r;
-      for (int s = 0; s < k; ++s)
-        if (ids[t * k + s] == e) {
-          perm[pos] = t * k + s;
-          break;
-        }
+  // 5. tile plans: one warp per plan
+  for (int p = warp; p < pa.n_plans; p += nw) {
+    int* to = tile_off + p * (max_items + 1);
+    int carry = 0;
+    for (int base = 0; base < pa.n_items[p]; base += 32) {
+      const int i = base + lane;
+      int v = 0;
+      if (i < pa.n_items[p]) {
+        const int n = pa.items[p][i];
+        v = plan_tiles(pa, p, srank[n], cnt[n]);
+      }
+      int incl = v;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int x = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += x;
+      }
+      if (i < pa.n_items[p]) {
+        to[i] = carry + incl - v;
+        if (p >= PLAN_STREAM) stoff[(p - PLAN_STREAM) * (max_items + 1) + i] = carry + incl - v;
+      }
+      carry += __shfl_sync(0xffffffffu, incl, 31);
+    }
+    if (lane == 0) {
+      to[pa.n_items[p]] = carry;
+      if (p >= PLAN_STREAM) stoff[(p - PLAN_STREAM) * (max_items + 1) + pa.n_items[p]] = carry;
     }
   }
-  // 6. rows of every (assignment, path level)
+  // 6. scatter from the assignments: bucket rows, node rows, permutation
   for (int a = tid; a < T * k; a += nth) {
     const int t = a / k, e = ids[a];
-    const int len = (e >= 0 && e < E) ? path_len[e] : 0;
+    const bool valid = e >= 0 && e < E;
+    const int len = valid ? splen[e] : 0;
+    if (valid) perm[off[N + 1 + e] + rk[(N + e) * Tp + t]] = a;
     for (int l = 0; l < D; ++l) {
       int row = -1;
       if (l < len) {
-        const int n = paths[e * LX_MAX_DEPTH + l];
+        const int n = spaths[e * LX_MAX_DEPTH + l];
         row = off[n] + rk[n * Tp + t];
+        node_tok[row] = t;   // (t, n) pairs shared by several slots write the same values
+        row_node[row] = n;
       }
       node_row[(size_t)a * D + l] = row;
     }
   }
-  // 7. tile plans
-  for (int p = 0; p < pa.n_plans; ++p) {
-    int* to = tile_off + p * (max_items + 1);
-    int carry = 0;
-    for (int base = 0; base < pa.n_items[p]; base += nth) {
-      const int i = base + tid;
-      int v = 0;
-      if (i < pa.n_items[p]) {
-        const int n = pa.items[p][i];
-        v = plan_tiles(pa, p, rank[n], cnt[n]);
-      }
-      int total;
-      const int ex = block_excl_scan(v, &total);
-      if (i < pa.n_items[p]) to[i] = carry + ex;
-      carry += total;
-    }
-    if (tid == 0) to[pa.n_items[p]] = carry;
-    __syncthreads();
+  __syncthreads();
+  // 7. streaming tile descriptors (plans and item lists from shared memory)
+  if (stiles) {
+    const int* its[N_OPS];
+    for (int op = 0; op < N_OPS; ++op)
+      its[op] = pa.shape[PLAN_STREAM + op].on_anchors ? sitems : sitems + n_anc;
+    expand_stream_tiles(pa, stoff, max_items + 1, its, off, srank, stiles, stile_cnt, stile_cap);
   }
 }
 
@@ -340,21 +423,24 @@ static PlanArgs make_plans(const lx_layer* L, int n_plans) {
 }
 
 bool bucket_small_fits(const lx_layer* L, int T, int k) {
-  return T <= SB_MAX_T && sb_smem(T, k, L->N + L->E) <= SB_SMEM_LIMIT;
+  return T <= SB_MAX_T &&
+         sb_smem(T, k, L->N + L->E, L->E, L->N, op_max_items(L)) <= SB_SMEM_LIMIT;
 }
 
 lx_status launch_bucket_small(lx_layer* L, const float* logits, const int* ids_in, int T, int k,
                               int* topk_id, float* topk_w, cudaStream_t s) {
   Workspace& w = L->ws;
-  const size_t smem = sb_smem(T, k, L->N + L->E);
+  const size_t smem = sb_smem(T, k, L->N + L->E, L->E, L->N, op_max_items(L));
   const PlanArgs pa = make_plans(L, N_PLANS);
-  LX_CUDA(cudaFuncSetAttribute(k_bucket_small, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               (int)smem));
+  static bool done[64] = {};
+  LX_CUDA(smem_cap_once((const void*)k_bucket_small, (int)SB_SMEM_LIMIT, L->device, done));
   ProfScope ps(L, s, logits ? "topk_bucket_small" : "bucket_small");
   k_bucket_small<<<1, SB_THREADS, smem, s>>>(logits, ids_in, T, k, L->E, L->N, L->max_depth,
                                              L->d_paths, L->d_path_len, L->d_rank, topk_id, topk_w,
                                              w.key_off, w.node_tok, w.row_node, w.node_row, w.perm,
-                                             w.tile_off, op_max_items(L), pa);
+                                             w.tile_off, op_max_items(L), pa,
+                                             L->stream_ok ? w.stiles : nullptr, w.stile_cnt,
+                                             w.stile_cap);
   LX_CUDA(cudaGetLastError());
   return LX_OK;
 }
@@ -382,7 +468,8 @@ lx_status launch_bucket(lx_layer* L, const int* topk_id, int T, int k, cudaStrea
     const PlanArgs pa = make_plans(L, N_PLANS);
     ProfScope ps(L, s, "bucket_offsets");
     k_offsets_plan<<<1, 1024, 0, s>>>(w.key_cnt, L->N, L->E, w.key_off, L->d_rank, w.tile_off,
-                                      op_max_items(L), pa);
+                                      op_max_items(L), pa, L->stream_ok ? w.stiles : nullptr,
+                                      w.stile_cnt, w.stile_cap);
     LX_CUDA(cudaGetLastError());
   }
   {
@@ -488,7 +575,7 @@ extern "C" lx_status lx_bucket_noalloc(lx_layer* L, const int32_t* topk_id, int3
   LX_CUDA(cudaGetLastError());
   const PlanArgs pa = make_plans(L, N_OPS);
   k_offsets_plan<<<1, 1024, 0, s>>>(key_cnt, L->N, L->E, key_off, L->d_rank, tile_off,
-                                    op_max_items(L), pa);
+                                    op_max_items(L), pa, nullptr, nullptr, 0);
   LX_CUDA(cudaGetLastError());
   k_scatter<<<dim3((T + 255) / 256, (unsigned)keys), 256, 0, s>>>(
       marks, rank_in, key_off, topk_id, T, k, L->N, Tp, node_tok, row_node, perm);

@@ -71,7 +71,12 @@ k_grouped_gemm(GemmArgs g) {
       for (int idx = threadIdx.x; idx < G_BN * G_BK; idx += GG_THREADS) {
         const int j = idx / G_BK, kk = idx % G_BK;
         float v = 0.f;
-        if (col0 + j < Ng && k0 + kk < K) v = to_f32(W[(size_t)(col0 + j) * K + k0 + kk]);
+        if (col0 + j < Ng && k0 + kk < K) {
+          const int c = col0 + j, kx = k0 + kk;
+          const size_t wi = g.tiled ? ((((size_t)(c >> 6) * (K >> 6) + (kx >> 6)) * 64 + (c & 63)) * 64 + (kx & 63))
+                                    : (size_t)c * K + kx;
+          v = to_f32(W[wi]);
+        }
         Ws[kk][j] = v;
       }
       __syncthreads();
@@ -101,55 +106,108 @@ k_grouped_gemm(GemmArgs g) {
 
 __device__ __forceinline__ float silu_f(float v) { return v / (1.f + expf(-v)); }
 
-// z[row] for every (token, node) row
+// One CTA per token.  Its k selected experts' gated SwiGLU outputs,
+//   a_s = g_s * silu(sum_l h_gate[row(s,l)]) * sum_l h_up[row(s,l)],
+// are added, slot by slot in ascending order, into the z row of every node on
+// the slot's path: z[(t,n)] = sum_{s : n in path(e_s)} a_s.  Each thread owns
+// four columns; its per-row partial sums live in its own shared-memory slice.
+constexpr int SW_T = 256;
+
+
 template <typename TZ>
-__global__ void k_swiglu_aggregate(const int* __restrict__ key_off, int N,
-                                   const int* __restrict__ node_tok,
-                                   const int* __restrict__ row_node,
-                                   const int* __restrict__ topk_id,
-                                   const float* __restrict__ topk_w,
-                                   const int* __restrict__ node_row, int k, int D, int E,
-                                   const int* __restrict__ paths, const int* __restrict__ path_len,
-                                   const float* __restrict__ h, int I, TZ* __restrict__ z) {
-  const int R = key_off[N];
-  for (int row = blockIdx.x; row < R; row += gridDim.x) {
-    const int t = node_tok[row];
-    const int n = row_node[row];
-    for (int i = threadIdx.x; i < I; i += blockDim.x) {
-      float acc = 0.f;
-      for (int s = 0; s < k; ++s) {
-        const long a = (long)t * k + s;
-        const int e = topk_id[a];
-        if (e < 0 || e >= E) continue;
-        const int len = path_len[e];
-        bool on_path = false;
-        for (int l = 0; l < len; ++l) on_path |= paths[e * LX_MAX_DEPTH + l] == n;
-        if (!on_path) continue;
-        float pg = 0.f, pu = 0.f;
-        for (int l = 0; l < len; ++l) {
-          const int rr = node_row[a * D + l];
-          if (rr < 0) continue;
-          pg += h[(size_t)rr * 2 * I + i];
-          pu += h[(size_t)rr * 2 * I + I + i];
+__device__ __forceinline__ void store4(TZ* p, float4 v);
+template <>
+__device__ __forceinline__ void store4<float>(float* p, float4 v) {
+  *reinterpret_cast<float4*>(p) = v;
+}
+template <>
+__device__ __forceinline__ void store4<__nv_bfloat16>(__nv_bfloat16* p, float4 v) {
+  __nv_bfloat162 a = __floats2bfloat162_rn(v.x, v.y), b = __floats2bfloat162_rn(v.z, v.w);
+  uint2 u;
+  u.x = *reinterpret_cast<uint32_t*>(&a);
+  u.y = *reinterpret_cast<uint32_t*>(&b);
+  *reinterpret_cast<uint2*>(p) = u;
+}
+
+template <typename TZ>
+__global__ void __launch_bounds__(SW_T)
+k_swiglu_aggregate(const int* __restrict__ topk_id, const float* __restrict__ topk_w,
+                   const int* __restrict__ node_row, int T, int k, int D,
+                   const float* __restrict__ h, int I, TZ* __restrict__ z) {
+  extern __shared__ float4 zacc[];  // [distinct rows][SW_T]
+  __shared__ int rows[LX_MAX_K * LX_MAX_DEPTH], lrow[LX_MAX_K * LX_MAX_DEPTH];
+  __shared__ int drow[LX_MAX_K * LX_MAX_DEPTH];
+  __shared__ float gw[LX_MAX_K];
+  __shared__ int nd_s;
+  const int kD = k * D;
+  for (int t = blockIdx.x; t < T; t += gridDim.x) {
+    for (int j = threadIdx.x; j < kD; j += blockDim.x) rows[j] = node_row[(size_t)t * kD + j];
+    for (int j = threadIdx.x; j < k; j += blockDim.x) gw[j] = topk_w[(size_t)t * k + j];
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      int nd = 0;
+      for (int j = 0; j < kD; ++j) {
+        const int r = rows[j];
+        int d = -1;
+        if (r >= 0) {
+          for (int q = 0; q < nd; ++q)
+            if (drow[q] == r) d = q;
+          if (d < 0) { d = nd; drow[nd++] = r; }
         }
-        acc = fmaf(topk_w[a], silu_f(pg) * pu, acc);
+        lrow[j] = d;
       }
-      z[(size_t)row * I + i] = from_f32<TZ>(acc);
+      nd_s = nd;
     }
+    __syncthreads();
+    const int nd = nd_s;
+    for (int c0 = 0; c0 < I; c0 += 4 * SW_T) {
+      const int i = c0 + 4 * threadIdx.x;
+      if (i < I) {
+        for (int d = 0; d < nd; ++d) zacc[d * SW_T + threadIdx.x] = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 4
+        for (int sl = 0; sl < k; ++sl) {
+          float4 pg = make_float4(0.f, 0.f, 0.f, 0.f), pu = pg;
+          for (int l = 0; l < D; ++l) {
+            const int r = rows[sl * D + l];
+            if (r < 0) continue;
+            const float4 a = *reinterpret_cast<const float4*>(h + (size_t)r * 2 * I + i);
+            const float4 b = *reinterpret_cast<const float4*>(h + (size_t)r * 2 * I + I + i);
+            pg.x += a.x; pg.y += a.y; pg.z += a.z; pg.w += a.w;
+            pu.x += b.x; pu.y += b.y; pu.z += b.z; pu.w += b.w;
+          }
+          const float g = gw[sl];
+          const float4 act = make_float4(g * silu_f(pg.x) * pu.x, g * silu_f(pg.y) * pu.y,
+                                         g * silu_f(pg.z) * pu.z, g * silu_f(pg.w) * pu.w);
+          for (int l = 0; l < D; ++l) {
+            const int d = lrow[sl * D + l];
+            if (d < 0) continue;
+            float4& acc = zacc[d * SW_T + threadIdx.x];
+            acc.x += act.x; acc.y += act.y; acc.z += act.z; acc.w += act.w;
+          }
+        }
+        for (int d = 0; d < nd; ++d) store4<TZ>(z + (size_t)drow[d] * I + i, zacc[d * SW_T + threadIdx.x]);
+      }
+    }
+    __syncthreads();
   }
 }
 
-// y[t] = sum of ypart over t's distinct rows, ascending
+// y[t] = sum of ypart over t's distinct rows in ascending row (= node) order;
+// each thread owns four columns and issues four rows' loads at a time.
 template <typename TY>
-__global__ void k_combine(const int* __restrict__ node_row, int k, int D,
-                          const float* __restrict__ ypart, int H, TY* __restrict__ y, int T) {
+__global__ void __launch_bounds__(256)
+k_combine(const int* __restrict__ node_row, int k, int D, const float* __restrict__ ypart, int H,
+          TY* __restrict__ y, int T) {
+  __shared__ int raw_s[LX_MAX_K * LX_MAX_DEPTH];
   __shared__ int rows_s[LX_MAX_K * LX_MAX_DEPTH];
   __shared__ int nrows_s;
   for (int t = blockIdx.x; t < T; t += gridDim.x) {
+    for (int j = threadIdx.x; j < k * D; j += blockDim.x) raw_s[j] = node_row[(long)t * k * D + j];
+    __syncthreads();
     if (threadIdx.x == 0) {
       int m = 0;
       for (int j = 0; j < k * D; ++j) {
-        const int r = node_row[(long)t * k * D + j];
+        const int r = raw_s[j];
         if (r < 0) continue;
         bool dup = false;
         for (int q = 0; q < m; ++q) dup |= rows_s[q] == r;
@@ -162,10 +220,24 @@ __global__ void k_combine(const int* __restrict__ node_row, int k, int D,
     }
     __syncthreads();
     const int m = nrows_s;
-    for (int c = threadIdx.x; c < H; c += blockDim.x) {
-      float acc = 0.f;
-      for (int q = 0; q < m; ++q) acc += ypart[(size_t)rows_s[q] * H + c];
-      y[(size_t)t * H + c] = from_f32<TY>(acc);
+    for (int c = 4 * threadIdx.x; c < H; c += 4 * blockDim.x) {
+      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+      int q = 0;
+      for (; q + 4 <= m; q += 4) {
+        float4 v[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+          v[u] = *reinterpret_cast<const float4*>(ypart + (size_t)rows_s[q + u] * H + c);
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          acc.x += v[u].x; acc.y += v[u].y; acc.z += v[u].z; acc.w += v[u].w;
+        }
+      }
+      for (; q < m; ++q) {
+        const float4 v = *reinterpret_cast<const float4*>(ypart + (size_t)rows_s[q] * H + c);
+        acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
+      }
+      store4<TY>(y + (size_t)t * H + c, acc);
     }
     __syncthreads();
   }
@@ -173,18 +245,21 @@ __global__ void k_combine(const int* __restrict__ node_row, int k, int D,
 
 }  // namespace
 
-lx_status launch_swiglu(lx_layer* L, int k, void* z, bool z_bf16, cudaStream_t s) {
+lx_status launch_swiglu(lx_layer* L, int T, int k, void* z, bool z_bf16, cudaStream_t s) {
   Workspace& w = L->ws;
   ProfScope ps(L, s, z_bf16 ? "swiglu" : "generic_swiglu");
-  const dim3 grid(L->num_sms * 8);
-  if (z_bf16)
-    k_swiglu_aggregate<__nv_bfloat16><<<grid, 256, 0, s>>>(
-        w.key_off, L->N, w.node_tok, w.row_node, w.topk_id, w.topk_w, w.node_row, k,
-        L->max_depth, L->E, L->d_paths, L->d_path_len, w.h, L->I, (__nv_bfloat16*)z);
-  else
-    k_swiglu_aggregate<float><<<grid, 256, 0, s>>>(
-        w.key_off, L->N, w.node_tok, w.row_node, w.topk_id, w.topk_w, w.node_row, k,
-        L->max_depth, L->E, L->d_paths, L->d_path_len, w.h, L->I, (float*)z);
+  const int grid = std::min(T, L->num_sms * 8);
+  const size_t smem = sizeof(float4) * SW_T * k * L->max_depth;
+  static bool done_b[64] = {}, done_f[64] = {};
+  if (z_bf16) {
+    LX_CUDA(smem_cap_once((const void*)k_swiglu_aggregate<__nv_bfloat16>, 200 * 1024, L->device, done_b));
+    k_swiglu_aggregate<__nv_bfloat16><<<grid, SW_T, smem, s>>>(
+        w.topk_id, w.topk_w, w.node_row, T, k, L->max_depth, w.h, L->I, (__nv_bfloat16*)z);
+  } else {
+    LX_CUDA(smem_cap_once((const void*)k_swiglu_aggregate<float>, 200 * 1024, L->device, done_f));
+    k_swiglu_aggregate<float><<<grid, SW_T, smem, s>>>(w.topk_id, w.topk_w, w.node_row, T, k,
+                                                       L->max_depth, w.h, L->I, (float*)z);
+  }
   LX_CUDA(cudaGetLastError());
   return LX_OK;
 }
@@ -222,6 +297,7 @@ lx_status run_gemm(lx_layer* L, const void* A, long lda, const int* gather,
   g.shape = sh;
   g.out = out;
   g.ldo = ldo;
+  g.tiled = L->tiled ? 1 : 0;
   ProfScope ps(L, s, name);
   k_grouped_gemm<TA, TW, op><<<L->num_sms * 4, GG_THREADS, 0, s>>>(g);
   LX_CUDA(cudaGetLastError());
@@ -240,7 +316,7 @@ lx_status generic_impl(lx_layer* L, const void* x, int T, int k, void* y, cudaSt
                            2 * rmax, s, "generic_up_V")));
   LX_TRY((run_gemm<float, TX, OP_UP_U>(L, w.P, 2 * rmax, nullptr,
                               (const void* const*)L->d_w_upU, w.h, 2 * I, s, "generic_up_U")));
-  LX_TRY(launch_swiglu(L, k, w.z, false, s));
+  LX_TRY(launch_swiglu(L, T, k, w.z, false, s));
   // z-side products
   LX_TRY((run_gemm<float, TX, OP_DN_ANCHOR>(L, w.z, I, nullptr, (const void* const*)L->d_w_dn,
                               w.ypart, H, s, "generic_dn_anchor")));

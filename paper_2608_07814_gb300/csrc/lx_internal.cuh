@@ -53,27 +53,40 @@ __device__ __forceinline__ bool topk_better(float v, int i, float bv, int bi) {
   return v > bv || (v == bv && i < bi);
 }
 
-__device__ __forceinline__ void warp_topk(const float* lt, int E, int k, int& sel_id,
-                                          float& sel_w) {
+template <int EPL>  // candidates per lane: E <= 32 * EPL
+__device__ __forceinline__ void warp_topk_t(const float* lt, int E, int k, int& sel_id,
+                                            float& sel_w) {
   const int lane = threadIdx.x & 31;
+  float v[EPL];  // this lane's candidates e = lane + 32 i, in registers
+#pragma unroll
+  for (int i = 0; i < EPL; ++i) {
+    const int e = lane + 32 * i;
+    v[i] = e < E ? lt[e] : 0.f;
+  }
   uint32_t taken = 0;  // bit i <-> expert lane + 32 i
   float m = 0.f, denom = 0.f, selv = 0.f;
   int seli = 0;
   for (int j = 0; j < k; ++j) {
     float bv = -INFINITY;
     int bi = 0x7fffffff;
-    for (int i = 0, e = lane; e < E; ++i, e += 32)
-      if (!((taken >> i) & 1u) && topk_better(lt[e], e, bv, bi)) { bv = lt[e]; bi = e; }
+#pragma unroll
+    for (int i = 0; i < EPL; ++i) {
+      const int e = lane + 32 * i;
+      if (e < E && !((taken >> i) & 1u) && topk_better(v[i], e, bv, bi)) { bv = v[i]; bi = e; }
+    }
 #pragma unroll
     for (int off = 16; off >= 1; off >>= 1) {
       const float ov = __shfl_xor_sync(0xffffffffu, bv, off);
       const int oi = __shfl_xor_sync(0xffffffffu, bi, off);
       if (topk_better(ov, oi, bv, bi)) { bv = ov; bi = oi; }
     }
-    if (bi == 0x7fffffff) {
+    if (bi == 0x7fffffff) {  // only NaNs left: lowest free id
       int fi = 0x7fffffff;
-      for (int i = 0, e = lane; e < E; ++i, e += 32)
-        if (!((taken >> i) & 1u)) { fi = e; break; }
+#pragma unroll
+      for (int i = EPL - 1; i >= 0; --i) {
+        const int e = lane + 32 * i;
+        if (e < E && !((taken >> i) & 1u)) fi = e;
+      }
 #pragma unroll
       for (int off = 16; off >= 1; off >>= 1) fi = min(fi, __shfl_xor_sync(0xffffffffu, fi, off));
       bi = fi;
@@ -87,6 +100,15 @@ __device__ __forceinline__ void warp_topk(const float* lt, int E, int k, int& se
   }
   sel_id = seli;
   sel_w = selv / denom;
+}
+
+__device__ __forceinline__ void warp_topk(const float* lt, int E, int k, int& sel_id,
+                                          float& sel_w) {
+  if (E <= 32) warp_topk_t<1>(lt, E, k, sel_id, sel_w);
+  else if (E <= 64) warp_topk_t<2>(lt, E, k, sel_id, sel_w);
+  else if (E <= 128) warp_topk_t<4>(lt, E, k, sel_id, sel_w);
+  else if (E <= 256) warp_topk_t<8>(lt, E, k, sel_id, sel_w);
+  else warp_topk_t<32>(lt, E, k, sel_id, sel_w);
 }
 
 // ---------------------------------------------------------------------------
@@ -105,7 +127,8 @@ enum OpKind {
 
 // Tile plans: plan p < N_OPS is op p for the generic kernel (32-token x
 // 64-column tiles); plan N_OPS + p is op p for the streaming kernel (64-token
-// x 64-weight-row tiles).
+// x 64-weight-row blocks; ops with a short K take several column blocks per
+// tile, see stream_col_blocks).
 constexpr int N_PLANS = 2 * N_OPS;
 constexpr int PLAN_STREAM = N_OPS;
 
@@ -132,6 +155,7 @@ struct GemmArgs {
   OpShape shape;
   float* out;
   long ldo;
+  int tiled;               // W stored as [rows/64][K/64][64][64] tiles
 };
 
 // Streaming (decode) grouped GEMM: one op of a launch
@@ -151,9 +175,33 @@ struct StreamOp {
   const int* rank;
 };
 
+// The streaming launches: group 0 = {UP_ANCHOR, UP_V}, 1 = {UP_U},
+// 2 = {DN_ANCHOR, DN_V}, 3 = {DN_U}.  Each group's tiles are expanded on the
+// device into a flat list of descriptors
+//   a = {op, node, row0 (first weight row in the group), tok0 (first node row)}
+//   b = {M (tokens), K, Ng (rows per group), grp | column blocks << 4}
+constexpr int N_STREAM_GROUPS = 4;
+__host__ __device__ inline int stream_group_op(int g, int j) {
+  const int ops[N_STREAM_GROUPS][2] = {{OP_UP_ANCHOR, OP_UP_V}, {OP_UP_U, -1},
+                                       {OP_DN_ANCHOR, OP_DN_V}, {OP_DN_U, -1}};
+  return ops[g][j];
+}
+
+// Column blocks (of 64 weight rows) per streaming tile.  Measured on GB300:
+// one block per tile (more, smaller tiles spread over more CTAs) streams the
+// short-K factor products faster than grouping blocks, so tiles keep one.
+__host__ __device__ inline int stream_col_blocks(int K, int ncol) {
+  (void)K;
+  (void)ncol;
+  return 1;
+}
+
 struct StreamLaunch {
-  StreamOp op[2];
+  StreamOp op[2];            // op[j] serves descriptors whose op id is op_id[j]
+  int op_id[2];
   int n_ops;
+  const int4* tiles;         // [n_tiles][2] descriptors of this launch's group
+  const int* n_tiles;        // device count
   int* err;                  // device error word (LX_ERR_TIMEOUT on a bounded wait)
 };
 
@@ -188,6 +236,9 @@ struct Workspace {
   __nv_bfloat16* Pb = nullptr;  // [Rmax][2 rmax]
   __nv_bfloat16* zb = nullptr;  // [Rmax][I]
   __nv_bfloat16* Qb = nullptr;  // [Rmax][rmax]
+  int4* stiles = nullptr;       // [N_STREAM_GROUPS][stile_cap][2] tile descriptors
+  int* stile_cnt = nullptr;     // [N_STREAM_GROUPS]
+  int stile_cap = 0;
   int* err = nullptr;           // device error word
 };
 
@@ -217,6 +268,7 @@ struct lx_layer {
   const void** d_w_dnU = nullptr;   // per node: corr Ud [H][r] (null for anchors)
   CUtensorMap* d_tmaps = nullptr;   // [N_OPS][N] TMA descriptors (bf16 layers)
   bool stream_ok = false;           // the streaming kernels support this layer
+  bool tiled = false;               // weights stored as 64x64 tiles (see lx_api.cu)
   std::vector<const void*> h_w_up, h_w_upU, h_w_dn, h_w_dnU;  // same, host copies
   void* router_w = nullptr;         // [E][H]
   float* router_bias = nullptr;     // [E] or null
@@ -231,6 +283,16 @@ struct lx_layer {
 };
 
 namespace lx {
+
+// Raises a kernel's dynamic shared-memory cap once per device (the flag array
+// belongs to the calling launcher).
+inline cudaError_t smem_cap_once(const void* func, int bytes, int device, bool (&done)[64]) {
+  if (device >= 0 && device < 64 && done[device]) return cudaSuccess;
+  const cudaError_t e =
+      cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e == cudaSuccess && device >= 0 && device < 64) done[device] = true;
+  return e;
+}
 
 // Launch-time timing helper: records events around a launch when profiling.
 struct ProfScope {
@@ -247,7 +309,7 @@ lx_status launch_router_logits(lx_layer* L, const void* x, int T, float* logits,
 lx_status launch_bucket(lx_layer* L, const int* topk_id, int T, int k, cudaStream_t s);
 lx_status launch_generic_experts(lx_layer* L, const void* x, int T, int k, void* y,
                                  cudaStream_t s);
-lx_status launch_swiglu(lx_layer* L, int k, void* z, bool z_bf16, cudaStream_t s);
+lx_status launch_swiglu(lx_layer* L, int T, int k, void* z, bool z_bf16, cudaStream_t s);
 lx_status launch_combine(lx_layer* L, int T, int k, void* y, cudaStream_t s);
 lx_status launch_fast_experts(lx_layer* L, const void* x, int T, int k, void* y, cudaStream_t s);
 lx_status launch_stream(lx_layer* L, const StreamLaunch& P, cudaStream_t s, const char* name);

@@ -8,8 +8,8 @@
 // 16, 8, 4, 2, 1; the bias (if any) is added last.
 //
 // One CTA computes the logits of 8 tokens for a slice of the experts (all
-// experts when T is large, 16 per CTA when T is small, so that a decode batch
-// still spreads the 0.5 MB router matrix over many SMs).  Each warp owns one
+// experts when T is large, one per warp when T is small, so that a decode
+// batch still spreads the 0.5 MB router matrix over many SMs).  Each warp owns one
 // expert at a time and issues its weight loads in groups of 8 independent
 // 16-byte loads before using them.
 #include "lx_internal.cuh"
@@ -129,17 +129,18 @@ lx_status launch_router_logits(lx_layer* L, const void* x, int T, float* logits,
   if (smem > 200 * 1024) return fail(LX_ERR_SHAPE, "router token tile exceeds shared memory");
   const int tiles = (T + RT_TOK - 1) / RT_TOK;
   // few token tiles: slice the experts so the router matrix spreads over the SMs
-  const int per_cta = tiles >= L->num_sms ? L->E : 16;
+  const int per_cta = tiles >= L->num_sms ? L->E : RT_THREADS / 32;
   const dim3 grid(tiles, (L->E + per_cta - 1) / per_cta);
   ProfScope ps(L, s, "router");
+  static bool done_bf16[64] = {}, done_f32[64] = {};
   if (L->dtype == LX_BF16) {
     auto kern = k_router_logits<__nv_bfloat16>;
-    LX_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+    LX_CUDA(smem_cap_once((const void*)kern, 200 * 1024, L->device, done_bf16));
     kern<<<grid, RT_THREADS, smem, s>>>((const __nv_bfloat16*)x, (const __nv_bfloat16*)L->router_w,
                                         L->router_bias, T, L->E, L->H, per_cta, logits);
   } else {
     auto kern = k_router_logits<float>;
-    LX_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+    LX_CUDA(smem_cap_once((const void*)kern, 200 * 1024, L->device, done_f32));
     kern<<<grid, RT_THREADS, smem, s>>>((const float*)x, (const float*)L->router_w, L->router_bias,
                                         T, L->E, L->H, per_cta, logits);
   }
