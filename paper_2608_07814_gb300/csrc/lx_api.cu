@@ -95,29 +95,11 @@ static lx_status ensure_workspace(lx_layer* L, int T, int k, cudaStream_t s) {
   const long keys = (long)L->N + L->E;
   const long Rmax = std::max<long>(1, (long)cT * std::min<long>(L->N, (long)ck * D));
   const long rmax = std::max(1, L->max_rank);
-  // streaming tile descriptors: per launch group, at most ceil(T/64) token
-  // blocks of every node's column tiles
-  long scap = 0;
-  if (L->stream_ok) {
-    const long tb = (cT + stream_tile_tokens() - 1) / stream_tile_tokens();
-    for (int g = 0; g < N_STREAM_GROUPS; ++g) {
-      long tot = 0;
-      for (int j = 0; j < 2; ++j) {
-        const int op = stream_group_op(g, j);
-        if (op < 0) continue;
-        const OpShape sh = op_shape(L, op);
-        for (int n : (sh.on_anchors ? L->anchors : L->corrs)) {
-          const long Ng = sh.n_const + (long)sh.n_rank * L->rank[n];
-          tot += tb * sh.groups * ((Ng + stream_tile_rows() - 1) / stream_tile_rows());
-        }
-      }
-      scap = std::max(scap, tot);
-    }
-  }
   struct Item { void** p; size_t bytes; };
   std::vector<Item> items = {
       {(void**)&w.logits, sizeof(float) * cT * L->E},
       {(void**)&w.topk_id, sizeof(int) * cT * ck},
+      {(void**)&w.tile_cnt, sizeof(int) * ((cT + 7) / 8)},
       {(void**)&w.topk_w, sizeof(float) * cT * ck},
       {(void**)&w.marks, (size_t)keys * Tp},
       {(void**)&w.rank_in, sizeof(int) * keys * Tp},
@@ -136,8 +118,9 @@ static lx_status ensure_workspace(lx_layer* L, int T, int k, cudaStream_t s) {
       {(void**)&w.Pb, 2 * Rmax * 2 * rmax},
       {(void**)&w.zb, 2 * Rmax * L->I},
       {(void**)&w.Qb, 2 * Rmax * rmax},
-      {(void**)&w.stiles, sizeof(int4) * 2 * N_STREAM_GROUPS * std::max<long>(1, scap)},
-      {(void**)&w.stile_cnt, sizeof(int) * N_STREAM_GROUPS},
+      {(void**)&w.act, sizeof(int) * std::max(1, L->n_anchor + L->n_corr)},
+      {(void**)&w.act_n, sizeof(int) * 2},
+      {(void**)&w.sctr, sizeof(int) * N_STREAM_GROUPS},
       {(void**)&w.err, 256},
   };
   size_t total = 0;
@@ -161,11 +144,11 @@ static lx_status ensure_workspace(lx_layer* L, int T, int k, cudaStream_t s) {
   w.base = base;
   w.bytes = total;
   e = cudaMemsetAsync(w.err, 0, sizeof(int), s);
+  if (e == cudaSuccess) e = cudaMemsetAsync(w.tile_cnt, 0, sizeof(int) * ((cT + 7) / 8), s);
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
   if (e != cudaSuccess) return cuda_fail(e, "clear workspace error word");
   w.cap_T = cT;
   w.cap_k = ck;
-  w.stile_cap = (int)scap;
   L->last_T = L->last_k = 0;
   return LX_OK;
 }
@@ -179,24 +162,19 @@ static lx_status check_call(lx_layer* L, int T, int k) {
   return LX_OK;
 }
 
-// Logits, top-k and bucketing of T tokens (single-CTA bucketing for small T).
-static lx_status route_and_bucket(lx_layer* L, const void* x, int T, int k, int* ids, float* w,
-                                  float* logits_user, cudaStream_t s) {
-  float* logits = logits_user ? logits_user : L->ws.logits;
-  LX_TRY(launch_router_logits(L, x, T, logits, s));
-  if (bucket_small_fits(L, T, k)) {
-    LX_TRY(launch_bucket_small(L, logits, nullptr, T, k, ids, w, s));
-  } else {
-    LX_TRY(launch_topk(L, logits, T, k, ids, w, s));
-    LX_TRY(launch_bucket(L, ids, T, k, s));
-  }
-  return LX_OK;
-}
-
 static lx_status bucket_ids(lx_layer* L, const int* ids, int T, int k, cudaStream_t s) {
   if (bucket_small_fits(L, T, k)) return launch_bucket_small(L, nullptr, ids, T, k, nullptr, nullptr, s);
   return launch_bucket(L, ids, T, k, s);
 }
+
+// Logits, top-k and bucketing of T tokens (single-CTA bucketing for small T).
+static lx_status route_and_bucket(lx_layer* L, const void* x, int T, int k, int* ids, float* w,
+                                  float* logits_user, cudaStream_t s) {
+  float* logits = logits_user ? logits_user : L->ws.logits;
+  LX_TRY(launch_router(L, x, T, k, logits, ids, w, s));
+  return bucket_ids(L, ids, T, k, s);
+}
+
 
 // Largest batch the weight-streaming (decode) kernels take; beyond it every
 // weight would be re-streamed per 64-token block.

@@ -107,58 +107,39 @@ __device__ __forceinline__ int plan_tiles(const PlanArgs& pa, int p, int r, int 
 }
 
 
-// Expands the streaming plans (plans PLAN_STREAM + op) into one flat list of
-// tile descriptors per launch group (see StreamLaunch).  Called by one CTA
-// after the plans are written; node_off and rank may live in shared memory.
-__device__ void expand_stream_tiles(const PlanArgs& pa, const int* tile_off, int toff_stride,
-                                    const int* const* items, const int* node_off, const int* rank,
-                                    int4* tiles, int* cnt, int cap) {
-  for (int g = 0; g < N_STREAM_GROUPS; ++g) {
-    int tot[2] = {0, 0};
-    for (int j = 0; j < 2; ++j) {
-      const int op = stream_group_op(g, j);
-      if (op >= 0) tot[j] = tile_off[op * toff_stride + pa.n_items[PLAN_STREAM + op]];
+
+// Compact lists of the active anchors and corrections (bucket size > 0), in
+// node-table order, and zeroed tile counters for the streaming launches.  One
+// CTA; warps 0 and 1 each compact one list.
+__device__ void publish_active(const int* cnt, const int* anchors, int n_anchor,
+                               const int* corrs, int n_corr, int* act, int* act_n, int* sctr) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (warp < 2) {
+    const int* list = warp == 0 ? anchors : corrs;
+    const int n = warp == 0 ? n_anchor : n_corr;
+    int* out = act + (warp == 0 ? 0 : n_anchor);
+    int base = 0;
+    for (int i0 = 0; i0 < n; i0 += 32) {
+      const int i = i0 + lane;
+      const int node = i < n ? list[i] : -1;
+      const bool a = node >= 0 && cnt[node] > 0;
+      const uint32_t b = __ballot_sync(0xffffffffu, a);
+      if (a) out[base + __popc(b & ((1u << lane) - 1u))] = node;
+      base += __popc(b);
     }
-    const int total = min(tot[0] + tot[1], cap);
-    if (threadIdx.x == 0) cnt[g] = total;
-    int4* out = tiles + (size_t)g * cap * 2;
-    for (int idx = threadIdx.x; idx < total; idx += blockDim.x) {
-      const int j = idx < tot[0] ? 0 : 1;
-      const int op = stream_group_op(g, j);
-      const int p = PLAN_STREAM + op;
-      const int local0 = idx - (j ? tot[0] : 0);
-      const int* to = tile_off + op * toff_stride;
-      int lo = 0, hi = pa.n_items[p];
-      while (hi - lo > 1) {
-        const int mid = (lo + hi) >> 1;
-        if (to[mid] <= local0) lo = mid; else hi = mid;
-      }
-      const int n = items[op][lo];
-      const int local = local0 - to[lo];
-      const OpShape sh = pa.shape[p];
-      const int r = rank[n];
-      const int Ng = sh.n_const + sh.n_rank * r, K = sh.k_const + sh.k_rank * r;
-      const int ncol = (Ng + pa.bn[p] - 1) / pa.bn[p];
-      const int ncb = stream_col_blocks(K, ncol);
-      const int nct = (ncol + ncb - 1) / ncb;
-      const int per_tb = nct * sh.groups;
-      const int tb = local / per_tb, rem = local % per_tb;
-      const int ct = rem % nct;
-      const int tok0 = node_off[n] + tb * pa.bm[p];
-      const int M = min(pa.bm[p], node_off[n + 1] - tok0);
-      const int cbs = min(ncb, ncol - ct * ncb);
-      out[2 * idx] = make_int4(op, n, ct * ncb * pa.bn[p], tok0);
-      out[2 * idx + 1] = make_int4(M, K, Ng, (rem / nct) | (cbs << 4));
-    }
+    if (lane == 0) act_n[warp] = base;
   }
+  if (threadIdx.x < N_STREAM_GROUPS) sctr[threadIdx.x] = 0;
 }
 
 // one CTA: node/expert offsets and the tile prefix of every plan
 __global__ void k_offsets_plan(const int* __restrict__ key_cnt, int N, int E,
                                int* __restrict__ key_off, const int* __restrict__ rank,
                                int* __restrict__ tile_off, int max_items, PlanArgs pa,
-                               int4* __restrict__ stiles, int* __restrict__ stile_cnt,
-                               int stile_cap) {
+                               const int* __restrict__ anchors, int n_anchor,
+                               const int* __restrict__ corrs, int n_corr, int* __restrict__ act,
+                               int* __restrict__ act_n, int* __restrict__ sctr) {
+  if (act) publish_active(key_cnt, anchors, n_anchor, corrs, n_corr, act, act_n, sctr);
   // node offsets then expert offsets
   for (int part = 0; part < 2; ++part) {
     const int n0 = part == 0 ? 0 : N, cnt = part == 0 ? N : E;
@@ -192,12 +173,6 @@ __global__ void k_offsets_plan(const int* __restrict__ key_cnt, int N, int E,
     }
     if (threadIdx.x == 0) to[pa.n_items[p]] = carry;
     __syncthreads();
-  }
-  if (stiles) {
-    const int* its[N_OPS];
-    for (int op = 0; op < N_OPS; ++op) its[op] = pa.items[PLAN_STREAM + op];
-    expand_stream_tiles(pa, tile_off + PLAN_STREAM * (max_items + 1), max_items + 1, its, key_off,
-                        rank, stiles, stile_cnt, stile_cap);
   }
 }
 
@@ -258,8 +233,7 @@ constexpr size_t SB_SMEM_LIMIT = 160 * 1024;
 __host__ __device__ inline size_t sb_smem(int T, int k, int keys, int E, int N, int max_items) {
   const size_t Tp = ((size_t)T + 15) / 16 * 16;
   return (size_t)T * k * 4 + 2 * (size_t)keys * Tp + (size_t)keys * 4 + ((size_t)keys + 2) * 4 +
-         (size_t)E * (LX_MAX_DEPTH + 1) * 4 + (size_t)N * 4 +
-         (size_t)N_OPS * (max_items + 1) * 4 + (size_t)N * 4 + 64;
+         (size_t)E * (LX_MAX_DEPTH + 1) * 4 + (size_t)N * 4 + 64;
 }
 
 __global__ void __launch_bounds__(SB_THREADS)
@@ -269,7 +243,9 @@ k_bucket_small(const float* __restrict__ logits, const int* __restrict__ ids_in,
                int* __restrict__ topk_id, float* __restrict__ topk_w, int* __restrict__ key_off_g,
                int* __restrict__ node_tok, int* __restrict__ row_node, int* __restrict__ node_row,
                int* __restrict__ perm, int* __restrict__ tile_off, int max_items, PlanArgs pa,
-               int4* __restrict__ stiles, int* __restrict__ stile_cnt, int stile_cap) {
+               const int* __restrict__ anchors, int n_anchor, const int* __restrict__ corrs,
+               int n_corr, int* __restrict__ act, int* __restrict__ act_n,
+               int* __restrict__ sctr) {
   extern __shared__ __align__(16) unsigned char sm[];
   const int keys = N + E;
   const int Tp = (T + 15) & ~15;
@@ -281,16 +257,11 @@ k_bucket_small(const float* __restrict__ logits, const int* __restrict__ ids_in,
   int* spaths = off + keys + 2;                 // [E][LX_MAX_DEPTH]
   int* splen = spaths + E * LX_MAX_DEPTH;       // [E]
   int* srank = splen + E;                       // [N]
-  int* stoff = srank + N;                       // [N_OPS][max_items+1] streaming plans
-  int* sitems = stoff + N_OPS * (max_items + 1); // anchors then corrections
   const int tid = threadIdx.x, nth = blockDim.x;
   const int warp = tid >> 5, lane = tid & 31, nw = nth >> 5;
   for (int i = tid; i < E * LX_MAX_DEPTH; i += nth) spaths[i] = paths[i];
   for (int i = tid; i < E; i += nth) splen[i] = path_len[i];
   for (int i = tid; i < N; i += nth) srank[i] = rank[i];
-  const int n_anc = pa.n_items[PLAN_STREAM + OP_UP_ANCHOR], n_cor = pa.n_items[PLAN_STREAM + OP_UP_V];
-  for (int i = tid; i < n_anc; i += nth) sitems[i] = pa.items[PLAN_STREAM + OP_UP_ANCHOR][i];
-  for (int i = tid; i < n_cor; i += nth) sitems[n_anc + i] = pa.items[PLAN_STREAM + OP_UP_V][i];
   {
     uint32_t* m32 = reinterpret_cast<uint32_t*>(marks);  // keys*Tp is a multiple of 16
     for (int i = tid; i < keys * Tp / 4; i += nth) m32[i] = 0;
@@ -350,6 +321,7 @@ k_bucket_small(const float* __restrict__ logits, const int* __restrict__ ids_in,
     __syncthreads();
   }
   for (int i = tid; i < keys + 2; i += nth) key_off_g[i] = off[i];
+  publish_active(cnt, anchors, n_anchor, corrs, n_corr, act, act_n, sctr);
   // 5. tile plans: one warp per plan
   for (int p = warp; p < pa.n_plans; p += nw) {
     int* to = tile_off + p * (max_items + 1);
@@ -367,16 +339,10 @@ k_bucket_small(const float* __restrict__ logits, const int* __restrict__ ids_in,
         const int x = __shfl_up_sync(0xffffffffu, incl, o);
         if (lane >= o) incl += x;
       }
-      if (i < pa.n_items[p]) {
-        to[i] = carry + incl - v;
-        if (p >= PLAN_STREAM) stoff[(p - PLAN_STREAM) * (max_items + 1) + i] = carry + incl - v;
-      }
+      if (i < pa.n_items[p]) to[i] = carry + incl - v;
       carry += __shfl_sync(0xffffffffu, incl, 31);
     }
-    if (lane == 0) {
-      to[pa.n_items[p]] = carry;
-      if (p >= PLAN_STREAM) stoff[(p - PLAN_STREAM) * (max_items + 1) + pa.n_items[p]] = carry;
-    }
+    if (lane == 0) to[pa.n_items[p]] = carry;
   }
   // 6. scatter from the assignments: bucket rows, node rows, permutation
   for (int a = tid; a < T * k; a += nth) {
@@ -394,14 +360,6 @@ k_bucket_small(const float* __restrict__ logits, const int* __restrict__ ids_in,
       }
       node_row[(size_t)a * D + l] = row;
     }
-  }
-  __syncthreads();
-  // 7. streaming tile descriptors (plans and item lists from shared memory)
-  if (stiles) {
-    const int* its[N_OPS];
-    for (int op = 0; op < N_OPS; ++op)
-      its[op] = pa.shape[PLAN_STREAM + op].on_anchors ? sitems : sitems + n_anc;
-    expand_stream_tiles(pa, stoff, max_items + 1, its, off, srank, stiles, stile_cnt, stile_cap);
   }
 }
 
@@ -431,16 +389,16 @@ lx_status launch_bucket_small(lx_layer* L, const float* logits, const int* ids_i
                               int* topk_id, float* topk_w, cudaStream_t s) {
   Workspace& w = L->ws;
   const size_t smem = sb_smem(T, k, L->N + L->E, L->E, L->N, op_max_items(L));
-  const PlanArgs pa = make_plans(L, N_PLANS);
+  const PlanArgs pa = make_plans(L, N_OPS);
   static bool done[64] = {};
   LX_CUDA(smem_cap_once((const void*)k_bucket_small, (int)SB_SMEM_LIMIT, L->device, done));
   ProfScope ps(L, s, logits ? "topk_bucket_small" : "bucket_small");
   k_bucket_small<<<1, SB_THREADS, smem, s>>>(logits, ids_in, T, k, L->E, L->N, L->max_depth,
                                              L->d_paths, L->d_path_len, L->d_rank, topk_id, topk_w,
                                              w.key_off, w.node_tok, w.row_node, w.node_row, w.perm,
-                                             w.tile_off, op_max_items(L), pa,
-                                             L->stream_ok ? w.stiles : nullptr, w.stile_cnt,
-                                             w.stile_cap);
+                                             w.tile_off, op_max_items(L), pa, L->d_anchors,
+                                             L->n_anchor, L->d_corrs, L->n_corr, w.act, w.act_n,
+                                             w.sctr);
   LX_CUDA(cudaGetLastError());
   return LX_OK;
 }
@@ -465,11 +423,11 @@ lx_status launch_bucket(lx_layer* L, const int* topk_id, int T, int k, cudaStrea
     LX_CUDA(cudaGetLastError());
   }
   {
-    const PlanArgs pa = make_plans(L, N_PLANS);
+    const PlanArgs pa = make_plans(L, N_OPS);
     ProfScope ps(L, s, "bucket_offsets");
     k_offsets_plan<<<1, 1024, 0, s>>>(w.key_cnt, L->N, L->E, w.key_off, L->d_rank, w.tile_off,
-                                      op_max_items(L), pa, L->stream_ok ? w.stiles : nullptr,
-                                      w.stile_cnt, w.stile_cap);
+                                      op_max_items(L), pa, L->d_anchors, L->n_anchor, L->d_corrs,
+                                      L->n_corr, w.act, w.act_n, w.sctr);
     LX_CUDA(cudaGetLastError());
   }
   {
@@ -575,7 +533,8 @@ extern "C" lx_status lx_bucket_noalloc(lx_layer* L, const int32_t* topk_id, int3
   LX_CUDA(cudaGetLastError());
   const PlanArgs pa = make_plans(L, N_OPS);
   k_offsets_plan<<<1, 1024, 0, s>>>(key_cnt, L->N, L->E, key_off, L->d_rank, tile_off,
-                                    op_max_items(L), pa, nullptr, nullptr, 0);
+                                    op_max_items(L), pa, nullptr, 0, nullptr, 0, nullptr, nullptr,
+                                    nullptr);
   LX_CUDA(cudaGetLastError());
   k_scatter<<<dim3((T + 255) / 256, (unsigned)keys), 256, 0, s>>>(
       marks, rank_in, key_off, topk_id, T, k, L->N, Tp, node_tok, row_node, perm);

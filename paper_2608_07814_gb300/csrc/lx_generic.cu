@@ -144,19 +144,33 @@ k_swiglu_aggregate(const int* __restrict__ topk_id, const float* __restrict__ to
     for (int j = threadIdx.x; j < kD; j += blockDim.x) rows[j] = node_row[(size_t)t * kD + j];
     for (int j = threadIdx.x; j < k; j += blockDim.x) gw[j] = topk_w[(size_t)t * k + j];
     __syncthreads();
-    if (threadIdx.x == 0) {
-      int nd = 0;
-      for (int j = 0; j < kD; ++j) {
-        const int r = rows[j];
-        int d = -1;
-        if (r >= 0) {
-          for (int q = 0; q < nd; ++q)
-            if (drow[q] == r) d = q;
-          if (d < 0) { d = nd; drow[nd++] = r; }
+    // distinct rows, numbered in order of first appearance (entry j owns the
+    // number of first appearances before it)
+    if (threadIdx.x < 32) {
+      const int lane = threadIdx.x;
+      int base = 0;
+      for (int j0 = 0; j0 < kD; j0 += 32) {
+        const int j = j0 + lane;
+        const int r = j < kD ? rows[j] : -1;
+        bool first = r >= 0;
+        for (int q = 0; q < j && first; ++q) first = rows[q] != r;
+        const uint32_t fm = __ballot_sync(0xffffffffu, first);
+        if (first) {
+          const int d = base + __popc(fm & ((1u << lane) - 1u));
+          drow[d] = r;
         }
-        lrow[j] = d;
+        base += __popc(fm);
       }
-      nd_s = nd;
+      if (lane == 0) nd_s = base;
+    }
+    __syncthreads();
+    for (int j = threadIdx.x; j < kD; j += blockDim.x) {
+      const int r = rows[j];
+      int d = -1;
+      if (r >= 0)
+        for (int q = 0; q < nd_s; ++q)
+          if (drow[q] == r) d = q;
+      lrow[j] = d;
     }
     __syncthreads();
     const int nd = nd_s;
@@ -204,19 +218,33 @@ k_combine(const int* __restrict__ node_row, int k, int D, const float* __restric
   for (int t = blockIdx.x; t < T; t += gridDim.x) {
     for (int j = threadIdx.x; j < k * D; j += blockDim.x) raw_s[j] = node_row[(long)t * k * D + j];
     __syncthreads();
-    if (threadIdx.x == 0) {
-      int m = 0;
-      for (int j = 0; j < k * D; ++j) {
-        const int r = raw_s[j];
-        if (r < 0) continue;
-        bool dup = false;
-        for (int q = 0; q < m; ++q) dup |= rows_s[q] == r;
-        if (dup) continue;
-        int p = m++;  // insertion sort, ascending
-        while (p > 0 && rows_s[p - 1] > r) { rows_s[p] = rows_s[p - 1]; --p; }
-        rows_s[p] = r;
+    // distinct rows in ascending order: each first occurrence takes the rank
+    // of its value among the distinct values
+    for (int j = threadIdx.x; j < k * D; j += blockDim.x) {
+      const int r = raw_s[j];
+      bool first = r >= 0;
+      for (int q = 0; q < j && first; ++q) first = raw_s[q] != r;
+      if (first) {
+        int rank = 0;
+        for (int q = 0; q < k * D; ++q) {
+          const int v = raw_s[q];
+          bool fq = v >= 0 && v < r;
+          for (int u = 0; u < q && fq; ++u) fq = raw_s[u] != v;
+          rank += fq;
+        }
+        rows_s[rank] = r;
       }
-      nrows_s = m;
+    }
+    if (threadIdx.x < 32) {
+      int cntd = 0;
+      for (int j0 = 0; j0 < k * D; j0 += 32) {
+        const int j = j0 + threadIdx.x;
+        const int r = j < k * D ? raw_s[j] : -1;
+        bool first = r >= 0;
+        for (int q = 0; q < j && first; ++q) first = raw_s[q] != r;
+        cntd += __popc(__ballot_sync(0xffffffffu, first));
+      }
+      if (threadIdx.x == 0) nrows_s = cntd;
     }
     __syncthreads();
     const int m = nrows_s;

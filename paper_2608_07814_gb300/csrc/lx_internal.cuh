@@ -161,8 +161,9 @@ struct GemmArgs {
 // Streaming (decode) grouped GEMM: one op of a launch
 struct StreamOp {
   const CUtensorMap* tmaps;  // [n_nodes] weight tensor maps of this op
-  const int* items;          // node ids
-  int n_items;
+  const int* items;          // active node ids (compact list written by the bucketing)
+  const int* n_active;       // device count of items
+  int n_items;               // upper bound of the count (host)
   const int* tile_off;       // [n_items+1] stream plan
   const int* node_off;
   const int* gather;         // row -> X row (token ids), or null = identity
@@ -173,13 +174,14 @@ struct StreamOp {
   int out_f32;
   OpShape shape;
   const int* rank;
+  int ncol_max;              // column tiles of the widest node of this op
+  int ntb;                   // token blocks (64 tokens) of the largest possible bucket
 };
 
 // The streaming launches: group 0 = {UP_ANCHOR, UP_V}, 1 = {UP_U},
-// 2 = {DN_ANCHOR, DN_V}, 3 = {DN_U}.  Each group's tiles are expanded on the
-// device into a flat list of descriptors
-//   a = {op, node, row0 (first weight row in the group), tok0 (first node row)}
-//   b = {M (tokens), K, Ng (rows per group), grp | column blocks << 4}
+// 2 = {DN_ANCHOR, DN_V}, 3 = {DN_U}.  A launch's tile index runs over
+// op 0's (item, token block, group, column tile) grid, then op 1's; tiles of
+// inactive nodes or beyond a node's columns are skipped.
 constexpr int N_STREAM_GROUPS = 4;
 __host__ __device__ inline int stream_group_op(int g, int j) {
   const int ops[N_STREAM_GROUPS][2] = {{OP_UP_ANCHOR, OP_UP_V}, {OP_UP_U, -1},
@@ -197,11 +199,9 @@ __host__ __device__ inline int stream_col_blocks(int K, int ncol) {
 }
 
 struct StreamLaunch {
-  StreamOp op[2];            // op[j] serves descriptors whose op id is op_id[j]
-  int op_id[2];
+  StreamOp op[2];
   int n_ops;
-  const int4* tiles;         // [n_tiles][2] descriptors of this launch's group
-  const int* n_tiles;        // device count
+  int* ctr;                  // tile counter of this launch (zeroed by the bucketing)
   int* err;                  // device error word (LX_ERR_TIMEOUT on a bounded wait)
 };
 
@@ -215,6 +215,7 @@ struct Workspace {
   // routing
   float* logits = nullptr;   // [T][E]
   int* topk_id = nullptr;    // [T][k]
+  int* tile_cnt = nullptr;   // [T/8] router slices done per token tile (self-resetting)
   float* topk_w = nullptr;   // [T][k]
   // bucketing
   uint8_t* marks = nullptr;  // [(N+E)][Tp]
@@ -236,9 +237,9 @@ struct Workspace {
   __nv_bfloat16* Pb = nullptr;  // [Rmax][2 rmax]
   __nv_bfloat16* zb = nullptr;  // [Rmax][I]
   __nv_bfloat16* Qb = nullptr;  // [Rmax][rmax]
-  int4* stiles = nullptr;       // [N_STREAM_GROUPS][stile_cap][2] tile descriptors
-  int* stile_cnt = nullptr;     // [N_STREAM_GROUPS]
-  int stile_cap = 0;
+  int* act = nullptr;           // [n_anchor + n_corr] active anchors, then active corrections
+  int* act_n = nullptr;         // [2] their counts
+  int* sctr = nullptr;          // [N_STREAM_GROUPS] streaming tile counters
   int* err = nullptr;           // device error word
 };
 
@@ -305,7 +306,8 @@ struct ProfScope {
 };
 
 // kernels / launchers (defined in the .cu files)
-lx_status launch_router_logits(lx_layer* L, const void* x, int T, float* logits, cudaStream_t s);
+lx_status launch_router(lx_layer* L, const void* x, int T, int k, float* logits, int* topk_id,
+                        float* topk_w, cudaStream_t s);
 lx_status launch_bucket(lx_layer* L, const int* topk_id, int T, int k, cudaStream_t s);
 lx_status launch_generic_experts(lx_layer* L, const void* x, int T, int k, void* y,
                                  cudaStream_t s);
@@ -313,8 +315,6 @@ lx_status launch_swiglu(lx_layer* L, int T, int k, void* z, bool z_bf16, cudaStr
 lx_status launch_combine(lx_layer* L, int T, int k, void* y, cudaStream_t s);
 lx_status launch_fast_experts(lx_layer* L, const void* x, int T, int k, void* y, cudaStream_t s);
 lx_status launch_stream(lx_layer* L, const StreamLaunch& P, cudaStream_t s, const char* name);
-lx_status launch_topk(lx_layer* L, const float* logits, int T, int k, int* topk_id,
-                      float* topk_w, cudaStream_t s);
 lx_status launch_bucket_small(lx_layer* L, const float* logits, const int* ids_in, int T, int k,
                               int* topk_id, float* topk_w, cudaStream_t s);
 bool bucket_small_fits(const lx_layer* L, int T, int k);

@@ -1,4 +1,5 @@
-// Router: logits in the canonical fp32 order, then top-k and softmax gates.
+// Router: logits in the canonical fp32 order, then top-k and softmax gates,
+// in one launch.
 //
 // The router is the MoE layer's own, unchanged by compression (Sec. 1, Fig. 1;
 // Sec. 3.2 Stage 1).  Logit order (fixed so that the top-k decision is
@@ -12,6 +13,8 @@
 // batch still spreads the 0.5 MB router matrix over many SMs).  Each warp owns one
 // expert at a time and issues its weight loads in groups of 8 independent
 // 16-byte loads before using them.
+#include <algorithm>
+
 #include "lx_internal.cuh"
 
 namespace lx {
@@ -49,7 +52,9 @@ __device__ __forceinline__ void load8<__nv_bfloat16>(const __nv_bfloat16* p, flo
 template <typename T>
 __global__ void __launch_bounds__(RT_THREADS)
 k_router_logits(const T* __restrict__ x, const T* __restrict__ W, const float* __restrict__ bias,
-                int Ttok, int E, int H, int experts_per_cta, float* __restrict__ logits) {
+                int Ttok, int E, int H, int experts_per_cta, float* __restrict__ logits,
+                int* __restrict__ tile_cnt, int k, int* __restrict__ topk_id,
+                float* __restrict__ topk_w) {
   extern __shared__ __align__(16) unsigned char smem[];
   T* xs = reinterpret_cast<T*>(smem);
   const int t0 = blockIdx.x * RT_TOK;
@@ -104,28 +109,41 @@ k_router_logits(const T* __restrict__ x, const T* __restrict__ W, const float* _
         logits[(size_t)(t0 + tt) * E + e] = bias ? __fadd_rn(acc[tt], b) : acc[tt];
     }
   }
-}
-
-__global__ void k_topk(const float* __restrict__ logits, int T, int E, int k,
-                       int* __restrict__ topk_id, float* __restrict__ topk_w) {
-  const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  const int lane = threadIdx.x & 31;
-  if (warp >= T) return;
-  int id;
-  float w;
-  warp_topk(logits + (size_t)warp * E, E, k, id, w);
-  if (lane < k) {
-    topk_id[(size_t)warp * k + lane] = id;
-    topk_w[(size_t)warp * k + lane] = w;
+  // The last CTA to finish this token tile's expert slices takes its top-k
+  // (no CTA waits for another; the counter is reset for the next call).
+  __shared__ int s_last;
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    const int old = atomicAdd(&tile_cnt[blockIdx.x], 1);
+    s_last = old == (int)gridDim.y - 1;
   }
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  float* ls = reinterpret_cast<float*>(smem);  // reuse the token tile's space
+  for (int i = threadIdx.x; i < nt * E; i += blockDim.x)
+    ls[i] = __ldcg(logits + (size_t)t0 * E + i);
+  __syncthreads();
+  for (int tt = warp; tt < nt; tt += nw) {
+    int id;
+    float w;
+    warp_topk(ls + tt * E, E, k, id, w);
+    if (lane < k) {
+      topk_id[(size_t)(t0 + tt) * k + lane] = id;
+      topk_w[(size_t)(t0 + tt) * k + lane] = w;
+    }
+  }
+  if (threadIdx.x == 0) tile_cnt[blockIdx.x] = 0;
 }
 
 }  // namespace
 
-lx_status launch_router_logits(lx_layer* L, const void* x, int T, float* logits, cudaStream_t s) {
+lx_status launch_router(lx_layer* L, const void* x, int T, int k, float* logits, int* topk_id,
+                        float* topk_w, cudaStream_t s) {
   if (reinterpret_cast<uintptr_t>(x) % 16)
     return fail(LX_ERR_ARG, "x must be 16-byte aligned");
-  const size_t smem = (size_t)RT_TOK * L->H * L->esz;
+  const size_t smem = std::max((size_t)RT_TOK * L->H * L->esz, (size_t)RT_TOK * L->E * 4);
   if (smem > 200 * 1024) return fail(LX_ERR_SHAPE, "router token tile exceeds shared memory");
   const int tiles = (T + RT_TOK - 1) / RT_TOK;
   // few token tiles: slice the experts so the router matrix spreads over the SMs
@@ -137,21 +155,15 @@ lx_status launch_router_logits(lx_layer* L, const void* x, int T, float* logits,
     auto kern = k_router_logits<__nv_bfloat16>;
     LX_CUDA(smem_cap_once((const void*)kern, 200 * 1024, L->device, done_bf16));
     kern<<<grid, RT_THREADS, smem, s>>>((const __nv_bfloat16*)x, (const __nv_bfloat16*)L->router_w,
-                                        L->router_bias, T, L->E, L->H, per_cta, logits);
+                                        L->router_bias, T, L->E, L->H, per_cta, logits,
+                                        L->ws.tile_cnt, k, topk_id, topk_w);
   } else {
     auto kern = k_router_logits<float>;
     LX_CUDA(smem_cap_once((const void*)kern, 200 * 1024, L->device, done_f32));
     kern<<<grid, RT_THREADS, smem, s>>>((const float*)x, (const float*)L->router_w, L->router_bias,
-                                        T, L->E, L->H, per_cta, logits);
+                                        T, L->E, L->H, per_cta, logits, L->ws.tile_cnt, k,
+                                        topk_id, topk_w);
   }
-  LX_CUDA(cudaGetLastError());
-  return LX_OK;
-}
-
-lx_status launch_topk(lx_layer* L, const float* logits, int T, int k, int* topk_id, float* topk_w,
-                      cudaStream_t s) {
-  ProfScope ps(L, s, "topk");
-  k_topk<<<(T + 7) / 8, 256, 0, s>>>(logits, T, L->E, k, topk_id, topk_w);
   LX_CUDA(cudaGetLastError());
   return LX_OK;
 }

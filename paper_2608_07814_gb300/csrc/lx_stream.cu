@@ -21,6 +21,8 @@
 //     word and drains the CTA's copies in flight before returning.
 #include <cuda.h>
 
+#include <algorithm>
+
 
 #include "lx_internal.cuh"
 
@@ -34,8 +36,9 @@ constexpr int SW_BOX = 64;          // K per stage = one TMA box of 64 K x 64 ro
 constexpr int SW_BOX_BYTES = SW_BOX * SW_ROWS * 2;
 constexpr int SW_XROW = SW_BOX * 2 + 16;           // padded token row in shared memory
 constexpr int SW_STAGE_BYTES = SW_BOX_BYTES + SW_TOK * SW_XROW;  // 17 KiB, 1024-aligned
-constexpr int SW_STAGES = 6;
+constexpr int SW_STAGES = 4;
 constexpr int SW_CONSUMERS = 2;
+constexpr int SW_MT = SW_ROWS / (16 * SW_CONSUMERS);  // 16-row MMA tiles per consumer warp
 constexpr int SW_THREADS = 32 * (1 + SW_CONSUMERS);
 constexpr unsigned long long SW_TIMEOUT_CYCLES = 4000000000ull;  // ~2 s
 static_assert(SW_STAGE_BYTES % 1024 == 0, "stages must keep the 128B-swizzle alignment");
@@ -52,19 +55,30 @@ __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
 }
 
+// Consumer release of a stage.  The stage's shared-memory reads are complete
+// (their values fed the MMAs before this point in program order), so no
+// release ordering is needed -- which keeps the arrive from waiting on the
+// consumer's earlier global stores.
+__device__ __forceinline__ void mbar_arrive_relaxed(uint32_t bar) {
+  asm volatile("mbarrier.arrive.relaxed.cta.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
 __device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
   asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
                : "memory");
 }
 
+// try_wait with a suspend-time hint: a waiting thread is parked by the
+// hardware (up to ~0.5 us per call) instead of spinning on issue slots that
+// the working warps of the SM need.
 __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
       "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
       "selp.u32 %0, 1, 0, p;\n\t}"
       : "=r"(ok)
-      : "r"(bar), "r"(parity)
+      : "r"(bar), "r"(parity), "r"(500)
       : "memory");
   return ok != 0;
 }
@@ -122,27 +136,42 @@ __device__ __forceinline__ uint4 lds_v4(uint32_t addr) {
 
 struct TileInfo {
   int op, node, grp, row0, tok0, M, Ng, K, ncb;
+  bool active;
 };
 
-__device__ __forceinline__ void fetch_tile(const StreamLaunch& P, int tile, int total, int4& a,
-                                           int4& b) {
-  if (tile < total) {
-    a = P.tiles[2 * tile];
-    b = P.tiles[2 * tile + 1];
-  }
+__device__ __forceinline__ int op_tiles(const StreamOp& op) {
+  return *op.n_active * op.ntb * op.shape.groups * op.ncol_max;
 }
 
-__device__ __forceinline__ void unpack_tile(const StreamLaunch& P, const int4& a, const int4& b,
+// Tile index -> (op, node, token block, group, column tile).
+__device__ __forceinline__ void decode_tile(const StreamLaunch& P, int tile, int tiles0,
                                             TileInfo& ti) {
-  ti.op = (P.n_ops > 1 && a.x == P.op_id[1]) ? 1 : 0;
-  ti.node = a.y;
-  ti.row0 = a.z;
-  ti.tok0 = a.w;
-  ti.M = b.x;
-  ti.K = b.y;
-  ti.Ng = b.z;
-  ti.grp = b.w & 15;
-  ti.ncb = b.w >> 4;
+  int o = 0, local = tile;
+  if (P.n_ops > 1 && tile >= tiles0) {
+    o = 1;
+    local = tile - tiles0;
+  }
+  const StreamOp& op = P.op[o];
+  const int per_tb = op.shape.groups * op.ncol_max;
+  const int per_item = op.ntb * per_tb;
+  const int item = local / per_item;
+  int rem = local - item * per_item;
+  const int tb = rem / per_tb;
+  rem -= tb * per_tb;
+  const int grp = rem / op.ncol_max, ct = rem - grp * op.ncol_max;
+  const int n = op.items[item];
+  const int r = op.rank[n];
+  const int b0 = op.node_off[n], b1 = op.node_off[n + 1];
+  ti.op = o;
+  ti.node = n;
+  ti.grp = grp;
+  ti.row0 = ct * SW_ROWS;
+  ti.Ng = op.shape.n_const + op.shape.n_rank * r;
+  ti.K = op.shape.k_const + op.shape.k_rank * r;
+  ti.tok0 = b0 + tb * SW_TOK;
+  ti.M = min(SW_TOK, b1 - ti.tok0);
+  ti.ncb = 1;
+  ti.active = ti.M > 0 && ti.row0 < ti.Ng;
 }
 
 template <int NT>
@@ -153,11 +182,11 @@ __device__ __forceinline__ bool consume_tile(const StreamLaunch& P, const TileIn
   const int lane = threadIdx.x & 31, cw = (threadIdx.x >> 5) - 1;
   const int g = lane >> 2, q = lane & 3;
   const int nkb = (ti.K + SW_BOX - 1) / SW_BOX;
-  const int wrow = cw * 32 + g;  // first of this lane's weight rows inside a 64-row block
+  const int wrow = cw * 16 * SW_MT + g;  // first of this lane's weight rows in a 64-row block
   for (int cb = 0; cb < ti.ncb; ++cb) {
-    float acc[2][NT][4];
+    float acc[SW_MT][NT][4];
 #pragma unroll
-    for (int i = 0; i < 2; ++i)
+    for (int i = 0; i < SW_MT; ++i)
 #pragma unroll
       for (int j = 0; j < NT; ++j)
 #pragma unroll
@@ -176,7 +205,7 @@ __device__ __forceinline__ bool consume_tile(const StreamLaunch& P, const TileIn
           xv[j] = lds_v4(xbox + (8 * j + g) * SW_XROW + c * 64 + 16 * q);
         const uint32_t unit = ((c * 4 + q) ^ g) * 16;  // 128-byte swizzle (row & 7 == g)
 #pragma unroll
-        for (int i = 0; i < 2; ++i) {
+        for (int i = 0; i < SW_MT; ++i) {
           const uint4 w0 = lds_v4(wbox + (wrow + 16 * i) * 128 + unit);
           const uint4 w1 = lds_v4(wbox + (wrow + 16 * i + 8) * 128 + unit);
 #pragma unroll
@@ -187,11 +216,11 @@ __device__ __forceinline__ bool consume_tile(const StreamLaunch& P, const TileIn
         }
       }
       __syncwarp();
-      if (lane == 0) mbar_arrive(empty0 + 8 * s);
+      if (lane == 0) mbar_arrive_relaxed(empty0 + 8 * s);
     }
     // epilogue: D[weight row][token] -> out[token row][grp*Ng + weight row]
 #pragma unroll
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < SW_MT; ++i) {
 #pragma unroll
       for (int j = 0; j < NT; ++j) {
 #pragma unroll
@@ -218,12 +247,13 @@ k_stream_gemm(const __grid_constant__ StreamLaunch P) {
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + SW_STAGES * SW_STAGE_BYTES);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(bars + 2 * SW_STAGES);
   const __nv_bfloat16** xsrc = reinterpret_cast<const __nv_bfloat16**>(bars + 2 * SW_STAGES + 2);
+  TileInfo* slot = reinterpret_cast<TileInfo*>(xsrc + 2 * SW_TOK);  // [SW_STAGES]
   const uint32_t smem_base = smem_u32(smem);
   const uint32_t full0 = smem_u32(bars), empty0 = full0 + 8 * SW_STAGES;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
     for (int s = 0; s < SW_STAGES; ++s) {
-      // the producer lane's expect_tx arrival plus one cp.async arrival per producer lane
+      // the producer lane's arrival plus one cp.async arrival per producer lane
       mbar_init(full0 + 8 * s, 1 + 32);
       mbar_init(empty0 + 8 * s, SW_CONSUMERS);
     }
@@ -231,56 +261,116 @@ k_stream_gemm(const __grid_constant__ StreamLaunch P) {
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   __syncthreads();
-  const int total = *P.n_tiles;
   uint32_t it = 0;
   if (warp == 0) {
-    // ---- producer warp: lane 0 waits and issues the weight box, every lane
-    // copies up to two token rows of the stage
-    bool ok = true;
-    int4 na = make_int4(0, 0, 0, 0), nb = na;
-    fetch_tile(P, blockIdx.x, total, na, nb);
-    for (int tile = blockIdx.x; tile < total && ok; tile += gridDim.x) {
-      TileInfo ti;
-      unpack_tile(P, na, nb, ti);
-      fetch_tile(P, tile + gridDim.x, total, na, nb);  // next descriptor in flight
-      const StreamOp& op = P.op[ti.op];
-      const CUtensorMap* map = op.tmaps + ti.node;
-      const int rt0 = (ti.grp * ti.Ng + ti.row0) / SW_ROWS;
-      const long acol = (long)ti.grp * ti.K;
-      __syncwarp();  // earlier readers of xsrc are done
+    // ---- producer warp.  Tiles are claimed from the launch's counter one
+    // ahead of use; the decoded tile rides in the shared slot of its first
+    // stage.  Lane 0 waits and issues the weight box, all lanes copy token rows.
+    const int tiles0 = op_tiles(P.op[0]);
+    const int total = tiles0 + (P.n_ops > 1 ? op_tiles(P.op[1]) : 0);
+    // token-row sources of a tile, double-buffered so the next tile's are
+    // prepared while the current one streams
+    auto prepare = [&](const TileInfo& t, int buf) {
+      const StreamOp& op = P.op[t.op];
+      const long acol = (long)t.grp * t.K;
 #pragma unroll
       for (int h = 0; h < 2; ++h) {
         const int m = lane + 32 * h;
-        if (m < ti.M) {
-          const int row = ti.tok0 + m;
+        if (t.active && m < t.M) {
+          const int row = t.tok0 + m;
           const long r = op.gather ? op.gather[row] : row;
-          xsrc[m] = op.X + r * op.ldx + acol;
+          xsrc[buf * SW_TOK + m] = op.X + r * op.ldx + acol;
+        }
+      }
+    };
+    int cur = lane == 0 ? atomicAdd(P.ctr, 1) : 0;
+    cur = __shfl_sync(0xffffffffu, cur, 0);
+    TileInfo ti;
+    if (cur < total) {
+      decode_tile(P, cur, tiles0, ti);
+      prepare(ti, 0);
+    }
+    __syncwarp();
+    int buf = 0;
+    bool ok = true;
+    while (cur < total && ok) {
+      int nxt = lane == 0 ? atomicAdd(P.ctr, 1) : 0;  // next claim in flight
+      TileInfo tn;
+      bool prepared = false;
+      if (ti.active) {
+        const StreamOp& op = P.op[ti.op];
+        const CUtensorMap* map = op.tmaps + ti.node;
+        const int rt0 = (ti.grp * ti.Ng + ti.row0) / SW_ROWS;
+        const __nv_bfloat16* const* xs = xsrc + buf * SW_TOK;
+        const int nkb = (ti.K + SW_BOX - 1) / SW_BOX;
+        for (int cb = 0; cb < ti.ncb && ok; ++cb) {
+          for (int kb = 0; kb < nkb; ++kb, ++it) {
+            const uint32_t s = it % SW_STAGES;
+            int good = 1;
+            if (lane == 0) {
+              good = mbar_wait(empty0 + 8 * s, ((it / SW_STAGES) & 1) ^ 1, abort_flag) ? 1 : 0;
+              if (good) {
+                if (cb == 0 && kb == 0) slot[s] = ti;
+                mbar_expect_tx(full0 + 8 * s, SW_BOX_BYTES);
+              }
+            }
+            good = __shfl_sync(0xffffffffu, good, 0);
+            if (!good) {
+              ok = false;
+              break;
+            }
+            const uint32_t wbox = smem_base + s * SW_STAGE_BYTES;
+            if (lane == 0) tma_load_tile(wbox, map, kb, rt0 + cb, full0 + 8 * s);
+            // token rows: M rows x 128 bytes as 16-byte pieces over the 32 lanes
+            for (int piece = lane; piece < ti.M * 8; piece += 32) {
+              const int m = piece >> 3, u = piece & 7;
+              cp_async16(wbox + SW_BOX_BYTES + m * SW_XROW + u * 16, xs[m] + kb * SW_BOX + u * 8);
+            }
+            cp_async_arrive(full0 + 8 * s);
+            if (!prepared && cb == 0 && (kb == 1 || kb == nkb - 1)) {
+              // the next tile: decode and prepare its rows while these stages stream
+              nxt = __shfl_sync(0xffffffffu, nxt, 0);
+              if (nxt < total) {
+                decode_tile(P, nxt, tiles0, tn);
+                prepare(tn, buf ^ 1);
+                if (lane == 0 && tn.active)
+                  asm volatile("prefetch.tensormap [%0];" ::"l"(
+                      reinterpret_cast<uint64_t>(P.op[tn.op].tmaps + tn.node)) : "memory");
+              }
+              prepared = true;
+            }
+          }
+        }
+      }
+      if (!prepared) {
+        nxt = __shfl_sync(0xffffffffu, nxt, 0);
+        if (nxt < total) {
+          decode_tile(P, nxt, tiles0, tn);
+          prepare(tn, buf ^ 1);
         }
       }
       __syncwarp();
-      const int nkb = (ti.K + SW_BOX - 1) / SW_BOX;
-      for (int cb = 0; cb < ti.ncb && ok; ++cb) {
-        for (int kb = 0; kb < nkb; ++kb, ++it) {
-          const uint32_t s = it % SW_STAGES;
-          int good = 1;
-          if (lane == 0) {
-            good = mbar_wait(empty0 + 8 * s, ((it / SW_STAGES) & 1) ^ 1, abort_flag) ? 1 : 0;
-            if (good) mbar_expect_tx(full0 + 8 * s, SW_BOX_BYTES);
-          }
-          good = __shfl_sync(0xffffffffu, good, 0);
-          if (!good) {
-            ok = false;
-            break;
-          }
-          const uint32_t wbox = smem_base + s * SW_STAGE_BYTES;
-          if (lane == 0) tma_load_tile(wbox, map, kb, rt0 + cb, full0 + 8 * s);
-          // token rows: M rows x 128 bytes as 16-byte pieces over the 32 lanes
-          for (int piece = lane; piece < ti.M * 8; piece += 32) {
-            const int m = piece >> 3, u = piece & 7;
-            cp_async16(wbox + SW_BOX_BYTES + m * SW_XROW + u * 16, xsrc[m] + kb * SW_BOX + u * 8);
-          }
-          cp_async_arrive(full0 + 8 * s);
+      cur = nxt;
+      ti = tn;
+      buf ^= 1;
+    }
+    if (ok) {
+      // sentinel stage: tells the consumers that no tile follows
+      const uint32_t s = it % SW_STAGES;
+      int good = 1;
+      if (lane == 0) {
+        good = mbar_wait(empty0 + 8 * s, ((it / SW_STAGES) & 1) ^ 1, abort_flag) ? 1 : 0;
+        if (good) {
+          slot[s].op = -1;
+          mbar_arrive(full0 + 8 * s);
         }
+      }
+      good = __shfl_sync(0xffffffffu, good, 0);
+      if (good) {
+        cp_async_arrive(full0 + 8 * s);
+        ++it;
+      } else {
+        ok = false;
       }
     }
     if (!ok && lane == 0) {
@@ -294,13 +384,18 @@ k_stream_gemm(const __grid_constant__ StreamLaunch P) {
     }
     return;
   }
-  // ---- consumers
-  int4 na = make_int4(0, 0, 0, 0), nb = na;
-  fetch_tile(P, blockIdx.x, total, na, nb);
-  for (int tile = blockIdx.x; tile < total; tile += gridDim.x) {
-    TileInfo ti;
-    unpack_tile(P, na, nb, ti);
-    fetch_tile(P, tile + gridDim.x, total, na, nb);
+  // ---- consumers: the first stage of every tile carries its description
+  while (true) {
+    const uint32_t s = it % SW_STAGES;
+    if (!mbar_wait(full0 + 8 * s, (it / SW_STAGES) & 1, abort_flag)) {
+      if (lane == 0) {
+        atomicExch(P.err, LX_ERR_TIMEOUT);
+        *abort_flag = 1;
+      }
+      return;
+    }
+    const TileInfo ti = slot[s];
+    if (ti.op < 0) return;  // sentinel
     const int nt = (ti.M + 7) / 8;
     bool ok;
     if (nt <= 1) ok = consume_tile<1>(P, ti, smem_base, full0, empty0, it, abort_flag);
@@ -320,7 +415,8 @@ k_stream_gemm(const __grid_constant__ StreamLaunch P) {
 }  // namespace
 
 int stream_smem_bytes() {
-  return SW_STAGES * SW_STAGE_BYTES + 2 * SW_STAGES * 8 + 16 + SW_TOK * 8 + 1024;
+  return SW_STAGES * SW_STAGE_BYTES + 2 * SW_STAGES * 8 + 16 + 2 * SW_TOK * 8 +
+         SW_STAGES * (int)sizeof(TileInfo) + 1024;
 }
 
 lx_status launch_stream(lx_layer* L, const StreamLaunch& P, cudaStream_t s, const char* name) {
@@ -328,17 +424,18 @@ lx_status launch_stream(lx_layer* L, const StreamLaunch& P, cudaStream_t s, cons
   static bool done[64] = {};
   LX_CUDA(smem_cap_once((const void*)k_stream_gemm, smem, L->device, done));
   ProfScope ps(L, s, name);
-  k_stream_gemm<<<L->num_sms * 2, SW_THREADS, smem, s>>>(P);
+  k_stream_gemm<<<L->num_sms * 3, SW_THREADS, smem, s>>>(P);
   LX_CUDA(cudaGetLastError());
   return LX_OK;
 }
 
-static StreamOp make_op(lx_layer* L, int op, const __nv_bfloat16* X, long ldx, const int* gather,
-                        void* out, long ldo, bool out_f32) {
+static StreamOp make_op(lx_layer* L, int op, int T, const __nv_bfloat16* X, long ldx,
+                        const int* gather, void* out, long ldo, bool out_f32) {
   StreamOp o;
   o.shape = op_shape(L, op);
   o.tmaps = L->d_tmaps + (size_t)op * L->N;
-  o.items = o.shape.on_anchors ? L->d_anchors : L->d_corrs;
+  o.items = o.shape.on_anchors ? L->ws.act : L->ws.act + L->n_anchor;
+  o.n_active = L->ws.act_n + (o.shape.on_anchors ? 0 : 1);
   o.n_items = o.shape.on_anchors ? L->n_anchor : L->n_corr;
   o.tile_off = nullptr;
   o.node_off = L->ws.key_off;
@@ -349,25 +446,25 @@ static StreamOp make_op(lx_layer* L, int op, const __nv_bfloat16* X, long ldx, c
   o.ldo = ldo;
   o.out_f32 = out_f32 ? 1 : 0;
   o.rank = L->d_rank;
+  int ng_max = 0;
+  for (int n : (o.shape.on_anchors ? L->anchors : L->corrs))
+    ng_max = std::max(ng_max, o.shape.n_const + o.shape.n_rank * L->rank[n]);
+  o.ncol_max = (ng_max + SW_ROWS - 1) / SW_ROWS;
+  o.ntb = (T + SW_TOK - 1) / SW_TOK;
   return o;
 }
 
-// One launch of launch group g (its tile list was built during bucketing).
+// One streaming launch (launch group g) over up to two ops' tile grids.
 static lx_status run_stream(lx_layer* L, int g, const StreamOp& o0, const StreamOp* o1,
                             cudaStream_t s, const char* name) {
   StreamLaunch P;
-  P.op[0] = o0;
-  P.op_id[0] = stream_group_op(g, 0);
-  P.n_ops = 1;
-  P.op_id[1] = -1;
-  if (o1) {
-    P.op[1] = *o1;
-    P.op_id[1] = stream_group_op(g, 1);
-    P.n_ops = 2;
+  P.n_ops = 0;
+  for (const StreamOp* o : {&o0, o1}) {
+    if (!o || o->n_items == 0) continue;
+    P.op[P.n_ops++] = *o;
   }
-  if (o0.n_items == 0 && (!o1 || o1->n_items == 0)) return LX_OK;
-  P.tiles = L->ws.stiles + (size_t)g * L->ws.stile_cap * 2;
-  P.n_tiles = L->ws.stile_cnt + g;
+  if (P.n_ops == 0) return LX_OK;
+  P.ctr = L->ws.sctr + g;
   P.err = L->ws.err;
   return launch_stream(L, P, s, name);
 }
@@ -378,18 +475,18 @@ lx_status launch_fast_experts(lx_layer* L, const void* x, int T, int k, void* y,
   const long H = L->H, I = L->I, rmax = L->max_rank;
   const __nv_bfloat16* xb = static_cast<const __nv_bfloat16*>(x);
   // x-side: shared anchor gate/up, and x V of every correction
-  const StreamOp up_v = make_op(L, OP_UP_V, xb, H, w.node_tok, w.Pb, 2 * rmax, false);
-  LX_TRY(run_stream(L, 0, make_op(L, OP_UP_ANCHOR, xb, H, w.node_tok, w.h, 2 * I, true), &up_v,
+  const StreamOp up_v = make_op(L, OP_UP_V, T, xb, H, w.node_tok, w.Pb, 2 * rmax, false);
+  LX_TRY(run_stream(L, 0, make_op(L, OP_UP_ANCHOR, T, xb, H, w.node_tok, w.h, 2 * I, true), &up_v,
                     s, "stream_up_anchor_V"));
-  LX_TRY(run_stream(L, 1, make_op(L, OP_UP_U, w.Pb, 2 * rmax, nullptr, w.h, 2 * I, true),
+  LX_TRY(run_stream(L, 1, make_op(L, OP_UP_U, T, w.Pb, 2 * rmax, nullptr, w.h, 2 * I, true),
                     nullptr, s, "stream_up_U"));
   LX_TRY(launch_swiglu(L, T, k, w.zb, true, s));
   // z-side: shared anchor down projection, and z Vd of every correction
-  const StreamOp dn_v = make_op(L, OP_DN_V, w.zb, I, nullptr, w.Qb, rmax, false);
-  LX_TRY(run_stream(L, 2, make_op(L, OP_DN_ANCHOR, w.zb, I, nullptr, w.ypart, H, true), &dn_v,
+  const StreamOp dn_v = make_op(L, OP_DN_V, T, w.zb, I, nullptr, w.Qb, rmax, false);
+  LX_TRY(run_stream(L, 2, make_op(L, OP_DN_ANCHOR, T, w.zb, I, nullptr, w.ypart, H, true), &dn_v,
                     s, "stream_dn_anchor_V"));
-  LX_TRY(run_stream(L, 3, make_op(L, OP_DN_U, w.Qb, rmax, nullptr, w.ypart, H, true), nullptr, s,
-                    "stream_dn_U"));
+  LX_TRY(run_stream(L, 3, make_op(L, OP_DN_U, T, w.Qb, rmax, nullptr, w.ypart, H, true), nullptr,
+                    s, "stream_dn_U"));
   LX_TRY(launch_combine(L, T, k, y, s));
   return LX_OK;
 }
