@@ -167,6 +167,22 @@ def kernel_bytes(name, st, src, esz):
     return table.get(name)
 
 
+def kernel_flops(name, st, src):
+    """Dense multiply-add FLOPs per launch of a tensor-core kernel: 2 x (rows of
+    each node's bucket) x (its output columns) x (its K), over real rows only."""
+    H, I = src.d_model, src.d_ff
+    Ra, rr = st["R_anchor"], st["corr_r_rows"]
+    table = {
+        "tc_up_anchor": 2 * Ra * 2 * I * H,
+        "tc_up_V": 2 * rr * 2 * H,
+        "tc_up_U": 2 * rr * 2 * I,
+        "tc_dn_anchor": 2 * Ra * H * I,
+        "tc_dn_V": 2 * rr * I,
+        "tc_dn_U": 2 * rr * H,
+    }
+    return table.get(name)
+
+
 def step_bytes(st, src, esz):
     from paper_2608_07814_gb300 import cost
     c = cost.step_counts(src.d_model, src.d_ff, src.n_experts, src.node_parent, src.node_rank,
@@ -275,7 +291,7 @@ def run_lx(args, rank, world, local_rank):
     per_copy = [L.read_profile(cap=1 << 20) for L in layers]
     totals, counts = {}, {}
     launches = 0
-    kbytes = {}
+    kbytes, kflops = {}, {}
     for c, recs in enumerate(per_copy):
         steps_of_copy = [i for i in range(args.steps) if i % n_copies == c]
         per_step = len(recs) // max(1, len(steps_of_copy))
@@ -288,6 +304,9 @@ def run_lx(args, rank, world, local_rank):
             b = kernel_bytes(name, stats[step_i % n_batches], src, esz)
             if b is not None:
                 kbytes[name] = kbytes.get(name, 0.0) + b
+            f = kernel_flops(name, stats[step_i % n_batches], src)
+            if f is not None:
+                kflops[name] = kflops.get(name, 0.0) + f
 
     # e2e: host buffers, copies inside the timed region, a read of every result
     xh = [lx.host_to_torch(x, src.dtype).pin_memory() for x in xs_host]
@@ -335,6 +354,16 @@ def run_lx(args, rank, world, local_rank):
                 "unit": "GB/s", "frac": round(ach / hbm, 4), "traffic": traffic_for(dom),
                 "algorithmic_bytes_per_launch": round(bytes_per_launch),
                 "avg_launch_us": round(avg_ms * 1e3, 2), "peak_source": f"{peak_kind} hbm_gbs"}
+    elif dom in kflops:
+        # a contraction on the tensor cores, timed alone per launch: burst bf16 peak
+        tf = float(peaks["bf16_tflops"])
+        flops_per_launch = kflops[dom] / counts[dom]
+        ach = flops_per_launch / (avg_ms * 1e-3) / 1e12
+        roof = {"kernel": dom, "bound": "tensor", "achieved": round(ach, 1), "peak": tf,
+                "unit": "TFLOP/s", "frac": round(ach / tf, 4), "traffic": traffic_for(dom),
+                "algorithmic_flops_per_launch": round(flops_per_launch),
+                "avg_launch_us": round(avg_ms * 1e3, 2),
+                "peak_source": f"{peak_kind} bf16_tflops (burst)"}
     sb = [step_bytes(stats[i % n_batches], src, esz)["bytes"] for i in range(args.steps)]
     step_gbs = sum(sb) / (ms * 1e-3) / 1e9
     tokens = T * args.steps * world

@@ -83,6 +83,30 @@ OpShape op_shape(const lx_layer* L, int op) {
 
 int op_max_items(const lx_layer* L) { return std::max(L->n_anchor, L->n_corr); }
 
+static PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
+  void* fn = nullptr;
+  cudaDriverEntryPointQueryResult q;
+  cudaError_t ce = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000,
+                                                    cudaEnableDefault, &q);
+  if (ce != cudaSuccess || q != cudaDriverEntryPointSuccess || !fn) return nullptr;
+  return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+}
+
+// TMA map of a bf16 activation buffer [rows][ld] read as 128-row x 64-column
+// boxes (the tensor-core A operand when its rows are already in node-row order)
+static bool encode_rows_map(CUtensorMap* m, void* base, long rows, long ld) {
+  auto encode = get_encode();
+  if (!encode) return false;
+  const cuuint64_t dims[2] = {(cuuint64_t)ld, (cuuint64_t)rows};
+  const cuuint64_t strides[1] = {(cuuint64_t)ld * 2};
+  const cuuint32_t box[2] = {64, (cuuint32_t)tc_tile_tokens()};
+  const cuuint32_t estr[2] = {1, 1};
+  return encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, dims, strides, box, estr,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) ==
+         CUDA_SUCCESS;
+}
+
 // ---------------------------------------------------------------------------
 // workspace
 // ---------------------------------------------------------------------------
@@ -120,7 +144,8 @@ static lx_status ensure_workspace(lx_layer* L, int T, int k, cudaStream_t s) {
       {(void**)&w.Qb, 2 * Rmax * rmax},
       {(void**)&w.act, sizeof(int) * std::max(1, L->n_anchor + L->n_corr)},
       {(void**)&w.act_n, sizeof(int) * 2},
-      {(void**)&w.sctr, sizeof(int) * N_STREAM_GROUPS},
+      {(void**)&w.sctr, sizeof(int) * N_TILE_COUNTERS},
+      {(void**)&w.xmaps, sizeof(CUtensorMap) * 3},
       {(void**)&w.err, 256},
   };
   size_t total = 0;
@@ -149,6 +174,18 @@ static lx_status ensure_workspace(lx_layer* L, int T, int k, cudaStream_t s) {
   if (e != cudaSuccess) return cuda_fail(e, "clear workspace error word");
   w.cap_T = cT;
   w.cap_k = ck;
+  w.rows_cap = Rmax;
+  if (L->stream_ok) {
+    CUtensorMap maps[3];
+    std::memset(maps, 0, sizeof(maps));
+    const bool okm = encode_rows_map(&maps[0], w.Pb, Rmax, 2 * rmax) &&
+                     encode_rows_map(&maps[1], w.zb, Rmax, L->I) &&
+                     encode_rows_map(&maps[2], w.Qb, Rmax, rmax);
+    if (!okm) return fail(LX_ERR_CUDA, "cuTensorMapEncodeTiled(activation maps) failed");
+    e = cudaMemcpyAsync(w.xmaps, maps, sizeof(maps), cudaMemcpyHostToDevice, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return cuda_fail(e, "copy activation maps");
+  }
   L->last_T = L->last_k = 0;
   return LX_OK;
 }
@@ -184,18 +221,19 @@ static bool use_stream(const lx_layer* L, int T) {
   return L->path_mode == LX_PATH_AUTO && L->stream_ok && T <= kStreamMaxT;
 }
 
+// Larger batches: the tensor-core kernels (same layer requirements).
+static bool use_tc(const lx_layer* L, int T) {
+  return L->path_mode == LX_PATH_AUTO && L->stream_ok && T > kStreamMaxT;
+}
+
 // TMA descriptors of every weight matrix the streaming kernels read: each
 // matrix is a 4-D tensor {64 K, 64 rows, K/64 tiles, rows/64 tiles} over the
 // tiled layout, read one 64x64 box (8 KiB, contiguous) at a time.
 static lx_status encode_tensor_maps(lx_layer* L, cudaStream_t s) {
   L->stream_ok = false;
   if (!L->tiled) return LX_OK;
-  void* fn = nullptr;
-  cudaDriverEntryPointQueryResult q;
-  cudaError_t ce = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000,
-                                                    cudaEnableDefault, &q);
-  if (ce != cudaSuccess || q != cudaDriverEntryPointSuccess || !fn) return LX_OK;
-  auto encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  auto encode = get_encode();
+  if (!encode) return LX_OK;
   std::vector<CUtensorMap> maps((size_t)N_OPS * L->N);
   std::memset(maps.data(), 0, maps.size() * sizeof(CUtensorMap));
   for (int op = 0; op < N_OPS; ++op) {
@@ -530,6 +568,8 @@ extern "C" lx_status lx_moe_forward(lx_layer* L, const void* x, int32_t T, int32
   L->last_k = k;
   if (use_stream(L, T)) {
     LX_TRY(launch_fast_experts(L, x, T, k, y, s));
+  } else if (use_tc(L, T)) {
+    LX_TRY(launch_tc_experts(L, x, T, k, y, s));
   } else {
     LX_TRY(launch_generic_experts(L, x, T, k, y, s));
   }

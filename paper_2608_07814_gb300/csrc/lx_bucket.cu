@@ -99,7 +99,7 @@ __device__ __forceinline__ int plan_tiles(const PlanArgs& pa, int p, int r, int 
   const OpShape sh = pa.shape[p];
   const int Ng = sh.n_const + sh.n_rank * r;
   int ncol = (Ng + pa.bn[p] - 1) / pa.bn[p];
-  if (p >= PLAN_STREAM) {
+  if (p >= PLAN_STREAM && p < PLAN_TC) {
     const int ncb = stream_col_blocks(sh.k_const + sh.k_rank * r, ncol);
     ncol = (ncol + ncb - 1) / ncb;
   }
@@ -129,7 +129,7 @@ __device__ void publish_active(const int* cnt, const int* anchors, int n_anchor,
     }
     if (lane == 0) act_n[warp] = base;
   }
-  if (threadIdx.x < N_STREAM_GROUPS) sctr[threadIdx.x] = 0;
+  if (threadIdx.x < N_TILE_COUNTERS) sctr[threadIdx.x] = 0;
 }
 
 // one CTA: node/expert offsets and the tile prefix of every plan
@@ -374,8 +374,8 @@ static PlanArgs make_plans(const lx_layer* L, int n_plans) {
     pa.shape[p] = op_shape(L, op);
     pa.items[p] = pa.shape[p].on_anchors ? L->d_anchors : L->d_corrs;
     pa.n_items[p] = pa.shape[p].on_anchors ? L->n_anchor : L->n_corr;
-    pa.bm[p] = p < N_OPS ? G_BM : stream_tile_tokens();
-    pa.bn[p] = p < N_OPS ? G_BN : stream_tile_rows();
+    pa.bm[p] = p < PLAN_STREAM ? G_BM : p < PLAN_TC ? stream_tile_tokens() : tc_tile_tokens();
+    pa.bn[p] = p < PLAN_STREAM ? G_BN : p < PLAN_TC ? stream_tile_rows() : tc_tile_cols();
   }
   return pa;
 }
@@ -423,7 +423,7 @@ lx_status launch_bucket(lx_layer* L, const int* topk_id, int T, int k, cudaStrea
     LX_CUDA(cudaGetLastError());
   }
   {
-    const PlanArgs pa = make_plans(L, N_OPS);
+    const PlanArgs pa = make_plans(L, N_PLANS);
     ProfScope ps(L, s, "bucket_offsets");
     k_offsets_plan<<<1, 1024, 0, s>>>(w.key_cnt, L->N, L->E, w.key_off, L->d_rank, w.tile_off,
                                       op_max_items(L), pa, L->d_anchors, L->n_anchor, L->d_corrs,

@@ -129,8 +129,10 @@ enum OpKind {
 // 64-column tiles); plan N_OPS + p is op p for the streaming kernel (64-token
 // x 64-weight-row blocks; ops with a short K take several column blocks per
 // tile, see stream_col_blocks).
-constexpr int N_PLANS = 2 * N_OPS;
+constexpr int N_PLANS = 3 * N_OPS;
 constexpr int PLAN_STREAM = N_OPS;
+constexpr int PLAN_TC = 2 * N_OPS;   // tensor-core tiles: 128 tokens x 256 columns
+constexpr int N_TILE_COUNTERS = 16;  // dynamic tile counters, zeroed by the bucketing
 
 // Per-op shape rule: for node n with rank r, each group has
 //   N_g = n_const + n_rank * r output columns and K = k_const + k_rank * r.
@@ -205,11 +207,34 @@ struct StreamLaunch {
   int* err;                  // device error word (LX_ERR_TIMEOUT on a bounded wait)
 };
 
+// Tensor-core (prefill) grouped GEMM: one op per launch
+struct TcLaunch {
+  OpShape shape;
+  const int* items;          // node ids of the op's plan
+  int n_items;
+  const int* tile_off;       // [n_items+1] tensor-core plan
+  const int* node_off;
+  const int* rank;
+  const CUtensorMap* wmaps;  // [n_nodes] weight tensor maps of the op
+  const __nv_bfloat16* X;    // gathered A rows (with gather), else unused
+  long ldx;
+  const int* gather;         // row -> X row, or null: A from xmap (rows in node-row order)
+  const CUtensorMap* xmap;   // TMA map of the A buffer when gather is null
+  int xcol;                  // column offset of A inside xmap
+  void* out;
+  long ldo;
+  int out_f32;
+  long rows_cap;             // rows of the output buffer (bounds check)
+  int* ctr;                  // dynamic tile counter (zeroed by the bucketing)
+  int* err;
+};
+
 // ---------------------------------------------------------------------------
 // device workspace of one forward
 // ---------------------------------------------------------------------------
 struct Workspace {
   int cap_T = 0, cap_k = 0;
+  long rows_cap = 0;            // Rmax
   void* base = nullptr;
   size_t bytes = 0;
   // routing
@@ -239,7 +264,8 @@ struct Workspace {
   __nv_bfloat16* Qb = nullptr;  // [Rmax][rmax]
   int* act = nullptr;           // [n_anchor + n_corr] active anchors, then active corrections
   int* act_n = nullptr;         // [2] their counts
-  int* sctr = nullptr;          // [N_STREAM_GROUPS] streaming tile counters
+  int* sctr = nullptr;          // [N_TILE_COUNTERS] streaming / tensor-core tile counters
+  CUtensorMap* xmaps = nullptr; // [3] TMA maps of Pb, zb, Qb (tensor-core A operands)
   int* err = nullptr;           // device error word
 };
 
@@ -314,6 +340,10 @@ lx_status launch_generic_experts(lx_layer* L, const void* x, int T, int k, void*
 lx_status launch_swiglu(lx_layer* L, int T, int k, void* z, bool z_bf16, cudaStream_t s);
 lx_status launch_combine(lx_layer* L, int T, int k, void* y, cudaStream_t s);
 lx_status launch_fast_experts(lx_layer* L, const void* x, int T, int k, void* y, cudaStream_t s);
+lx_status launch_tc_experts(lx_layer* L, const void* x, int T, int k, void* y, cudaStream_t s);
+int tc_tile_tokens();
+int tc_tile_cols();
+lx_status launch_tc(lx_layer* L, const TcLaunch& P, cudaStream_t s, const char* name);
 lx_status launch_stream(lx_layer* L, const StreamLaunch& P, cudaStream_t s, const char* name);
 lx_status launch_bucket_small(lx_layer* L, const float* logits, const int* ids_in, int T, int k,
                               int* topk_id, float* topk_w, cudaStream_t s);

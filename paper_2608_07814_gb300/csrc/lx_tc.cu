@@ -1,0 +1,522 @@
+// Tensor-core grouped GEMM for large token counts (prefill), sm_103a tcgen05.
+//
+// out[rows of node n][cols] = X[rows][K] . W_n[cols][K]^T for every active
+// node, in tiles of 128 tokens (rows of the node's bucket) x BN <= 256 output
+// columns over the full K -- the dense anchor and factor contractions of the
+// amortised forward (Sec. 5.1), each evaluated once per (token, node).
+//
+// One persistent CTA per SM, 8 warps:
+//   warp 0      producer: claims tiles from the launch's counter (one ahead),
+//               loads the weight boxes (64 rows x 64 K, 128B swizzle, tiled
+//               layout) with TMA, and the 128 token rows either with one TMA
+//               box (rows already contiguous in node-row order: P, z, Q) or
+//               with 16-byte cp.async gathers (x rows by token id); gathered
+//               rows are made visible to the tensor core's async proxy with
+//               fence.proxy.async before the stage is marked full;
+//   warp 1      allocates 256 TMEM columns; lane 0 issues tcgen05.mma
+//               (kind::f16, bf16 x bf16 -> fp32, M=128, N=BN, K=16 per
+//               instruction) and commits stage releases and accumulator-ready
+//               signals with tcgen05.commit;
+//   warps 4..7  epilogue: tcgen05.ld (32 lanes x 16 columns per load) from the
+//               accumulator and row-wise stores to global memory.
+// Every wait is bounded; a wait that gives up records LX_ERR_TIMEOUT, makes the
+// other roles stop, drains the CTA's copies and MMAs in flight and frees TMEM.
+#include <cuda.h>
+
+#include <algorithm>
+
+#include "lx_internal.cuh"
+
+namespace lx {
+
+namespace {
+
+constexpr int TC_BM = 128;          // tokens per tile (UMMA M)
+constexpr int TC_BN = 256;          // max output columns per tile (UMMA N)
+constexpr int TC_BK = 64;           // K per stage (one 128-byte swizzle row)
+constexpr int TC_STAGES = 4;
+constexpr int TC_A_BYTES = TC_BM * TC_BK * 2;   // 16 KiB
+constexpr int TC_B_BYTES = TC_BN * TC_BK * 2;   // 32 KiB
+constexpr int TC_STAGE_BYTES = TC_A_BYTES + TC_B_BYTES;
+constexpr int TC_THREADS = 256;
+constexpr int TC_TMEM_COLS = 256;
+constexpr unsigned long long TC_TIMEOUT_CYCLES = 4000000000ull;  // ~2 s
+static_assert(TC_STAGE_BYTES % 1024 == 0, "stages keep the 1024-byte swizzle alignment");
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// bounded wait; false on timeout or when the CTA aborts
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const unsigned long long t0 = clock64();
+  while (true) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (abort_flag && *abort_flag) return false;
+    if (clock64() - t0 > TC_TIMEOUT_CYCLES) return false;
+  }
+}
+
+__device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap* map, int c0, int c1,
+                                            int c2, int c3, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3, %4, %5}], [%6];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(bar)
+      : "memory");
+}
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int c0, int c1,
+                                            uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(bar)
+      : "memory");
+}
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst),
+               "l"(reinterpret_cast<uint64_t>(src))
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+__device__ __forceinline__ void fence_proxy_async() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// ---- tcgen05 ---------------------------------------------------------------
+// Shared-memory matrix descriptor of a K-major tile whose rows are 128 bytes
+// (64 bf16) with the 128-byte swizzle, rows packed (8-row atoms 1024 bytes
+// apart): start address >> 4 at bits 0..13, leading-dimension offset (unused
+// for this layout, 16 bytes) at bits 16..29, stride between 8-row atoms
+// (1024 bytes) at bits 32..45, descriptor version 1 at bits 46..47, swizzle
+// mode 2 (128-byte) at bits 61..63.
+__device__ __forceinline__ uint64_t smem_desc(uint32_t addr) {
+  return (uint64_t)((addr >> 4) & 0x3FFF) | ((uint64_t)(16 >> 4) << 16) |
+         ((uint64_t)(1024 >> 4) << 32) | (1ull << 46) | (2ull << 61);
+}
+
+// Instruction descriptor, kind::f16: D fp32 (bits 4..5 = 1), A and B bf16
+// (bits 7..9 = 1, bits 10..12 = 1), both K-major (bits 15, 16 = 0),
+// N >> 3 at bits 17..22, M >> 4 at bits 24..28.
+__host__ __device__ constexpr uint32_t instr_desc(int M, int N) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) |
+         ((uint32_t)(M >> 4) << 24);
+}
+
+static_assert(instr_desc(128, 256) == 0x08400490u, "M=128 N=256 bf16->f32 descriptor");
+static_assert(instr_desc(128, 64) == 0x08100490u, "M=128 N=64 bf16->f32 descriptor");
+
+__device__ __forceinline__ void tc_mma(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
+                                       uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(tmem_d),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+__device__ __forceinline__ void tc_commit(uint32_t bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+      : "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_ld16(uint32_t taddr, float (&v)[16]) {
+  uint32_t r[16];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+struct TcTile {
+  int node, grp, row0, tok0, M, Ng, K, BN;  // BN < 0: sentinel
+};
+
+// tile index -> (node, token block, group, column block) through the plan prefix
+__device__ __forceinline__ void tc_decode(const TcLaunch& P, int tile, TcTile& t) {
+  const int* to = P.tile_off;
+  int lo = 0, hi = P.n_items;
+  while (hi - lo > 1) {
+    const int mid = (lo + hi) >> 1;
+    if (to[mid] <= tile) lo = mid; else hi = mid;
+  }
+  const int n = P.items[lo];
+  const int local = tile - to[lo];
+  const int r = P.rank[n];
+  t.Ng = P.shape.n_const + P.shape.n_rank * r;
+  t.K = P.shape.k_const + P.shape.k_rank * r;
+  const int ncol = (t.Ng + TC_BN - 1) / TC_BN;
+  const int per_tb = ncol * P.shape.groups;
+  const int tb = local / per_tb, rem = local % per_tb;
+  t.grp = rem / ncol;
+  t.row0 = (rem % ncol) * TC_BN;
+  t.BN = min(TC_BN, t.Ng - t.row0);
+  t.node = n;
+  t.tok0 = P.node_off[n] + tb * TC_BM;
+  t.M = min(TC_BM, P.node_off[n + 1] - t.tok0);
+}
+
+__global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant__ TcLaunch P) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + TC_STAGES * TC_STAGE_BYTES);
+  // full[S], empty[S], tmem_full, tmem_empty, drain
+  const uint32_t full0 = smem_u32(bars), empty0 = full0 + 8 * TC_STAGES;
+  const uint32_t tfull = empty0 + 8 * TC_STAGES, tempty = tfull + 8, drain = tempty + 8;
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(bars + 2 * TC_STAGES + 3);
+  uint32_t* tmem_base_s = reinterpret_cast<uint32_t*>(bars + 2 * TC_STAGES + 4);
+  TcTile* slot = reinterpret_cast<TcTile*>(bars + 2 * TC_STAGES + 5);  // [TC_STAGES]
+  TcTile* eslot = slot + TC_STAGES;                                     // epilogue hand-off
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t smem_base = smem_u32(smem);
+  uint32_t prod_it = 0;  // stages the producer issued
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < TC_STAGES; ++s) {
+      mbar_init(full0 + 8 * s, 1 + 32);  // producer arrival + one per producer lane
+      mbar_init(empty0 + 8 * s, 1);      // tcgen05.commit
+    }
+    mbar_init(tfull, 2);   // MMA thread's arrival (tile info written) + tcgen05.commit
+    mbar_init(tempty, 4);  // one arrival per epilogue warp
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(tmem_base_s)),
+                 "r"(TC_TMEM_COLS)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_base_s;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer
+    const int total = P.tile_off[P.n_items];
+    int cur = lane == 0 ? atomicAdd(P.ctr, 1) : 0;
+    cur = __shfl_sync(0xffffffffu, cur, 0);
+    TcTile t;
+    if (cur < total) tc_decode(P, cur, t);
+    uint32_t it = 0;
+    bool ok = true;
+    bool pending = false;  // a gathered stage waits for its fence + arrivals
+    uint32_t pend_s = 0;
+    while (cur < total && ok) {
+      int nxt = lane == 0 ? atomicAdd(P.ctr, 1) : 0;
+      // token row sources of this tile (lane handles rows lane + 32 h)
+      const __nv_bfloat16* src[4];
+#pragma unroll
+      for (int h = 0; h < 4; ++h) {
+        const int m = lane + 32 * h;
+        src[h] = nullptr;
+        if (P.gather && m < t.M) src[h] = P.X + (long)P.gather[t.tok0 + m] * P.ldx;
+      }
+      const int nkb = (t.K + TC_BK - 1) / TC_BK;
+      const int rt0 = (t.grp * t.Ng + t.row0) / 64;  // first 64-row weight tile
+      const int nbox = (t.BN + 63) / 64;
+      for (int kb = 0; kb < nkb; ++kb, ++it) {
+        const uint32_t s = it % TC_STAGES;
+        int good = 1;
+        if (lane == 0) {
+          good = mbar_wait(empty0 + 8 * s, ((it / TC_STAGES) & 1) ^ 1, abort_flag) ? 1 : 0;
+          if (good) {
+            if (kb == 0) slot[s] = t;
+            mbar_expect_tx(full0 + 8 * s, nbox * 8192 + (P.gather ? 0 : TC_A_BYTES));
+          }
+        }
+        good = __shfl_sync(0xffffffffu, good, 0);
+        if (!good) {
+          ok = false;
+          break;
+        }
+        const uint32_t a_s = smem_base + s * TC_STAGE_BYTES, b_s = a_s + TC_A_BYTES;
+        if (lane == 0) {
+          for (int b = 0; b < nbox; ++b)
+            tma_load_4d(b_s + b * 8192, P.wmaps + t.node, 0, 0, kb, rt0 + b, full0 + 8 * s);
+          if (!P.gather)
+            tma_load_2d(a_s, P.xmap, (int)(t.grp * t.K) + kb * TC_BK + P.xcol, t.tok0,
+                        full0 + 8 * s);
+        }
+        if (P.gather) {
+          // 128 rows x 128 bytes in the 128-byte swizzle: chunk u of row m goes
+          // to u ^ (m & 7)
+#pragma unroll
+          for (int h = 0; h < 4; ++h) {
+            const int m = lane + 32 * h;
+            if (src[h]) {
+#pragma unroll
+              for (int u = 0; u < 8; ++u)
+                cp_async16(a_s + m * 128 + ((u ^ (m & 7)) << 4), src[h] + kb * TC_BK + 8 * u);
+            }
+          }
+          cp_async_commit();
+          if (pending) {  // the previous gathered stage has landed: publish it
+            cp_async_wait<1>();
+            fence_proxy_async();
+            mbar_arrive(full0 + 8 * pend_s);
+          }
+          pending = true;
+          pend_s = s;
+        } else {
+          mbar_arrive(full0 + 8 * s);
+        }
+      }
+      nxt = __shfl_sync(0xffffffffu, nxt, 0);
+      cur = nxt;
+      if (cur < total) tc_decode(P, cur, t);
+    }
+    if (pending) {
+      cp_async_wait<0>();
+      fence_proxy_async();
+      mbar_arrive(full0 + 8 * pend_s);
+    }
+    if (ok) {
+      // sentinel stage
+      const uint32_t s = it % TC_STAGES;
+      int good = 1;
+      if (lane == 0) {
+        good = mbar_wait(empty0 + 8 * s, ((it / TC_STAGES) & 1) ^ 1, abort_flag) ? 1 : 0;
+        if (good) {
+          slot[s].BN = -1;
+          mbar_arrive(full0 + 8 * s);
+        }
+      }
+      good = __shfl_sync(0xffffffffu, good, 0);
+      if (good) {
+        mbar_arrive(full0 + 8 * s);
+        ++it;
+      } else {
+        ok = false;
+      }
+    }
+    if (!ok && lane == 0) {
+      atomicExch(P.err, LX_ERR_TIMEOUT);
+      *abort_flag = 1;
+    }
+    prod_it = it;
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      uint32_t it = 0, tiles = 0;
+      bool ok = true;
+      while (ok) {
+        const uint32_t s = it % TC_STAGES;
+        if (!mbar_wait(full0 + 8 * s, (it / TC_STAGES) & 1, abort_flag)) { ok = false; break; }
+        const TcTile t = slot[s];
+        // the accumulator must have been drained by the epilogue
+        if (!mbar_wait(tempty, (tiles & 1) ^ 1, abort_flag)) { ok = false; break; }
+        eslot[0] = t;       // tile info for the epilogue, released by this arrival
+        mbar_arrive(tfull);
+        if (t.BN < 0) {     // sentinel: the second arrival completes the phase
+          mbar_arrive(tfull);
+          ++it;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t idesc = instr_desc(TC_BM, t.BN);
+        const int nkb = (t.K + TC_BK - 1) / TC_BK;
+        for (int kb = 0; kb < nkb; ++kb, ++it) {
+          const uint32_t s2 = it % TC_STAGES;
+          if (!mbar_wait(full0 + 8 * s2, (it / TC_STAGES) & 1, abort_flag)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t a_s = smem_base + s2 * TC_STAGE_BYTES, b_s = a_s + TC_A_BYTES;
+#pragma unroll
+          for (int k = 0; k < TC_BK / 16; ++k)
+            tc_mma(tmem, smem_desc(a_s + 32 * k), smem_desc(b_s + 32 * k), idesc,
+                   (kb | k) != 0 ? 1u : 0u);
+          tc_commit(empty0 + 8 * s2);  // frees the stage once these MMAs are done
+        }
+        if (!ok) break;
+        tc_commit(tfull);  // accumulator ready
+        ++tiles;
+      }
+      if (!ok) {
+        atomicExch(P.err, LX_ERR_TIMEOUT);
+        *abort_flag = 1;
+        tc_commit(drain);  // arrives once every MMA issued so far has completed
+        mbar_wait(drain, 0, nullptr);
+      }
+    }
+    __syncwarp();
+  } else if (warp >= 4) {
+    // ------------------------------------------------------------ epilogue
+    const int ew = warp - 4;  // TMEM lanes 32 ew .. 32 ew + 31
+    uint32_t tiles = 0;
+    while (true) {
+      if (!mbar_wait(tfull, tiles & 1, abort_flag)) {
+        if (lane == 0) {
+          atomicExch(P.err, LX_ERR_TIMEOUT);
+          *abort_flag = 1;
+        }
+        break;
+      }
+      tc_fence_after();
+      const TcTile t = eslot[0];
+      if (t.BN < 0) break;
+      const int m = 32 * ew + lane;  // accumulator row = token within the tile
+      const bool row_ok = m < t.M && t.tok0 >= 0 && (long)t.tok0 + m < P.rows_cap &&
+                          (long)t.grp * t.Ng + t.row0 + t.BN <= P.ldo;
+      const size_t obase = (size_t)(t.tok0 + m) * P.ldo + (size_t)t.grp * t.Ng + t.row0;
+      for (int c0 = 0; c0 < t.BN; c0 += 16) {
+        float v[16];
+        tc_ld16(tmem + ((uint32_t)(32 * ew) << 16) + (uint32_t)c0, v);
+        if (row_ok) {
+          if (P.out_f32) {
+            float4* o = reinterpret_cast<float4*>(static_cast<float*>(P.out) + obase + c0);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) o[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+          } else {
+            uint4* o = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(P.out) + obase + c0);
+#pragma unroll
+            for (int q = 0; q < 2; ++q) {
+              uint32_t u[4];
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                __nv_bfloat162 b2 = __floats2bfloat162_rn(v[8 * q + 2 * e], v[8 * q + 2 * e + 1]);
+                u[e] = *reinterpret_cast<uint32_t*>(&b2);
+              }
+              o[q] = make_uint4(u[0], u[1], u[2], u[3]);
+            }
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(tempty);
+      ++tiles;
+    }
+  }
+  // all roles meet before the TMEM is released
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                 "r"(TC_TMEM_COLS)
+                 : "memory");
+  } else if (warp == 0 && lane == 0 && *abort_flag) {
+    // an aborted CTA may leave weight/activation copies in flight: wait (bounded)
+    // for the last stages the producer issued before shared memory goes away
+    const uint32_t first = prod_it > TC_STAGES ? prod_it - TC_STAGES : 0;
+    for (uint32_t j = first; j < prod_it; ++j)
+      mbar_wait(full0 + 8 * (j % TC_STAGES), (j / TC_STAGES) & 1, nullptr);
+  }
+}
+
+}  // namespace
+
+int tc_tile_tokens() { return TC_BM; }
+int tc_tile_cols() { return TC_BN; }
+
+static int tc_smem_bytes() {
+  return TC_STAGES * TC_STAGE_BYTES + 8 * (2 * TC_STAGES + 5) + 2 * TC_STAGES * (int)sizeof(TcTile) +
+         64 + 1024;
+}
+
+lx_status launch_tc(lx_layer* L, const TcLaunch& P, cudaStream_t s, const char* name) {
+  const int smem = tc_smem_bytes();
+  static bool done[64] = {};
+  LX_CUDA(smem_cap_once((const void*)k_tc_gemm, smem, L->device, done));
+  ProfScope ps(L, s, name);
+  k_tc_gemm<<<L->num_sms, TC_THREADS, smem, s>>>(P);
+  LX_CUDA(cudaGetLastError());
+  return LX_OK;
+}
+
+static TcLaunch tc_op(lx_layer* L, int op, const __nv_bfloat16* X, long ldx, const int* gather,
+                      const CUtensorMap* xmap, int xcol, void* out, long ldo, bool out_f32,
+                      int counter) {
+  Workspace& w = L->ws;
+  TcLaunch P;
+  P.shape = op_shape(L, op);
+  P.items = P.shape.on_anchors ? L->d_anchors : L->d_corrs;
+  P.n_items = P.shape.on_anchors ? L->n_anchor : L->n_corr;
+  P.tile_off = w.tile_off + (PLAN_TC + op) * (op_max_items(L) + 1);
+  P.node_off = w.key_off;
+  P.rank = L->d_rank;
+  P.wmaps = L->d_tmaps + (size_t)op * L->N;
+  P.X = X;
+  P.ldx = ldx;
+  P.gather = gather;
+  P.xmap = xmap;
+  P.xcol = xcol;
+  P.out = out;
+  P.ldo = ldo;
+  P.out_f32 = out_f32 ? 1 : 0;
+  P.ctr = w.sctr + N_STREAM_GROUPS + counter;
+  P.err = w.err;
+  P.rows_cap = w.rows_cap;
+  return P;
+}
+
+// The prefill forward: every (token, node) product on the tensor cores.
+lx_status launch_tc_experts(lx_layer* L, const void* x, int T, int k, void* y, cudaStream_t s) {
+  Workspace& w = L->ws;
+  const long H = L->H, I = L->I, rmax = L->max_rank;
+  const __nv_bfloat16* xb = static_cast<const __nv_bfloat16*>(x);
+  auto run = [&](const TcLaunch& P, const char* name) -> lx_status {
+    if (P.n_items == 0) return LX_OK;
+    return launch_tc(L, P, s, name);
+  };
+  LX_TRY(run(tc_op(L, OP_UP_ANCHOR, xb, H, w.node_tok, nullptr, 0, w.h, 2 * I, true, 0),
+             "tc_up_anchor"));
+  LX_TRY(run(tc_op(L, OP_UP_V, xb, H, w.node_tok, nullptr, 0, w.Pb, 2 * rmax, false, 1), "tc_up_V"));
+  LX_TRY(run(tc_op(L, OP_UP_U, nullptr, 0, nullptr, w.xmaps + 0, 0, w.h, 2 * I, true, 2),
+             "tc_up_U"));
+  LX_TRY(launch_swiglu(L, T, k, w.zb, true, s));
+  LX_TRY(run(tc_op(L, OP_DN_ANCHOR, nullptr, 0, nullptr, w.xmaps + 1, 0, w.ypart, H, true, 3),
+             "tc_dn_anchor"));
+  LX_TRY(run(tc_op(L, OP_DN_V, nullptr, 0, nullptr, w.xmaps + 1, 0, w.Qb, rmax, false, 4),
+             "tc_dn_V"));
+  LX_TRY(run(tc_op(L, OP_DN_U, nullptr, 0, nullptr, w.xmaps + 2, 0, w.ypart, H, true, 5),
+             "tc_dn_U"));
+  LX_TRY(launch_combine(L, T, k, y, s));
+  return LX_OK;
+}
+
+}  // namespace lx

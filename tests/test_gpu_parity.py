@@ -145,6 +145,29 @@ def test_stream_generic_boundary(T):
     check_forward(src, L, x, src.top_k)
 
 
+@pytest.mark.parametrize("name", STREAM)
+@pytest.mark.parametrize("T", [300, 1031])
+def test_tensor_core_path(name, T):
+    """Batches above the streaming limit run on the tcgen05 kernels."""
+    src, L = installed(name, SMALL[name])
+    x = synth.tokens(src, T, seed=500 + T)
+    ids, _ = check_route(src, L, x, src.top_k)
+    check_buckets(src, L, ids)
+    check_forward(src, L, x, src.top_k)
+
+
+def test_tensor_core_one_cluster_many_token_blocks():
+    """Every token on one cluster: each node bucket spans several 128-row blocks."""
+    src = synth.flat_layer(256, 128, [4] * 4, 64, 4, "bf16", seed=12, factor_std="visible")
+    src.router_bias = np.zeros(16, np.float32)
+    src.router_bias[src.meta["clusters"][1]] = 50.0
+    L = lx.Layer(src)
+    x = synth.tokens(src, 700, seed=4)
+    ids, _ = check_route(src, L, x, 4)
+    check_buckets(src, L, ids)
+    check_forward(src, L, x, 4)
+
+
 def test_tiny_fp32_config_full():
     """The tiny fp32 workload: 256 tokens, top-2, rank-8 SVD members."""
     src, L = installed("tiny_fp32", SMALL["tiny_fp32"])
