@@ -271,11 +271,193 @@ k_combine(const int* __restrict__ node_row, int k, int D, const float* __restric
   }
 }
 
+// ---------------------------------------------------------------------------
+// Warp-per-token SwiGLU aggregation and combine (k <= 8, k * D <= 32).
+//
+// A warp reads the token's k * D path rows (node_row), finds its distinct rows
+// with match/ballot/shuffle (no block barrier), and keeps them, in ascending
+// order, in a per-warp shared-memory block with, for each distinct row, the
+// bit mask of the top-k slots whose path passes through it.
+// ---------------------------------------------------------------------------
+constexpr int WT_WARPS = 8;
+constexpr int WT_SLOTS = 8;
+
+struct WarpRows {
+  int rows[32];       // entry j = slot j / D, level j % D (-1: none)
+  int drow[32];       // distinct rows, ascending
+  unsigned dmask[32]; // slots whose path holds distinct row d
+  float g[WT_SLOTS];
+  int nd;
+};
+
+__device__ __forceinline__ void warp_token_rows(const int* __restrict__ node_row_t, int kD, int D,
+                                                WarpRows& wr) {
+  const int lane = threadIdx.x & 31;
+  const int v = lane < kD ? node_row_t[lane] : -1;
+  const int key = v >= 0 ? v : INT_MAX;
+  const unsigned same = __match_any_sync(0xffffffffu, key);
+  const bool first = key != INT_MAX && lane == __ffs(same) - 1;
+  const unsigned fm = __ballot_sync(0xffffffffu, first);
+  // rank of this entry's row among the distinct rows (the loop is warp-uniform)
+  int rank = 0;
+  for (unsigned b = fm; b; b &= b - 1) {
+    const int q = __ffs(b) - 1;
+    rank += __shfl_sync(0xffffffffu, key, q) < key;
+  }
+  if (lane < kD) wr.rows[lane] = v;
+  if (first) wr.drow[rank] = key;
+  unsigned mask = 0;
+  for (int j = 0; j < kD; ++j) {
+    const int rj = __shfl_sync(0xffffffffu, key != INT_MAX ? rank : -1, j);
+    if (rj == lane) mask |= 1u << (j / D);
+  }
+  if (lane < 32) wr.dmask[lane] = mask;
+  if (lane == 0) wr.nd = __popc(fm);
+  __syncwarp();
+}
+
+template <typename TZ, int D>
+__global__ void __launch_bounds__(WT_WARPS * 32, 2)
+k_swiglu_warp(const float* __restrict__ topk_w, const int* __restrict__ node_row, int T, int k,
+              const float* __restrict__ h, int I, TZ* __restrict__ z, int cols_per_item) {
+  __shared__ WarpRows wrs[WT_WARPS];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  WarpRows& wr = wrs[warp];
+  const int kD = k * D;
+  const int per_tok = (I + cols_per_item - 1) / cols_per_item;
+  const long items = (long)T * per_tok;
+  for (long it = (long)blockIdx.x * WT_WARPS + warp; it < items; it += (long)gridDim.x * WT_WARPS) {
+    const int t = (int)(it / per_tok);
+    const int c_begin = (int)(it % per_tok) * cols_per_item;
+    const int c_end = min(I, c_begin + cols_per_item);
+    warp_token_rows(node_row + (size_t)t * kD, kD, D, wr);
+    if (lane < k) wr.g[lane] = topk_w[(size_t)t * k + lane];
+    __syncwarp();
+    const int nd = wr.nd;
+    for (int c = c_begin + 4 * lane; c < c_end; c += 128) {
+      float4 act[WT_SLOTS];
+#pragma unroll
+      for (int sl = 0; sl < WT_SLOTS; ++sl) {
+        act[sl] = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (sl < k) {
+          float4 pg = make_float4(0.f, 0.f, 0.f, 0.f), pu = pg;
+#pragma unroll
+          for (int l = 0; l < D; ++l) {  // path order: anchor first
+            const int r = wr.rows[sl * D + l];
+            if (r >= 0) {
+              const float4 a = __ldg(reinterpret_cast<const float4*>(h + (size_t)r * 2 * I + c));
+              const float4 b = __ldg(reinterpret_cast<const float4*>(h + (size_t)r * 2 * I + I + c));
+              pg.x += a.x; pg.y += a.y; pg.z += a.z; pg.w += a.w;
+              pu.x += b.x; pu.y += b.y; pu.z += b.z; pu.w += b.w;
+            }
+          }
+          const float g = wr.g[sl];
+          act[sl] = make_float4(g * silu_f(pg.x) * pu.x, g * silu_f(pg.y) * pu.y,
+                                g * silu_f(pg.z) * pu.z, g * silu_f(pg.w) * pu.w);
+        }
+      }
+      for (int d = 0; d < nd; ++d) {
+        const unsigned m = wr.dmask[d];
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int sl = 0; sl < WT_SLOTS; ++sl) {  // slots ascending
+          if ((m >> sl) & 1u) {
+            acc.x += act[sl].x; acc.y += act[sl].y; acc.z += act[sl].z; acc.w += act[sl].w;
+          }
+        }
+        store4<TZ>(z + (size_t)wr.drow[d] * I + c, acc);
+      }
+    }
+    __syncwarp();
+  }
+}
+
+// y[t] = sum of ypart over t's distinct rows in ascending row order
+template <typename TY>
+__global__ void __launch_bounds__(WT_WARPS * 32, 2)
+k_combine_warp(const int* __restrict__ node_row, int k, int D, const float* __restrict__ ypart,
+               int H, TY* __restrict__ y, int T, int cols_per_item) {
+  __shared__ WarpRows wrs[WT_WARPS];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  WarpRows& wr = wrs[warp];
+  const int kD = k * D;
+  const int per_tok = (H + cols_per_item - 1) / cols_per_item;
+  const long items = (long)T * per_tok;
+  for (long it = (long)blockIdx.x * WT_WARPS + warp; it < items; it += (long)gridDim.x * WT_WARPS) {
+    const int t = (int)(it / per_tok);
+    const int c_begin = (int)(it % per_tok) * cols_per_item;
+    const int c_end = min(H, c_begin + cols_per_item);
+    warp_token_rows(node_row + (size_t)t * kD, kD, D, wr);
+    const int nd = wr.nd;
+    for (int c = c_begin + 4 * lane; c < c_end; c += 128) {
+      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+      int q = 0;
+      for (; q + 8 <= nd; q += 8) {
+        float4 v[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+          v[u] = __ldg(reinterpret_cast<const float4*>(ypart + (size_t)wr.drow[q + u] * H + c));
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          acc.x += v[u].x; acc.y += v[u].y; acc.z += v[u].z; acc.w += v[u].w;
+        }
+      }
+      for (; q < nd; ++q) {
+        const float4 v = __ldg(reinterpret_cast<const float4*>(ypart + (size_t)wr.drow[q] * H + c));
+        acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
+      }
+      store4<TY>(y + (size_t)t * H + c, acc);
+    }
+    __syncwarp();
+  }
+}
+
 }  // namespace
+
+static bool warp_kernels_fit(const lx_layer* L, int k) {
+  return k <= WT_SLOTS && k * L->max_depth <= 32 && L->I % 4 == 0 && L->H % 4 == 0;
+}
+
+// Columns per warp work item: whole rows when the batch alone fills the GPU
+// (the distinct-row search then runs once per token), else 128-column blocks
+// so that a small batch still spreads over the SMs.
+static int warp_item_cols(const lx_layer* L, int T, int width) {
+  const long want = (long)L->num_sms * 4 * WT_WARPS;
+  const int blocks = (width + 127) / 128;
+  int per = blocks;
+  while (per > 1 && (long)T * ((blocks + per - 1) / per) < want) per = (per + 1) / 2;
+  return per * 128;
+}
+
+static int warp_grid(const lx_layer* L, int T, int width, int cols) {
+  const long items = (long)T * ((width + cols - 1) / cols);
+  return (int)std::min<long>((items + WT_WARPS - 1) / WT_WARPS, (long)L->num_sms * 4);
+}
+
+template <typename TZ>
+static void launch_swiglu_warp(lx_layer* L, int T, int k, TZ* z, cudaStream_t s) {
+  Workspace& w = L->ws;
+  const int cols = warp_item_cols(L, T, L->I);
+  const int grid = warp_grid(L, T, L->I, cols);
+  switch (L->max_depth) {
+    case 1: k_swiglu_warp<TZ, 1><<<grid, WT_WARPS * 32, 0, s>>>(w.topk_w, w.node_row, T, k, w.h, L->I, z, cols); break;
+    case 2: k_swiglu_warp<TZ, 2><<<grid, WT_WARPS * 32, 0, s>>>(w.topk_w, w.node_row, T, k, w.h, L->I, z, cols); break;
+    case 3: k_swiglu_warp<TZ, 3><<<grid, WT_WARPS * 32, 0, s>>>(w.topk_w, w.node_row, T, k, w.h, L->I, z, cols); break;
+    default: k_swiglu_warp<TZ, 4><<<grid, WT_WARPS * 32, 0, s>>>(w.topk_w, w.node_row, T, k, w.h, L->I, z, cols); break;
+  }
+}
 
 lx_status launch_swiglu(lx_layer* L, int T, int k, void* z, bool z_bf16, cudaStream_t s) {
   Workspace& w = L->ws;
   ProfScope ps(L, s, z_bf16 ? "swiglu" : "generic_swiglu");
+  if (warp_kernels_fit(L, k)) {
+    if (z_bf16)
+      launch_swiglu_warp(L, T, k, static_cast<__nv_bfloat16*>(z), s);
+    else
+      launch_swiglu_warp(L, T, k, static_cast<float*>(z), s);
+    LX_CUDA(cudaGetLastError());
+    return LX_OK;
+  }
   const int grid = std::min(T, L->num_sms * 8);
   const size_t smem = sizeof(float4) * SW_T * k * L->max_depth;
   static bool done_b[64] = {}, done_f[64] = {};
@@ -295,6 +477,18 @@ lx_status launch_swiglu(lx_layer* L, int T, int k, void* z, bool z_bf16, cudaStr
 lx_status launch_combine(lx_layer* L, int T, int k, void* y, cudaStream_t s) {
   Workspace& w = L->ws;
   ProfScope ps(L, s, "combine");
+  if (warp_kernels_fit(L, k)) {
+    const int cols = warp_item_cols(L, T, L->H);
+    const int g2 = warp_grid(L, T, L->H, cols);
+    if (L->dtype == LX_BF16)
+      k_combine_warp<__nv_bfloat16><<<g2, WT_WARPS * 32, 0, s>>>(
+          w.node_row, k, L->max_depth, w.ypart, L->H, (__nv_bfloat16*)y, T, cols);
+    else
+      k_combine_warp<float><<<g2, WT_WARPS * 32, 0, s>>>(w.node_row, k, L->max_depth, w.ypart,
+                                                          L->H, (float*)y, T, cols);
+    LX_CUDA(cudaGetLastError());
+    return LX_OK;
+  }
   const int grid = std::min(T, L->num_sms * 8);
   if (L->dtype == LX_BF16)
     k_combine<__nv_bfloat16><<<grid, 256, 0, s>>>(w.node_row, k, L->max_depth, w.ypart, L->H,

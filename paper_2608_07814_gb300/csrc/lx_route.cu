@@ -8,11 +8,20 @@
 // multiply-adds, and the 32 lane partials are added pairwise at offsets
 // 16, 8, 4, 2, 1; the bias (if any) is added last.
 //
-// One CTA computes the logits of 8 tokens for a slice of the experts (all
-// experts when T is large, one per warp when T is small, so that a decode
-// batch still spreads the 0.5 MB router matrix over many SMs).  Each warp owns one
+// Small batches (k_router_logits): one CTA computes the logits of 8 tokens
+// for a slice of the experts (one expert per warp, so that a decode batch
+// still spreads the 0.5 MB router matrix over many SMs).  Each warp owns one
 // expert at a time and issues its weight loads in groups of 8 independent
 // 16-byte loads before using them.
+//
+// Large bf16 batches (k_router_tiled): persistent CTAs walk tiles of 8
+// tokens.  A thread holds the lane partials of 8 tokens x 8 experts for its
+// lane's chunks (64 accumulators), so every widened weight value serves 8
+// tokens and every widened token value 8 experts.  The 32 lane partials are
+// then combined by a transpose-reduce whose pairs are those of the canonical
+// order (lane l with lane l ^ 16, then ^ 8, ^ 4, ^ 2, ^ 1; IEEE addition is
+// commutative, so each sum is bit-identical), leaving lane l with the logits
+// of entries 2l and 2l + 1 of the 8 x 8 block.
 #include <algorithm>
 
 #include "lx_internal.cuh"
@@ -137,15 +146,163 @@ k_router_logits(const T* __restrict__ x, const T* __restrict__ W, const float* _
   if (threadIdx.x == 0) tile_cnt[blockIdx.x] = 0;
 }
 
+constexpr int RTT_TOK = 8;         // tokens per tile (one token per warp in the top-k)
+constexpr int RTT_THREADS = 256;   // 8 warps, each on 8-expert groups
+
+__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+
+// x tile rows [t0, t0 + nt) into shared memory (16-byte cp.async), zeros after
+__device__ __forceinline__ void rtt_load_tile(const __nv_bfloat16* x, int t0, int nt, int H,
+                                              __nv_bfloat16* xs) {
+  const int vec_per_tok = H / 8;
+  for (int i = threadIdx.x; i < RTT_TOK * vec_per_tok; i += blockDim.x) {
+    const int r = i / vec_per_tok;
+    uint4* d = reinterpret_cast<uint4*>(xs) + i;
+    if (r < nt) {
+      const uint32_t da = static_cast<uint32_t>(__cvta_generic_to_shared(d));
+      asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(da),
+                   "l"(reinterpret_cast<const uint4*>(x + (size_t)t0 * H) + i)
+                   : "memory");
+    } else {
+      *d = make_uint4(0, 0, 0, 0);
+    }
+  }
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+
+__global__ void __launch_bounds__(RTT_THREADS, 1)
+k_router_tiled(const __nv_bfloat16* __restrict__ x, const __nv_bfloat16* __restrict__ W,
+               const float* __restrict__ bias, int Ttok, int E, int H,
+               float* __restrict__ logits, int k, int* __restrict__ topk_id,
+               float* __restrict__ topk_w) {
+  extern __shared__ __align__(16) unsigned char smem[];
+  __nv_bfloat16* xs0 = reinterpret_cast<__nv_bfloat16*>(smem);
+  __nv_bfloat16* xs1 = xs0 + (size_t)RTT_TOK * H;
+  float* ls = reinterpret_cast<float*>(xs1 + (size_t)RTT_TOK * H);  // [RTT_TOK][E]
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nchunk = H / 8, nj = (nchunk + 31) / 32;
+  const int ngroups = (E + 7) / 8;
+  const int ntiles = (Ttok + RTT_TOK - 1) / RTT_TOK;
+  int buf = 0;
+  if ((int)blockIdx.x < ntiles) {
+    const int t0 = blockIdx.x * RTT_TOK;
+    rtt_load_tile(x, t0, min(RTT_TOK, Ttok - t0), H, xs0);
+  }
+  for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x, buf ^= 1) {
+    const int t0 = tile * RTT_TOK, nt = min(RTT_TOK, Ttok - t0);
+    const __nv_bfloat16* xs = buf ? xs1 : xs0;
+    asm volatile("cp.async.wait_group 0;" ::: "memory");
+    __syncthreads();
+    // the next tile streams in while this one is computed
+    const int nxt = tile + gridDim.x;
+    if (nxt < ntiles) {
+      const int n0 = nxt * RTT_TOK;
+      rtt_load_tile(x, n0, min(RTT_TOK, Ttok - n0), H, buf ? xs0 : xs1);
+    }
+    for (int g = warp; g < ngroups; g += RTT_THREADS / 32) {
+      float acc[64];  // [token tt][expert ee] partials of this lane
+#pragma unroll
+      for (int a = 0; a < 64; ++a) acc[a] = 0.f;
+      for (int j = 0; j < nj; ++j) {
+        const int q = lane + 32 * j;  // this lane's chunk
+        if (q >= nchunk) break;
+        uint4 wr[8], xr[8];
+#pragma unroll
+        for (int ee = 0; ee < 8; ++ee) {
+          const int e = 8 * g + ee;
+          const uint4* wrow = reinterpret_cast<const uint4*>(W + (size_t)e * H);
+          wr[ee] = e < E ? __ldg(wrow + q) : make_uint4(0, 0, 0, 0);
+          // the next chunk of this expert row heads for L1 while this one is used
+          if (e < E && q + 32 < nchunk)
+            asm volatile("prefetch.global.L1 [%0];" ::"l"(wrow + q + 32));
+        }
+#pragma unroll
+        for (int tt = 0; tt < 8; ++tt)
+          xr[tt] = reinterpret_cast<const uint4*>(xs + (size_t)tt * H)[q];
+#pragma unroll
+        for (int wd = 0; wd < 4; ++wd) {
+#pragma unroll
+          for (int hf = 0; hf < 2; ++hf) {  // element 2 wd + hf of the chunk, ascending
+            float xv[8], wv[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+              const uint32_t xw = wd == 0 ? xr[i].x : wd == 1 ? xr[i].y : wd == 2 ? xr[i].z : xr[i].w;
+              const uint32_t ww = wd == 0 ? wr[i].x : wd == 1 ? wr[i].y : wd == 2 ? wr[i].z : wr[i].w;
+              xv[i] = hf ? bf16_hi(xw) : bf16_lo(xw);
+              wv[i] = hf ? bf16_hi(ww) : bf16_lo(ww);
+            }
+#pragma unroll
+            for (int tt = 0; tt < 8; ++tt)
+#pragma unroll
+              for (int ee = 0; ee < 8; ++ee)
+                acc[tt * 8 + ee] = __fmaf_rn(xv[tt], wv[ee], acc[tt * 8 + ee]);
+          }
+        }
+      }
+      // transpose-reduce: at offset o, the lane with bit o clear keeps the lower
+      // half of its live entries and adds its partner's copy of them
+#pragma unroll
+      for (int o = 16, n = 64; o >= 1; o >>= 1, n >>= 1) {
+        const bool upper = (lane & o) != 0;
+#pragma unroll
+        for (int a = 0; a < n / 2; ++a) {
+          const float send = upper ? acc[a] : acc[a + n / 2];
+          const float keep = upper ? acc[a + n / 2] : acc[a];
+          acc[a] = __fadd_rn(keep, __shfl_xor_sync(0xffffffffu, send, o));
+        }
+      }
+      // lane l now holds entries 2l, 2l + 1: token l / 4, experts 2 (l % 4) + {0, 1}
+      const int tt = lane >> 2;
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const int e = 8 * g + 2 * (lane & 3) + h;
+        if (e < E) {
+          const float v = bias ? __fadd_rn(acc[h], bias[e]) : acc[h];
+          ls[tt * E + e] = v;
+          if (tt < nt) logits[(size_t)(t0 + tt) * E + e] = v;
+        }
+      }
+    }
+    __syncthreads();
+    if (warp < nt) {
+      int id;
+      float w;
+      warp_topk(ls + warp * E, E, k, id, w);
+      if (lane < k) {
+        topk_id[(size_t)(t0 + warp) * k + lane] = id;
+        topk_w[(size_t)(t0 + warp) * k + lane] = w;
+      }
+    }
+    // the logits block and the x buffer are reused two tiles on
+  }
+  asm volatile("cp.async.wait_group 0;" ::: "memory");
+}
+
 }  // namespace
 
 lx_status launch_router(lx_layer* L, const void* x, int T, int k, float* logits, int* topk_id,
                         float* topk_w, cudaStream_t s) {
   if (reinterpret_cast<uintptr_t>(x) % 16)
     return fail(LX_ERR_ARG, "x must be 16-byte aligned");
+  const int tiles = (T + RT_TOK - 1) / RT_TOK;
+  if (L->dtype == LX_BF16 && tiles >= L->num_sms && L->H % 8 == 0) {
+    // large batch: persistent register-tiled kernel
+    const size_t smem2 = 2 * (size_t)RTT_TOK * L->H * 2 + (size_t)RTT_TOK * L->E * 4;
+    if (smem2 <= 200 * 1024) {
+      static bool done_t[64] = {};
+      LX_CUDA(smem_cap_once((const void*)k_router_tiled, 200 * 1024, L->device, done_t));
+      ProfScope ps(L, s, "router");
+      const int grid = std::min(tiles, L->num_sms);
+      k_router_tiled<<<grid, RTT_THREADS, smem2, s>>>(
+          (const __nv_bfloat16*)x, (const __nv_bfloat16*)L->router_w, L->router_bias, T, L->E,
+          L->H, logits, k, topk_id, topk_w);
+      LX_CUDA(cudaGetLastError());
+      return LX_OK;
+    }
+  }
   const size_t smem = std::max((size_t)RT_TOK * L->H * L->esz, (size_t)RT_TOK * L->E * 4);
   if (smem > 200 * 1024) return fail(LX_ERR_SHAPE, "router token tile exceeds shared memory");
-  const int tiles = (T + RT_TOK - 1) / RT_TOK;
   // few token tiles: slice the experts so the router matrix spreads over the SMs
   const int per_cta = tiles >= L->num_sms ? L->E : RT_THREADS / 32;
   const dim3 grid(tiles, (L->E + per_cta - 1) / per_cta);

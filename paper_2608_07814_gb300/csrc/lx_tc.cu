@@ -10,15 +10,18 @@
 //               loads the weight boxes (64 rows x 64 K, 128B swizzle, tiled
 //               layout) with TMA, and the 128 token rows either with one TMA
 //               box (rows already contiguous in node-row order: P, z, Q) or
-//               with 16-byte cp.async gathers (x rows by token id); gathered
-//               rows are made visible to the tensor core's async proxy with
-//               fence.proxy.async before the stage is marked full;
-//   warp 1      allocates 256 TMEM columns; lane 0 issues tcgen05.mma
-//               (kind::f16, bf16 x bf16 -> fp32, M=128, N=BN, K=16 per
-//               instruction) and commits stage releases and accumulator-ready
-//               signals with tcgen05.commit;
-//   warps 4..7  epilogue: tcgen05.ld (32 lanes x 16 columns per load) from the
-//               accumulator and row-wise stores to global memory.
+//               with 16-byte cp.async gathers (x rows by token id, eight lanes
+//               per 128-byte row so one instruction touches four rows);
+//               gathered rows are made visible to the tensor core's async
+//               proxy with fence.proxy.async before the stage is marked full;
+//   warp 1      allocates 512 TMEM columns (two 256-column accumulators, so
+//               the epilogue of one tile overlaps the MMAs of the next); lane 0
+//               issues tcgen05.mma (kind::f16, bf16 x bf16 -> fp32, M=128,
+//               N=BN, K=16 per instruction) and commits stage releases and
+//               accumulator-ready signals with tcgen05.commit;
+//   warps 4..7  epilogue: tcgen05.ld (32 lanes x 32 columns per load), a
+//               transpose through a per-warp shared-memory block, and stores
+//               of whole 128-byte row segments.
 // Every wait is bounded; a wait that gives up records LX_ERR_TIMEOUT, makes the
 // other roles stop, drains the CTA's copies and MMAs in flight and frees TMEM.
 #include <cuda.h>
@@ -39,9 +42,13 @@ constexpr int TC_A_BYTES = TC_BM * TC_BK * 2;   // 16 KiB
 constexpr int TC_B_BYTES = TC_BN * TC_BK * 2;   // 32 KiB
 constexpr int TC_STAGE_BYTES = TC_A_BYTES + TC_B_BYTES;
 constexpr int TC_THREADS = 256;
-constexpr int TC_TMEM_COLS = 256;
+constexpr int TC_ACC_COLS = 256;                 // one accumulator
+constexpr int TC_TMEM_COLS = 2 * TC_ACC_COLS;    // double-buffered
+constexpr int TC_EPI_LD = 36;                    // staging row stride (floats)
+constexpr int TC_EPI_BYTES = 32 * TC_EPI_LD * 4; // per epilogue warp
 constexpr unsigned long long TC_TIMEOUT_CYCLES = 4000000000ull;  // ~2 s
 static_assert(TC_STAGE_BYTES % 1024 == 0, "stages keep the 1024-byte swizzle alignment");
+static_assert(TC_STAGES <= 8 && TC_STAGES >= 2, "in-flight stage ring packs 4-bit stage ids");
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -154,18 +161,22 @@ __device__ __forceinline__ void tc_fence_after() {
 __device__ __forceinline__ void tc_fence_before() {
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
 }
-__device__ __forceinline__ void tc_ld16(uint32_t taddr, float (&v)[16]) {
-  uint32_t r[16];
+// 32 TMEM lanes x 32 consecutive columns: register i of lane l = column i of lane l
+__device__ __forceinline__ void tc_ld32(uint32_t taddr, float (&v)[32]) {
+  uint32_t r[32];
   asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
-      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
       : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
         "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
-        "=r"(r[14]), "=r"(r[15])
+        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
+        "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
+        "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
       : "r"(taddr));
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 #pragma unroll
-  for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
 struct TcTile {
@@ -200,14 +211,15 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + TC_STAGES * TC_STAGE_BYTES);
-  // full[S], empty[S], tmem_full, tmem_empty, drain
+  float* epi = reinterpret_cast<float*>(smem + TC_STAGES * TC_STAGE_BYTES);  // [4][32][EPI_LD]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + TC_STAGES * TC_STAGE_BYTES + 4 * TC_EPI_BYTES);
+  // full[S], empty[S], tmem_full[2], tmem_empty[2], drain
   const uint32_t full0 = smem_u32(bars), empty0 = full0 + 8 * TC_STAGES;
-  const uint32_t tfull = empty0 + 8 * TC_STAGES, tempty = tfull + 8, drain = tempty + 8;
-  volatile int* abort_flag = reinterpret_cast<volatile int*>(bars + 2 * TC_STAGES + 3);
-  uint32_t* tmem_base_s = reinterpret_cast<uint32_t*>(bars + 2 * TC_STAGES + 4);
-  TcTile* slot = reinterpret_cast<TcTile*>(bars + 2 * TC_STAGES + 5);  // [TC_STAGES]
-  TcTile* eslot = slot + TC_STAGES;                                     // epilogue hand-off
+  const uint32_t tfull0 = empty0 + 8 * TC_STAGES, tempty0 = tfull0 + 16, drain = tempty0 + 16;
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(bars + 2 * TC_STAGES + 5);
+  uint32_t* tmem_base_s = reinterpret_cast<uint32_t*>(bars + 2 * TC_STAGES + 6);
+  TcTile* slot = reinterpret_cast<TcTile*>(bars + 2 * TC_STAGES + 7);     // [TC_STAGES]
+  TcTile* eslot = slot + TC_STAGES;                                         // [2] epilogue hand-off
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t smem_base = smem_u32(smem);
   uint32_t prod_it = 0;  // stages the producer issued
@@ -217,8 +229,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
       mbar_init(full0 + 8 * s, 1 + 32);  // producer arrival + one per producer lane
       mbar_init(empty0 + 8 * s, 1);      // tcgen05.commit
     }
-    mbar_init(tfull, 2);   // MMA thread's arrival (tile info written) + tcgen05.commit
-    mbar_init(tempty, 4);  // one arrival per epilogue warp
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(tfull0 + 8 * b, 2);   // MMA thread's arrival (tile info written) + tcgen05.commit
+      mbar_init(tempty0 + 8 * b, 4);  // one arrival per epilogue warp
+    }
     mbar_init(drain, 1);
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -244,17 +258,21 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
     if (cur < total) tc_decode(P, cur, t);
     uint32_t it = 0;
     bool ok = true;
-    bool pending = false;  // a gathered stage waits for its fence + arrivals
-    uint32_t pend_s = 0;
+    const int r8 = lane >> 3, u = lane & 7;  // gather: row within a group of 4, 16-byte chunk
+    // Gathered stages still in flight (cp.async groups not yet waited for), oldest
+    // first, four bits per stage index: up to TC_STAGES - 1 stages of token rows
+    // stay in flight before the oldest is published to the MMA issuer.
+    uint32_t pq = 0;
+    int np = 0;
     while (cur < total && ok) {
       int nxt = lane == 0 ? atomicAdd(P.ctr, 1) : 0;
-      // token row sources of this tile (lane handles rows lane + 32 h)
-      const __nv_bfloat16* src[4];
+      int trow[TC_BM / 4];  // token of row 4 i + r8 of this tile, or -1
+      if (P.gather) {
 #pragma unroll
-      for (int h = 0; h < 4; ++h) {
-        const int m = lane + 32 * h;
-        src[h] = nullptr;
-        if (P.gather && m < t.M) src[h] = P.X + (long)P.gather[t.tok0 + m] * P.ldx;
+        for (int i = 0; i < TC_BM / 4; ++i) {
+          const int m = 4 * i + r8;
+          trow[i] = m < t.M ? __ldg(P.gather + t.tok0 + m) : -1;
+        }
       }
       const int nkb = (t.K + TC_BK - 1) / TC_BK;
       const int rt0 = (t.grp * t.Ng + t.row0) / 64;  // first 64-row weight tile
@@ -283,25 +301,24 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
                         full0 + 8 * s);
         }
         if (P.gather) {
-          // 128 rows x 128 bytes in the 128-byte swizzle: chunk u of row m goes
-          // to u ^ (m & 7)
+          // row m (128 bytes of K) in the 128-byte swizzle: chunk u goes to u ^ (m & 7);
+          // eight lanes cover one row, one instruction four rows
+          const __nv_bfloat16* xk = P.X + kb * TC_BK + 8 * u;
 #pragma unroll
-          for (int h = 0; h < 4; ++h) {
-            const int m = lane + 32 * h;
-            if (src[h]) {
-#pragma unroll
-              for (int u = 0; u < 8; ++u)
-                cp_async16(a_s + m * 128 + ((u ^ (m & 7)) << 4), src[h] + kb * TC_BK + 8 * u);
-            }
+          for (int i = 0; i < TC_BM / 4; ++i) {
+            const int m = 4 * i + r8;
+            if (trow[i] >= 0)
+              cp_async16(a_s + m * 128 + ((u ^ (m & 7)) << 4), xk + (long)trow[i] * P.ldx);
           }
           cp_async_commit();
-          if (pending) {  // the previous gathered stage has landed: publish it
-            cp_async_wait<1>();
+          pq |= s << (4 * np);
+          if (++np == TC_STAGES - 1) {  // publish the oldest gathered stage
+            cp_async_wait<TC_STAGES - 2>();
             fence_proxy_async();
-            mbar_arrive(full0 + 8 * pend_s);
+            mbar_arrive(full0 + 8 * (pq & 15u));
+            pq >>= 4;
+            --np;
           }
-          pending = true;
-          pend_s = s;
         } else {
           mbar_arrive(full0 + 8 * s);
         }
@@ -310,10 +327,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
       cur = nxt;
       if (cur < total) tc_decode(P, cur, t);
     }
-    if (pending) {
+    if (np > 0) {  // publish what is still in flight
       cp_async_wait<0>();
       fence_proxy_async();
-      mbar_arrive(full0 + 8 * pend_s);
+      for (; np > 0; --np, pq >>= 4) mbar_arrive(full0 + 8 * (pq & 15u));
     }
     if (ok) {
       // sentinel stage
@@ -348,16 +365,18 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
         const uint32_t s = it % TC_STAGES;
         if (!mbar_wait(full0 + 8 * s, (it / TC_STAGES) & 1, abort_flag)) { ok = false; break; }
         const TcTile t = slot[s];
-        // the accumulator must have been drained by the epilogue
-        if (!mbar_wait(tempty, (tiles & 1) ^ 1, abort_flag)) { ok = false; break; }
-        eslot[0] = t;       // tile info for the epilogue, released by this arrival
-        mbar_arrive(tfull);
-        if (t.BN < 0) {     // sentinel: the second arrival completes the phase
-          mbar_arrive(tfull);
+        const uint32_t b = tiles & 1;
+        // this accumulator must have been drained by the epilogue (two tiles ago)
+        if (!mbar_wait(tempty0 + 8 * b, ((tiles >> 1) & 1) ^ 1, abort_flag)) { ok = false; break; }
+        eslot[b] = t;  // tile info for the epilogue, released by this arrival
+        mbar_arrive(tfull0 + 8 * b);
+        if (t.BN < 0) {  // sentinel: the second arrival completes the phase
+          mbar_arrive(tfull0 + 8 * b);
           ++it;
           break;
         }
         tc_fence_after();
+        const uint32_t d = tmem + b * TC_ACC_COLS;
         const uint32_t idesc = instr_desc(TC_BM, t.BN);
         const int nkb = (t.K + TC_BK - 1) / TC_BK;
         for (int kb = 0; kb < nkb; ++kb, ++it) {
@@ -367,12 +386,12 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
           const uint32_t a_s = smem_base + s2 * TC_STAGE_BYTES, b_s = a_s + TC_A_BYTES;
 #pragma unroll
           for (int k = 0; k < TC_BK / 16; ++k)
-            tc_mma(tmem, smem_desc(a_s + 32 * k), smem_desc(b_s + 32 * k), idesc,
+            tc_mma(d, smem_desc(a_s + 32 * k), smem_desc(b_s + 32 * k), idesc,
                    (kb | k) != 0 ? 1u : 0u);
           tc_commit(empty0 + 8 * s2);  // frees the stage once these MMAs are done
         }
         if (!ok) break;
-        tc_commit(tfull);  // accumulator ready
+        tc_commit(tfull0 + 8 * b);  // accumulator ready
         ++tiles;
       }
       if (!ok) {
@@ -386,9 +405,11 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
   } else if (warp >= 4) {
     // ------------------------------------------------------------ epilogue
     const int ew = warp - 4;  // TMEM lanes 32 ew .. 32 ew + 31
+    float* stg = epi + ew * 32 * TC_EPI_LD;
     uint32_t tiles = 0;
     while (true) {
-      if (!mbar_wait(tfull, tiles & 1, abort_flag)) {
+      const uint32_t b = tiles & 1;
+      if (!mbar_wait(tfull0 + 8 * b, (tiles >> 1) & 1, abort_flag)) {
         if (lane == 0) {
           atomicExch(P.err, LX_ERR_TIMEOUT);
           *abort_flag = 1;
@@ -396,38 +417,46 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
         break;
       }
       tc_fence_after();
-      const TcTile t = eslot[0];
+      const TcTile t = eslot[b];
       if (t.BN < 0) break;
-      const int m = 32 * ew + lane;  // accumulator row = token within the tile
-      const bool row_ok = m < t.M && t.tok0 >= 0 && (long)t.tok0 + m < P.rows_cap &&
-                          (long)t.grp * t.Ng + t.row0 + t.BN <= P.ldo;
-      const size_t obase = (size_t)(t.tok0 + m) * P.ldo + (size_t)t.grp * t.Ng + t.row0;
-      for (int c0 = 0; c0 < t.BN; c0 += 16) {
-        float v[16];
-        tc_ld16(tmem + ((uint32_t)(32 * ew) << 16) + (uint32_t)c0, v);
-        if (row_ok) {
-          if (P.out_f32) {
-            float4* o = reinterpret_cast<float4*>(static_cast<float*>(P.out) + obase + c0);
+      const bool tile_ok = t.tok0 >= 0 && (long)t.grp * t.Ng + t.row0 + t.BN <= P.ldo;
+      const long col0 = (long)t.grp * t.Ng + t.row0;
+      for (int c0 = 0; c0 < t.BN; c0 += 32) {
+        float v[32];
+        tc_ld32(tmem + b * TC_ACC_COLS + ((uint32_t)(32 * ew) << 16) + (uint32_t)c0, v);
+        // lane = accumulator row: stage the 32 x 32 block row-major
+        float4* srow = reinterpret_cast<float4*>(stg + lane * TC_EPI_LD);
 #pragma unroll
-            for (int q = 0; q < 4; ++q) o[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-          } else {
-            uint4* o = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(P.out) + obase + c0);
+        for (int q = 0; q < 8; ++q)
+          srow[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+        __syncwarp();
+        // eight lanes per row, four rows per pass: whole 128-byte (f32) segments
+        const int cq = lane & 7;
 #pragma unroll
-            for (int q = 0; q < 2; ++q) {
-              uint32_t u[4];
-#pragma unroll
-              for (int e = 0; e < 4; ++e) {
-                __nv_bfloat162 b2 = __floats2bfloat162_rn(v[8 * q + 2 * e], v[8 * q + 2 * e + 1]);
-                u[e] = *reinterpret_cast<uint32_t*>(&b2);
-              }
-              o[q] = make_uint4(u[0], u[1], u[2], u[3]);
+        for (int j = 0; j < 8; ++j) {
+          const int rr = 4 * j + (lane >> 3);
+          const int m = 32 * ew + rr;
+          const long grow = (long)t.tok0 + m;
+          if (tile_ok && m < t.M && grow < P.rows_cap) {
+            const float4 f = *reinterpret_cast<const float4*>(stg + rr * TC_EPI_LD + 4 * cq);
+            const size_t o = (size_t)grow * P.ldo + col0 + c0 + 4 * cq;
+            if (P.out_f32) {
+              *reinterpret_cast<float4*>(static_cast<float*>(P.out) + o) = f;
+            } else {
+              __nv_bfloat162 lo = __floats2bfloat162_rn(f.x, f.y);
+              __nv_bfloat162 hi = __floats2bfloat162_rn(f.z, f.w);
+              uint2 pk;
+              pk.x = *reinterpret_cast<uint32_t*>(&lo);
+              pk.y = *reinterpret_cast<uint32_t*>(&hi);
+              *reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(P.out) + o) = pk;
             }
           }
         }
+        __syncwarp();
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(tempty);
+      if (lane == 0) mbar_arrive(tempty0 + 8 * b);
       ++tiles;
     }
   }
@@ -454,8 +483,8 @@ int tc_tile_tokens() { return TC_BM; }
 int tc_tile_cols() { return TC_BN; }
 
 static int tc_smem_bytes() {
-  return TC_STAGES * TC_STAGE_BYTES + 8 * (2 * TC_STAGES + 5) + 2 * TC_STAGES * (int)sizeof(TcTile) +
-         64 + 1024;
+  return TC_STAGES * TC_STAGE_BYTES + 4 * TC_EPI_BYTES + 8 * (2 * TC_STAGES + 7) +
+         3 * TC_STAGES * (int)sizeof(TcTile) + 1024;
 }
 
 lx_status launch_tc(lx_layer* L, const TcLaunch& P, cudaStream_t s, const char* name) {

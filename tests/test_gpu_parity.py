@@ -156,6 +156,20 @@ def test_tensor_core_path(name, T):
     check_forward(src, L, x, src.top_k)
 
 
+BF16_SMALL = [n for n in sorted(SMALL) if "fp32" not in n]
+
+
+@pytest.mark.parametrize("name", BF16_SMALL)
+@pytest.mark.parametrize("T", [1217, 2003])
+def test_router_large_batch(name, T):
+    """Batches of >= 152 8-token tiles take the register-tiled router: logits,
+    top-k and gates stay bit-exact (ragged expert groups and chunk counts)."""
+    src, L = installed(name, SMALL[name])
+    x = synth.tokens(src, T, seed=700 + T)
+    ids, _ = check_route(src, L, x, src.top_k)
+    check_buckets(src, L, ids)
+
+
 def test_tensor_core_one_cluster_many_token_blocks():
     """Every token on one cluster: each node bucket spans several 128-row blocks."""
     src = synth.flat_layer(256, 128, [4] * 4, 64, 4, "bf16", seed=12, factor_std="visible")
