@@ -110,6 +110,9 @@ static bool encode_rows_map(CUtensorMap* m, void* base, long rows, long ld) {
 // ---------------------------------------------------------------------------
 // workspace
 // ---------------------------------------------------------------------------
+// Batches up to this size take the weight-streaming kernels.
+constexpr int kStreamMaxT = 256;
+
 static lx_status ensure_workspace(lx_layer* L, int T, int k, cudaStream_t s) {
   Workspace& w = L->ws;
   if (T <= w.cap_T && k <= w.cap_k) return LX_OK;
@@ -119,6 +122,11 @@ static lx_status ensure_workspace(lx_layer* L, int T, int k, cudaStream_t s) {
   const long keys = (long)L->N + L->E;
   const long Rmax = std::max<long>(1, (long)cT * std::min<long>(L->N, (long)ck * D));
   const long rmax = std::max(1, L->max_rank);
+  // split-K partial rows of the streaming path (batches up to kStreamMaxT)
+  const long Rsplit =
+      L->stream_ok ? std::max<long>(1, (long)std::min(cT, kStreamMaxT) *
+                                           std::min<long>(L->N, (long)ck * D))
+                   : 0;
   struct Item { void** p; size_t bytes; };
   std::vector<Item> items = {
       {(void**)&w.logits, sizeof(float) * cT * L->E},
@@ -146,6 +154,8 @@ static lx_status ensure_workspace(lx_layer* L, int T, int k, cudaStream_t s) {
       {(void**)&w.act_n, sizeof(int) * 2},
       {(void**)&w.sctr, sizeof(int) * N_TILE_COUNTERS},
       {(void**)&w.xmaps, sizeof(CUtensorMap) * 3},
+      {(void**)&w.hsplit, sizeof(float) * (LX_STREAM_MAX_SPLIT - 1) * Rsplit * 2 * L->I},
+      {(void**)&w.ysplit, sizeof(float) * (LX_STREAM_MAX_SPLIT - 1) * Rsplit * L->H},
       {(void**)&w.err, 256},
   };
   size_t total = 0;
@@ -175,6 +185,8 @@ static lx_status ensure_workspace(lx_layer* L, int T, int k, cudaStream_t s) {
   w.cap_T = cT;
   w.cap_k = ck;
   w.rows_cap = Rmax;
+  w.split_rows = Rsplit;
+  if (Rsplit == 0) w.hsplit = w.ysplit = nullptr;
   if (L->stream_ok) {
     CUtensorMap maps[3];
     std::memset(maps, 0, sizeof(maps));
@@ -215,7 +227,6 @@ static lx_status route_and_bucket(lx_layer* L, const void* x, int T, int k, int*
 
 // Largest batch the weight-streaming (decode) kernels take; beyond it every
 // weight would be re-streamed per 64-token block.
-constexpr int kStreamMaxT = 256;
 
 static bool use_stream(const lx_layer* L, int T) {
   return L->path_mode == LX_PATH_AUTO && L->stream_ok && T <= kStreamMaxT;

@@ -288,6 +288,7 @@ struct WarpRows {
   unsigned dmask[32]; // slots whose path holds distinct row d
   float g[WT_SLOTS];
   int nd;
+  unsigned anchor_rows;  // bit d: distinct row d belongs to an anchor
 };
 
 __device__ __forceinline__ void warp_token_rows(const int* __restrict__ node_row_t, int kD, int D,
@@ -306,20 +307,30 @@ __device__ __forceinline__ void warp_token_rows(const int* __restrict__ node_row
   }
   if (lane < kD) wr.rows[lane] = v;
   if (first) wr.drow[rank] = key;
-  unsigned mask = 0;
+  // entry j holds its path's anchor if it is the path's last valid level
+  // (paths are stored from the expert's own node up to the anchor)
+  const int v_next = __shfl_down_sync(0xffffffffu, v, 1);
+  const bool anchor_entry = v >= 0 && (lane % D == D - 1 || lane + 1 >= kD || v_next < 0);
+  const unsigned am = __ballot_sync(0xffffffffu, anchor_entry);
+  unsigned mask = 0, anc = 0;
   for (int j = 0; j < kD; ++j) {
     const int rj = __shfl_sync(0xffffffffu, key != INT_MAX ? rank : -1, j);
     if (rj == lane) mask |= 1u << (j / D);
+    if (rj >= 0 && ((am >> j) & 1u)) anc |= 1u << rj;
   }
-  if (lane < 32) wr.dmask[lane] = mask;
-  if (lane == 0) wr.nd = __popc(fm);
+  wr.dmask[lane] = mask;
+  if (lane == 0) {
+    wr.nd = __popc(fm);
+    wr.anchor_rows = anc;
+  }
   __syncwarp();
 }
 
-template <typename TZ, int D>
+template <typename TZ, int D, bool SPLIT>
 __global__ void __launch_bounds__(WT_WARPS * 32, 2)
 k_swiglu_warp(const float* __restrict__ topk_w, const int* __restrict__ node_row, int T, int k,
-              const float* __restrict__ h, int I, TZ* __restrict__ z, int cols_per_item) {
+              const float* __restrict__ h, int I, TZ* __restrict__ z, int cols_per_item,
+              const SplitParts hs) {
   __shared__ WarpRows wrs[WT_WARPS];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   WarpRows& wr = wrs[warp];
@@ -349,6 +360,15 @@ k_swiglu_warp(const float* __restrict__ topk_w, const int* __restrict__ node_row
               const float4 b = __ldg(reinterpret_cast<const float4*>(h + (size_t)r * 2 * I + I + c));
               pg.x += a.x; pg.y += a.y; pg.z += a.z; pg.w += a.w;
               pu.x += b.x; pu.y += b.y; pu.z += b.z; pu.w += b.w;
+              if (SPLIT && (l + 1 == D || wr.rows[sl * D + l + 1] < 0)) {  // anchor: split partials
+                for (int sp = 1; sp < hs.splits; ++sp) {
+                  const float* hp = hs.part + (sp - 1) * hs.stride + (size_t)r * 2 * I;
+                  const float4 a2 = __ldg(reinterpret_cast<const float4*>(hp + c));
+                  const float4 b2 = __ldg(reinterpret_cast<const float4*>(hp + I + c));
+                  pg.x += a2.x; pg.y += a2.y; pg.z += a2.z; pg.w += a2.w;
+                  pu.x += b2.x; pu.y += b2.y; pu.z += b2.z; pu.w += b2.w;
+                }
+              }
             }
           }
           const float g = wr.g[sl];
@@ -376,7 +396,7 @@ k_swiglu_warp(const float* __restrict__ topk_w, const int* __restrict__ node_row
 template <typename TY>
 __global__ void __launch_bounds__(WT_WARPS * 32, 2)
 k_combine_warp(const int* __restrict__ node_row, int k, int D, const float* __restrict__ ypart,
-               int H, TY* __restrict__ y, int T, int cols_per_item) {
+               int H, TY* __restrict__ y, int T, int cols_per_item, const SplitParts ys) {
   __shared__ WarpRows wrs[WT_WARPS];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   WarpRows& wr = wrs[warp];
@@ -406,6 +426,16 @@ k_combine_warp(const int* __restrict__ node_row, int k, int D, const float* __re
         const float4 v = __ldg(reinterpret_cast<const float4*>(ypart + (size_t)wr.drow[q] * H + c));
         acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
       }
+      if (ys.splits > 1) {  // anchor rows' split-K partials: rows ascending, then splits
+        for (unsigned b = wr.anchor_rows; b; b &= b - 1) {
+          const int d = __ffs(b) - 1;
+          for (int sp = 1; sp < ys.splits; ++sp) {
+            const float4 v = __ldg(reinterpret_cast<const float4*>(
+                ys.part + (sp - 1) * ys.stride + (size_t)wr.drow[d] * H + c));
+            acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
+          }
+        }
+      }
       store4<TY>(y + (size_t)t * H + c, acc);
     }
     __syncwarp();
@@ -414,7 +444,7 @@ k_combine_warp(const int* __restrict__ node_row, int k, int D, const float* __re
 
 }  // namespace
 
-static bool warp_kernels_fit(const lx_layer* L, int k) {
+bool warp_kernels_fit(const lx_layer* L, int k) {
   return k <= WT_SLOTS && k * L->max_depth <= 32 && L->I % 4 == 0 && L->H % 4 == 0;
 }
 
@@ -434,27 +464,40 @@ static int warp_grid(const lx_layer* L, int T, int width, int cols) {
   return (int)std::min<long>((items + WT_WARPS - 1) / WT_WARPS, (long)L->num_sms * 4);
 }
 
-template <typename TZ>
-static void launch_swiglu_warp(lx_layer* L, int T, int k, TZ* z, cudaStream_t s) {
+template <typename TZ, int D>
+static void launch_swiglu_d(lx_layer* L, int T, int k, TZ* z, cudaStream_t s, const SplitParts& hs,
+                            int grid, int cols) {
   Workspace& w = L->ws;
+  if (hs.splits > 1)
+    k_swiglu_warp<TZ, D, true><<<grid, WT_WARPS * 32, 0, s>>>(w.topk_w, w.node_row, T, k, w.h,
+                                                              L->I, z, cols, hs);
+  else
+    k_swiglu_warp<TZ, D, false><<<grid, WT_WARPS * 32, 0, s>>>(w.topk_w, w.node_row, T, k, w.h,
+                                                               L->I, z, cols, hs);
+}
+
+template <typename TZ>
+static void launch_swiglu_warp(lx_layer* L, int T, int k, TZ* z, cudaStream_t s,
+                               const SplitParts& hs) {
   const int cols = warp_item_cols(L, T, L->I);
   const int grid = warp_grid(L, T, L->I, cols);
   switch (L->max_depth) {
-    case 1: k_swiglu_warp<TZ, 1><<<grid, WT_WARPS * 32, 0, s>>>(w.topk_w, w.node_row, T, k, w.h, L->I, z, cols); break;
-    case 2: k_swiglu_warp<TZ, 2><<<grid, WT_WARPS * 32, 0, s>>>(w.topk_w, w.node_row, T, k, w.h, L->I, z, cols); break;
-    case 3: k_swiglu_warp<TZ, 3><<<grid, WT_WARPS * 32, 0, s>>>(w.topk_w, w.node_row, T, k, w.h, L->I, z, cols); break;
-    default: k_swiglu_warp<TZ, 4><<<grid, WT_WARPS * 32, 0, s>>>(w.topk_w, w.node_row, T, k, w.h, L->I, z, cols); break;
+    case 1: launch_swiglu_d<TZ, 1>(L, T, k, z, s, hs, grid, cols); break;
+    case 2: launch_swiglu_d<TZ, 2>(L, T, k, z, s, hs, grid, cols); break;
+    case 3: launch_swiglu_d<TZ, 3>(L, T, k, z, s, hs, grid, cols); break;
+    default: launch_swiglu_d<TZ, 4>(L, T, k, z, s, hs, grid, cols); break;
   }
 }
 
-lx_status launch_swiglu(lx_layer* L, int T, int k, void* z, bool z_bf16, cudaStream_t s) {
+lx_status launch_swiglu(lx_layer* L, int T, int k, void* z, bool z_bf16, cudaStream_t s,
+                        SplitParts hs) {
   Workspace& w = L->ws;
   ProfScope ps(L, s, z_bf16 ? "swiglu" : "generic_swiglu");
   if (warp_kernels_fit(L, k)) {
     if (z_bf16)
-      launch_swiglu_warp(L, T, k, static_cast<__nv_bfloat16*>(z), s);
+      launch_swiglu_warp(L, T, k, static_cast<__nv_bfloat16*>(z), s, hs);
     else
-      launch_swiglu_warp(L, T, k, static_cast<float*>(z), s);
+      launch_swiglu_warp(L, T, k, static_cast<float*>(z), s, hs);
     LX_CUDA(cudaGetLastError());
     return LX_OK;
   }
@@ -474,7 +517,7 @@ lx_status launch_swiglu(lx_layer* L, int T, int k, void* z, bool z_bf16, cudaStr
   return LX_OK;
 }
 
-lx_status launch_combine(lx_layer* L, int T, int k, void* y, cudaStream_t s) {
+lx_status launch_combine(lx_layer* L, int T, int k, void* y, cudaStream_t s, SplitParts ys) {
   Workspace& w = L->ws;
   ProfScope ps(L, s, "combine");
   if (warp_kernels_fit(L, k)) {
@@ -482,10 +525,10 @@ lx_status launch_combine(lx_layer* L, int T, int k, void* y, cudaStream_t s) {
     const int g2 = warp_grid(L, T, L->H, cols);
     if (L->dtype == LX_BF16)
       k_combine_warp<__nv_bfloat16><<<g2, WT_WARPS * 32, 0, s>>>(
-          w.node_row, k, L->max_depth, w.ypart, L->H, (__nv_bfloat16*)y, T, cols);
+          w.node_row, k, L->max_depth, w.ypart, L->H, (__nv_bfloat16*)y, T, cols, ys);
     else
       k_combine_warp<float><<<g2, WT_WARPS * 32, 0, s>>>(w.node_row, k, L->max_depth, w.ypart,
-                                                          L->H, (float*)y, T, cols);
+                                                          L->H, (float*)y, T, cols, ys);
     LX_CUDA(cudaGetLastError());
     return LX_OK;
   }

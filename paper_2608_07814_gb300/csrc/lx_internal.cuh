@@ -178,6 +178,12 @@ struct StreamOp {
   const int* rank;
   int ncol_max;              // column tiles of the widest node of this op
   int ntb;                   // token blocks (64 tokens) of the largest possible bucket
+  // split-K: K-range s of a tile (kbs 64-wide K blocks) writes fp32 partial s,
+  // partial 0 to `out`, partial s >= 1 to split_out + (s - 1) * split_stride
+  int nsplit;
+  int kbs;
+  float* split_out;
+  long split_stride;
 };
 
 // The streaming launches: group 0 = {UP_ANCHOR, UP_V}, 1 = {UP_U},
@@ -266,6 +272,11 @@ struct Workspace {
   int* act_n = nullptr;         // [2] their counts
   int* sctr = nullptr;          // [N_TILE_COUNTERS] streaming / tensor-core tile counters
   CUtensorMap* xmaps = nullptr; // [3] TMA maps of Pb, zb, Qb (tensor-core A operands)
+  // split-K partials of the anchor products on the streaming path:
+  // [LX_STREAM_MAX_SPLIT - 1][split_rows][2I] and [..][split_rows][H]
+  float* hsplit = nullptr;
+  float* ysplit = nullptr;
+  long split_rows = 0;
   int* err = nullptr;           // device error word
 };
 
@@ -337,8 +348,20 @@ lx_status launch_router(lx_layer* L, const void* x, int T, int k, float* logits,
 lx_status launch_bucket(lx_layer* L, const int* topk_id, int T, int k, cudaStream_t s);
 lx_status launch_generic_experts(lx_layer* L, const void* x, int T, int k, void* y,
                                  cudaStream_t s);
-lx_status launch_swiglu(lx_layer* L, int T, int k, void* z, bool z_bf16, cudaStream_t s);
-lx_status launch_combine(lx_layer* L, int T, int k, void* y, cudaStream_t s);
+// Anchor split-K partials the SwiGLU / combine kernels add to the anchor rows
+// (the last node of each expert's path): partial s >= 1 of row r at
+// part + (s - 1) * stride + r * width.
+struct SplitParts {
+  const float* part = nullptr;
+  int splits = 1;
+  long stride = 0;
+};
+constexpr int LX_STREAM_MAX_SPLIT = 4;
+bool warp_kernels_fit(const lx_layer* L, int k);
+lx_status launch_swiglu(lx_layer* L, int T, int k, void* z, bool z_bf16, cudaStream_t s,
+                        SplitParts hs = SplitParts());
+lx_status launch_combine(lx_layer* L, int T, int k, void* y, cudaStream_t s,
+                         SplitParts ys = SplitParts());
 lx_status launch_fast_experts(lx_layer* L, const void* x, int T, int k, void* y, cudaStream_t s);
 lx_status launch_tc_experts(lx_layer* L, const void* x, int T, int k, void* y, cudaStream_t s);
 int tc_tile_tokens();

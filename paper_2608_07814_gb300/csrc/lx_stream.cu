@@ -5,8 +5,10 @@
 // touched weight byte once from HBM (Sec. 5.2: the projections run at about one
 // FLOP per byte), so the kernel is organised around the weight stream:
 //
-//   * one tile = 64 weight rows (output columns) x 64 tokens of one node,
-//     over the full K;
+//   * one tile = 64 weight rows (output columns) x 32 tokens of one node,
+//     over the full K or, for the anchors, one of up to four K ranges (split-K:
+//     every range writes an fp32 partial that the next kernel adds in order),
+//     so that the tiles left at the end of a launch are short;
 //   * a producer warp streams the tile's weights with 2-D TMA loads
 //     (cp.async.bulk.tensor, 64x64 bf16 boxes, 128-byte swizzle) into a
 //     4-stage shared-memory ring guarded by mbarriers;
@@ -31,17 +33,23 @@ namespace lx {
 namespace {
 
 constexpr int SW_ROWS = 64;         // weight rows per tile
-constexpr int SW_TOK = 64;          // tokens per tile
+// Tokens per tile.  Decode buckets are small (at 64 tokens top-8 over 32
+// clusters the median anchor bucket holds a handful of tokens), so a 32-token
+// slot keeps the stage at 13 KiB and four CTAs of four stages fit an SM:
+// 128 KiB of weights in flight per SM.  Larger buckets take several token blocks.
+constexpr int SW_TOK = 32;
 constexpr int SW_BOX = 64;          // K per stage = one TMA box of 64 K x 64 rows
 constexpr int SW_BOX_BYTES = SW_BOX * SW_ROWS * 2;
 constexpr int SW_XROW = SW_BOX * 2 + 16;           // padded token row in shared memory
-constexpr int SW_STAGE_BYTES = SW_BOX_BYTES + SW_TOK * SW_XROW;  // 17 KiB, 1024-aligned
+constexpr int SW_STAGE_BYTES = (SW_BOX_BYTES + SW_TOK * SW_XROW + 1023) / 1024 * 1024;
 constexpr int SW_STAGES = 4;
+constexpr int SW_CTAS_PER_SM = 4;
 constexpr int SW_CONSUMERS = 2;
 constexpr int SW_MT = SW_ROWS / (16 * SW_CONSUMERS);  // 16-row MMA tiles per consumer warp
 constexpr int SW_THREADS = 32 * (1 + SW_CONSUMERS);
 constexpr unsigned long long SW_TIMEOUT_CYCLES = 4000000000ull;  // ~2 s
 static_assert(SW_STAGE_BYTES % 1024 == 0, "stages must keep the 128B-swizzle alignment");
+static_assert(SW_TOK % 8 == 0 && SW_TOK <= 64, "token slot: whole 8-token MMA columns");
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -136,14 +144,15 @@ __device__ __forceinline__ uint4 lds_v4(uint32_t addr) {
 
 struct TileInfo {
   int op, node, grp, row0, tok0, M, Ng, K, ncb;
+  int kb0, nkb, split;  // K blocks [kb0, kb0 + nkb) of split `split`
   bool active;
 };
 
 __device__ __forceinline__ int op_tiles(const StreamOp& op) {
-  return *op.n_active * op.ntb * op.shape.groups * op.ncol_max;
+  return *op.n_active * op.ntb * op.shape.groups * op.ncol_max * op.nsplit;
 }
 
-// Tile index -> (op, node, token block, group, column tile).
+// Tile index -> (op, node, token block, group, column tile, K split).
 __device__ __forceinline__ void decode_tile(const StreamLaunch& P, int tile, int tiles0,
                                             TileInfo& ti) {
   int o = 0, local = tile;
@@ -152,13 +161,16 @@ __device__ __forceinline__ void decode_tile(const StreamLaunch& P, int tile, int
     local = tile - tiles0;
   }
   const StreamOp& op = P.op[o];
-  const int per_tb = op.shape.groups * op.ncol_max;
+  // (item, token block, group, column tile, split), split fastest
+  const int per_tb = op.shape.groups * op.ncol_max * op.nsplit;
   const int per_item = op.ntb * per_tb;
   const int item = local / per_item;
   int rem = local - item * per_item;
   const int tb = rem / per_tb;
   rem -= tb * per_tb;
-  const int grp = rem / op.ncol_max, ct = rem - grp * op.ncol_max;
+  const int grp = rem / (op.ncol_max * op.nsplit);
+  rem -= grp * op.ncol_max * op.nsplit;
+  const int ct = rem / op.nsplit, split = rem - ct * op.nsplit;
   const int n = op.items[item];
   const int r = op.rank[n];
   const int b0 = op.node_off[n], b1 = op.node_off[n + 1];
@@ -171,7 +183,11 @@ __device__ __forceinline__ void decode_tile(const StreamLaunch& P, int tile, int
   ti.tok0 = b0 + tb * SW_TOK;
   ti.M = min(SW_TOK, b1 - ti.tok0);
   ti.ncb = 1;
-  ti.active = ti.M > 0 && ti.row0 < ti.Ng;
+  const int nkb_all = (ti.K + SW_BOX - 1) / SW_BOX;
+  ti.split = split;
+  ti.kb0 = split * op.kbs;
+  ti.nkb = min(op.kbs, nkb_all - ti.kb0);
+  ti.active = ti.M > 0 && ti.row0 < ti.Ng && ti.nkb > 0;
 }
 
 template <int NT>
@@ -181,8 +197,11 @@ __device__ __forceinline__ bool consume_tile(const StreamLaunch& P, const TileIn
   const StreamOp& op = P.op[ti.op];
   const int lane = threadIdx.x & 31, cw = (threadIdx.x >> 5) - 1;
   const int g = lane >> 2, q = lane & 3;
-  const int nkb = (ti.K + SW_BOX - 1) / SW_BOX;
+  const int nkb = ti.nkb;
   const int wrow = cw * 16 * SW_MT + g;  // first of this lane's weight rows in a 64-row block
+  // split 0 (and unsplit tiles) write `out`; split s >= 1 its fp32 partial
+  float* const out_f = ti.split == 0 ? static_cast<float*>(op.out)
+                                     : op.split_out + (ti.split - 1) * op.split_stride;
   for (int cb = 0; cb < ti.ncb; ++cb) {
     float acc[SW_MT][NT][4];
 #pragma unroll
@@ -229,7 +248,7 @@ __device__ __forceinline__ bool consume_tile(const StreamLaunch& P, const TileIn
           const int m = 8 * j + 2 * q + (c & 1);
           if (wr < ti.Ng && m < ti.M) {
             const size_t o = (size_t)(ti.tok0 + m) * op.ldo + (size_t)ti.grp * ti.Ng + wr;
-            if (op.out_f32) static_cast<float*>(op.out)[o] = acc[i][j][c];
+            if (op.out_f32) out_f[o] = acc[i][j][c];
             else static_cast<__nv_bfloat16*>(op.out)[o] = __float2bfloat16_rn(acc[i][j][c]);
           }
         }
@@ -274,7 +293,7 @@ k_stream_gemm(const __grid_constant__ StreamLaunch P) {
       const StreamOp& op = P.op[t.op];
       const long acol = (long)t.grp * t.K;
 #pragma unroll
-      for (int h = 0; h < 2; ++h) {
+      for (int h = 0; h < (SW_TOK + 31) / 32; ++h) {
         const int m = lane + 32 * h;
         if (t.active && m < t.M) {
           const int row = t.tok0 + m;
@@ -302,7 +321,7 @@ k_stream_gemm(const __grid_constant__ StreamLaunch P) {
         const CUtensorMap* map = op.tmaps + ti.node;
         const int rt0 = (ti.grp * ti.Ng + ti.row0) / SW_ROWS;
         const __nv_bfloat16* const* xs = xsrc + buf * SW_TOK;
-        const int nkb = (ti.K + SW_BOX - 1) / SW_BOX;
+        const int nkb = ti.nkb, kb0 = ti.kb0;
         for (int cb = 0; cb < ti.ncb && ok; ++cb) {
           for (int kb = 0; kb < nkb; ++kb, ++it) {
             const uint32_t s = it % SW_STAGES;
@@ -320,11 +339,12 @@ k_stream_gemm(const __grid_constant__ StreamLaunch P) {
               break;
             }
             const uint32_t wbox = smem_base + s * SW_STAGE_BYTES;
-            if (lane == 0) tma_load_tile(wbox, map, kb, rt0 + cb, full0 + 8 * s);
+            if (lane == 0) tma_load_tile(wbox, map, kb0 + kb, rt0 + cb, full0 + 8 * s);
             // token rows: M rows x 128 bytes as 16-byte pieces over the 32 lanes
             for (int piece = lane; piece < ti.M * 8; piece += 32) {
               const int m = piece >> 3, u = piece & 7;
-              cp_async16(wbox + SW_BOX_BYTES + m * SW_XROW + u * 16, xs[m] + kb * SW_BOX + u * 8);
+              cp_async16(wbox + SW_BOX_BYTES + m * SW_XROW + u * 16,
+                         xs[m] + (kb0 + kb) * SW_BOX + u * 8);
             }
             cp_async_arrive(full0 + 8 * s);
             if (!prepared && cb == 0 && (kb == 1 || kb == nkb - 1)) {
@@ -400,8 +420,9 @@ k_stream_gemm(const __grid_constant__ StreamLaunch P) {
     bool ok;
     if (nt <= 1) ok = consume_tile<1>(P, ti, smem_base, full0, empty0, it, abort_flag);
     else if (nt <= 2) ok = consume_tile<2>(P, ti, smem_base, full0, empty0, it, abort_flag);
-    else if (nt <= 4) ok = consume_tile<4>(P, ti, smem_base, full0, empty0, it, abort_flag);
-    else ok = consume_tile<8>(P, ti, smem_base, full0, empty0, it, abort_flag);
+    else if (SW_TOK <= 32 || nt <= 4)
+      ok = consume_tile<SW_TOK <= 32 ? SW_TOK / 8 : 4>(P, ti, smem_base, full0, empty0, it, abort_flag);
+    else ok = consume_tile<SW_TOK / 8>(P, ti, smem_base, full0, empty0, it, abort_flag);
     if (!ok) {
       if (lane == 0) {
         atomicExch(P.err, LX_ERR_TIMEOUT);
@@ -424,7 +445,7 @@ lx_status launch_stream(lx_layer* L, const StreamLaunch& P, cudaStream_t s, cons
   static bool done[64] = {};
   LX_CUDA(smem_cap_once((const void*)k_stream_gemm, smem, L->device, done));
   ProfScope ps(L, s, name);
-  k_stream_gemm<<<L->num_sms * 3, SW_THREADS, smem, s>>>(P);
+  k_stream_gemm<<<L->num_sms * SW_CTAS_PER_SM, SW_THREADS, smem, s>>>(P);
   LX_CUDA(cudaGetLastError());
   return LX_OK;
 }
@@ -451,7 +472,28 @@ static StreamOp make_op(lx_layer* L, int op, int T, const __nv_bfloat16* X, long
     ng_max = std::max(ng_max, o.shape.n_const + o.shape.n_rank * L->rank[n]);
   o.ncol_max = (ng_max + SW_ROWS - 1) / SW_ROWS;
   o.ntb = (T + SW_TOK - 1) / SW_TOK;
+  o.nsplit = 1;
+  o.kbs = 1 << 20;
+  o.split_out = nullptr;
+  o.split_stride = 0;
   return o;
+}
+
+// Split the anchor op's K into at most LX_STREAM_MAX_SPLIT ranges of about
+// kStreamSplitBlocks 64-wide blocks (a 64 KB weight slice per tile), so that
+// the last tiles of a launch are short.  Partials go to `part`.
+constexpr int kStreamSplitBlocks = 8;
+static void split_op(lx_layer* L, StreamOp& o, float* part, long stride) {
+  if (!part) return;
+  const int K = o.shape.k_const;  // anchors: K does not depend on a rank
+  const int nkb = (K + SW_BOX - 1) / SW_BOX;
+  int ns = std::min(LX_STREAM_MAX_SPLIT, (nkb + kStreamSplitBlocks - 1) / kStreamSplitBlocks);
+  if (ns <= 1) return;
+  o.kbs = (nkb + ns - 1) / ns;
+  o.nsplit = (nkb + o.kbs - 1) / o.kbs;
+  o.split_out = part;
+  o.split_stride = stride;
+  (void)L;
 }
 
 // One streaming launch (launch group g) over up to two ops' tile grids.
@@ -474,20 +516,37 @@ lx_status launch_fast_experts(lx_layer* L, const void* x, int T, int k, void* y,
   Workspace& w = L->ws;
   const long H = L->H, I = L->I, rmax = L->max_rank;
   const __nv_bfloat16* xb = static_cast<const __nv_bfloat16*>(x);
-  // x-side: shared anchor gate/up, and x V of every correction
+  const bool split = w.hsplit && w.ysplit && warp_kernels_fit(L, k) &&
+                     (long)T * std::min<long>(L->N, (long)k * L->max_depth) <= w.split_rows;
+  // x-side: x V of every correction (whole-K tiles, claimed first), and the
+  // shared anchor gate/up in split-K slices
+  StreamOp up_a = make_op(L, OP_UP_ANCHOR, T, xb, H, w.node_tok, w.h, 2 * I, true);
+  if (split) split_op(L, up_a, w.hsplit, w.split_rows * 2 * I);
   const StreamOp up_v = make_op(L, OP_UP_V, T, xb, H, w.node_tok, w.Pb, 2 * rmax, false);
-  LX_TRY(run_stream(L, 0, make_op(L, OP_UP_ANCHOR, T, xb, H, w.node_tok, w.h, 2 * I, true), &up_v,
-                    s, "stream_up_anchor_V"));
+  LX_TRY(run_stream(L, 0, up_v, &up_a, s, "stream_up_anchor_V"));
   LX_TRY(run_stream(L, 1, make_op(L, OP_UP_U, T, w.Pb, 2 * rmax, nullptr, w.h, 2 * I, true),
                     nullptr, s, "stream_up_U"));
-  LX_TRY(launch_swiglu(L, T, k, w.zb, true, s));
-  // z-side: shared anchor down projection, and z Vd of every correction
+  SplitParts hs, ys;
+  if (up_a.nsplit > 1) {
+    hs.part = up_a.split_out;
+    hs.splits = up_a.nsplit;
+    hs.stride = up_a.split_stride;
+  }
+  LX_TRY(launch_swiglu(L, T, k, w.zb, true, s, hs));
+  // z-side: z Vd of every correction first, then the shared anchor down
+  // projection in split-K slices
+  StreamOp dn_a = make_op(L, OP_DN_ANCHOR, T, w.zb, I, nullptr, w.ypart, H, true);
+  if (split) split_op(L, dn_a, w.ysplit, w.split_rows * H);
   const StreamOp dn_v = make_op(L, OP_DN_V, T, w.zb, I, nullptr, w.Qb, rmax, false);
-  LX_TRY(run_stream(L, 2, make_op(L, OP_DN_ANCHOR, T, w.zb, I, nullptr, w.ypart, H, true), &dn_v,
-                    s, "stream_dn_anchor_V"));
+  LX_TRY(run_stream(L, 2, dn_v, &dn_a, s, "stream_dn_anchor_V"));
   LX_TRY(run_stream(L, 3, make_op(L, OP_DN_U, T, w.Qb, rmax, nullptr, w.ypart, H, true), nullptr,
                     s, "stream_dn_U"));
-  LX_TRY(launch_combine(L, T, k, y, s));
+  if (dn_a.nsplit > 1) {
+    ys.part = dn_a.split_out;
+    ys.splits = dn_a.nsplit;
+    ys.stride = dn_a.split_stride;
+  }
+  LX_TRY(launch_combine(L, T, k, y, s, ys));
   return LX_OK;
 }
 

@@ -114,6 +114,12 @@ SMALL = {
                                                         seed=14, factor_std="visible"),
     "stream_tree": lambda: synth.tree_layer(256, 192, 2, 4, 3, 128, 64, 8, "bf16", seed=15,
                                             factor_std="visible", skew=synth.TREE_SKEW),
+    # K long enough for split-K anchor tiles on the streaming path (ragged last split)
+    "stream_split_ragged": lambda: synth.flat_layer(1088, 448, [4] * 4, 64, 4, "bf16", seed=16,
+                                                    factor_std="visible", skew=synth.QWEN_SKEW),
+    "stream_split_tree": lambda: synth.tree_layer(1024, 640, 2, 4, 3, 128, 64, 8, "bf16",
+                                                  seed=17, factor_std="visible",
+                                                  skew=synth.TREE_SKEW),
 }
 
 STREAM = [n for n in SMALL if n.startswith("stream")]
@@ -264,6 +270,18 @@ FULL = {
 def test_qwen_decode_batches(T):
     src, L = installed("qwen", FULL["qwen"])
     x = synth.tokens(src, T, seed=T)
+    ids, _ = check_route(src, L, x, 8)
+    check_buckets(src, L, ids)
+    check_forward(src, L, x, 8)
+
+
+@pytest.mark.parametrize("name", ["high_e", "tree"])
+@pytest.mark.parametrize("T", [1, 64])
+def test_full_layers_decode(name, T):
+    """Decode batches of the other full-size layers (split-K anchor tiles with
+    three and four K ranges, depth-3 tree paths)."""
+    src, L = installed(name, FULL[name])
+    x = synth.tokens(src, T, seed=40 + T)
     ids, _ = check_route(src, L, x, 8)
     check_buckets(src, L, ids)
     check_forward(src, L, x, 8)
