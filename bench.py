@@ -251,7 +251,7 @@ def run_lx(args, rank, world, local_rank):
             layers[i % n_copies].moe_forward(xs[i % n_batches], k, ys[i % n_batches])
 
     # One profiled pass of the same steps fills each layer's event pool, so the
-    # capture below creates no events.
+    # instrumented capture below creates no events.
     for L in layers:
         L.read_profile()
         L.set_profiling(True)
@@ -259,14 +259,25 @@ def run_lx(args, rank, world, local_rank):
     torch.cuda.synchronize()
     for L in layers:
         L.read_profile(cap=1 << 20)
-    graph = None
+    graph = graph_prof = None
     if not args.no_graph:
-        # The timed region is one CUDA graph of the K forwards: the GPU runs the
-        # launches back to back, with the library's per-kernel events as
-        # external event nodes stamped by the replay.
+        # Two CUDA graphs of the same K forwards: `graph_prof` carries the
+        # library's per-kernel events (external event nodes stamped by the
+        # replay; dependent launch off) and gives the kernel durations;
+        # `graph` has no events (dependent launch on) and gives the step time.
+        graph_prof = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph_prof):
+            steps(args.steps)
+    for L in layers:
+        L.set_profiling(False)
+    if not args.no_graph:
         graph = torch.cuda.CUDAGraph()
         with torch.cuda.graph(graph):
             steps(args.steps)
+        graph.replay()  # untimed replay: first-launch costs of the graph
+        torch.cuda.synchronize()
+
+    # timed region 1: the step time (no instrumentation)
     if world > 1:
         torch.distributed.barrier()
     torch.cuda.synchronize()
@@ -284,8 +295,19 @@ def run_lx(args, rank, world, local_rank):
     t_wall1 = time.time()
     clocks.mark(t_wall0, t_wall1)
     ms = ev0.elapsed_time(ev1)
-    for L in layers:
-        L.set_profiling(False)
+
+    # timed region 2: the same steps with per-kernel events
+    t_p0 = time.time()
+    if graph_prof is not None:
+        graph_prof.replay()
+    else:
+        for L in layers:
+            L.set_profiling(True)
+        steps(args.steps)
+        for L in layers:
+            L.set_profiling(False)
+    torch.cuda.synchronize()
+    clocks.mark(t_p0, time.time())
 
     # per-kernel device times of the timed launches (in launch order per copy)
     per_copy = [L.read_profile(cap=1 << 20) for L in layers]
@@ -380,8 +402,9 @@ def run_lx(args, rank, world, local_rank):
                    "l2": f"{n_copies} rotating device copies of the layer and 8 token batches "
                          "(inputs larger than L2)",
                    "parallelism": f"replica per GPU x{world}",
-                   "timing": "one CUDA graph of the K forwards" if graph is not None
-                             else "K forwards launched one by one"},
+                   "timing": ("one CUDA graph of the K forwards (kernel durations from a "
+                              "second, event-instrumented graph of the same forwards)")
+                             if graph is not None else "K forwards launched one by one"},
         "roofline": roof,
         "kernels": {n: {"launches": counts[n], "avg_us": round(totals[n] / counts[n] * 1e3, 2),
                         "share": round(totals[n] / sum(totals.values()), 4)} for n in totals},

@@ -3,6 +3,7 @@
 #include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <cstdlib>
 #include <cstring>
 #include <string>
 #include <vector>
@@ -338,6 +339,11 @@ extern "C" lx_status lx_load_compressed_layer(const lx_layer_desc* d, const void
   LX_TRY(validate_desc(d, node_w, router_w));
   cudaStream_t s = (cudaStream_t)stream;
   lx_layer* L = new lx_layer();
+  {
+    // LX_PDL=0 turns programmatic dependent launch off (for A/B timing)
+    const char* pdl = std::getenv("LX_PDL");
+    L->pdl = !(pdl && pdl[0] == '0');
+  }
   L->H = d->d_model;
   L->I = d->d_ff;
   L->E = d->n_experts;

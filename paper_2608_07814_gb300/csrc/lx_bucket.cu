@@ -22,6 +22,7 @@ constexpr int SCAN_THREADS = 512;
 __global__ void k_mark(const int* __restrict__ topk_id, int T, int k, int N, int E, long Tp,
                        const int* __restrict__ paths, const int* __restrict__ path_len,
                        uint8_t* __restrict__ marks) {
+  pdl_wait();
   const int t = blockIdx.x * blockDim.x + threadIdx.x;
   if (t >= T) return;
   for (int s = 0; s < k; ++s) {
@@ -64,6 +65,7 @@ __device__ int block_excl_scan(int v, int* total) {
 __global__ void __launch_bounds__(SCAN_THREADS)
 k_key_scan(const uint8_t* __restrict__ marks, int T, long Tp, int* __restrict__ rank_in,
            int* __restrict__ key_cnt) {
+  pdl_wait();
   const int key = blockIdx.x;
   const uint8_t* m = marks + (size_t)key * Tp;
   int* r = rank_in + (size_t)key * Tp;
@@ -139,6 +141,7 @@ __global__ void k_offsets_plan(const int* __restrict__ key_cnt, int N, int E,
                                const int* __restrict__ anchors, int n_anchor,
                                const int* __restrict__ corrs, int n_corr, int* __restrict__ act,
                                int* __restrict__ act_n, int* __restrict__ sctr) {
+  pdl_wait();
   if (act) publish_active(key_cnt, anchors, n_anchor, corrs, n_corr, act, act_n, sctr);
   // node offsets then expert offsets
   for (int part = 0; part < 2; ++part) {
@@ -180,6 +183,7 @@ __global__ void k_scatter(const uint8_t* __restrict__ marks, const int* __restri
                           const int* __restrict__ key_off, const int* __restrict__ topk_id, int T,
                           int k, int N, long Tp, int* __restrict__ node_tok,
                           int* __restrict__ row_node, int* __restrict__ perm) {
+  pdl_wait();
   const int key = blockIdx.y;
   const int t = blockIdx.x * blockDim.x + threadIdx.x;
   if (t >= T) return;
@@ -205,6 +209,7 @@ __global__ void k_node_row(const int* __restrict__ topk_id, int T, int k, int E,
                            const int* __restrict__ paths, const int* __restrict__ path_len,
                            const int* __restrict__ key_off, const int* __restrict__ rank_in,
                            int* __restrict__ node_row) {
+  pdl_wait();
   const long a = (long)blockIdx.x * blockDim.x + threadIdx.x;
   if (a >= (long)T * k) return;
   const int t = (int)(a / k);
@@ -246,6 +251,7 @@ k_bucket_small(const float* __restrict__ logits, const int* __restrict__ ids_in,
                const int* __restrict__ anchors, int n_anchor, const int* __restrict__ corrs,
                int n_corr, int* __restrict__ act, int* __restrict__ act_n,
                int* __restrict__ sctr) {
+  pdl_wait();
   extern __shared__ __align__(16) unsigned char sm[];
   const int keys = N + E;
   const int Tp = (T + 15) & ~15;
@@ -393,7 +399,7 @@ lx_status launch_bucket_small(lx_layer* L, const float* logits, const int* ids_i
   static bool done[64] = {};
   LX_CUDA(smem_cap_once((const void*)k_bucket_small, (int)SB_SMEM_LIMIT, L->device, done));
   ProfScope ps(L, s, logits ? "topk_bucket_small" : "bucket_small");
-  k_bucket_small<<<1, SB_THREADS, smem, s>>>(logits, ids_in, T, k, L->E, L->N, L->max_depth,
+  launch_k(L, k_bucket_small, 1, SB_THREADS, smem, s, logits, ids_in, T, k, L->E, L->N, L->max_depth,
                                              L->d_paths, L->d_path_len, L->d_rank, topk_id, topk_w,
                                              w.key_off, w.node_tok, w.row_node, w.node_row, w.perm,
                                              w.tile_off, op_max_items(L), pa, L->d_anchors,
@@ -413,19 +419,19 @@ lx_status launch_bucket(lx_layer* L, const int* topk_id, int T, int k, cudaStrea
   }
   {
     ProfScope ps(L, s, "bucket_mark");
-    k_mark<<<(T + 255) / 256, 256, 0, s>>>(topk_id, T, k, L->N, L->E, Tp, L->d_paths,
-                                           L->d_path_len, w.marks);
+    launch_k(L, k_mark, (T + 255) / 256, 256, 0, s, topk_id, T, k, L->N, L->E, Tp, L->d_paths,
+             L->d_path_len, w.marks);
     LX_CUDA(cudaGetLastError());
   }
   {
     ProfScope ps(L, s, "bucket_scan");
-    k_key_scan<<<keys, SCAN_THREADS, 0, s>>>(w.marks, T, Tp, w.rank_in, w.key_cnt);
+    launch_k(L, k_key_scan, keys, SCAN_THREADS, 0, s, w.marks, T, Tp, w.rank_in, w.key_cnt);
     LX_CUDA(cudaGetLastError());
   }
   {
     const PlanArgs pa = make_plans(L, N_PLANS);
     ProfScope ps(L, s, "bucket_offsets");
-    k_offsets_plan<<<1, 1024, 0, s>>>(w.key_cnt, L->N, L->E, w.key_off, L->d_rank, w.tile_off,
+    launch_k(L, k_offsets_plan, 1, 1024, 0, s, w.key_cnt, L->N, L->E, w.key_off, L->d_rank, w.tile_off,
                                       op_max_items(L), pa, L->d_anchors, L->n_anchor, L->d_corrs,
                                       L->n_corr, w.act, w.act_n, w.sctr);
     LX_CUDA(cudaGetLastError());
@@ -433,16 +439,15 @@ lx_status launch_bucket(lx_layer* L, const int* topk_id, int T, int k, cudaStrea
   {
     ProfScope ps(L, s, "bucket_scatter");
     const dim3 grid((T + 255) / 256, keys);
-    k_scatter<<<grid, 256, 0, s>>>(w.marks, w.rank_in, w.key_off, topk_id, T, k, L->N, Tp,
+    launch_k(L, k_scatter, grid, 256, 0, s, w.marks, w.rank_in, w.key_off, topk_id, T, k, L->N, Tp,
                                    w.node_tok, w.row_node, w.perm);
     LX_CUDA(cudaGetLastError());
   }
   {
     ProfScope ps(L, s, "bucket_node_row");
     const long A = (long)T * k;
-    k_node_row<<<(unsigned)((A + 255) / 256), 256, 0, s>>>(topk_id, T, k, L->E, L->max_depth, Tp,
-                                                           L->d_paths, L->d_path_len, w.key_off,
-                                                           w.rank_in, w.node_row);
+    launch_k(L, k_node_row, (unsigned)((A + 255) / 256), 256, 0, s, topk_id, T, k, L->E,
+             L->max_depth, Tp, L->d_paths, L->d_path_len, w.key_off, w.rank_in, w.node_row);
     LX_CUDA(cudaGetLastError());
   }
   return LX_OK;

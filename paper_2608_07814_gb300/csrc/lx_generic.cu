@@ -24,6 +24,7 @@ constexpr int GG_THREADS = 256;
 template <typename TA, typename TW, int OPK>
 __global__ void __launch_bounds__(GG_THREADS)
 k_grouped_gemm(GemmArgs g) {
+  pdl_wait();
   __shared__ float As[G_BK][G_BM + 1];
   __shared__ float Ws[G_BK][G_BN + 1];
   const int total = g.tile_off[g.n_items];
@@ -134,6 +135,7 @@ __global__ void __launch_bounds__(SW_T)
 k_swiglu_aggregate(const int* __restrict__ topk_id, const float* __restrict__ topk_w,
                    const int* __restrict__ node_row, int T, int k, int D,
                    const float* __restrict__ h, int I, TZ* __restrict__ z) {
+  pdl_wait();
   extern __shared__ float4 zacc[];  // [distinct rows][SW_T]
   __shared__ int rows[LX_MAX_K * LX_MAX_DEPTH], lrow[LX_MAX_K * LX_MAX_DEPTH];
   __shared__ int drow[LX_MAX_K * LX_MAX_DEPTH];
@@ -212,6 +214,7 @@ template <typename TY>
 __global__ void __launch_bounds__(256)
 k_combine(const int* __restrict__ node_row, int k, int D, const float* __restrict__ ypart, int H,
           TY* __restrict__ y, int T) {
+  pdl_wait();
   __shared__ int raw_s[LX_MAX_K * LX_MAX_DEPTH];
   __shared__ int rows_s[LX_MAX_K * LX_MAX_DEPTH];
   __shared__ int nrows_s;
@@ -331,6 +334,7 @@ __global__ void __launch_bounds__(WT_WARPS * 32, 2)
 k_swiglu_warp(const float* __restrict__ topk_w, const int* __restrict__ node_row, int T, int k,
               const float* __restrict__ h, int I, TZ* __restrict__ z, int cols_per_item,
               const SplitParts hs) {
+  pdl_wait();
   __shared__ WarpRows wrs[WT_WARPS];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   WarpRows& wr = wrs[warp];
@@ -397,6 +401,7 @@ template <typename TY>
 __global__ void __launch_bounds__(WT_WARPS * 32, 2)
 k_combine_warp(const int* __restrict__ node_row, int k, int D, const float* __restrict__ ypart,
                int H, TY* __restrict__ y, int T, int cols_per_item, const SplitParts ys) {
+  pdl_wait();
   __shared__ WarpRows wrs[WT_WARPS];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   WarpRows& wr = wrs[warp];
@@ -469,10 +474,10 @@ static void launch_swiglu_d(lx_layer* L, int T, int k, TZ* z, cudaStream_t s, co
                             int grid, int cols) {
   Workspace& w = L->ws;
   if (hs.splits > 1)
-    k_swiglu_warp<TZ, D, true><<<grid, WT_WARPS * 32, 0, s>>>(w.topk_w, w.node_row, T, k, w.h,
+    launch_k(L, k_swiglu_warp<TZ, D, true>, grid, WT_WARPS * 32, 0, s, w.topk_w, w.node_row, T, k, w.h,
                                                               L->I, z, cols, hs);
   else
-    k_swiglu_warp<TZ, D, false><<<grid, WT_WARPS * 32, 0, s>>>(w.topk_w, w.node_row, T, k, w.h,
+    launch_k(L, k_swiglu_warp<TZ, D, false>, grid, WT_WARPS * 32, 0, s, w.topk_w, w.node_row, T, k, w.h,
                                                                L->I, z, cols, hs);
 }
 
@@ -506,11 +511,11 @@ lx_status launch_swiglu(lx_layer* L, int T, int k, void* z, bool z_bf16, cudaStr
   static bool done_b[64] = {}, done_f[64] = {};
   if (z_bf16) {
     LX_CUDA(smem_cap_once((const void*)k_swiglu_aggregate<__nv_bfloat16>, 200 * 1024, L->device, done_b));
-    k_swiglu_aggregate<__nv_bfloat16><<<grid, SW_T, smem, s>>>(
+    launch_k(L, k_swiglu_aggregate<__nv_bfloat16>, grid, SW_T, smem, s, 
         w.topk_id, w.topk_w, w.node_row, T, k, L->max_depth, w.h, L->I, (__nv_bfloat16*)z);
   } else {
     LX_CUDA(smem_cap_once((const void*)k_swiglu_aggregate<float>, 200 * 1024, L->device, done_f));
-    k_swiglu_aggregate<float><<<grid, SW_T, smem, s>>>(w.topk_id, w.topk_w, w.node_row, T, k,
+    launch_k(L, k_swiglu_aggregate<float>, grid, SW_T, smem, s, w.topk_id, w.topk_w, w.node_row, T, k,
                                                        L->max_depth, w.h, L->I, (float*)z);
   }
   LX_CUDA(cudaGetLastError());
@@ -524,20 +529,20 @@ lx_status launch_combine(lx_layer* L, int T, int k, void* y, cudaStream_t s, Spl
     const int cols = warp_item_cols(L, T, L->H);
     const int g2 = warp_grid(L, T, L->H, cols);
     if (L->dtype == LX_BF16)
-      k_combine_warp<__nv_bfloat16><<<g2, WT_WARPS * 32, 0, s>>>(
+      launch_k(L, k_combine_warp<__nv_bfloat16>, g2, WT_WARPS * 32, 0, s, 
           w.node_row, k, L->max_depth, w.ypart, L->H, (__nv_bfloat16*)y, T, cols, ys);
     else
-      k_combine_warp<float><<<g2, WT_WARPS * 32, 0, s>>>(w.node_row, k, L->max_depth, w.ypart,
+      launch_k(L, k_combine_warp<float>, g2, WT_WARPS * 32, 0, s, w.node_row, k, L->max_depth, w.ypart,
                                                           L->H, (float*)y, T, cols, ys);
     LX_CUDA(cudaGetLastError());
     return LX_OK;
   }
   const int grid = std::min(T, L->num_sms * 8);
   if (L->dtype == LX_BF16)
-    k_combine<__nv_bfloat16><<<grid, 256, 0, s>>>(w.node_row, k, L->max_depth, w.ypart, L->H,
+    launch_k(L, k_combine<__nv_bfloat16>, grid, 256, 0, s, w.node_row, k, L->max_depth, w.ypart, L->H,
                                                   (__nv_bfloat16*)y, T);
   else
-    k_combine<float><<<grid, 256, 0, s>>>(w.node_row, k, L->max_depth, w.ypart, L->H, (float*)y, T);
+    launch_k(L, k_combine<float>, grid, 256, 0, s, w.node_row, k, L->max_depth, w.ypart, L->H, (float*)y, T);
   LX_CUDA(cudaGetLastError());
   return LX_OK;
 }
@@ -564,7 +569,7 @@ lx_status run_gemm(lx_layer* L, const void* A, long lda, const int* gather,
   g.ldo = ldo;
   g.tiled = L->tiled ? 1 : 0;
   ProfScope ps(L, s, name);
-  k_grouped_gemm<TA, TW, op><<<L->num_sms * 4, GG_THREADS, 0, s>>>(g);
+  launch_k(L, k_grouped_gemm<TA, TW, op>, L->num_sms * 4, GG_THREADS, 0, s, g);
   LX_CUDA(cudaGetLastError());
   return LX_OK;
 }

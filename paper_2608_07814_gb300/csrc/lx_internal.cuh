@@ -316,6 +316,7 @@ struct lx_layer {
   lx::Workspace ws;
   int last_T = 0, last_k = 0;       // last bucketing
   bool profiling = false;
+  bool pdl = true;                  // programmatic dependent launch between kernels
   std::vector<lx::ProfRec> prof;
   std::vector<cudaEvent_t> event_pool;
 };
@@ -330,6 +331,35 @@ inline cudaError_t smem_cap_once(const void* func, int bytes, int device, bool (
       cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
   if (e == cudaSuccess && device >= 0 && device < 64) done[device] = true;
   return e;
+}
+
+// Kernel launch with programmatic dependent launch: the next kernel of the
+// stream may be scheduled while this one drains, and every kernel of the
+// library starts with griddepcontrol.wait (pdl_wait), which returns once its
+// predecessor has completed and its writes are visible.  Off while profiling,
+// so that the per-kernel events time one kernel each.  Launch errors surface
+// through cudaGetLastError at the call site.
+template <typename... KArgs, typename... Args>
+inline void launch_k(const lx_layer* L, void (*kern)(KArgs...), dim3 grid, dim3 block,
+                     size_t smem, cudaStream_t s, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = (L->pdl && !L->profiling) ? 1 : 0;
+  (void)cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
+}
+
+// Device side of the dependent launch: wait for the predecessor grid, then let
+// the successor be scheduled on SMs this grid leaves free.
+__device__ __forceinline__ void pdl_wait() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 
 // Launch-time timing helper: records events around a launch when profiling.

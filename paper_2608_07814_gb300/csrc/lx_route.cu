@@ -64,6 +64,7 @@ k_router_logits(const T* __restrict__ x, const T* __restrict__ W, const float* _
                 int Ttok, int E, int H, int experts_per_cta, float* __restrict__ logits,
                 int* __restrict__ tile_cnt, int k, int* __restrict__ topk_id,
                 float* __restrict__ topk_w) {
+  pdl_wait();
   extern __shared__ __align__(16) unsigned char smem[];
   T* xs = reinterpret_cast<T*>(smem);
   const int t0 = blockIdx.x * RT_TOK;
@@ -176,6 +177,7 @@ k_router_tiled(const __nv_bfloat16* __restrict__ x, const __nv_bfloat16* __restr
                const float* __restrict__ bias, int Ttok, int E, int H,
                float* __restrict__ logits, int k, int* __restrict__ topk_id,
                float* __restrict__ topk_w) {
+  pdl_wait();
   extern __shared__ __align__(16) unsigned char smem[];
   __nv_bfloat16* xs0 = reinterpret_cast<__nv_bfloat16*>(smem);
   __nv_bfloat16* xs1 = xs0 + (size_t)RTT_TOK * H;
@@ -294,7 +296,7 @@ lx_status launch_router(lx_layer* L, const void* x, int T, int k, float* logits,
       LX_CUDA(smem_cap_once((const void*)k_router_tiled, 200 * 1024, L->device, done_t));
       ProfScope ps(L, s, "router");
       const int grid = std::min(tiles, L->num_sms);
-      k_router_tiled<<<grid, RTT_THREADS, smem2, s>>>(
+      launch_k(L, k_router_tiled, grid, RTT_THREADS, smem2, s, 
           (const __nv_bfloat16*)x, (const __nv_bfloat16*)L->router_w, L->router_bias, T, L->E,
           L->H, logits, k, topk_id, topk_w);
       LX_CUDA(cudaGetLastError());
@@ -311,13 +313,13 @@ lx_status launch_router(lx_layer* L, const void* x, int T, int k, float* logits,
   if (L->dtype == LX_BF16) {
     auto kern = k_router_logits<__nv_bfloat16>;
     LX_CUDA(smem_cap_once((const void*)kern, 200 * 1024, L->device, done_bf16));
-    kern<<<grid, RT_THREADS, smem, s>>>((const __nv_bfloat16*)x, (const __nv_bfloat16*)L->router_w,
+    launch_k(L, kern, grid, RT_THREADS, smem, s, (const __nv_bfloat16*)x, (const __nv_bfloat16*)L->router_w,
                                         L->router_bias, T, L->E, L->H, per_cta, logits,
                                         L->ws.tile_cnt, k, topk_id, topk_w);
   } else {
     auto kern = k_router_logits<float>;
     LX_CUDA(smem_cap_once((const void*)kern, 200 * 1024, L->device, done_f32));
-    kern<<<grid, RT_THREADS, smem, s>>>((const float*)x, (const float*)L->router_w, L->router_bias,
+    launch_k(L, kern, grid, RT_THREADS, smem, s, (const float*)x, (const float*)L->router_w, L->router_bias,
                                         T, L->E, L->H, per_cta, logits, L->ws.tile_cnt, k,
                                         topk_id, topk_w);
   }

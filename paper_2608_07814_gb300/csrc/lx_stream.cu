@@ -260,6 +260,7 @@ __device__ __forceinline__ bool consume_tile(const StreamLaunch& P, const TileIn
 
 __global__ void __launch_bounds__(SW_THREADS)
 k_stream_gemm(const __grid_constant__ StreamLaunch P) {
+  pdl_wait();
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -445,7 +446,7 @@ lx_status launch_stream(lx_layer* L, const StreamLaunch& P, cudaStream_t s, cons
   static bool done[64] = {};
   LX_CUDA(smem_cap_once((const void*)k_stream_gemm, smem, L->device, done));
   ProfScope ps(L, s, name);
-  k_stream_gemm<<<L->num_sms * SW_CTAS_PER_SM, SW_THREADS, smem, s>>>(P);
+  launch_k(L, k_stream_gemm, L->num_sms * SW_CTAS_PER_SM, SW_THREADS, smem, s, P);
   LX_CUDA(cudaGetLastError());
   return LX_OK;
 }

@@ -208,6 +208,7 @@ __device__ __forceinline__ void tc_decode(const TcLaunch& P, int tile, TcTile& t
 }
 
 __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant__ TcLaunch P) {
+  pdl_wait();
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -492,7 +493,7 @@ lx_status launch_tc(lx_layer* L, const TcLaunch& P, cudaStream_t s, const char* 
   static bool done[64] = {};
   LX_CUDA(smem_cap_once((const void*)k_tc_gemm, smem, L->device, done));
   ProfScope ps(L, s, name);
-  k_tc_gemm<<<L->num_sms, TC_THREADS, smem, s>>>(P);
+  launch_k(L, k_tc_gemm, L->num_sms, TC_THREADS, smem, s, P);
   LX_CUDA(cudaGetLastError());
   return LX_OK;
 }
