@@ -190,14 +190,14 @@ def step_bytes(st, src, esz):
     return c
 
 
-def traffic_for(kernel):
-    """dram bytes per launch from the committed ncu summary, if the kernel's
-    source is unchanged since the capture; else None."""
+def traffic_for(kernel, workload):
+    """dram bytes per launch from the committed ncu summary, if it was taken on
+    this workload and the kernel's source is unchanged since; else None."""
     p = os.path.join(ROOT, "profiles", "traffic.json")
     if not os.path.exists(p):
         return None
     d = json.load(open(p)).get(kernel)
-    if not d:
+    if not d or d.get("workload") != workload:
         return None
     src = os.path.join(ROOT, d["source"])
     if not os.path.exists(src):
@@ -205,6 +205,29 @@ def traffic_for(kernel):
     if hashlib.sha256(open(src, "rb").read()).hexdigest() != d["sha256"]:
         return None
     return d["bytes_per_launch"]
+
+
+# ----------------------------------------------------------------------------
+# ranks: one replica per GPU on its own token batches (weak scaling)
+# ----------------------------------------------------------------------------
+def max_over_ranks(values, world, device=None):
+    """Element-wise max of per-rank timings; every rank calls it and gets the max."""
+    if world <= 1:
+        return [float(v) for v in values]
+    import torch
+    t = torch.tensor([float(v) for v in values], dtype=torch.float64, device=device)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return [float(v) for v in t]
+
+
+def whole_job_rate(units_per_rank_step, steps, world, ms):
+    """Units processed by all ranks per second, over the slowest rank's time."""
+    return units_per_rank_step * steps * world / (ms * 1e-3)
+
+
+def batch_seed(rank, b):
+    """Seed of batch b on a rank: every rank draws its own tokens."""
+    return 1000 * rank + b
 
 
 # ----------------------------------------------------------------------------
@@ -227,7 +250,7 @@ def run_lx(args, rank, world, local_rank):
     for L in layers:
         L.reserve(T, k)
     n_batches = 8
-    xs_host = [synth.tokens(src, T, seed=1000 * rank + b) for b in range(n_batches)]
+    xs_host = [synth.tokens(src, T, seed=batch_seed(rank, b)) for b in range(n_batches)]
     xs = [lx.host_to_torch(x, src.dtype).to(dev) for x in xs_host]
     ys = [torch.empty_like(x) for x in xs]
     stream = torch.cuda.current_stream()
@@ -357,10 +380,7 @@ def run_lx(args, rank, world, local_rank):
     clk = clocks.stop()
 
     # max over ranks
-    if world > 1:
-        t = torch.tensor([ms, ms_e2e], dtype=torch.float64, device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms, ms_e2e = float(t[0]), float(t[1])
+    ms, ms_e2e = max_over_ranks([ms, ms_e2e], world, dev)
     if rank != 0:
         return None
 
@@ -373,7 +393,7 @@ def run_lx(args, rank, world, local_rank):
         bytes_per_launch = kbytes[dom] / counts[dom]
         ach = bytes_per_launch / (avg_ms * 1e-3) / 1e9
         roof = {"kernel": dom, "bound": "hbm", "achieved": round(ach, 1), "peak": hbm,
-                "unit": "GB/s", "frac": round(ach / hbm, 4), "traffic": traffic_for(dom),
+                "unit": "GB/s", "frac": round(ach / hbm, 4), "traffic": traffic_for(dom, args.workload),
                 "algorithmic_bytes_per_launch": round(bytes_per_launch),
                 "avg_launch_us": round(avg_ms * 1e3, 2), "peak_source": f"{peak_kind} hbm_gbs"}
     elif dom in kflops:
@@ -382,7 +402,7 @@ def run_lx(args, rank, world, local_rank):
         flops_per_launch = kflops[dom] / counts[dom]
         ach = flops_per_launch / (avg_ms * 1e-3) / 1e12
         roof = {"kernel": dom, "bound": "tensor", "achieved": round(ach, 1), "peak": tf,
-                "unit": "TFLOP/s", "frac": round(ach / tf, 4), "traffic": traffic_for(dom),
+                "unit": "TFLOP/s", "frac": round(ach / tf, 4), "traffic": traffic_for(dom, args.workload),
                 "algorithmic_flops_per_launch": round(flops_per_launch),
                 "avg_launch_us": round(avg_ms * 1e3, 2),
                 "peak_source": f"{peak_kind} bf16_tflops (burst)"}
@@ -391,7 +411,8 @@ def run_lx(args, rank, world, local_rank):
     tokens = T * args.steps * world
     amort = np.mean([st["T"] * st["k"] / max(1, st["R_anchor"]) for st in stats])
     line = {
-        "metric": METRIC, "value": round(tokens / (ms * 1e-3), 1), "unit": "tokens/s",
+        "metric": METRIC, "value": round(whole_job_rate(T, args.steps, world, ms), 1),
+        "unit": "tokens/s",
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": round(ms / args.steps, 5), "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16" if src.dtype == "bf16" else "f32",
@@ -411,7 +432,7 @@ def run_lx(args, rank, world, local_rank):
         "step_roofline": {"algorithmic_bytes_per_step": round(float(np.mean(sb))),
                           "achieved_gbs": round(step_gbs, 1), "frac": round(step_gbs / hbm, 4)},
         "amortisation": round(float(amort), 3),
-        "e2e": {"value": round(T * k_e2e * world / (ms_e2e * 1e-3), 1), "unit": "tokens/s",
+        "e2e": {"value": round(whole_job_rate(T, k_e2e, world, ms_e2e), 1), "unit": "tokens/s",
                 "steps": k_e2e, "h2d_bytes_per_step": int(xs[0].numel() * xs[0].element_size()),
                 "d2h_bytes_per_step": int(ys[0].numel() * ys[0].element_size())},
         "gpu_launches": launches,
