@@ -157,12 +157,12 @@ def kernel_bytes(name, st, src, esz):
         "generic_dn_anchor": ta * H * I * esz + Ra * I * 4 + Ra * H * 4,
         "generic_dn_V": rt * I * esz + Rc * I * 4 + rr * 4,
         "generic_dn_U": rt * H * esz + rr * 4 + Rc * H * 4,
-        # streaming kernels: weights once, activations in, results out
+        # streaming kernels: weights once, activations in, results out (bf16)
         "stream_up_anchor_V": (ta * 2 * I * H + rt * 2 * H) * esz + Ra_c * H * esz
-                              + Ra * 2 * I * 4 + rr * 2 * 2,
-        "stream_up_U": rt * 2 * I * esz + rr * 2 * 2 + Rc * 2 * I * 4,
-        "stream_dn_anchor_V": (ta * H * I + rt * I) * esz + Ra_c * I * 2 + Ra * H * 4 + rr * 2,
-        "stream_dn_U": rt * H * esz + rr * 2 + Rc * H * 4,
+                              + Ra * 2 * I * 2 + rr * 2 * 2,
+        "stream_up_U": rt * 2 * I * esz + rr * 2 * 2 + Rc * 2 * I * 2,
+        "stream_dn_anchor_V": (ta * H * I + rt * I) * esz + Ra_c * I * 2 + Ra * H * 2 + rr * 2,
+        "stream_dn_U": rt * H * esz + rr * 2 + Rc * H * 2,
     }
     return table.get(name)
 
@@ -408,7 +408,6 @@ def run_lx(args, rank, world, local_rank):
                 "peak_source": f"{peak_kind} bf16_tflops (burst)"}
     sb = [step_bytes(stats[i % n_batches], src, esz)["bytes"] for i in range(args.steps)]
     step_gbs = sum(sb) / (ms * 1e-3) / 1e9
-    tokens = T * args.steps * world
     amort = np.mean([st["T"] * st["k"] / max(1, st["R_anchor"]) for st in stats])
     line = {
         "metric": METRIC, "value": round(whole_job_rate(T, args.steps, world, ms), 1),

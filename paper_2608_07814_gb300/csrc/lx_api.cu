@@ -93,14 +93,15 @@ static PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
   return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
 }
 
-// TMA map of a bf16 activation buffer [rows][ld] read as 128-row x 64-column
-// boxes (the tensor-core A operand when its rows are already in node-row order)
-static bool encode_rows_map(CUtensorMap* m, void* base, long rows, long ld) {
+// TMA map of a bf16 activation buffer [rows][ld] read as box_rows x 64-column
+// boxes with the 128-byte swizzle (an A operand whose rows are already in
+// node-row order)
+static bool encode_rows_map(CUtensorMap* m, void* base, long rows, long ld, int box_rows) {
   auto encode = get_encode();
   if (!encode) return false;
   const cuuint64_t dims[2] = {(cuuint64_t)ld, (cuuint64_t)rows};
   const cuuint64_t strides[1] = {(cuuint64_t)ld * 2};
-  const cuuint32_t box[2] = {64, (cuuint32_t)tc_tile_tokens()};
+  const cuuint32_t box[2] = {64, (cuuint32_t)box_rows};
   const cuuint32_t estr[2] = {1, 1};
   return encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, dims, strides, box, estr,
                 CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -155,8 +156,11 @@ static lx_status ensure_workspace(lx_layer* L, int T, int k, cudaStream_t s) {
       {(void**)&w.act_n, sizeof(int) * 2},
       {(void**)&w.sctr, sizeof(int) * N_TILE_COUNTERS},
       {(void**)&w.xmaps, sizeof(CUtensorMap) * 3},
-      {(void**)&w.hsplit, sizeof(float) * (LX_STREAM_MAX_SPLIT - 1) * Rsplit * 2 * L->I},
-      {(void**)&w.ysplit, sizeof(float) * (LX_STREAM_MAX_SPLIT - 1) * Rsplit * L->H},
+      {(void**)&w.smaps, sizeof(CUtensorMap) * 3},
+      {(void**)&w.gmap, sizeof(CUtensorMap)},
+      {(void**)&w.xg, L->stream_ok ? (size_t)2 * Rmax * L->H : 0},
+      {(void**)&w.hsplit, sizeof(float) * LX_STREAM_MAX_SPLIT * Rsplit * 2 * L->I},
+      {(void**)&w.ysplit, sizeof(float) * LX_STREAM_MAX_SPLIT * Rsplit * L->H},
       {(void**)&w.err, 256},
   };
   size_t total = 0;
@@ -186,16 +190,27 @@ static lx_status ensure_workspace(lx_layer* L, int T, int k, cudaStream_t s) {
   w.cap_T = cT;
   w.cap_k = ck;
   w.rows_cap = Rmax;
+  w.hb = reinterpret_cast<__nv_bfloat16*>(w.h);
+  w.yb = reinterpret_cast<__nv_bfloat16*>(w.ypart);
   w.split_rows = Rsplit;
   if (Rsplit == 0) w.hsplit = w.ysplit = nullptr;
   if (L->stream_ok) {
-    CUtensorMap maps[3];
+    CUtensorMap maps[7];
     std::memset(maps, 0, sizeof(maps));
-    const bool okm = encode_rows_map(&maps[0], w.Pb, Rmax, 2 * rmax) &&
-                     encode_rows_map(&maps[1], w.zb, Rmax, L->I) &&
-                     encode_rows_map(&maps[2], w.Qb, Rmax, rmax);
+    const int tb = tc_tile_tokens(), sb = stream_tile_tokens();
+    const bool okm = encode_rows_map(&maps[0], w.Pb, Rmax, 2 * rmax, tb) &&
+                     encode_rows_map(&maps[1], w.zb, Rmax, L->I, tb) &&
+                     encode_rows_map(&maps[2], w.Qb, Rmax, rmax, tb) &&
+                     encode_rows_map(&maps[3], w.Pb, Rmax, 2 * rmax, sb) &&
+                     encode_rows_map(&maps[4], w.zb, Rmax, L->I, sb) &&
+                     encode_rows_map(&maps[5], w.Qb, Rmax, rmax, sb) &&
+                     encode_rows_map(&maps[6], w.xg, Rmax, L->H, tb);
     if (!okm) return fail(LX_ERR_CUDA, "cuTensorMapEncodeTiled(activation maps) failed");
-    e = cudaMemcpyAsync(w.xmaps, maps, sizeof(maps), cudaMemcpyHostToDevice, s);
+    e = cudaMemcpyAsync(w.xmaps, maps, 3 * sizeof(CUtensorMap), cudaMemcpyHostToDevice, s);
+    if (e == cudaSuccess)
+      e = cudaMemcpyAsync(w.smaps, maps + 3, 3 * sizeof(CUtensorMap), cudaMemcpyHostToDevice, s);
+    if (e == cudaSuccess)
+      e = cudaMemcpyAsync(w.gmap, maps + 6, sizeof(CUtensorMap), cudaMemcpyHostToDevice, s);
     if (e == cudaSuccess) e = cudaStreamSynchronize(s);
     if (e != cudaSuccess) return cuda_fail(e, "copy activation maps");
   }
@@ -229,13 +244,15 @@ static lx_status route_and_bucket(lx_layer* L, const void* x, int T, int k, int*
 // Largest batch the weight-streaming (decode) kernels take; beyond it every
 // weight would be re-streamed per 64-token block.
 
-static bool use_stream(const lx_layer* L, int T) {
-  return L->path_mode == LX_PATH_AUTO && L->stream_ok && T <= kStreamMaxT;
+static bool use_stream(const lx_layer* L, int T, int k) {
+  return L->path_mode == LX_PATH_AUTO && L->stream_ok && warp_kernels_fit(L, k) &&
+         T <= kStreamMaxT;
 }
 
 // Larger batches: the tensor-core kernels (same layer requirements).
-static bool use_tc(const lx_layer* L, int T) {
-  return L->path_mode == LX_PATH_AUTO && L->stream_ok && T > kStreamMaxT;
+static bool use_tc(const lx_layer* L, int T, int k) {
+  return L->path_mode == LX_PATH_AUTO && L->stream_ok && warp_kernels_fit(L, k) &&
+         T > kStreamMaxT;
 }
 
 // TMA descriptors of every weight matrix the streaming kernels read: each
@@ -583,9 +600,9 @@ extern "C" lx_status lx_moe_forward(lx_layer* L, const void* x, int32_t T, int32
   LX_TRY(route_and_bucket(L, x, T, k, w.topk_id, w.topk_w, nullptr, s));
   L->last_T = T;
   L->last_k = k;
-  if (use_stream(L, T)) {
+  if (use_stream(L, T, k)) {
     LX_TRY(launch_fast_experts(L, x, T, k, y, s));
-  } else if (use_tc(L, T)) {
+  } else if (use_tc(L, T, k)) {
     LX_TRY(launch_tc_experts(L, x, T, k, y, s));
   } else {
     LX_TRY(launch_generic_experts(L, x, T, k, y, s));

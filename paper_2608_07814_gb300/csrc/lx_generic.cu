@@ -11,6 +11,7 @@
 //   anchor:     ypart[(t,n)] = z Wd^T;   correction: ypart[(t,n)] = (z Vd) Ud^T
 // y_t is the sum of ypart over t's rows in ascending node order.
 #include <algorithm>
+#include <type_traits>
 
 #include "lx_internal.cuh"
 
@@ -329,10 +330,60 @@ __device__ __forceinline__ void warp_token_rows(const int* __restrict__ node_row
   __syncwarp();
 }
 
-template <typename TZ, int D, bool SPLIT>
+// CPL consecutive columns of one row (CPL = 1: one float per lane, for small
+// batches, where every row load of a token can then be in flight at once;
+// CPL = 4: one 16-byte load)
+template <int CPL>
+struct Cols {
+  float v[CPL];
+};
+template <int CPL>
+__device__ __forceinline__ Cols<CPL> ld_cols(const float* p) {
+  Cols<CPL> r;
+  if constexpr (CPL == 4) {
+    const float4 f = __ldg(reinterpret_cast<const float4*>(p));
+    r.v[0] = f.x; r.v[1] = f.y; r.v[2] = f.z; r.v[3] = f.w;
+  } else {
+#pragma unroll
+    for (int i = 0; i < CPL; ++i) r.v[i] = __ldg(p + i);
+  }
+  return r;
+}
+template <int CPL>
+__device__ __forceinline__ Cols<CPL> ld_cols(const __nv_bfloat16* p) {
+  Cols<CPL> r;
+  if constexpr (CPL == 4) {
+    const uint2 u = __ldg(reinterpret_cast<const uint2*>(p));
+    r.v[0] = __uint_as_float(u.x << 16); r.v[1] = __uint_as_float(u.x & 0xFFFF0000u);
+    r.v[2] = __uint_as_float(u.y << 16); r.v[3] = __uint_as_float(u.y & 0xFFFF0000u);
+  } else {
+#pragma unroll
+    for (int i = 0; i < CPL; ++i) r.v[i] = __bfloat162float(p[i]);
+  }
+  return r;
+}
+template <typename T, int CPL>
+__device__ __forceinline__ void st_cols(T* p, const Cols<CPL>& c) {
+  if constexpr (CPL == 4) {
+    store4<T>(p, make_float4(c.v[0], c.v[1], c.v[2], c.v[3]));
+  } else if constexpr (std::is_same<T, float>::value) {
+#pragma unroll
+    for (int i = 0; i < CPL; ++i) p[i] = c.v[i];
+  } else {
+#pragma unroll
+    for (int i = 0; i < CPL; ++i) p[i] = __float2bfloat16_rn(c.v[i]);
+  }
+}
+template <int CPL>
+__device__ __forceinline__ void add_cols(Cols<CPL>& a, const Cols<CPL>& b) {
+#pragma unroll
+  for (int i = 0; i < CPL; ++i) a.v[i] += b.v[i];
+}
+
+template <typename TH, typename TZ, int D, bool SPLIT, int CPL>
 __global__ void __launch_bounds__(WT_WARPS * 32, 2)
 k_swiglu_warp(const float* __restrict__ topk_w, const int* __restrict__ node_row, int T, int k,
-              const float* __restrict__ h, int I, TZ* __restrict__ z, int cols_per_item,
+              const TH* __restrict__ h, int I, TZ* __restrict__ z, int cols_per_item,
               const SplitParts hs) {
   pdl_wait();
   __shared__ WarpRows wrs[WT_WARPS];
@@ -349,57 +400,61 @@ k_swiglu_warp(const float* __restrict__ topk_w, const int* __restrict__ node_row
     if (lane < k) wr.g[lane] = topk_w[(size_t)t * k + lane];
     __syncwarp();
     const int nd = wr.nd;
-    for (int c = c_begin + 4 * lane; c < c_end; c += 128) {
-      float4 act[WT_SLOTS];
+    for (int c = c_begin + CPL * lane; c < c_end; c += 32 * CPL) {
+      Cols<CPL> act[WT_SLOTS];
 #pragma unroll
       for (int sl = 0; sl < WT_SLOTS; ++sl) {
-        act[sl] = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (sl < k) {
-          float4 pg = make_float4(0.f, 0.f, 0.f, 0.f), pu = pg;
 #pragma unroll
-          for (int l = 0; l < D; ++l) {  // path order: anchor first
+        for (int i = 0; i < CPL; ++i) act[sl].v[i] = 0.f;
+        if (sl < k) {
+          Cols<CPL> pg, pu;
+#pragma unroll
+          for (int i = 0; i < CPL; ++i) pg.v[i] = pu.v[i] = 0.f;
+#pragma unroll
+          for (int l = 0; l < D; ++l) {  // path order: the expert's node up to its anchor
             const int r = wr.rows[sl * D + l];
             if (r >= 0) {
-              const float4 a = __ldg(reinterpret_cast<const float4*>(h + (size_t)r * 2 * I + c));
-              const float4 b = __ldg(reinterpret_cast<const float4*>(h + (size_t)r * 2 * I + I + c));
-              pg.x += a.x; pg.y += a.y; pg.z += a.z; pg.w += a.w;
-              pu.x += b.x; pu.y += b.y; pu.z += b.z; pu.w += b.w;
-              if (SPLIT && (l + 1 == D || wr.rows[sl * D + l + 1] < 0)) {  // anchor: split partials
-                for (int sp = 1; sp < hs.splits; ++sp) {
-                  const float* hp = hs.part + (sp - 1) * hs.stride + (size_t)r * 2 * I;
-                  const float4 a2 = __ldg(reinterpret_cast<const float4*>(hp + c));
-                  const float4 b2 = __ldg(reinterpret_cast<const float4*>(hp + I + c));
-                  pg.x += a2.x; pg.y += a2.y; pg.z += a2.z; pg.w += a2.w;
-                  pu.x += b2.x; pu.y += b2.y; pu.z += b2.z; pu.w += b2.w;
+              if (SPLIT && (l + 1 == D || wr.rows[sl * D + l + 1] < 0)) {
+                // anchor row: its split-K partials, in split order
+#pragma unroll
+                for (int sp = 0; sp < LX_STREAM_MAX_SPLIT; ++sp) {
+                  if (sp < hs.splits) {
+                    const float* hp = hs.part + sp * hs.stride + (size_t)r * 2 * I;
+                    add_cols(pg, ld_cols<CPL>(hp + c));
+                    add_cols(pu, ld_cols<CPL>(hp + I + c));
+                  }
                 }
+              } else {
+                add_cols(pg, ld_cols<CPL>(h + (size_t)r * 2 * I + c));
+                add_cols(pu, ld_cols<CPL>(h + (size_t)r * 2 * I + I + c));
               }
             }
           }
           const float g = wr.g[sl];
-          act[sl] = make_float4(g * silu_f(pg.x) * pu.x, g * silu_f(pg.y) * pu.y,
-                                g * silu_f(pg.z) * pu.z, g * silu_f(pg.w) * pu.w);
+#pragma unroll
+          for (int i = 0; i < CPL; ++i) act[sl].v[i] = g * silu_f(pg.v[i]) * pu.v[i];
         }
       }
       for (int d = 0; d < nd; ++d) {
         const unsigned m = wr.dmask[d];
-        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+        Cols<CPL> acc;
 #pragma unroll
-        for (int sl = 0; sl < WT_SLOTS; ++sl) {  // slots ascending
-          if ((m >> sl) & 1u) {
-            acc.x += act[sl].x; acc.y += act[sl].y; acc.z += act[sl].z; acc.w += act[sl].w;
-          }
-        }
-        store4<TZ>(z + (size_t)wr.drow[d] * I + c, acc);
+        for (int i = 0; i < CPL; ++i) acc.v[i] = 0.f;
+#pragma unroll
+        for (int sl = 0; sl < WT_SLOTS; ++sl)  // slots ascending
+          if ((m >> sl) & 1u) add_cols(acc, act[sl]);
+        st_cols<TZ, CPL>(z + (size_t)wr.drow[d] * I + c, acc);
       }
     }
     __syncwarp();
   }
 }
 
-// y[t] = sum of ypart over t's distinct rows in ascending row order
-template <typename TY>
+// y[t] = sum of ypart over t's distinct rows in ascending row order (an
+// anchor row split into K ranges contributes its partials in split order)
+template <typename TP, typename TY, int CPL>
 __global__ void __launch_bounds__(WT_WARPS * 32, 2)
-k_combine_warp(const int* __restrict__ node_row, int k, int D, const float* __restrict__ ypart,
+k_combine_warp(const int* __restrict__ node_row, int k, int D, const TP* __restrict__ ypart,
                int H, TY* __restrict__ y, int T, int cols_per_item, const SplitParts ys) {
   pdl_wait();
   __shared__ WarpRows wrs[WT_WARPS];
@@ -414,34 +469,37 @@ k_combine_warp(const int* __restrict__ node_row, int k, int D, const float* __re
     const int c_end = min(H, c_begin + cols_per_item);
     warp_token_rows(node_row + (size_t)t * kD, kD, D, wr);
     const int nd = wr.nd;
-    for (int c = c_begin + 4 * lane; c < c_end; c += 128) {
-      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-      int q = 0;
-      for (; q + 8 <= nd; q += 8) {
-        float4 v[8];
+    for (int c = c_begin + CPL * lane; c < c_end; c += 32 * CPL) {
+      Cols<CPL> acc;
 #pragma unroll
-        for (int u = 0; u < 8; ++u)
-          v[u] = __ldg(reinterpret_cast<const float4*>(ypart + (size_t)wr.drow[q + u] * H + c));
+      for (int i = 0; i < CPL; ++i) acc.v[i] = 0.f;
+      if (ys.splits > 1) {
+        for (int d = 0; d < nd; ++d) {
+          const size_t ro = (size_t)wr.drow[d] * H + c;
+          if ((wr.anchor_rows >> d) & 1u) {
+            Cols<CPL> v[LX_STREAM_MAX_SPLIT];
 #pragma unroll
-        for (int u = 0; u < 8; ++u) {
-          acc.x += v[u].x; acc.y += v[u].y; acc.z += v[u].z; acc.w += v[u].w;
-        }
-      }
-      for (; q < nd; ++q) {
-        const float4 v = __ldg(reinterpret_cast<const float4*>(ypart + (size_t)wr.drow[q] * H + c));
-        acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
-      }
-      if (ys.splits > 1) {  // anchor rows' split-K partials: rows ascending, then splits
-        for (unsigned b = wr.anchor_rows; b; b &= b - 1) {
-          const int d = __ffs(b) - 1;
-          for (int sp = 1; sp < ys.splits; ++sp) {
-            const float4 v = __ldg(reinterpret_cast<const float4*>(
-                ys.part + (sp - 1) * ys.stride + (size_t)wr.drow[d] * H + c));
-            acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
+            for (int sp = 0; sp < LX_STREAM_MAX_SPLIT; ++sp)
+              if (sp < ys.splits) v[sp] = ld_cols<CPL>(ys.part + sp * ys.stride + ro);
+#pragma unroll
+            for (int sp = 0; sp < LX_STREAM_MAX_SPLIT; ++sp)
+              if (sp < ys.splits) add_cols(acc, v[sp]);
+          } else {
+            add_cols(acc, ld_cols<CPL>(ypart + ro));
           }
         }
+      } else {
+        int q = 0;
+        for (; q + 8 <= nd; q += 8) {
+          Cols<CPL> v[8];
+#pragma unroll
+          for (int u = 0; u < 8; ++u) v[u] = ld_cols<CPL>(ypart + (size_t)wr.drow[q + u] * H + c);
+#pragma unroll
+          for (int u = 0; u < 8; ++u) add_cols(acc, v[u]);
+        }
+        for (; q < nd; ++q) add_cols(acc, ld_cols<CPL>(ypart + (size_t)wr.drow[q] * H + c));
       }
-      store4<TY>(y + (size_t)t * H + c, acc);
+      st_cols<TY, CPL>(y + (size_t)t * H + c, acc);
     }
     __syncwarp();
   }
@@ -454,14 +512,14 @@ bool warp_kernels_fit(const lx_layer* L, int k) {
 }
 
 // Columns per warp work item: whole rows when the batch alone fills the GPU
-// (the distinct-row search then runs once per token), else 128-column blocks
-// so that a small batch still spreads over the SMs.
-static int warp_item_cols(const lx_layer* L, int T, int width) {
+// (the distinct-row search then runs once per token), else blocks of `unit`
+// columns so that a small batch still spreads over the SMs.
+static int warp_item_cols(const lx_layer* L, int T, int width, int unit) {
   const long want = (long)L->num_sms * 4 * WT_WARPS;
-  const int blocks = (width + 127) / 128;
+  const int blocks = (width + unit - 1) / unit;
   int per = blocks;
   while (per > 1 && (long)T * ((blocks + per - 1) / per) < want) per = (per + 1) / 2;
-  return per * 128;
+  return per * unit;
 }
 
 static int warp_grid(const lx_layer* L, int T, int width, int cols) {
@@ -469,74 +527,95 @@ static int warp_grid(const lx_layer* L, int T, int width, int cols) {
   return (int)std::min<long>((items + WT_WARPS - 1) / WT_WARPS, (long)L->num_sms * 4);
 }
 
-template <typename TZ, int D>
-static void launch_swiglu_d(lx_layer* L, int T, int k, TZ* z, cudaStream_t s, const SplitParts& hs,
-                            int grid, int cols) {
-  Workspace& w = L->ws;
-  if (hs.splits > 1)
-    launch_k(L, k_swiglu_warp<TZ, D, true>, grid, WT_WARPS * 32, 0, s, w.topk_w, w.node_row, T, k, w.h,
-                                                              L->I, z, cols, hs);
-  else
-    launch_k(L, k_swiglu_warp<TZ, D, false>, grid, WT_WARPS * 32, 0, s, w.topk_w, w.node_row, T, k, w.h,
-                                                               L->I, z, cols, hs);
+// One float per lane for batches too small to fill the GPU with 128-column items.
+static bool narrow_cols(const lx_layer* L, int T, int width) {
+  return (long)T * ((width + 127) / 128) < (long)L->num_sms * 4 * WT_WARPS;
 }
 
-template <typename TZ>
-static void launch_swiglu_warp(lx_layer* L, int T, int k, TZ* z, cudaStream_t s,
-                               const SplitParts& hs) {
-  const int cols = warp_item_cols(L, T, L->I);
+template <typename TH, typename TZ, int D, int CPL>
+static void launch_swiglu_c(lx_layer* L, int T, int k, const TH* h, TZ* z, cudaStream_t s,
+                            const SplitParts& hs) {
+  Workspace& w = L->ws;
+  const int cols = warp_item_cols(L, T, L->I, 32 * CPL);
   const int grid = warp_grid(L, T, L->I, cols);
+  if (hs.splits > 1)
+    launch_k(L, k_swiglu_warp<TH, TZ, D, true, CPL>, grid, WT_WARPS * 32, 0, s, w.topk_w,
+             w.node_row, T, k, h, L->I, z, cols, hs);
+  else
+    launch_k(L, k_swiglu_warp<TH, TZ, D, false, CPL>, grid, WT_WARPS * 32, 0, s, w.topk_w,
+             w.node_row, T, k, h, L->I, z, cols, hs);
+}
+
+template <typename TH, typename TZ, int D>
+static void launch_swiglu_d(lx_layer* L, int T, int k, const TH* h, TZ* z, cudaStream_t s,
+                            const SplitParts& hs) {
+  if (narrow_cols(L, T, L->I))
+    launch_swiglu_c<TH, TZ, D, 1>(L, T, k, h, z, s, hs);
+  else
+    launch_swiglu_c<TH, TZ, D, 4>(L, T, k, h, z, s, hs);
+}
+
+template <typename TH, typename TZ>
+static void launch_swiglu_warp(lx_layer* L, int T, int k, const TH* h, TZ* z, cudaStream_t s,
+                               const SplitParts& hs) {
   switch (L->max_depth) {
-    case 1: launch_swiglu_d<TZ, 1>(L, T, k, z, s, hs, grid, cols); break;
-    case 2: launch_swiglu_d<TZ, 2>(L, T, k, z, s, hs, grid, cols); break;
-    case 3: launch_swiglu_d<TZ, 3>(L, T, k, z, s, hs, grid, cols); break;
-    default: launch_swiglu_d<TZ, 4>(L, T, k, z, s, hs, grid, cols); break;
+    case 1: launch_swiglu_d<TH, TZ, 1>(L, T, k, h, z, s, hs); break;
+    case 2: launch_swiglu_d<TH, TZ, 2>(L, T, k, h, z, s, hs); break;
+    case 3: launch_swiglu_d<TH, TZ, 3>(L, T, k, h, z, s, hs); break;
+    default: launch_swiglu_d<TH, TZ, 4>(L, T, k, h, z, s, hs); break;
   }
 }
 
-lx_status launch_swiglu(lx_layer* L, int T, int k, void* z, bool z_bf16, cudaStream_t s,
-                        SplitParts hs) {
+// (the combine reads few rows per token: 16-byte columns measured faster at
+// every batch size)
+template <typename TP, typename TY>
+static void launch_combine_warp(lx_layer* L, int T, int k, const TP* ypart, TY* y, cudaStream_t s,
+                                const SplitParts& ys) {
   Workspace& w = L->ws;
-  ProfScope ps(L, s, z_bf16 ? "swiglu" : "generic_swiglu");
+  const int cols = warp_item_cols(L, T, L->H, 128);
+  const int grid = warp_grid(L, T, L->H, cols);
+  launch_k(L, k_combine_warp<TP, TY, 4>, grid, WT_WARPS * 32, 0, s, w.node_row, k, L->max_depth,
+           ypart, L->H, y, T, cols, ys);
+}
+
+lx_status launch_swiglu(lx_layer* L, int T, int k, bool bf16, cudaStream_t s, SplitParts hs) {
+  Workspace& w = L->ws;
+  ProfScope ps(L, s, bf16 ? "swiglu" : "generic_swiglu");
   if (warp_kernels_fit(L, k)) {
-    if (z_bf16)
-      launch_swiglu_warp(L, T, k, static_cast<__nv_bfloat16*>(z), s, hs);
+    if (bf16)
+      launch_swiglu_warp(L, T, k, w.hb, w.zb, s, hs);
     else
-      launch_swiglu_warp(L, T, k, static_cast<float*>(z), s, hs);
+      launch_swiglu_warp(L, T, k, w.h, w.z, s, hs);
     LX_CUDA(cudaGetLastError());
     return LX_OK;
   }
+  // large k or deep paths: the block-per-token form (generic path only)
+  if (bf16 || hs.splits > 1) return fail(LX_ERR_STATE, "bf16 SwiGLU needs k <= 8, k * depth <= 32");
   const int grid = std::min(T, L->num_sms * 8);
   const size_t smem = sizeof(float4) * SW_T * k * L->max_depth;
-  static bool done_b[64] = {}, done_f[64] = {};
-  if (z_bf16) {
-    LX_CUDA(smem_cap_once((const void*)k_swiglu_aggregate<__nv_bfloat16>, 200 * 1024, L->device, done_b));
-    launch_k(L, k_swiglu_aggregate<__nv_bfloat16>, grid, SW_T, smem, s, 
-        w.topk_id, w.topk_w, w.node_row, T, k, L->max_depth, w.h, L->I, (__nv_bfloat16*)z);
-  } else {
-    LX_CUDA(smem_cap_once((const void*)k_swiglu_aggregate<float>, 200 * 1024, L->device, done_f));
-    launch_k(L, k_swiglu_aggregate<float>, grid, SW_T, smem, s, w.topk_id, w.topk_w, w.node_row, T, k,
-                                                       L->max_depth, w.h, L->I, (float*)z);
-  }
+  static bool done_f[64] = {};
+  LX_CUDA(smem_cap_once((const void*)k_swiglu_aggregate<float>, 200 * 1024, L->device, done_f));
+  launch_k(L, k_swiglu_aggregate<float>, grid, SW_T, smem, s, w.topk_id, w.topk_w, w.node_row, T,
+           k, L->max_depth, w.h, L->I, w.z);
   LX_CUDA(cudaGetLastError());
   return LX_OK;
 }
 
-lx_status launch_combine(lx_layer* L, int T, int k, void* y, cudaStream_t s, SplitParts ys) {
+lx_status launch_combine(lx_layer* L, int T, int k, void* y, bool bf16, cudaStream_t s,
+                         SplitParts ys) {
   Workspace& w = L->ws;
   ProfScope ps(L, s, "combine");
   if (warp_kernels_fit(L, k)) {
-    const int cols = warp_item_cols(L, T, L->H);
-    const int g2 = warp_grid(L, T, L->H, cols);
-    if (L->dtype == LX_BF16)
-      launch_k(L, k_combine_warp<__nv_bfloat16>, g2, WT_WARPS * 32, 0, s, 
-          w.node_row, k, L->max_depth, w.ypart, L->H, (__nv_bfloat16*)y, T, cols, ys);
+    if (bf16)
+      launch_combine_warp(L, T, k, L->ws.yb, static_cast<__nv_bfloat16*>(y), s, ys);
+    else if (L->dtype == LX_BF16)
+      launch_combine_warp(L, T, k, L->ws.ypart, static_cast<__nv_bfloat16*>(y), s, ys);
     else
-      launch_k(L, k_combine_warp<float>, g2, WT_WARPS * 32, 0, s, w.node_row, k, L->max_depth, w.ypart,
-                                                          L->H, (float*)y, T, cols, ys);
+      launch_combine_warp(L, T, k, L->ws.ypart, static_cast<float*>(y), s, ys);
     LX_CUDA(cudaGetLastError());
     return LX_OK;
   }
+  if (bf16 || ys.splits > 1) return fail(LX_ERR_STATE, "bf16 combine needs k <= 8, k * depth <= 32");
   const int grid = std::min(T, L->num_sms * 8);
   if (L->dtype == LX_BF16)
     launch_k(L, k_combine<__nv_bfloat16>, grid, 256, 0, s, w.node_row, k, L->max_depth, w.ypart, L->H,
@@ -586,7 +665,7 @@ lx_status generic_impl(lx_layer* L, const void* x, int T, int k, void* y, cudaSt
                            2 * rmax, s, "generic_up_V")));
   LX_TRY((run_gemm<float, TX, OP_UP_U>(L, w.P, 2 * rmax, nullptr,
                               (const void* const*)L->d_w_upU, w.h, 2 * I, s, "generic_up_U")));
-  LX_TRY(launch_swiglu(L, T, k, w.z, false, s));
+  LX_TRY(launch_swiglu(L, T, k, false, s));
   // z-side products
   LX_TRY((run_gemm<float, TX, OP_DN_ANCHOR>(L, w.z, I, nullptr, (const void* const*)L->d_w_dn,
                               w.ypart, H, s, "generic_dn_anchor")));
@@ -594,7 +673,7 @@ lx_status generic_impl(lx_layer* L, const void* x, int T, int k, void* y, cudaSt
                               rmax, s, "generic_dn_V")));
   LX_TRY((run_gemm<float, TX, OP_DN_U>(L, w.Q, rmax, nullptr, (const void* const*)L->d_w_dnU,
                               w.ypart, H, s, "generic_dn_U")));
-  LX_TRY(launch_combine(L, T, k, y, s));
+  LX_TRY(launch_combine(L, T, k, y, false, s));
   return LX_OK;
 }
 

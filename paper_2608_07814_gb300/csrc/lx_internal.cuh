@@ -170,6 +170,7 @@ struct StreamOp {
   const int* node_off;
   const int* gather;         // row -> X row (token ids), or null = identity
   const __nv_bfloat16* X;    // activations, bf16
+  const CUtensorMap* xmap;   // TMA map of X (rows in node-row order) when gather is null
   long ldx;
   void* out;                 // fp32 or bf16
   long ldo;
@@ -177,9 +178,10 @@ struct StreamOp {
   OpShape shape;
   const int* rank;
   int ncol_max;              // column tiles of the widest node of this op
+  int ncb;                   // 64-row column blocks per tile
   int ntb;                   // token blocks (64 tokens) of the largest possible bucket
-  // split-K: K-range s of a tile (kbs 64-wide K blocks) writes fp32 partial s,
-  // partial 0 to `out`, partial s >= 1 to split_out + (s - 1) * split_stride
+  // split-K: K-range s of a tile (kbs 64-wide K blocks) writes fp32 partial s
+  // to split_out + s * split_stride (`out` is not written)
   int nsplit;
   int kbs;
   float* split_out;
@@ -264,7 +266,11 @@ struct Workspace {
   float* z = nullptr;        // [Rmax][I]
   float* Q = nullptr;        // [Rmax][rmax]
   float* ypart = nullptr;    // [Rmax][H]
-  // streaming path intermediates (bf16 operands of the next product)
+  // streaming and tensor-core path intermediates, bf16: pre-activations hb
+  // [Rmax][2I] and down partials yb [Rmax][H] (aliasing h and ypart, which only
+  // the generic path uses), and the operands of the next product
+  __nv_bfloat16* hb = nullptr;
+  __nv_bfloat16* yb = nullptr;
   __nv_bfloat16* Pb = nullptr;  // [Rmax][2 rmax]
   __nv_bfloat16* zb = nullptr;  // [Rmax][I]
   __nv_bfloat16* Qb = nullptr;  // [Rmax][rmax]
@@ -272,8 +278,11 @@ struct Workspace {
   int* act_n = nullptr;         // [2] their counts
   int* sctr = nullptr;          // [N_TILE_COUNTERS] streaming / tensor-core tile counters
   CUtensorMap* xmaps = nullptr; // [3] TMA maps of Pb, zb, Qb (tensor-core A operands)
-  // split-K partials of the anchor products on the streaming path:
-  // [LX_STREAM_MAX_SPLIT - 1][split_rows][2I] and [..][split_rows][H]
+  CUtensorMap* smaps = nullptr; // [3] the same buffers in streaming-tile boxes
+  __nv_bfloat16* xg = nullptr;  // [Rmax][H] token rows in node-row order (tensor-core path)
+  CUtensorMap* gmap = nullptr;  // TMA map of xg (tensor-core A operand boxes)
+  // split-K partials of the anchor products on the streaming path (fp32):
+  // [LX_STREAM_MAX_SPLIT][split_rows][2I] and [..][split_rows][H]
   float* hsplit = nullptr;
   float* ysplit = nullptr;
   long split_rows = 0;
@@ -378,9 +387,9 @@ lx_status launch_router(lx_layer* L, const void* x, int T, int k, float* logits,
 lx_status launch_bucket(lx_layer* L, const int* topk_id, int T, int k, cudaStream_t s);
 lx_status launch_generic_experts(lx_layer* L, const void* x, int T, int k, void* y,
                                  cudaStream_t s);
-// Anchor split-K partials the SwiGLU / combine kernels add to the anchor rows
-// (the last node of each expert's path): partial s >= 1 of row r at
-// part + (s - 1) * stride + r * width.
+// Anchor split-K partials the SwiGLU / combine kernels read for the anchor rows
+// (the last node of each expert's path) in place of h / ypart: partial s of
+// row r at part + s * stride + r * width, summed in split order.
 struct SplitParts {
   const float* part = nullptr;
   int splits = 1;
@@ -388,9 +397,11 @@ struct SplitParts {
 };
 constexpr int LX_STREAM_MAX_SPLIT = 4;
 bool warp_kernels_fit(const lx_layer* L, int k);
-lx_status launch_swiglu(lx_layer* L, int T, int k, void* z, bool z_bf16, cudaStream_t s,
+// bf16 = true: the streaming / tensor-core form (h = hb, z = zb, ypart = yb,
+// all bf16); false: the generic form (fp32 h, z, ypart)
+lx_status launch_swiglu(lx_layer* L, int T, int k, bool bf16, cudaStream_t s,
                         SplitParts hs = SplitParts());
-lx_status launch_combine(lx_layer* L, int T, int k, void* y, cudaStream_t s,
+lx_status launch_combine(lx_layer* L, int T, int k, void* y, bool bf16, cudaStream_t s,
                          SplitParts ys = SplitParts());
 lx_status launch_fast_experts(lx_layer* L, const void* x, int T, int k, void* y, cudaStream_t s);
 lx_status launch_tc_experts(lx_layer* L, const void* x, int T, int k, void* y, cudaStream_t s);

@@ -14,10 +14,11 @@
 //     4-stage shared-memory ring guarded by mbarriers;
 //   * two consumer warps (32 weight rows each) multiply with mma.sync
 //     m16n8k16 (weights as the 16-row operand, tokens as the 8-column
-//     operand).  Inside each 32-wide K chunk the contraction index is
+//     operand).  Inside each 64-wide K box the contraction index is
 //     permuted so that every lane reads 8 consecutive K values of a weight
-//     row (one 16-byte shared load) and of a token row (one 16-byte global
-//     load); the same permutation on both operands leaves the sum unchanged;
+//     row and of a token row (16-byte shared loads, conflict-free under the
+//     128-byte swizzle); the same permutation on both operands leaves the sum
+//     unchanged;
 //   * persistent CTAs walk a device-built tile list; every mbarrier wait is
 //     bounded, and a wait that gives up records LX_ERR_TIMEOUT in a device
 //     word and drains the CTA's copies in flight before returning.
@@ -35,15 +36,19 @@ namespace {
 constexpr int SW_ROWS = 64;         // weight rows per tile
 // Tokens per tile.  Decode buckets are small (at 64 tokens top-8 over 32
 // clusters the median anchor bucket holds a handful of tokens), so a 32-token
-// slot keeps the stage at 13 KiB and four CTAs of four stages fit an SM:
-// 128 KiB of weights in flight per SM.  Larger buckets take several token blocks.
+// slot keeps the stage at 12 KiB and five CTAs of three stages fit an SM (more
+// CTAs streaming measured faster than fewer CTAs with deeper rings).  Larger
+// buckets take several token blocks.
 constexpr int SW_TOK = 32;
 constexpr int SW_BOX = 64;          // K per stage = one TMA box of 64 K x 64 rows
 constexpr int SW_BOX_BYTES = SW_BOX * SW_ROWS * 2;
-constexpr int SW_XROW = SW_BOX * 2 + 16;           // padded token row in shared memory
-constexpr int SW_STAGE_BYTES = (SW_BOX_BYTES + SW_TOK * SW_XROW + 1023) / 1024 * 1024;
-constexpr int SW_STAGES = 4;
-constexpr int SW_CTAS_PER_SM = 4;
+// Token rows of a stage: SW_TOK rows x 128 bytes in the 128-byte swizzle (the
+// layout a TMA box of contiguous rows lands in; gathered rows are written in
+// the same layout by cp.async).
+constexpr int SW_XBYTES = SW_TOK * SW_BOX * 2;
+constexpr int SW_STAGE_BYTES = SW_BOX_BYTES + SW_XBYTES;
+constexpr int SW_STAGES = 3;
+constexpr int SW_CTAS_PER_SM = 5;
 constexpr int SW_CONSUMERS = 2;
 constexpr int SW_MT = SW_ROWS / (16 * SW_CONSUMERS);  // 16-row MMA tiles per consumer warp
 constexpr int SW_THREADS = 32 * (1 + SW_CONSUMERS);
@@ -112,6 +117,15 @@ __device__ __forceinline__ void tma_load_tile(uint32_t dst, const CUtensorMap* m
       : "memory");
 }
 
+// SW_TOK contiguous rows x 64 columns of a bf16 activation buffer (2-D map)
+__device__ __forceinline__ void tma_load_rows(uint32_t dst, const CUtensorMap* map, int col,
+                                              int row, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(col), "r"(row), "r"(bar)
+      : "memory");
+}
 // 16-byte asynchronous copy global -> shared on the load/store path (cp.async);
 // the TMA unit is kept for the weight boxes, whose requests it serialises.
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
@@ -177,12 +191,12 @@ __device__ __forceinline__ void decode_tile(const StreamLaunch& P, int tile, int
   ti.op = o;
   ti.node = n;
   ti.grp = grp;
-  ti.row0 = ct * SW_ROWS;
+  ti.row0 = ct * SW_ROWS * op.ncb;
   ti.Ng = op.shape.n_const + op.shape.n_rank * r;
   ti.K = op.shape.k_const + op.shape.k_rank * r;
   ti.tok0 = b0 + tb * SW_TOK;
   ti.M = min(SW_TOK, b1 - ti.tok0);
-  ti.ncb = 1;
+  ti.ncb = min(op.ncb, (ti.Ng - ti.row0 + SW_ROWS - 1) / SW_ROWS);
   const int nkb_all = (ti.K + SW_BOX - 1) / SW_BOX;
   ti.split = split;
   ti.kb0 = split * op.kbs;
@@ -199,9 +213,8 @@ __device__ __forceinline__ bool consume_tile(const StreamLaunch& P, const TileIn
   const int g = lane >> 2, q = lane & 3;
   const int nkb = ti.nkb;
   const int wrow = cw * 16 * SW_MT + g;  // first of this lane's weight rows in a 64-row block
-  // split 0 (and unsplit tiles) write `out`; split s >= 1 its fp32 partial
-  float* const out_f = ti.split == 0 ? static_cast<float*>(op.out)
-                                     : op.split_out + (ti.split - 1) * op.split_stride;
+  // split-K tiles write their fp32 partial, the others `out`
+  float* const part = op.nsplit > 1 ? op.split_out + ti.split * op.split_stride : nullptr;
   for (int cb = 0; cb < ti.ncb; ++cb) {
     float acc[SW_MT][NT][4];
 #pragma unroll
@@ -217,12 +230,17 @@ __device__ __forceinline__ bool consume_tile(const StreamLaunch& P, const TileIn
       const uint32_t xbox = wbox + SW_BOX_BYTES;
 #pragma unroll
       for (int c = 0; c < 2; ++c) {
+        // Lane q of half c reads the 16-byte K unit u = 2q + c of its rows (the
+        // same unit of the weight and of the token row, so the MMA sum is a
+        // permutation of K), stored at u ^ (r & 7) by the 128-byte swizzle with
+        // r & 7 == g.  Rows g and g + 1 then read units of opposite parity:
+        // the 8 lanes of a shared-memory phase touch 8 distinct bank groups.
+        const uint32_t unit = (((q << 1) | c) ^ g) * 16;
         // token rows 8j+g beyond M hold stale data; they only reach masked columns
         uint4 xv[NT];
 #pragma unroll
         for (int j = 0; j < NT; ++j)
-          xv[j] = lds_v4(xbox + (8 * j + g) * SW_XROW + c * 64 + 16 * q);
-        const uint32_t unit = ((c * 4 + q) ^ g) * 16;  // 128-byte swizzle (row & 7 == g)
+          xv[j] = lds_v4(xbox + (8 * j + g) * 128 + unit);
 #pragma unroll
         for (int i = 0; i < SW_MT; ++i) {
           const uint4 w0 = lds_v4(wbox + (wrow + 16 * i) * 128 + unit);
@@ -248,7 +266,8 @@ __device__ __forceinline__ bool consume_tile(const StreamLaunch& P, const TileIn
           const int m = 8 * j + 2 * q + (c & 1);
           if (wr < ti.Ng && m < ti.M) {
             const size_t o = (size_t)(ti.tok0 + m) * op.ldo + (size_t)ti.grp * ti.Ng + wr;
-            if (op.out_f32) out_f[o] = acc[i][j][c];
+            if (part) part[o] = acc[i][j][c];
+            else if (op.out_f32) static_cast<float*>(op.out)[o] = acc[i][j][c];
             else static_cast<__nv_bfloat16*>(op.out)[o] = __float2bfloat16_rn(acc[i][j][c]);
           }
         }
@@ -292,6 +311,7 @@ k_stream_gemm(const __grid_constant__ StreamLaunch P) {
     // prepared while the current one streams
     auto prepare = [&](const TileInfo& t, int buf) {
       const StreamOp& op = P.op[t.op];
+      if (!op.gather) return;  // contiguous rows come by TMA
       const long acol = (long)t.grp * t.K;
 #pragma unroll
       for (int h = 0; h < (SW_TOK + 31) / 32; ++h) {
@@ -331,7 +351,7 @@ k_stream_gemm(const __grid_constant__ StreamLaunch P) {
               good = mbar_wait(empty0 + 8 * s, ((it / SW_STAGES) & 1) ^ 1, abort_flag) ? 1 : 0;
               if (good) {
                 if (cb == 0 && kb == 0) slot[s] = ti;
-                mbar_expect_tx(full0 + 8 * s, SW_BOX_BYTES);
+                mbar_expect_tx(full0 + 8 * s, SW_BOX_BYTES + (op.gather ? 0 : SW_XBYTES));
               }
             }
             good = __shfl_sync(0xffffffffu, good, 0);
@@ -340,12 +360,22 @@ k_stream_gemm(const __grid_constant__ StreamLaunch P) {
               break;
             }
             const uint32_t wbox = smem_base + s * SW_STAGE_BYTES;
-            if (lane == 0) tma_load_tile(wbox, map, kb0 + kb, rt0 + cb, full0 + 8 * s);
-            // token rows: M rows x 128 bytes as 16-byte pieces over the 32 lanes
-            for (int piece = lane; piece < ti.M * 8; piece += 32) {
-              const int m = piece >> 3, u = piece & 7;
-              cp_async16(wbox + SW_BOX_BYTES + m * SW_XROW + u * 16,
-                         xs[m] + (kb0 + kb) * SW_BOX + u * 8);
+            if (lane == 0) {
+              tma_load_tile(wbox, map, kb0 + kb, rt0 + cb, full0 + 8 * s);
+              // contiguous token rows: one box of SW_TOK rows (rows past the
+              // bucket belong to the next node and are never stored)
+              if (!op.gather)
+                tma_load_rows(wbox + SW_BOX_BYTES, op.xmap,
+                              (int)(ti.grp * ti.K) + (kb0 + kb) * SW_BOX, ti.tok0, full0 + 8 * s);
+            }
+            if (op.gather) {
+              // gathered token rows: M rows x 128 bytes as 16-byte pieces over
+              // the 32 lanes, piece u of row m to 16-byte unit u ^ (m & 7)
+              for (int piece = lane; piece < ti.M * 8; piece += 32) {
+                const int m = piece >> 3, u = piece & 7;
+                cp_async16(wbox + SW_BOX_BYTES + m * 128 + ((u ^ (m & 7)) << 4),
+                           xs[m] + (kb0 + kb) * SW_BOX + u * 8);
+              }
             }
             cp_async_arrive(full0 + 8 * s);
             if (!prepared && cb == 0 && (kb == 1 || kb == nkb - 1)) {
@@ -451,8 +481,11 @@ lx_status launch_stream(lx_layer* L, const StreamLaunch& P, cudaStream_t s, cons
   return LX_OK;
 }
 
+constexpr int kStreamUBlocks = 1;
+
 static StreamOp make_op(lx_layer* L, int op, int T, const __nv_bfloat16* X, long ldx,
-                        const int* gather, void* out, long ldo, bool out_f32) {
+                        const int* gather, const CUtensorMap* xmap, void* out, long ldo,
+                        bool out_f32) {
   StreamOp o;
   o.shape = op_shape(L, op);
   o.tmaps = L->d_tmaps + (size_t)op * L->N;
@@ -463,6 +496,7 @@ static StreamOp make_op(lx_layer* L, int op, int T, const __nv_bfloat16* X, long
   o.node_off = L->ws.key_off;
   o.gather = gather;
   o.X = X;
+  o.xmap = xmap;
   o.ldx = ldx;
   o.out = out;
   o.ldo = ldo;
@@ -471,7 +505,10 @@ static StreamOp make_op(lx_layer* L, int op, int T, const __nv_bfloat16* X, long
   int ng_max = 0;
   for (int n : (o.shape.on_anchors ? L->anchors : L->corrs))
     ng_max = std::max(ng_max, o.shape.n_const + o.shape.n_rank * L->rank[n]);
-  o.ncol_max = (ng_max + SW_ROWS - 1) / SW_ROWS;
+  // short-K factor products (U) take several column blocks per tile, so that
+  // a tile streams more than two stages
+  o.ncb = (op == OP_UP_U || op == OP_DN_U) ? kStreamUBlocks : 1;
+  o.ncol_max = ((ng_max + SW_ROWS - 1) / SW_ROWS + o.ncb - 1) / o.ncb;
   o.ntb = (T + SW_TOK - 1) / SW_TOK;
   o.nsplit = 1;
   o.kbs = 1 << 20;
@@ -521,11 +558,12 @@ lx_status launch_fast_experts(lx_layer* L, const void* x, int T, int k, void* y,
                      (long)T * std::min<long>(L->N, (long)k * L->max_depth) <= w.split_rows;
   // x-side: x V of every correction (whole-K tiles, claimed first), and the
   // shared anchor gate/up in split-K slices
-  StreamOp up_a = make_op(L, OP_UP_ANCHOR, T, xb, H, w.node_tok, w.h, 2 * I, true);
+  StreamOp up_a = make_op(L, OP_UP_ANCHOR, T, xb, H, w.node_tok, nullptr, w.hb, 2 * I, false);
   if (split) split_op(L, up_a, w.hsplit, w.split_rows * 2 * I);
-  const StreamOp up_v = make_op(L, OP_UP_V, T, xb, H, w.node_tok, w.Pb, 2 * rmax, false);
+  const StreamOp up_v = make_op(L, OP_UP_V, T, xb, H, w.node_tok, nullptr, w.Pb, 2 * rmax, false);
   LX_TRY(run_stream(L, 0, up_v, &up_a, s, "stream_up_anchor_V"));
-  LX_TRY(run_stream(L, 1, make_op(L, OP_UP_U, T, w.Pb, 2 * rmax, nullptr, w.h, 2 * I, true),
+  LX_TRY(run_stream(L, 1,
+                    make_op(L, OP_UP_U, T, w.Pb, 2 * rmax, nullptr, w.smaps + 0, w.hb, 2 * I, false),
                     nullptr, s, "stream_up_U"));
   SplitParts hs, ys;
   if (up_a.nsplit > 1) {
@@ -533,21 +571,22 @@ lx_status launch_fast_experts(lx_layer* L, const void* x, int T, int k, void* y,
     hs.splits = up_a.nsplit;
     hs.stride = up_a.split_stride;
   }
-  LX_TRY(launch_swiglu(L, T, k, w.zb, true, s, hs));
+  LX_TRY(launch_swiglu(L, T, k, true, s, hs));
   // z-side: z Vd of every correction first, then the shared anchor down
   // projection in split-K slices
-  StreamOp dn_a = make_op(L, OP_DN_ANCHOR, T, w.zb, I, nullptr, w.ypart, H, true);
+  StreamOp dn_a = make_op(L, OP_DN_ANCHOR, T, w.zb, I, nullptr, w.smaps + 1, w.yb, H, false);
   if (split) split_op(L, dn_a, w.ysplit, w.split_rows * H);
-  const StreamOp dn_v = make_op(L, OP_DN_V, T, w.zb, I, nullptr, w.Qb, rmax, false);
+  const StreamOp dn_v = make_op(L, OP_DN_V, T, w.zb, I, nullptr, w.smaps + 1, w.Qb, rmax, false);
   LX_TRY(run_stream(L, 2, dn_v, &dn_a, s, "stream_dn_anchor_V"));
-  LX_TRY(run_stream(L, 3, make_op(L, OP_DN_U, T, w.Qb, rmax, nullptr, w.ypart, H, true), nullptr,
-                    s, "stream_dn_U"));
+  LX_TRY(run_stream(L, 3,
+                    make_op(L, OP_DN_U, T, w.Qb, rmax, nullptr, w.smaps + 2, w.yb, H, false),
+                    nullptr, s, "stream_dn_U"));
   if (dn_a.nsplit > 1) {
     ys.part = dn_a.split_out;
     ys.splits = dn_a.nsplit;
     ys.stride = dn_a.split_stride;
   }
-  LX_TRY(launch_combine(L, T, k, y, s, ys));
+  LX_TRY(launch_combine(L, T, k, y, true, s, ys));
   return LX_OK;
 }
 

@@ -27,6 +27,7 @@
 #include <cuda.h>
 
 #include <algorithm>
+#include <climits>
 
 #include "lx_internal.cuh"
 
@@ -183,17 +184,30 @@ struct TcTile {
   int node, grp, row0, tok0, M, Ng, K, BN;  // BN < 0: sentinel
 };
 
-// tile index -> (node, token block, group, column block) through the plan prefix
-__device__ __forceinline__ void tc_decode(const TcLaunch& P, int tile, TcTile& t) {
+// Tile index -> (node, token block, group, column block) through the plan
+// prefix, by the whole producer warp: one round of independent loads of the
+// prefix and ballots count the items whose first tile is <= `tile` (the
+// prefix is non-decreasing and starts at 0), instead of a chain of dependent
+// loads of a binary search.
+__device__ __forceinline__ void tc_decode_warp(const TcLaunch& P, int tile, TcTile& t) {
+  const int lane = threadIdx.x & 31;
   const int* to = P.tile_off;
-  int lo = 0, hi = P.n_items;
-  while (hi - lo > 1) {
-    const int mid = (lo + hi) >> 1;
-    if (to[mid] <= tile) lo = mid; else hi = mid;
+  int cnt = 0;
+  for (int i0 = 0; i0 < P.n_items; i0 += 256) {
+    int v[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int i = i0 + lane + 32 * j;
+      v[j] = i < P.n_items ? __ldg(to + i) : INT_MAX;
+    }
+#pragma unroll
+    for (int j = 0; j < 8; ++j) cnt += __popc(__ballot_sync(0xffffffffu, v[j] <= tile));
   }
-  const int n = P.items[lo];
-  const int local = tile - to[lo];
-  const int r = P.rank[n];
+  const int lo = cnt - 1;
+  const int n = __ldg(P.items + lo);
+  const int local = tile - __ldg(to + lo);
+  const int r = __ldg(P.rank + n);
+  const int b0 = __ldg(P.node_off + n), b1 = __ldg(P.node_off + n + 1);
   t.Ng = P.shape.n_const + P.shape.n_rank * r;
   t.K = P.shape.k_const + P.shape.k_rank * r;
   const int ncol = (t.Ng + TC_BN - 1) / TC_BN;
@@ -203,8 +217,18 @@ __device__ __forceinline__ void tc_decode(const TcLaunch& P, int tile, TcTile& t
   t.row0 = (rem % ncol) * TC_BN;
   t.BN = min(TC_BN, t.Ng - t.row0);
   t.node = n;
-  t.tok0 = P.node_off[n] + tb * TC_BM;
-  t.M = min(TC_BM, P.node_off[n + 1] - t.tok0);
+  t.tok0 = b0 + tb * TC_BM;
+  t.M = min(TC_BM, b1 - t.tok0);
+}
+
+// gathered token of row 4 i + r8 of a tile, or -1 past the bucket
+__device__ __forceinline__ void tc_load_trow(const TcLaunch& P, const TcTile& t, int r8,
+                                             int (&tr)[TC_BM / 4]) {
+#pragma unroll
+  for (int i = 0; i < TC_BM / 4; ++i) {
+    const int m = 4 * i + r8;
+    tr[i] = m < t.M ? __ldg(P.gather + t.tok0 + m) : -1;
+  }
 }
 
 __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant__ TcLaunch P) {
@@ -253,28 +277,27 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
   if (warp == 0) {
     // ------------------------------------------------------------ producer
     const int total = P.tile_off[P.n_items];
+    const int r8 = lane >> 3, u = lane & 7;  // gather: row within a group of 4, 16-byte chunk
     int cur = lane == 0 ? atomicAdd(P.ctr, 1) : 0;
     cur = __shfl_sync(0xffffffffu, cur, 0);
     TcTile t;
-    if (cur < total) tc_decode(P, cur, t);
+    int trow[TC_BM / 4];  // token of row 4 i + r8 of the current tile, or -1
+    if (cur < total) {
+      tc_decode_warp(P, cur, t);
+      if (P.gather) tc_load_trow(P, t, r8, trow);
+    }
+    int claim = lane == 0 ? atomicAdd(P.ctr, 1) : 0;  // the next tile, claimed one ahead
     uint32_t it = 0;
     bool ok = true;
-    const int r8 = lane >> 3, u = lane & 7;  // gather: row within a group of 4, 16-byte chunk
     // Gathered stages still in flight (cp.async groups not yet waited for), oldest
     // first, four bits per stage index: up to TC_STAGES - 1 stages of token rows
     // stay in flight before the oldest is published to the MMA issuer.
     uint32_t pq = 0;
     int np = 0;
     while (cur < total && ok) {
-      int nxt = lane == 0 ? atomicAdd(P.ctr, 1) : 0;
-      int trow[TC_BM / 4];  // token of row 4 i + r8 of this tile, or -1
-      if (P.gather) {
-#pragma unroll
-        for (int i = 0; i < TC_BM / 4; ++i) {
-          const int m = 4 * i + r8;
-          trow[i] = m < t.M ? __ldg(P.gather + t.tok0 + m) : -1;
-        }
-      }
+      TcTile tn;
+      int trow_n[TC_BM / 4];
+      int nxt = total;
       const int nkb = (t.K + TC_BK - 1) / TC_BK;
       const int rt0 = (t.grp * t.Ng + t.row0) / 64;  // first 64-row weight tile
       const int nbox = (t.BN + 63) / 64;
@@ -323,10 +346,24 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
         } else {
           mbar_arrive(full0 + 8 * s);
         }
+        if (kb == 0) {
+          // the next tile: decoded (and its token rows looked up) while this
+          // one streams
+          nxt = __shfl_sync(0xffffffffu, claim, 0);
+          if (nxt < total) {
+            tc_decode_warp(P, nxt, tn);
+            if (P.gather) tc_load_trow(P, tn, r8, trow_n);
+          }
+        }
       }
-      nxt = __shfl_sync(0xffffffffu, nxt, 0);
+      if (!ok) break;
       cur = nxt;
-      if (cur < total) tc_decode(P, cur, t);
+      if (cur < total) {
+        t = tn;
+#pragma unroll
+        for (int i = 0; i < TC_BM / 4; ++i) trow[i] = trow_n[i];
+        claim = lane == 0 ? atomicAdd(P.ctr, 1) : 0;
+      }
     }
     if (np > 0) {  // publish what is still in flight
       cp_async_wait<0>();
@@ -524,6 +561,27 @@ static TcLaunch tc_op(lx_layer* L, int op, const __nv_bfloat16* X, long ldx, con
   return P;
 }
 
+namespace {
+
+// xg[r] = x[node_tok[r]] for the rows r < R of this forward (R = the node
+// rows, key_off[N]): one warp per row, 16-byte loads and stores.
+__global__ void __launch_bounds__(256)
+k_gather_rows(const __nv_bfloat16* __restrict__ x, int H, const int* __restrict__ node_tok,
+              const int* __restrict__ rows_total, long rows_cap, __nv_bfloat16* __restrict__ xg) {
+  pdl_wait();
+  const long R = min((long)*rows_total, rows_cap);
+  const int lane = threadIdx.x & 31;
+  const long warps = (long)gridDim.x * (blockDim.x >> 5);
+  const int vec = H / 8;
+  for (long r = (long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); r < R; r += warps) {
+    const uint4* src = reinterpret_cast<const uint4*>(x + (size_t)node_tok[r] * H);
+    uint4* dst = reinterpret_cast<uint4*>(xg + (size_t)r * H);
+    for (int i = lane; i < vec; i += 32) dst[i] = __ldg(src + i);
+  }
+}
+
+}  // namespace
+
 // The prefill forward: every (token, node) product on the tensor cores.
 lx_status launch_tc_experts(lx_layer* L, const void* x, int T, int k, void* y, cudaStream_t s) {
   Workspace& w = L->ws;
@@ -533,19 +591,27 @@ lx_status launch_tc_experts(lx_layer* L, const void* x, int T, int k, void* y, c
     if (P.n_items == 0) return LX_OK;
     return launch_tc(L, P, s, name);
   };
-  LX_TRY(run(tc_op(L, OP_UP_ANCHOR, xb, H, w.node_tok, nullptr, 0, w.h, 2 * I, true, 0),
+  // token rows in node-row order once, so that every A tile below is a TMA box
+  {
+    ProfScope ps(L, s, "gather_rows");
+    launch_k(L, k_gather_rows, L->num_sms * 8, 256, 0, s, xb, (int)H, w.node_tok,
+             w.key_off + L->N, w.rows_cap, w.xg);
+    LX_CUDA(cudaGetLastError());
+  }
+  LX_TRY(run(tc_op(L, OP_UP_ANCHOR, nullptr, 0, nullptr, w.gmap, 0, w.hb, 2 * I, false, 0),
              "tc_up_anchor"));
-  LX_TRY(run(tc_op(L, OP_UP_V, xb, H, w.node_tok, nullptr, 0, w.Pb, 2 * rmax, false, 1), "tc_up_V"));
-  LX_TRY(run(tc_op(L, OP_UP_U, nullptr, 0, nullptr, w.xmaps + 0, 0, w.h, 2 * I, true, 2),
+  LX_TRY(run(tc_op(L, OP_UP_V, nullptr, 0, nullptr, w.gmap, 0, w.Pb, 2 * rmax, false, 1),
+             "tc_up_V"));
+  LX_TRY(run(tc_op(L, OP_UP_U, nullptr, 0, nullptr, w.xmaps + 0, 0, w.hb, 2 * I, false, 2),
              "tc_up_U"));
-  LX_TRY(launch_swiglu(L, T, k, w.zb, true, s));
-  LX_TRY(run(tc_op(L, OP_DN_ANCHOR, nullptr, 0, nullptr, w.xmaps + 1, 0, w.ypart, H, true, 3),
+  LX_TRY(launch_swiglu(L, T, k, true, s));
+  LX_TRY(run(tc_op(L, OP_DN_ANCHOR, nullptr, 0, nullptr, w.xmaps + 1, 0, w.yb, H, false, 3),
              "tc_dn_anchor"));
   LX_TRY(run(tc_op(L, OP_DN_V, nullptr, 0, nullptr, w.xmaps + 1, 0, w.Qb, rmax, false, 4),
              "tc_dn_V"));
-  LX_TRY(run(tc_op(L, OP_DN_U, nullptr, 0, nullptr, w.xmaps + 2, 0, w.ypart, H, true, 5),
+  LX_TRY(run(tc_op(L, OP_DN_U, nullptr, 0, nullptr, w.xmaps + 2, 0, w.yb, H, false, 5),
              "tc_dn_U"));
-  LX_TRY(launch_combine(L, T, k, y, s));
+  LX_TRY(launch_combine(L, T, k, y, true, s));
   return LX_OK;
 }
 
