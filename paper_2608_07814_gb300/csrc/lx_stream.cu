@@ -48,6 +48,10 @@ constexpr int SW_BOX_BYTES = SW_BOX * SW_ROWS * 2;
 constexpr int SW_XBYTES = SW_TOK * SW_BOX * 2;
 constexpr int SW_STAGE_BYTES = SW_BOX_BYTES + SW_XBYTES;
 constexpr int SW_STAGES = 3;
+// bf16 output staging per consumer warp: SW_TOK token rows of its 32 output
+// columns, rows padded to 80 bytes (conflict-free writes and 16-byte reads)
+constexpr int SW_OST = 40;
+constexpr int SW_OST_BYTES = 2 * SW_TOK * SW_OST * 2;
 constexpr int SW_CTAS_PER_SM = 5;
 constexpr int SW_CONSUMERS = 2;
 constexpr int SW_MT = SW_ROWS / (16 * SW_CONSUMERS);  // 16-row MMA tiles per consumer warp
@@ -207,7 +211,8 @@ __device__ __forceinline__ void decode_tile(const StreamLaunch& P, int tile, int
 template <int NT>
 __device__ __forceinline__ bool consume_tile(const StreamLaunch& P, const TileInfo& ti,
                                              uint32_t smem_base, uint32_t full0, uint32_t empty0,
-                                             uint32_t& it, volatile int* abort_flag) {
+                                             uint32_t& it, volatile int* abort_flag,
+                                             __nv_bfloat16* ost) {
   const StreamOp& op = P.op[ti.op];
   const int lane = threadIdx.x & 31, cw = (threadIdx.x >> 5) - 1;
   const int g = lane >> 2, q = lane & 3;
@@ -256,6 +261,33 @@ __device__ __forceinline__ bool consume_tile(const StreamLaunch& P, const TileIn
       if (lane == 0) mbar_arrive_relaxed(empty0 + 8 * s);
     }
     // epilogue: D[weight row][token] -> out[token row][grp*Ng + weight row]
+    if (!part && !op.out_f32) {
+      // bf16: stage the warp's 32 columns x 8 NT tokens, then 16-byte row pieces
+      __nv_bfloat16* st = ost + cw * (SW_TOK * SW_OST);
+#pragma unroll
+      for (int i = 0; i < SW_MT; ++i)
+#pragma unroll
+        for (int j = 0; j < NT; ++j)
+#pragma unroll
+          for (int c = 0; c < 4; ++c)
+            st[(8 * j + 2 * q + (c & 1)) * SW_OST + 16 * i + g + (c >= 2 ? 8 : 0)] =
+                __float2bfloat16_rn(acc[i][j][c]);
+      __syncwarp();
+      const int ch = lane & 3;
+      const int wr0 = ti.row0 + cb * SW_ROWS + cw * 16 * SW_MT + 8 * ch;
+#pragma unroll
+      for (int pss = 0; pss < NT; ++pss) {
+        const int m = 8 * pss + (lane >> 2);
+        if (m < ti.M && wr0 < ti.Ng) {
+          const uint4 v = *reinterpret_cast<const uint4*>(st + m * SW_OST + 8 * ch);
+          *reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(op.out) +
+                                    (size_t)(ti.tok0 + m) * op.ldo + (size_t)ti.grp * ti.Ng +
+                                    wr0) = v;
+        }
+      }
+      __syncwarp();
+      continue;
+    }
 #pragma unroll
     for (int i = 0; i < SW_MT; ++i) {
 #pragma unroll
@@ -277,13 +309,14 @@ __device__ __forceinline__ bool consume_tile(const StreamLaunch& P, const TileIn
   return true;
 }
 
-__global__ void __launch_bounds__(SW_THREADS)
+__global__ void __launch_bounds__(SW_THREADS, SW_CTAS_PER_SM)
 k_stream_gemm(const __grid_constant__ StreamLaunch P) {
   pdl_wait();
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + SW_STAGES * SW_STAGE_BYTES);
+  __nv_bfloat16* ost = reinterpret_cast<__nv_bfloat16*>(smem + SW_STAGES * SW_STAGE_BYTES);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + SW_STAGES * SW_STAGE_BYTES + SW_OST_BYTES);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(bars + 2 * SW_STAGES);
   const __nv_bfloat16** xsrc = reinterpret_cast<const __nv_bfloat16**>(bars + 2 * SW_STAGES + 2);
   TileInfo* slot = reinterpret_cast<TileInfo*>(xsrc + 2 * SW_TOK);  // [SW_STAGES]
@@ -449,11 +482,11 @@ k_stream_gemm(const __grid_constant__ StreamLaunch P) {
     if (ti.op < 0) return;  // sentinel
     const int nt = (ti.M + 7) / 8;
     bool ok;
-    if (nt <= 1) ok = consume_tile<1>(P, ti, smem_base, full0, empty0, it, abort_flag);
-    else if (nt <= 2) ok = consume_tile<2>(P, ti, smem_base, full0, empty0, it, abort_flag);
+    if (nt <= 1) ok = consume_tile<1>(P, ti, smem_base, full0, empty0, it, abort_flag, ost);
+    else if (nt <= 2) ok = consume_tile<2>(P, ti, smem_base, full0, empty0, it, abort_flag, ost);
     else if (SW_TOK <= 32 || nt <= 4)
-      ok = consume_tile<SW_TOK <= 32 ? SW_TOK / 8 : 4>(P, ti, smem_base, full0, empty0, it, abort_flag);
-    else ok = consume_tile<SW_TOK / 8>(P, ti, smem_base, full0, empty0, it, abort_flag);
+      ok = consume_tile<SW_TOK <= 32 ? SW_TOK / 8 : 4>(P, ti, smem_base, full0, empty0, it, abort_flag, ost);
+    else ok = consume_tile<SW_TOK / 8>(P, ti, smem_base, full0, empty0, it, abort_flag, ost);
     if (!ok) {
       if (lane == 0) {
         atomicExch(P.err, LX_ERR_TIMEOUT);
@@ -467,7 +500,7 @@ k_stream_gemm(const __grid_constant__ StreamLaunch P) {
 }  // namespace
 
 int stream_smem_bytes() {
-  return SW_STAGES * SW_STAGE_BYTES + 2 * SW_STAGES * 8 + 16 + 2 * SW_TOK * 8 +
+  return SW_STAGES * SW_STAGE_BYTES + SW_OST_BYTES + 2 * SW_STAGES * 8 + 16 + 2 * SW_TOK * 8 +
          SW_STAGES * (int)sizeof(TileInfo) + 1024;
 }
 

@@ -459,38 +459,65 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
       if (t.BN < 0) break;
       const bool tile_ok = t.tok0 >= 0 && (long)t.grp * t.Ng + t.row0 + t.BN <= P.ldo;
       const long col0 = (long)t.grp * t.Ng + t.row0;
-      for (int c0 = 0; c0 < t.BN; c0 += 32) {
-        float v[32];
-        tc_ld32(tmem + b * TC_ACC_COLS + ((uint32_t)(32 * ew) << 16) + (uint32_t)c0, v);
-        // lane = accumulator row: stage the 32 x 32 block row-major
-        float4* srow = reinterpret_cast<float4*>(stg + lane * TC_EPI_LD);
+      const int cq = lane & 7;
+      if (P.out_f32) {
+        for (int c0 = 0; c0 < t.BN; c0 += 32) {
+          float v[32];
+          tc_ld32(tmem + b * TC_ACC_COLS + ((uint32_t)(32 * ew) << 16) + (uint32_t)c0, v);
+          // lane = accumulator row: stage the 32 x 32 block row-major
+          float4* srow = reinterpret_cast<float4*>(stg + lane * TC_EPI_LD);
 #pragma unroll
-        for (int q = 0; q < 8; ++q)
-          srow[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-        __syncwarp();
-        // eight lanes per row, four rows per pass: whole 128-byte (f32) segments
-        const int cq = lane & 7;
+          for (int q = 0; q < 8; ++q)
+            srow[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+          __syncwarp();
+          // eight lanes per row, four rows per pass: whole 128-byte segments
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          const int rr = 4 * j + (lane >> 3);
-          const int m = 32 * ew + rr;
-          const long grow = (long)t.tok0 + m;
-          if (tile_ok && m < t.M && grow < P.rows_cap) {
-            const float4 f = *reinterpret_cast<const float4*>(stg + rr * TC_EPI_LD + 4 * cq);
-            const size_t o = (size_t)grow * P.ldo + col0 + c0 + 4 * cq;
-            if (P.out_f32) {
-              *reinterpret_cast<float4*>(static_cast<float*>(P.out) + o) = f;
-            } else {
-              __nv_bfloat162 lo = __floats2bfloat162_rn(f.x, f.y);
-              __nv_bfloat162 hi = __floats2bfloat162_rn(f.z, f.w);
-              uint2 pk;
-              pk.x = *reinterpret_cast<uint32_t*>(&lo);
-              pk.y = *reinterpret_cast<uint32_t*>(&hi);
-              *reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(P.out) + o) = pk;
+          for (int j = 0; j < 8; ++j) {
+            const int rr = 4 * j + (lane >> 3);
+            const int m = 32 * ew + rr;
+            const long grow = (long)t.tok0 + m;
+            if (tile_ok && m < t.M && grow < P.rows_cap) {
+              const float4 f = *reinterpret_cast<const float4*>(stg + rr * TC_EPI_LD + 4 * cq);
+              *reinterpret_cast<float4*>(static_cast<float*>(P.out) + (size_t)grow * P.ldo +
+                                         col0 + c0 + 4 * cq) = f;
             }
           }
+          __syncwarp();
         }
-        __syncwarp();
+      } else {
+        // bf16: 64 columns per pass, converted before staging, so that a row
+        // segment is again 128 bytes
+        for (int c0 = 0; c0 < t.BN; c0 += 64) {
+          uint32_t pk[32];
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            float v[32];
+            tc_ld32(tmem + b * TC_ACC_COLS + ((uint32_t)(32 * ew) << 16) + (uint32_t)(c0 + 32 * h),
+                    v);
+#pragma unroll
+            for (int e = 0; e < 16; ++e) {
+              __nv_bfloat162 b2 = __floats2bfloat162_rn(v[2 * e], v[2 * e + 1]);
+              pk[16 * h + e] = *reinterpret_cast<uint32_t*>(&b2);
+            }
+          }
+          uint4* srow = reinterpret_cast<uint4*>(stg + lane * TC_EPI_LD);
+#pragma unroll
+          for (int q = 0; q < 8; ++q)
+            srow[q] = make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
+          __syncwarp();
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const int rr = 4 * j + (lane >> 3);
+            const int m = 32 * ew + rr;
+            const long grow = (long)t.tok0 + m;
+            if (tile_ok && m < t.M && grow < P.rows_cap) {
+              const uint4 u4 = *reinterpret_cast<const uint4*>(stg + rr * TC_EPI_LD + 4 * cq);
+              *reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(P.out) + (size_t)grow * P.ldo +
+                                        col0 + c0 + 8 * cq) = u4;
+            }
+          }
+          __syncwarp();
+        }
       }
       tc_fence_before();
       __syncwarp();
