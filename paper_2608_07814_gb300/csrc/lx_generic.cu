@@ -362,6 +362,34 @@ __device__ __forceinline__ Cols<CPL> ld_cols(const __nv_bfloat16* p) {
   }
   return r;
 }
+// CPL raw bf16 values (CPL = 4: one 8-byte load) and their widening
+template <int CPL>
+struct RawB {
+  uint32_t w[(CPL + 1) / 2];
+};
+template <int CPL>
+__device__ __forceinline__ RawB<CPL> ld_raw(const __nv_bfloat16* p) {
+  RawB<CPL> r;
+  if constexpr (CPL == 4) {
+    const uint2 u = __ldg(reinterpret_cast<const uint2*>(p));
+    r.w[0] = u.x;
+    r.w[1] = u.y;
+  } else {
+    r.w[0] = (uint32_t)__ldg(reinterpret_cast<const unsigned short*>(p));
+  }
+  return r;
+}
+template <int CPL>
+__device__ __forceinline__ void add_raw(Cols<CPL>& a, const RawB<CPL>& r, bool valid) {
+  if constexpr (CPL == 4) {
+    if (valid) {
+      a.v[0] += __uint_as_float(r.w[0] << 16); a.v[1] += __uint_as_float(r.w[0] & 0xFFFF0000u);
+      a.v[2] += __uint_as_float(r.w[1] << 16); a.v[3] += __uint_as_float(r.w[1] & 0xFFFF0000u);
+    }
+  } else {
+    if (valid) a.v[0] += __uint_as_float(r.w[0] << 16);
+  }
+}
 template <typename T, int CPL>
 __device__ __forceinline__ void st_cols(T* p, const Cols<CPL>& c) {
   if constexpr (CPL == 4) {
@@ -402,6 +430,64 @@ k_swiglu_warp(const float* __restrict__ topk_w, const int* __restrict__ node_row
     const int nd = wr.nd;
     for (int c = c_begin + CPL * lane; c < c_end; c += 32 * CPL) {
       Cols<CPL> act[WT_SLOTS];
+      if constexpr (sizeof(TH) == 2) {
+        // bf16 rows: every load of this column block first (invalid entries
+        // read row 0 and are masked), so that they are all in flight at once
+        RawB<CPL> rg[WT_SLOTS][D], ru[WT_SLOTS][D];
+        bool val[WT_SLOTS][D], anc[WT_SLOTS][D];
+        constexpr int NS = SPLIT ? LX_STREAM_MAX_SPLIT : 1;
+        Cols<CPL> sg[WT_SLOTS][NS], su[WT_SLOTS][NS];  // the anchor row's split-K partials
+#pragma unroll
+        for (int sl = 0; sl < WT_SLOTS; ++sl) {
+          int ra = 0;
+#pragma unroll
+          for (int l = 0; l < D; ++l) {
+            const int r = sl < k ? wr.rows[sl * D + l] : -1;
+            const int rn = (sl < k && l + 1 < D) ? wr.rows[sl * D + l + 1] : -1;
+            val[sl][l] = r >= 0;
+            anc[sl][l] = SPLIT && r >= 0 && rn < 0;  // the path's anchor row
+            if (anc[sl][l]) ra = r;
+            const __nv_bfloat16* hp = reinterpret_cast<const __nv_bfloat16*>(h) +
+                                      (size_t)(r >= 0 ? r : 0) * 2 * I + c;
+            rg[sl][l] = ld_raw<CPL>(hp);
+            ru[sl][l] = ld_raw<CPL>(hp + I);
+          }
+          if constexpr (SPLIT) {
+#pragma unroll
+            for (int sp = 0; sp < NS; ++sp) {
+              const float* hp2 =
+                  hs.part + (long)(sp < hs.splits ? sp : 0) * hs.stride + (size_t)ra * 2 * I + c;
+              sg[sl][sp] = ld_cols<CPL>(hp2);
+              su[sl][sp] = ld_cols<CPL>(hp2 + I);
+            }
+          }
+        }
+#pragma unroll
+        for (int sl = 0; sl < WT_SLOTS; ++sl) {
+          Cols<CPL> pg, pu;
+#pragma unroll
+          for (int i = 0; i < CPL; ++i) pg.v[i] = pu.v[i] = 0.f;
+#pragma unroll
+          for (int l = 0; l < D; ++l) {  // path order: the expert's node up to its anchor
+            if (anc[sl][l]) {
+              // anchor row: its split-K partials (not h), in split order
+#pragma unroll
+              for (int sp = 0; sp < NS; ++sp) {
+                if (sp < hs.splits) {
+                  add_cols(pg, sg[sl][sp]);
+                  add_cols(pu, su[sl][sp]);
+                }
+              }
+            } else {
+              add_raw(pg, rg[sl][l], val[sl][l]);
+              add_raw(pu, ru[sl][l], val[sl][l]);
+            }
+          }
+          const float g = sl < k ? wr.g[sl] : 0.f;
+#pragma unroll
+          for (int i = 0; i < CPL; ++i) act[sl].v[i] = g * silu_f(pg.v[i]) * pu.v[i];
+        }
+      } else {
 #pragma unroll
       for (int sl = 0; sl < WT_SLOTS; ++sl) {
 #pragma unroll
@@ -434,6 +520,7 @@ k_swiglu_warp(const float* __restrict__ topk_w, const int* __restrict__ node_row
 #pragma unroll
           for (int i = 0; i < CPL; ++i) act[sl].v[i] = g * silu_f(pg.v[i]) * pu.v[i];
         }
+      }
       }
       for (int d = 0; d < nd; ++d) {
         const unsigned m = wr.dmask[d];
@@ -538,18 +625,22 @@ static void launch_swiglu_c(lx_layer* L, int T, int k, const TH* h, TZ* z, cudaS
   Workspace& w = L->ws;
   const int cols = warp_item_cols(L, T, L->I, 32 * CPL);
   const int grid = warp_grid(L, T, L->I, cols);
-  if (hs.splits > 1)
-    launch_k(L, k_swiglu_warp<TH, TZ, D, true, CPL>, grid, WT_WARPS * 32, 0, s, w.topk_w,
-             w.node_row, T, k, h, L->I, z, cols, hs);
-  else
-    launch_k(L, k_swiglu_warp<TH, TZ, D, false, CPL>, grid, WT_WARPS * 32, 0, s, w.topk_w,
-             w.node_row, T, k, h, L->I, z, cols, hs);
+  if constexpr (CPL == 1) {
+    if (hs.splits > 1) {
+      launch_k(L, k_swiglu_warp<TH, TZ, D, true, CPL>, grid, WT_WARPS * 32, 0, s, w.topk_w,
+               w.node_row, T, k, h, L->I, z, cols, hs);
+      return;
+    }
+  }
+  launch_k(L, k_swiglu_warp<TH, TZ, D, false, CPL>, grid, WT_WARPS * 32, 0, s, w.topk_w,
+           w.node_row, T, k, h, L->I, z, cols, hs);
 }
 
 template <typename TH, typename TZ, int D>
 static void launch_swiglu_d(lx_layer* L, int T, int k, const TH* h, TZ* z, cudaStream_t s,
                             const SplitParts& hs) {
-  if (narrow_cols(L, T, L->I))
+  // split partials (small batches only) take the one-column-per-lane form
+  if (narrow_cols(L, T, L->I) || hs.splits > 1)
     launch_swiglu_c<TH, TZ, D, 1>(L, T, k, h, z, s, hs);
   else
     launch_swiglu_c<TH, TZ, D, 4>(L, T, k, h, z, s, hs);
