@@ -539,7 +539,7 @@ k_swiglu_warp(const float* __restrict__ topk_w, const int* __restrict__ node_row
 
 // y[t] = sum of ypart over t's distinct rows in ascending row order (an
 // anchor row split into K ranges contributes its partials in split order)
-template <typename TP, typename TY, int CPL>
+template <typename TP, typename TY, int CPL, bool SPLIT>
 __global__ void __launch_bounds__(WT_WARPS * 32, 2)
 k_combine_warp(const int* __restrict__ node_row, int k, int D, const TP* __restrict__ ypart,
                int H, TY* __restrict__ y, int T, int cols_per_item, const SplitParts ys) {
@@ -560,19 +560,37 @@ k_combine_warp(const int* __restrict__ node_row, int k, int D, const TP* __restr
       Cols<CPL> acc;
 #pragma unroll
       for (int i = 0; i < CPL; ++i) acc.v[i] = 0.f;
-      if (ys.splits > 1) {
-        for (int d = 0; d < nd; ++d) {
-          const size_t ro = (size_t)wr.drow[d] * H + c;
-          if ((wr.anchor_rows >> d) & 1u) {
-            Cols<CPL> v[LX_STREAM_MAX_SPLIT];
+      if constexpr (SPLIT) {
+        // four distinct rows per batch, every load of the batch first: an
+        // anchor row contributes its split partials (fp32, split order), any
+        // other row its ypart row
+        constexpr int NS = LX_STREAM_MAX_SPLIT;
+        for (int q0 = 0; q0 < nd; q0 += 4) {
+          Cols<CPL> v[4][NS];
+          bool isa[4];
 #pragma unroll
-            for (int sp = 0; sp < LX_STREAM_MAX_SPLIT; ++sp)
-              if (sp < ys.splits) v[sp] = ld_cols<CPL>(ys.part + sp * ys.stride + ro);
+          for (int u = 0; u < 4; ++u) {
+            const int d = q0 + u < nd ? q0 + u : q0;
+            const size_t ro = (size_t)wr.drow[d] * H + c;
+            isa[u] = q0 + u < nd && ((wr.anchor_rows >> d) & 1u);
+            if (isa[u]) {
 #pragma unroll
-            for (int sp = 0; sp < LX_STREAM_MAX_SPLIT; ++sp)
-              if (sp < ys.splits) add_cols(acc, v[sp]);
-          } else {
-            add_cols(acc, ld_cols<CPL>(ypart + ro));
+              for (int sp = 0; sp < NS; ++sp)
+                v[u][sp] = ld_cols<CPL>(ys.part + (long)(sp < ys.splits ? sp : 0) * ys.stride + ro);
+            } else {
+              v[u][0] = ld_cols<CPL>(ypart + ro);
+            }
+          }
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            if (q0 + u >= nd) break;
+            if (isa[u]) {
+#pragma unroll
+              for (int sp = 0; sp < NS; ++sp)
+                if (sp < ys.splits) add_cols(acc, v[u][sp]);
+            } else {
+              add_cols(acc, v[u][0]);
+            }
           }
         }
       } else {
@@ -665,8 +683,12 @@ static void launch_combine_warp(lx_layer* L, int T, int k, const TP* ypart, TY* 
   Workspace& w = L->ws;
   const int cols = warp_item_cols(L, T, L->H, 128);
   const int grid = warp_grid(L, T, L->H, cols);
-  launch_k(L, k_combine_warp<TP, TY, 4>, grid, WT_WARPS * 32, 0, s, w.node_row, k, L->max_depth,
-           ypart, L->H, y, T, cols, ys);
+  if (ys.splits > 1)
+    launch_k(L, k_combine_warp<TP, TY, 4, true>, grid, WT_WARPS * 32, 0, s, w.node_row, k,
+             L->max_depth, ypart, L->H, y, T, cols, ys);
+  else
+    launch_k(L, k_combine_warp<TP, TY, 4, false>, grid, WT_WARPS * 32, 0, s, w.node_row, k,
+             L->max_depth, ypart, L->H, y, T, cols, ys);
 }
 
 lx_status launch_swiglu(lx_layer* L, int T, int k, bool bf16, cudaStream_t s, SplitParts hs) {
