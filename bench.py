@@ -167,6 +167,20 @@ def kernel_bytes(name, st, src, esz):
     return table.get(name)
 
 
+def fp32_alu_peak_tflops(peaks):
+    """fp32 FMA peak of the GB300: 152 SMs x 128 FP32 lanes x 2 FLOP x the
+    maximum SM clock (MEASURED_PEAKS sm_max_mhz, else 2070 MHz)."""
+    mhz = float(peaks.get("sm_max_mhz", 2070.0))
+    return 152 * 128 * 2 * mhz * 1e6 / 1e12
+
+
+def kernel_alu_flops(name, st, src):
+    """fp32 multiply-add FLOPs of the CUDA-core kernels: the router's logits."""
+    if name == "router":
+        return 2 * st["T"] * src.n_experts * src.d_model
+    return None
+
+
 def kernel_flops(name, st, src):
     """Dense multiply-add FLOPs per launch of a tensor-core kernel: 2 x (rows of
     each node's bucket) x (its output columns) x (its K), over real rows only."""
@@ -336,7 +350,7 @@ def run_lx(args, rank, world, local_rank):
     per_copy = [L.read_profile(cap=1 << 20) for L in layers]
     totals, counts = {}, {}
     launches = 0
-    kbytes, kflops = {}, {}
+    kbytes, kflops, kalu = {}, {}, {}
     for c, recs in enumerate(per_copy):
         steps_of_copy = [i for i in range(args.steps) if i % n_copies == c]
         per_step = len(recs) // max(1, len(steps_of_copy))
@@ -352,6 +366,9 @@ def run_lx(args, rank, world, local_rank):
             f = kernel_flops(name, stats[step_i % n_batches], src)
             if f is not None:
                 kflops[name] = kflops.get(name, 0.0) + f
+            a = kernel_alu_flops(name, stats[step_i % n_batches], src)
+            if a is not None:
+                kalu[name] = kalu.get(name, 0.0) + a
 
     # e2e: host buffers, copies inside the timed region, a read of every result
     xh = [lx.host_to_torch(x, src.dtype).pin_memory() for x in xs_host]
@@ -389,7 +406,16 @@ def run_lx(args, rank, world, local_rank):
     dom = max(totals, key=totals.get)
     avg_ms = totals[dom] / counts[dom]
     roof = None
-    if dom in kbytes:
+    if dom in kalu and src.dtype == "bf16" and T > 256:
+        # the large-batch router: fp32 FMAs on the CUDA cores
+        alu = fp32_alu_peak_tflops(peaks)
+        fl = kalu[dom] / counts[dom]
+        ach = fl / (avg_ms * 1e-3) / 1e12
+        roof = {"kernel": dom, "bound": "alu", "achieved": round(ach, 2), "peak": round(alu, 1),
+                "unit": "TFLOP/s", "frac": round(ach / alu, 4), "traffic": traffic_for(dom, args.workload),
+                "algorithmic_flops_per_launch": round(fl), "avg_launch_us": round(avg_ms * 1e3, 2),
+                "peak_source": "derived fp32 FMA peak (152 SMs x 128 lanes x 2 x max SM clock)"}
+    elif dom in kbytes:
         bytes_per_launch = kbytes[dom] / counts[dom]
         ach = bytes_per_launch / (avg_ms * 1e-3) / 1e9
         roof = {"kernel": dom, "bound": "hbm", "achieved": round(ach, 1), "peak": hbm,
@@ -406,6 +432,18 @@ def run_lx(args, rank, world, local_rank):
                 "algorithmic_flops_per_launch": round(flops_per_launch),
                 "avg_launch_us": round(avg_ms * 1e3, 2),
                 "peak_source": f"{peak_kind} bf16_tflops (burst)"}
+    def kernel_frac(n):
+        """this kernel's own roofline fraction (streaming: HBM, tensor-core:
+        bf16 burst, large-batch router: fp32 ALU), from its event times"""
+        t = totals[n] / counts[n] * 1e-3
+        if n in kflops:
+            return {"frac_bf16": round(kflops[n] / counts[n] / t / 1e12 / float(peaks["bf16_tflops"]), 4)}
+        if n in kalu and src.dtype == "bf16" and T > 256:
+            return {"frac_alu": round(kalu[n] / counts[n] / t / 1e12 / fp32_alu_peak_tflops(peaks), 4)}
+        if n in kbytes:
+            return {"frac_hbm": round(kbytes[n] / counts[n] / t / 1e9 / hbm, 4)}
+        return {}
+
     sb = [step_bytes(stats[i % n_batches], src, esz)["bytes"] for i in range(args.steps)]
     step_gbs = sum(sb) / (ms * 1e-3) / 1e9
     amort = np.mean([st["T"] * st["k"] / max(1, st["R_anchor"]) for st in stats])
@@ -427,7 +465,8 @@ def run_lx(args, rank, world, local_rank):
                              if graph is not None else "K forwards launched one by one"},
         "roofline": roof,
         "kernels": {n: {"launches": counts[n], "avg_us": round(totals[n] / counts[n] * 1e3, 2),
-                        "share": round(totals[n] / sum(totals.values()), 4)} for n in totals},
+                        "share": round(totals[n] / sum(totals.values()), 4),
+                        **kernel_frac(n)} for n in totals},
         "step_roofline": {"algorithmic_bytes_per_step": round(float(np.mean(sb))),
                           "achieved_gbs": round(step_gbs, 1), "frac": round(step_gbs / hbm, 4)},
         "amortisation": round(float(amort), 3),

@@ -227,17 +227,19 @@ static lx_status check_call(lx_layer* L, int T, int k) {
   return LX_OK;
 }
 
-static lx_status bucket_ids(lx_layer* L, const int* ids, int T, int k, cudaStream_t s) {
-  if (bucket_small_fits(L, T, k)) return launch_bucket_small(L, nullptr, ids, T, k, nullptr, nullptr, s);
+static lx_status bucket_ids(lx_layer* L, const int* ids, int T, int k, cudaStream_t s,
+                            bool plans) {
+  if (bucket_small_fits(L, T, k))
+    return launch_bucket_small(L, nullptr, ids, T, k, nullptr, nullptr, s, plans);
   return launch_bucket(L, ids, T, k, s);
 }
 
 // Logits, top-k and bucketing of T tokens (single-CTA bucketing for small T).
 static lx_status route_and_bucket(lx_layer* L, const void* x, int T, int k, int* ids, float* w,
-                                  float* logits_user, cudaStream_t s) {
+                                  float* logits_user, cudaStream_t s, bool plans) {
   float* logits = logits_user ? logits_user : L->ws.logits;
   LX_TRY(launch_router(L, x, T, k, logits, ids, w, s));
-  return bucket_ids(L, ids, T, k, s);
+  return bucket_ids(L, ids, T, k, s, plans);
 }
 
 
@@ -569,7 +571,7 @@ extern "C" lx_status lx_route(lx_layer* L, const void* x, int32_t T, int32_t k, 
   if (!x || !topk_id || !topk_w) return fail(LX_ERR_ARG, "NULL x/topk_id/topk_w");
   cudaStream_t s = (cudaStream_t)stream;
   LX_TRY(ensure_workspace(L, T, k, s));
-  LX_TRY(route_and_bucket(L, x, T, k, topk_id, topk_w, logits, s));
+  LX_TRY(route_and_bucket(L, x, T, k, topk_id, topk_w, logits, s, false));
   L->last_T = T;
   L->last_k = k;
   return LX_OK;
@@ -582,7 +584,7 @@ extern "C" lx_status lx_bucket(lx_layer* L, const int32_t* topk_id, int32_t T, i
   if (!topk_id) return fail(LX_ERR_ARG, "NULL topk_id");
   cudaStream_t s = (cudaStream_t)stream;
   LX_TRY(ensure_workspace(L, T, k, s));
-  LX_TRY(bucket_ids(L, topk_id, T, k, s));
+  LX_TRY(bucket_ids(L, topk_id, T, k, s, false));
   L->last_T = T;
   L->last_k = k;
   return LX_OK;
@@ -597,7 +599,8 @@ extern "C" lx_status lx_moe_forward(lx_layer* L, const void* x, int32_t T, int32
   cudaStream_t s = (cudaStream_t)stream;
   LX_TRY(ensure_workspace(L, T, k, s));
   Workspace& w = L->ws;
-  LX_TRY(route_and_bucket(L, x, T, k, w.topk_id, w.topk_w, nullptr, s));
+  // the generic GEMMs read the tile plans; the streaming kernels do not
+  LX_TRY(route_and_bucket(L, x, T, k, w.topk_id, w.topk_w, nullptr, s, !use_stream(L, T, k)));
   L->last_T = T;
   L->last_k = k;
   if (use_stream(L, T, k)) {

@@ -265,12 +265,20 @@ k_bucket_small(const float* __restrict__ logits, const int* __restrict__ ids_in,
   int* srank = splen + E;                       // [N]
   const int tid = threadIdx.x, nth = blockDim.x;
   const int warp = tid >> 5, lane = tid & 31, nw = nth >> 5;
-  for (int i = tid; i < E * LX_MAX_DEPTH; i += nth) spaths[i] = paths[i];
-  for (int i = tid; i < E; i += nth) splen[i] = path_len[i];
-  for (int i = tid; i < N; i += nth) srank[i] = rank[i];
   {
     uint32_t* m32 = reinterpret_cast<uint32_t*>(marks);  // keys*Tp is a multiple of 16
     for (int i = tid; i < keys * Tp / 4; i += nth) m32[i] = 0;
+  }
+  // the layer's tables and the given ids in one pass (one round trip)
+  {
+    const int n_paths = E * LX_MAX_DEPTH, n_tab = n_paths + E + N;
+    const int n_all = n_tab + (logits ? 0 : T * k);
+    for (int i = tid; i < n_all; i += nth) {
+      if (i < n_paths) spaths[i] = paths[i];
+      else if (i < n_paths + E) splen[i - n_paths] = path_len[i - n_paths];
+      else if (i < n_tab) srank[i - n_paths - E] = rank[i - n_paths - E];
+      else ids[i - n_tab] = ids_in[i - n_tab];
+    }
   }
   // 1. routing (or the given ids)
   if (logits) {
@@ -284,8 +292,6 @@ k_bucket_small(const float* __restrict__ logits, const int* __restrict__ ids_in,
         topk_w[(size_t)t * k + lane] = w;
       }
     }
-  } else {
-    for (int i = tid; i < T * k; i += nth) ids[i] = ids_in[i];
   }
   __syncthreads();
   // 2. marks
@@ -392,10 +398,10 @@ bool bucket_small_fits(const lx_layer* L, int T, int k) {
 }
 
 lx_status launch_bucket_small(lx_layer* L, const float* logits, const int* ids_in, int T, int k,
-                              int* topk_id, float* topk_w, cudaStream_t s) {
+                              int* topk_id, float* topk_w, cudaStream_t s, bool plans) {
   Workspace& w = L->ws;
   const size_t smem = sb_smem(T, k, L->N + L->E, L->E, L->N, op_max_items(L));
-  const PlanArgs pa = make_plans(L, N_OPS);
+  const PlanArgs pa = make_plans(L, plans ? N_OPS : 0);
   static bool done[64] = {};
   LX_CUDA(smem_cap_once((const void*)k_bucket_small, (int)SB_SMEM_LIMIT, L->device, done));
   ProfScope ps(L, s, logits ? "topk_bucket_small" : "bucket_small");

@@ -409,8 +409,10 @@ int tc_tile_tokens();
 int tc_tile_cols();
 lx_status launch_tc(lx_layer* L, const TcLaunch& P, cudaStream_t s, const char* name);
 lx_status launch_stream(lx_layer* L, const StreamLaunch& P, cudaStream_t s, const char* name);
+// plans = false: skip the generic GEMMs' tile plans (not read by the
+// streaming kernels or by lx_get_buckets)
 lx_status launch_bucket_small(lx_layer* L, const float* logits, const int* ids_in, int T, int k,
-                              int* topk_id, float* topk_w, cudaStream_t s);
+                              int* topk_id, float* topk_w, cudaStream_t s, bool plans = true);
 bool bucket_small_fits(const lx_layer* L, int T, int k);
 int stream_tile_rows();
 int stream_tile_tokens();

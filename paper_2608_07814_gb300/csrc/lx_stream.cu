@@ -551,14 +551,18 @@ static StreamOp make_op(lx_layer* L, int op, int T, const __nv_bfloat16* X, long
 }
 
 // Split the anchor op's K into at most LX_STREAM_MAX_SPLIT ranges of about
-// kStreamSplitBlocks 64-wide blocks (a 64 KB weight slice per tile), so that
-// the last tiles of a launch are short.  Partials go to `part`.
-constexpr int kStreamSplitBlocks = 8;
-static void split_op(lx_layer* L, StreamOp& o, float* part, long stride) {
+// `blocks` 64-wide blocks, so that the last tiles of a launch are short.
+// Partials go to `part`.  Measured on GB300 at a decode batch of 64: the
+// gate/up side (K = H) gains with 8-block (64 KB) ranges; the down side
+// (K = I) is faster unsplit up to 16 blocks, where the partials' extra traffic
+// outweighs the shorter tail.
+constexpr int kStreamSplitBlocksUp = 8;
+constexpr int kStreamSplitBlocksDown = 16;
+static void split_op(lx_layer* L, StreamOp& o, float* part, long stride, int blocks) {
   if (!part) return;
   const int K = o.shape.k_const;  // anchors: K does not depend on a rank
   const int nkb = (K + SW_BOX - 1) / SW_BOX;
-  int ns = std::min(LX_STREAM_MAX_SPLIT, (nkb + kStreamSplitBlocks - 1) / kStreamSplitBlocks);
+  int ns = std::min(LX_STREAM_MAX_SPLIT, (nkb + blocks - 1) / blocks);
   if (ns <= 1) return;
   o.kbs = (nkb + ns - 1) / ns;
   o.nsplit = (nkb + o.kbs - 1) / o.kbs;
@@ -592,7 +596,7 @@ lx_status launch_fast_experts(lx_layer* L, const void* x, int T, int k, void* y,
   // x-side: x V of every correction (whole-K tiles, claimed first), and the
   // shared anchor gate/up in split-K slices
   StreamOp up_a = make_op(L, OP_UP_ANCHOR, T, xb, H, w.node_tok, nullptr, w.hb, 2 * I, false);
-  if (split) split_op(L, up_a, w.hsplit, w.split_rows * 2 * I);
+  if (split) split_op(L, up_a, w.hsplit, w.split_rows * 2 * I, kStreamSplitBlocksUp);
   const StreamOp up_v = make_op(L, OP_UP_V, T, xb, H, w.node_tok, nullptr, w.Pb, 2 * rmax, false);
   LX_TRY(run_stream(L, 0, up_v, &up_a, s, "stream_up_anchor_V"));
   LX_TRY(run_stream(L, 1,
@@ -608,7 +612,7 @@ lx_status launch_fast_experts(lx_layer* L, const void* x, int T, int k, void* y,
   // z-side: z Vd of every correction first, then the shared anchor down
   // projection in split-K slices
   StreamOp dn_a = make_op(L, OP_DN_ANCHOR, T, w.zb, I, nullptr, w.smaps + 1, w.yb, H, false);
-  if (split) split_op(L, dn_a, w.ysplit, w.split_rows * H);
+  if (split) split_op(L, dn_a, w.ysplit, w.split_rows * H, kStreamSplitBlocksDown);
   const StreamOp dn_v = make_op(L, OP_DN_V, T, w.zb, I, nullptr, w.smaps + 1, w.Qb, rmax, false);
   LX_TRY(run_stream(L, 2, dn_v, &dn_a, s, "stream_dn_anchor_V"));
   LX_TRY(run_stream(L, 3,
