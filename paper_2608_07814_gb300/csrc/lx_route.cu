@@ -17,7 +17,8 @@
 // Large bf16 batches (k_router_tiled): persistent CTAs walk tiles of 8
 // tokens.  A thread holds the lane partials of 8 tokens x 8 experts for its
 // lane's chunks (64 accumulators), so every widened weight value serves 8
-// tokens and every widened token value 8 experts.  The 32 lane partials are
+// tokens and every widened token value 8 experts; the weight chunks (read
+// through L2) are software-pipelined one chunk ahead.  The 32 lane partials are
 // then combined by a transpose-reduce whose pairs are those of the canonical
 // order (lane l with lane l ^ 16, then ^ 8, ^ 4, ^ 2, ^ 1; IEEE addition is
 // commutative, so each sum is bit-identical), leaving lane l with the logits
@@ -206,32 +207,42 @@ k_router_tiled(const __nv_bfloat16* __restrict__ x, const __nv_bfloat16* __restr
       float acc[64];  // [token tt][expert ee] partials of this lane
 #pragma unroll
       for (int a = 0; a < 64; ++a) acc[a] = 0.f;
+      // weight chunks are software-pipelined one chunk ahead (raw bf16 in
+      // registers); token words come from shared memory per element pair
+      uint4 wr[8];
+      const int q_first = lane;
+#pragma unroll
+      for (int ee = 0; ee < 8; ++ee) {
+        const int e = 8 * g + ee;
+        wr[ee] = (e < E && q_first < nchunk)
+                     ? __ldg(reinterpret_cast<const uint4*>(W + (size_t)e * H) + q_first)
+                     : make_uint4(0, 0, 0, 0);
+      }
       for (int j = 0; j < nj; ++j) {
         const int q = lane + 32 * j;  // this lane's chunk
         if (q >= nchunk) break;
-        uint4 wr[8], xr[8];
+        uint4 wn[8];
+        const int qn = q + 32;
 #pragma unroll
         for (int ee = 0; ee < 8; ++ee) {
           const int e = 8 * g + ee;
-          const uint4* wrow = reinterpret_cast<const uint4*>(W + (size_t)e * H);
-          wr[ee] = e < E ? __ldg(wrow + q) : make_uint4(0, 0, 0, 0);
-          // the next chunk of this expert row heads for L1 while this one is used
-          if (e < E && q + 32 < nchunk)
-            asm volatile("prefetch.global.L1 [%0];" ::"l"(wrow + q + 32));
+          wn[ee] = (e < E && qn < nchunk)
+                       ? __ldg(reinterpret_cast<const uint4*>(W + (size_t)e * H) + qn)
+                       : make_uint4(0, 0, 0, 0);
         }
-#pragma unroll
-        for (int tt = 0; tt < 8; ++tt)
-          xr[tt] = reinterpret_cast<const uint4*>(xs + (size_t)tt * H)[q];
+        const uint32_t* xw = reinterpret_cast<const uint32_t*>(xs) + 4 * q;  // chunk q, token 0
 #pragma unroll
         for (int wd = 0; wd < 4; ++wd) {
+          uint32_t xt[8];
+#pragma unroll
+          for (int tt = 0; tt < 8; ++tt) xt[tt] = xw[(size_t)tt * (H / 2) + wd];
 #pragma unroll
           for (int hf = 0; hf < 2; ++hf) {  // element 2 wd + hf of the chunk, ascending
             float xv[8], wv[8];
 #pragma unroll
             for (int i = 0; i < 8; ++i) {
-              const uint32_t xw = wd == 0 ? xr[i].x : wd == 1 ? xr[i].y : wd == 2 ? xr[i].z : xr[i].w;
               const uint32_t ww = wd == 0 ? wr[i].x : wd == 1 ? wr[i].y : wd == 2 ? wr[i].z : wr[i].w;
-              xv[i] = hf ? bf16_hi(xw) : bf16_lo(xw);
+              xv[i] = hf ? bf16_hi(xt[i]) : bf16_lo(xt[i]);
               wv[i] = hf ? bf16_hi(ww) : bf16_lo(ww);
             }
 #pragma unroll
@@ -241,6 +252,8 @@ k_router_tiled(const __nv_bfloat16* __restrict__ x, const __nv_bfloat16* __restr
                 acc[tt * 8 + ee] = __fmaf_rn(xv[tt], wv[ee], acc[tt * 8 + ee]);
           }
         }
+#pragma unroll
+        for (int ee = 0; ee < 8; ++ee) wr[ee] = wn[ee];
       }
       // transpose-reduce: at offset o, the lane with bit o clear keeps the lower
       // half of its live entries and adds its partner's copy of them
