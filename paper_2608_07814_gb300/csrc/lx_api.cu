@@ -227,19 +227,20 @@ static lx_status check_call(lx_layer* L, int T, int k) {
   return LX_OK;
 }
 
+// plan_first: which tile plans the forward's GEMMs read (0 = generic, PLAN_TC =
+// tensor-core, -1 = none: the streaming kernels and lx_get_buckets read none)
 static lx_status bucket_ids(lx_layer* L, const int* ids, int T, int k, cudaStream_t s,
-                            bool plans) {
+                            int plan_first) {
   if (bucket_small_fits(L, T, k))
-    return launch_bucket_small(L, nullptr, ids, T, k, nullptr, nullptr, s, plans);
-  return launch_bucket(L, ids, T, k, s);
+    return launch_bucket_small(L, nullptr, ids, T, k, nullptr, nullptr, s, plan_first == 0);
+  return launch_bucket(L, ids, T, k, s, plan_first);
 }
 
-// Logits, top-k and bucketing of T tokens (single-CTA bucketing for small T).
 static lx_status route_and_bucket(lx_layer* L, const void* x, int T, int k, int* ids, float* w,
-                                  float* logits_user, cudaStream_t s, bool plans) {
+                                  float* logits_user, cudaStream_t s, int plan_first) {
   float* logits = logits_user ? logits_user : L->ws.logits;
   LX_TRY(launch_router(L, x, T, k, logits, ids, w, s));
-  return bucket_ids(L, ids, T, k, s, plans);
+  return bucket_ids(L, ids, T, k, s, plan_first);
 }
 
 
@@ -571,7 +572,7 @@ extern "C" lx_status lx_route(lx_layer* L, const void* x, int32_t T, int32_t k, 
   if (!x || !topk_id || !topk_w) return fail(LX_ERR_ARG, "NULL x/topk_id/topk_w");
   cudaStream_t s = (cudaStream_t)stream;
   LX_TRY(ensure_workspace(L, T, k, s));
-  LX_TRY(route_and_bucket(L, x, T, k, topk_id, topk_w, logits, s, false));
+  LX_TRY(route_and_bucket(L, x, T, k, topk_id, topk_w, logits, s, -1));
   L->last_T = T;
   L->last_k = k;
   return LX_OK;
@@ -584,7 +585,7 @@ extern "C" lx_status lx_bucket(lx_layer* L, const int32_t* topk_id, int32_t T, i
   if (!topk_id) return fail(LX_ERR_ARG, "NULL topk_id");
   cudaStream_t s = (cudaStream_t)stream;
   LX_TRY(ensure_workspace(L, T, k, s));
-  LX_TRY(bucket_ids(L, topk_id, T, k, s, false));
+  LX_TRY(bucket_ids(L, topk_id, T, k, s, -1));
   L->last_T = T;
   L->last_k = k;
   return LX_OK;
@@ -599,8 +600,9 @@ extern "C" lx_status lx_moe_forward(lx_layer* L, const void* x, int32_t T, int32
   cudaStream_t s = (cudaStream_t)stream;
   LX_TRY(ensure_workspace(L, T, k, s));
   Workspace& w = L->ws;
-  // the generic GEMMs read the tile plans; the streaming kernels do not
-  LX_TRY(route_and_bucket(L, x, T, k, w.topk_id, w.topk_w, nullptr, s, !use_stream(L, T, k)));
+  // the generic and tensor-core GEMMs read tile plans; the streaming kernels do not
+  const int plan_first = use_stream(L, T, k) ? -1 : use_tc(L, T, k) ? PLAN_TC : 0;
+  LX_TRY(route_and_bucket(L, x, T, k, w.topk_id, w.topk_w, nullptr, s, plan_first));
   L->last_T = T;
   L->last_k = k;
   if (use_stream(L, T, k)) {

@@ -94,6 +94,7 @@ struct PlanArgs {
   OpShape shape[N_PLANS];
   int bm[N_PLANS], bn[N_PLANS];  // token rows and output columns per tile
   int n_plans;
+  int first;                      // plan p fills tile-plan slot first + p
 };
 
 // tiles of one node in one plan
@@ -160,7 +161,7 @@ __global__ void k_offsets_plan(const int* __restrict__ key_cnt, int N, int E,
     __syncthreads();
   }
   for (int p = 0; p < pa.n_plans; ++p) {
-    int* to = tile_off + p * (max_items + 1);
+    int* to = tile_off + (pa.first + p) * (max_items + 1);
     int carry = 0;
     for (int base = 0; base < pa.n_items[p]; base += blockDim.x) {
       const int i = base + threadIdx.x;
@@ -336,7 +337,7 @@ k_bucket_small(const float* __restrict__ logits, const int* __restrict__ ids_in,
   publish_active(cnt, anchors, n_anchor, corrs, n_corr, act, act_n, sctr);
   // 5. tile plans: one warp per plan
   for (int p = warp; p < pa.n_plans; p += nw) {
-    int* to = tile_off + p * (max_items + 1);
+    int* to = tile_off + (pa.first + p) * (max_items + 1);
     int carry = 0;
     for (int base = 0; base < pa.n_items[p]; base += 32) {
       const int i = base + lane;
@@ -378,16 +379,20 @@ k_bucket_small(const float* __restrict__ logits, const int* __restrict__ ids_in,
 }  // namespace
 
 // plans 0..N_OPS-1: generic tiles; N_OPS..2*N_OPS-1: streaming tiles
-static PlanArgs make_plans(const lx_layer* L, int n_plans) {
+// Plans for slots [first, first + n_plans): 0 = the generic GEMMs' six ops,
+// PLAN_TC = the tensor-core GEMMs' six ops.
+static PlanArgs make_plans(const lx_layer* L, int n_plans, int first = 0) {
   PlanArgs pa;
   pa.n_plans = n_plans;
+  pa.first = first;
   for (int p = 0; p < n_plans; ++p) {
-    const int op = p % N_OPS;
+    const int slot = first + p;
+    const int op = slot % N_OPS;
     pa.shape[p] = op_shape(L, op);
     pa.items[p] = pa.shape[p].on_anchors ? L->d_anchors : L->d_corrs;
     pa.n_items[p] = pa.shape[p].on_anchors ? L->n_anchor : L->n_corr;
-    pa.bm[p] = p < PLAN_STREAM ? G_BM : p < PLAN_TC ? stream_tile_tokens() : tc_tile_tokens();
-    pa.bn[p] = p < PLAN_STREAM ? G_BN : p < PLAN_TC ? stream_tile_rows() : tc_tile_cols();
+    pa.bm[p] = slot < PLAN_STREAM ? G_BM : slot < PLAN_TC ? stream_tile_tokens() : tc_tile_tokens();
+    pa.bn[p] = slot < PLAN_STREAM ? G_BN : slot < PLAN_TC ? stream_tile_rows() : tc_tile_cols();
   }
   return pa;
 }
@@ -415,7 +420,8 @@ lx_status launch_bucket_small(lx_layer* L, const float* logits, const int* ids_i
   return LX_OK;
 }
 
-lx_status launch_bucket(lx_layer* L, const int* topk_id, int T, int k, cudaStream_t s) {
+lx_status launch_bucket(lx_layer* L, const int* topk_id, int T, int k, cudaStream_t s,
+                        int plan_first) {
   Workspace& w = L->ws;
   const long Tp = (w.cap_T + 15) / 16 * 16;
   const int keys = L->N + L->E;
@@ -435,7 +441,7 @@ lx_status launch_bucket(lx_layer* L, const int* topk_id, int T, int k, cudaStrea
     LX_CUDA(cudaGetLastError());
   }
   {
-    const PlanArgs pa = make_plans(L, N_PLANS);
+    const PlanArgs pa = plan_first < 0 ? make_plans(L, 0) : make_plans(L, N_OPS, plan_first);
     ProfScope ps(L, s, "bucket_offsets");
     launch_k(L, k_offsets_plan, 1, 1024, 0, s, w.key_cnt, L->N, L->E, w.key_off, L->d_rank, w.tile_off,
                                       op_max_items(L), pa, L->d_anchors, L->n_anchor, L->d_corrs,

@@ -384,7 +384,10 @@ struct ProfScope {
 // kernels / launchers (defined in the .cu files)
 lx_status launch_router(lx_layer* L, const void* x, int T, int k, float* logits, int* topk_id,
                         float* topk_w, cudaStream_t s);
-lx_status launch_bucket(lx_layer* L, const int* topk_id, int T, int k, cudaStream_t s);
+// plan_first: tile plans for the generic GEMMs (0), the tensor-core GEMMs
+// (PLAN_TC), or none (-1)
+lx_status launch_bucket(lx_layer* L, const int* topk_id, int T, int k, cudaStream_t s,
+                        int plan_first);
 lx_status launch_generic_experts(lx_layer* L, const void* x, int T, int k, void* y,
                                  cudaStream_t s);
 // Anchor split-K partials the SwiGLU / combine kernels read for the anchor rows
