@@ -164,6 +164,9 @@ def kernel_bytes(name, st, src, esz):
         "stream_dn_anchor_V": (ta * H * I + rt * I) * esz + Ra_c * I * 2 + Ra * H * 2 + rr * 2,
         "stream_dn_U": rt * H * esz + rr * 2 + Rc * H * 2,
     }
+    # the fused streaming launches: {V, anchor gate/up, U} and {Vd, anchor down, Ud}
+    table["stream_up"] = table["stream_up_anchor_V"] + table["stream_up_U"]
+    table["stream_dn"] = table["stream_dn_anchor_V"] + table["stream_dn_U"]
     return table.get(name)
 
 

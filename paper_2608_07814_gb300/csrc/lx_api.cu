@@ -154,7 +154,7 @@ static lx_status ensure_workspace(lx_layer* L, int T, int k, cudaStream_t s) {
       {(void**)&w.Qb, 2 * Rmax * rmax},
       {(void**)&w.act, sizeof(int) * std::max(1, L->n_anchor + L->n_corr)},
       {(void**)&w.act_n, sizeof(int) * 2},
-      {(void**)&w.sctr, sizeof(int) * N_TILE_COUNTERS},
+      {(void**)&w.sctr, sizeof(int) * sctr_ints(L)},
       {(void**)&w.xmaps, sizeof(CUtensorMap) * 3},
       {(void**)&w.smaps, sizeof(CUtensorMap) * 3},
       {(void**)&w.gmap, sizeof(CUtensorMap)},

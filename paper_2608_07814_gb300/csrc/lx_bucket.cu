@@ -115,7 +115,8 @@ __device__ __forceinline__ int plan_tiles(const PlanArgs& pa, int p, int r, int 
 // node-table order, and zeroed tile counters for the streaming launches.  One
 // CTA; warps 0 and 1 each compact one list.
 __device__ void publish_active(const int* cnt, const int* anchors, int n_anchor,
-                               const int* corrs, int n_corr, int* act, int* act_n, int* sctr) {
+                               const int* corrs, int n_corr, int* act, int* act_n, int* sctr,
+                               int n_sctr) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (warp < 2) {
     const int* list = warp == 0 ? anchors : corrs;
@@ -132,7 +133,7 @@ __device__ void publish_active(const int* cnt, const int* anchors, int n_anchor,
     }
     if (lane == 0) act_n[warp] = base;
   }
-  if (threadIdx.x < N_TILE_COUNTERS) sctr[threadIdx.x] = 0;
+  for (int i = threadIdx.x; i < n_sctr; i += blockDim.x) sctr[i] = 0;
 }
 
 // one CTA: node/expert offsets and the tile prefix of every plan
@@ -141,9 +142,9 @@ __global__ void k_offsets_plan(const int* __restrict__ key_cnt, int N, int E,
                                int* __restrict__ tile_off, int max_items, PlanArgs pa,
                                const int* __restrict__ anchors, int n_anchor,
                                const int* __restrict__ corrs, int n_corr, int* __restrict__ act,
-                               int* __restrict__ act_n, int* __restrict__ sctr) {
+                               int* __restrict__ act_n, int* __restrict__ sctr, int n_sctr) {
   pdl_wait();
-  if (act) publish_active(key_cnt, anchors, n_anchor, corrs, n_corr, act, act_n, sctr);
+  if (act) publish_active(key_cnt, anchors, n_anchor, corrs, n_corr, act, act_n, sctr, n_sctr);
   // node offsets then expert offsets
   for (int part = 0; part < 2; ++part) {
     const int n0 = part == 0 ? 0 : N, cnt = part == 0 ? N : E;
@@ -251,7 +252,7 @@ k_bucket_small(const float* __restrict__ logits, const int* __restrict__ ids_in,
                int* __restrict__ perm, int* __restrict__ tile_off, int max_items, PlanArgs pa,
                const int* __restrict__ anchors, int n_anchor, const int* __restrict__ corrs,
                int n_corr, int* __restrict__ act, int* __restrict__ act_n,
-               int* __restrict__ sctr) {
+               int* __restrict__ sctr, int n_sctr) {
   pdl_wait();
   extern __shared__ __align__(16) unsigned char sm[];
   const int keys = N + E;
@@ -334,7 +335,7 @@ k_bucket_small(const float* __restrict__ logits, const int* __restrict__ ids_in,
     __syncthreads();
   }
   for (int i = tid; i < keys + 2; i += nth) key_off_g[i] = off[i];
-  publish_active(cnt, anchors, n_anchor, corrs, n_corr, act, act_n, sctr);
+  publish_active(cnt, anchors, n_anchor, corrs, n_corr, act, act_n, sctr, n_sctr);
   // 5. tile plans: one warp per plan
   for (int p = warp; p < pa.n_plans; p += nw) {
     int* to = tile_off + (pa.first + p) * (max_items + 1);
@@ -415,7 +416,7 @@ lx_status launch_bucket_small(lx_layer* L, const float* logits, const int* ids_i
                                              w.key_off, w.node_tok, w.row_node, w.node_row, w.perm,
                                              w.tile_off, op_max_items(L), pa, L->d_anchors,
                                              L->n_anchor, L->d_corrs, L->n_corr, w.act, w.act_n,
-                                             w.sctr);
+                                             w.sctr, sctr_ints(L));
   LX_CUDA(cudaGetLastError());
   return LX_OK;
 }
@@ -445,7 +446,7 @@ lx_status launch_bucket(lx_layer* L, const int* topk_id, int T, int k, cudaStrea
     ProfScope ps(L, s, "bucket_offsets");
     launch_k(L, k_offsets_plan, 1, 1024, 0, s, w.key_cnt, L->N, L->E, w.key_off, L->d_rank, w.tile_off,
                                       op_max_items(L), pa, L->d_anchors, L->n_anchor, L->d_corrs,
-                                      L->n_corr, w.act, w.act_n, w.sctr);
+                                      L->n_corr, w.act, w.act_n, w.sctr, sctr_ints(L));
     LX_CUDA(cudaGetLastError());
   }
   {
@@ -551,7 +552,7 @@ extern "C" lx_status lx_bucket_noalloc(lx_layer* L, const int32_t* topk_id, int3
   const PlanArgs pa = make_plans(L, N_OPS);
   k_offsets_plan<<<1, 1024, 0, s>>>(key_cnt, L->N, L->E, key_off, L->d_rank, tile_off,
                                     op_max_items(L), pa, nullptr, 0, nullptr, 0, nullptr, nullptr,
-                                    nullptr);
+                                    nullptr, 0);
   LX_CUDA(cudaGetLastError());
   k_scatter<<<dim3((T + 255) / 256, (unsigned)keys), 256, 0, s>>>(
       marks, rank_in, key_off, topk_id, T, k, L->N, Tp, node_tok, row_node, perm);

@@ -186,6 +186,14 @@ struct StreamOp {
   int kbs;
   float* split_out;
   long split_stride;
+  // in-launch dependency of a factor product on the rows another op of the
+  // same launch writes: a tile of `sig`'s op adds 1 to sig[node * STREAM_DEP_TB
+  // + token block] once its rows are stored; a tile of `dep`'s op waits
+  // (bounded) until dep[...] reaches ceil(dep_nrank * rank / 64), the column
+  // tiles of its node's producer op
+  int* sig;
+  const int* dep;
+  int dep_nrank;
 };
 
 // The streaming launches: group 0 = {UP_ANCHOR, UP_V}, 1 = {UP_U},
@@ -208,8 +216,10 @@ __host__ __device__ inline int stream_col_blocks(int K, int ncol) {
   return 1;
 }
 
+constexpr int STREAM_DEP_TB = 8;  // token blocks per node covered by the dependency counters
+
 struct StreamLaunch {
-  StreamOp op[2];
+  StreamOp op[3];
   int n_ops;
   int* ctr;                  // tile counter of this launch (zeroed by the bucketing)
   int* err;                  // device error word (LX_ERR_TIMEOUT on a bounded wait)
@@ -276,7 +286,8 @@ struct Workspace {
   __nv_bfloat16* Qb = nullptr;  // [Rmax][rmax]
   int* act = nullptr;           // [n_anchor + n_corr] active anchors, then active corrections
   int* act_n = nullptr;         // [2] their counts
-  int* sctr = nullptr;          // [N_TILE_COUNTERS] streaming / tensor-core tile counters
+  int* sctr = nullptr;          // [sctr_ints] streaming / tensor-core tile counters, then the
+                                // streaming launches' dependency counters [2][N][STREAM_DEP_TB]
   CUtensorMap* xmaps = nullptr; // [3] TMA maps of Pb, zb, Qb (tensor-core A operands)
   CUtensorMap* smaps = nullptr; // [3] the same buffers in streaming-tile boxes
   __nv_bfloat16* xg = nullptr;  // [Rmax][H] token rows in node-row order (tensor-core path)
@@ -331,6 +342,9 @@ struct lx_layer {
 };
 
 namespace lx {
+
+// ints of the counter block zeroed by every bucketing
+inline int sctr_ints(const lx_layer* L) { return N_TILE_COUNTERS + 2 * L->N * STREAM_DEP_TB; }
 
 // Raises a kernel's dynamic shared-memory cap once per device (the flag array
 // belongs to the calling launcher).

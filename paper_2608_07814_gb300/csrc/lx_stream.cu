@@ -25,6 +25,7 @@
 #include <cuda.h>
 
 #include <algorithm>
+#include <initializer_list>
 
 
 #include "lx_internal.cuh"
@@ -111,6 +112,20 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatil
   }
 }
 
+// Bounded wait for an in-launch dependency counter (acquire); false on
+// timeout or when the CTA aborts.
+__device__ __forceinline__ bool dep_wait(const int* p, int need, volatile int* abort_flag) {
+  const unsigned long long t0 = clock64();
+  while (true) {
+    int v;
+    asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    if (v >= need) return true;
+    if (*abort_flag) return false;
+    if (clock64() - t0 > SW_TIMEOUT_CYCLES) return false;
+    __nanosleep(128);
+  }
+}
+
 // one 64x64 tile (box) of a tiled weight matrix: K tile kt of row tile rt
 __device__ __forceinline__ void tma_load_tile(uint32_t dst, const CUtensorMap* map, int kt, int rt,
                                               uint32_t bar) {
@@ -162,6 +177,7 @@ __device__ __forceinline__ uint4 lds_v4(uint32_t addr) {
 
 struct TileInfo {
   int op, node, grp, row0, tok0, M, Ng, K, ncb;
+  int tb;               // token block of the node's bucket
   int kb0, nkb, split;  // K blocks [kb0, kb0 + nkb) of split `split`
   bool active;
 };
@@ -171,10 +187,14 @@ __device__ __forceinline__ int op_tiles(const StreamOp& op) {
 }
 
 // Tile index -> (op, node, token block, group, column tile, K split).
+// tiles0 / tiles1: first tile of op 1 / op 2 (the ops' tiles are consecutive)
 __device__ __forceinline__ void decode_tile(const StreamLaunch& P, int tile, int tiles0,
-                                            TileInfo& ti) {
+                                            int tiles1, TileInfo& ti) {
   int o = 0, local = tile;
-  if (P.n_ops > 1 && tile >= tiles0) {
+  if (P.n_ops > 2 && tile >= tiles1) {
+    o = 2;
+    local = tile - tiles1;
+  } else if (P.n_ops > 1 && tile >= tiles0) {
     o = 1;
     local = tile - tiles0;
   }
@@ -193,6 +213,7 @@ __device__ __forceinline__ void decode_tile(const StreamLaunch& P, int tile, int
   const int r = op.rank[n];
   const int b0 = op.node_off[n], b1 = op.node_off[n + 1];
   ti.op = o;
+  ti.tb = tb;
   ti.node = n;
   ti.grp = grp;
   ti.row0 = ct * SW_ROWS * op.ncb;
@@ -285,6 +306,12 @@ __device__ __forceinline__ bool consume_tile(const StreamLaunch& P, const TileIn
                                     wr0) = v;
         }
       }
+      if (op.sig) {
+        // this warp's half of the column tile is stored: count it
+        __threadfence();
+        __syncwarp();
+        if (lane == 0) atomicAdd(op.sig + ti.node * STREAM_DEP_TB + ti.tb, 1);
+      }
       __syncwarp();
       continue;
     }
@@ -339,7 +366,8 @@ k_stream_gemm(const __grid_constant__ StreamLaunch P) {
     // ahead of use; the decoded tile rides in the shared slot of its first
     // stage.  Lane 0 waits and issues the weight box, all lanes copy token rows.
     const int tiles0 = op_tiles(P.op[0]);
-    const int total = tiles0 + (P.n_ops > 1 ? op_tiles(P.op[1]) : 0);
+    const int tiles1 = tiles0 + (P.n_ops > 1 ? op_tiles(P.op[1]) : 0);
+    const int total = tiles1 + (P.n_ops > 2 ? op_tiles(P.op[2]) : 0);
     // token-row sources of a tile, double-buffered so the next tile's are
     // prepared while the current one streams
     auto prepare = [&](const TileInfo& t, int buf) {
@@ -360,7 +388,7 @@ k_stream_gemm(const __grid_constant__ StreamLaunch P) {
     cur = __shfl_sync(0xffffffffu, cur, 0);
     TileInfo ti;
     if (cur < total) {
-      decode_tile(P, cur, tiles0, ti);
+      decode_tile(P, cur, tiles0, tiles1, ti);
       prepare(ti, 0);
     }
     __syncwarp();
@@ -376,6 +404,19 @@ k_stream_gemm(const __grid_constant__ StreamLaunch P) {
         const int rt0 = (ti.grp * ti.Ng + ti.row0) / SW_ROWS;
         const __nv_bfloat16* const* xs = xsrc + buf * SW_TOK;
         const int nkb = ti.nkb, kb0 = ti.kb0;
+        if (op.dep) {
+          // the token rows of this tile are written by another op of this
+          // launch: wait for every column tile of them (both consumer warps'
+          // halves), then order the async-proxy row loads after the acquire
+          int good = 1;
+          if (lane == 0) {
+            const int need = SW_CONSUMERS * ((op.dep_nrank * ti.K + SW_ROWS - 1) / SW_ROWS);
+            good = dep_wait(op.dep + ti.node * STREAM_DEP_TB + ti.tb, need, abort_flag) ? 1 : 0;
+            asm volatile("fence.proxy.async.global;" ::: "memory");
+          }
+          good = __shfl_sync(0xffffffffu, good, 0);
+          if (!good) ok = false;
+        }
         for (int cb = 0; cb < ti.ncb && ok; ++cb) {
           for (int kb = 0; kb < nkb; ++kb, ++it) {
             const uint32_t s = it % SW_STAGES;
@@ -415,7 +456,7 @@ k_stream_gemm(const __grid_constant__ StreamLaunch P) {
               // the next tile: decode and prepare its rows while these stages stream
               nxt = __shfl_sync(0xffffffffu, nxt, 0);
               if (nxt < total) {
-                decode_tile(P, nxt, tiles0, tn);
+                decode_tile(P, nxt, tiles0, tiles1, tn);
                 prepare(tn, buf ^ 1);
                 if (lane == 0 && tn.active)
                   asm volatile("prefetch.tensormap [%0];" ::"l"(
@@ -429,7 +470,7 @@ k_stream_gemm(const __grid_constant__ StreamLaunch P) {
       if (!prepared) {
         nxt = __shfl_sync(0xffffffffu, nxt, 0);
         if (nxt < total) {
-          decode_tile(P, nxt, tiles0, tn);
+          decode_tile(P, nxt, tiles0, tiles1, tn);
           prepare(tn, buf ^ 1);
         }
       }
@@ -547,6 +588,9 @@ static StreamOp make_op(lx_layer* L, int op, int T, const __nv_bfloat16* X, long
   o.kbs = 1 << 20;
   o.split_out = nullptr;
   o.split_stride = 0;
+  o.sig = nullptr;
+  o.dep = nullptr;
+  o.dep_nrank = 0;
   return o;
 }
 
@@ -571,12 +615,13 @@ static void split_op(lx_layer* L, StreamOp& o, float* part, long stride, int blo
   (void)L;
 }
 
-// One streaming launch (launch group g) over up to two ops' tile grids.
-static lx_status run_stream(lx_layer* L, int g, const StreamOp& o0, const StreamOp* o1,
+// One streaming launch (launch group g) over up to three ops' tile grids, in
+// claim order.
+static lx_status run_stream(lx_layer* L, int g, std::initializer_list<const StreamOp*> ops,
                             cudaStream_t s, const char* name) {
   StreamLaunch P;
   P.n_ops = 0;
-  for (const StreamOp* o : {&o0, o1}) {
+  for (const StreamOp* o : ops) {
     if (!o || o->n_items == 0) continue;
     P.op[P.n_ops++] = *o;
   }
@@ -586,22 +631,28 @@ static lx_status run_stream(lx_layer* L, int g, const StreamOp& o0, const Stream
   return launch_stream(L, P, s, name);
 }
 
-// The decode forward: every touched weight byte is streamed once.
+// The decode forward: every touched weight byte is streamed once.  Two
+// streaming launches: {x V of every correction, the shared anchor gate/up,
+// then P U of every correction (each waits for its P rows)} and the same on
+// the z side; the factor products fill the tail of the anchor products.
 lx_status launch_fast_experts(lx_layer* L, const void* x, int T, int k, void* y, cudaStream_t s) {
   Workspace& w = L->ws;
   const long H = L->H, I = L->I, rmax = L->max_rank;
   const __nv_bfloat16* xb = static_cast<const __nv_bfloat16*>(x);
   const bool split = w.hsplit && w.ysplit && warp_kernels_fit(L, k) &&
                      (long)T * std::min<long>(L->N, (long)k * L->max_depth) <= w.split_rows;
-  // x-side: x V of every correction (whole-K tiles, claimed first), and the
-  // shared anchor gate/up in split-K slices
+  int* dep_up = w.sctr + N_TILE_COUNTERS;
+  int* dep_dn = dep_up + (size_t)L->N * STREAM_DEP_TB;
+  // x-side: x V of every correction (whole-K tiles, claimed first), the shared
+  // anchor gate/up in split-K slices, then the corrections' U products
+  StreamOp up_v = make_op(L, OP_UP_V, T, xb, H, w.node_tok, nullptr, w.Pb, 2 * rmax, false);
+  up_v.sig = dep_up;
   StreamOp up_a = make_op(L, OP_UP_ANCHOR, T, xb, H, w.node_tok, nullptr, w.hb, 2 * I, false);
   if (split) split_op(L, up_a, w.hsplit, w.split_rows * 2 * I, kStreamSplitBlocksUp);
-  const StreamOp up_v = make_op(L, OP_UP_V, T, xb, H, w.node_tok, nullptr, w.Pb, 2 * rmax, false);
-  LX_TRY(run_stream(L, 0, up_v, &up_a, s, "stream_up_anchor_V"));
-  LX_TRY(run_stream(L, 1,
-                    make_op(L, OP_UP_U, T, w.Pb, 2 * rmax, nullptr, w.smaps + 0, w.hb, 2 * I, false),
-                    nullptr, s, "stream_up_U"));
+  StreamOp up_u = make_op(L, OP_UP_U, T, w.Pb, 2 * rmax, nullptr, w.smaps + 0, w.hb, 2 * I, false);
+  up_u.dep = dep_up;
+  up_u.dep_nrank = 2;  // P = [x Vg | x Vu]: 2r columns
+  LX_TRY(run_stream(L, 0, {&up_v, &up_a, &up_u}, s, "stream_up"));
   SplitParts hs, ys;
   if (up_a.nsplit > 1) {
     hs.part = up_a.split_out;
@@ -609,15 +660,16 @@ lx_status launch_fast_experts(lx_layer* L, const void* x, int T, int k, void* y,
     hs.stride = up_a.split_stride;
   }
   LX_TRY(launch_swiglu(L, T, k, true, s, hs));
-  // z-side: z Vd of every correction first, then the shared anchor down
-  // projection in split-K slices
+  // z-side: z Vd of every correction first, the shared anchor down
+  // projection, then the corrections' Ud products
+  StreamOp dn_v = make_op(L, OP_DN_V, T, w.zb, I, nullptr, w.smaps + 1, w.Qb, rmax, false);
+  dn_v.sig = dep_dn;
   StreamOp dn_a = make_op(L, OP_DN_ANCHOR, T, w.zb, I, nullptr, w.smaps + 1, w.yb, H, false);
   if (split) split_op(L, dn_a, w.ysplit, w.split_rows * H, kStreamSplitBlocksDown);
-  const StreamOp dn_v = make_op(L, OP_DN_V, T, w.zb, I, nullptr, w.smaps + 1, w.Qb, rmax, false);
-  LX_TRY(run_stream(L, 2, dn_v, &dn_a, s, "stream_dn_anchor_V"));
-  LX_TRY(run_stream(L, 3,
-                    make_op(L, OP_DN_U, T, w.Qb, rmax, nullptr, w.smaps + 2, w.yb, H, false),
-                    nullptr, s, "stream_dn_U"));
+  StreamOp dn_u = make_op(L, OP_DN_U, T, w.Qb, rmax, nullptr, w.smaps + 2, w.yb, H, false);
+  dn_u.dep = dep_dn;
+  dn_u.dep_nrank = 1;  // Q = z Vd: r columns
+  LX_TRY(run_stream(L, 2, {&dn_v, &dn_a, &dn_u}, s, "stream_dn"));
   if (dn_a.nsplit > 1) {
     ys.part = dn_a.split_out;
     ys.splits = dn_a.nsplit;
