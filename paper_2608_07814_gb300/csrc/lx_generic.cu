@@ -107,6 +107,9 @@ k_grouped_gemm(GemmArgs g) {
 }
 
 __device__ __forceinline__ float silu_f(float v) { return v / (1.f + expf(-v)); }
+// the bf16 paths' SiLU: CUDA's fast exponential and division intrinsics (their
+// error is far below the bf16 rounding of the operands)
+__device__ __forceinline__ float silu_fast(float v) { return __fdividef(v, 1.f + __expf(-v)); }
 
 // One CTA per token.  Its k selected experts' gated SwiGLU outputs,
 //   a_s = g_s * silu(sum_l h_gate[row(s,l)]) * sum_l h_up[row(s,l)],
@@ -288,6 +291,7 @@ constexpr int WT_SLOTS = 8;
 
 struct WarpRows {
   int rows[32];       // entry j = slot j / D, level j % D (-1: none)
+  int lrow[32];       // entry j: index of its row among the distinct rows (-1: none)
   int drow[32];       // distinct rows, ascending
   unsigned dmask[32]; // slots whose path holds distinct row d
   float g[WT_SLOTS];
@@ -309,7 +313,10 @@ __device__ __forceinline__ void warp_token_rows(const int* __restrict__ node_row
     const int q = __ffs(b) - 1;
     rank += __shfl_sync(0xffffffffu, key, q) < key;
   }
-  if (lane < kD) wr.rows[lane] = v;
+  if (lane < kD) {
+    wr.rows[lane] = v;
+    wr.lrow[lane] = key != INT_MAX ? rank : -1;
+  }
   if (first) wr.drow[rank] = key;
   // entry j holds its path's anchor if it is the path's last valid level
   // (paths are stored from the expert's own node up to the anchor)
@@ -343,6 +350,9 @@ __device__ __forceinline__ Cols<CPL> ld_cols(const float* p) {
   if constexpr (CPL == 4) {
     const float4 f = __ldg(reinterpret_cast<const float4*>(p));
     r.v[0] = f.x; r.v[1] = f.y; r.v[2] = f.z; r.v[3] = f.w;
+  } else if constexpr (CPL == 2) {
+    const float2 f = __ldg(reinterpret_cast<const float2*>(p));
+    r.v[0] = f.x; r.v[1] = f.y;
   } else {
 #pragma unroll
     for (int i = 0; i < CPL; ++i) r.v[i] = __ldg(p + i);
@@ -356,6 +366,9 @@ __device__ __forceinline__ Cols<CPL> ld_cols(const __nv_bfloat16* p) {
     const uint2 u = __ldg(reinterpret_cast<const uint2*>(p));
     r.v[0] = __uint_as_float(u.x << 16); r.v[1] = __uint_as_float(u.x & 0xFFFF0000u);
     r.v[2] = __uint_as_float(u.y << 16); r.v[3] = __uint_as_float(u.y & 0xFFFF0000u);
+  } else if constexpr (CPL == 2) {
+    const uint32_t u = __ldg(reinterpret_cast<const unsigned int*>(p));
+    r.v[0] = __uint_as_float(u << 16); r.v[1] = __uint_as_float(u & 0xFFFF0000u);
   } else {
 #pragma unroll
     for (int i = 0; i < CPL; ++i) r.v[i] = __bfloat162float(p[i]);
@@ -374,6 +387,8 @@ __device__ __forceinline__ RawB<CPL> ld_raw(const __nv_bfloat16* p) {
     const uint2 u = __ldg(reinterpret_cast<const uint2*>(p));
     r.w[0] = u.x;
     r.w[1] = u.y;
+  } else if constexpr (CPL == 2) {
+    r.w[0] = __ldg(reinterpret_cast<const unsigned int*>(p));
   } else {
     r.w[0] = (uint32_t)__ldg(reinterpret_cast<const unsigned short*>(p));
   }
@@ -386,6 +401,10 @@ __device__ __forceinline__ void add_raw(Cols<CPL>& a, const RawB<CPL>& r, bool v
       a.v[0] += __uint_as_float(r.w[0] << 16); a.v[1] += __uint_as_float(r.w[0] & 0xFFFF0000u);
       a.v[2] += __uint_as_float(r.w[1] << 16); a.v[3] += __uint_as_float(r.w[1] & 0xFFFF0000u);
     }
+  } else if constexpr (CPL == 2) {
+    if (valid) {
+      a.v[0] += __uint_as_float(r.w[0] << 16); a.v[1] += __uint_as_float(r.w[0] & 0xFFFF0000u);
+    }
   } else {
     if (valid) a.v[0] += __uint_as_float(r.w[0] << 16);
   }
@@ -394,6 +413,8 @@ template <typename T, int CPL>
 __device__ __forceinline__ void st_cols(T* p, const Cols<CPL>& c) {
   if constexpr (CPL == 4) {
     store4<T>(p, make_float4(c.v[0], c.v[1], c.v[2], c.v[3]));
+  } else if constexpr (CPL == 2 && std::is_same<T, __nv_bfloat16>::value) {
+    *reinterpret_cast<__nv_bfloat162*>(p) = __floats2bfloat162_rn(c.v[0], c.v[1]);
   } else if constexpr (std::is_same<T, float>::value) {
 #pragma unroll
     for (int i = 0; i < CPL; ++i) p[i] = c.v[i];
@@ -414,6 +435,7 @@ k_swiglu_warp(const float* __restrict__ topk_w, const int* __restrict__ node_row
               const TH* __restrict__ h, int I, TZ* __restrict__ z, int cols_per_item,
               const SplitParts hs) {
   pdl_wait();
+  extern __shared__ float zsm[];  // bf16 path: [warp][k * D rows][32 lanes * CPL]
   __shared__ WarpRows wrs[WT_WARPS];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   WarpRows& wr = wrs[warp];
@@ -485,8 +507,34 @@ k_swiglu_warp(const float* __restrict__ topk_w, const int* __restrict__ node_row
           }
           const float g = sl < k ? wr.g[sl] : 0.f;
 #pragma unroll
-          for (int i = 0; i < CPL; ++i) act[sl].v[i] = g * silu_f(pg.v[i]) * pu.v[i];
+          for (int i = 0; i < CPL; ++i) act[sl].v[i] = g * silu_fast(pg.v[i]) * pu.v[i];
         }
+        // z: every slot's act into the accumulators of the distinct rows on its
+        // path, slots in ascending order; then each distinct row out once
+        float* zacc = zsm + (size_t)warp * kD * 32 * CPL;
+        for (int d = 0; d < nd; ++d)
+#pragma unroll
+          for (int i = 0; i < CPL; ++i) zacc[(d * 32 + lane) * CPL + i] = 0.f;
+#pragma unroll
+        for (int sl = 0; sl < WT_SLOTS; ++sl) {
+          if (sl < k) {
+#pragma unroll
+            for (int l = 0; l < D; ++l) {
+              const int d = wr.lrow[sl * D + l];
+              if (d >= 0) {
+#pragma unroll
+                for (int i = 0; i < CPL; ++i) zacc[(d * 32 + lane) * CPL + i] += act[sl].v[i];
+              }
+            }
+          }
+        }
+        for (int d = 0; d < nd; ++d) {
+          Cols<CPL> zc;
+#pragma unroll
+          for (int i = 0; i < CPL; ++i) zc.v[i] = zacc[(d * 32 + lane) * CPL + i];
+          st_cols<TZ, CPL>(z + (size_t)wr.drow[d] * I + c, zc);
+        }
+        continue;
       } else {
 #pragma unroll
       for (int sl = 0; sl < WT_SLOTS; ++sl) {
@@ -643,14 +691,25 @@ static void launch_swiglu_c(lx_layer* L, int T, int k, const TH* h, TZ* z, cudaS
   Workspace& w = L->ws;
   const int cols = warp_item_cols(L, T, L->I, 32 * CPL);
   const int grid = warp_grid(L, T, L->I, cols);
+  const size_t zs = sizeof(TH) == 2 ? (size_t)WT_WARPS * k * D * 32 * CPL * 4 : 0;
+  if (zs > 0) {  // the accumulators plus the static rows may pass the 48 KB default
+    static bool done_s[64] = {}, done_n[64] = {};
+    if constexpr (CPL == 1) {
+      if (hs.splits > 1)
+        (void)smem_cap_once((const void*)k_swiglu_warp<TH, TZ, D, true, CPL>, 128 * 1024,
+                            L->device, done_s);
+    }
+    (void)smem_cap_once((const void*)k_swiglu_warp<TH, TZ, D, false, CPL>, 128 * 1024, L->device,
+                        done_n);
+  }
   if constexpr (CPL == 1) {
     if (hs.splits > 1) {
-      launch_k(L, k_swiglu_warp<TH, TZ, D, true, CPL>, grid, WT_WARPS * 32, 0, s, w.topk_w,
+      launch_k(L, k_swiglu_warp<TH, TZ, D, true, CPL>, grid, WT_WARPS * 32, zs, s, w.topk_w,
                w.node_row, T, k, h, L->I, z, cols, hs);
       return;
     }
   }
-  launch_k(L, k_swiglu_warp<TH, TZ, D, false, CPL>, grid, WT_WARPS * 32, 0, s, w.topk_w,
+  launch_k(L, k_swiglu_warp<TH, TZ, D, false, CPL>, grid, WT_WARPS * 32, zs, s, w.topk_w,
            w.node_row, T, k, h, L->I, z, cols, hs);
 }
 
@@ -658,6 +717,7 @@ template <typename TH, typename TZ, int D>
 static void launch_swiglu_d(lx_layer* L, int T, int k, const TH* h, TZ* z, cudaStream_t s,
                             const SplitParts& hs) {
   // split partials (small batches only) take the one-column-per-lane form
+  // (measured on GB300: four columns per lane beat two for large batches)
   if (narrow_cols(L, T, L->I) || hs.splits > 1)
     launch_swiglu_c<TH, TZ, D, 1>(L, T, k, h, z, s, hs);
   else
