@@ -142,6 +142,22 @@ def test_stream_path_serves_layer(name):
     assert L.info()["stream_path"] == 1
 
 
+@pytest.mark.parametrize("name", STREAM)
+@pytest.mark.parametrize("T", [1, 37, 200, 256])
+def test_forward_buckets(name, T):
+    """The bucketing a streaming forward runs (fused with the router for small
+    batches) is bit-exact too: read back after the forward."""
+    src, L = installed(name, SMALL[name])
+    x = synth.tokens(src, T, seed=900 + T)
+    check_forward(src, L, x, src.top_k)
+    b = L.get_buckets()
+    torch.cuda.synchronize()
+    o_ids, _, _ = oracle.route(src, x, src.top_k)
+    ref = oracle.buckets(src, o_ids)
+    for key in ("node_off", "node_tok", "node_row", "expert_off", "perm"):
+        assert np.array_equal(b[key].cpu().numpy(), ref[key]), key
+
+
 @pytest.mark.parametrize("T", [64, 256, 257])
 def test_stream_generic_boundary(T):
     src, L = installed("stream_flat", SMALL["stream_flat"])
