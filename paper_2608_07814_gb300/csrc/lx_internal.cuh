@@ -221,6 +221,10 @@ constexpr int STREAM_DEP_TB = 8;  // token blocks per node covered by the depend
 struct StreamLaunch {
   StreamOp op[3];
   int n_ops;
+  // 1: the launch's weights and tile lists do not depend on the preceding
+  // kernel (only its token rows do): the producer issues the first tile's
+  // weight boxes before griddepcontrol.wait
+  int early_weights;
   int* ctr;                  // tile counter of this launch (zeroed by the bucketing)
   int* err;                  // device error word (LX_ERR_TIMEOUT on a bounded wait)
 };

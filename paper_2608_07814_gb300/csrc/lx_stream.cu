@@ -338,7 +338,8 @@ __device__ __forceinline__ bool consume_tile(const StreamLaunch& P, const TileIn
 
 __global__ void __launch_bounds__(SW_THREADS, SW_CTAS_PER_SM)
 k_stream_gemm(const __grid_constant__ StreamLaunch P) {
-  pdl_wait();
+  if (!P.early_weights) pdl_wait();
+  else asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -392,6 +393,27 @@ k_stream_gemm(const __grid_constant__ StreamLaunch P) {
       prepare(ti, 0);
     }
     __syncwarp();
+    // Dependent launch whose weights do not depend on the preceding kernel: the
+    // first tile's first weight boxes go out before the wait for it (stage
+    // it < npre already holds its box and expected bytes); token rows after.
+    uint32_t npre = 0;
+    if (P.early_weights) {
+      if (cur < total && ti.active && ti.ncb >= 1) {
+        const StreamOp& op = P.op[ti.op];
+        npre = (uint32_t)min(ti.nkb, SW_STAGES);
+        if (lane == 0) {
+          const int rt0 = (ti.grp * ti.Ng + ti.row0) / SW_ROWS;
+          for (uint32_t kb = 0; kb < npre; ++kb) {  // fresh stages: nothing to wait for
+            const uint32_t wbox = smem_base + kb * SW_STAGE_BYTES;
+            if (kb == 0) slot[0] = ti;
+            mbar_expect_tx(full0 + 8 * kb, SW_BOX_BYTES + (op.gather ? 0 : SW_XBYTES));
+            tma_load_tile(wbox, op.tmaps + ti.node, ti.kb0 + kb, rt0, full0 + 8 * kb);
+          }
+        }
+      }
+      __syncwarp();
+      asm volatile("griddepcontrol.wait;" ::: "memory");
+    }
     int buf = 0;
     bool ok = true;
     while (cur < total && ok) {
@@ -421,7 +443,8 @@ k_stream_gemm(const __grid_constant__ StreamLaunch P) {
           for (int kb = 0; kb < nkb; ++kb, ++it) {
             const uint32_t s = it % SW_STAGES;
             int good = 1;
-            if (lane == 0) {
+            const bool pre = it < npre;  // weight box issued before the dependency wait
+            if (lane == 0 && !pre) {
               good = mbar_wait(empty0 + 8 * s, ((it / SW_STAGES) & 1) ^ 1, abort_flag) ? 1 : 0;
               if (good) {
                 if (cb == 0 && kb == 0) slot[s] = ti;
@@ -435,7 +458,7 @@ k_stream_gemm(const __grid_constant__ StreamLaunch P) {
             }
             const uint32_t wbox = smem_base + s * SW_STAGE_BYTES;
             if (lane == 0) {
-              tma_load_tile(wbox, map, kb0 + kb, rt0 + cb, full0 + 8 * s);
+              if (!pre) tma_load_tile(wbox, map, kb0 + kb, rt0 + cb, full0 + 8 * s);
               // contiguous token rows: one box of SW_TOK rows (rows past the
               // bucket belong to the next node and are never stored)
               if (!op.gather)
@@ -628,6 +651,9 @@ static lx_status run_stream(lx_layer* L, int g, std::initializer_list<const Stre
   if (P.n_ops == 0) return LX_OK;
   P.ctr = L->ws.sctr + g;
   P.err = L->ws.err;
+  // the z-side launch follows the SwiGLU kernel, whose output only its token
+  // rows read
+  P.early_weights = g == 2 ? 1 : 0;
   return launch_stream(L, P, s, name);
 }
 
