@@ -136,7 +136,18 @@ LX_API lx_status lx_bucket(lx_layer* layer, const int32_t* topk_id, int32_t T, i
 /*
  * The compressed-MoE forward: route, bucket, shared anchor GEMMs with the
  * low-rank corrections and SwiGLU, down-projection and weighted combine.
- *   x: device [T][H], y: device [T][H] (layer dtype); y may not alias x.
+ *   x: device [T][H], y: device [T][H] (layer dtype), 16-byte aligned; y may
+ *   not alias x.
+ * Kernels: bf16 layers whose H, I and ranks are multiples of 64 (with k <= 8,
+ * k * max_depth <= 32) take the weight-streaming kernels for T <= 256 and the
+ * tcgen05 tensor-core kernels above; every other layer, and LX_PATH_GENERIC,
+ * the CUDA-core kernels.  All products accumulate in fp32; on the streaming
+ * and tensor-core paths the intermediates that cross device memory (the
+ * gate/up pre-activations, x V, the SwiGLU aggregate, z Vd and the down
+ * partials) are stored as bf16, on the CUDA-core path as fp32.
+ * Errors: LX_ERR_ARG (k, T, alignment, aliasing, null pointers), LX_ERR_OOM /
+ * LX_ERR_CUDA while growing the workspace; a kernel's bounded wait that gave up
+ * is reported by lx_layer_info (device_error).
  */
 LX_API lx_status lx_moe_forward(lx_layer* layer, const void* x, int32_t T, int32_t k, void* y,
                          void* stream);
@@ -165,7 +176,8 @@ typedef struct {
   int32_t last_rows;          /* node_off[n_nodes] of the last bucketing (synchronises) */
   int32_t device_error;       /* lx_status recorded by a kernel (e.g. LX_ERR_TIMEOUT when a
                                  bounded device-side wait gave up), 0 if none (synchronises) */
-  int32_t stream_path;        /* 1 if the weight-streaming (TMA) decode kernels serve the layer */
+  int32_t stream_path;        /* 1 if the weight-streaming (T <= 256) and tcgen05 (T > 256)
+                                 kernels serve the layer under LX_PATH_AUTO */
 } lx_layer_info_t;
 
 LX_API lx_status lx_layer_info(lx_layer* layer, lx_layer_info_t* info);
@@ -178,7 +190,9 @@ LX_API lx_status lx_set_path(lx_layer* layer, int32_t path);
 
 /*
  * Kernel timing.  While enabled, every kernel the layer launches is bracketed by
- * CUDA events on its stream.  lx_read_profile synchronises on the last event,
+ * CUDA events on its stream (and kernels are launched without programmatic
+ * dependent launch, so each event pair times one kernel; the events add the
+ * launch latency to each).  lx_read_profile synchronises on the last event,
  * writes up to `cap` records of the launches since the previous read (oldest
  * first) and clears the list; *n receives the number written.
  */

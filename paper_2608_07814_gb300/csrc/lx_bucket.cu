@@ -101,11 +101,7 @@ struct PlanArgs {
 __device__ __forceinline__ int plan_tiles(const PlanArgs& pa, int p, int r, int rows) {
   const OpShape sh = pa.shape[p];
   const int Ng = sh.n_const + sh.n_rank * r;
-  int ncol = (Ng + pa.bn[p] - 1) / pa.bn[p];
-  if (p >= PLAN_STREAM && p < PLAN_TC) {
-    const int ncb = stream_col_blocks(sh.k_const + sh.k_rank * r, ncol);
-    ncol = (ncol + ncb - 1) / ncb;
-  }
+  const int ncol = (Ng + pa.bn[p] - 1) / pa.bn[p];
   return ((rows + pa.bm[p] - 1) / pa.bm[p]) * sh.groups * ncol;
 }
 
@@ -392,8 +388,8 @@ static PlanArgs make_plans(const lx_layer* L, int n_plans, int first = 0) {
     pa.shape[p] = op_shape(L, op);
     pa.items[p] = pa.shape[p].on_anchors ? L->d_anchors : L->d_corrs;
     pa.n_items[p] = pa.shape[p].on_anchors ? L->n_anchor : L->n_corr;
-    pa.bm[p] = slot < PLAN_STREAM ? G_BM : slot < PLAN_TC ? stream_tile_tokens() : tc_tile_tokens();
-    pa.bn[p] = slot < PLAN_STREAM ? G_BN : slot < PLAN_TC ? stream_tile_rows() : tc_tile_cols();
+    pa.bm[p] = slot < PLAN_TC ? G_BM : tc_tile_tokens();
+    pa.bn[p] = slot < PLAN_TC ? G_BN : tc_tile_cols();
   }
   return pa;
 }

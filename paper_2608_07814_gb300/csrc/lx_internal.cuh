@@ -125,13 +125,12 @@ enum OpKind {
   N_OPS = 6
 };
 
-// Tile plans: plan p < N_OPS is op p for the generic kernel (32-token x
-// 64-column tiles); plan N_OPS + p is op p for the streaming kernel (64-token
-// x 64-weight-row blocks; ops with a short K take several column blocks per
-// tile, see stream_col_blocks).
-constexpr int N_PLANS = 3 * N_OPS;
-constexpr int PLAN_STREAM = N_OPS;
-constexpr int PLAN_TC = 2 * N_OPS;   // tensor-core tiles: 128 tokens x 256 columns
+// Tile plans (prefix of the tiles per node, built by the bucketing): plan p <
+// N_OPS is op p for the generic kernel (32-token x 64-column tiles); plan
+// PLAN_TC + p is op p for the tensor-core kernel (128 tokens x 256 columns).
+// The streaming kernels decode their tiles from the active-node lists instead.
+constexpr int N_PLANS = 2 * N_OPS;
+constexpr int PLAN_TC = N_OPS;
 constexpr int N_TILE_COUNTERS = 16;  // dynamic tile counters, zeroed by the bucketing
 
 // Per-op shape rule: for node n with rank r, each group has
@@ -187,34 +186,19 @@ struct StreamOp {
   float* split_out;
   long split_stride;
   // in-launch dependency of a factor product on the rows another op of the
-  // same launch writes: a tile of `sig`'s op adds 1 to sig[node * STREAM_DEP_TB
-  // + token block] once its rows are stored; a tile of `dep`'s op waits
-  // (bounded) until dep[...] reaches ceil(dep_nrank * rank / 64), the column
-  // tiles of its node's producer op
+  // same launch writes: each consumer warp of a tile of `sig`'s op adds 1 to
+  // sig[node * STREAM_DEP_TB + token block] once its half of the rows is
+  // stored; a tile of `dep`'s op waits (bounded) until dep[...] reaches
+  // 2 * ceil(dep_nrank * rank / 64), both halves of every column tile of its
+  // node's producer op
   int* sig;
   const int* dep;
   int dep_nrank;
 };
 
-// The streaming launches: group 0 = {UP_ANCHOR, UP_V}, 1 = {UP_U},
-// 2 = {DN_ANCHOR, DN_V}, 3 = {DN_U}.  A launch's tile index runs over
-// op 0's (item, token block, group, column tile) grid, then op 1's; tiles of
-// inactive nodes or beyond a node's columns are skipped.
+// Dynamic tile counters of the launches: 0 = the x-side streaming launch, 2 =
+// the z-side one, N_STREAM_GROUPS + op = the tensor-core launch of op.
 constexpr int N_STREAM_GROUPS = 4;
-__host__ __device__ inline int stream_group_op(int g, int j) {
-  const int ops[N_STREAM_GROUPS][2] = {{OP_UP_ANCHOR, OP_UP_V}, {OP_UP_U, -1},
-                                       {OP_DN_ANCHOR, OP_DN_V}, {OP_DN_U, -1}};
-  return ops[g][j];
-}
-
-// Column blocks (of 64 weight rows) per streaming tile.  Measured on GB300:
-// one block per tile (more, smaller tiles spread over more CTAs) streams the
-// short-K factor products faster than grouping blocks, so tiles keep one.
-__host__ __device__ inline int stream_col_blocks(int K, int ncol) {
-  (void)K;
-  (void)ncol;
-  return 1;
-}
 
 constexpr int STREAM_DEP_TB = 8;  // token blocks per node covered by the dependency counters
 
