@@ -136,8 +136,8 @@ LX_API lx_status lx_bucket(lx_layer* layer, const int32_t* topk_id, int32_t T, i
 /*
  * The compressed-MoE forward: route, bucket, shared anchor GEMMs with the
  * low-rank corrections and SwiGLU, down-projection and weighted combine.
- *   x: device [T][H], y: device [T][H] (layer dtype), 16-byte aligned; y may
- *   not alias x.
+ *   x: device [T][H], y: device [T][H] (layer dtype), both 16-byte aligned;
+ *   y may not overlap x.
  * Kernels: bf16 layers whose H, I and ranks are multiples of 64 (with k <= 8,
  * k * max_depth <= 32) take the weight-streaming kernels for T <= 256 and the
  * tcgen05 tensor-core kernels above; every other layer, and LX_PATH_GENERIC,

@@ -596,7 +596,13 @@ extern "C" lx_status lx_moe_forward(lx_layer* L, const void* x, int32_t T, int32
   LX_TRY(check_call(L, T, k));
   if (T == 0) return LX_OK;
   if (!x || !y) return fail(LX_ERR_ARG, "NULL x/y");
-  if (x == y) return fail(LX_ERR_ARG, "y may not alias x");
+  if (reinterpret_cast<uintptr_t>(x) % 16 || reinterpret_cast<uintptr_t>(y) % 16)
+    return fail(LX_ERR_ARG, "x and y must be 16-byte aligned");
+  {
+    const uintptr_t xb = reinterpret_cast<uintptr_t>(x), yb = reinterpret_cast<uintptr_t>(y);
+    const uintptr_t bytes = (uintptr_t)T * L->H * L->esz;
+    if (xb < yb + bytes && yb < xb + bytes) return fail(LX_ERR_ARG, "y may not overlap x");
+  }
   cudaStream_t s = (cudaStream_t)stream;
   LX_TRY(ensure_workspace(L, T, k, s));
   Workspace& w = L->ws;

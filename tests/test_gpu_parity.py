@@ -269,6 +269,14 @@ def test_call_errors():
     with pytest.raises(lx.LxError) as e:
         L.moe_forward(x, 2, y=x)                   # aliasing
     assert e.value.status == lx.LX_ERR_ARG
+    ybig = torch.zeros(4 * 64 + 1, dtype=torch.float32, device="cuda")
+    with pytest.raises(lx.LxError) as e:
+        L.moe_forward(x, 2, y=ybig[1:].view(4, 64))  # misaligned y
+    assert e.value.status == lx.LX_ERR_ARG
+    xy = torch.zeros(8 * 64, dtype=torch.float32, device="cuda")
+    with pytest.raises(lx.LxError) as e:
+        L.moe_forward(xy[:4 * 64].view(4, 64), 2, y=xy[2 * 64:6 * 64].view(4, 64))  # overlap
+    assert e.value.status == lx.LX_ERR_ARG
 
 
 # ----------------------------------------------------------------------------
