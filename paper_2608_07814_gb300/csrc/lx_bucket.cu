@@ -107,25 +107,34 @@ __device__ __forceinline__ int plan_tiles(const PlanArgs& pa, int p, int r, int 
 
 
 
-// Compact lists of the active anchors and corrections (bucket size > 0), in
-// node-table order, and zeroed tile counters for the streaming launches.  One
-// CTA; warps 0 and 1 each compact one list.
+// Work items of the streaming launches: one (node, token block) pair per
+// `blk` rows of every active node's bucket, anchors then corrections, in
+// node-table order, packed as node * STREAM_DEP_TB + block; and zeroed tile
+// counters.  blk = 0 (batches the streaming kernels do not take) publishes
+// empty lists.  One CTA; warps 0 and 1 each compact one list.
 __device__ void publish_active(const int* cnt, const int* anchors, int n_anchor,
-                               const int* corrs, int n_corr, int* act, int* act_n, int* sctr,
-                               int n_sctr) {
+                               const int* corrs, int n_corr, int blk, int* act, int* act_n,
+                               int* sctr, int n_sctr) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (warp < 2) {
     const int* list = warp == 0 ? anchors : corrs;
     const int n = warp == 0 ? n_anchor : n_corr;
-    int* out = act + (warp == 0 ? 0 : n_anchor);
+    int* out = act + (warp == 0 ? 0 : n_anchor * STREAM_DEP_TB);
     int base = 0;
-    for (int i0 = 0; i0 < n; i0 += 32) {
+    for (int i0 = 0; i0 < n && blk > 0; i0 += 32) {
       const int i = i0 + lane;
       const int node = i < n ? list[i] : -1;
-      const bool a = node >= 0 && cnt[node] > 0;
-      const uint32_t b = __ballot_sync(0xffffffffu, a);
-      if (a) out[base + __popc(b & ((1u << lane) - 1u))] = node;
-      base += __popc(b);
+      // blocks of this node's bucket (the host passes blk only for batches of
+      // at most STREAM_DEP_TB blocks)
+      const int nb = node >= 0 ? (cnt[node] + blk - 1) / blk : 0;
+      int incl = nb;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int x = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += x;
+      }
+      for (int b = 0; b < nb; ++b) out[base + incl - nb + b] = node * STREAM_DEP_TB + b;
+      base += __shfl_sync(0xffffffffu, incl, 31);
     }
     if (lane == 0) act_n[warp] = base;
   }
@@ -137,10 +146,12 @@ __global__ void k_offsets_plan(const int* __restrict__ key_cnt, int N, int E,
                                int* __restrict__ key_off, const int* __restrict__ rank,
                                int* __restrict__ tile_off, int max_items, PlanArgs pa,
                                const int* __restrict__ anchors, int n_anchor,
-                               const int* __restrict__ corrs, int n_corr, int* __restrict__ act,
-                               int* __restrict__ act_n, int* __restrict__ sctr, int n_sctr) {
+                               const int* __restrict__ corrs, int n_corr, int blk,
+                               int* __restrict__ act, int* __restrict__ act_n,
+                               int* __restrict__ sctr, int n_sctr) {
   pdl_wait();
-  if (act) publish_active(key_cnt, anchors, n_anchor, corrs, n_corr, act, act_n, sctr, n_sctr);
+  if (act)
+    publish_active(key_cnt, anchors, n_anchor, corrs, n_corr, blk, act, act_n, sctr, n_sctr);
   // node offsets then expert offsets
   for (int part = 0; part < 2; ++part) {
     const int n0 = part == 0 ? 0 : N, cnt = part == 0 ? N : E;
@@ -247,7 +258,7 @@ k_bucket_small(const float* __restrict__ logits, const int* __restrict__ ids_in,
                int* __restrict__ node_tok, int* __restrict__ row_node, int* __restrict__ node_row,
                int* __restrict__ perm, int* __restrict__ tile_off, int max_items, PlanArgs pa,
                const int* __restrict__ anchors, int n_anchor, const int* __restrict__ corrs,
-               int n_corr, int* __restrict__ act, int* __restrict__ act_n,
+               int n_corr, int blk, int* __restrict__ act, int* __restrict__ act_n,
                int* __restrict__ sctr, int n_sctr) {
   pdl_wait();
   extern __shared__ __align__(16) unsigned char sm[];
@@ -331,7 +342,7 @@ k_bucket_small(const float* __restrict__ logits, const int* __restrict__ ids_in,
     __syncthreads();
   }
   for (int i = tid; i < keys + 2; i += nth) key_off_g[i] = off[i];
-  publish_active(cnt, anchors, n_anchor, corrs, n_corr, act, act_n, sctr, n_sctr);
+  publish_active(cnt, anchors, n_anchor, corrs, n_corr, blk, act, act_n, sctr, n_sctr);
   // 5. tile plans: one warp per plan
   for (int p = warp; p < pa.n_plans; p += nw) {
     int* to = tile_off + (pa.first + p) * (max_items + 1);
@@ -394,6 +405,13 @@ static PlanArgs make_plans(const lx_layer* L, int n_plans, int first = 0) {
   return pa;
 }
 
+// Token rows per streaming work item, or 0 for batches the streaming kernels
+// do not take (more blocks than the dependency counters cover).
+static int stream_item_rows(int T) {
+  const int blk = stream_tile_tokens();
+  return T <= STREAM_DEP_TB * blk ? blk : 0;
+}
+
 bool bucket_small_fits(const lx_layer* L, int T, int k) {
   return T <= SB_MAX_T &&
          sb_smem(T, k, L->N + L->E, L->E, L->N, op_max_items(L)) <= SB_SMEM_LIMIT;
@@ -411,8 +429,9 @@ lx_status launch_bucket_small(lx_layer* L, const float* logits, const int* ids_i
                                              L->d_paths, L->d_path_len, L->d_rank, topk_id, topk_w,
                                              w.key_off, w.node_tok, w.row_node, w.node_row, w.perm,
                                              w.tile_off, op_max_items(L), pa, L->d_anchors,
-                                             L->n_anchor, L->d_corrs, L->n_corr, w.act, w.act_n,
-                                             w.sctr, sctr_ints(L));
+                                             L->n_anchor, L->d_corrs, L->n_corr,
+                                             stream_item_rows(T), w.act, w.act_n, w.sctr,
+                                             sctr_ints(L));
   LX_CUDA(cudaGetLastError());
   return LX_OK;
 }
@@ -442,7 +461,8 @@ lx_status launch_bucket(lx_layer* L, const int* topk_id, int T, int k, cudaStrea
     ProfScope ps(L, s, "bucket_offsets");
     launch_k(L, k_offsets_plan, 1, 1024, 0, s, w.key_cnt, L->N, L->E, w.key_off, L->d_rank, w.tile_off,
                                       op_max_items(L), pa, L->d_anchors, L->n_anchor, L->d_corrs,
-                                      L->n_corr, w.act, w.act_n, w.sctr, sctr_ints(L));
+                                      L->n_corr, stream_item_rows(T), w.act, w.act_n, w.sctr,
+                                      sctr_ints(L));
     LX_CUDA(cudaGetLastError());
   }
   {
@@ -547,8 +567,8 @@ extern "C" lx_status lx_bucket_noalloc(lx_layer* L, const int32_t* topk_id, int3
   LX_CUDA(cudaGetLastError());
   const PlanArgs pa = make_plans(L, N_OPS);
   k_offsets_plan<<<1, 1024, 0, s>>>(key_cnt, L->N, L->E, key_off, L->d_rank, tile_off,
-                                    op_max_items(L), pa, nullptr, 0, nullptr, 0, nullptr, nullptr,
-                                    nullptr, 0);
+                                    op_max_items(L), pa, nullptr, 0, nullptr, 0, 0, nullptr,
+                                    nullptr, nullptr, 0);
   LX_CUDA(cudaGetLastError());
   k_scatter<<<dim3((T + 255) / 256, (unsigned)keys), 256, 0, s>>>(
       marks, rank_in, key_off, topk_id, T, k, L->N, Tp, node_tok, row_node, perm);

@@ -162,7 +162,7 @@ struct GemmArgs {
 // Streaming (decode) grouped GEMM: one op of a launch
 struct StreamOp {
   const CUtensorMap* tmaps;  // [n_nodes] weight tensor maps of this op
-  const int* items;          // active node ids (compact list written by the bucketing)
+  const int* items;          // work items node * STREAM_DEP_TB + token block (written by the bucketing)
   const int* n_active;       // device count of items
   int n_items;               // upper bound of the count (host)
   const int* tile_off;       // [n_items+1] stream plan
@@ -178,7 +178,6 @@ struct StreamOp {
   const int* rank;
   int ncol_max;              // column tiles of the widest node of this op
   int ncb;                   // 64-row column blocks per tile
-  int ntb;                   // token blocks (64 tokens) of the largest possible bucket
   // split-K: K-range s of a tile (kbs 64-wide K blocks) writes fp32 partial s
   // to split_out + s * split_stride (`out` is not written)
   int nsplit;
@@ -272,7 +271,8 @@ struct Workspace {
   __nv_bfloat16* Pb = nullptr;  // [Rmax][2 rmax]
   __nv_bfloat16* zb = nullptr;  // [Rmax][I]
   __nv_bfloat16* Qb = nullptr;  // [Rmax][rmax]
-  int* act = nullptr;           // [n_anchor + n_corr] active anchors, then active corrections
+  int* act = nullptr;           // [STREAM_DEP_TB * (n_anchor + n_corr)] streaming work items:
+                                // (anchor, token block) pairs, then (correction, token block)
   int* act_n = nullptr;         // [2] their counts
   int* sctr = nullptr;          // [sctr_ints] streaming / tensor-core tile counters, then the
                                 // streaming launches' dependency counters [2][N][STREAM_DEP_TB]

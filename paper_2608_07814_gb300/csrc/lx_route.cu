@@ -12,7 +12,8 @@
 // for a slice of the experts (one expert per warp, so that a decode batch
 // still spreads the 0.5 MB router matrix over many SMs).  Each warp owns one
 // expert at a time and issues its weight loads in groups of 8 independent
-// 16-byte loads before using them.
+// 16-byte loads before using them; the first group goes out before the wait
+// for the preceding kernel, since the router matrix does not depend on it.
 //
 // Large bf16 batches (k_router_tiled): persistent CTAs walk tiles of 8
 // tokens.  A thread holds the lane partials of 8 tokens x 8 experts for its
@@ -65,34 +66,47 @@ k_router_logits(const T* __restrict__ x, const T* __restrict__ W, const float* _
                 int Ttok, int E, int H, int experts_per_cta, float* __restrict__ logits,
                 int* __restrict__ tile_cnt, int k, int* __restrict__ topk_id,
                 float* __restrict__ topk_w) {
-  pdl_wait();
   extern __shared__ __align__(16) unsigned char smem[];
   T* xs = reinterpret_cast<T*>(smem);
   const int t0 = blockIdx.x * RT_TOK;
   const int nt = min(RT_TOK, Ttok - t0);
   const int e_begin = blockIdx.y * experts_per_cta;
   const int e_end = min(E, e_begin + experts_per_cta);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
+  const int nchunk = H / 8;
+  // weight chunks q0 + 32u (u < RT_PREF) of expert e: independent 16-byte loads
+  float wv[RT_PREF][8];
+  auto load_w = [&](int e, int q0) {
+#pragma unroll
+    for (int u = 0; u < RT_PREF; ++u) {
+      const int q = q0 + 32 * u;
+      if (q < nchunk) load8(W + (size_t)e * H + 8 * q, wv[u]);
+    }
+  };
+  // The router matrix is a layer constant: the first expert's weights are
+  // requested before the wait for the preceding kernel (which may write x).
+  int e = e_begin + warp;
+  if (e < e_end) load_w(e, lane);
+  pdl_wait();
   {
+    // the token tile: every 16-byte piece in flight at once
     const int vec_per_tok = H * (int)sizeof(T) / 16;
     const uint4* src = reinterpret_cast<const uint4*>(x + (size_t)t0 * H);
     uint4* dst = reinterpret_cast<uint4*>(xs);
-    for (int i = threadIdx.x; i < nt * vec_per_tok; i += blockDim.x) dst[i] = src[i];
+    for (int i = threadIdx.x; i < nt * vec_per_tok; i += blockDim.x) {
+      const uint32_t da = static_cast<uint32_t>(__cvta_generic_to_shared(dst + i));
+      asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(da), "l"(src + i) : "memory");
+    }
+    asm volatile("cp.async.commit_group;" ::: "memory");
+    asm volatile("cp.async.wait_group 0;" ::: "memory");
   }
   __syncthreads();
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
-  const int nchunk = H / 8;
-  for (int e = e_begin + warp; e < e_end; e += nw) {
+  for (; e < e_end; e += nw) {
     float acc[RT_TOK];
 #pragma unroll
     for (int tt = 0; tt < RT_TOK; ++tt) acc[tt] = 0.f;
-    const T* w = W + (size_t)e * H;
     for (int q0 = lane; q0 < nchunk; q0 += 32 * RT_PREF) {
-      float wv[RT_PREF][8];
-#pragma unroll
-      for (int u = 0; u < RT_PREF; ++u) {
-        const int q = q0 + 32 * u;
-        if (q < nchunk) load8(w + 8 * q, wv[u]);
-      }
+      if (q0 != lane) load_w(e, q0);  // the expert's first chunks are already loaded
 #pragma unroll
       for (int u = 0; u < RT_PREF; ++u) {
         const int q = q0 + 32 * u;
@@ -119,6 +133,7 @@ k_router_logits(const T* __restrict__ x, const T* __restrict__ W, const float* _
       for (int tt = 0; tt < nt; ++tt)
         logits[(size_t)(t0 + tt) * E + e] = bias ? __fadd_rn(acc[tt], b) : acc[tt];
     }
+    if (e + nw < e_end) load_w(e + nw, lane);  // the next expert's first chunks
   }
   // The last CTA to finish this token tile's expert slices takes its top-k
   // (no CTA waits for another; the counter is reset for the next call).

@@ -1,7 +1,7 @@
 // Weight-streaming grouped GEMM for small token counts (decode).
 //
 // out[rows of node n][cols] = X[rows][K] . W_n[cols][K]^T for every active node,
-// where X holds at most 64 rows per tile.  Decode is bound by reading each
+// where X holds at most 32 rows per tile.  Decode is bound by reading each
 // touched weight byte once from HBM (Sec. 5.2: the projections run at about one
 // FLOP per byte), so the kernel is organised around the weight stream:
 //
@@ -9,9 +9,9 @@
 //     over the full K or, for the anchors, one of up to four K ranges (split-K:
 //     every range writes an fp32 partial that the next kernel adds in order),
 //     so that the tiles left at the end of a launch are short;
-//   * a producer warp streams the tile's weights with 2-D TMA loads
+//   * a producer warp streams the tile's weights with TMA loads
 //     (cp.async.bulk.tensor, 64x64 bf16 boxes, 128-byte swizzle) into a
-//     4-stage shared-memory ring guarded by mbarriers;
+//     3-stage shared-memory ring guarded by mbarriers;
 //   * two consumer warps (32 weight rows each) multiply with mma.sync
 //     m16n8k16 (weights as the 16-row operand, tokens as the 8-column
 //     operand).  Inside each 64-wide K box the contraction index is
@@ -19,7 +19,8 @@
 //     row and of a token row (16-byte shared loads, conflict-free under the
 //     128-byte swizzle); the same permutation on both operands leaves the sum
 //     unchanged;
-//   * persistent CTAs walk a device-built tile list; every mbarrier wait is
+//   * persistent CTAs claim tiles from a device-built list of (node, token
+//     block) work items, each near the end of the previous tile; every mbarrier wait is
 //     bounded, and a wait that gives up records LX_ERR_TIMEOUT in a device
 //     word and drains the CTA's copies in flight before returning.
 #include <cuda.h>
@@ -58,6 +59,9 @@ constexpr int SW_CONSUMERS = 2;
 constexpr int SW_MT = SW_ROWS / (16 * SW_CONSUMERS);  // 16-row MMA tiles per consumer warp
 constexpr int SW_THREADS = 32 * (1 + SW_CONSUMERS);
 constexpr unsigned long long SW_TIMEOUT_CYCLES = 4000000000ull;  // ~2 s
+// stages of the current tile still to be issued when the next tile is decoded
+// (measured at a decode batch of 64: 1 before 3 before 6)
+constexpr int kClaimLead = 1;
 static_assert(SW_STAGE_BYTES % 1024 == 0, "stages must keep the 128B-swizzle alignment");
 static_assert(SW_TOK % 8 == 0 && SW_TOK <= 64, "token slot: whole 8-token MMA columns");
 
@@ -183,7 +187,7 @@ struct TileInfo {
 };
 
 __device__ __forceinline__ int op_tiles(const StreamOp& op) {
-  return *op.n_active * op.ntb * op.shape.groups * op.ncol_max * op.nsplit;
+  return *op.n_active * op.shape.groups * op.ncol_max * op.nsplit;
 }
 
 // Tile index -> (op, node, token block, group, column tile, K split).
@@ -199,17 +203,15 @@ __device__ __forceinline__ void decode_tile(const StreamLaunch& P, int tile, int
     local = tile - tiles0;
   }
   const StreamOp& op = P.op[o];
-  // (item, token block, group, column tile, split), split fastest
-  const int per_tb = op.shape.groups * op.ncol_max * op.nsplit;
-  const int per_item = op.ntb * per_tb;
+  // (work item = node and token block, group, column tile, split), split fastest
+  const int per_item = op.shape.groups * op.ncol_max * op.nsplit;
   const int item = local / per_item;
   int rem = local - item * per_item;
-  const int tb = rem / per_tb;
-  rem -= tb * per_tb;
   const int grp = rem / (op.ncol_max * op.nsplit);
   rem -= grp * op.ncol_max * op.nsplit;
   const int ct = rem / op.nsplit, split = rem - ct * op.nsplit;
-  const int n = op.items[item];
+  const int packed = op.items[item];
+  const int n = packed / STREAM_DEP_TB, tb = packed - n * STREAM_DEP_TB;
   const int r = op.rank[n];
   const int b0 = op.node_off[n], b1 = op.node_off[n + 1];
   ti.op = o;
@@ -363,9 +365,10 @@ k_stream_gemm(const __grid_constant__ StreamLaunch P) {
   __syncthreads();
   uint32_t it = 0;
   if (warp == 0) {
-    // ---- producer warp.  Tiles are claimed from the launch's counter one
-    // ahead of use; the decoded tile rides in the shared slot of its first
-    // stage.  Lane 0 waits and issues the weight box, all lanes copy token rows.
+    // ---- producer warp.  Tiles are claimed from the launch's counter while
+    // the previous tile's last stages stream; the decoded tile rides in the
+    // shared slot of its first stage.  Lane 0 waits and issues the weight box,
+    // all lanes copy token rows.
     const int tiles0 = op_tiles(P.op[0]);
     const int tiles1 = tiles0 + (P.n_ops > 1 ? op_tiles(P.op[1]) : 0);
     const int total = tiles1 + (P.n_ops > 2 ? op_tiles(P.op[2]) : 0);
@@ -385,8 +388,11 @@ k_stream_gemm(const __grid_constant__ StreamLaunch P) {
         }
       }
     };
-    int cur = lane == 0 ? atomicAdd(P.ctr, 1) : 0;
-    cur = __shfl_sync(0xffffffffu, cur, 0);
+    // CTA b starts on tile b; later tiles come from the counter, offset by the
+    // grid (a first claim by every CTA at once would be a contended round
+    // trip).  A factor-product tile among the first ones waits only for tiles
+    // of lower index, i.e. of CTAs dispatched no later than its own.
+    int cur = blockIdx.x;
     TileInfo ti;
     if (cur < total) {
       decode_tile(P, cur, tiles0, tiles1, ti);
@@ -417,15 +423,21 @@ k_stream_gemm(const __grid_constant__ StreamLaunch P) {
     int buf = 0;
     bool ok = true;
     while (cur < total && ok) {
-      int nxt = lane == 0 ? atomicAdd(P.ctr, 1) : 0;  // next claim in flight
+      int nxt = 0;
       TileInfo tn;
-      bool prepared = false;
+      bool claimed = false, prepared = false;
       if (ti.active) {
         const StreamOp& op = P.op[ti.op];
         const CUtensorMap* map = op.tmaps + ti.node;
         const int rt0 = (ti.grp * ti.Ng + ti.row0) / SW_ROWS;
         const __nv_bfloat16* const* xs = xsrc + buf * SW_TOK;
         const int nkb = ti.nkb, kb0 = ti.kb0;
+        // The next tile is claimed kClaimLead stages before this tile's last
+        // one and decoded a stage later: a tile claimed earlier would wait
+        // behind a long one (whole-K factor tiles stream 32 stages) instead of
+        // going to a CTA that is about to be free.
+        const int nst = ti.ncb * nkb;
+        const int jd = max(nst - 1 - kClaimLead, min(1, nst - 1)), jc = max(jd - 1, 0);
         if (op.dep) {
           // the token rows of this tile are written by another op of this
           // launch: wait for every column tile of them (both consumer warps'
@@ -441,6 +453,11 @@ k_stream_gemm(const __grid_constant__ StreamLaunch P) {
         }
         for (int cb = 0; cb < ti.ncb && ok; ++cb) {
           for (int kb = 0; kb < nkb; ++kb, ++it) {
+            const int j = cb * nkb + kb;
+            if (j == jc) {
+              if (lane == 0) nxt = (int)gridDim.x + atomicAdd(P.ctr, 1);  // in flight until j == jd
+              claimed = true;
+            }
             const uint32_t s = it % SW_STAGES;
             int good = 1;
             const bool pre = it < npre;  // weight box issued before the dependency wait
@@ -475,7 +492,7 @@ k_stream_gemm(const __grid_constant__ StreamLaunch P) {
               }
             }
             cp_async_arrive(full0 + 8 * s);
-            if (!prepared && cb == 0 && (kb == 1 || kb == nkb - 1)) {
+            if (j == jd) {
               // the next tile: decode and prepare its rows while these stages stream
               nxt = __shfl_sync(0xffffffffu, nxt, 0);
               if (nxt < total) {
@@ -490,6 +507,7 @@ k_stream_gemm(const __grid_constant__ StreamLaunch P) {
           }
         }
       }
+      if (!claimed && lane == 0) nxt = (int)gridDim.x + atomicAdd(P.ctr, 1);
       if (!prepared) {
         nxt = __shfl_sync(0xffffffffu, nxt, 0);
         if (nxt < total) {
@@ -580,13 +598,13 @@ lx_status launch_stream(lx_layer* L, const StreamLaunch& P, cudaStream_t s, cons
 
 constexpr int kStreamUBlocks = 1;
 
-static StreamOp make_op(lx_layer* L, int op, int T, const __nv_bfloat16* X, long ldx,
+static StreamOp make_op(lx_layer* L, int op, const __nv_bfloat16* X, long ldx,
                         const int* gather, const CUtensorMap* xmap, void* out, long ldo,
                         bool out_f32) {
   StreamOp o;
   o.shape = op_shape(L, op);
   o.tmaps = L->d_tmaps + (size_t)op * L->N;
-  o.items = o.shape.on_anchors ? L->ws.act : L->ws.act + L->n_anchor;
+  o.items = L->ws.act + (o.shape.on_anchors ? 0 : (size_t)L->n_anchor * STREAM_DEP_TB);
   o.n_active = L->ws.act_n + (o.shape.on_anchors ? 0 : 1);
   o.n_items = o.shape.on_anchors ? L->n_anchor : L->n_corr;
   o.tile_off = nullptr;
@@ -606,7 +624,6 @@ static StreamOp make_op(lx_layer* L, int op, int T, const __nv_bfloat16* X, long
   // a tile streams more than two stages
   o.ncb = (op == OP_UP_U || op == OP_DN_U) ? kStreamUBlocks : 1;
   o.ncol_max = ((ng_max + SW_ROWS - 1) / SW_ROWS + o.ncb - 1) / o.ncb;
-  o.ntb = (T + SW_TOK - 1) / SW_TOK;
   o.nsplit = 1;
   o.kbs = 1 << 20;
   o.split_out = nullptr;
@@ -671,11 +688,11 @@ lx_status launch_fast_experts(lx_layer* L, const void* x, int T, int k, void* y,
   int* dep_dn = dep_up + (size_t)L->N * STREAM_DEP_TB;
   // x-side: x V of every correction (whole-K tiles, claimed first), the shared
   // anchor gate/up in split-K slices, then the corrections' U products
-  StreamOp up_v = make_op(L, OP_UP_V, T, xb, H, w.node_tok, nullptr, w.Pb, 2 * rmax, false);
+  StreamOp up_v = make_op(L, OP_UP_V, xb, H, w.node_tok, nullptr, w.Pb, 2 * rmax, false);
   up_v.sig = dep_up;
-  StreamOp up_a = make_op(L, OP_UP_ANCHOR, T, xb, H, w.node_tok, nullptr, w.hb, 2 * I, false);
+  StreamOp up_a = make_op(L, OP_UP_ANCHOR, xb, H, w.node_tok, nullptr, w.hb, 2 * I, false);
   if (split) split_op(L, up_a, w.hsplit, w.split_rows * 2 * I, kStreamSplitBlocksUp);
-  StreamOp up_u = make_op(L, OP_UP_U, T, w.Pb, 2 * rmax, nullptr, w.smaps + 0, w.hb, 2 * I, false);
+  StreamOp up_u = make_op(L, OP_UP_U, w.Pb, 2 * rmax, nullptr, w.smaps + 0, w.hb, 2 * I, false);
   up_u.dep = dep_up;
   up_u.dep_nrank = 2;  // P = [x Vg | x Vu]: 2r columns
   LX_TRY(run_stream(L, 0, {&up_v, &up_a, &up_u}, s, "stream_up"));
@@ -688,11 +705,11 @@ lx_status launch_fast_experts(lx_layer* L, const void* x, int T, int k, void* y,
   LX_TRY(launch_swiglu(L, T, k, true, s, hs));
   // z-side: z Vd of every correction first, the shared anchor down
   // projection, then the corrections' Ud products
-  StreamOp dn_v = make_op(L, OP_DN_V, T, w.zb, I, nullptr, w.smaps + 1, w.Qb, rmax, false);
+  StreamOp dn_v = make_op(L, OP_DN_V, w.zb, I, nullptr, w.smaps + 1, w.Qb, rmax, false);
   dn_v.sig = dep_dn;
-  StreamOp dn_a = make_op(L, OP_DN_ANCHOR, T, w.zb, I, nullptr, w.smaps + 1, w.yb, H, false);
+  StreamOp dn_a = make_op(L, OP_DN_ANCHOR, w.zb, I, nullptr, w.smaps + 1, w.yb, H, false);
   if (split) split_op(L, dn_a, w.ysplit, w.split_rows * H, kStreamSplitBlocksDown);
-  StreamOp dn_u = make_op(L, OP_DN_U, T, w.Qb, rmax, nullptr, w.smaps + 2, w.yb, H, false);
+  StreamOp dn_u = make_op(L, OP_DN_U, w.Qb, rmax, nullptr, w.smaps + 2, w.yb, H, false);
   dn_u.dep = dep_dn;
   dn_u.dep_nrank = 1;  // Q = z Vd: r columns
   LX_TRY(run_stream(L, 2, {&dn_v, &dn_a, &dn_u}, s, "stream_dn"));
