@@ -49,47 +49,58 @@ template <> __device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(flo
 // logit is never preferred; if only NaNs remain the lowest free id is taken,
 // so ids always stay in [0, E).
 // ---------------------------------------------------------------------------
-__device__ __forceinline__ bool topk_better(float v, int i, float bv, int bi) {
-  return v > bv || (v == bv && i < bi);
+// Order-preserving integer key of a non-NaN logit (+0 and -0 map alike, as
+// they compare equal); 0 marks "no candidate" and lies below every logit.
+__device__ __forceinline__ uint32_t topk_key(float v) {
+  const uint32_t u = __float_as_uint(v == 0.f ? 0.f : v);
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+__device__ __forceinline__ float topk_key_value(uint32_t key) {
+  return __uint_as_float((key & 0x80000000u) ? (key & 0x7fffffffu) : ~key);
 }
 
+// Each round: every lane's best free candidate (largest key, then lowest id),
+// the warp maximum of the keys and the lowest id holding it by two warp
+// reductions (redux.sync).
 template <int EPL>  // candidates per lane: E <= 32 * EPL
 __device__ __forceinline__ void warp_topk_t(const float* lt, int E, int k, int& sel_id,
                                             float& sel_w) {
   const int lane = threadIdx.x & 31;
-  float v[EPL];  // this lane's candidates e = lane + 32 i, in registers
+  uint32_t key[EPL];  // this lane's candidates e = lane + 32 i (0: absent or NaN)
 #pragma unroll
   for (int i = 0; i < EPL; ++i) {
     const int e = lane + 32 * i;
-    v[i] = e < E ? lt[e] : 0.f;
+    const float v = e < E ? lt[e] : 0.f;
+    key[i] = (e < E && v == v) ? topk_key(v) : 0u;
   }
   uint32_t taken = 0;  // bit i <-> expert lane + 32 i
   float m = 0.f, denom = 0.f, selv = 0.f;
   int seli = 0;
   for (int j = 0; j < k; ++j) {
-    float bv = -INFINITY;
-    int bi = 0x7fffffff;
+    uint32_t bk = 0;
+    int be = 0x7fffffff;
 #pragma unroll
     for (int i = 0; i < EPL; ++i) {
-      const int e = lane + 32 * i;
-      if (e < E && !((taken >> i) & 1u) && topk_better(v[i], e, bv, bi)) { bv = v[i]; bi = e; }
+      const uint32_t ki = ((taken >> i) & 1u) ? 0u : key[i];
+      if (ki > bk) {  // ascending i: the first of equal keys (lowest id) stays
+        bk = ki;
+        be = lane + 32 * i;
+      }
     }
-#pragma unroll
-    for (int off = 16; off >= 1; off >>= 1) {
-      const float ov = __shfl_xor_sync(0xffffffffu, bv, off);
-      const int oi = __shfl_xor_sync(0xffffffffu, bi, off);
-      if (topk_better(ov, oi, bv, bi)) { bv = ov; bi = oi; }
-    }
-    if (bi == 0x7fffffff) {  // only NaNs left: lowest free id
+    const uint32_t mk = __reduce_max_sync(0xffffffffu, bk);
+    int bi;
+    float bv;
+    if (mk != 0u) {
+      bi = __reduce_min_sync(0xffffffffu, bk == mk ? be : 0x7fffffff);
+      bv = topk_key_value(mk);
+    } else {  // only NaNs left: lowest free id
       int fi = 0x7fffffff;
 #pragma unroll
       for (int i = EPL - 1; i >= 0; --i) {
         const int e = lane + 32 * i;
         if (e < E && !((taken >> i) & 1u)) fi = e;
       }
-#pragma unroll
-      for (int off = 16; off >= 1; off >>= 1) fi = min(fi, __shfl_xor_sync(0xffffffffu, fi, off));
-      bi = fi;
+      bi = __reduce_min_sync(0xffffffffu, fi);
       bv = lt[bi];
     }
     if ((bi & 31) == lane) taken |= 1u << (bi >> 5);
@@ -386,6 +397,7 @@ struct ProfScope {
 // kernels / launchers (defined in the .cu files)
 lx_status launch_router(lx_layer* L, const void* x, int T, int k, float* logits, int* topk_id,
                         float* topk_w, cudaStream_t s);
+bool router_is_tiled(const lx_layer* L, int T);
 // plan_first: tile plans for the generic GEMMs (0), the tensor-core GEMMs
 // (PLAN_TC), or none (-1)
 lx_status launch_bucket(lx_layer* L, const int* topk_id, int T, int k, cudaStream_t s,

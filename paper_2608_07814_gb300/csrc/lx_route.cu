@@ -311,25 +311,29 @@ k_router_tiled(const __nv_bfloat16* __restrict__ x, const __nv_bfloat16* __restr
 
 }  // namespace
 
+bool router_is_tiled(const lx_layer* L, int T) {
+  const int tiles = (T + RT_TOK - 1) / RT_TOK;
+  return L->dtype == LX_BF16 && tiles >= L->num_sms && L->H % 8 == 0 &&
+         2 * (size_t)RTT_TOK * L->H * 2 + (size_t)RTT_TOK * L->E * 4 <= 200 * 1024;
+}
+
 lx_status launch_router(lx_layer* L, const void* x, int T, int k, float* logits, int* topk_id,
                         float* topk_w, cudaStream_t s) {
   if (reinterpret_cast<uintptr_t>(x) % 16)
     return fail(LX_ERR_ARG, "x must be 16-byte aligned");
   const int tiles = (T + RT_TOK - 1) / RT_TOK;
-  if (L->dtype == LX_BF16 && tiles >= L->num_sms && L->H % 8 == 0) {
+  if (router_is_tiled(L, T)) {
     // large batch: persistent register-tiled kernel
     const size_t smem2 = 2 * (size_t)RTT_TOK * L->H * 2 + (size_t)RTT_TOK * L->E * 4;
-    if (smem2 <= 200 * 1024) {
-      static bool done_t[64] = {};
-      LX_CUDA(smem_cap_once((const void*)k_router_tiled, 200 * 1024, L->device, done_t));
-      ProfScope ps(L, s, "router");
-      const int grid = std::min(tiles, L->num_sms);
-      launch_k(L, k_router_tiled, grid, RTT_THREADS, smem2, s, 
-          (const __nv_bfloat16*)x, (const __nv_bfloat16*)L->router_w, L->router_bias, T, L->E,
-          L->H, logits, k, topk_id, topk_w);
-      LX_CUDA(cudaGetLastError());
-      return LX_OK;
-    }
+    static bool done_t[64] = {};
+    LX_CUDA(smem_cap_once((const void*)k_router_tiled, 200 * 1024, L->device, done_t));
+    ProfScope ps(L, s, "router");
+    const int grid = std::min(tiles, L->num_sms);
+    launch_k(L, k_router_tiled, grid, RTT_THREADS, smem2, s, (const __nv_bfloat16*)x,
+             (const __nv_bfloat16*)L->router_w, L->router_bias, T, L->E, L->H, logits, k, topk_id,
+             topk_w);
+    LX_CUDA(cudaGetLastError());
+    return LX_OK;
   }
   const size_t smem = std::max((size_t)RT_TOK * L->H * L->esz, (size_t)RT_TOK * L->E * 4);
   if (smem > 200 * 1024) return fail(LX_ERR_SHAPE, "router token tile exceeds shared memory");
