@@ -130,13 +130,23 @@ __device__ __forceinline__ bool dep_wait(const int* p, int need, volatile int* a
   }
 }
 
+// L2 policy of the weight boxes: every weight byte is read once per launch, so
+// its lines are evicted first and the activations, factor projections and
+// split-K partials the launch writes stay in L2 for the kernels that read them.
+__device__ __forceinline__ uint64_t evict_first_policy() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+
 // one 64x64 tile (box) of a tiled weight matrix: K tile kt of row tile rt
 __device__ __forceinline__ void tma_load_tile(uint32_t dst, const CUtensorMap* map, int kt, int rt,
-                                              uint32_t bar) {
+                                              uint32_t bar, uint64_t policy) {
   asm volatile(
       "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
-      " [%0], [%1, {%2, %3, %4, %5}], [%6];" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(0), "r"(0), "r"(kt), "r"(rt), "r"(bar)
+      ".L2::cache_hint [%0], [%1, {%2, %3, %4, %5}], [%6], %7;" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(0), "r"(0), "r"(kt), "r"(rt), "r"(bar),
+      "l"(policy)
       : "memory");
 }
 
@@ -369,6 +379,7 @@ k_stream_gemm(const __grid_constant__ StreamLaunch P) {
     // the previous tile's last stages stream; the decoded tile rides in the
     // shared slot of its first stage.  Lane 0 waits and issues the weight box,
     // all lanes copy token rows.
+    const uint64_t wpol = evict_first_policy();
     const int tiles0 = op_tiles(P.op[0]);
     const int tiles1 = tiles0 + (P.n_ops > 1 ? op_tiles(P.op[1]) : 0);
     const int total = tiles1 + (P.n_ops > 2 ? op_tiles(P.op[2]) : 0);
@@ -413,7 +424,7 @@ k_stream_gemm(const __grid_constant__ StreamLaunch P) {
             const uint32_t wbox = smem_base + kb * SW_STAGE_BYTES;
             if (kb == 0) slot[0] = ti;
             mbar_expect_tx(full0 + 8 * kb, SW_BOX_BYTES + (op.gather ? 0 : SW_XBYTES));
-            tma_load_tile(wbox, op.tmaps + ti.node, ti.kb0 + kb, rt0, full0 + 8 * kb);
+            tma_load_tile(wbox, op.tmaps + ti.node, ti.kb0 + kb, rt0, full0 + 8 * kb, wpol);
           }
         }
       }
@@ -475,7 +486,7 @@ k_stream_gemm(const __grid_constant__ StreamLaunch P) {
             }
             const uint32_t wbox = smem_base + s * SW_STAGE_BYTES;
             if (lane == 0) {
-              if (!pre) tma_load_tile(wbox, map, kb0 + kb, rt0 + cb, full0 + 8 * s);
+              if (!pre) tma_load_tile(wbox, map, kb0 + kb, rt0 + cb, full0 + 8 * s, wpol);
               // contiguous token rows: one box of SW_TOK rows (rows past the
               // bucket belong to the next node and are never stored)
               if (!op.gather)
