@@ -299,10 +299,9 @@ struct WarpRows {
   unsigned anchor_rows;  // bit d: distinct row d belongs to an anchor
 };
 
-__device__ __forceinline__ void warp_token_rows(const int* __restrict__ node_row_t, int kD, int D,
-                                                WarpRows& wr) {
+// v: entry `lane` of the token's node rows (-1 for lanes >= kD)
+__device__ __forceinline__ void warp_token_rows(int v, int kD, int D, WarpRows& wr) {
   const int lane = threadIdx.x & 31;
-  const int v = lane < kD ? node_row_t[lane] : -1;
   const int key = v >= 0 ? v : INT_MAX;
   const unsigned same = __match_any_sync(0xffffffffu, key);
   const bool first = key != INT_MAX && lane == __ffs(same) - 1;
@@ -434,7 +433,6 @@ __global__ void __launch_bounds__(WT_WARPS * 32, 2)
 k_swiglu_warp(const float* __restrict__ topk_w, const int* __restrict__ node_row, int T, int k,
               const TH* __restrict__ h, int I, TZ* __restrict__ z, int cols_per_item,
               const SplitParts hs) {
-  pdl_wait();
   extern __shared__ float zsm[];  // bf16 path: [warp][k * D rows][32 lanes * CPL]
   __shared__ WarpRows wrs[WT_WARPS];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -442,12 +440,24 @@ k_swiglu_warp(const float* __restrict__ topk_w, const int* __restrict__ node_row
   const int kD = k * D;
   const int per_tok = (I + cols_per_item - 1) / cols_per_item;
   const long items = (long)T * per_tok;
-  for (long it = (long)blockIdx.x * WT_WARPS + warp; it < items; it += (long)gridDim.x * WT_WARPS) {
+  long it = (long)blockIdx.x * WT_WARPS + warp;
+  // The routing tables (node rows, gates) come from the routing and bucketing
+  // kernels, at least two launches before this one: the first item's entries
+  // are loaded before the wait for the preceding kernel.
+  int v_pre = -1;
+  float g_pre = 0.f;
+  if (it < items) {
+    const int t = (int)(it / per_tok);
+    if (lane < kD) v_pre = node_row[(size_t)t * kD + lane];
+    if (lane < k) g_pre = topk_w[(size_t)t * k + lane];
+  }
+  pdl_wait();
+  for (bool first = true; it < items; it += (long)gridDim.x * WT_WARPS, first = false) {
     const int t = (int)(it / per_tok);
     const int c_begin = (int)(it % per_tok) * cols_per_item;
     const int c_end = min(I, c_begin + cols_per_item);
-    warp_token_rows(node_row + (size_t)t * kD, kD, D, wr);
-    if (lane < k) wr.g[lane] = topk_w[(size_t)t * k + lane];
+    warp_token_rows(first ? v_pre : (lane < kD ? node_row[(size_t)t * kD + lane] : -1), kD, D, wr);
+    if (lane < k) wr.g[lane] = first ? g_pre : topk_w[(size_t)t * k + lane];
     __syncwarp();
     const int nd = wr.nd;
     for (int c = c_begin + CPL * lane; c < c_end; c += 32 * CPL) {
@@ -591,18 +601,23 @@ template <typename TP, typename TY, int CPL, bool SPLIT>
 __global__ void __launch_bounds__(WT_WARPS * 32, 2)
 k_combine_warp(const int* __restrict__ node_row, int k, int D, const TP* __restrict__ ypart,
                int H, TY* __restrict__ y, int T, int cols_per_item, const SplitParts ys) {
-  pdl_wait();
   __shared__ WarpRows wrs[WT_WARPS];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   WarpRows& wr = wrs[warp];
   const int kD = k * D;
   const int per_tok = (H + cols_per_item - 1) / cols_per_item;
   const long items = (long)T * per_tok;
-  for (long it = (long)blockIdx.x * WT_WARPS + warp; it < items; it += (long)gridDim.x * WT_WARPS) {
+  long it = (long)blockIdx.x * WT_WARPS + warp;
+  // node rows come from the bucketing, several launches before this one: the
+  // first item's entries are loaded before the wait for the preceding kernel
+  int v_pre = -1;
+  if (it < items && lane < kD) v_pre = node_row[(size_t)(it / per_tok) * kD + lane];
+  pdl_wait();
+  for (bool first = true; it < items; it += (long)gridDim.x * WT_WARPS, first = false) {
     const int t = (int)(it / per_tok);
     const int c_begin = (int)(it % per_tok) * cols_per_item;
     const int c_end = min(H, c_begin + cols_per_item);
-    warp_token_rows(node_row + (size_t)t * kD, kD, D, wr);
+    warp_token_rows(first ? v_pre : (lane < kD ? node_row[(size_t)t * kD + lane] : -1), kD, D, wr);
     const int nd = wr.nd;
     for (int c = c_begin + CPL * lane; c < c_end; c += 32 * CPL) {
       Cols<CPL> acc;
