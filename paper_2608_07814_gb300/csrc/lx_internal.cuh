@@ -139,7 +139,7 @@ enum OpKind {
 // Tile plans (prefix of the tiles per node, built by the bucketing): plan p <
 // N_OPS is op p for the generic kernel (32-token x 64-column tiles); plan
 // PLAN_TC + p is op p for the tensor-core kernel (128 tokens x 256 columns).
-// The streaming kernels decode their tiles from the active-node lists instead.
+// The streaming kernels decode their tiles from the streaming work items instead.
 constexpr int N_PLANS = 2 * N_OPS;
 constexpr int PLAN_TC = N_OPS;
 constexpr int N_TILE_COUNTERS = 16;  // dynamic tile counters, zeroed by the bucketing

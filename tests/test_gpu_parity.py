@@ -234,16 +234,22 @@ def test_ties_go_to_lower_id():
             assert sorted(pos, key=pos.get) == sorted(pos)
 
 
-def test_all_tokens_on_one_cluster():
+@pytest.mark.parametrize("T", [70, 255, 256])
+def test_all_tokens_on_one_cluster(T):
+    """Every token on one cluster of a streaming-capable layer: each of its
+    nodes' buckets spans up to the largest number of 32-token work items the
+    streaming path takes (8 at 256 tokens, one ragged at 255)."""
     src = synth.flat_layer(256, 128, [4] * 4, 64, 4, "bf16", seed=10, factor_std="visible")
     src.router_bias = np.zeros(16, np.float32)
     src.router_bias[src.meta["clusters"][2]] = 50.0
     L = lx.Layer(src)
-    x = synth.tokens(src, 70, seed=2)
+    assert L.info()["stream_path"] == 1
+    x = synth.tokens(src, T, seed=2)
     ids, _ = check_route(src, L, x, 4)
     assert set(np.unique(ids)) == set(src.meta["clusters"][2])
     check_buckets(src, L, ids)
     check_forward(src, L, x, 4)
+    assert L.info()["device_error"] == 0
 
 
 def test_zero_tokens_is_noop():
