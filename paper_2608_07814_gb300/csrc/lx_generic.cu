@@ -346,7 +346,12 @@ struct Cols {
 template <int CPL>
 __device__ __forceinline__ Cols<CPL> ld_cols(const float* p) {
   Cols<CPL> r;
-  if constexpr (CPL == 4) {
+  if constexpr (CPL == 8) {
+    const float4 f = __ldg(reinterpret_cast<const float4*>(p));
+    const float4 g = __ldg(reinterpret_cast<const float4*>(p + 4));
+    r.v[0] = f.x; r.v[1] = f.y; r.v[2] = f.z; r.v[3] = f.w;
+    r.v[4] = g.x; r.v[5] = g.y; r.v[6] = g.z; r.v[7] = g.w;
+  } else if constexpr (CPL == 4) {
     const float4 f = __ldg(reinterpret_cast<const float4*>(p));
     r.v[0] = f.x; r.v[1] = f.y; r.v[2] = f.z; r.v[3] = f.w;
   } else if constexpr (CPL == 2) {
@@ -361,7 +366,15 @@ __device__ __forceinline__ Cols<CPL> ld_cols(const float* p) {
 template <int CPL>
 __device__ __forceinline__ Cols<CPL> ld_cols(const __nv_bfloat16* p) {
   Cols<CPL> r;
-  if constexpr (CPL == 4) {
+  if constexpr (CPL == 8) {
+    const uint4 u = __ldg(reinterpret_cast<const uint4*>(p));
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      r.v[2 * i] = __uint_as_float(w[i] << 16);
+      r.v[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+    }
+  } else if constexpr (CPL == 4) {
     const uint2 u = __ldg(reinterpret_cast<const uint2*>(p));
     r.v[0] = __uint_as_float(u.x << 16); r.v[1] = __uint_as_float(u.x & 0xFFFF0000u);
     r.v[2] = __uint_as_float(u.y << 16); r.v[3] = __uint_as_float(u.y & 0xFFFF0000u);
@@ -410,7 +423,19 @@ __device__ __forceinline__ void add_raw(Cols<CPL>& a, const RawB<CPL>& r, bool v
 }
 template <typename T, int CPL>
 __device__ __forceinline__ void st_cols(T* p, const Cols<CPL>& c) {
-  if constexpr (CPL == 4) {
+  if constexpr (CPL == 8 && std::is_same<T, __nv_bfloat16>::value) {
+    uint4 u;
+    uint32_t* w = reinterpret_cast<uint32_t*>(&u);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const __nv_bfloat162 b = __floats2bfloat162_rn(c.v[2 * i], c.v[2 * i + 1]);
+      w[i] = *reinterpret_cast<const uint32_t*>(&b);
+    }
+    *reinterpret_cast<uint4*>(p) = u;
+  } else if constexpr (CPL == 8) {
+    store4<T>(p, make_float4(c.v[0], c.v[1], c.v[2], c.v[3]));
+    store4<T>(p + 4, make_float4(c.v[4], c.v[5], c.v[6], c.v[7]));
+  } else if constexpr (CPL == 4) {
     store4<T>(p, make_float4(c.v[0], c.v[1], c.v[2], c.v[3]));
   } else if constexpr (CPL == 2 && std::is_same<T, __nv_bfloat16>::value) {
     *reinterpret_cast<__nv_bfloat162*>(p) = __floats2bfloat162_rn(c.v[0], c.v[1]);
@@ -676,7 +701,7 @@ k_combine_warp(const int* __restrict__ node_row, int k, int D, const TP* __restr
 }  // namespace
 
 bool warp_kernels_fit(const lx_layer* L, int k) {
-  return k <= WT_SLOTS && k * L->max_depth <= 32 && L->I % 4 == 0 && L->H % 4 == 0;
+  return k <= WT_SLOTS && k * L->max_depth <= 32 && L->I % 4 == 0 && L->H % 8 == 0;
 }
 
 // Columns per warp work item: whole rows when the batch alone fills the GPU
@@ -756,14 +781,23 @@ template <typename TP, typename TY>
 static void launch_combine_warp(lx_layer* L, int T, int k, const TP* ypart, TY* y, cudaStream_t s,
                                 const SplitParts& ys) {
   Workspace& w = L->ws;
-  const int cols = warp_item_cols(L, T, L->H, 128);
+  if (ys.splits > 1 || narrow_cols(L, T, L->H)) {
+    const int cols = warp_item_cols(L, T, L->H, 128);
+    const int grid = warp_grid(L, T, L->H, cols);
+    if (ys.splits > 1)
+      launch_k(L, k_combine_warp<TP, TY, 4, true>, grid, WT_WARPS * 32, 0, s, w.node_row, k,
+               L->max_depth, ypart, L->H, y, T, cols, ys);
+    else
+      launch_k(L, k_combine_warp<TP, TY, 4, false>, grid, WT_WARPS * 32, 0, s, w.node_row, k,
+               L->max_depth, ypart, L->H, y, T, cols, ys);
+    return;
+  }
+  // large batches: eight columns per lane (16-byte bf16 loads), half the
+  // per-element address and loop instructions of four
+  const int cols = warp_item_cols(L, T, L->H, 256);
   const int grid = warp_grid(L, T, L->H, cols);
-  if (ys.splits > 1)
-    launch_k(L, k_combine_warp<TP, TY, 4, true>, grid, WT_WARPS * 32, 0, s, w.node_row, k,
-             L->max_depth, ypart, L->H, y, T, cols, ys);
-  else
-    launch_k(L, k_combine_warp<TP, TY, 4, false>, grid, WT_WARPS * 32, 0, s, w.node_row, k,
-             L->max_depth, ypart, L->H, y, T, cols, ys);
+  launch_k(L, k_combine_warp<TP, TY, 8, false>, grid, WT_WARPS * 32, 0, s, w.node_row, k,
+           L->max_depth, ypart, L->H, y, T, cols, ys);
 }
 
 lx_status launch_swiglu(lx_layer* L, int T, int k, bool bf16, cudaStream_t s, SplitParts hs) {
