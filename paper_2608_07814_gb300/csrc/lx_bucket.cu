@@ -247,7 +247,7 @@ constexpr size_t SB_SMEM_LIMIT = 160 * 1024;
 __host__ __device__ inline size_t sb_smem(int T, int k, int keys, int E, int N, int max_items) {
   const size_t Tp = ((size_t)T + 15) / 16 * 16;
   return (size_t)T * k * 4 + 2 * (size_t)keys * Tp + (size_t)keys * 4 + ((size_t)keys + 2) * 4 +
-         (size_t)E * (LX_MAX_DEPTH + 1) * 4 + (size_t)N * 4 + 64;
+         (size_t)E * (LX_MAX_DEPTH + 1) * 4 + 2 * (size_t)N * 4 + 64;
 }
 
 __global__ void __launch_bounds__(SB_THREADS)
@@ -260,7 +260,6 @@ k_bucket_small(const float* __restrict__ logits, const int* __restrict__ ids_in,
                const int* __restrict__ anchors, int n_anchor, const int* __restrict__ corrs,
                int n_corr, int blk, int* __restrict__ act, int* __restrict__ act_n,
                int* __restrict__ sctr, int n_sctr) {
-  pdl_wait();
   extern __shared__ __align__(16) unsigned char sm[];
   const int keys = N + E;
   const int Tp = (T + 15) & ~15;
@@ -272,23 +271,28 @@ k_bucket_small(const float* __restrict__ logits, const int* __restrict__ ids_in,
   int* spaths = off + keys + 2;                 // [E][LX_MAX_DEPTH]
   int* splen = spaths + E * LX_MAX_DEPTH;       // [E]
   int* srank = splen + E;                       // [N]
+  int* slist = srank + N;                       // [N]: the anchors, then the corrections
   const int tid = threadIdx.x, nth = blockDim.x;
   const int warp = tid >> 5, lane = tid & 31, nw = nth >> 5;
+  // Before the wait for the preceding kernel: zeroed marks and the layer's
+  // tables (constants of the layer) staged in shared memory.
   {
     uint32_t* m32 = reinterpret_cast<uint32_t*>(marks);  // keys*Tp is a multiple of 16
     for (int i = tid; i < keys * Tp / 4; i += nth) m32[i] = 0;
   }
-  // the layer's tables and the given ids in one pass (one round trip)
   {
     const int n_paths = E * LX_MAX_DEPTH, n_tab = n_paths + E + N;
-    const int n_all = n_tab + (logits ? 0 : T * k);
-    for (int i = tid; i < n_all; i += nth) {
+    for (int i = tid; i < n_tab + N; i += nth) {
       if (i < n_paths) spaths[i] = paths[i];
       else if (i < n_paths + E) splen[i - n_paths] = path_len[i - n_paths];
       else if (i < n_tab) srank[i - n_paths - E] = rank[i - n_paths - E];
-      else ids[i - n_tab] = ids_in[i - n_tab];
+      else if (i < n_tab + n_anchor) slist[i - n_tab] = anchors[i - n_tab];
+      else slist[i - n_tab] = corrs[i - n_tab - n_anchor];
     }
   }
+  pdl_wait();
+  if (!logits)  // the given ids (written by the preceding kernel)
+    for (int i = tid; i < T * k; i += nth) ids[i] = ids_in[i];
   // 1. routing (or the given ids)
   if (logits) {
     for (int t = warp; t < T; t += nw) {
@@ -342,7 +346,7 @@ k_bucket_small(const float* __restrict__ logits, const int* __restrict__ ids_in,
     __syncthreads();
   }
   for (int i = tid; i < keys + 2; i += nth) key_off_g[i] = off[i];
-  publish_active(cnt, anchors, n_anchor, corrs, n_corr, blk, act, act_n, sctr, n_sctr);
+  publish_active(cnt, slist, n_anchor, slist + n_anchor, n_corr, blk, act, act_n, sctr, n_sctr);
   // 5. tile plans: one warp per plan
   for (int p = warp; p < pa.n_plans; p += nw) {
     int* to = tile_off + (pa.first + p) * (max_items + 1);
