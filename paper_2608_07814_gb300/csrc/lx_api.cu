@@ -133,7 +133,7 @@ static lx_status ensure_workspace(lx_layer* L, int T, int k, cudaStream_t s) {
   std::vector<Item> items = {
       {(void**)&w.logits, sizeof(float) * cT * L->E},
       {(void**)&w.topk_id, sizeof(int) * cT * ck},
-      {(void**)&w.tile_cnt, sizeof(int) * ((cT + 7) / 8)},
+      {(void**)&w.tile_cnt, sizeof(int) * std::max(1, router_tile_counters(cT))},
       {(void**)&w.topk_w, sizeof(float) * cT * ck},
       {(void**)&w.marks, (size_t)keys * Tp},
       {(void**)&w.rank_in, sizeof(int) * keys * Tp},
@@ -184,7 +184,7 @@ static lx_status ensure_workspace(lx_layer* L, int T, int k, cudaStream_t s) {
   w.base = base;
   w.bytes = total;
   e = cudaMemsetAsync(w.err, 0, sizeof(int), s);
-  if (e == cudaSuccess) e = cudaMemsetAsync(w.tile_cnt, 0, sizeof(int) * ((cT + 7) / 8), s);
+  if (e == cudaSuccess) e = cudaMemsetAsync(w.tile_cnt, 0, sizeof(int) * std::max(1, router_tile_counters(cT)), s);
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
   if (e != cudaSuccess) return cuda_fail(e, "clear workspace error word");
   w.cap_T = cT;

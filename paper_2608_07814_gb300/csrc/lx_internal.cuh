@@ -256,7 +256,7 @@ struct Workspace {
   // routing
   float* logits = nullptr;   // [T][E]
   int* topk_id = nullptr;    // [T][k]
-  int* tile_cnt = nullptr;   // [T/8] router slices done per token tile (self-resetting)
+  int* tile_cnt = nullptr;   // [router_tile_counters(T)] router slices done per token tile (self-resetting)
   float* topk_w = nullptr;   // [T][k]
   // bucketing
   uint8_t* marks = nullptr;  // [(N+E)][Tp]
@@ -398,6 +398,7 @@ struct ProfScope {
 lx_status launch_router(lx_layer* L, const void* x, int T, int k, float* logits, int* topk_id,
                         float* topk_w, cudaStream_t s);
 bool router_is_tiled(const lx_layer* L, int T);
+int router_tile_counters(int T);  // token tiles of the small-batch router
 // plan_first: tile plans for the generic GEMMs (0), the tensor-core GEMMs
 // (PLAN_TC), or none (-1)
 lx_status launch_bucket(lx_layer* L, const int* topk_id, int T, int k, cudaStream_t s,

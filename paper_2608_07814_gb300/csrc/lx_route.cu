@@ -8,7 +8,7 @@
 // multiply-adds, and the 32 lane partials are added pairwise at offsets
 // 16, 8, 4, 2, 1; the bias (if any) is added last.
 //
-// Small batches (k_router_logits): one CTA computes the logits of 8 tokens
+// Small batches (k_router_logits): one CTA computes the logits of 4 tokens
 // for a slice of the experts (one expert per warp, so that a decode batch
 // still spreads the 0.5 MB router matrix over many SMs).  Each warp owns one
 // expert at a time and issues its weight loads in groups of 8 independent
@@ -32,7 +32,7 @@ namespace lx {
 
 namespace {
 
-constexpr int RT_TOK = 8;        // tokens per CTA
+constexpr int RT_TOK = 4;        // tokens per CTA (measured at a decode batch of 64: 4 before 2, 8, 1)
 constexpr int RT_THREADS = 256;  // 8 warps
 constexpr int RT_PREF = 8;       // 16-byte weight loads in flight per lane
 
@@ -312,7 +312,7 @@ k_router_tiled(const __nv_bfloat16* __restrict__ x, const __nv_bfloat16* __restr
 }  // namespace
 
 bool router_is_tiled(const lx_layer* L, int T) {
-  const int tiles = (T + RT_TOK - 1) / RT_TOK;
+  const int tiles = (T + RTT_TOK - 1) / RTT_TOK;
   return L->dtype == LX_BF16 && tiles >= L->num_sms && L->H % 8 == 0 &&
          2 * (size_t)RTT_TOK * L->H * 2 + (size_t)RTT_TOK * L->E * 4 <= 200 * 1024;
 }
@@ -358,5 +358,7 @@ lx_status launch_router(lx_layer* L, const void* x, int T, int k, float* logits,
   LX_CUDA(cudaGetLastError());
   return LX_OK;
 }
+
+int router_tile_counters(int T) { return (T + RT_TOK - 1) / RT_TOK; }
 
 }  // namespace lx
