@@ -316,35 +316,46 @@ k_bucket_small(const float* __restrict__ logits, const int* __restrict__ ids_in,
     for (int l = 0; l < len; ++l) marks[spaths[e * LX_MAX_DEPTH + l] * Tp + t] = 1;
   }
   __syncthreads();
-  // 3. per-key ranks in token order (warp ballots)
-  for (int key = warp; key < keys; key += nw) {
-    int running = 0;
+  // 3. per-key ranks in token order (warp ballots; four keys per warp at a
+  // time, so that their ballot chains overlap)
+  for (int kb0 = warp; kb0 < keys; kb0 += 4 * nw) {
+    int running[4] = {0, 0, 0, 0};
     for (int t0 = 0; t0 < T; t0 += 32) {
       const int t = t0 + lane;
-      const bool m = t < T && marks[key * Tp + t];
-      const uint32_t b = __ballot_sync(0xffffffffu, m);
-      if (m) rk[key * Tp + t] = (uint8_t)(running + __popc(b & ((1u << lane) - 1u)));
-      running += __popc(b);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int key = kb0 + j * nw;
+        const bool m = key < keys && t < T && marks[key * Tp + t];
+        const uint32_t b = __ballot_sync(0xffffffffu, m);
+        if (m) rk[key * Tp + t] = (uint8_t)(running[j] + __popc(b & ((1u << lane) - 1u)));
+        running[j] += __popc(b);
+      }
     }
-    if (lane == 0) cnt[key] = running;
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      if (lane == 0 && kb0 + j * nw < keys) cnt[kb0 + j * nw] = running[j];
   }
   __syncthreads();
-  // 4. node offsets then expert offsets
-  for (int part = 0; part < 2; ++part) {
-    const int n0 = part == 0 ? 0 : N, n = part == 0 ? N : E;
-    const int o0 = part == 0 ? 0 : N + 1;
+  // 4. node offsets (warp 0) and expert offsets (warp 1): warp scans with a carry
+  if (warp < 2) {
+    const int n0 = warp == 0 ? 0 : N, n = warp == 0 ? N : E;
+    const int o0 = warp == 0 ? 0 : N + 1;
     int carry = 0;
-    for (int base = 0; base < n; base += nth) {
-      const int i = base + tid;
+    for (int base = 0; base < n; base += 32) {
+      const int i = base + lane;
       const int v = i < n ? cnt[n0 + i] : 0;
-      int total;
-      const int ex = block_excl_scan(v, &total);
-      if (i < n) off[o0 + i] = carry + ex;
-      carry += total;
+      int incl = v;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int x = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += x;
+      }
+      if (i < n) off[o0 + i] = carry + incl - v;
+      carry += __shfl_sync(0xffffffffu, incl, 31);
     }
-    if (tid == 0) off[o0 + n] = carry;
-    __syncthreads();
+    if (lane == 0) off[o0 + n] = carry;
   }
+  __syncthreads();
   for (int i = tid; i < keys + 2; i += nth) key_off_g[i] = off[i];
   publish_active(cnt, slist, n_anchor, slist + n_anchor, n_corr, blk, act, act_n, sctr, n_sctr);
   // 5. tile plans: one warp per plan

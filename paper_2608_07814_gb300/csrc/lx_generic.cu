@@ -781,19 +781,15 @@ template <typename TP, typename TY>
 static void launch_combine_warp(lx_layer* L, int T, int k, const TP* ypart, TY* y, cudaStream_t s,
                                 const SplitParts& ys) {
   Workspace& w = L->ws;
-  if (ys.splits > 1 || narrow_cols(L, T, L->H)) {
+  if (ys.splits > 1) {
     const int cols = warp_item_cols(L, T, L->H, 128);
     const int grid = warp_grid(L, T, L->H, cols);
-    if (ys.splits > 1)
-      launch_k(L, k_combine_warp<TP, TY, 4, true>, grid, WT_WARPS * 32, 0, s, w.node_row, k,
-               L->max_depth, ypart, L->H, y, T, cols, ys);
-    else
-      launch_k(L, k_combine_warp<TP, TY, 4, false>, grid, WT_WARPS * 32, 0, s, w.node_row, k,
-               L->max_depth, ypart, L->H, y, T, cols, ys);
+    launch_k(L, k_combine_warp<TP, TY, 4, true>, grid, WT_WARPS * 32, 0, s, w.node_row, k,
+             L->max_depth, ypart, L->H, y, T, cols, ys);
     return;
   }
-  // large batches: eight columns per lane (16-byte bf16 loads), half the
-  // per-element address and loop instructions of four
+  // eight columns per lane (16-byte bf16 loads): half the per-element address
+  // and loop instructions of four (measured faster at decode and prefill)
   const int cols = warp_item_cols(L, T, L->H, 256);
   const int grid = warp_grid(L, T, L->H, cols);
   launch_k(L, k_combine_warp<TP, TY, 8, false>, grid, WT_WARPS * 32, 0, s, w.node_row, k,
