@@ -44,13 +44,22 @@ WORKLOADS = {
     "prefill": ("qwen", 8192, "Qwen3-30B-A3B-shaped compressed MoE layer, prefill of 8192 tokens"),
     "high_e": ("high_e", 4096, "E=256 (32 clusters of 8, rank 64), H=2560, I=1536, 4096 tokens"),
     "tree": ("tree", 2048, "BTExperts depth-2 tree (8 roots, 32 rank-192 subs, 96 rank-64 leaves), 2048 tokens"),
+    "binary_decode64": ("binary", 64, "BTExperts Fig. 2 binary trees with -1/+1 edges (16 roots, "
+                        "rank-128/64 internal corrections, 128 rank-64 leaf experts), decode batch of 64 tokens"),
+    "binary": ("binary", 2048, "BTExperts Fig. 2 binary trees with -1/+1 edges (16 roots, "
+               "rank-128/64 internal corrections, 128 rank-64 leaf experts), 2048 tokens"),
+    "single_base_decode64": ("single_base", 64, "single shared base with 128 rank-128 experts, "
+                             "H=2048, I=768, top-8, decode batch of 64 tokens"),
+    "single_base": ("single_base", 2048, "single shared base with 128 rank-128 experts, "
+                    "H=2048, I=768, top-8, 2048 tokens"),
 }
 
 
 def make_layer(kind):
     import synth
     return {"qwen": synth.qwen_decode_layer, "high_e": synth.high_e_layer,
-            "tree": synth.btexperts_tree_layer}[kind]()
+            "tree": synth.btexperts_tree_layer, "binary": synth.btexperts_binary_layer,
+            "single_base": synth.d2moe_base_layer}[kind]()
 
 
 def load_peaks():

@@ -11,11 +11,15 @@
  *     V = A_m^T [in][r]:  Ug [I][r], Vg [H][r], Uu [I][r], Vu [H][r],
  *     Ud [H][r], Vd [I][r]   (row-major);
  *   - expert e is the sum of the contributions on the root path of
- *     expert_node[e]:  W_e = W_anchor + sum_{corrections n on the path} U_n V_n^T.
+ *     expert_node[e]:  W_e = W_anchor + sum_{corrections n on the path} s_n U_n V_n^T,
+ *     s_n = +1 unless the descriptor labels the edge into n with -1 (Fig. 2).
  * Flat LorExperts: one anchor per cluster (the dominant maps to it, so it
  * carries no correction) and one rank-r child per member; a protection-set
  * singleton is an anchor without children.  BTExperts: anchors are tree roots
- * (which need not be experts), corrections at any depth <= LX_MAX_DEPTH - 1.
+ * (which need not be experts), corrections at any depth <= LX_MAX_DEPTH - 1,
+ * e.g. Fig. 2's binary tree with signed edges and experts at the leaves.  A
+ * single shared base (Sec. 5.2's single-shared-component layout) is one anchor
+ * that is no expert, with every expert a correction below it.
  *
  * The forward (Sec. 5.1, "computed once per token and broadcast") routes every
  * token top-k over all E experts with the unchanged router (Sec. 1, Fig. 1),
@@ -79,6 +83,10 @@ typedef struct {
   const int32_t* node_parent; /* host [n_nodes]: -1 for an anchor, else parent id */
   const int32_t* node_rank;   /* host [n_nodes]: 0 for an anchor, 1..min(I,H) else */
   const int32_t* expert_node; /* host [n_experts]: node defining expert e */
+  const int8_t* node_sign;    /* host [n_nodes] or NULL: sign s_n in {+1, -1} of the edge
+                                 into node n (Fig. 2 labels the edges of the BTExperts tree
+                                 -1/+1); a correction then contributes s_n U_n V_n^T.
+                                 Anchors must carry +1.  NULL = every edge +1. */
 } lx_layer_desc;
 
 /*
@@ -89,10 +97,13 @@ typedef struct {
  *                Element type = desc->dtype (bf16 as uint16 bit patterns).
  *   router_w:    host [E][H] (desc->dtype).
  *   router_bias: host [E] fp32 added to the logits, or NULL.
- * Copies (and repacks) everything to device memory owned by the layer;
- * synchronises `stream`.  Errors: LX_ERR_ARG (null pointers), LX_ERR_SHAPE
- * (sizes, cycles, depth > LX_MAX_DEPTH, anchor with rank != 0, correction rank
- * outside 1..min(I,H), H or I not a multiple of 8), LX_ERR_OOM, LX_ERR_CUDA.
+ * Copies (and repacks) everything to device memory owned by the layer; a
+ * correction whose edge sign is -1 is stored with negated U factors (exact), so
+ * every kernel sees an unsigned tree.  Synchronises `stream`.  Errors:
+ * LX_ERR_ARG (null pointers), LX_ERR_SHAPE (sizes, cycles, depth >
+ * LX_MAX_DEPTH, anchor with rank != 0, correction rank outside 1..min(I,H),
+ * H or I not a multiple of 8, a sign other than +1/-1 or an anchor sign of -1),
+ * LX_ERR_OOM, LX_ERR_CUDA.
  */
 LX_API lx_status lx_load_compressed_layer(const lx_layer_desc* desc, const void* const* node_w,
                                    const void* router_w, const float* router_bias,

@@ -12,7 +12,9 @@ except the router logits, see below):
    Sec. 3.2 Stage 3(iii) "installation"; Sec. 5 tree: an expert's weights are the
    sum of the contributions on its root path).  For every projection
    p in {gate, up, down}:  ``W_e^p = W_anchor^p + sum_{n on path(e), n != anchor}
-   U_n^p (V_n^p)^T``  with ``U = B`` ([out, r]) and ``V = A^T`` ([in, r]).
+   s_n U_n^p (V_n^p)^T``  with ``U = B`` ([out, r]), ``V = A^T`` ([in, r]) and
+   ``s_n`` in {+1, -1} the label of the edge into n (Fig. 2; +1 when the layer
+   carries no signs).
 2. Routing (Sec. 1 and Fig. 1: top-k over all E experts by the unchanged
    router; Sec. 5.2 "top-k routing").  Logits ``l = x W_r^T (+ b)`` in the
    canonical fp32 order of ``router_canonical.c``; top-k by (logit descending,
@@ -44,7 +46,7 @@ from . import _clib
 
 __all__ = [
     "router_logits", "topk", "gates", "route", "expert_weights", "silu",
-    "expert_output", "moe_forward", "buckets", "build",
+    "expert_output", "moe_forward", "buckets", "build", "edge_sign",
 ]
 
 
@@ -121,14 +123,21 @@ def _correction(layer: CompressedLayer, n: int, p: int) -> np.ndarray:
     return U @ V.T
 
 
+def edge_sign(layer: CompressedLayer, n: int) -> float:
+    """Sign of the edge into node n (Fig. 2's -1/+1 labels); +1 without signs."""
+    signs = getattr(layer, "node_sign", None)
+    return 1.0 if signs is None else float(signs[n])
+
+
 def expert_weights(layer: CompressedLayer, e: int):
     """(W_gate [I,H], W_up [I,H], W_down [H,I]) of expert e, float64."""
     path = _path(layer, e)
     anchor = path[-1]
     Ws = [from_storage(a, layer.dtype).copy() for a in layer.node_w[anchor]]
     for n in path[:-1]:
+        s = edge_sign(layer, n)
         for p in range(3):
-            Ws[p] += _correction(layer, n, p)
+            Ws[p] += s * _correction(layer, n, p)
     return tuple(Ws)
 
 

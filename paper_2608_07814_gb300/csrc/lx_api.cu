@@ -340,7 +340,24 @@ static lx_status validate_desc(const lx_layer_desc* d, const void* const* node_w
   for (long e = 0; e < E; ++e)
     if (d->expert_node[e] < 0 || d->expert_node[e] >= N)
       return fail(LX_ERR_SHAPE, "expert_node out of range");
+  if (d->node_sign)
+    for (long n = 0; n < N; ++n) {
+      const int sg = d->node_sign[n];
+      if (sg != 1 && sg != -1) return fail(LX_ERR_SHAPE, "node_sign must be +1 or -1");
+      if (d->node_parent[n] < 0 && sg != 1) return fail(LX_ERR_SHAPE, "anchor with node_sign -1");
+    }
   return LX_OK;
+}
+
+// Flips the sign bit of every element (bf16 or fp32): exact negation.
+static void negate_bytes(void* buf, size_t n_elems, int esz) {
+  if (esz == 2) {
+    uint16_t* p = (uint16_t*)buf;
+    for (size_t i = 0; i < n_elems; ++i) p[i] ^= 0x8000u;
+  } else {
+    uint32_t* p = (uint32_t*)buf;
+    for (size_t i = 0; i < n_elems; ++i) p[i] ^= 0x80000000u;
+  }
 }
 
 // dst[c][r] = src[r][c] for a [rows][cols] matrix of esz-byte elements
@@ -442,6 +459,8 @@ extern "C" lx_status lx_load_compressed_layer(const lx_layer_desc* d, const void
     char* dst = (char*)L->arena + p.off;
     const int n = p.node;
     const void* const* w = node_w + 6 * (size_t)n;
+    // edge sign -1 (Fig. 2): the correction enters as (-U) V^T
+    const bool negative = d->node_sign && d->node_sign[n] < 0;
     stage.resize(p.bytes);
     if (L->parent[n] < 0) {
       if (p.slot == 0) {
@@ -461,12 +480,14 @@ extern "C" lx_status lx_load_compressed_layer(const lx_layer_desc* d, const void
       } else if (p.slot == 1) {
         std::memcpy(stage.data(), w[0], I * r * esz);
         std::memcpy(stage.data() + I * r * esz, w[2], I * r * esz);
+        if (negative) negate_bytes(stage.data(), (size_t)2 * I * r, (int)esz);
         L->h_w_upU[n] = dst;
       } else if (p.slot == 2) {  // Vd [I][r] -> [r][I]
         transpose_bytes(w[5], stage.data(), I, r, esz);
         L->h_w_dn[n] = dst;
       } else {
         std::memcpy(stage.data(), w[4], H * r * esz);
+        if (negative) negate_bytes(stage.data(), (size_t)H * r, (int)esz);
         L->h_w_dnU[n] = dst;
       }
     }

@@ -44,7 +44,8 @@ class LayerDesc(ctypes.Structure):
                 ("n_experts", ctypes.c_int32), ("n_nodes", ctypes.c_int32),
                 ("dtype", ctypes.c_int32), ("node_parent", ctypes.POINTER(ctypes.c_int32)),
                 ("node_rank", ctypes.POINTER(ctypes.c_int32)),
-                ("expert_node", ctypes.POINTER(ctypes.c_int32))]
+                ("expert_node", ctypes.POINTER(ctypes.c_int32)),
+                ("node_sign", ctypes.POINTER(ctypes.c_int8))]
 
 
 class LayerInfo(ctypes.Structure):
@@ -122,7 +123,7 @@ class Layer:
 
     ``src`` is any object with the fields of ``synth.CompressedLayer``
     (d_model, d_ff, n_experts, dtype in {'f32','bf16'}, node_parent, node_rank,
-    expert_node, node_w, router_w, router_bias)."""
+    expert_node, node_w, router_w, router_bias, and optionally node_sign)."""
 
     def __init__(self, src, stream: Optional[torch.cuda.Stream] = None):
         L = lib()
@@ -137,6 +138,10 @@ class Layer:
         rank = np.ascontiguousarray(src.node_rank, np.int32)
         enode = np.ascontiguousarray(src.expert_node, np.int32)
         self._keep += [parent, rank, enode]
+        sign = getattr(src, "node_sign", None)
+        if sign is not None:
+            sign = np.ascontiguousarray(sign, np.int8)
+            self._keep.append(sign)
         N = parent.shape[0]
         ptrs = (ctypes.c_void_p * (6 * N))()
         for n, ws in enumerate(src.node_w):
@@ -154,7 +159,9 @@ class Layer:
                          LX_BF16 if src.dtype == "bf16" else LX_F32,
                          parent.ctypes.data_as(ctypes.POINTER(ctypes.c_int32)),
                          rank.ctypes.data_as(ctypes.POINTER(ctypes.c_int32)),
-                         enode.ctypes.data_as(ctypes.POINTER(ctypes.c_int32)))
+                         enode.ctypes.data_as(ctypes.POINTER(ctypes.c_int32)),
+                         None if sign is None else sign.ctypes.data_as(
+                             ctypes.POINTER(ctypes.c_int8)))
         h = ctypes.c_void_p()
         st = L.lx_load_compressed_layer(ctypes.byref(desc), ptrs, ctypes.c_void_p(rw.ctypes.data),
                                         None if bias is None else ctypes.c_void_p(bias.ctypes.data),

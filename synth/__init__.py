@@ -19,7 +19,15 @@ A layer is described by a *node table* (LorExperts Sec. 3.1; BTExperts Sec. 5):
 The flat LorExperts layout has one anchor per cluster (the dominant expert maps
 to it directly) and one rank-r child per member.  The BTExperts layout used here
 has non-expert root anchors, rank-192 sub-dominant children (experts) and rank-64
-leaf grandchildren (experts).
+leaf grandchildren (experts).  Two further layouts: a binary BTExperts tree in the
+shape of Fig. 2 (non-expert root and internal corrections, experts at the
+leaves, optionally with the figure's -1/+1 edge signs), and a single shared base
+(one non-expert anchor, every expert a rank-r correction to it: the
+single-shared-component layout the paper contrasts with, Sec. 5.2).
+
+Edge signs: ``node_sign[n]`` in {+1, -1} multiplies correction n's contribution
+``U_n V_n^T`` (the label on the edge from n's parent to n in Fig. 2); ``None``
+means every edge is +1.  Anchors always carry +1.
 
 Storage dtypes: ``'f32'`` (float32 arrays), ``'bf16'`` (uint16 arrays holding
 bfloat16 bit patterns) and ``'f64'`` (float64; accepted by the oracle only, used
@@ -45,8 +53,8 @@ import numpy as np
 __all__ = [
     "CompressedLayer", "bf16_bits", "bf16_to_f32", "to_storage", "from_storage",
     "tiny_layer", "flat_layer", "tree_layer", "qwen_decode_layer",
-    "qwen_prefill_layer", "high_e_layer", "btexperts_tree_layer", "tokens",
-    "CONFIGS",
+    "qwen_prefill_layer", "high_e_layer", "btexperts_tree_layer", "binary_tree_layer",
+    "single_base_layer", "btexperts_binary_layer", "d2moe_base_layer", "tokens", "CONFIGS",
 ]
 
 ANCHOR_SLOTS = ("gate", "up", "down")
@@ -106,6 +114,7 @@ class CompressedLayer:
     top_k: int
     name: str = ""
     meta: dict = dataclasses.field(default_factory=dict)
+    node_sign: Optional[np.ndarray] = None   # int8 [n_nodes] of +1/-1, or None (all +1)
 
     @property
     def n_nodes(self) -> int:
@@ -306,6 +315,116 @@ def tree_layer(H: int, I: int, n_roots: int, subs_per_root: int, leaves_per_sub:
 
 
 # ----------------------------------------------------------------------------
+# BTExperts binary tree (Fig. 2): per root anchor a complete binary tree of
+# corrections; internal corrections are shared, the leaves are the experts.
+# ----------------------------------------------------------------------------
+def binary_tree_layer(H: int, I: int, n_roots: int, levels: int, ranks: Sequence[int],
+                      top_k: int, dtype: str = "bf16", seed: int = 0, factor_std=None,
+                      signed: bool = False, zero_dominants: bool = False,
+                      zero_factors: bool = False,
+                      skew: Optional[Tuple[float, float, float, int]] = None,
+                      name: str = "binary-tree") -> CompressedLayer:
+    """``levels`` correction levels below each root (level 1 has 2 nodes, level
+    ``levels`` has 2**levels leaves, the experts); ``ranks[l-1]`` is the rank of
+    level l.  ``signed`` labels the edge to every left child -1 and to every
+    right child +1, as Fig. 2 does for the internal levels (the figure gives the
+    leaf edges no label; here they carry the same alternation)."""
+    assert 1 <= levels and len(ranks) == levels
+    rng = np.random.default_rng(seed)
+    leaves_per_root = 2 ** levels
+    E = n_roots * leaves_per_root
+    ids = [int(e) for e in rng.permutation(E)]
+    parent = [-1] * n_roots
+    nrank = [0] * n_roots
+    sign = [1] * n_roots
+    node_w = [_anchor(rng, H, I, dtype, zero=zero_dominants) for _ in range(n_roots)]
+    expert_node = np.zeros(E, np.int32)
+    it = iter(ids)
+    root_groups, pair_groups = [], []
+    for rt in range(n_roots):
+        frontier = [rt]
+        for lev in range(1, levels + 1):
+            nxt = []
+            for pn in frontier:
+                for side in (0, 1):
+                    parent.append(pn)
+                    r = int(ranks[lev - 1])
+                    nrank.append(r)
+                    sign.append((-1 if side == 0 else 1) if signed else 1)
+                    node_w.append(_corr_factors(rng, H, I, r, _factor_std(r, factor_std),
+                                                dtype, zero=zero_factors))
+                    nxt.append(len(parent) - 1)
+            frontier = nxt
+        leaves = []
+        for ln in frontier:
+            e = next(it)
+            expert_node[e] = ln
+            leaves.append(e)
+        root_groups.append(leaves)
+        # co-activation groups: the leaves below each level-(levels-1) node
+        # (pairs of siblings; the whole root's leaves when levels == 1)
+        step = 2 if levels > 1 else leaves_per_root
+        for j in range(0, leaves_per_root, step):
+            pair_groups.append(leaves[j:j + step])
+    if skew is None:
+        Wr = _normal(rng, (E, H), 0.02)
+        bias = None
+    else:
+        s, beta, rho, n_dead = skew
+        Wr = _router(rng, E, H, pair_groups, rho * 0.5, outer=root_groups, rho_outer=rho * 0.45)
+        cand = [e for g in pair_groups for e in g[1:]]
+        dead = rng.choice(cand, size=min(n_dead, len(cand)), replace=False) if n_dead else []
+        bias = _zipf_bias(rng, E, pair_groups, s, beta, dead)
+    return CompressedLayer(
+        d_model=H, d_ff=I, n_experts=E, dtype=dtype,
+        node_parent=np.asarray(parent, np.int32), node_rank=np.asarray(nrank, np.int32),
+        expert_node=expert_node, node_w=node_w, router_w=to_storage(Wr, dtype),
+        router_bias=bias, top_k=top_k, name=name,
+        meta={"roots": root_groups, "pairs": pair_groups, "seed": seed},
+        node_sign=np.asarray(sign, np.int8) if signed else None)
+
+
+# ----------------------------------------------------------------------------
+# single shared base: one non-expert anchor, every expert a rank-r correction
+# ----------------------------------------------------------------------------
+def single_base_layer(H: int, I: int, E: int, rank, top_k: int, dtype: str = "bf16",
+                      seed: int = 0, factor_std=None, group: int = 4,
+                      zero_dominants: bool = False, zero_factors: bool = False,
+                      skew: Optional[Tuple[float, float, float, int]] = None,
+                      name: str = "single-base") -> CompressedLayer:
+    """One shared base anchor (not an expert) and E rank-r experts below it.
+    Router co-activation groups of ``group`` consecutive shuffled experts."""
+    rng = np.random.default_rng(seed)
+    ids = [int(e) for e in rng.permutation(E)]
+    ranks = list(rank) if isinstance(rank, (list, tuple, np.ndarray)) else [int(rank)] * E
+    parent, nrank = [-1], [0]
+    node_w = [_anchor(rng, H, I, dtype, zero=zero_dominants)]
+    expert_node = np.zeros(E, np.int32)
+    for j, e in enumerate(ids):
+        r = int(ranks[j])
+        parent.append(0)
+        nrank.append(r)
+        node_w.append(_corr_factors(rng, H, I, r, _factor_std(r, factor_std), dtype,
+                                    zero=zero_factors))
+        expert_node[e] = len(parent) - 1
+    groups = [ids[j:j + group] for j in range(0, E, group)]
+    if skew is None:
+        Wr = _normal(rng, (E, H), 0.02)
+        bias = None
+    else:
+        s, beta, rho, n_dead = skew
+        Wr = _router(rng, E, H, groups, rho)
+        cand = [e for g in groups for e in g[1:]]
+        dead = rng.choice(cand, size=min(n_dead, len(cand)), replace=False) if n_dead else []
+        bias = _zipf_bias(rng, E, groups, s, beta, dead)
+    return CompressedLayer(
+        d_model=H, d_ff=I, n_experts=E, dtype=dtype,
+        node_parent=np.asarray(parent, np.int32), node_rank=np.asarray(nrank, np.int32),
+        expert_node=expert_node, node_w=node_w, router_w=to_storage(Wr, dtype),
+        router_bias=bias, top_k=top_k, name=name, meta={"groups": groups, "seed": seed})
+
+
+# ----------------------------------------------------------------------------
 # the five workloads
 # ----------------------------------------------------------------------------
 def _svd_factors(R: np.ndarray, r: int):
@@ -397,6 +516,22 @@ def btexperts_tree_layer(seed: int = 5, factor_std=None, **kw) -> CompressedLaye
     """H=2048, I=768, 8 root anchors x 4 rank-192 sub-dominants x 3 rank-64 leaves."""
     return tree_layer(2048, 768, 8, 4, 3, 192, 64, 8, "bf16", seed, factor_std,
                       skew=TREE_SKEW, name="btexperts-tree-layer", **kw)
+
+
+def btexperts_binary_layer(seed: int = 6, factor_std=None, signed: bool = True,
+                           **kw) -> CompressedLayer:
+    """H=2048, I=768, E=128 top-8: 16 root anchors, each a Fig. 2 binary tree of
+    rank-128 / rank-64 internal corrections and rank-64 leaf experts (8 per root,
+    root paths of 4 nodes), edge signs -1/+1."""
+    return binary_tree_layer(2048, 768, 16, 3, [128, 64, 64], 8, "bf16", seed, factor_std,
+                             signed=signed, skew=TREE_SKEW, name="btexperts-binary-layer",
+                             **kw)
+
+
+def d2moe_base_layer(seed: int = 7, factor_std=None, **kw) -> CompressedLayer:
+    """H=2048, I=768, E=128 top-8 rank-128 experts over one shared base."""
+    return single_base_layer(2048, 768, 128, 128, 8, "bf16", seed, factor_std,
+                             skew=QWEN_SKEW, name="single-base-layer", **kw)
 
 
 def tokens(layer: CompressedLayer, T: int, seed: int = 0) -> np.ndarray:

@@ -62,6 +62,10 @@ def _base():
     (lambda l: l.node_rank.__setitem__(3, 0), lx.LX_ERR_SHAPE),      # correction rank 0
     (lambda l: l.node_rank.__setitem__(3, 33), lx.LX_ERR_SHAPE),     # rank > min(I,H)
     (lambda l: l.expert_node.__setitem__(1, 99), lx.LX_ERR_SHAPE),
+    (lambda l: setattr(l, "node_sign", np.asarray([1, 1, 2, 1, 1, 1, 1, 1], np.int8)),
+     lx.LX_ERR_SHAPE),                                                # sign not +-1
+    (lambda l: setattr(l, "node_sign", np.asarray([-1, 1, 1, 1, 1, 1, 1, 1], np.int8)),
+     lx.LX_ERR_SHAPE),                                                # negative anchor edge
 ])
 def test_invalid_layers_rejected_on_host(L, mutate, status):
     layer = copy.deepcopy(_base())
@@ -101,3 +105,5 @@ def test_null_arguments(L):
 @pytest.mark.skipif(torch.cuda.is_available(), reason="checks the no-GPU error path")
 def test_valid_layer_without_gpu_reports_cuda_error(L):
     assert _load_status(_base()) == lx.LX_ERR_CUDA
+    signed = synth.binary_tree_layer(64, 32, 1, 3, [8, 8, 8], 2, "f32", seed=0, signed=True)
+    assert _load_status(signed) == lx.LX_ERR_CUDA      # passes validation

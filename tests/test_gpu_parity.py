@@ -120,6 +120,19 @@ SMALL = {
     "stream_split_tree": lambda: synth.tree_layer(1024, 640, 2, 4, 3, 128, 64, 8, "bf16",
                                                   seed=17, factor_std="visible",
                                                   skew=synth.TREE_SKEW),
+    # Fig. 2 binary trees with -1/+1 edges (root paths of four nodes: k * depth = 32)
+    "stream_binary_signed": lambda: synth.binary_tree_layer(
+        256, 192, 2, 3, [128, 64, 64], 8, "bf16", seed=18, factor_std="visible", signed=True,
+        skew=synth.TREE_SKEW),
+    "binary_signed_fp32": lambda: synth.binary_tree_layer(
+        128, 64, 2, 3, [16, 8, 8], 4, "f32", seed=19, factor_std="visible", signed=True,
+        skew=synth.TREE_SKEW),
+    # one shared base below which every expert is a correction
+    "stream_single_base": lambda: synth.single_base_layer(
+        512, 384, 24, 64, 8, "bf16", seed=20, factor_std="visible", skew=synth.QWEN_SKEW),
+    "single_base_fp32_mixed_rank": lambda: synth.single_base_layer(
+        64, 96, 12, [8, 16, 24, 40, 8, 64, 1, 2, 3, 5, 7, 9], 4, "f32", seed=21,
+        factor_std="visible"),
 }
 
 STREAM = [n for n in SMALL if n.startswith("stream")]
@@ -293,6 +306,8 @@ FULL = {
     "qwen_visible": lambda: synth.qwen_decode_layer(factor_std="visible"),
     "high_e": lambda: synth.high_e_layer(),
     "tree": lambda: synth.btexperts_tree_layer(factor_std="visible"),
+    "binary": lambda: synth.btexperts_binary_layer(factor_std="visible"),
+    "single_base": lambda: synth.d2moe_base_layer(factor_std="visible"),
 }
 
 
@@ -305,7 +320,7 @@ def test_qwen_decode_batches(T):
     check_forward(src, L, x, 8)
 
 
-@pytest.mark.parametrize("name", ["high_e", "tree"])
+@pytest.mark.parametrize("name", ["high_e", "tree", "binary", "single_base"])
 @pytest.mark.parametrize("T", [1, 64])
 def test_full_layers_decode(name, T):
     """Decode batches of the other full-size layers (split-K anchor tiles with
@@ -329,7 +344,8 @@ def _sample(T, n=24, seed=0):
     return np.unique(np.concatenate([[0, T - 1], rng.choice(T, n, replace=False)]))
 
 
-@pytest.mark.parametrize("name,T", [("qwen", 8192), ("high_e", 4096), ("tree", 2048)])
+@pytest.mark.parametrize("name,T", [("qwen", 8192), ("high_e", 4096), ("tree", 2048),
+                                    ("binary", 2048), ("single_base", 2048)])
 def test_full_size_sampled(name, T):
     src, L = installed(name, FULL[name])
     x = synth.tokens(src, T, seed=11)

@@ -220,8 +220,10 @@ def _flat_from_tree(tree):
                 for p in range(3):
                     acc[p] = acc[p] + f64(w[p])
             else:
+                sg = 1.0 if tree.node_sign is None else float(tree.node_sign[n])
                 for p in range(3):
-                    acc[p] = acc[p] + np.einsum("ir,jr->ij", f64(w[2 * p]), f64(w[2 * p + 1]))
+                    acc[p] = acc[p] + sg * np.einsum("ir,jr->ij", f64(w[2 * p]),
+                                                     f64(w[2 * p + 1]))
             n = int(tree.node_parent[n])
         node_w.append(tuple(acc))
     return synth.CompressedLayer(
@@ -247,6 +249,75 @@ def test_tree_equals_flat():
     zero = synth.tree_layer(64, 48, 2, 2, 3, 12, 4, 4, "f32", seed=11, zero_factors=True,
                             skew=synth.TREE_SKEW)
     assert rel_err(oracle.moe_forward(zero, x, routing=(ids, g)), y_tree) > 1e-2
+
+
+# ----------------------------------------------------------------------------
+# BTExperts variants: Fig. 2's binary tree with -1/+1 edges, and a single shared
+# base (the single-shared-component layout of Sec. 5.2)
+# ----------------------------------------------------------------------------
+def test_signed_binary_tree_equals_flat():
+    """A Fig. 2 binary tree with signed edges is the flat layer whose experts are
+    the signed sums along their root paths (summed independently above)."""
+    tree = synth.binary_tree_layer(64, 48, 2, 3, [12, 8, 4], 4, "f32", seed=21,
+                                   factor_std="visible", signed=True, skew=synth.TREE_SKEW)
+    assert tree.node_sign is not None and set(np.unique(tree.node_sign)) == {-1, 1}
+    assert max(len(tree.path(e)) for e in range(tree.n_experts)) == 4
+    x = synth.tokens(tree, 50, seed=3)
+    ids, g, _ = oracle.route(tree, x)
+    flat = _flat_from_tree(tree)
+    y_tree = oracle.moe_forward(tree, x, routing=(ids, g))
+    y_flat = oracle.moe_forward(flat, synth.from_storage(x, "f32"), routing=(ids, g))
+    assert rel_err(y_tree, y_flat) < 1e-12
+    # the signs matter: the unsigned tree is another function
+    tree.node_sign = None
+    assert rel_err(oracle.moe_forward(tree, x, routing=(ids, g)), y_tree) > 1e-2
+
+
+def test_sibling_edges_cancel():
+    """Two leaves below one root through edges -1 and +1 that carry the same
+    factors average to the root and differ by twice the correction."""
+    tree = synth.binary_tree_layer(32, 24, 1, 1, [6], 2, "f64", seed=22,
+                                   factor_std="visible", signed=True)
+    left, right = int(tree.expert_node[0]), int(tree.expert_node[1])
+    tree.node_w[right] = tree.node_w[left]
+    e_left, e_right = (0, 1) if tree.node_sign[left] < 0 else (1, 0)
+    Wl = oracle.expert_weights(tree, e_left)
+    Wr = oracle.expert_weights(tree, e_right)
+    root = tree.node_w[0]
+    fac = tree.node_w[left]
+    for p in range(3):
+        assert np.allclose(0.5 * (Wl[p] + Wr[p]), root[p], rtol=0, atol=1e-15)
+        assert np.allclose(Wr[p] - Wl[p], 2.0 * np.einsum("ir,jr->ij", fac[2 * p], fac[2 * p + 1]),
+                           rtol=0, atol=1e-14)
+
+
+def test_single_base_full_rank_equals_uncompressed():
+    """One shared base (not an expert) with every expert a full-rank correction
+    (Eq. svd / factors of W_e - base) is the uncompressed MoE."""
+    rng = np.random.default_rng(23)
+    H, I, E = 32, 48, 6
+    dense = [tuple(rng.standard_normal(s) * 0.02 for s in [(I, H), (I, H), (H, I)])
+             for _ in range(E)]
+    base = tuple(np.mean([d[p] for d in dense], axis=0) for p in range(3))
+    node_w = [tuple(synth.to_storage(b, "f32") for b in base)]
+    for e in range(E):
+        fac = []
+        for p in range(3):
+            B, At = synth._svd_factors(dense[e][p] - synth.from_storage(node_w[0][p], "f32"),
+                                       min(H, I))
+            fac += [B, At]
+        node_w.append(tuple(synth.to_storage(f, "f32") for f in fac))
+    layer = synth.CompressedLayer(
+        d_model=H, d_ff=I, n_experts=E, dtype="f32",
+        node_parent=np.asarray([-1] + [0] * E, np.int32),
+        node_rank=np.asarray([0] + [min(H, I)] * E, np.int32),
+        expert_node=np.arange(1, E + 1, dtype=np.int32), node_w=node_w,
+        router_w=synth.to_storage(rng.standard_normal((E, H)) * 0.02, "f32"),
+        router_bias=None, top_k=3)
+    x = synth.tokens(layer, 40, seed=4)
+    ids, g, _ = oracle.route(layer, x)
+    ref = dense_moe_torch(dense, synth.from_storage(x, "f32"), ids, g)
+    assert rel_err(oracle.moe_forward(layer, x), ref) < 1e-5
 
 
 # ----------------------------------------------------------------------------
@@ -370,6 +441,10 @@ def _mut_uniform_gates(logits, ids):
     return np.full(ids.shape, 1.0 / ids.shape[1])
 
 
+def _mut_unsigned(layer, n):
+    return 1.0
+
+
 def _pins_pass():
     try:
         test_full_rank_reconstruction_equals_uncompressed()
@@ -378,6 +453,9 @@ def _pins_pass():
         test_gates_closed_form()
         test_swiglu_closed_form()
         test_tree_equals_flat()
+        test_signed_binary_tree_equals_flat()
+        test_sibling_edges_cancel()
+        test_single_base_full_rank_equals_uncompressed()
     except AssertionError:
         return False
     return True
@@ -390,6 +468,7 @@ def _pins_pass():
     ("silu", _mut_sigmoid),
     ("topk", _mut_topk_high_id),
     ("gates", _mut_uniform_gates),
+    ("edge_sign", _mut_unsigned),
 ])
 def test_planted_mistakes_fail_a_pin(monkeypatch, target, mutant):
     assert _pins_pass()
