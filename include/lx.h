@@ -254,6 +254,38 @@ LX_API lx_status lx_bucket_noalloc(lx_layer* layer, const int32_t* topk_id, int3
                                    int32_t* node_off, int32_t* node_tok, int32_t* node_row,
                                    int32_t* expert_off, int32_t* perm, void* stream);
 
+/*
+ * Router profiling statistics (Sec. 3.2 Stage 1 accumulates per-layer firing
+ * counts N_e by reading the router; Sec. 2.2 weights the expert co-activation
+ * graph by normalised pointwise mutual information, NPMI, and Stage 2's
+ * Coact-NPMI variant clusters on 1 - NPMI).  Standalone: no layer needed.
+ *
+ * lx_coact_accumulate ADDS one batch of top-k assignments to the counters:
+ *   topk_id: device [T][k] int32.  A token's selected set is the set of its ids
+ *            in [0, E); ids outside are skipped and a repeated id counts once.
+ *   fire:    device [E] uint64 or NULL:  fire[e] += tokens whose set holds e (N_e)
+ *   coact:   device [E][E] uint64 row-major or NULL:  coact[i][j] += tokens
+ *            whose set holds both i and j; coact[i][i] += N_i.
+ * The caller zeroes the counters before the first batch; counts are exact
+ * (integer) and independent of launch order.  Stream-ordered; no allocation.
+ * Errors: LX_ERR_ARG (T < 0, k outside 1..LX_MAX_K, E outside
+ * 1..LX_MAX_EXPERTS, fire and coact both NULL, topk_id NULL with T > 0).
+ * T == 0 is a no-op.
+ */
+LX_API lx_status lx_coact_accumulate(const int32_t* topk_id, int32_t T, int32_t k, int32_t E,
+                                     uint64_t* fire, uint64_t* coact, void* stream);
+
+/*
+ * lx_coact_npmi: NPMI matrix of accumulated counts over n_tokens tokens, in
+ * float64:  with p_i = coact[i][i] / n and p_ij = coact[i][j] / n,
+ *   npmi[i][j] = ln(p_ij / (p_i p_j)) / (-ln p_ij)   for 0 < p_ij < 1,
+ *              = -1 for p_ij = 0 (never together), +1 for p_ij = 1.
+ *   coact: device [E][E] uint64 (from lx_coact_accumulate); npmi: device [E][E]
+ *   double out.  Errors: LX_ERR_ARG (E out of range, n_tokens < 0, NULL).
+ */
+LX_API lx_status lx_coact_npmi(const uint64_t* coact, int32_t E, int64_t n_tokens, double* npmi,
+                               void* stream);
+
 /* Message of the last failed call on this thread ("" if none). */
 LX_API const char* lx_last_error(void);
 

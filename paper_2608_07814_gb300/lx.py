@@ -28,7 +28,8 @@ LX_MAX_DEPTH, LX_MAX_K, LX_MAX_EXPERTS = 4, 32, 1024
 EXPORTS = [
     "lx_load_compressed_layer", "lx_free_layer", "lx_reserve", "lx_route", "lx_bucket",
     "lx_moe_forward", "lx_get_buckets", "lx_layer_info", "lx_set_path", "lx_set_profiling",
-    "lx_read_profile", "lx_last_error", "lx_bucket_noalloc",
+    "lx_read_profile", "lx_last_error", "lx_bucket_noalloc", "lx_coact_accumulate",
+    "lx_coact_npmi",
 ]
 LX_NOALLOC_SCRATCH_BYTES = 16 << 20
 
@@ -86,6 +87,8 @@ def lib() -> ctypes.CDLL:
             "lx_set_profiling": [vp, i32],
             "lx_read_profile": [vp, ctypes.POINTER(KernelTime), i32, ctypes.POINTER(i32)],
             "lx_bucket_noalloc": [vp, vp, i32, i32, vp, vp, vp, vp, vp, vp],
+            "lx_coact_accumulate": [vp, i32, i32, i32, vp, vp, vp],
+            "lx_coact_npmi": [vp, i32, ctypes.c_int64, vp, vp],
         }
         for name, args in sig.items():
             f = getattr(L, name)
@@ -242,3 +245,30 @@ class Layer:
         out["node_row"] = out["node_row"][:T * k * D]
         out["perm"] = out["perm"][:T * k]
         return out
+
+
+# ----------------------------------------------------------------------------
+# router profiling statistics (standalone calls, no layer)
+# ----------------------------------------------------------------------------
+def coact_accumulate(topk_id: torch.Tensor, E: int, fire: Optional[torch.Tensor] = None,
+                     coact: Optional[torch.Tensor] = None, stream=None):
+    """Adds the batch topk_id [T, k] (int32, device) to the uint64 counters
+    fire [E] and coact [E, E] (int64 tensors holding the unsigned counts;
+    allocated zeroed when omitted).  Returns (fire, coact)."""
+    dev = topk_id.device
+    if fire is None:
+        fire = torch.zeros(E, dtype=torch.int64, device=dev)
+    if coact is None:
+        coact = torch.zeros((E, E), dtype=torch.int64, device=dev)
+    T, k = topk_id.shape
+    _check(lib().lx_coact_accumulate(_ptr(topk_id), T, k, E, _ptr(fire), _ptr(coact),
+                                     _stream(stream)))
+    return fire, coact
+
+
+def coact_npmi(coact: torch.Tensor, n_tokens: int, stream=None) -> torch.Tensor:
+    """float64 [E, E] NPMI of the counts coact [E, E] over n_tokens tokens."""
+    E = coact.shape[0]
+    out = torch.empty((E, E), dtype=torch.float64, device=coact.device)
+    _check(lib().lx_coact_npmi(_ptr(coact), E, n_tokens, _ptr(out), _stream(stream)))
+    return out

@@ -107,3 +107,19 @@ def test_valid_layer_without_gpu_reports_cuda_error(L):
     assert _load_status(_base()) == lx.LX_ERR_CUDA
     signed = synth.binary_tree_layer(64, 32, 1, 3, [8, 8, 8], 2, "f32", seed=0, signed=True)
     assert _load_status(signed) == lx.LX_ERR_CUDA      # passes validation
+
+
+def test_statistics_calls_rejected_on_host(L):
+    """Argument checks of the router-statistics calls come before any CUDA call."""
+    buf = ctypes.c_void_p(8)  # never dereferenced: every call below fails validation
+    assert L.lx_coact_accumulate(buf, -1, 4, 16, buf, buf, None) == lx.LX_ERR_ARG
+    assert L.lx_coact_accumulate(buf, 4, 0, 16, buf, buf, None) == lx.LX_ERR_ARG
+    assert L.lx_coact_accumulate(buf, 4, 33, 16, buf, buf, None) == lx.LX_ERR_ARG
+    assert L.lx_coact_accumulate(buf, 4, 4, 0, buf, buf, None) == lx.LX_ERR_ARG
+    assert L.lx_coact_accumulate(buf, 4, 4, 1025, buf, buf, None) == lx.LX_ERR_ARG
+    assert L.lx_coact_accumulate(buf, 4, 4, 16, None, None, None) == lx.LX_ERR_ARG
+    assert L.lx_coact_accumulate(None, 4, 4, 16, buf, None, None) == lx.LX_ERR_ARG
+    assert L.lx_coact_accumulate(None, 0, 4, 16, buf, None, None) == lx.LX_OK   # T = 0
+    assert L.lx_coact_npmi(None, 16, 4, buf, None) == lx.LX_ERR_ARG
+    assert L.lx_coact_npmi(buf, 0, 4, buf, None) == lx.LX_ERR_ARG
+    assert L.lx_coact_npmi(buf, 16, -1, buf, None) == lx.LX_ERR_ARG
