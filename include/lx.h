@@ -286,6 +286,53 @@ LX_API lx_status lx_coact_accumulate(const int32_t* topk_id, int32_t T, int32_t 
 LX_API lx_status lx_coact_npmi(const uint64_t* coact, int32_t E, int64_t n_tokens, double* npmi,
                                void* stream);
 
+/*
+ * Neuron alignment of a member expert to its dominant (Sec. 3.2 Stage 3 (i)).
+ * Standalone: the experts are given as plain matrices, not as a layer.
+ * Neuron i of an expert is a_i = (gate[i][:], up[i][:], down[:][i]), length 3H.
+ *
+ * lx_align_cost: C[i][j] = ||a_i||^2 + ||b_j||^2 - 2 a_i . b_j (Eq. cost) for
+ * dominant neurons a_i and member neurons b_j, fp32 accumulation.
+ *   dtype: LX_F32 or LX_BF16 (bf16 as uint16 bit patterns); d_model H, d_ff I
+ *          multiples of 8.
+ *   dom_gate, dom_up, mem_gate, mem_up: device [I][H]; dom_down, mem_down:
+ *          device [H][I] (row-major, the x W^T storage of lx_load_compressed_layer);
+ *   cost:  device [I][I] fp32 out.  Every pointer 16-byte aligned.
+ * Stream-ordered; no allocation.  Errors: LX_ERR_ARG (dtype, NULL, alignment),
+ * LX_ERR_SHAPE (sizes).
+ */
+LX_API lx_status lx_align_cost(int32_t dtype, int32_t d_model, int32_t d_ff,
+                               const void* dom_gate, const void* dom_up, const void* dom_down,
+                               const void* mem_gate, const void* mem_up, const void* mem_down,
+                               float* cost, void* stream);
+
+/*
+ * lx_lap_solve (host): the permutation P minimising sum_i cost[i][P(i)]
+ * (Eq. assign), solved exactly (shortest augmenting paths with dual
+ * potentials, the scheme of Jonker and Volgenant; float64 arithmetic, O(n^3)).
+ *   cost:   HOST [n][n] fp32 (e.g. copied back from lx_align_cost), finite;
+ *   assign: HOST [n] int32 out, assign[i] = P(i);
+ *   total:  HOST double out (sum_i cost[i][P(i)] in float64), or NULL.
+ * Among several optimal permutations any one may be returned.  Errors:
+ * LX_ERR_ARG (n outside 1..65536, NULL, a NaN or infinite cost).
+ */
+LX_API lx_status lx_lap_solve(const float* cost, int32_t n, int32_t* assign, double* total);
+
+/*
+ * lx_permute_neurons: the aligned member, neuron i <- neuron perm[i]:
+ *   gate_out[i][:] = gate[perm[i]][:], up_out likewise,
+ *   down_out[:][i] = down[:][perm[i]]   (bit-exact copies).
+ *   perm: device [I] int32, a permutation of 0..I-1 (an entry outside that
+ *         range yields a zero neuron);  weights as lx_align_cost, outputs
+ *         device buffers of the same shapes that overlap no input.
+ * Stream-ordered; no allocation.  Errors: LX_ERR_ARG (dtype, NULL, alignment,
+ * overlap), LX_ERR_SHAPE (sizes).
+ */
+LX_API lx_status lx_permute_neurons(int32_t dtype, int32_t d_model, int32_t d_ff,
+                                    const int32_t* perm, const void* gate, const void* up,
+                                    const void* down, void* gate_out, void* up_out, void* down_out,
+                                    void* stream);
+
 /* Message of the last failed call on this thread ("" if none). */
 LX_API const char* lx_last_error(void);
 

@@ -36,14 +36,16 @@ def neuron_vectors(gate: np.ndarray, up: np.ndarray, down: np.ndarray) -> np.nda
     return np.concatenate([g, u, d.T], axis=1)
 
 
-def cost_matrix(dom, mem) -> np.ndarray:
-    """C[i, j] = ||a_i - b_j||^2 for dom = (gate, up, down), mem likewise."""
+def cost_matrix(dom, mem, rows=None) -> np.ndarray:
+    """C[i, j] = ||a_i - b_j||^2 for dom = (gate, up, down), mem likewise;
+    only the dominant neurons ``rows`` (all by default), in that order."""
     A = neuron_vectors(*dom)
     B = neuron_vectors(*mem)
-    C = np.empty((A.shape[0], B.shape[0]), np.float64)
-    for i in range(A.shape[0]):
+    rows = np.arange(A.shape[0]) if rows is None else np.asarray(rows, np.int64)
+    C = np.empty((len(rows), B.shape[0]), np.float64)
+    for q, i in enumerate(rows):
         diff = B - A[i]
-        C[i] = np.sum(diff * diff, axis=1)
+        C[q] = np.sum(diff * diff, axis=1)
     return C
 
 

@@ -1,0 +1,293 @@
+// Neuron alignment of a member to its dominant (Sec. 3.2 Stage 3 (i)).
+//
+// Neuron i of an expert is the vector a_i = (gate[i, :], up[i, :], down[:, i])
+// of length 3H (the x W^T storage: gate/up [I][H], down [H][I]).  The matching
+// cost is C[i][j] = ||a_i||^2 + ||b_j||^2 - 2 a_i . b_j (Eq. cost), the optimal
+// matching minimises sum_i C[i][P(i)] (Eq. assign), and the aligned member takes
+// the member's neuron P(i) as its neuron i.
+//
+// k_align_cost: one 64 x 64 tile of C per CTA, fp32 multiply-adds over the
+// three K segments (gate rows, up rows: K-major; down columns: MN-major) staged
+// through shared memory in 32-deep chunks; the tile's row norms are summed
+// from the same staged chunks, so every operand byte is read once per tile.
+// k_permute_rows / k_permute_cols: gathers (bit-exact copies).
+// lx_lap_solve: the exact assignment on the host (shortest augmenting paths
+// with dual potentials, the augmentation scheme of Jonker and Volgenant).
+#include <algorithm>
+#include <limits>
+#include <vector>
+
+#include "lx_internal.cuh"
+
+namespace lx {
+namespace {
+
+constexpr int AC_TILE = 64;     // rows (dominant neurons) and columns (member neurons) per CTA
+constexpr int AC_KC = 32;       // K chunk
+constexpr int AC_LD = AC_TILE + 4;
+constexpr int AC_THREADS = 256;
+
+// 8 consecutive elements starting at p (16-byte aligned for bf16, 32 for fp32)
+__device__ __forceinline__ void load8(const __nv_bfloat16* p, float (&v)[8]) {
+  const uint4 q = *reinterpret_cast<const uint4*>(p);
+  const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&q);
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    const float2 f = __bfloat1622float2(h[e]);
+    v[2 * e] = f.x;
+    v[2 * e + 1] = f.y;
+  }
+}
+__device__ __forceinline__ void load8(const float* p, float (&v)[8]) {
+  const float4 a = *reinterpret_cast<const float4*>(p);
+  const float4 b = *reinterpret_cast<const float4*>(p + 4);
+  v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+  v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+}
+
+// Stages the chunk (segment seg, K offset h0, length kc <= 32) of the neuron
+// vectors of rows r0 .. r0+63 into S[k][row] (zero beyond I or kc).
+//   seg 0 / 1: rows of gate / up [I][H]  (element (i, h) at i*H + h)
+//   seg 2:     columns of down [H][I]    (element (i, h) at h*I + i)
+template <typename TW>
+__device__ __forceinline__ void stage_chunk(float (*S)[AC_LD], const TW* g, const TW* u,
+                                            const TW* d, int seg, int h0, int kc, int r0,
+                                            int H, int I, int tid) {
+  float v[8];
+  if (seg < 2) {
+    const TW* W = seg == 0 ? g : u;
+    const int row = tid >> 2, hq = (tid & 3) * 8;  // 64 rows x 4 groups of 8
+    const bool ok = r0 + row < I && hq < kc;
+    if (ok) load8(W + (size_t)(r0 + row) * H + h0 + hq, v);
+#pragma unroll
+    for (int e = 0; e < 8; ++e) S[hq + e][row] = ok ? v[e] : 0.f;
+  } else {
+    const int hr = tid >> 3, iq = (tid & 7) * 8;  // 32 K rows x 8 groups of 8 neurons
+    const bool ok = hr < kc && r0 + iq < I;
+    if (ok) load8(d + (size_t)(h0 + hr) * I + r0 + iq, v);
+#pragma unroll
+    for (int e = 0; e < 8; ++e) S[hr][iq + e] = ok ? v[e] : 0.f;
+  }
+}
+
+template <typename TW>
+__global__ void __launch_bounds__(AC_THREADS)
+k_align_cost(const TW* __restrict__ dg, const TW* __restrict__ du, const TW* __restrict__ dd,
+             const TW* __restrict__ mg, const TW* __restrict__ mu, const TW* __restrict__ md,
+             int H, int I, float* __restrict__ cost) {
+  __shared__ __align__(16) float As[AC_KC][AC_LD];
+  __shared__ __align__(16) float Bs[AC_KC][AC_LD];
+  __shared__ float na[AC_TILE], nb[AC_TILE];
+  const int tid = threadIdx.x;
+  const int i0 = blockIdx.y * AC_TILE, j0 = blockIdx.x * AC_TILE;
+  const int ty = tid >> 4, tx = tid & 15;
+  float acc[4][4] = {};
+  float nrm = 0.f;  // threads 0..63: |a_{i0+tid}|^2, 64..127: |b_{j0+tid-64}|^2
+  for (int seg = 0; seg < 3; ++seg) {
+    for (int h0 = 0; h0 < H; h0 += AC_KC) {
+      const int kc = min(AC_KC, H - h0);
+      stage_chunk(As, dg, du, dd, seg, h0, kc, i0, H, I, tid);
+      stage_chunk(Bs, mg, mu, md, seg, h0, kc, j0, H, I, tid);
+      __syncthreads();
+      if (tid < 2 * AC_TILE) {
+        float (*S)[AC_LD] = tid < AC_TILE ? As : Bs;
+        const int c = tid & (AC_TILE - 1);
+#pragma unroll 8
+        for (int k = 0; k < AC_KC; ++k) nrm = fmaf(S[k][c], S[k][c], nrm);
+      }
+#pragma unroll 8
+      for (int k = 0; k < AC_KC; ++k) {
+        const float4 a = *reinterpret_cast<const float4*>(&As[k][ty * 4]);
+        const float4 b = *reinterpret_cast<const float4*>(&Bs[k][tx * 4]);
+        const float av[4] = {a.x, a.y, a.z, a.w}, bv[4] = {b.x, b.y, b.z, b.w};
+#pragma unroll
+        for (int r = 0; r < 4; ++r)
+#pragma unroll
+          for (int c = 0; c < 4; ++c) acc[r][c] = fmaf(av[r], bv[c], acc[r][c]);
+      }
+      __syncthreads();
+    }
+  }
+  if (tid < AC_TILE) na[tid] = nrm;
+  else if (tid < 2 * AC_TILE) nb[tid - AC_TILE] = nrm;
+  __syncthreads();
+#pragma unroll
+  for (int r = 0; r < 4; ++r) {
+    const int i = i0 + ty * 4 + r;
+    if (i >= I) continue;
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      const int j = j0 + tx * 4 + c;
+      if (j < I) cost[(size_t)i * I + j] = na[ty * 4 + r] + nb[tx * 4 + c] - 2.f * acc[r][c];
+    }
+  }
+}
+
+// dst row i = src row perm[i] of a [rows][cols] matrix (16-byte pieces; a row
+// whose perm entry is outside [0, rows) is written as zeros)
+__global__ void k_permute_rows(const uint4* __restrict__ src, uint4* __restrict__ dst,
+                               const int* __restrict__ perm, int rows, int pieces) {
+  const int i = blockIdx.x;
+  const int p = perm[i];
+  const bool ok = p >= 0 && p < rows;
+  for (int q = threadIdx.x; q < pieces; q += blockDim.x)
+    dst[(size_t)i * pieces + q] = ok ? src[(size_t)p * pieces + q] : make_uint4(0u, 0u, 0u, 0u);
+}
+
+// dst[h][i] = src[h][perm[i]] of a [H][cols] matrix of esz-byte elements
+template <typename TE>
+__global__ void k_permute_cols(const TE* __restrict__ src, TE* __restrict__ dst,
+                               const int* __restrict__ perm, int rows, int cols) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= cols) return;
+  const int p = perm[i];
+  const bool ok = p >= 0 && p < cols;
+  for (int h = blockIdx.y; h < rows; h += gridDim.y)
+    dst[(size_t)h * cols + i] = ok ? src[(size_t)h * cols + p] : TE(0);
+}
+
+bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+lx_status check_expert_args(int32_t dtype, int32_t H, int32_t I) {
+  if (dtype != LX_F32 && dtype != LX_BF16) return fail(LX_ERR_ARG, "unknown dtype");
+  if (H < 8 || I < 8 || H % 8 || I % 8 || H > 65536 || I > 65536)
+    return fail(LX_ERR_SHAPE, "d_model and d_ff must be multiples of 8 in 8..65536");
+  return LX_OK;
+}
+
+}  // namespace
+}  // namespace lx
+
+extern "C" lx_status lx_align_cost(int32_t dtype, int32_t d_model, int32_t d_ff,
+                                   const void* dom_gate, const void* dom_up, const void* dom_down,
+                                   const void* mem_gate, const void* mem_up, const void* mem_down,
+                                   float* cost, void* stream) {
+  using namespace lx;
+  LX_TRY(check_expert_args(dtype, d_model, d_ff));
+  const void* ptrs[7] = {dom_gate, dom_up, dom_down, mem_gate, mem_up, mem_down, cost};
+  for (const void* p : ptrs) {
+    if (!p) return fail(LX_ERR_ARG, "NULL weight or cost pointer");
+    if (!aligned16(p)) return fail(LX_ERR_ARG, "weights and cost must be 16-byte aligned");
+  }
+  const int H = d_model, I = d_ff;
+  const dim3 grid((I + AC_TILE - 1) / AC_TILE, (I + AC_TILE - 1) / AC_TILE);
+  cudaStream_t s = (cudaStream_t)stream;
+  if (dtype == LX_BF16) {
+    using B = __nv_bfloat16;
+    k_align_cost<B><<<grid, AC_THREADS, 0, s>>>((const B*)dom_gate, (const B*)dom_up,
+                                                (const B*)dom_down, (const B*)mem_gate,
+                                                (const B*)mem_up, (const B*)mem_down, H, I, cost);
+  } else {
+    k_align_cost<float><<<grid, AC_THREADS, 0, s>>>(
+        (const float*)dom_gate, (const float*)dom_up, (const float*)dom_down,
+        (const float*)mem_gate, (const float*)mem_up, (const float*)mem_down, H, I, cost);
+  }
+  LX_CUDA(cudaGetLastError());
+  return LX_OK;
+}
+
+extern "C" lx_status lx_permute_neurons(int32_t dtype, int32_t d_model, int32_t d_ff,
+                                        const int32_t* perm, const void* gate, const void* up,
+                                        const void* down, void* gate_out, void* up_out,
+                                        void* down_out, void* stream) {
+  using namespace lx;
+  LX_TRY(check_expert_args(dtype, d_model, d_ff));
+  const void* ptrs[7] = {perm, gate, up, down, gate_out, up_out, down_out};
+  for (const void* p : ptrs)
+    if (!p) return fail(LX_ERR_ARG, "NULL pointer");
+  for (int q = 1; q < 7; ++q)
+    if (!aligned16(ptrs[q])) return fail(LX_ERR_ARG, "weights must be 16-byte aligned");
+  const int H = d_model, I = d_ff;
+  const size_t esz = dtype == LX_BF16 ? 2 : 4;
+  const size_t row_bytes = (size_t)H * esz, mat = (size_t)I * H * esz;
+  // the outputs may overlap no input (a gather cannot run in place)
+  const char* ins[3] = {(const char*)gate, (const char*)up, (const char*)down};
+  const char* outs[3] = {(const char*)gate_out, (const char*)up_out, (const char*)down_out};
+  for (const char* o : outs)
+    for (const char* in : ins)
+      if (o < in + mat && in < o + mat) return fail(LX_ERR_ARG, "outputs overlap the inputs");
+  cudaStream_t s = (cudaStream_t)stream;
+  const int pieces = (int)(row_bytes / 16);
+  k_permute_rows<<<I, 128, 0, s>>>((const uint4*)gate, (uint4*)gate_out, perm, I, pieces);
+  k_permute_rows<<<I, 128, 0, s>>>((const uint4*)up, (uint4*)up_out, perm, I, pieces);
+  const dim3 cg((I + 255) / 256, std::min(H, 4096));
+  if (dtype == LX_BF16)
+    k_permute_cols<unsigned short><<<cg, 256, 0, s>>>((const unsigned short*)down,
+                                                      (unsigned short*)down_out, perm, H, I);
+  else
+    k_permute_cols<unsigned int><<<cg, 256, 0, s>>>((const unsigned int*)down,
+                                                    (unsigned int*)down_out, perm, H, I);
+  LX_CUDA(cudaGetLastError());
+  return LX_OK;
+}
+
+// Exact linear assignment on the host: rows are added one at a time, each by a
+// shortest augmenting path (Dijkstra over the columns on reduced costs
+// c[i][j] - u[i] - v[j] >= 0), after which the dual potentials u, v are updated
+// so that every reduced cost stays non-negative and those on the matching are
+// zero -- the augmentation scheme of Jonker and Volgenant.  O(n^3), float64.
+extern "C" lx_status lx_lap_solve(const float* cost, int32_t n, int32_t* assign, double* total) {
+  using namespace lx;
+  if (n < 1 || n > 65536) return fail(LX_ERR_ARG, "n must be in 1..65536");
+  if (!cost || !assign) return fail(LX_ERR_ARG, "cost or assign is NULL");
+  for (long q = 0; q < (long)n * n; ++q)
+    if (!(cost[q] == cost[q]) || cost[q] == std::numeric_limits<float>::infinity() ||
+        cost[q] == -std::numeric_limits<float>::infinity())
+      return fail(LX_ERR_ARG, "cost holds a NaN or an infinity");
+  const double kInf = std::numeric_limits<double>::infinity();
+  // column 0 is a virtual column that holds the row being added
+  std::vector<double> u(n + 1, 0.0), v(n + 1, 0.0), dist(n + 1);
+  std::vector<int> row_of(n + 1, 0), prev(n + 1, 0);  // row_of[j]: row (1-based) on column j
+  std::vector<char> done(n + 1);
+  for (int r = 1; r <= n; ++r) {
+    row_of[0] = r;
+    int col = 0;
+    std::fill(dist.begin(), dist.end(), kInf);
+    std::fill(done.begin(), done.end(), 0);
+    // grow the shortest-path tree until it reaches a free column
+    while (true) {
+      done[col] = 1;
+      const int i = row_of[col];
+      const float* ci = cost + (size_t)(i - 1) * n;
+      double best = kInf;
+      int next = -1;
+      for (int j = 1; j <= n; ++j) {
+        if (done[j]) continue;
+        const double red = (double)ci[j - 1] - u[i] - v[j];
+        if (red < dist[j]) {
+          dist[j] = red;
+          prev[j] = col;
+        }
+        if (dist[j] < best) {
+          best = dist[j];
+          next = j;
+        }
+      }
+      // shift the potentials by the step length: tree columns keep zero
+      // reduced cost along the tree, the others' tentative distances shrink
+      for (int j = 0; j <= n; ++j) {
+        if (done[j]) {
+          u[row_of[j]] += best;
+          v[j] -= best;
+        } else {
+          dist[j] -= best;
+        }
+      }
+      col = next;
+      if (row_of[col] == 0) break;
+    }
+    // augment along the path back to the virtual column
+    while (col) {
+      const int p = prev[col];
+      row_of[col] = row_of[p];
+      col = p;
+    }
+  }
+  double sum = 0.0;
+  for (int j = 1; j <= n; ++j) {
+    assign[row_of[j] - 1] = j - 1;
+  }
+  for (int i = 0; i < n; ++i) sum += (double)cost[(size_t)i * n + assign[i]];
+  if (total) *total = sum;
+  return LX_OK;
+}

@@ -29,7 +29,7 @@ EXPORTS = [
     "lx_load_compressed_layer", "lx_free_layer", "lx_reserve", "lx_route", "lx_bucket",
     "lx_moe_forward", "lx_get_buckets", "lx_layer_info", "lx_set_path", "lx_set_profiling",
     "lx_read_profile", "lx_last_error", "lx_bucket_noalloc", "lx_coact_accumulate",
-    "lx_coact_npmi",
+    "lx_coact_npmi", "lx_align_cost", "lx_lap_solve", "lx_permute_neurons",
 ]
 LX_NOALLOC_SCRATCH_BYTES = 16 << 20
 
@@ -89,6 +89,9 @@ def lib() -> ctypes.CDLL:
             "lx_bucket_noalloc": [vp, vp, i32, i32, vp, vp, vp, vp, vp, vp],
             "lx_coact_accumulate": [vp, i32, i32, i32, vp, vp, vp],
             "lx_coact_npmi": [vp, i32, ctypes.c_int64, vp, vp],
+            "lx_align_cost": [i32, i32, i32, vp, vp, vp, vp, vp, vp, vp, vp],
+            "lx_lap_solve": [vp, i32, vp, ctypes.POINTER(ctypes.c_double)],
+            "lx_permute_neurons": [i32, i32, i32, vp, vp, vp, vp, vp, vp, vp, vp],
         }
         for name, args in sig.items():
             f = getattr(L, name)
@@ -272,3 +275,46 @@ def coact_npmi(coact: torch.Tensor, n_tokens: int, stream=None) -> torch.Tensor:
     out = torch.empty((E, E), dtype=torch.float64, device=coact.device)
     _check(lib().lx_coact_npmi(_ptr(coact), E, n_tokens, _ptr(out), _stream(stream)))
     return out
+
+
+# ----------------------------------------------------------------------------
+# neuron alignment (standalone calls on plain expert matrices)
+# ----------------------------------------------------------------------------
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.bfloat16:
+        return LX_BF16
+    if t.dtype == torch.float32:
+        return LX_F32
+    raise ValueError("expert matrices must be bf16 or fp32")
+
+
+def align_cost(dom, mem, stream=None) -> torch.Tensor:
+    """fp32 [I, I] cost of matching dominant neurons (rows) with member neurons
+    (columns); dom and mem are (gate [I,H], up [I,H], down [H,I]) device tensors."""
+    g = dom[0]
+    I, H = g.shape
+    cost = torch.empty((I, I), dtype=torch.float32, device=g.device)
+    _check(lib().lx_align_cost(_dtype_code(g), H, I, *[_ptr(t) for t in dom],
+                               *[_ptr(t) for t in mem], _ptr(cost), _stream(stream)))
+    return cost
+
+
+def lap_solve(cost: np.ndarray):
+    """(assign int32 [n], total float) of the exact assignment of a host cost."""
+    c = np.ascontiguousarray(cost, dtype=np.float32)
+    n = c.shape[0]
+    out = np.empty(n, np.int32)
+    tot = ctypes.c_double()
+    _check(lib().lx_lap_solve(ctypes.c_void_p(c.ctypes.data), n,
+                              ctypes.c_void_p(out.ctypes.data), ctypes.byref(tot)))
+    return out, tot.value
+
+
+def permute_neurons(perm: torch.Tensor, gate: torch.Tensor, up: torch.Tensor,
+                    down: torch.Tensor, stream=None):
+    """(gate, up, down) of the member with neuron i taken from neuron perm[i]."""
+    I, H = gate.shape
+    outs = (torch.empty_like(gate), torch.empty_like(up), torch.empty_like(down))
+    _check(lib().lx_permute_neurons(_dtype_code(gate), H, I, _ptr(perm), _ptr(gate), _ptr(up),
+                                    _ptr(down), *[_ptr(t) for t in outs], _stream(stream)))
+    return outs

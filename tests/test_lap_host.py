@@ -1,0 +1,70 @@
+"""The library's exact assignment solver (lx_lap_solve, host code behind the C
+ABI; Eq. assign) against SciPy's exact solver and brute force.  Runs without a
+GPU."""
+import itertools
+import os
+
+import numpy as np
+import pytest
+
+from oracle import align
+from paper_2608_07814_gb300 import build as lxbuild
+from paper_2608_07814_gb300 import lx
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not os.path.exists(lx.LIB_PATH):
+        lxbuild.build()
+    lx.lib()
+
+
+@pytest.mark.parametrize("n,seed", [(1, 0), (2, 1), (4, 2), (6, 3), (7, 4), (7, 5)])
+def test_brute_force(n, seed):
+    rng = np.random.default_rng(seed)
+    C = rng.random((n, n)).astype(np.float32)
+    if seed == 5:
+        C = np.round(C * 2).astype(np.float32)   # ties
+    P, tot = lx.lap_solve(C)
+    assert sorted(P.tolist()) == list(range(n))
+    best = min(sum(float(C[i, p[i]]) for i in range(n)) for p in itertools.permutations(range(n)))
+    assert abs(tot - best) <= 1e-9
+    assert abs(align.assignment_cost(C, P) - tot) <= 1e-9
+
+
+@pytest.mark.parametrize("n,kind", [(50, "uniform"), (200, "int"), (300, "neurons"),
+                                    (768, "neurons")])
+def test_matches_scipy_optimum(n, kind):
+    rng = np.random.default_rng(n)
+    if kind == "uniform":
+        C = rng.random((n, n)).astype(np.float32)
+    elif kind == "int":
+        C = rng.integers(0, 10, (n, n)).astype(np.float32)   # heavy ties
+    else:
+        # squared distances of neuron vectors, a planted permutation plus noise
+        H = 32
+        A = rng.standard_normal((n, 3 * H))
+        sigma = rng.permutation(n)
+        B = A[sigma] + 0.3 * rng.standard_normal((n, 3 * H))
+        C = ((A[:, None, :] - B[None, :, :]) ** 2).sum(-1).astype(np.float32)
+    P, tot = lx.lap_solve(C)
+    assert sorted(P.tolist()) == list(range(n))
+    ref = align.assignment_cost(C, align.assign(C))
+    assert abs(tot - ref) <= 1e-9 * max(1.0, abs(ref))
+    if kind == "neurons" and n == 300:
+        inv = np.empty(n, np.int64)
+        inv[sigma] = np.arange(n)
+        assert np.array_equal(P, inv)
+
+
+def test_negative_costs_and_rejects():
+    C = -np.arange(16, dtype=np.float32).reshape(4, 4)
+    P, tot = lx.lap_solve(C)
+    assert abs(tot - align.assignment_cost(C, align.assign(C))) <= 1e-9
+    bad = C.copy()
+    bad[1, 2] = np.nan
+    with pytest.raises(lx.LxError):
+        lx.lap_solve(bad)
+    bad[1, 2] = np.inf
+    with pytest.raises(lx.LxError):
+        lx.lap_solve(bad)
