@@ -55,6 +55,15 @@ WORKLOADS = {
 }
 
 
+# standalone kernels of the compression pipeline (timed on their own)
+OFFLINE = {
+    "coact": "router profiling statistics: co-activation counts of 8192-token batches of the "
+             "Qwen3-30B-A3B-shaped layer's top-8 routing (E=128)",
+    "align": "neuron alignment of one member to its dominant at the Qwen3-30B-A3B expert shape "
+             "(H=2048, I=768): cost matrix, exact assignment, permutation",
+}
+
+
 def make_layer(kind):
     import synth
     return {"qwen": synth.qwen_decode_layer, "high_e": synth.high_e_layer,
@@ -494,6 +503,123 @@ def run_lx(args, rank, world, local_rank):
     return line
 
 
+def _event_ms(fn, steps, warmup):
+    """Average ms per call of fn() over `steps` calls on the current stream
+    (CUDA events, synchronised on both sides), after `warmup` calls."""
+    import torch
+    for _ in range(warmup):
+        fn()
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(steps):
+        fn()
+    b.record()
+    torch.cuda.synchronize()
+    return a.elapsed_time(b) / steps
+
+
+def run_offline(args, rank, world, local_rank):
+    import torch
+    import synth
+    import oracle
+    from oracle import align as oalign, stats as ostats
+    from paper_2608_07814_gb300 import lx
+
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    peaks, peak_kind = load_peaks()
+    hbm = float(peaks["hbm_gbs"])
+    line = {"n_gpus": world, "steps": args.steps, "warmup": args.warmup, "scaling": "weak",
+            "vs_baseline": None, "data": "synthetic", "impl": "lx",
+            "config": {"workload": OFFLINE[args.workload]}}
+    if args.workload == "coact":
+        src = make_layer("qwen")
+        L = lx.Layer(src)
+        T, k, E, nb = 8192, 8, src.n_experts, 16
+        ids = []
+        for b in range(nb):
+            x = lx.host_to_torch(synth.tokens(src, T, seed=batch_seed(rank, b)), "bf16").to(dev)
+            ids.append(L.route(x, k)[0])
+        fire = torch.zeros(E, dtype=torch.int64, device=dev)
+        coact = torch.zeros((E, E), dtype=torch.int64, device=dev)
+        it = [0]
+
+        def step():
+            lx.coact_accumulate(ids[it[0] % nb], E, fire, coact)
+            it[0] += 1
+        ms = _event_ms(step, args.steps, args.warmup)
+        byts = T * k * 4 + 2 * E * E * 8
+        t_npmi = _event_ms(lambda: lx.coact_npmi(coact, T * nb), 20, 3)
+        host_ids = [i.cpu().numpy() for i in ids[:2]]
+        t0 = time.time()
+        for h in host_ids:
+            ostats.coact_counts(h[:1024], E)
+        cpu = 2 * 1024 / (time.time() - t0)
+        line.update({"metric": "router-statistics tokens/s (co-activation counts)",
+                     "value": round(whole_job_rate(T, 1, world, ms), 1), "unit": "tokens/s",
+                     "ms_per_step": round(ms, 5), "higher_is_better": True, "dtype": "int64",
+                     "gpu_launches": args.steps,
+                     "roofline": {"kernel": "k_coact_smem", "bound": "hbm",
+                                  "achieved": round(byts / (ms * 1e-3) / 1e9, 1), "peak": hbm,
+                                  "unit": "GB/s", "frac": round(byts / (ms * 1e-3) / 1e9 / hbm, 5),
+                                  "traffic": None, "note": "latency-bound: 256 KB of ids per launch"},
+                     "npmi_us": round(t_npmi * 1e3, 2),
+                     "cpu_baseline": {"value": round(cpu, 1), "unit": "tokens/s", "cores": 1,
+                                      "kind": "oracle", "sample": "2 x 1024 tokens"}})
+        line["config"].update({"tokens_per_step": T, "n_experts": E, "top_k": k,
+                               "l2": "16 rotating id batches (4 MB, L2-resident)"})
+    else:
+        H, I = 2048, 768
+        rng = np.random.default_rng(rank)
+        draw = lambda s: synth.to_storage(rng.standard_normal(s).astype(np.float32) * 0.02, "bf16")
+        dom = [draw((I, H)), draw((I, H)), draw((H, I))]
+        mems = [[draw((I, H)), draw((I, H)), draw((H, I))] for _ in range(4)]
+        dd = tuple(lx.host_to_torch(w, "bf16").to(dev) for w in dom)
+        md = [tuple(lx.host_to_torch(w, "bf16").to(dev) for w in m) for m in mems]
+        it = [0]
+
+        def step():
+            lx.align_cost(dd, md[it[0] % 4])
+            it[0] += 1
+        ms = _event_ms(step, args.steps, args.warmup)
+        cost = lx.align_cost(dd, md[0]).cpu().numpy()
+        t0 = time.time()
+        P, _ = lx.lap_solve(cost)
+        lap_s = time.time() - t0
+        Pd = torch.from_numpy(P).to(dev)
+        ms_perm = _event_ms(lambda: lx.permute_neurons(Pd, *md[1]), 20, 3)
+        flops = 2.0 * I * I * 3 * H + 2.0 * 2 * I * 3 * H
+        alu = fp32_alu_peak_tflops(peaks)
+        ach = flops / (ms * 1e-3) / 1e12
+        pbytes = 2 * 3 * I * H * 2 + I * 4
+        t0 = time.time()
+        oalign.assign(oalign.cost_matrix(tuple(synth.from_storage(w, "bf16") for w in dom),
+                                         tuple(synth.from_storage(w, "bf16") for w in mems[0]),
+                                         rows=np.arange(64)))
+        cpu_rows = 64 / (time.time() - t0)
+        line.update({"metric": "neuron-alignment cost matrices/s (one member vs its dominant)",
+                     "value": round(1e3 / ms * world, 2), "unit": "matrices/s",
+                     "ms_per_step": round(ms, 5), "higher_is_better": True, "dtype": "f32",
+                     "gpu_launches": args.steps,
+                     "roofline": {"kernel": "k_align_cost", "bound": "alu", "achieved": round(ach, 2),
+                                  "peak": round(alu, 1), "unit": "TFLOP/s",
+                                  "frac": round(ach / alu, 4), "traffic": None,
+                                  "peak_source": "fp32 FMA: 152 SMs x 128 lanes x 2 x sm_max_mhz"},
+                     "lap_host_s": round(lap_s, 3),
+                     "permute": {"us": round(ms_perm * 1e3, 2),
+                                 "gbs": round(pbytes / (ms_perm * 1e-3) / 1e9, 1),
+                                 "frac_hbm": round(pbytes / (ms_perm * 1e-3) / 1e9 / hbm, 4)},
+                     "e2e": {"value": round(1.0 / (ms * 1e-3 + lap_s + ms_perm * 1e-3), 3),
+                             "unit": "members aligned/s (cost + host assignment + permutation)",
+                             "h2d_bytes_per_step": 0, "d2h_bytes_per_step": I * I * 4},
+                     "cpu_baseline": {"value": round(cpu_rows / I, 5), "unit": "matrices/s",
+                                      "cores": os.cpu_count(), "kind": "oracle",
+                                      "sample": "64 of the 768 cost rows (float64 definition)"}})
+        line["config"].update({"d_model": H, "d_ff": I, "l2": "4 rotating members (L2-resident)"})
+    return line
+
+
 def cpu_baseline(src, xs_host, T, budget_s):
     """The oracle, as it stands, on a bounded sample of the same workload."""
     import oracle
@@ -550,7 +676,7 @@ def main():
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=400)
     ap.add_argument("--warmup", type=int, default=20)
-    ap.add_argument("--workload", default="decode64", choices=sorted(WORKLOADS))
+    ap.add_argument("--workload", default="decode64", choices=sorted(WORKLOADS) + sorted(OFFLINE))
     ap.add_argument("--impl", default="lx", choices=["lx", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
@@ -570,7 +696,10 @@ def main():
         import torch
         torch.cuda.set_device(local_rank)
         torch.distributed.init_process_group("nccl")
-    if args.impl == "reference":
+    if args.workload in OFFLINE:
+        line = run_offline(args, rank, world, local_rank) if args.impl == "lx" else \
+            {"impl": "reference", "unavailable": "the reference arm times the forward only"}
+    elif args.impl == "reference":
         line = run_reference(args, rank, world)
     else:
         line = run_lx(args, rank, world, local_rank)
