@@ -61,6 +61,9 @@ OFFLINE = {
              "Qwen3-30B-A3B-shaped layer's top-8 routing (E=128)",
     "align": "neuron alignment of one member to its dominant at the Qwen3-30B-A3B expert shape "
              "(H=2048, I=768): cost matrix, exact assignment, permutation",
+    "compress": "compression of one member at the Qwen3-30B-A3B expert shape (H=2048, I=768): "
+                "rank-128 randomized SVD (oversampling 8, 2 power iterations) of the gate, up "
+                "and down residuals with the symmetric split",
 }
 
 
@@ -569,6 +572,49 @@ def run_offline(args, rank, world, local_rank):
                                       "kind": "oracle", "sample": "2 x 1024 tokens"}})
         line["config"].update({"tokens_per_step": T, "n_experts": E, "top_k": k,
                                "l2": "16 rotating id batches (4 MB, L2-resident)"})
+    elif args.workload == "compress":
+        H, I, r, l, q = 2048, 768, 128, 136, 2
+        rng = np.random.default_rng(rank)
+        draw = lambda s: synth.to_storage(rng.standard_normal(s).astype(np.float32) * 0.02, "bf16")
+        shapes = [(I, H), (I, H), (H, I)]
+        dom = [draw(sh) for sh in shapes]
+        mem = [draw(sh) for sh in shapes]
+        oms = [rng.standard_normal((sh[1], l)).astype(np.float32) for sh in shapes]
+        dd = [lx.host_to_torch(w, "bf16").to(dev) for w in dom]
+        md = [lx.host_to_torch(w, "bf16").to(dev) for w in mem]
+        od = [torch.from_numpy(o).to(dev) for o in oms]
+        ws = torch.empty(max(lx.compress_workspace_bytes(a, b, l, r) for a, b in shapes),
+                         dtype=torch.uint8, device=dev)
+
+        def step():
+            for p in range(3):
+                lx.compress_factor(dd[p], md[p], od[p], r, q, workspace=ws)
+        ms = _event_ms(step, args.steps, args.warmup)
+        big = sum((2 + 2 * q) * 2.0 * a * b * l for a, b in shapes)        # the R-sized products
+        small = sum(2 * (1 + 2 * q) * 2 * (2.0 * a * l * l + a * l * l) + 2.0 * b * l * l
+                    + 2.0 * (a + b) * l * r for a, b in shapes)           # Grams, orthonormalisation
+        alu = fp32_alu_peak_tflops(peaks)
+        ach = (big + small) / (ms * 1e-3) / 1e12
+        t0 = time.time()
+        for p in range(3):
+            R = synth.from_storage(mem[p], "bf16") - synth.from_storage(dom[p], "bf16")
+            from oracle import compress as ocomp
+            ocomp.randomized_factors(R, r, oms[p].astype(np.float64), q)
+        cpu_s = time.time() - t0
+        line.update({"metric": "members compressed/s (gate, up and down residuals, rank 128)",
+                     "value": round(1e3 / ms * world, 3), "unit": "members/s",
+                     "ms_per_step": round(ms, 4), "higher_is_better": True, "dtype": "f32",
+                     "gpu_launches": args.steps * 3 * (2 + (1 + 2 * q) * 6 + 3 + 2),
+                     "roofline": {"kernel": "whole compression step", "bound": "alu",
+                                  "achieved": round(ach, 2), "peak": round(alu, 1),
+                                  "unit": "TFLOP/s", "frac": round(ach / alu, 4), "traffic": None,
+                                  "algorithmic_flops_per_step": round(big + small),
+                                  "peak_source": "fp32 FMA: 152 SMs x 128 lanes x 2 x sm_max_mhz"},
+                     "cpu_baseline": {"value": round(1.0 / cpu_s, 4), "unit": "members/s",
+                                      "cores": os.cpu_count(), "kind": "oracle",
+                                      "sample": "one member (3 projections), float64 numpy"}})
+        line["config"].update({"d_model": H, "d_ff": I, "rank": r, "oversampling": l - r,
+                               "power_iters": q, "l2": "one member (L2-resident)"})
     else:
         H, I = 2048, 768
         rng = np.random.default_rng(rank)

@@ -333,6 +333,38 @@ LX_API lx_status lx_permute_neurons(int32_t dtype, int32_t d_model, int32_t d_ff
                                     const void* down, void* gate_out, void* up_out, void* down_out,
                                     void* stream);
 
+/*
+ * Compression of one member projection (Sec. 3.2 Stage 3 (ii)): the residual
+ * R = W_mem - W_dom (Eq. svd; W_mem already aligned) and its rank-r randomized
+ * SVD with the symmetric split of Eq. factors:
+ *   U = U_r S_r^(1/2) [rows][r] (the paper's B_m),  V = V_r S_r^(1/2) [cols][r]
+ *   (A_m^T), so that U V^T ~ R, plus the singular values s [r].
+ * Solver: Y = R Omega, Q = orth(Y); power_iters times Q = orth(R orth(R^T Q));
+ * then the SVD of Q^T R through the l x l Gram (Jacobi, float64); products in
+ * fp32 (CUDA cores), Gram matrices, orthonormalisation (CholeskyQR, twice) and
+ * eigenvectors in float64.  The sign of each factor column is fixed so that the
+ * largest-magnitude entry of U's column is positive.  Singular values at or
+ * below 1e-6 of the largest give zero V columns.
+ *   dtype:      LX_F32 or LX_BF16 of w_dom / w_mem
+ *   rows, cols: the projection's [out][in] shape, multiples of 8 (gate / up:
+ *               [I][H], down: [H][I]); w_dom, w_mem device, 16-byte aligned
+ *   omega:      device [cols][l] fp32, the Gaussian test matrix (the caller
+ *               draws it: the random numbers are an input)
+ *   l, r:       1 <= r <= l <= min(rows, cols, 256) (l = r + oversampling)
+ *   power_iters 0..16
+ *   U, V, s:    device fp32 outputs [rows][r], [cols][r], [r]
+ *   workspace:  device, 256-byte aligned, >= lx_compress_workspace bytes
+ *               (caller-owned; nothing is allocated)
+ * Stream-ordered.  Errors: LX_ERR_ARG (dtype, NULL, alignment, power_iters,
+ * workspace too small), LX_ERR_SHAPE (sizes).
+ */
+LX_API lx_status lx_compress_workspace(int32_t rows, int32_t cols, int32_t l, int32_t r,
+                                       uint64_t* bytes);
+LX_API lx_status lx_compress_factor(int32_t dtype, int32_t rows, int32_t cols, const void* w_dom,
+                                    const void* w_mem, const float* omega, int32_t l, int32_t r,
+                                    int32_t power_iters, float* U, float* V, float* s,
+                                    void* workspace, uint64_t workspace_bytes, void* stream);
+
 /* Message of the last failed call on this thread ("" if none). */
 LX_API const char* lx_last_error(void);
 

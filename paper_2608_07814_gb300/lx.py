@@ -30,6 +30,7 @@ EXPORTS = [
     "lx_moe_forward", "lx_get_buckets", "lx_layer_info", "lx_set_path", "lx_set_profiling",
     "lx_read_profile", "lx_last_error", "lx_bucket_noalloc", "lx_coact_accumulate",
     "lx_coact_npmi", "lx_align_cost", "lx_lap_solve", "lx_permute_neurons",
+    "lx_compress_workspace", "lx_compress_factor",
 ]
 LX_NOALLOC_SCRATCH_BYTES = 16 << 20
 
@@ -92,6 +93,9 @@ def lib() -> ctypes.CDLL:
             "lx_align_cost": [i32, i32, i32, vp, vp, vp, vp, vp, vp, vp, vp],
             "lx_lap_solve": [vp, i32, vp, ctypes.POINTER(ctypes.c_double)],
             "lx_permute_neurons": [i32, i32, i32, vp, vp, vp, vp, vp, vp, vp, vp],
+            "lx_compress_workspace": [i32, i32, i32, i32, ctypes.POINTER(ctypes.c_uint64)],
+            "lx_compress_factor": [i32, i32, i32, vp, vp, vp, i32, i32, i32, vp, vp, vp, vp,
+                                   ctypes.c_uint64, vp],
         }
         for name, args in sig.items():
             f = getattr(L, name)
@@ -318,3 +322,32 @@ def permute_neurons(perm: torch.Tensor, gate: torch.Tensor, up: torch.Tensor,
     _check(lib().lx_permute_neurons(_dtype_code(gate), H, I, _ptr(perm), _ptr(gate), _ptr(up),
                                     _ptr(down), *[_ptr(t) for t in outs], _stream(stream)))
     return outs
+
+
+# ----------------------------------------------------------------------------
+# compression of one member projection
+# ----------------------------------------------------------------------------
+def compress_workspace_bytes(rows: int, cols: int, l: int, r: int) -> int:
+    b = ctypes.c_uint64()
+    _check(lib().lx_compress_workspace(rows, cols, l, r, ctypes.byref(b)))
+    return int(b.value)
+
+
+def compress_factor(w_dom: torch.Tensor, w_mem: torch.Tensor, omega: torch.Tensor, r: int,
+                    power_iters: int = 2, workspace: Optional[torch.Tensor] = None,
+                    stream=None):
+    """(U [rows, r], V [cols, r], s [r]) fp32 with U V^T ~ w_mem - w_dom; omega
+    is the fp32 [cols, l] Gaussian test matrix."""
+    rows, cols = w_dom.shape
+    l = omega.shape[1]
+    need = compress_workspace_bytes(rows, cols, l, r)
+    if workspace is None:
+        workspace = torch.empty(need, dtype=torch.uint8, device=w_dom.device)
+    dev = w_dom.device
+    U = torch.empty((rows, r), dtype=torch.float32, device=dev)
+    V = torch.empty((cols, r), dtype=torch.float32, device=dev)
+    s = torch.empty(r, dtype=torch.float32, device=dev)
+    _check(lib().lx_compress_factor(_dtype_code(w_dom), rows, cols, _ptr(w_dom), _ptr(w_mem),
+                                    _ptr(omega), l, r, power_iters, _ptr(U), _ptr(V), _ptr(s),
+                                    _ptr(workspace), workspace.numel(), _stream(stream)))
+    return U, V, s

@@ -46,7 +46,7 @@ def test_matches_scipy_optimum(n, kind):
         A = rng.standard_normal((n, 3 * H))
         sigma = rng.permutation(n)
         B = A[sigma] + 0.3 * rng.standard_normal((n, 3 * H))
-        C = ((A[:, None, :] - B[None, :, :]) ** 2).sum(-1).astype(np.float32)
+        C = ((A * A).sum(1)[:, None] + (B * B).sum(1)[None, :] - 2.0 * A @ B.T).astype(np.float32)
     P, tot = lx.lap_solve(C)
     assert sorted(P.tolist()) == list(range(n))
     ref = align.assignment_cost(C, align.assign(C))
