@@ -604,7 +604,7 @@ def run_offline(args, rank, world, local_rank):
         line.update({"metric": "members compressed/s (gate, up and down residuals, rank 128)",
                      "value": round(1e3 / ms * world, 3), "unit": "members/s",
                      "ms_per_step": round(ms, 4), "higher_is_better": True, "dtype": "f32",
-                     "gpu_launches": args.steps * 3 * (2 + (1 + 2 * q) * 6 + 3 + 2),
+                     "gpu_launches": args.steps * 3 * (7 + 6 * (1 + 2 * q) + 2 * q),
                      "roofline": {"kernel": "whole compression step", "bound": "alu",
                                   "achieved": round(ach, 2), "peak": round(alu, 1),
                                   "unit": "TFLOP/s", "frac": round(ach / alu, 4), "traffic": None,
