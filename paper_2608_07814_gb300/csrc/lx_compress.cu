@@ -9,14 +9,19 @@
 //               shared memory); its A operand is R (rows of W_mem - W_dom,
 //               formed on load), R^T (columns of the same), or an fp32 matrix.
 //   k_gram      G = X^T X in float64 (fp32 inputs, float64 products and sums).
-//   k_chol_inv  one CTA: Cholesky G + s I = L L^T (float64, a small relative
-//               shift keeps rank-deficient bases factorable) and T = L^-T
-//               (fp32) so that X T has orthonormal columns (CholeskyQR; run
-//               twice per orthonormalisation).
-//   k_jacobi    one CTA: cyclic parallel Jacobi eigensolver (float64) of the
-//               l x l Gram of the projected residual, the r largest
-//               eigenpairs and the fp32 matrices that turn the basis into the
-//               split factors.
+//   k_chol32    one CTA: Cholesky G + s I = L L^T (fp32 in shared memory; a
+//               small relative shift in the first of the two passes keeps
+//               rank-deficient bases factorable) and T = L^-T, so that X T has
+//               orthonormal columns (CholeskyQR, run twice per
+//               orthonormalisation).
+//   k_trmm      M = L1 L2, the triangular factor of R^T Q = Z2 M^T.
+//   k_onesided  one CTA: one-sided Jacobi SVD of M (fp32 rotations, shared
+//               memory), M W = U S.
+//   k_ritz      sigma_j = |M w_j| / |w_j| in float64 (Rayleigh quotients).
+//   k_finish    the r largest sigma and the fp32 matrices that turn the bases
+//               into the split factors.
+// Only the Gram sums and the Rayleigh quotients use float64: a single SM's
+// float64 rate is a small fraction of its fp32 rate on this GPU.
 //   k_sign      each factor column's largest-magnitude entry of U made
 //               positive (U and V negated together).
 #include <algorithm>
@@ -155,209 +160,235 @@ k_gram(const float* __restrict__ X, int n, int L, double* __restrict__ G) {
   if (i0 + ti < L && j0 + tj < L) G[(size_t)(i0 + ti) * L + j0 + tj] = acc;
 }
 
-// One CTA (blockDim >= L, L <= 256).  Lw [L][L] float64 workspace.
-// Cholesky of G + s I with s = 1e-11 * trace(G) (s = 1 when G = 0), then
-// X = L^-1 column by column (thread c solves L x = e_c) and T = X^T (fp32,
-// upper triangular), so that Y T = Y L^-T has orthonormal columns when
-// Y^T Y = G.
+// One CTA (L <= 256).  Cholesky of G + s I in fp32 (G float64, rounded once;
+// s = shift_rel * max diag(G)) in a packed lower triangle in shared memory
+// (L (L + 1) / 2 floats), pivots floored at 1e-30; then X = L^-1 by forward
+// substitution (thread c owns column c, kept in the global scratch Xg so that
+// a warp reads one contiguous piece of a row per step) and T = X^T, so that
+// Y T = Y L^-T has orthonormal columns when Y^T Y = G (CholeskyQR).  The factor
+// itself is written to Lout [L][L] (zero above the diagonal).  A zero Gram
+// gives Lout = T = 0.
 constexpr int CH_THREADS = 256;
 __global__ void __launch_bounds__(CH_THREADS)
-k_chol_inv(const double* __restrict__ G, int L, double* __restrict__ Lw,
-           double* __restrict__ Xw, float* __restrict__ T) {
-  __shared__ double s_shift;
-  const int tid = threadIdx.x;
+k_chol32(const double* __restrict__ G, int L, float shift_rel, float* __restrict__ Lout,
+         float* __restrict__ Xg, float* __restrict__ T) {
+  extern __shared__ float Ls[];
+  __shared__ double s_md;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nw = CH_THREADS / 32;
   if (tid == 0) {
-    double tr = 0.0;
-    for (int i = 0; i < L; ++i) tr += G[(size_t)i * L + i];
-    s_shift = tr > 0.0 ? 1e-11 * tr : 1.0;
+    double md = 0.0;
+    for (int i = 0; i < L; ++i) md = fmax(md, G[(size_t)i * L + i]);
+    s_md = md;
   }
   __syncthreads();
-  // lower triangle of G + s I (the upper triangle of Lw is never read)
-  for (int q = tid; q < L * L; q += CH_THREADS) {
-    const int i = q / L, j = q % L;
-    Lw[q] = j <= i ? G[q] + (i == j ? s_shift : 0.0) : 0.0;
+  const double md = s_md;
+  if (!(md > 0.0)) {
+    for (int q = tid; q < L * L; q += CH_THREADS) {
+      Lout[q] = 0.f;
+      T[q] = 0.f;
+    }
+    return;
   }
+  const float shift = (float)(shift_rel * md);
+  for (int i = warp; i < L; i += nw)
+    for (int j = lane; j <= i; j += 32)
+      Ls[i * (i + 1) / 2 + j] = (float)G[(size_t)i * L + j] + (i == j ? shift : 0.f);
   __syncthreads();
   for (int j = 0; j < L; ++j) {
-    if (tid == 0) {
-      const double d = Lw[(size_t)j * L + j];
-      Lw[(size_t)j * L + j] = sqrt(d > 1e-300 ? d : 1e-300);
-    }
+    const int jj = j * (j + 1) / 2 + j;
+    if (tid == 0) Ls[jj] = sqrtf(fmaxf(Ls[jj], 1e-30f));
     __syncthreads();
-    const double ljj = Lw[(size_t)j * L + j];
-    for (int i = j + 1 + tid; i < L; i += CH_THREADS) Lw[(size_t)i * L + j] /= ljj;
+    const float ljj = Ls[jj];
+    for (int i = j + 1 + tid; i < L; i += CH_THREADS) Ls[i * (i + 1) / 2 + j] /= ljj;
     __syncthreads();
-    // trailing update of the lower triangle: A[i][c] -= L[i][j] L[c][j], j < c <= i
-    const int w = L - j - 1;
-    for (int q = tid; q < w * w; q += CH_THREADS) {
-      const int i = j + 1 + q / w, c = j + 1 + q % w;
-      if (c <= i) Lw[(size_t)i * L + c] -= Lw[(size_t)i * L + j] * Lw[(size_t)c * L + j];
+    for (int i = j + 1 + warp; i < L; i += nw) {
+      const float lij = Ls[i * (i + 1) / 2 + j];
+      for (int c = j + 1 + lane; c <= i; c += 32) Ls[i * (i + 1) / 2 + c] -= lij * Ls[c * (c + 1) / 2 + j];
     }
     __syncthreads();
   }
-  // X = L^-1, row by row: thread c owns column c (x_i = -sum_{c<=k<i} L[i][k]
-  // x_k / L[i][i]); uniform loops, so a warp reads one broadcast L[i][k] and a
-  // contiguous piece of row k of X per step.  Each thread reads back only its
-  // own column, so the rows need no barrier between them.
+  for (int q = tid; q < L * L; q += CH_THREADS) {
+    const int i = q / L, c = q % L;
+    Lout[q] = c <= i ? Ls[i * (i + 1) / 2 + c] : 0.f;
+  }
   if (tid < L) {
     const int c = tid;
     for (int i = 0; i < L; ++i) {
-      double acc = 0.0;
+      const float* Li = Ls + i * (i + 1) / 2;
+      float acc = 0.f;
       for (int k = 0; k < i; ++k)
-        if (k >= c) acc = fma(Lw[(size_t)i * L + k], Xw[(size_t)k * L + c], acc);
-      const double lii = Lw[(size_t)i * L + i];
-      Xw[(size_t)i * L + c] = i < c ? 0.0 : (i == c ? 1.0 / lii : -acc / lii);
+        if (k >= c) acc = fmaf(Li[k], Xg[(size_t)k * L + c], acc);
+      Xg[(size_t)i * L + c] = i < c ? 0.f : (i == c ? 1.f / Li[i] : -acc / Li[i]);
     }
   }
   __syncthreads();
   for (int q = tid; q < L * L; q += CH_THREADS) {
     const int k = q / L, n = q % L;  // T[k][n] = X[n][k]
-    T[q] = (float)Xw[(size_t)n * L + k];
+    T[q] = Xg[(size_t)n * L + k];
   }
 }
 
-// Symmetric eigensolver for the l x l Gram S = Z^T Z (Z = R^T Q, so S = Bs Bs^T
-// for Bs = Q^T R), then the factor matrices of the r largest eigenpairs.
-// Cyclic Jacobi, parallel form: Lp = l rounded up to even; in each of the
-// Lp - 1 rounds of a sweep the indices are split into Lp / 2 disjoint pairs
-// (circle method: index Lp - 1 fixed, the others rotated), every pair's
-// rotation J = [[c, s], [-s, c]] zeroes its off-diagonal entry, and
-// A <- J^T A J, V <- V J are applied as independent 2 x 2 blocks (each entry
-// has one writer per round).  A padding index (odd l) stays decoupled: its row
-// and column are zero, so its rotations are the identity.  Sweeps stop when
-// the off-diagonal mass is below 1e-28 of the total (squared norms) or after
-// JB_MAX_SWEEPS.  A lives in shared memory when it fits, else in `Ag`.
-// Outputs, for c < r with i_c the c-th largest eigenvalue lambda (ties: lower
-// index first) and sigma_c = sqrt(max(lambda, 0)):
-//   sig[c] = sigma_c;  Wu[k][c] = V[k][i_c] sqrt(sigma_c);
-//   Wv[k][c] = V[k][i_c] / sqrt(sigma_c), or 0 when sigma_c <= 1e-6 sigma_0.
-// Q Wu = U_r S_r^(1/2) and Z Wv = V_r S_r^(1/2) (Eq. factors).
-constexpr int JB_THREADS = 512;
-constexpr int JB_MAX_L = 256;
-constexpr int JB_MAX_SWEEPS = 30;
+// Mt (column-major, Mt[j][i] = M[i][j]) of M = L1 L2 for lower-triangular
+// L1, L2 [L][L] (fp32, float64 sums).  CTA i, thread j.
+__global__ void k_trmm(const float* __restrict__ L1, const float* __restrict__ L2, int L,
+                       float* __restrict__ Mt) {
+  const int i = blockIdx.x, j = threadIdx.x;
+  if (j >= L) return;
+  double acc = 0.0;
+  for (int k = j; k <= i; ++k) acc = fma((double)L1[(size_t)i * L + k], (double)L2[(size_t)k * L + j], acc);
+  Mt[(size_t)j * L + i] = (float)acc;
+}
 
-__global__ void __launch_bounds__(JB_THREADS)
-k_jacobi(const double* __restrict__ S, int L, int r, double* __restrict__ Ag,
-         double* __restrict__ V, int a_in_smem, float* __restrict__ Wu,
-         float* __restrict__ Wv, float* __restrict__ sig) {
-  extern __shared__ double Asm[];
-  __shared__ double pc[JB_MAX_L / 2], ps[JB_MAX_L / 2];
-  __shared__ int pp[JB_MAX_L / 2], pq[JB_MAX_L / 2];
-  __shared__ int order[JB_MAX_L];
-  __shared__ double red[2][JB_THREADS / 32];
-  __shared__ int s_done;
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+// One-sided Jacobi SVD of M (Hestenes), one CTA: the columns of M are
+// orthogonalised by plane rotations applied from the right, M W = U S, W
+// orthogonal.  Lp = L rounded up to even (a zero padding column never rotates);
+// each round pairs the columns by the circle method, a warp takes a pair:
+// alpha = |m_p|^2, beta = |m_q|^2, gamma = m_p . m_q (fp32), and unless
+// |gamma| <= 1e-7 sqrt(alpha beta) rotates columns p, q of M and of W by the
+// angle that makes them orthogonal (zeta = (beta - alpha) / (2 gamma),
+// t = sign(zeta) / (|zeta| + sqrt(1 + zeta^2)), c = 1 / sqrt(1 + t^2), s = c t,
+// in float64).  Sweeps end when one makes no rotation, or after OS_MAX_SWEEPS.
+// M and W are column-major, in shared memory when they fit, else in Mg / Wg.
+// Output: Wt [L][L], Wt[j][k] = W[k][j].
+constexpr int OS_THREADS = 512;
+constexpr int OS_MAX_SWEEPS = 30;
+__global__ void __launch_bounds__(OS_THREADS)
+k_onesided(const float* __restrict__ Mt, int L, float* __restrict__ Mg, float* __restrict__ Wg,
+           int in_smem, float* __restrict__ Wt) {
+  extern __shared__ float osm[];
+  __shared__ int s_rot;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nw = OS_THREADS / 32;
   const int Lp = L + (L & 1), half = Lp / 2;
-  double* A = a_in_smem ? Asm : Ag;
-  for (int q = tid; q < Lp * Lp; q += JB_THREADS) {
-    const int i = q / Lp, j = q % Lp;
-    A[q] = (i < L && j < L) ? S[(size_t)i * L + j] : 0.0;
-    V[q] = i == j ? 1.0 : 0.0;
-  }
+  float* M = in_smem ? osm : Mg;                       // [Lp][L]
+  float* W = in_smem ? osm + (size_t)Lp * L : Wg;      // [Lp][Lp]
+  for (int q = tid; q < Lp * L; q += OS_THREADS) M[q] = q < L * L ? Mt[q] : 0.f;
+  for (int q = tid; q < Lp * Lp; q += OS_THREADS) W[q] = (q / Lp == q % Lp) ? 1.f : 0.f;
   __syncthreads();
-  for (int sweep = 0; sweep < JB_MAX_SWEEPS; ++sweep) {
-    // convergence: off-diagonal and total squared mass
-    double off = 0.0, tot = 0.0;
-    for (int q = tid; q < Lp * Lp; q += JB_THREADS) {
-      const double a = A[q];
-      tot += a * a;
-      if (q / Lp != q % Lp) off += a * a;
-    }
-    for (int o = 16; o; o >>= 1) {
-      off += __shfl_xor_sync(0xffffffffu, off, o);
-      tot += __shfl_xor_sync(0xffffffffu, tot, o);
-    }
-    if (lane == 0) {
-      red[0][warp] = off;
-      red[1][warp] = tot;
-    }
+  for (int sweep = 0; sweep < OS_MAX_SWEEPS; ++sweep) {
+    if (tid == 0) s_rot = 0;
     __syncthreads();
-    if (tid == 0) {
-      double o2 = 0.0, t2 = 0.0;
-      for (int w = 0; w < JB_THREADS / 32; ++w) {
-        o2 += red[0][w];
-        t2 += red[1][w];
-      }
-      s_done = (t2 == 0.0 || o2 <= 1e-28 * t2) ? 1 : 0;
-    }
-    __syncthreads();
-    if (s_done) break;
     for (int round = 0; round < Lp - 1; ++round) {
-      if (tid < half) {
+      for (int P = warp; P < half; P += nw) {
         int p, q;
-        if (tid == 0) {
+        if (P == 0) {
           p = round;
           q = Lp - 1;
         } else {
-          p = (round + tid) % (Lp - 1);
-          q = (round - tid + (Lp - 1)) % (Lp - 1);
+          p = (round + P) % (Lp - 1);
+          q = (round - P + (Lp - 1)) % (Lp - 1);
         }
-        const double app = A[(size_t)p * Lp + p], aqq = A[(size_t)q * Lp + q];
-        const double apq = A[(size_t)p * Lp + q];
-        double c = 1.0, s = 0.0;
-        if (apq != 0.0 && fabs(apq) > 1e-300) {
-          const double tau = (aqq - app) / (2.0 * apq);
-          const double t = (tau >= 0.0 ? 1.0 : -1.0) / (fabs(tau) + sqrt(1.0 + tau * tau));
-          c = 1.0 / sqrt(1.0 + t * t);
-          s = t * c;
+        float* mp = M + (size_t)p * L;
+        float* mq = M + (size_t)q * L;
+        float a = 0.f, b = 0.f, g = 0.f;
+        for (int i = lane; i < L; i += 32) {
+          const float x = mp[i], y = mq[i];
+          a = fmaf(x, x, a);
+          b = fmaf(y, y, b);
+          g = fmaf(x, y, g);
         }
-        pc[tid] = c;
-        ps[tid] = s;
-        pp[tid] = p;
-        pq[tid] = q;
-      }
-      __syncthreads();
-      // A <- J^T A J by 2 x 2 blocks (pair P rows, pair P2 columns)
-      for (int w = tid; w < half * half; w += JB_THREADS) {
-        const int P = w / half, P2 = w % half;
-        const int p = pp[P], q = pq[P], p2 = pp[P2], q2 = pq[P2];
-        const double c = pc[P], s = ps[P], c2 = pc[P2], s2 = ps[P2];
-        const double b00 = A[(size_t)p * Lp + p2], b01 = A[(size_t)p * Lp + q2];
-        const double b10 = A[(size_t)q * Lp + p2], b11 = A[(size_t)q * Lp + q2];
-        // rows: J^T B
-        const double r00 = c * b00 - s * b10, r01 = c * b01 - s * b11;
-        const double r10 = s * b00 + c * b10, r11 = s * b01 + c * b11;
-        // columns: (J^T B) J2
-        double n00 = c2 * r00 - s2 * r01, n01 = s2 * r00 + c2 * r01;
-        double n10 = c2 * r10 - s2 * r11, n11 = s2 * r10 + c2 * r11;
-        if (P == P2) n01 = n10 = 0.0;  // the entry this rotation annihilates
-        A[(size_t)p * Lp + p2] = n00;
-        A[(size_t)p * Lp + q2] = n01;
-        A[(size_t)q * Lp + p2] = n10;
-        A[(size_t)q * Lp + q2] = n11;
-      }
-      // V <- V J
-      for (int w = tid; w < Lp * half; w += JB_THREADS) {
-        const int i = w / half, P = w % half;
-        const int p = pp[P], q = pq[P];
-        const double c = pc[P], s = ps[P];
-        const double vp = V[(size_t)i * Lp + p], vq = V[(size_t)i * Lp + q];
-        V[(size_t)i * Lp + p] = c * vp - s * vq;
-        V[(size_t)i * Lp + q] = s * vp + c * vq;
+        for (int o = 16; o; o >>= 1) {
+          a += __shfl_xor_sync(0xffffffffu, a, o);
+          b += __shfl_xor_sync(0xffffffffu, b, o);
+          g += __shfl_xor_sync(0xffffffffu, g, o);
+        }
+        if (g == 0.f || fabsf(g) <= 1e-7f * sqrtf(a * b)) continue;  // warp-uniform
+        const double z = ((double)b - (double)a) / (2.0 * (double)g);
+        const double t = (z >= 0.0 ? 1.0 : -1.0) / (fabs(z) + sqrt(1.0 + z * z));
+        const double cd = 1.0 / sqrt(1.0 + t * t);
+        const float c = (float)cd, s = (float)(t * cd);
+        for (int i = lane; i < L; i += 32) {
+          const float x = mp[i], y = mq[i];
+          mp[i] = c * x - s * y;
+          mq[i] = s * x + c * y;
+        }
+        float* wp = W + (size_t)p * Lp;
+        float* wq = W + (size_t)q * Lp;
+        for (int k = lane; k < Lp; k += 32) {
+          const float x = wp[k], y = wq[k];
+          wp[k] = c * x - s * y;
+          wq[k] = s * x + c * y;
+        }
+        if (lane == 0) s_rot = 1;
       }
       __syncthreads();
     }
+    if (s_rot == 0) break;  // read after the round's barrier; every thread sees the same value
+    __syncthreads();        // before thread 0 clears s_rot for the next sweep
   }
-  // rank of every real index by (eigenvalue descending, index ascending)
-  for (int i = tid; i < L; i += JB_THREADS) {
-    const double li = A[(size_t)i * Lp + i];
+  for (int q = tid; q < L * L; q += OS_THREADS) {
+    const int j = q / L, k = q % L;
+    Wt[q] = W[(size_t)j * Lp + k];
+  }
+}
+
+// CTA j: v = M w_j in float64, sigma_j = |v| / |w_j| (the Rayleigh quotient of
+// the converged rotation, second-order accurate in the rotation's error);
+// MWn[j] = v / |w_j|, Wn[j] = w_j / |w_j| (fp32, column j stored contiguously).
+__global__ void __launch_bounds__(256)
+k_ritz(const float* __restrict__ Mt, const float* __restrict__ Wt, int L, float* __restrict__ MWn,
+       float* __restrict__ Wn, double* __restrict__ sig64) {
+  __shared__ float w[256];
+  __shared__ double red[2][8];
+  const int j = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  for (int k = tid; k < L; k += 256) w[k] = Wt[(size_t)j * L + k];
+  __syncthreads();
+  double v = 0.0, ww = 0.0;
+  if (tid < L) {
+    for (int k = 0; k < L; ++k) v = fma((double)Mt[(size_t)k * L + tid], (double)w[k], v);
+    ww = (double)w[tid] * (double)w[tid];
+  }
+  double v2 = v * v, w2 = ww;
+  for (int o = 16; o; o >>= 1) {
+    v2 += __shfl_xor_sync(0xffffffffu, v2, o);
+    w2 += __shfl_xor_sync(0xffffffffu, w2, o);
+  }
+  if (lane == 0) {
+    red[0][warp] = v2;
+    red[1][warp] = w2;
+  }
+  __syncthreads();
+  double tv = 0.0, tw = 0.0;
+  for (int q = 0; q < 8; ++q) {
+    tv += red[0][q];
+    tw += red[1][q];
+  }
+  const double nw_ = sqrt(tw);
+  if (tid < L) {
+    MWn[(size_t)j * L + tid] = nw_ > 0.0 ? (float)(v / nw_) : 0.f;
+    Wn[(size_t)j * L + tid] = nw_ > 0.0 ? (float)((double)w[tid] / nw_) : 0.f;
+  }
+  if (tid == 0) sig64[j] = nw_ > 0.0 ? sqrt(tv) / nw_ : 0.0;
+}
+
+// One CTA: the r largest sigma (ties: lower index first) and the fp32
+// matrices Wu [L][r] = MWn[i_c] / sqrt(sigma_c), Wv [L][r] = Wn[i_c] sqrt(sigma_c)
+// (zero for sigma_c <= 1e-6 sigma_0), so that Q Wu = U_r S_r^(1/2) and
+// Z2 Wv = V_r S_r^(1/2) (Eq. factors); sig [r] fp32.
+__global__ void __launch_bounds__(256)
+k_finish(const double* __restrict__ sig64, const float* __restrict__ MWn,
+         const float* __restrict__ Wn, int L, int r, float* __restrict__ Wu,
+         float* __restrict__ Wv, float* __restrict__ sig) {
+  __shared__ int order[256];
+  const int tid = threadIdx.x;
+  for (int i = tid; i < L; i += 256) {
+    const double si = sig64[i];
     int rk = 0;
     for (int j = 0; j < L; ++j) {
-      const double lj = A[(size_t)j * Lp + j];
-      rk += (lj > li || (lj == li && j < i)) ? 1 : 0;
+      const double sj = sig64[j];
+      rk += (sj > si || (sj == si && j < i)) ? 1 : 0;
     }
     order[rk] = i;
   }
   __syncthreads();
-  const double sig0 = sqrt(fmax(A[(size_t)order[0] * Lp + order[0]], 0.0));
-  for (int q = tid; q < L * r; q += JB_THREADS) {
+  const double s0 = sig64[order[0]];
+  for (int q = tid; q < L * r; q += 256) {
     const int k = q / r, c = q % r;
     const int i = order[c];
-    const double sg = sqrt(fmax(A[(size_t)i * Lp + i], 0.0));
-    const double rs = sqrt(sg);
-    const double v = V[(size_t)k * Lp + i];
-    Wu[q] = (float)(v * rs);
-    Wv[q] = (sg > 1e-6 * sig0 && sg > 0.0) ? (float)(v / rs) : 0.f;
+    const double sg = sig64[i];
+    const bool keep = sg > 1e-6 * s0 && sg > 0.0;
+    const float rs = (float)sqrt(sg);
+    Wu[q] = keep ? MWn[(size_t)i * L + k] / rs : 0.f;
+    Wv[q] = keep ? Wn[(size_t)i * L + k] * rs : 0.f;
     if (k == 0) sig[c] = (float)sg;
   }
 }
@@ -408,7 +439,8 @@ __global__ void k_sign(float* __restrict__ U, float* __restrict__ V, int rows, i
   }
 }
 
-bool g_jb_cap[64] = {};
+bool g_ch_cap[64] = {};
+bool g_os_cap[64] = {};
 
 }  // namespace
 }  // namespace lx
@@ -416,12 +448,13 @@ bool g_jb_cap[64] = {};
 namespace lx {
 namespace {
 constexpr int CP_MAX_L = 256;
+constexpr size_t CP_SMEM_CAP = 200 * 1024;
 
 size_t al256(size_t v) { return (v + 255) / 256 * 256; }
 
 struct CompressWs {
-  float *y0, *y1, *z0, *z1, *T, *Wu, *Wv;
-  double *G, *Lw, *Xw, *A, *V;
+  float *y0, *y1, *z0, *z1, *T, *Wu, *Wv, *L1, *L2, *Xg, *Mt, *Wt, *MWn, *Wn, *Mg, *Wg;
+  double *G, *sig64;
   size_t bytes;
 };
 
@@ -443,11 +476,17 @@ CompressWs carve(char* base, long rows, long cols, long l, long r) {
   w.T = (float*)take(4 * l * l);
   w.Wu = (float*)take(4 * l * r);
   w.Wv = (float*)take(4 * l * r);
+  w.L1 = (float*)take(4 * l * l);
+  w.L2 = (float*)take(4 * l * l);
+  w.Xg = (float*)take(4 * l * l);
+  w.Mt = (float*)take(4 * l * l);
+  w.Wt = (float*)take(4 * l * l);
+  w.MWn = (float*)take(4 * l * l);
+  w.Wn = (float*)take(4 * l * l);
+  w.Mg = (float*)take(4 * Lp * l);
+  w.Wg = (float*)take(4 * Lp * Lp);
   w.G = (double*)take(8 * l * l);
-  w.Lw = (double*)take(8 * l * l);
-  w.Xw = (double*)take(8 * l * l);
-  w.A = (double*)take(8 * Lp * Lp);
-  w.V = (double*)take(8 * Lp * Lp);
+  w.sig64 = (double*)take(8 * l);
   w.bytes = off;
   return w;
 }
@@ -477,13 +516,17 @@ lx_status run_compress(int rows, int cols, const TW* Wd, const TW* Wm, const flo
     const dim3 grid((l + GR_T - 1) / GR_T, (l + GR_T - 1) / GR_T);
     k_gram<<<grid, GR_T * GR_T, 0, s>>>(X, n, l, w.G);
   };
-  // CholeskyQR twice: X [n][l] -> orthonormal columns, result in X (tmp scratch)
+  const size_t ch_smem = sizeof(float) * (size_t)l * (l + 1) / 2;
+  LX_CUDA(smem_cap_once((const void*)k_chol32, (int)CP_SMEM_CAP, dev, g_ch_cap));
+  // CholeskyQR twice (the first pass shifted by 1e-6 of the largest Gram
+  // diagonal, so rank-deficient bases stay factorable); X [n][l] ends
+  // orthonormal, tmp is scratch; the two factors stay in L1, L2.
   auto orth2 = [&](float* X, float* tmp, int n) {
     gram(X, n);
-    k_chol_inv<<<1, CH_THREADS, 0, s>>>(w.G, l, w.Lw, w.Xw, w.T);
+    k_chol32<<<1, CH_THREADS, ch_smem, s>>>(w.G, l, 1e-6f, w.L1, w.Xg, w.T);
     gemm(A_F32, X, w.T, tmp, n, l, l);
     gram(tmp, n);
-    k_chol_inv<<<1, CH_THREADS, 0, s>>>(w.G, l, w.Lw, w.Xw, w.T);
+    k_chol32<<<1, CH_THREADS, ch_smem, s>>>(w.G, l, 0.f, w.L2, w.Xg, w.T);
     gemm(A_F32, tmp, w.T, X, n, l, l);
   };
   gemm(A_RES, nullptr, omega, w.y0, rows, l, cols);  // Y = R Omega
@@ -494,15 +537,19 @@ lx_status run_compress(int rows, int cols, const TW* Wd, const TW* Wm, const flo
     gemm(A_RES, nullptr, w.z0, w.y0, rows, l, cols);    // R Z
     orth2(w.y0, w.y1, rows);
   }
-  gemm(A_RES_T, nullptr, w.y0, w.z0, cols, l, rows);    // Z = R^T Q = Bs^T
-  gram(w.z0, cols);                                     // Bs Bs^T
+  // Z = R^T Q = Bs^T = Z2 (L1 L2)^T with Z2 orthonormal, so Bs = M Z2^T for
+  // M = L1 L2, and the SVD of Bs follows from the small SVD of M.
+  gemm(A_RES_T, nullptr, w.y0, w.z0, cols, l, rows);
+  orth2(w.z0, w.z1, cols);
+  k_trmm<<<l, 256, 0, s>>>(w.L1, w.L2, l, w.Mt);
   const int Lp = l + (l & 1);
-  const size_t a_bytes = (size_t)Lp * Lp * 8;
-  const bool in_smem = a_bytes <= 200 * 1024;
-  if (in_smem)
-    LX_CUDA(smem_cap_once((const void*)k_jacobi, 200 * 1024, dev, g_jb_cap));
-  k_jacobi<<<1, JB_THREADS, in_smem ? a_bytes : 0, s>>>(w.G, l, r, w.A, w.V, in_smem ? 1 : 0,
-                                                        w.Wu, w.Wv, sigma);
+  const size_t os_bytes = sizeof(float) * ((size_t)Lp * l + (size_t)Lp * Lp);
+  const bool os_smem = os_bytes <= CP_SMEM_CAP;
+  if (os_smem) LX_CUDA(smem_cap_once((const void*)k_onesided, (int)CP_SMEM_CAP, dev, g_os_cap));
+  k_onesided<<<1, OS_THREADS, os_smem ? os_bytes : 0, s>>>(w.Mt, l, w.Mg, w.Wg, os_smem ? 1 : 0,
+                                                          w.Wt);
+  k_ritz<<<l, 256, 0, s>>>(w.Mt, w.Wt, l, w.MWn, w.Wn, w.sig64);
+  k_finish<<<1, 256, 0, s>>>(w.sig64, w.MWn, w.Wn, l, r, w.Wu, w.Wv, sigma);
   gemm(A_F32, w.y0, w.Wu, U, rows, r, l);   // U_r S^(1/2)
   gemm(A_F32, w.z0, w.Wv, V, cols, r, l);   // V_r S^(1/2)
   k_sign<<<r, 256, 0, s>>>(U, V, rows, cols, r);
