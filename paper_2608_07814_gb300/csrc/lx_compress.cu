@@ -163,16 +163,18 @@ k_gram(const float* __restrict__ X, int n, int L, double* __restrict__ G) {
 // One CTA (L <= 256).  Cholesky of G + s I in fp32 (G float64, rounded once;
 // s = shift_rel * max diag(G)) in a packed lower triangle in shared memory
 // (L (L + 1) / 2 floats), pivots floored at 1e-30; then X = L^-1 by forward
-// substitution (thread c owns column c, kept in the global scratch Xg so that
-// a warp reads one contiguous piece of a row per step) and T = X^T, so that
-// Y T = Y L^-T has orthonormal columns when Y^T Y = G (CholeskyQR).  The factor
-// itself is written to Lout [L][L] (zero above the diagonal).  A zero Gram
-// gives Lout = T = 0.
+// substitution (thread c owns column c; X packed like L, in shared memory
+// when x_in_smem, else in the global scratch Xg, so that a warp reads one
+// contiguous piece of a row per step) and T = X^T, so that Y T = Y L^-T has
+// orthonormal columns when Y^T Y = G (CholeskyQR).  The factor itself is
+// written to Lout [L][L] (zero above the diagonal).  A zero Gram gives
+// Lout = T = 0.
 constexpr int CH_THREADS = 256;
 __global__ void __launch_bounds__(CH_THREADS)
 k_chol32(const double* __restrict__ G, int L, float shift_rel, float* __restrict__ Lout,
-         float* __restrict__ Xg, float* __restrict__ T) {
+         float* __restrict__ Xg, int x_in_smem, float* __restrict__ T) {
   extern __shared__ float Ls[];
+  float* Xp = x_in_smem ? Ls + L * (L + 1) / 2 : Xg;  // packed lower X
   __shared__ double s_md;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nw = CH_THREADS / 32;
   if (tid == 0) {
@@ -213,18 +215,17 @@ k_chol32(const double* __restrict__ G, int L, float shift_rel, float* __restrict
   }
   if (tid < L) {
     const int c = tid;
-    for (int i = 0; i < L; ++i) {
+    for (int i = c; i < L; ++i) {
       const float* Li = Ls + i * (i + 1) / 2;
       float acc = 0.f;
-      for (int k = 0; k < i; ++k)
-        if (k >= c) acc = fmaf(Li[k], Xg[(size_t)k * L + c], acc);
-      Xg[(size_t)i * L + c] = i < c ? 0.f : (i == c ? 1.f / Li[i] : -acc / Li[i]);
+      for (int k = c; k < i; ++k) acc = fmaf(Li[k], Xp[k * (k + 1) / 2 + c], acc);
+      Xp[i * (i + 1) / 2 + c] = i == c ? 1.f / Li[i] : -acc / Li[i];
     }
   }
   __syncthreads();
   for (int q = tid; q < L * L; q += CH_THREADS) {
-    const int k = q / L, n = q % L;  // T[k][n] = X[n][k]
-    T[q] = Xg[(size_t)n * L + k];
+    const int k = q / L, n = q % L;  // T[k][n] = X[n][k], zero below the diagonal
+    T[q] = k <= n ? Xp[n * (n + 1) / 2 + k] : 0.f;
   }
 }
 
@@ -244,13 +245,13 @@ __global__ void k_trmm(const float* __restrict__ L1, const float* __restrict__ L
 // orthogonal.  Lp = L rounded up to even (a zero padding column never rotates);
 // each round pairs the columns by the circle method, a warp takes a pair:
 // alpha = |m_p|^2, beta = |m_q|^2, gamma = m_p . m_q (fp32), and unless
-// |gamma| <= 1e-7 sqrt(alpha beta) rotates columns p, q of M and of W by the
+// |gamma| <= 1e-6 sqrt(alpha beta) (a little above the rounding of an fp32 dot
+// product, so that sweeps terminate) rotates columns p, q of M and of W by the
 // angle that makes them orthogonal (zeta = (beta - alpha) / (2 gamma),
-// t = sign(zeta) / (|zeta| + sqrt(1 + zeta^2)), c = 1 / sqrt(1 + t^2), s = c t,
-// in float64).  Sweeps end when one makes no rotation, or after OS_MAX_SWEEPS.
+// t = sign(zeta) / (|zeta| + sqrt(1 + zeta^2)), c = 1 / sqrt(1 + t^2), s = c t).  Sweeps end when one makes no rotation, or after OS_MAX_SWEEPS.
 // M and W are column-major, in shared memory when they fit, else in Mg / Wg.
 // Output: Wt [L][L], Wt[j][k] = W[k][j].
-constexpr int OS_THREADS = 512;
+constexpr int OS_THREADS = 1024;
 constexpr int OS_MAX_SWEEPS = 30;
 __global__ void __launch_bounds__(OS_THREADS)
 k_onesided(const float* __restrict__ Mt, int L, float* __restrict__ Mg, float* __restrict__ Wg,
@@ -291,11 +292,11 @@ k_onesided(const float* __restrict__ Mt, int L, float* __restrict__ Mg, float* _
           b += __shfl_xor_sync(0xffffffffu, b, o);
           g += __shfl_xor_sync(0xffffffffu, g, o);
         }
-        if (g == 0.f || fabsf(g) <= 1e-7f * sqrtf(a * b)) continue;  // warp-uniform
-        const double z = ((double)b - (double)a) / (2.0 * (double)g);
-        const double t = (z >= 0.0 ? 1.0 : -1.0) / (fabs(z) + sqrt(1.0 + z * z));
-        const double cd = 1.0 / sqrt(1.0 + t * t);
-        const float c = (float)cd, s = (float)(t * cd);
+        if (g == 0.f || fabsf(g) <= 1e-6f * sqrtf(a * b)) continue;  // warp-uniform
+        // (an overflowing zeta gives t = 0: no rotation, never a NaN)
+        const float z = (b - a) / (2.f * g);
+        const float t = (z >= 0.f ? 1.f : -1.f) / (fabsf(z) + sqrtf(1.f + z * z));
+        const float c = 1.f / sqrtf(1.f + t * t), s = t * c;
         for (int i = lane; i < L; i += 32) {
           const float x = mp[i], y = mq[i];
           mp[i] = c * x - s * y;
@@ -516,17 +517,19 @@ lx_status run_compress(int rows, int cols, const TW* Wd, const TW* Wm, const flo
     const dim3 grid((l + GR_T - 1) / GR_T, (l + GR_T - 1) / GR_T);
     k_gram<<<grid, GR_T * GR_T, 0, s>>>(X, n, l, w.G);
   };
-  const size_t ch_smem = sizeof(float) * (size_t)l * (l + 1) / 2;
+  const size_t tri = sizeof(float) * (size_t)l * (l + 1) / 2;
+  const bool x_smem = 2 * tri <= CP_SMEM_CAP;  // L and X both in shared memory
+  const size_t ch_smem = x_smem ? 2 * tri : tri;
   LX_CUDA(smem_cap_once((const void*)k_chol32, (int)CP_SMEM_CAP, dev, g_ch_cap));
   // CholeskyQR twice (the first pass shifted by 1e-6 of the largest Gram
   // diagonal, so rank-deficient bases stay factorable); X [n][l] ends
   // orthonormal, tmp is scratch; the two factors stay in L1, L2.
   auto orth2 = [&](float* X, float* tmp, int n) {
     gram(X, n);
-    k_chol32<<<1, CH_THREADS, ch_smem, s>>>(w.G, l, 1e-6f, w.L1, w.Xg, w.T);
+    k_chol32<<<1, CH_THREADS, ch_smem, s>>>(w.G, l, 1e-6f, w.L1, w.Xg, x_smem ? 1 : 0, w.T);
     gemm(A_F32, X, w.T, tmp, n, l, l);
     gram(tmp, n);
-    k_chol32<<<1, CH_THREADS, ch_smem, s>>>(w.G, l, 0.f, w.L2, w.Xg, w.T);
+    k_chol32<<<1, CH_THREADS, ch_smem, s>>>(w.G, l, 0.f, w.L2, w.Xg, x_smem ? 1 : 0, w.T);
     gemm(A_F32, tmp, w.T, X, n, l, l);
   };
   gemm(A_RES, nullptr, omega, w.y0, rows, l, cols);  // Y = R Omega
