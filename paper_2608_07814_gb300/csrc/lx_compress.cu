@@ -169,7 +169,7 @@ k_gram(const float* __restrict__ X, int n, int L, double* __restrict__ G) {
 // orthonormal columns when Y^T Y = G (CholeskyQR).  The factor itself is
 // written to Lout [L][L] (zero above the diagonal).  A zero Gram gives
 // Lout = T = 0.
-constexpr int CH_THREADS = 256;
+constexpr int CH_THREADS = 1024;
 __global__ void __launch_bounds__(CH_THREADS)
 k_chol32(const double* __restrict__ G, int L, float shift_rel, float* __restrict__ Lout,
          float* __restrict__ Xg, int x_in_smem, float* __restrict__ T) {

@@ -335,18 +335,22 @@ def compress_workspace_bytes(rows: int, cols: int, l: int, r: int) -> int:
 
 def compress_factor(w_dom: torch.Tensor, w_mem: torch.Tensor, omega: torch.Tensor, r: int,
                     power_iters: int = 2, workspace: Optional[torch.Tensor] = None,
-                    stream=None):
+                    stream=None, out=None):
     """(U [rows, r], V [cols, r], s [r]) fp32 with U V^T ~ w_mem - w_dom; omega
-    is the fp32 [cols, l] Gaussian test matrix."""
+    is the fp32 [cols, l] Gaussian test matrix.  ``out`` = preallocated
+    (U, V, s); independent projections may run concurrently on their own
+    streams, each with its own workspace."""
     rows, cols = w_dom.shape
     l = omega.shape[1]
     need = compress_workspace_bytes(rows, cols, l, r)
     if workspace is None:
         workspace = torch.empty(need, dtype=torch.uint8, device=w_dom.device)
     dev = w_dom.device
-    U = torch.empty((rows, r), dtype=torch.float32, device=dev)
-    V = torch.empty((cols, r), dtype=torch.float32, device=dev)
-    s = torch.empty(r, dtype=torch.float32, device=dev)
+    if out is None:
+        out = (torch.empty((rows, r), dtype=torch.float32, device=dev),
+               torch.empty((cols, r), dtype=torch.float32, device=dev),
+               torch.empty(r, dtype=torch.float32, device=dev))
+    U, V, s = out
     _check(lib().lx_compress_factor(_dtype_code(w_dom), rows, cols, _ptr(w_dom), _ptr(w_mem),
                                     _ptr(omega), l, r, power_iters, _ptr(U), _ptr(V), _ptr(s),
                                     _ptr(workspace), workspace.numel(), _stream(stream)))
