@@ -592,7 +592,7 @@ def run_offline(args, rank, world, local_rank):
         ms_seq = _event_ms(step, max(3, args.steps // 4), args.warmup)
         # a layer's members are independent: n_conc members (3 projections
         # each) in flight on their own streams, each with its own workspace
-        n_conc = 4
+        n_conc = 8
         streams = [torch.cuda.Stream(device=dev) for _ in range(3 * n_conc)]
         wss = [torch.empty(wsz, dtype=torch.uint8, device=dev) for _ in streams]
         outs = [(torch.empty((a, r), dtype=torch.float32, device=dev),

@@ -221,11 +221,12 @@ extern "C" lx_status lx_permute_neurons(int32_t dtype, int32_t d_model, int32_t 
   return LX_OK;
 }
 
-// Exact linear assignment on the host: rows are added one at a time, each by a
-// shortest augmenting path (Dijkstra over the columns on reduced costs
-// c[i][j] - u[i] - v[j] >= 0), after which the dual potentials u, v are updated
-// so that every reduced cost stays non-negative and those on the matching are
-// zero -- the augmentation scheme of Jonker and Volgenant.  O(n^3), float64.
+// Exact linear assignment on the host: Jonker and Volgenant's column reduction
+// assigns every column's cheapest row where that row is free; each remaining
+// row is then added by a shortest augmenting path (Dijkstra over the columns
+// on reduced costs c[i][j] - u[i] - v[j] >= 0), after which the dual
+// potentials u, v are updated so that every reduced cost stays non-negative
+// and those on the matching are zero -- JV's augmentation.  O(n^3), float64.
 extern "C" lx_status lx_lap_solve(const float* cost, int32_t n, int32_t* assign, double* total) {
   using namespace lx;
   if (n < 1 || n > 65536) return fail(LX_ERR_ARG, "n must be in 1..65536");
@@ -238,8 +239,29 @@ extern "C" lx_status lx_lap_solve(const float* cost, int32_t n, int32_t* assign,
   // column 0 is a virtual column that holds the row being added
   std::vector<double> u(n + 1, 0.0), v(n + 1, 0.0), dist(n + 1);
   std::vector<int> row_of(n + 1, 0), prev(n + 1, 0);  // row_of[j]: row (1-based) on column j
-  std::vector<char> done(n + 1);
+  std::vector<char> done(n + 1), row_used(n + 1, 0);
+  // JV column reduction: v_j = min_i c_ij, and column j takes its minimising
+  // row when that row is still free.  Reduced costs c - u - v stay >= 0 and
+  // every assigned pair is tight, so the augmentation below starts from a
+  // partial optimum.
+  for (int j = 1; j <= n; ++j) {
+    int best_i = 1;
+    double best = (double)cost[j - 1];
+    for (int i = 2; i <= n; ++i) {
+      const double c = (double)cost[(size_t)(i - 1) * n + (j - 1)];
+      if (c < best) {
+        best = c;
+        best_i = i;
+      }
+    }
+    v[j] = best;
+    if (!row_used[best_i]) {
+      row_used[best_i] = 1;
+      row_of[j] = best_i;
+    }
+  }
   for (int r = 1; r <= n; ++r) {
+    if (row_used[r]) continue;
     row_of[0] = r;
     int col = 0;
     std::fill(dist.begin(), dist.end(), kInf);
