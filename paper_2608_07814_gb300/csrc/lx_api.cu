@@ -149,9 +149,9 @@ static lx_status ensure_workspace(lx_layer* L, int T, int k, cudaStream_t s) {
       {(void**)&w.z, sizeof(float) * Rmax * L->I},
       {(void**)&w.Q, sizeof(float) * Rmax * rmax},
       {(void**)&w.ypart, sizeof(float) * Rmax * L->H},
-      {(void**)&w.Pb, 2 * Rmax * 2 * rmax},
-      {(void**)&w.zb, 2 * Rmax * L->I},
-      {(void**)&w.Qb, 2 * Rmax * rmax},
+      {(void**)&w.Pb, (size_t)2 * Rmax * 2 * rmax},
+      {(void**)&w.zb, (size_t)2 * Rmax * L->I},
+      {(void**)&w.Qb, (size_t)2 * Rmax * rmax},
       {(void**)&w.act, sizeof(int) * STREAM_DEP_TB * std::max(1, L->n_anchor + L->n_corr)},
       {(void**)&w.act_n, sizeof(int) * 2},
       {(void**)&w.sctr, sizeof(int) * sctr_ints(L)},
