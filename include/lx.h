@@ -319,6 +319,18 @@ LX_API lx_status lx_align_cost(int32_t dtype, int32_t d_model, int32_t d_ff,
 LX_API lx_status lx_lap_solve(const float* cost, int32_t n, int32_t* assign, double* total);
 
 /*
+ * lx_lap_solve_batch (host): lx_lap_solve for `count` independent problems
+ * (e.g. every member of a layer), spread over `threads` host threads
+ * (<= 0: the hardware concurrency).
+ *   costs:  HOST [count][n][n] fp32;  assign: HOST [count][n] int32 out;
+ *   totals: HOST [count] double out, or NULL.
+ * Every cost is checked before any problem is solved.  Errors: LX_ERR_ARG
+ * (n outside 1..65536, count < 0, NULL, a NaN or infinite cost).
+ */
+LX_API lx_status lx_lap_solve_batch(const float* costs, int32_t n, int32_t count, int32_t* assign,
+                                    double* totals, int32_t threads);
+
+/*
  * lx_permute_neurons: the aligned member, neuron i <- neuron perm[i]:
  *   gate_out[i][:] = gate[perm[i]][:], up_out likewise,
  *   down_out[:][i] = down[:][perm[i]]   (bit-exact copies).

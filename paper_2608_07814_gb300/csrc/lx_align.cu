@@ -14,7 +14,9 @@
 // lx_lap_solve: the exact assignment on the host (shortest augmenting paths
 // with dual potentials, the augmentation scheme of Jonker and Volgenant).
 #include <algorithm>
+#include <atomic>
 #include <limits>
+#include <thread>
 #include <vector>
 
 #include "lx_internal.cuh"
@@ -227,14 +229,17 @@ extern "C" lx_status lx_permute_neurons(int32_t dtype, int32_t d_model, int32_t 
 // on reduced costs c[i][j] - u[i] - v[j] >= 0), after which the dual
 // potentials u, v are updated so that every reduced cost stays non-negative
 // and those on the matching are zero -- JV's augmentation.  O(n^3), float64.
-extern "C" lx_status lx_lap_solve(const float* cost, int32_t n, int32_t* assign, double* total) {
-  using namespace lx;
-  if (n < 1 || n > 65536) return fail(LX_ERR_ARG, "n must be in 1..65536");
-  if (!cost || !assign) return fail(LX_ERR_ARG, "cost or assign is NULL");
-  for (long q = 0; q < (long)n * n; ++q)
+namespace {
+bool costs_finite(const float* cost, long count) {
+  for (long q = 0; q < count; ++q)
     if (!(cost[q] == cost[q]) || cost[q] == std::numeric_limits<float>::infinity() ||
         cost[q] == -std::numeric_limits<float>::infinity())
-      return fail(LX_ERR_ARG, "cost holds a NaN or an infinity");
+      return false;
+  return true;
+}
+
+// The solver proper (arguments already checked); thread-safe.
+void lap_solve_one(const float* cost, int32_t n, int32_t* assign, double* total) {
   const double kInf = std::numeric_limits<double>::infinity();
   // column 0 is a virtual column that holds the row being added
   std::vector<double> u(n + 1, 0.0), v(n + 1, 0.0), dist(n + 1);
@@ -311,5 +316,38 @@ extern "C" lx_status lx_lap_solve(const float* cost, int32_t n, int32_t* assign,
   }
   for (int i = 0; i < n; ++i) sum += (double)cost[(size_t)i * n + assign[i]];
   if (total) *total = sum;
+}
+}  // namespace
+
+extern "C" lx_status lx_lap_solve(const float* cost, int32_t n, int32_t* assign, double* total) {
+  using namespace lx;
+  if (n < 1 || n > 65536) return fail(LX_ERR_ARG, "n must be in 1..65536");
+  if (!cost || !assign) return fail(LX_ERR_ARG, "cost or assign is NULL");
+  if (!costs_finite(cost, (long)n * n)) return fail(LX_ERR_ARG, "cost holds a NaN or an infinity");
+  lap_solve_one(cost, n, assign, total);
+  return LX_OK;
+}
+
+extern "C" lx_status lx_lap_solve_batch(const float* costs, int32_t n, int32_t count,
+                                        int32_t* assign, double* totals, int32_t threads) {
+  using namespace lx;
+  if (n < 1 || n > 65536) return fail(LX_ERR_ARG, "n must be in 1..65536");
+  if (count < 0) return fail(LX_ERR_ARG, "count < 0");
+  if (count == 0) return LX_OK;
+  if (!costs || !assign) return fail(LX_ERR_ARG, "costs or assign is NULL");
+  const size_t nn = (size_t)n * n;
+  if (!costs_finite(costs, (long)(nn * count)))
+    return fail(LX_ERR_ARG, "a cost holds a NaN or an infinity");
+  int nt = threads > 0 ? threads : (int)std::thread::hardware_concurrency();
+  nt = std::max(1, std::min(nt, (int)count));
+  std::atomic<int> next(0);
+  auto work = [&]() {
+    for (int b = next.fetch_add(1); b < count; b = next.fetch_add(1))
+      lap_solve_one(costs + (size_t)b * nn, n, assign + (size_t)b * n, totals ? totals + b : nullptr);
+  };
+  std::vector<std::thread> pool;
+  for (int t = 1; t < nt; ++t) pool.emplace_back(work);
+  work();
+  for (auto& th : pool) th.join();
   return LX_OK;
 }

@@ -29,7 +29,7 @@ EXPORTS = [
     "lx_load_compressed_layer", "lx_free_layer", "lx_reserve", "lx_route", "lx_bucket",
     "lx_moe_forward", "lx_get_buckets", "lx_layer_info", "lx_set_path", "lx_set_profiling",
     "lx_read_profile", "lx_last_error", "lx_bucket_noalloc", "lx_coact_accumulate",
-    "lx_coact_npmi", "lx_align_cost", "lx_lap_solve", "lx_permute_neurons",
+    "lx_coact_npmi", "lx_align_cost", "lx_lap_solve", "lx_lap_solve_batch", "lx_permute_neurons",
     "lx_compress_workspace", "lx_compress_factor",
 ]
 LX_NOALLOC_SCRATCH_BYTES = 16 << 20
@@ -92,6 +92,7 @@ def lib() -> ctypes.CDLL:
             "lx_coact_npmi": [vp, i32, ctypes.c_int64, vp, vp],
             "lx_align_cost": [i32, i32, i32, vp, vp, vp, vp, vp, vp, vp, vp],
             "lx_lap_solve": [vp, i32, vp, ctypes.POINTER(ctypes.c_double)],
+            "lx_lap_solve_batch": [vp, i32, i32, vp, vp, i32],
             "lx_permute_neurons": [i32, i32, i32, vp, vp, vp, vp, vp, vp, vp, vp],
             "lx_compress_workspace": [i32, i32, i32, i32, ctypes.POINTER(ctypes.c_uint64)],
             "lx_compress_factor": [i32, i32, i32, vp, vp, vp, i32, i32, i32, vp, vp, vp, vp,
@@ -314,11 +315,26 @@ def lap_solve(cost: np.ndarray):
     return out, tot.value
 
 
+def lap_solve_batch(costs: np.ndarray, threads: int = 0):
+    """(assign int32 [count, n], totals float64 [count]) of independent host
+    costs [count, n, n], solved on `threads` host threads (0: all cores)."""
+    c = np.ascontiguousarray(costs, dtype=np.float32)
+    count, n = c.shape[0], c.shape[1]
+    out = np.empty((count, n), np.int32)
+    tot = np.empty(count, np.float64)
+    _check(lib().lx_lap_solve_batch(ctypes.c_void_p(c.ctypes.data), n, count,
+                                    ctypes.c_void_p(out.ctypes.data),
+                                    ctypes.c_void_p(tot.ctypes.data), threads))
+    return out, tot
+
+
 def permute_neurons(perm: torch.Tensor, gate: torch.Tensor, up: torch.Tensor,
-                    down: torch.Tensor, stream=None):
-    """(gate, up, down) of the member with neuron i taken from neuron perm[i]."""
+                    down: torch.Tensor, stream=None, out=None):
+    """(gate, up, down) of the member with neuron i taken from neuron perm[i]
+    (into ``out`` when given)."""
     I, H = gate.shape
-    outs = (torch.empty_like(gate), torch.empty_like(up), torch.empty_like(down))
+    outs = out if out is not None else (torch.empty_like(gate), torch.empty_like(up),
+                                        torch.empty_like(down))
     _check(lib().lx_permute_neurons(_dtype_code(gate), H, I, _ptr(perm), _ptr(gate), _ptr(up),
                                     _ptr(down), *[_ptr(t) for t in outs], _stream(stream)))
     return outs

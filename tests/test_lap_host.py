@@ -68,3 +68,23 @@ def test_negative_costs_and_rejects():
     bad[1, 2] = np.inf
     with pytest.raises(lx.LxError):
         lx.lap_solve(bad)
+
+
+def test_batch_matches_single_solves_on_threads():
+    rng = np.random.default_rng(11)
+    n, count = 120, 9
+    costs = rng.random((count, n, n)).astype(np.float32)
+    costs[3] = np.round(costs[3] * 3)          # ties in one problem
+    P, tot = lx.lap_solve_batch(costs, threads=4)
+    for b in range(count):
+        Pb, tb = lx.lap_solve(costs[b])
+        assert abs(tot[b] - tb) <= 1e-9 * max(1.0, abs(tb))
+        assert sorted(P[b].tolist()) == list(range(n))
+        ref = align.assignment_cost(costs[b], align.assign(costs[b]))
+        assert abs(tot[b] - ref) <= 1e-9 * max(1.0, abs(ref))
+    bad = costs.copy()
+    bad[7, 1, 1] = np.nan
+    with pytest.raises(lx.LxError):
+        lx.lap_solve_batch(bad)
+    P0, t0 = lx.lap_solve_batch(costs[:0])
+    assert P0.shape == (0, n)
