@@ -10,6 +10,8 @@
 // three K segments (gate rows, up rows: K-major; down columns: MN-major) staged
 // through shared memory in 32-deep chunks; the tile's row norms are summed
 // from the same staged chunks, so every operand byte is read once per tile.
+// k_align_cost_mma: the same tile for bf16 experts on the tensor cores
+// (mma.sync, bf16 inputs, fp32 accumulation).
 // k_permute_rows / k_permute_cols: gathers (bit-exact copies).
 // lx_lap_solve: the exact assignment on the host (shortest augmenting paths
 // with dual potentials, the augmentation scheme of Jonker and Volgenant).
@@ -125,6 +127,174 @@ k_align_cost(const TW* __restrict__ dg, const TW* __restrict__ du, const TW* __r
   }
 }
 
+// Tensor-core form of the cost for bf16 experts: the same tile of C, with the
+// products a_i . b_j on mma.sync m16n8k16 (bf16 inputs, fp32 accumulation:
+// every product is exact, as on the CUDA-core path).  Per 64-deep K chunk the
+// 64 dominant rows (A) and 64 member rows (B) are staged K-major in shared
+// memory as 128-byte rows with the 128-byte XOR swizzle (unit u of row r at
+// unit u ^ (r & 7)); gate/up chunks are copied as 16-byte units, down chunks
+// (columns of [H][I]) are transposed in registers from 8 x 8 blocks.  Lane
+// (g, q) feeds the MMA its own 16-byte K unit 2q + c of both operands, a K
+// permutation shared by A and B (the sum over K is unchanged).  The next
+// chunk's global loads are issued before the current chunk's MMAs (register
+// double buffering).  Row norms are summed from the staged chunks.
+constexpr int AM_TILE = 64;
+constexpr int AM_THREADS = 256;
+constexpr int AM_ROWB = 128;  // bytes per staged row (64 bf16)
+
+__device__ __forceinline__ void am_mma(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2,
+                                       uint32_t a3, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 "
+      "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// this thread's part of chunk (seg, h0, kc) of A (rows i0..) and B (rows j0..)
+struct AmRegs {
+  uint4 v[8];
+};
+
+__device__ __forceinline__ void am_load(AmRegs& R, const __nv_bfloat16* dg, const __nv_bfloat16* du,
+                                        const __nv_bfloat16* dd, const __nv_bfloat16* mg,
+                                        const __nv_bfloat16* mu, const __nv_bfloat16* md, int seg,
+                                        int h0, int kc, int i0, int j0, int H, int I, int tid) {
+  const uint4 z = make_uint4(0u, 0u, 0u, 0u);
+  if (seg < 2) {
+    // 2 units of A and 2 of B per thread: index q = tid + 256 v, row q / 8, unit q % 8
+#pragma unroll
+    for (int v = 0; v < 4; ++v) {
+      const int qi = tid + AM_THREADS * (v & 1);
+      const int row = qi >> 3, u = qi & 7;
+      const bool isA = v < 2;
+      const int r0 = isA ? i0 : j0;
+      const __nv_bfloat16* W = isA ? (seg == 0 ? dg : du) : (seg == 0 ? mg : mu);
+      const bool ok = r0 + row < I && u * 8 < kc;
+      R.v[v] = ok ? *reinterpret_cast<const uint4*>(W + (size_t)(r0 + row) * H + h0 + u * 8) : z;
+    }
+  } else if (tid < 2 * AM_TILE) {
+    // one 8 x 8 block (8 K rows x 8 neurons) of the down matrix [H][I]
+    const bool isA = tid < AM_TILE;
+    const int b = tid & (AM_TILE - 1), hb = b >> 3, ib = b & 7;
+    const __nv_bfloat16* W = isA ? dd : md;
+    const int n0 = (isA ? i0 : j0) + ib * 8;
+#pragma unroll
+    for (int rr = 0; rr < 8; ++rr) {
+      const bool ok = hb * 8 + rr < kc && n0 < I;
+      R.v[rr] = ok ? *reinterpret_cast<const uint4*>(W + (size_t)(h0 + hb * 8 + rr) * I + n0) : z;
+    }
+  }
+}
+
+__device__ __forceinline__ void am_store(const AmRegs& R, unsigned char* As, unsigned char* Bs,
+                                         int seg, int tid) {
+  if (seg < 2) {
+#pragma unroll
+    for (int v = 0; v < 4; ++v) {
+      const int qi = tid + AM_THREADS * (v & 1);
+      const int row = qi >> 3, u = qi & 7;
+      unsigned char* S = v < 2 ? As : Bs;
+      *reinterpret_cast<uint4*>(S + row * AM_ROWB + ((u ^ (row & 7)) << 4)) = R.v[v];
+    }
+  } else if (tid < 2 * AM_TILE) {
+    const bool isA = tid < AM_TILE;
+    const int b = tid & (AM_TILE - 1), hb = b >> 3, ib = b & 7;
+    unsigned char* S = isA ? As : Bs;
+    const uint32_t* w = reinterpret_cast<const uint32_t*>(R.v);  // w[rr * 4 + word]
+#pragma unroll
+    for (int ii = 0; ii < 8; ++ii) {
+      // neuron ii: element ii of K rows rr = 0..7, packed two K values per word
+      const uint32_t sel = (ii & 1) ? 0x7632u : 0x5410u;
+      const int wd = ii >> 1;
+      uint4 o;
+      o.x = __byte_perm(w[0 * 4 + wd], w[1 * 4 + wd], sel);
+      o.y = __byte_perm(w[2 * 4 + wd], w[3 * 4 + wd], sel);
+      o.z = __byte_perm(w[4 * 4 + wd], w[5 * 4 + wd], sel);
+      o.w = __byte_perm(w[6 * 4 + wd], w[7 * 4 + wd], sel);
+      const int row = ib * 8 + ii;
+      *reinterpret_cast<uint4*>(S + row * AM_ROWB + ((hb ^ (row & 7)) << 4)) = o;
+    }
+  }
+}
+
+__global__ void __launch_bounds__(AM_THREADS)
+k_align_cost_mma(const __nv_bfloat16* __restrict__ dg, const __nv_bfloat16* __restrict__ du,
+                 const __nv_bfloat16* __restrict__ dd, const __nv_bfloat16* __restrict__ mg,
+                 const __nv_bfloat16* __restrict__ mu, const __nv_bfloat16* __restrict__ md,
+                 int H, int I, float* __restrict__ cost) {
+  __shared__ __align__(128) unsigned char sA[2][AM_TILE * AM_ROWB];
+  __shared__ __align__(128) unsigned char sB[2][AM_TILE * AM_ROWB];
+  __shared__ float s_norm[2][2 * AM_TILE];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int g = lane >> 2, q = lane & 3;
+  const int wm = warp & 3, wn = warp >> 2;  // 16 rows x 32 columns per warp
+  const int i0 = blockIdx.y * AM_TILE, j0 = blockIdx.x * AM_TILE;
+  const int nch = (H + 63) / 64, total = 3 * nch;
+  float acc[4][4] = {};
+  float nrm = 0.f;  // row (tid & 127) of A (< 64) or B, units 4 (tid >> 7) .. +3
+  AmRegs R;
+  am_load(R, dg, du, dd, mg, mu, md, 0, 0, min(64, H), i0, j0, H, I, tid);
+  am_store(R, sA[0], sB[0], 0, tid);
+  __syncthreads();
+  for (int t = 0; t < total; ++t) {
+    const int buf = t & 1;
+    if (t + 1 < total) {
+      const int seg = (t + 1) / nch, h0 = ((t + 1) % nch) * 64;
+      am_load(R, dg, du, dd, mg, mu, md, seg, h0, min(64, H - h0), i0, j0, H, I, tid);
+    }
+    const unsigned char* A = sA[buf];
+    const unsigned char* B = sB[buf];
+#pragma unroll
+    for (int c = 0; c < 2; ++c) {
+      const int unit = (((q << 1) | c) ^ g) << 4;
+      const int ra = 16 * wm + g;
+      const uint4 w0 = *reinterpret_cast<const uint4*>(A + ra * AM_ROWB + unit);
+      const uint4 w1 = *reinterpret_cast<const uint4*>(A + (ra + 8) * AM_ROWB + unit);
+#pragma unroll
+      for (int nj = 0; nj < 4; ++nj) {
+        const uint4 xv = *reinterpret_cast<const uint4*>(B + (32 * wn + 8 * nj + g) * AM_ROWB + unit);
+        am_mma(acc[nj], w0.x, w1.x, w0.y, w1.y, xv.x, xv.y);
+        am_mma(acc[nj], w0.z, w1.z, w0.w, w1.w, xv.z, xv.w);
+      }
+    }
+    {
+      const int r = tid & 127, half = tid >> 7;
+      const unsigned char* S = r < AM_TILE ? A : B;
+      const int row = r & (AM_TILE - 1);
+#pragma unroll
+      for (int uu = 0; uu < 4; ++uu) {
+        const int u = half * 4 + uu;
+        const uint4 v = *reinterpret_cast<const uint4*>(S + row * AM_ROWB + ((u ^ (row & 7)) << 4));
+        const __nv_bfloat162* h2 = reinterpret_cast<const __nv_bfloat162*>(&v);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float2 f = __bfloat1622float2(h2[e]);
+          nrm = fmaf(f.x, f.x, nrm);
+          nrm = fmaf(f.y, f.y, nrm);
+        }
+      }
+    }
+    if (t + 1 < total) am_store(R, sA[buf ^ 1], sB[buf ^ 1], (t + 1) / nch, tid);
+    __syncthreads();
+  }
+  s_norm[tid >> 7][tid & 127] = nrm;
+  __syncthreads();
+#pragma unroll
+  for (int nj = 0; nj < 4; ++nj)
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      const int rl = 16 * wm + g + (c >= 2 ? 8 : 0);
+      const int cl = 32 * wn + 8 * nj + 2 * q + (c & 1);
+      const int i = i0 + rl, j = j0 + cl;
+      if (i < I && j < I) {
+        const float na = s_norm[0][rl] + s_norm[1][rl];
+        const float nb = s_norm[0][AM_TILE + cl] + s_norm[1][AM_TILE + cl];
+        cost[(size_t)i * I + j] = na + nb - 2.f * acc[nj][c];
+      }
+    }
+}
+
 // dst row i = src row perm[i] of a [rows][cols] matrix (16-byte pieces; a row
 // whose perm entry is outside [0, rows) is written as zeros)
 __global__ void k_permute_rows(const uint4* __restrict__ src, uint4* __restrict__ dst,
@@ -176,9 +346,9 @@ extern "C" lx_status lx_align_cost(int32_t dtype, int32_t d_model, int32_t d_ff,
   cudaStream_t s = (cudaStream_t)stream;
   if (dtype == LX_BF16) {
     using B = __nv_bfloat16;
-    k_align_cost<B><<<grid, AC_THREADS, 0, s>>>((const B*)dom_gate, (const B*)dom_up,
-                                                (const B*)dom_down, (const B*)mem_gate,
-                                                (const B*)mem_up, (const B*)mem_down, H, I, cost);
+    k_align_cost_mma<<<grid, AM_THREADS, 0, s>>>((const B*)dom_gate, (const B*)dom_up,
+                                                 (const B*)dom_down, (const B*)mem_gate,
+                                                 (const B*)mem_up, (const B*)mem_down, H, I, cost);
   } else {
     k_align_cost<float><<<grid, AC_THREADS, 0, s>>>(
         (const float*)dom_gate, (const float*)dom_up, (const float*)dom_down,
