@@ -136,12 +136,14 @@ k_cgemm(const TW* __restrict__ Wm, const TW* __restrict__ Wd, const float* __res
 }
 
 // G [L][L] = X^T X for X [n][L] fp32 row-major; float64 products and sums in
-// ascending row order.  16 x 16 outputs per CTA.
+// ascending row order.  16 x 16 outputs per CTA; only the tiles on or below
+// the diagonal are computed (the Cholesky reads the lower triangle alone).
 constexpr int GR_T = 16;
 constexpr int GR_KC = 32;
 __global__ void __launch_bounds__(GR_T * GR_T)
 k_gram(const float* __restrict__ X, int n, int L, double* __restrict__ G) {
   __shared__ double Xi[GR_KC][GR_T], Xj[GR_KC][GR_T];
+  if (blockIdx.x > blockIdx.y) return;  // strictly above the diagonal
   const int ti = threadIdx.x / GR_T, tj = threadIdx.x % GR_T;
   const int i0 = blockIdx.y * GR_T, j0 = blockIdx.x * GR_T;
   double acc = 0.0;
@@ -176,6 +178,7 @@ k_chol32(const double* __restrict__ G, int L, float shift_rel, float* __restrict
   extern __shared__ float Ls[];
   float* Xp = x_in_smem ? Ls + L * (L + 1) / 2 : Xg;  // packed lower X
   __shared__ double s_md;
+  __shared__ float s_diag[256];  // the factor's diagonal (Ls keeps the raw pivots)
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nw = CH_THREADS / 32;
   if (tid == 0) {
     double md = 0.0;
@@ -197,10 +200,10 @@ k_chol32(const double* __restrict__ G, int L, float shift_rel, float* __restrict
       Ls[i * (i + 1) / 2 + j] = (float)G[(size_t)i * L + j] + (i == j ? shift : 0.f);
   __syncthreads();
   for (int j = 0; j < L; ++j) {
-    const int jj = j * (j + 1) / 2 + j;
-    if (tid == 0) Ls[jj] = sqrtf(fmaxf(Ls[jj], 1e-30f));
-    __syncthreads();
-    const float ljj = Ls[jj];
+    // every thread takes the pivot from the raw entry, which nothing writes
+    // after the previous step's barrier; the factor's diagonal goes to s_diag
+    const float ljj = sqrtf(fmaxf(Ls[j * (j + 1) / 2 + j], 1e-30f));
+    if (tid == 0) s_diag[j] = ljj;
     for (int i = j + 1 + tid; i < L; i += CH_THREADS) Ls[i * (i + 1) / 2 + j] /= ljj;
     __syncthreads();
     for (int i = j + 1 + warp; i < L; i += nw) {
@@ -209,6 +212,8 @@ k_chol32(const double* __restrict__ G, int L, float shift_rel, float* __restrict
     }
     __syncthreads();
   }
+  for (int j = tid; j < L; j += CH_THREADS) Ls[j * (j + 1) / 2 + j] = s_diag[j];
+  __syncthreads();
   for (int q = tid; q < L * L; q += CH_THREADS) {
     const int i = q / L, c = q % L;
     Lout[q] = c <= i ? Ls[i * (i + 1) / 2 + c] : 0.f;
@@ -275,8 +280,10 @@ k_onesided(const float* __restrict__ Mt, int L, float* __restrict__ Mg, float* _
           p = round;
           q = Lp - 1;
         } else {
-          p = (round + P) % (Lp - 1);
-          q = (round - P + (Lp - 1)) % (Lp - 1);
+          p = round + P;
+          if (p >= Lp - 1) p -= Lp - 1;
+          q = round - P;
+          if (q < 0) q += Lp - 1;
         }
         float* mp = M + (size_t)p * L;
         float* mq = M + (size_t)q * L;
@@ -297,17 +304,17 @@ k_onesided(const float* __restrict__ Mt, int L, float* __restrict__ Mg, float* _
         const float z = (b - a) / (2.f * g);
         const float t = (z >= 0.f ? 1.f : -1.f) / (fabsf(z) + sqrtf(1.f + z * z));
         const float c = 1.f / sqrtf(1.f + t * t), s = t * c;
-        for (int i = lane; i < L; i += 32) {
-          const float x = mp[i], y = mq[i];
-          mp[i] = c * x - s * y;
-          mq[i] = s * x + c * y;
-        }
         float* wp = W + (size_t)p * Lp;
         float* wq = W + (size_t)q * Lp;
-        for (int k = lane; k < Lp; k += 32) {
-          const float x = wp[k], y = wq[k];
-          wp[k] = c * x - s * y;
-          wq[k] = s * x + c * y;
+        for (int i = lane; i < Lp; i += 32) {  // Lp >= L: one loop for M and W
+          if (i < L) {
+            const float x = mp[i], y = mq[i];
+            mp[i] = c * x - s * y;
+            mq[i] = s * x + c * y;
+          }
+          const float x = wp[i], y = wq[i];
+          wp[i] = c * x - s * y;
+          wq[i] = s * x + c * y;
         }
         if (lane == 0) s_rot = 1;
       }
