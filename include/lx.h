@@ -352,11 +352,16 @@ LX_API lx_status lx_permute_neurons(int32_t dtype, int32_t d_model, int32_t d_ff
  *   U = U_r S_r^(1/2) [rows][r] (the paper's B_m),  V = V_r S_r^(1/2) [cols][r]
  *   (A_m^T), so that U V^T ~ R, plus the singular values s [r].
  * Solver: Y = R Omega, Q = orth(Y); power_iters times Q = orth(R orth(R^T Q));
- * then the SVD of Q^T R through the l x l Gram (Jacobi, float64); products in
- * fp32 (CUDA cores), Gram matrices, orthonormalisation (CholeskyQR, twice) and
- * eigenvectors in float64.  The sign of each factor column is fixed so that the
+ * then the SVD of Bs = Q^T R: Z = R^T Q is orthonormalised too, Z = Z2 M^T with
+ * M the l x l triangular factor, and the small SVD of M (one-sided Jacobi)
+ * gives Bs's.  orth is CholeskyQR run twice (float64 Gram sums, fp32 Cholesky;
+ * the first pass is shifted by 1e-6 of the largest Gram diagonal); the
+ * products with R are fp32 (CUDA cores); singular values are float64 Rayleigh
+ * quotients.  The sign of each factor column is fixed so that the
  * largest-magnitude entry of U's column is positive.  Singular values at or
- * below 1e-6 of the largest give zero V columns.
+ * below 1e-6 of the largest give zero U and V columns.  The call is latency
+ * bound (one-CTA stages): independent projections run concurrently when given
+ * their own streams and workspaces.
  *   dtype:      LX_F32 or LX_BF16 of w_dom / w_mem
  *   rows, cols: the projection's [out][in] shape, multiples of 8 (gate / up:
  *               [I][H], down: [H][I]); w_dom, w_mem device, 16-byte aligned
