@@ -123,3 +123,32 @@ def test_statistics_calls_rejected_on_host(L):
     assert L.lx_coact_npmi(None, 16, 4, buf, None) == lx.LX_ERR_ARG
     assert L.lx_coact_npmi(buf, 0, 4, buf, None) == lx.LX_ERR_ARG
     assert L.lx_coact_npmi(buf, 16, -1, buf, None) == lx.LX_ERR_ARG
+
+
+def _declared_arity():
+    """{name: parameter count} of every LX_API function in include/lx.h."""
+    src = open(os.path.join(ROOT, "include", "lx.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    out = {}
+    for m in re.finditer(r"LX_API\s+[\w\s\*]+?\b(lx_\w+)\s*\(([^)]*)\)\s*;", src, flags=re.S):
+        params = m.group(2).strip()
+        out[m.group(1)] = 0 if params in ("", "void") else len(params.split(","))
+    return out
+
+
+def test_binding_arity_matches_header(L):
+    arity = _declared_arity()
+    assert sorted(arity) == sorted(lx.EXPORTS)
+    for name, n in arity.items():
+        f = getattr(L, name)
+        got = len(f.argtypes) if f.argtypes is not None else 0
+        assert got == n, f"{name}: binding declares {got} arguments, the header {n}"
+
+
+def test_layer_desc_struct_matches_header():
+    """lx_layer_desc's fields, in order, as the binding lays them out."""
+    src = open(os.path.join(ROOT, "include", "lx.h")).read()
+    body = re.search(r"typedef struct \{(.*?)\} lx_layer_desc;", src, flags=re.S).group(1)
+    body = re.sub(r"/\*.*?\*/", "", body, flags=re.S)
+    fields = re.findall(r"\b(\w+)\s*;", body)
+    assert fields == [f for f, _ in lx.LayerDesc._fields_]
