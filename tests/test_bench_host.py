@@ -6,6 +6,7 @@ import os
 import socket
 import sys
 
+import numpy as np
 import pytest
 import torch
 import torch.multiprocessing as mp
@@ -64,3 +65,42 @@ def test_reference_arm_only_rank0_works():
     class A:
         workload, ref_tokens, warmup, steps = "decode64", 2, 3, 1
     assert bench.run_reference(A(), rank=1, world=2) is None
+
+
+def _routed_stats(src, T, seed):
+    import oracle
+    import synth
+    x = synth.tokens(src, T, seed=seed)
+    ids, _, _ = oracle.route(src, x)
+    b = oracle.buckets(src, ids)
+    return bench.routing_stats(src, b["node_off"], T, src.top_k), b
+
+
+def test_tensor_core_flop_table_sums_to_the_cost_model():
+    """The six tensor-core GEMMs' FLOPs (bench.kernel_flops) add up to the
+    amortised forward's expert FLOPs (cost.step_counts) on the realised
+    routing: each (token, node) pair counted once, anchors 2*3IH, rank-r
+    corrections 2*3r(I+H)."""
+    import synth
+    from paper_2608_07814_gb300 import cost
+    for src in (synth.tree_layer(256, 192, 2, 4, 3, 128, 64, 8, "bf16", seed=15,
+                                 skew=synth.TREE_SKEW),
+                synth.flat_layer(320, 448, [1, 3, 1, 5, 2], [64, 128, 192, 64, 64, 128, 192], 3,
+                                 "bf16", seed=14)):
+        st, b = _routed_stats(src, 300, seed=3)
+        total = sum(bench.kernel_flops(n, st, src) for n in
+                    ("tc_up_anchor", "tc_up_V", "tc_up_U", "tc_dn_anchor", "tc_dn_V", "tc_dn_U"))
+        ref = cost.step_counts(src.d_model, src.d_ff, src.n_experts, src.node_parent,
+                               src.node_rank, st["cnt"], 300, 2, 2)["expert_flops"]
+        assert total == ref
+
+
+def test_routing_stats_match_the_buckets():
+    import synth
+    src = synth.flat_layer(256, 128, [4] * 4, 64, 4, "bf16", seed=10, skew=synth.QWEN_SKEW)
+    st, b = _routed_stats(src, 200, seed=1)
+    cnt = np.diff(b["node_off"].astype(np.int64))
+    anchors = np.asarray(src.node_parent) < 0
+    assert st["R_anchor"] + st["R_corr"] == len(b["node_tok"])
+    assert st["touched_anchor"] == int(np.sum((cnt > 0) & anchors))
+    assert st["corr_r_rows"] == int(np.sum(cnt[~anchors] * np.asarray(src.node_rank)[~anchors]))
