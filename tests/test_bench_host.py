@@ -104,3 +104,21 @@ def test_routing_stats_match_the_buckets():
     assert st["R_anchor"] + st["R_corr"] == len(b["node_tok"])
     assert st["touched_anchor"] == int(np.sum((cnt > 0) & anchors))
     assert st["corr_r_rows"] == int(np.sum(cnt[~anchors] * np.asarray(src.node_rank)[~anchors]))
+
+
+def test_streaming_weight_bytes_match_the_cost_model():
+    """The weight bytes inside the four streaming ops' byte counts (the part
+    that scales with the element size, less the gathered token rows) are the
+    cost model's touched-weight bytes: every touched node's weights once."""
+    import synth
+    from paper_2608_07814_gb300 import cost
+    src = synth.tree_layer(256, 192, 2, 4, 3, 128, 64, 8, "bf16", seed=15, skew=synth.TREE_SKEW)
+    st, b = _routed_stats(src, 64, seed=2)
+    ops = ("stream_up_anchor_V", "stream_up_U", "stream_dn_anchor_V", "stream_dn_U")
+    scaled = sum(bench.kernel_bytes(n, st, src, 2) - bench.kernel_bytes(n, st, src, 0) for n in ops)
+    x_rows = (st["R_anchor"] + st["R_corr"]) * src.d_model * 2
+    ref = cost.step_counts(src.d_model, src.d_ff, src.n_experts, src.node_parent, src.node_rank,
+                           st["cnt"], 64, 2, 2)["weight_bytes"]
+    assert scaled - x_rows == ref
+    assert bench.kernel_bytes("stream_up", st, src, 2) + bench.kernel_bytes("stream_dn", st, src, 2) \
+        == sum(bench.kernel_bytes(n, st, src, 2) for n in ops)
