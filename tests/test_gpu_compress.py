@@ -14,6 +14,8 @@ projection shapes), a decaying spectrum, an exactly rank-5 residual (recovered
 exactly), a zero residual (the dominant compressed against itself gives zero
 factors), and an odd l.
 """
+import ctypes
+
 import numpy as np
 import pytest
 import torch
@@ -89,7 +91,7 @@ def test_compress_factor(rows, cols, dtype, r, l, q, kind):
 def test_workspace_query_and_rejects():
     assert lx.compress_workspace_bytes(768, 2048, 136, 128) > 0
     L = lx.lib()
-    b = __import__("ctypes").c_uint64()
+    b = ctypes.c_uint64()
     assert L.lx_compress_workspace(768, 2048, 257, 128, b) == lx.LX_ERR_SHAPE   # l > 256
     assert L.lx_compress_workspace(768, 2048, 100, 128, b) == lx.LX_ERR_SHAPE   # l < r
     assert L.lx_compress_workspace(770, 2048, 136, 128, b) == lx.LX_ERR_SHAPE   # rows % 8
