@@ -2,8 +2,9 @@
 oracle (oracle/compress.py), through the C ABI, on the same residual and the
 same Gaussian test matrix.
 
-Bar, derived from the arithmetic (fp32 products, float64 small factorisations;
-the same algorithm, so only rounding separates the two):
+Bar, derived from the arithmetic (fp32 products, Cholesky factors and Jacobi
+rotations; float64 Gram sums and Rayleigh quotients; the same subspaces as the
+oracle's float64 algorithm, so only rounding separates the two):
   * the rank-r approximation U V^T within 1e-4 of max|U_ref V_ref^T|;
   * singular values within 1e-5 of the largest;
   * ||R - U V^T||_F within 1e-5 (relative) of the oracle's;
