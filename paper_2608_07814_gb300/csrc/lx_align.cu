@@ -394,8 +394,9 @@ extern "C" lx_status lx_permute_neurons(int32_t dtype, int32_t d_model, int32_t 
 }
 
 // Exact linear assignment on the host: Jonker and Volgenant's column reduction
-// assigns every column's cheapest row where that row is free; each remaining
-// row is then added by a shortest augmenting path (Dijkstra over the columns
+// assigns every column's cheapest row where that row is free, their augmenting
+// row reduction assigns most of the rest; each remaining row is then added by
+// a shortest augmenting path (Dijkstra over the columns
 // on reduced costs c[i][j] - u[i] - v[j] >= 0), after which the dual
 // potentials u, v are updated so that every reduced cost stays non-negative
 // and those on the matching are zero -- JV's augmentation.  O(n^3), float64.
@@ -434,6 +435,75 @@ void lap_solve_one(const float* cost, int32_t n, int32_t* assign, double* total)
       row_used[best_i] = 1;
       row_of[j] = best_i;
     }
+  }
+  // JV augmenting row reduction, two passes over the free rows: a free row i
+  // takes the column j1 minimising c_ij - v_j; if that beats the runner-up j2
+  // strictly, v_j1 drops by the gap (so j1 and j2 tie for row i) and the row
+  // that held j1, if any, is processed next; on a tie the row takes j2 when j1
+  // is held, and a displaced row waits for the next pass.  Every assigned row
+  // keeps a column of least c_ij - v_j (lowering a v only raises c - v), so
+  // u_i = that least value makes c - u - v >= 0 with the matching tight.  A
+  // step limit hands whatever is left to the augmentation below, which is exact
+  // from any such state.
+  std::vector<int> col_of(n + 1, 0);
+  for (int j = 1; j <= n; ++j)
+    if (row_of[j]) col_of[row_of[j]] = j;
+  if (n > 1) {
+    std::vector<int> freel, later;
+    for (int i = 1; i <= n; ++i)
+      if (!row_used[i]) freel.push_back(i);
+    for (int pass = 0; pass < 2 && !freel.empty(); ++pass) {
+      later.clear();
+      size_t k = 0;
+      long steps = 0;
+      const long max_steps = 16L * n;
+      while (k < freel.size()) {
+        if (++steps > max_steps) {
+          for (; k < freel.size(); ++k) later.push_back(freel[k]);
+          break;
+        }
+        const int i = freel[k++];
+        const float* ci = cost + (size_t)(i - 1) * n;
+        double u1 = (double)ci[0] - v[1], u2 = kInf;
+        int j1 = 1, j2 = 0;
+        for (int j = 2; j <= n; ++j) {
+          const double h = (double)ci[j - 1] - v[j];
+          if (h < u2) {
+            if (h >= u1) {
+              u2 = h;
+              j2 = j;
+            } else {
+              u2 = u1;
+              u1 = h;
+              j2 = j1;
+              j1 = j;
+            }
+          }
+        }
+        int i0 = row_of[j1];
+        const bool strict = u1 < u2;
+        if (strict) {
+          v[j1] -= u2 - u1;
+        } else if (i0 != 0) {
+          j1 = j2;
+          i0 = row_of[j1];
+        }
+        if (i0 != 0) {
+          col_of[i0] = 0;
+          row_used[i0] = 0;
+        }
+        row_of[j1] = i;
+        col_of[i] = j1;
+        row_used[i] = 1;
+        if (i0 != 0) {
+          if (strict) freel[--k] = i0;  // the displaced row goes next
+          else later.push_back(i0);
+        }
+      }
+      freel.swap(later);
+    }
+    for (int i = 1; i <= n; ++i)
+      if (row_used[i]) u[i] = (double)cost[(size_t)(i - 1) * n + (col_of[i] - 1)] - v[col_of[i]];
   }
   for (int r = 1; r <= n; ++r) {
     if (row_used[r]) continue;

@@ -88,3 +88,34 @@ def test_batch_matches_single_solves_on_threads():
         lx.lap_solve_batch(bad)
     P0, t0 = lx.lap_solve_batch(costs[:0])
     assert P0.shape == (0, n)
+
+
+@pytest.mark.parametrize("seed", [0, 1, 2])
+def test_optimum_on_adversarial_families(seed):
+    """Ties, constant matrices, identical rows, negative and large costs,
+    rank-one and squared-distance costs: the optimum equals SciPy's."""
+    rng = np.random.default_rng(100 + seed)
+    for n in list(range(1, 10)) * 4 + [17, 40]:
+        for kind in range(8):
+            if kind == 0:
+                C = rng.random((n, n))
+            elif kind == 1:
+                C = rng.integers(0, 3, (n, n))
+            elif kind == 2:
+                C = np.full((n, n), 7.0)
+            elif kind == 3:
+                C = np.tile(rng.random(n), (n, 1))
+            elif kind == 4:
+                C = -rng.random((n, n)) * 1e3
+            elif kind == 5:
+                C = rng.random((n, n)) * 1e6 - 5e5
+            elif kind == 6:
+                a, b = rng.standard_normal((n, 5)), rng.standard_normal((n, 5))
+                C = (a * a).sum(1)[:, None] + (b * b).sum(1)[None, :] - 2 * a @ b.T
+            else:
+                C = np.outer(rng.random(n), rng.random(n))
+            C = C.astype(np.float32)
+            P, tot = lx.lap_solve(C)
+            assert sorted(P.tolist()) == list(range(n))
+            ref = align.assignment_cost(C, align.assign(C))
+            assert abs(align.assignment_cost(C, P) - ref) <= 1e-9 * max(1.0, abs(ref))
