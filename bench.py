@@ -506,20 +506,27 @@ def run_lx(args, rank, world, local_rank):
     return line
 
 
-def _event_ms(fn, steps, warmup):
+def _event_ms(fn, steps, warmup, world=1):
     """Average ms per call of fn() over `steps` calls on the current stream
-    (CUDA events, synchronised on both sides), after `warmup` calls."""
+    (CUDA events, synchronised on both sides), after `warmup` calls; with
+    several ranks a barrier precedes the timed calls and the slowest rank's
+    time is returned."""
     import torch
     for _ in range(warmup):
         fn()
     torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
     a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     a.record()
     for _ in range(steps):
         fn()
     b.record()
     torch.cuda.synchronize()
-    return a.elapsed_time(b) / steps
+    ms = a.elapsed_time(b) / steps
+    if world > 1:
+        ms = max_over_ranks([ms], world, torch.device("cuda", torch.cuda.current_device()))[0]
+    return ms
 
 
 def run_offline(args, rank, world, local_rank):
@@ -551,7 +558,7 @@ def run_offline(args, rank, world, local_rank):
         def step():
             lx.coact_accumulate(ids[it[0] % nb], E, fire, coact)
             it[0] += 1
-        ms = _event_ms(step, args.steps, args.warmup)
+        ms = _event_ms(step, args.steps, args.warmup, world)
         byts = T * k * 4 + 2 * E * E * 8
         t_npmi = _event_ms(lambda: lx.coact_npmi(coact, T * nb), 20, 3)
         host_ids = [i.cpu().numpy() for i in ids[:2]]
@@ -613,7 +620,7 @@ def run_offline(args, rank, world, local_rank):
                 e = torch.cuda.Event()
                 e.record(st)
                 main.wait_event(e)
-        ms = _event_ms(step_conc, args.steps, args.warmup) / n_conc
+        ms = _event_ms(step_conc, args.steps, args.warmup, world) / n_conc
         big = sum((2 + 2 * q) * 2.0 * a * b * l for a, b in shapes)        # the R-sized products
         small = sum(2 * (1 + 2 * q) * 2 * (2.0 * a * l * l + a * l * l) + 2.0 * b * l * l
                     + 2.0 * (a + b) * l * r for a, b in shapes)           # Grams, orthonormalisation
@@ -655,7 +662,7 @@ def run_offline(args, rank, world, local_rank):
         def step():
             lx.align_cost(dd, md[it[0] % 4])
             it[0] += 1
-        ms = _event_ms(step, args.steps, args.warmup)
+        ms = _event_ms(step, args.steps, args.warmup, world)
         cost = lx.align_cost(dd, md[0]).cpu().numpy()
         t0 = time.time()
         P, _ = lx.lap_solve(cost)
@@ -720,7 +727,7 @@ def run_offline(args, rank, world, local_rank):
                                       "cores": os.cpu_count(), "kind": "oracle",
                                       "sample": "64 of the 768 cost rows (float64 definition)"}})
         line["config"].update({"d_model": H, "d_ff": I, "l2": "4 rotating members (L2-resident)"})
-    return line
+    return line if rank == 0 else None
 
 
 def cpu_baseline(src, xs_host, T, budget_s):
