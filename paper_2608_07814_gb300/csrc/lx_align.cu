@@ -13,8 +13,10 @@
 // k_align_cost_mma: the same tile for bf16 experts on the tensor cores
 // (mma.sync, bf16 inputs, fp32 accumulation).
 // k_permute_rows / k_permute_cols: gathers (bit-exact copies).
-// lx_lap_solve: the exact assignment on the host (shortest augmenting paths
-// with dual potentials, the augmentation scheme of Jonker and Volgenant).
+// lx_lap_solve / lx_lap_solve_batch: the exact assignment on the host (Jonker
+// and Volgenant: column reduction, augmenting row reduction, then shortest
+// augmenting paths with dual potentials); the batch form spreads independent
+// problems over host threads.
 #include <algorithm>
 #include <atomic>
 #include <limits>

@@ -20,10 +20,10 @@
 //   k_ritz      sigma_j = |M w_j| / |w_j| in float64 (Rayleigh quotients).
 //   k_finish    the r largest sigma and the fp32 matrices that turn the bases
 //               into the split factors.
-// Only the Gram sums and the Rayleigh quotients use float64: a single SM's
-// float64 rate is a small fraction of its fp32 rate on this GPU.
 //   k_sign      each factor column's largest-magnitude entry of U made
 //               positive (U and V negated together).
+// Only the Gram sums and the Rayleigh quotients use float64: a single SM's
+// float64 rate is a small fraction of its fp32 rate on this GPU.
 #include <algorithm>
 #include <cmath>
 
