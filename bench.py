@@ -271,9 +271,210 @@ def batch_seed(rank, b):
 # ----------------------------------------------------------------------------
 # the CUDA arm
 # ----------------------------------------------------------------------------
+def workload_config(src, T, desc):
+    """The workload's `config` (identical in both arms)."""
+    return {"workload": desc, "d_model": src.d_model, "d_ff": src.d_ff,
+            "n_experts": src.n_experts, "top_k": src.top_k, "n_nodes": src.n_nodes,
+            "tokens_per_step": T, "layer_bytes": src.weight_bytes(),
+            "l2": "inputs larger than L2 (GPU arm: rotating device copies of the layer for "
+                  "decode batches, 8 token batches; the reference arm runs on the host cores)"}
+
+
+def time_steps(layers, xs, ys, k, steps, warmup, world, clocks, graph=True):
+    """Step time and per-kernel device times of `steps` forwards.
+
+    The step time comes from one CUDA graph of the forwards without
+    instrumentation (dependent launch on); the kernel durations from a second
+    graph of the same forwards with the library's CUDA events around every
+    launch.  Barrier + synchronize on both sides of the timed region; the max
+    over ranks is taken by the caller."""
+    import torch
+    n_copies, n_batches = len(layers), len(xs)
+    stream = torch.cuda.current_stream()
+
+    def run(n):
+        for i in range(n):
+            layers[i % n_copies].moe_forward(xs[i % n_batches], k, ys[i % n_batches])
+
+    for i in range(warmup):
+        layers[i % n_copies].moe_forward(xs[i % n_batches], k, ys[i % n_batches])
+    torch.cuda.synchronize()
+    # one profiled pass fills each layer's event pool, so that the instrumented
+    # capture below creates no events
+    for L in layers:
+        L.read_profile()
+        L.set_profiling(True)
+    run(steps)
+    torch.cuda.synchronize()
+    for L in layers:
+        L.read_profile(cap=1 << 20)
+    g = gp = None
+    if graph:
+        gp = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(gp):
+            run(steps)
+    for L in layers:
+        L.set_profiling(False)
+    if graph:
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            run(steps)
+        g.replay()  # untimed replay: first-launch costs of the graph
+        torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0 = time.time()
+    ev0.record(stream)
+    if g is not None:
+        g.replay()
+    else:
+        run(steps)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    clocks.mark(t0, time.time())
+    ms = ev0.elapsed_time(ev1)
+    t1 = time.time()
+    if gp is not None:
+        gp.replay()
+    else:
+        for L in layers:
+            L.set_profiling(True)
+        run(steps)
+        for L in layers:
+            L.set_profiling(False)
+    torch.cuda.synchronize()
+    clocks.mark(t1, time.time())
+    per_copy = [L.read_profile(cap=1 << 20) for L in layers]
+    del g, gp
+    return ms, per_copy
+
+
+def kernel_tables(per_copy, steps, n_copies, stats, src):
+    """Per-kernel totals, launch counts and algorithmic bytes / FLOPs of the
+    timed launches (records are in launch order per layer copy)."""
+    esz = 2 if src.dtype == "bf16" else 4
+    totals, counts, kbytes, kflops, kalu = {}, {}, {}, {}, {}
+    launches = 0
+    for c, recs in enumerate(per_copy):
+        steps_of_copy = [i for i in range(steps) if i % n_copies == c]
+        per_step = len(recs) // max(1, len(steps_of_copy))
+        for j, (name, kms) in enumerate(recs):
+            totals[name] = totals.get(name, 0.0) + kms
+            counts[name] = counts.get(name, 0) + 1
+            if name != "bucket_clear":
+                launches += 1
+            st = stats[(steps_of_copy[j // per_step] if per_step else 0) % len(stats)]
+            for table, f in ((kbytes, kernel_bytes(name, st, src, esz)),
+                             (kflops, kernel_flops(name, st, src)),
+                             (kalu, kernel_alu_flops(name, st, src))):
+                if f is not None:
+                    table[name] = table.get(name, 0.0) + f
+    return totals, counts, kbytes, kflops, kalu, launches
+
+
+def roofline_summary(src, T, ms, steps, stats, tabs, peaks, peak_kind, workload):
+    """Dominant kernel's roofline, per-kernel fractions and the step roofline."""
+    totals, counts, kbytes, kflops, kalu, launches = tabs
+    esz = 2 if src.dtype == "bf16" else 4
+    hbm = float(peaks["hbm_gbs"])
+    tf, tfs = float(peaks["bf16_tflops"]), float(peaks["bf16_tflops_sustained"])
+    alu = fp32_alu_peak_tflops(peaks)
+    dom = max(totals, key=totals.get)
+    avg_ms = totals[dom] / counts[dom]
+    roof = None
+    if dom in kalu and src.dtype == "bf16" and T > 256:
+        # the large-batch router: fp32 FMAs on the CUDA cores
+        fl = kalu[dom] / counts[dom]
+        ach = fl / (avg_ms * 1e-3) / 1e12
+        roof = {"kernel": dom, "bound": "alu", "achieved": round(ach, 2), "peak": round(alu, 1),
+                "unit": "TFLOP/s", "frac": round(ach / alu, 4), "traffic": traffic_for(dom, workload),
+                "algorithmic_flops_per_launch": round(fl), "avg_launch_us": round(avg_ms * 1e3, 2),
+                "peak_source": "derived fp32 FMA peak (152 SMs x 128 lanes x 2 x max SM clock)"}
+    elif dom in kbytes:
+        b = kbytes[dom] / counts[dom]
+        ach = b / (avg_ms * 1e-3) / 1e9
+        roof = {"kernel": dom, "bound": "hbm", "achieved": round(ach, 1), "peak": hbm,
+                "unit": "GB/s", "frac": round(ach / hbm, 4), "traffic": traffic_for(dom, workload),
+                "algorithmic_bytes_per_launch": round(b), "avg_launch_us": round(avg_ms * 1e3, 2),
+                "peak_source": f"{peak_kind} hbm_gbs"}
+    elif dom in kflops:
+        fl = kflops[dom] / counts[dom]
+        ach = fl / (avg_ms * 1e-3) / 1e12
+        roof = {"kernel": dom, "bound": "tensor", "achieved": round(ach, 1), "peak": tf,
+                "unit": "TFLOP/s", "frac": round(ach / tf, 4), "traffic": traffic_for(dom, workload),
+                "algorithmic_flops_per_launch": round(fl), "avg_launch_us": round(avg_ms * 1e3, 2),
+                "peak_source": f"{peak_kind} bf16_tflops (burst)"}
+
+    def kernel_frac(n):
+        t = totals[n] / counts[n] * 1e-3
+        if n in kflops:
+            return {"frac_bf16": round(kflops[n] / counts[n] / t / 1e12 / tf, 4)}
+        if n in kalu and src.dtype == "bf16" and T > 256:
+            return {"frac_alu": round(kalu[n] / counts[n] / t / 1e12 / alu, 4)}
+        if n in kbytes:
+            return {"frac_hbm": round(kbytes[n] / counts[n] / t / 1e9 / hbm, 4)}
+        return {}
+
+    cs = [step_bytes(stats[i % len(stats)], src, esz) for i in range(steps)]
+    sec = ms * 1e-3
+    step_b = sum(c["bytes"] for c in cs)
+    step_f = sum(c["flops"] for c in cs)
+    step = {"algorithmic_bytes_per_step": round(step_b / steps),
+            "algorithmic_flops_per_step": round(step_f / steps),
+            "achieved_gbs": round(step_b / sec / 1e9, 1),
+            "achieved_tflops": round(step_f / sec / 1e12, 1)}
+    if T <= 256:
+        step.update({"bound": "hbm", "frac": round(step_b / sec / 1e9 / hbm, 4),
+                     "frac_nominal_8tbs": round(step_b / sec / 1e9 / 8000.0, 4),
+                     "peak": f"{peak_kind} hbm_gbs {hbm}"})
+    else:
+        step.update({"bound": "tensor", "frac": round(step_f / sec / 1e12 / tf, 4),
+                     "frac_sustained": round(step_f / sec / 1e12 / tfs, 4),
+                     "peak": f"{peak_kind} bf16_tflops {tf} (burst), {tfs} (sustained)"})
+    amort = float(np.mean([st["T"] * st["k"] / max(1, st["R_anchor"]) for st in stats]))
+    kernels = {n: {"launches": counts[n], "avg_us": round(totals[n] / counts[n] * 1e3, 2),
+                   "share": round(totals[n] / sum(totals.values()), 4), **kernel_frac(n)}
+               for n in totals}
+    return roof, kernels, step, round(amort, 3), launches
+
+
+def setup_workload(src, T, n_copies, rank, dev, layers=None):
+    """Installed layer copies, 8 token batches on the device and their hosts."""
+    import synth
+    from paper_2608_07814_gb300 import lx
+    if layers is None:
+        layers = [lx.Layer(src) for _ in range(n_copies)]
+    for L in layers:
+        L.reserve(T, src.top_k)
+    xs_host = [synth.tokens(src, T, seed=batch_seed(rank, b)) for b in range(8)]
+    xs = [lx.host_to_torch(x, src.dtype).to(dev) for x in xs_host]
+    ys = [torch_empty_like(x) for x in xs]
+    return layers, xs_host, xs, ys
+
+
+def torch_empty_like(x):
+    import torch
+    return torch.empty_like(x)
+
+
+def batch_stats(src, layer, xs, ys, T):
+    """Routing statistics of every batch (outside the timed region)."""
+    import torch
+    stats = []
+    for b in range(len(xs)):
+        layer.moe_forward(xs[b], src.top_k, ys[b])
+        bk = layer.get_buckets()
+        torch.cuda.synchronize()
+        stats.append(routing_stats(src, bk["node_off"].cpu().numpy(), T, src.top_k))
+    return stats
+
+
 def run_lx(args, rank, world, local_rank):
     import torch
-    import synth
     from paper_2608_07814_gb300 import lx
 
     torch.cuda.set_device(local_rank)
@@ -281,128 +482,26 @@ def run_lx(args, rank, world, local_rank):
     kind, T, desc = WORKLOADS[args.workload]
     src = make_layer(kind)
     k = src.top_k
-    esz = 2 if src.dtype == "bf16" else 4
-    wbytes = src.weight_bytes()
     n_copies = args.copies if args.copies else (4 if T <= 512 else 1)
-    layers = [lx.Layer(src) for _ in range(n_copies)]
-    for L in layers:
-        L.reserve(T, k)
-    n_batches = 8
-    xs_host = [synth.tokens(src, T, seed=batch_seed(rank, b)) for b in range(n_batches)]
-    xs = [lx.host_to_torch(x, src.dtype).to(dev) for x in xs_host]
-    ys = [torch.empty_like(x) for x in xs]
-    stream = torch.cuda.current_stream()
-
-    # routing statistics of every batch (outside the timed region)
-    stats = []
-    for b in range(n_batches):
-        layers[0].moe_forward(xs[b], k, ys[b])
-        bk = layers[0].get_buckets()
-        torch.cuda.synchronize()
-        stats.append(routing_stats(src, bk["node_off"].cpu().numpy(), T, k))
+    layers, xs_host, xs, ys = setup_workload(src, T, n_copies, rank, dev)
+    stats = batch_stats(src, layers[0], xs, ys, T)
+    peaks, peak_kind = load_peaks()
 
     clocks = Clocks(local_rank)
     clocks.start()
-    for i in range(args.warmup):
-        layers[i % n_copies].moe_forward(xs[i % n_batches], k, ys[i % n_batches])
-    torch.cuda.synchronize()
-
-    def steps(n):
-        for i in range(n):
-            layers[i % n_copies].moe_forward(xs[i % n_batches], k, ys[i % n_batches])
-
-    # One profiled pass of the same steps fills each layer's event pool, so the
-    # instrumented capture below creates no events.
-    for L in layers:
-        L.read_profile()
-        L.set_profiling(True)
-    steps(args.steps)
-    torch.cuda.synchronize()
-    for L in layers:
-        L.read_profile(cap=1 << 20)
-    graph = graph_prof = None
-    if not args.no_graph:
-        # Two CUDA graphs of the same K forwards: `graph_prof` carries the
-        # library's per-kernel events (external event nodes stamped by the
-        # replay; dependent launch off) and gives the kernel durations;
-        # `graph` has no events (dependent launch on) and gives the step time.
-        graph_prof = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(graph_prof):
-            steps(args.steps)
-    for L in layers:
-        L.set_profiling(False)
-    if not args.no_graph:
-        graph = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(graph):
-            steps(args.steps)
-        graph.replay()  # untimed replay: first-launch costs of the graph
-        torch.cuda.synchronize()
-
-    # timed region 1: the step time (no instrumentation)
-    if world > 1:
-        torch.distributed.barrier()
-    torch.cuda.synchronize()
-    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    t_wall0 = time.time()
-    ev0.record(stream)
-    if graph is not None:
-        graph.replay()
-    else:
-        steps(args.steps)
-    ev1.record(stream)
-    torch.cuda.synchronize()
-    if world > 1:
-        torch.distributed.barrier()
-    t_wall1 = time.time()
-    clocks.mark(t_wall0, t_wall1)
-    ms = ev0.elapsed_time(ev1)
-
-    # timed region 2: the same steps with per-kernel events
-    t_p0 = time.time()
-    if graph_prof is not None:
-        graph_prof.replay()
-    else:
-        for L in layers:
-            L.set_profiling(True)
-        steps(args.steps)
-        for L in layers:
-            L.set_profiling(False)
-    torch.cuda.synchronize()
-    clocks.mark(t_p0, time.time())
-
-    # per-kernel device times of the timed launches (in launch order per copy)
-    per_copy = [L.read_profile(cap=1 << 20) for L in layers]
-    totals, counts = {}, {}
-    launches = 0
-    kbytes, kflops, kalu = {}, {}, {}
-    for c, recs in enumerate(per_copy):
-        steps_of_copy = [i for i in range(args.steps) if i % n_copies == c]
-        per_step = len(recs) // max(1, len(steps_of_copy))
-        for j, (name, kms) in enumerate(recs):
-            totals[name] = totals.get(name, 0.0) + kms
-            counts[name] = counts.get(name, 0) + 1
-            if name != "bucket_clear":
-                launches += 1
-            step_i = steps_of_copy[j // per_step] if per_step else 0
-            b = kernel_bytes(name, stats[step_i % n_batches], src, esz)
-            if b is not None:
-                kbytes[name] = kbytes.get(name, 0.0) + b
-            f = kernel_flops(name, stats[step_i % n_batches], src)
-            if f is not None:
-                kflops[name] = kflops.get(name, 0.0) + f
-            a = kernel_alu_flops(name, stats[step_i % n_batches], src)
-            if a is not None:
-                kalu[name] = kalu.get(name, 0.0) + a
+    ms, per_copy = time_steps(layers, xs, ys, k, args.steps, args.warmup, world, clocks,
+                              graph=not args.no_graph)
 
     # e2e: host buffers, copies inside the timed region, a read of every result
+    stream = torch.cuda.current_stream()
     xh = [lx.host_to_torch(x, src.dtype).pin_memory() for x in xs_host]
     yh = [torch.empty_like(x).pin_memory() for x in xh]
     xd, yd = torch.empty_like(xs[0]), torch.empty_like(xs[0])
     k_e2e = max(3, min(args.steps, 200))
     for i in range(3):
-        xd.copy_(xh[i % n_batches], non_blocking=True)
+        xd.copy_(xh[i % len(xh)], non_blocking=True)
         layers[i % n_copies].moe_forward(xd, k, yd)
-        yh[i % n_batches].copy_(yd, non_blocking=True)
+        yh[i % len(xh)].copy_(yd, non_blocking=True)
     torch.cuda.synchronize()
     if world > 1:
         torch.distributed.barrier()
@@ -410,67 +509,32 @@ def run_lx(args, rank, world, local_rank):
     t_e2e0 = time.time()
     e0.record(stream)
     for i in range(k_e2e):
-        xd.copy_(xh[i % n_batches], non_blocking=True)
+        xd.copy_(xh[i % len(xh)], non_blocking=True)
         layers[i % n_copies].moe_forward(xd, k, yd)
-        yh[i % n_batches].copy_(yd, non_blocking=True)
+        yh[i % len(xh)].copy_(yd, non_blocking=True)
         stream.synchronize()
     e1.record(stream)
     torch.cuda.synchronize()
     clocks.mark(t_e2e0, time.time())
     ms_e2e = e0.elapsed_time(e1)
+
+    # the other workloads of the metric, at one GPU, in the same run
+    per_config = None
+    if world == 1 and not args.no_per_config and args.workload == "decode64":
+        per_config = run_per_config(args, rank, dev, src, layers, clocks, peaks, peak_kind)
     clk = clocks.stop()
 
-    # max over ranks
     ms, ms_e2e = max_over_ranks([ms, ms_e2e], world, dev)
     if rank != 0:
         return None
-
-    peaks, peak_kind = load_peaks()
-    hbm = float(peaks["hbm_gbs"])
-    dom = max(totals, key=totals.get)
-    avg_ms = totals[dom] / counts[dom]
-    roof = None
-    if dom in kalu and src.dtype == "bf16" and T > 256:
-        # the large-batch router: fp32 FMAs on the CUDA cores
-        alu = fp32_alu_peak_tflops(peaks)
-        fl = kalu[dom] / counts[dom]
-        ach = fl / (avg_ms * 1e-3) / 1e12
-        roof = {"kernel": dom, "bound": "alu", "achieved": round(ach, 2), "peak": round(alu, 1),
-                "unit": "TFLOP/s", "frac": round(ach / alu, 4), "traffic": traffic_for(dom, args.workload),
-                "algorithmic_flops_per_launch": round(fl), "avg_launch_us": round(avg_ms * 1e3, 2),
-                "peak_source": "derived fp32 FMA peak (152 SMs x 128 lanes x 2 x max SM clock)"}
-    elif dom in kbytes:
-        bytes_per_launch = kbytes[dom] / counts[dom]
-        ach = bytes_per_launch / (avg_ms * 1e-3) / 1e9
-        roof = {"kernel": dom, "bound": "hbm", "achieved": round(ach, 1), "peak": hbm,
-                "unit": "GB/s", "frac": round(ach / hbm, 4), "traffic": traffic_for(dom, args.workload),
-                "algorithmic_bytes_per_launch": round(bytes_per_launch),
-                "avg_launch_us": round(avg_ms * 1e3, 2), "peak_source": f"{peak_kind} hbm_gbs"}
-    elif dom in kflops:
-        # a contraction on the tensor cores, timed alone per launch: burst bf16 peak
-        tf = float(peaks["bf16_tflops"])
-        flops_per_launch = kflops[dom] / counts[dom]
-        ach = flops_per_launch / (avg_ms * 1e-3) / 1e12
-        roof = {"kernel": dom, "bound": "tensor", "achieved": round(ach, 1), "peak": tf,
-                "unit": "TFLOP/s", "frac": round(ach / tf, 4), "traffic": traffic_for(dom, args.workload),
-                "algorithmic_flops_per_launch": round(flops_per_launch),
-                "avg_launch_us": round(avg_ms * 1e3, 2),
-                "peak_source": f"{peak_kind} bf16_tflops (burst)"}
-    def kernel_frac(n):
-        """this kernel's own roofline fraction (streaming: HBM, tensor-core:
-        bf16 burst, large-batch router: fp32 ALU), from its event times"""
-        t = totals[n] / counts[n] * 1e-3
-        if n in kflops:
-            return {"frac_bf16": round(kflops[n] / counts[n] / t / 1e12 / float(peaks["bf16_tflops"]), 4)}
-        if n in kalu and src.dtype == "bf16" and T > 256:
-            return {"frac_alu": round(kalu[n] / counts[n] / t / 1e12 / fp32_alu_peak_tflops(peaks), 4)}
-        if n in kbytes:
-            return {"frac_hbm": round(kbytes[n] / counts[n] / t / 1e9 / hbm, 4)}
-        return {}
-
-    sb = [step_bytes(stats[i % n_batches], src, esz)["bytes"] for i in range(args.steps)]
-    step_gbs = sum(sb) / (ms * 1e-3) / 1e9
-    amort = np.mean([st["T"] * st["k"] / max(1, st["R_anchor"]) for st in stats])
+    tabs = kernel_tables(per_copy, args.steps, n_copies, stats, src)
+    roof, kernels, step, amort, launches = roofline_summary(
+        src, T, ms, args.steps, stats, tabs, peaks, peak_kind, args.workload)
+    config = workload_config(src, T, desc)
+    config.update({"layer_copies": n_copies, "parallelism": f"replica per GPU x{world}",
+                   "timing": ("one CUDA graph of the K forwards (kernel durations from a "
+                              "second, event-instrumented graph of the same forwards)")
+                             if not args.no_graph else "K forwards launched one by one"})
     line = {
         "metric": METRIC, "value": round(whole_job_rate(T, args.steps, world, ms), 1),
         "unit": "tokens/s",
@@ -478,22 +542,11 @@ def run_lx(args, rank, world, local_rank):
         "ms_per_step": round(ms / args.steps, 5), "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16" if src.dtype == "bf16" else "f32",
         "data": "synthetic (seeded Gaussian weights and tokens, Zipf-skewed cluster-correlated router)",
-        "config": {"workload": desc, "d_model": src.d_model, "d_ff": src.d_ff,
-                   "n_experts": src.n_experts, "top_k": k, "n_nodes": src.n_nodes,
-                   "tokens_per_step": T, "layer_bytes": wbytes, "layer_copies": n_copies,
-                   "l2": f"{n_copies} rotating device copies of the layer and 8 token batches "
-                         "(inputs larger than L2)",
-                   "parallelism": f"replica per GPU x{world}",
-                   "timing": ("one CUDA graph of the K forwards (kernel durations from a "
-                              "second, event-instrumented graph of the same forwards)")
-                             if graph is not None else "K forwards launched one by one"},
+        "config": config,
         "roofline": roof,
-        "kernels": {n: {"launches": counts[n], "avg_us": round(totals[n] / counts[n] * 1e3, 2),
-                        "share": round(totals[n] / sum(totals.values()), 4),
-                        **kernel_frac(n)} for n in totals},
-        "step_roofline": {"algorithmic_bytes_per_step": round(float(np.mean(sb))),
-                          "achieved_gbs": round(step_gbs, 1), "frac": round(step_gbs / hbm, 4)},
-        "amortisation": round(float(amort), 3),
+        "kernels": kernels,
+        "step_roofline": step,
+        "amortisation": amort,
         "e2e": {"value": round(whole_job_rate(T, k_e2e, world, ms_e2e), 1), "unit": "tokens/s",
                 "steps": k_e2e, "h2d_bytes_per_step": int(xs[0].numel() * xs[0].element_size()),
                 "d2h_bytes_per_step": int(ys[0].numel() * ys[0].element_size())},
@@ -501,9 +554,57 @@ def run_lx(args, rank, world, local_rank):
         "clocks": clk,
         "impl": "lx",
     }
+    if per_config is not None:
+        line["per_config"] = per_config
     if world == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(src, xs_host, T, args.cpu_seconds)
+        line["cpu_baseline"] = cpu_baseline(src, xs_host, T, args.cpu_seconds, n_tokens=8)
     return line
+
+
+# the other workloads reported beside the headline (name, layer kind, T, steps)
+PER_CONFIG = [("decode1", 20), ("decode8", 20), ("decode32", 20), ("prefill", 10),
+              ("high_e", 10), ("tree", 10)]
+
+
+def run_per_config(args, rank, dev, qwen_src, qwen_layers, clocks, peaks, peak_kind):
+    """Each of the metric's other workloads: tokens/s, the step roofline, the
+    dominant kernel's roofline, the amortisation and a bounded oracle baseline.
+    The Qwen-shaped layer copies of the headline are reused."""
+    import torch
+    out = {}
+    made = {"qwen": qwen_src}
+    for name, steps in PER_CONFIG:
+        kind, T, desc = WORKLOADS[name]
+        t_start = time.time()
+        if kind not in made:
+            made[kind] = make_layer(kind)
+        src = made[kind]
+        reuse = qwen_layers if kind == "qwen" else None
+        layers, xs_host, xs, ys = setup_workload(src, T, len(reuse) if reuse else 1, rank, dev,
+                                                 layers=reuse)
+        stats = batch_stats(src, layers[0], xs, ys, T)
+        ms, per_copy = time_steps(layers, xs, ys, src.top_k, steps, 3, 1, clocks,
+                                  graph=not args.no_graph)
+        tabs = kernel_tables(per_copy, steps, len(layers), stats, src)
+        roof, kernels, step, amort, launches = roofline_summary(
+            src, T, ms, steps, stats, tabs, peaks, peak_kind, name)
+        entry = {"workload": desc, "tokens_per_step": T, "steps": steps, "warmup": 3,
+                 "value": round(whole_job_rate(T, steps, 1, ms), 1), "unit": "tokens/s",
+                 "ms_per_step": round(ms / steps, 5), "layer_copies": len(layers),
+                 "step_roofline": step, "roofline": roof, "amortisation": amort,
+                 "gpu_launches": launches,
+                 "kernels": {n: v for n, v in kernels.items() if v["share"] >= 0.02}}
+        if not args.no_cpu_baseline:
+            entry["cpu_baseline"] = cpu_baseline(src, xs_host, T, args.cfg_cpu_seconds,
+                                                 n_tokens=8 if T <= 8 else 4, n_batches=2)
+        entry["wall_s"] = round(time.time() - t_start, 1)
+        out[name] = entry
+        if reuse is None:
+            for L in layers:
+                L.free()
+        del xs, ys
+        torch.cuda.empty_cache()
+    return out
 
 
 def _event_ms(fn, steps, warmup, world=1):
@@ -730,23 +831,40 @@ def run_offline(args, rank, world, local_rank):
     return line if rank == 0 else None
 
 
-def cpu_baseline(src, xs_host, T, budget_s):
-    """The oracle, as it stands, on a bounded sample of the same workload."""
+_RECON = {}   # id(layer) -> {expert: reconstructed float64 weights}
+
+
+def cpu_baseline(src, xs_host, T, budget_s, n_tokens=8, n_batches=8):
+    """The oracle, as it stands, on a bounded sample of the same workload:
+    routing plus the standard MoE forward of the first `n_tokens` tokens of
+    `n_batches` batches, from experts reconstructed beforehand (the
+    reconstruction is timed separately, and shared by the workloads of one layer)."""
     import oracle
-    done, t0 = 0, time.time()
-    b = 0
-    n = min(T, 64)
+    n = min(T, n_tokens)
+    samples = [x[:n] for x in xs_host[:n_batches]]
+    t0 = time.time()
+    ids = np.unique(np.concatenate([oracle.route(src, x)[0].ravel() for x in samples]))
+    cache = _RECON.setdefault(id(src), {})
+    missing = [int(e) for e in ids if int(e) not in cache]
+    cache.update(oracle.reconstruct(src, missing) if missing else {})
+    experts = {int(e): cache[int(e)] for e in ids}
+    recon_s = time.time() - t0
+    done, b, t0 = 0, 0, time.time()
     while True:
-        oracle.moe_forward(src, xs_host[b % len(xs_host)][:n])
+        oracle.moe_forward(src, samples[b % len(samples)], experts=experts)
         done += n
         b += 1
-        if time.time() - t0 > budget_s or b >= 4 * len(xs_host):
+        if time.time() - t0 > budget_s or b >= 8 * len(samples):
             break
     el = time.time() - t0
     return {"value": round(done / el, 3), "unit": "tokens/s", "cores": os.cpu_count(),
             "kind": "oracle", "seconds": round(el, 2),
-            "sample": f"{b} batch(es) of {n} tokens of the same workload (routing, fp64 "
-                      "reconstruction of every selected expert, standard MoE forward)"}
+            "reconstruction_s": round(recon_s, 2),
+            "sample": f"{b} batch(es) of the first {n} tokens of the workload's batches: "
+                      "canonical-fp32 routing and the float64 standard MoE forward, timed; "
+                      f"the float64 reconstruction of the {len(experts)} experts they select "
+                      "is done beforehand (reconstruction_s: the part not already done for "
+                      "an earlier workload of the same layer)"}
 
 
 # ----------------------------------------------------------------------------
@@ -755,25 +873,31 @@ def cpu_baseline(src, xs_host, T, budget_s):
 def run_reference(args, rank, world):
     if rank != 0:
         return None
+    import oracle
     import synth
     kind, T, desc = WORKLOADS[args.workload]
     src = make_layer(kind)
     n = min(T, args.ref_tokens)
     xs = [synth.tokens(src, T, seed=b)[:n] for b in range(4)]
-    import oracle
+    ids = np.concatenate([oracle.route(src, x)[0].ravel() for x in xs])
+    t0 = time.time()
+    experts = oracle.reconstruct(src, ids)
+    recon_s = time.time() - t0
     for i in range(args.warmup):
-        oracle.moe_forward(src, xs[i % 4])
+        oracle.moe_forward(src, xs[i % 4], experts=experts)
     t0 = time.time()
     for i in range(args.steps):
-        oracle.moe_forward(src, xs[i % 4])
+        oracle.moe_forward(src, xs[i % 4], experts=experts)
     el = time.time() - t0
     v = n * args.steps / el
-    sample = f"{n} of the {T} tokens of each step's batch"
+    sample = (f"{n} of the {T} tokens of each step's batch: canonical-fp32 routing and the "
+              f"float64 standard MoE forward, from the {len(experts)} experts the samples "
+              f"select, reconstructed beforehand in {recon_s:.1f} s")
     return {"metric": METRIC, "value": round(v, 3), "unit": "tokens/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": round(el / args.steps * 1e3, 3), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": desc, "tokens_per_step": T},
+            "config": workload_config(src, T, desc),
             "impl": "reference",
             "cpu_baseline": {"value": round(v, 3), "unit": "tokens/s", "cores": os.cpu_count(),
                              "kind": "oracle", "sample": sample},
@@ -789,7 +913,11 @@ def main():
     ap.add_argument("--workload", default="decode64", choices=sorted(WORKLOADS) + sorted(OFFLINE))
     ap.add_argument("--impl", default="lx", choices=["lx", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--cfg-cpu-seconds", type=float, default=3.0,
+                    help="oracle seconds per workload of per_config")
+    ap.add_argument("--no-per-config", action="store_true",
+                    help="report the headline workload only")
     ap.add_argument("--ref-tokens", type=int, default=8)
     ap.add_argument("--no-graph", action="store_true",
                     help="launch the timed steps one by one instead of as one CUDA graph")

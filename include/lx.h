@@ -21,7 +21,7 @@
  * single shared base (Sec. 5.2's single-shared-component layout) is one anchor
  * that is no expert, with every expert a correction below it.
  *
- * The forward (Sec. 5.1, "computed once per token and broadcast") routes every
+ * The forward (Sec. 5.1: each shared product evaluated once per token) routes every
  * token top-k over all E experts with the unchanged router (Sec. 1, Fig. 1),
  * evaluates each anchor's product once per (token, anchor) and each correction
  * once per (token, node), applies SwiGLU per selected expert and combines
@@ -145,8 +145,10 @@ LX_API lx_status lx_bucket(lx_layer* layer, const int32_t* topk_id, int32_t T, i
                     void* stream);
 
 /*
- * The compressed-MoE forward: route, bucket, shared anchor GEMMs with the
- * low-rank corrections and SwiGLU, down-projection and weighted combine.
+ * The compressed-MoE forward (Sec. 5.1: a dominant's or ancestor's product is
+ * evaluated one time per token and reused by every selected expert below it;
+ * Sec. 3.1: a member's projection is W_dom + B_m A_m, never re-materialised): route, bucket, shared anchor GEMMs with the low-rank
+ * corrections and SwiGLU, down-projection and weighted combine.
  *   x: device [T][H], y: device [T][H] (layer dtype), both 16-byte aligned;
  *   y may not overlap x.
  * Kernels: bf16 layers whose H, I and ranks are multiples of 64 (with k <= 8,
@@ -165,7 +167,10 @@ LX_API lx_status lx_moe_forward(lx_layer* layer, const void* x, int32_t T, int32
 
 /*
  * Copies the last bucketing (from lx_bucket, lx_route or lx_moe_forward) into
- * caller device buffers (stream-ordered).  With D = info.max_depth:
+ * caller device buffers (stream-ordered).  The buckets are the (token, node)
+ * pairs whose products the forward evaluates once and shares (Sec. 5.1): node
+ * n's bucket holds every token that selected an expert whose root path
+ * contains n.  With D = info.max_depth:
  *   node_off   [n_nodes+1]  exclusive prefix of the node bucket sizes
  *   node_tok   [T*k*D]      capacity; first node_off[n_nodes] entries written:
  *                           node n's tokens ascending, nodes in id order
@@ -215,6 +220,37 @@ LX_API lx_status lx_set_profiling(lx_layer* layer, int32_t enable);
 LX_API lx_status lx_read_profile(lx_layer* layer, lx_kernel_time* out, int32_t cap, int32_t* n);
 
 /*
+ * Bounded device-side waits.  The kernels wait in two places: the weight
+ * streaming kernels (T <= 256) wait inside a launch for the rows another tile
+ * of the same launch writes (a factor product U after its x V), and every
+ * kernel with a TMA/tensor-core pipeline waits on shared-memory barriers.
+ * Each wait gives up after a bound, records LX_ERR_TIMEOUT in the layer's
+ * device error word (lx_layer_info's device_error), makes the CTA's other
+ * roles stop, lets the CTA's copies and tensor-core operations in flight
+ * finish and frees its tensor memory; the launch then ends normally, so the
+ * CUDA context stays usable, and that forward's output is undefined.
+ *
+ * lx_set_wait_limit: the bound in SM clock cycles of every later wait of the
+ * layer's kernels (0 restores the default, 4e9 cycles, about 2 s at the GB300's
+ * clock).  Copies that are already in flight are always waited for with the
+ * default bound.  Errors: LX_ERR_ARG (NULL layer).
+ *
+ * lx_inject_unmet_wait (test hook): from the next forward on, the wait at
+ * `site` waits for a condition that nothing fulfils -- LX_WAIT_STREAM_DEP: one
+ * arrival more than the streaming producer tiles make; LX_WAIT_TC_MMA: a
+ * barrier that only the abort path arrives on, before the tensor-core MMA
+ * issuer's first tile -- so that it runs out after the bound.  LX_WAIT_NONE
+ * turns the hook off.  Errors: LX_ERR_ARG (NULL layer, unknown site).
+ *
+ * lx_clear_device_error: zeroes the device error word (stream-ordered on the
+ * legacy default stream; synchronises the device).  Errors: LX_ERR_ARG.
+ */
+typedef enum { LX_WAIT_NONE = 0, LX_WAIT_STREAM_DEP = 1, LX_WAIT_TC_MMA = 2 } lx_wait_site;
+LX_API lx_status lx_set_wait_limit(lx_layer* layer, uint64_t cycles);
+LX_API lx_status lx_inject_unmet_wait(lx_layer* layer, int32_t site);
+LX_API lx_status lx_clear_device_error(lx_layer* layer);
+
+/*
  * Size of the fixed device array that lx_bucket_noalloc uses as scratch.  The
  * array is a static device variable of the library, so every GPU on which the
  * library's code is loaded holds these bytes until the process exits.
@@ -240,10 +276,13 @@ LX_API lx_status lx_read_profile(lx_layer* layer, lx_kernel_time* out, int32_t c
  *   expert_off [E+1], perm [T*k].
  * Must be called with the layer's device current.  The first call on a device
  * looks up the array's device address (cudaGetSymbolAddress) and caches it;
- * make that first call before any stream capture.  The call needs
- * 5*(n_nodes+E)*round_up(T,16) + 4*T*k*D bytes (plus small tables, each part
- * rounded up to 256 bytes) of the array and returns LX_ERR_SHAPE, launching
- * nothing, when that exceeds LX_NOALLOC_SCRATCH_BYTES.
+ * make that first call before any stream capture.  With keys = n_nodes + E
+ * and Tp = round_up(T, 16), the call needs
+ *   r(keys*Tp) + r(4*keys*Tp) + r(4*keys) + r(4*(keys+2)) + r(4*T*k*D)
+ * bytes of the array, r(v) = v rounded up to 256, and returns LX_ERR_SHAPE,
+ * launching nothing, when that exceeds LX_NOALLOC_SCRATCH_BYTES (the
+ * Qwen3-30B-A3B-shaped layer, keys = 256, k = 8, D = 2: T <= 12480).
+ * T == 0 writes zeros to node_off and expert_off (if not NULL) and nothing else.
  * All calls in the process share the one array per device and the array keeps
  * the previous call's contents (the call clears what must start at zero):
  * calls whose GPU work can overlap (different streams, or different layers on

@@ -16,7 +16,7 @@ except the router logits, see below):
    ``s_n`` in {+1, -1} the label of the edge into n (Fig. 2; +1 when the layer
    carries no signs).
 2. Routing (Sec. 1 and Fig. 1: top-k over all E experts by the unchanged
-   router; Sec. 5.2 "top-k routing").  Logits ``l = x W_r^T (+ b)`` in the
+   router; Sec. 5.2 names the routing top-k).  Logits ``l = x W_r^T (+ b)`` in the
    canonical fp32 order of ``router_canonical.c``; top-k by (logit descending,
    expert id ascending); gates = softmax over the k selected logits (float64).
 3. The standard MoE forward on the reconstructed experts (Sec. 5.1, the
@@ -24,7 +24,7 @@ except the router logits, see below):
    with expert e = id[t, s] and gate g = gate[t, s],
    ``out[t, s] = g * W_e^down (silu(W_e^gate x_t) * (W_e^up x_t))``,
    ``silu(z) = z / (1 + exp(-z))``, and ``y_t = sum_s out[t, s]`` in slot order.
-4. Bucketing (what "computed once per token and broadcast", Sec. 5.1, needs):
+4. Bucketing (what Sec. 5.1's one evaluation per token of each shared product needs):
    per node n, the ascending list of tokens whose selected experts' root paths
    contain n; per (assignment, path level) the row of that (token, node) pair;
    per expert, its assignments in ascending token order.  Written as plain
@@ -150,12 +150,21 @@ def expert_output(Wg: np.ndarray, Wu: np.ndarray, Wd: np.ndarray, xs: np.ndarray
     return (silu(xs @ Wg.T) * (xs @ Wu.T)) @ Wd.T
 
 
+def reconstruct(layer: CompressedLayer, experts: Sequence[int]) -> Dict[int, tuple]:
+    """{e: expert_weights(layer, e)} for the given experts (step 1 done ahead of
+    the forward, so that a timing of the forward can leave it out)."""
+    return {int(e): expert_weights(layer, int(e)) for e in np.unique(np.asarray(experts))}
+
+
 def moe_forward(layer: CompressedLayer, x: np.ndarray, k: Optional[int] = None,
-                token_subset: Optional[Sequence[int]] = None, routing=None) -> np.ndarray:
+                token_subset: Optional[Sequence[int]] = None, routing=None,
+                experts: Optional[Dict[int, tuple]] = None) -> np.ndarray:
     """y [T, H] float64 (or [len(token_subset), H]).
 
     Routing is decided on all T tokens' canonical logits (only the subset's rows
-    are needed, and routing is per token, so only those rows are routed)."""
+    are needed, and routing is per token, so only those rows are routed).
+    ``experts`` may hold reconstructed weights from ``reconstruct``; an expert
+    missing from it is reconstructed here."""
     k = layer.top_k if k is None else k
     toks = np.arange(x.shape[0]) if token_subset is None else np.asarray(token_subset, np.int64)
     xs = x[toks]
@@ -167,7 +176,10 @@ def moe_forward(layer: CompressedLayer, x: np.ndarray, k: Optional[int] = None,
     n, H = X.shape
     out = np.zeros((n, k, H), np.float64)
     for e in np.unique(ids):
-        Wg, Wu, Wd = expert_weights(layer, int(e))
+        if experts is not None and int(e) in experts:
+            Wg, Wu, Wd = experts[int(e)]
+        else:
+            Wg, Wu, Wd = expert_weights(layer, int(e))
         rows, slots = np.nonzero(ids == e)
         out[rows, slots] = g[rows, slots][:, None] * expert_output(Wg, Wu, Wd, X[rows])
     y = np.zeros((n, H), np.float64)

@@ -6,8 +6,8 @@ TEST INFRASTRUCTURE ONLY (like the rest of ``oracle``): imported by the tests,
 An expert's intermediate neurons have no canonical order, so a member is
 permuted to match its dominant before the residual is decomposed:
 
-* neuron i of an expert is the concatenation of its gate, up and down columns
-  (in the ``x W^T`` storage used here: row i of gate [I, H], row i of up
+* neuron i of an expert is one vector: its gate, up and down weights joined
+  end to end (in the ``x W^T`` storage used here: row i of gate [I, H], row i of up
   [I, H] and column i of down [H, I]), a vector of length 3H;
 * the cost of matching dominant neuron i with member neuron j is the squared
   distance ``C[i, j] = ||a_i - b_j||^2`` (Eq. cost), computed here from the

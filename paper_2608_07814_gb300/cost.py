@@ -7,8 +7,9 @@ Per token and projection, an anchor (a dominant or a tree root) costs ``2*I*H``
 FLOPs and ``I*H`` weight elements; a rank-r correction costs ``2*r*(I+H)``
 FLOPs and ``r*(I+H)`` elements (``x V`` then ``(x V) U^T``).  The amortised
 forward evaluates each anchor once per (token, anchor) and each correction once
-per (token, correction node) -- Sec. 5.1 ("computed once per token and
-broadcast") and the Sec. 5.2 display equation:
+per (token, correction node) -- Sec. 5.1 (a shared product is evaluated one
+time per token and reused by every selected expert below it) and the Sec. 5.2
+display equation:
 
     speedup = k * 2IH / (2IH + k * 2r(I+H))      (gate_proj, k co-selected
                                                   members of one cluster)

@@ -701,6 +701,30 @@ extern "C" lx_status lx_set_path(lx_layer* L, int32_t path) {
   return LX_OK;
 }
 
+extern "C" lx_status lx_set_wait_limit(lx_layer* L, uint64_t cycles) {
+  if (!L) return fail(LX_ERR_ARG, "layer is NULL");
+  L->wait_cycles = cycles;
+  return LX_OK;
+}
+
+extern "C" lx_status lx_inject_unmet_wait(lx_layer* L, int32_t site) {
+  if (!L) return fail(LX_ERR_ARG, "layer is NULL");
+  if (site != LX_WAIT_NONE && site != LX_WAIT_STREAM_DEP && site != LX_WAIT_TC_MMA)
+    return fail(LX_ERR_ARG, "unknown wait site");
+  L->unmet_wait = site;
+  return LX_OK;
+}
+
+extern "C" lx_status lx_clear_device_error(lx_layer* L) {
+  if (!L) return fail(LX_ERR_ARG, "layer is NULL");
+  if (L->ws.base) {
+    LX_CUDA(cudaDeviceSynchronize());
+    LX_CUDA(cudaMemset(L->ws.err, 0, sizeof(int)));
+    LX_CUDA(cudaDeviceSynchronize());
+  }
+  return LX_OK;
+}
+
 extern "C" lx_status lx_set_profiling(lx_layer* L, int32_t enable) {
   if (!L) return fail(LX_ERR_ARG, "layer is NULL");
   L->profiling = enable != 0;

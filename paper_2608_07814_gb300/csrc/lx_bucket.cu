@@ -541,14 +541,21 @@ extern "C" lx_status lx_bucket_noalloc(lx_layer* L, const int32_t* topk_id, int3
   if (!L) return fail(LX_ERR_ARG, "layer is NULL");
   if (T < 0) return fail(LX_ERR_ARG, "T < 0");
   if (k < 1 || k > LX_MAX_K || k > L->E) return fail(LX_ERR_ARG, "k must be in 1..min(E, LX_MAX_K)");
-  if (T == 0) return LX_OK;
+  cudaStream_t s = (cudaStream_t)stream;
+  if (T == 0) {
+    // no assignments: every bucket is empty, so both offset arrays are zero
+    if (node_off) LX_CUDA(cudaMemsetAsync(node_off, 0, sizeof(int) * (L->N + 1), s));
+    if (expert_off) LX_CUDA(cudaMemsetAsync(expert_off, 0, sizeof(int) * (L->E + 1), s));
+    return LX_OK;
+  }
   if (!topk_id || !node_off || !node_tok || !node_row || !expert_off || !perm)
     return fail(LX_ERR_ARG, "NULL topk_id or output pointer");
   int dev = -1;
   LX_CUDA(cudaGetDevice(&dev));
   if (dev != L->device) return fail(LX_ERR_ARG, "the layer's device must be current");
 
-  // carve the scratch: marks, ranks, counts, offsets, row->node, tile plans
+  // carve the scratch: marks, ranks, counts, offsets, row->node (no tile plans:
+  // nothing reads them here)
   const long Tp = ((long)T + 15) / 16 * 16;
   const long keys = (long)L->N + L->E;
   const long D = L->max_depth;
@@ -557,8 +564,7 @@ extern "C" lx_status lx_bucket_noalloc(lx_layer* L, const int32_t* topk_id, int3
   const size_t b_cnt = round256(sizeof(int) * (size_t)keys);
   const size_t b_off = round256(sizeof(int) * (size_t)(keys + 2));
   const size_t b_rown = round256(sizeof(int) * (size_t)T * k * D);
-  const size_t b_tile = round256(sizeof(int) * (size_t)N_OPS * (op_max_items(L) + 1));
-  const size_t need = b_marks + b_rank + b_cnt + b_off + b_rown + b_tile;
+  const size_t need = b_marks + b_rank + b_cnt + b_off + b_rown;
   if (need > (size_t)LX_NOALLOC_SCRATCH_BYTES)
     return fail(LX_ERR_SHAPE, "lx_bucket_noalloc: T=" + std::to_string(T) + " needs " +
                                   std::to_string(need) + " scratch bytes, the fixed array has " +
@@ -571,17 +577,15 @@ extern "C" lx_status lx_bucket_noalloc(lx_layer* L, const int32_t* topk_id, int3
   int* key_cnt = reinterpret_cast<int*>(p += b_rank);
   int* key_off = reinterpret_cast<int*>(p += b_cnt);
   int* row_node = reinterpret_cast<int*>(p += b_off);
-  int* tile_off = reinterpret_cast<int*>(p += b_rown);
 
-  cudaStream_t s = (cudaStream_t)stream;
   LX_CUDA(cudaMemsetAsync(marks, 0, (size_t)keys * Tp, s));  // previous call's marks
   k_mark<<<(T + 255) / 256, 256, 0, s>>>(topk_id, T, k, L->N, L->E, Tp, L->d_paths,
                                          L->d_path_len, marks);
   LX_CUDA(cudaGetLastError());
   k_key_scan<<<(unsigned)keys, SCAN_THREADS, 0, s>>>(marks, T, Tp, rank_in, key_cnt);
   LX_CUDA(cudaGetLastError());
-  const PlanArgs pa = make_plans(L, N_OPS);
-  k_offsets_plan<<<1, 1024, 0, s>>>(key_cnt, L->N, L->E, key_off, L->d_rank, tile_off,
+  const PlanArgs pa = make_plans(L, 0);
+  k_offsets_plan<<<1, 1024, 0, s>>>(key_cnt, L->N, L->E, key_off, L->d_rank, nullptr,
                                     op_max_items(L), pa, nullptr, 0, nullptr, 0, 0, nullptr,
                                     nullptr, nullptr, 0);
   LX_CUDA(cudaGetLastError());

@@ -221,6 +221,8 @@ struct StreamLaunch {
   int early_weights;
   int* ctr;                  // tile counter of this launch (zeroed by the bucketing)
   int* err;                  // device error word (LX_ERR_TIMEOUT on a bounded wait)
+  unsigned long long wait_cycles;  // bound of every wait (SM clock cycles)
+  int unmet_wait;            // lx_wait_site whose wait is made to run out (test hook), 0 = none
 };
 
 // Tensor-core (prefill) grouped GEMM: one op per launch
@@ -243,6 +245,8 @@ struct TcLaunch {
   long rows_cap;             // rows of the output buffer (bounds check)
   int* ctr;                  // dynamic tile counter (zeroed by the bucketing)
   int* err;
+  unsigned long long wait_cycles;  // bound of every wait (SM clock cycles)
+  int unmet_wait;            // lx_wait_site whose wait is made to run out (test hook), 0 = none
 };
 
 // ---------------------------------------------------------------------------
@@ -336,11 +340,19 @@ struct lx_layer {
   int last_T = 0, last_k = 0;       // last bucketing
   bool profiling = false;
   bool pdl = true;                  // programmatic dependent launch between kernels
+  unsigned long long wait_cycles = 0;  // bound of the kernels' device-side waits (0: default)
+  int unmet_wait = 0;               // lx_wait_site made to run out (test hook), 0 = none
   std::vector<lx::ProfRec> prof;
   std::vector<cudaEvent_t> event_pool;
 };
 
 namespace lx {
+
+// Default bound of every device-side wait: about 2 s at the GB300's clock.
+constexpr unsigned long long kDefaultWaitCycles = 4000000000ull;
+inline unsigned long long wait_limit(const lx_layer* L) {
+  return L->wait_cycles ? L->wait_cycles : kDefaultWaitCycles;
+}
 
 // ints of the counter block zeroed by every bucketing
 inline int sctr_ints(const lx_layer* L) { return N_TILE_COUNTERS + 2 * L->N * STREAM_DEP_TB; }

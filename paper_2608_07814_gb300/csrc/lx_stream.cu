@@ -105,27 +105,30 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   return ok != 0;
 }
 
-// Bounded wait: false if the phase did not complete in time or the CTA aborted.
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag) {
+// Bounded wait: false if the phase did not complete within `limit` SM clock
+// cycles or the CTA aborted.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+                                          unsigned long long limit) {
   if (mbar_try_wait(bar, parity)) return true;
   const unsigned long long t0 = clock64();
   while (true) {
     if (mbar_try_wait(bar, parity)) return true;
     if (*abort_flag) return false;
-    if (clock64() - t0 > SW_TIMEOUT_CYCLES) return false;
+    if (clock64() - t0 > limit) return false;
   }
 }
 
 // Bounded wait for an in-launch dependency counter (acquire); false on
 // timeout or when the CTA aborts.
-__device__ __forceinline__ bool dep_wait(const int* p, int need, volatile int* abort_flag) {
+__device__ __forceinline__ bool dep_wait(const int* p, int need, volatile int* abort_flag,
+                                         unsigned long long limit) {
   const unsigned long long t0 = clock64();
   while (true) {
     int v;
     asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
     if (v >= need) return true;
     if (*abort_flag) return false;
-    if (clock64() - t0 > SW_TIMEOUT_CYCLES) return false;
+    if (clock64() - t0 > limit) return false;
     __nanosleep(128);
   }
 }
@@ -263,7 +266,7 @@ __device__ __forceinline__ bool consume_tile(const StreamLaunch& P, const TileIn
         for (int c = 0; c < 4; ++c) acc[i][j][c] = 0.f;
     for (int kb = 0; kb < nkb; ++kb, ++it) {
       const uint32_t s = it % SW_STAGES;
-      if (!mbar_wait(full0 + 8 * s, (it / SW_STAGES) & 1, abort_flag)) return false;
+      if (!mbar_wait(full0 + 8 * s, (it / SW_STAGES) & 1, abort_flag, P.wait_cycles)) return false;
       const uint32_t wbox = smem_base + s * SW_STAGE_BYTES;
       const uint32_t xbox = wbox + SW_BOX_BYTES;
 #pragma unroll
@@ -455,8 +458,12 @@ k_stream_gemm(const __grid_constant__ StreamLaunch P) {
           // halves), then order the async-proxy row loads after the acquire
           int good = 1;
           if (lane == 0) {
-            const int need = SW_CONSUMERS * ((op.dep_nrank * ti.K + SW_ROWS - 1) / SW_ROWS);
-            good = dep_wait(op.dep + ti.node * STREAM_DEP_TB + ti.tb, need, abort_flag) ? 1 : 0;
+            // (an injected unmet wait asks for one arrival more than the
+            // producer tiles ever make, so that the bounded wait runs out)
+            const int need = SW_CONSUMERS * ((op.dep_nrank * ti.K + SW_ROWS - 1) / SW_ROWS) +
+                             (P.unmet_wait == LX_WAIT_STREAM_DEP ? 1 : 0);
+            good = dep_wait(op.dep + ti.node * STREAM_DEP_TB + ti.tb, need, abort_flag,
+                            P.wait_cycles) ? 1 : 0;
             asm volatile("fence.proxy.async.global;" ::: "memory");
           }
           good = __shfl_sync(0xffffffffu, good, 0);
@@ -473,7 +480,8 @@ k_stream_gemm(const __grid_constant__ StreamLaunch P) {
             int good = 1;
             const bool pre = it < npre;  // weight box issued before the dependency wait
             if (lane == 0 && !pre) {
-              good = mbar_wait(empty0 + 8 * s, ((it / SW_STAGES) & 1) ^ 1, abort_flag) ? 1 : 0;
+              good = mbar_wait(empty0 + 8 * s, ((it / SW_STAGES) & 1) ^ 1, abort_flag,
+                               P.wait_cycles) ? 1 : 0;
               if (good) {
                 if (cb == 0 && kb == 0) slot[s] = ti;
                 mbar_expect_tx(full0 + 8 * s, SW_BOX_BYTES + (op.gather ? 0 : SW_XBYTES));
@@ -536,7 +544,8 @@ k_stream_gemm(const __grid_constant__ StreamLaunch P) {
       const uint32_t s = it % SW_STAGES;
       int good = 1;
       if (lane == 0) {
-        good = mbar_wait(empty0 + 8 * s, ((it / SW_STAGES) & 1) ^ 1, abort_flag) ? 1 : 0;
+        good = mbar_wait(empty0 + 8 * s, ((it / SW_STAGES) & 1) ^ 1, abort_flag, P.wait_cycles)
+                   ? 1 : 0;
         if (good) {
           slot[s].op = -1;
           mbar_arrive(full0 + 8 * s);
@@ -553,18 +562,19 @@ k_stream_gemm(const __grid_constant__ StreamLaunch P) {
     if (!ok && lane == 0) {
       atomicExch(P.err, LX_ERR_TIMEOUT);
       *abort_flag = 1;
-      // drain: every issued stage's copies must land before the CTA exits
+      // drain: every issued stage's copies must land before the CTA exits (the
+      // copies were issued, so these waits end; they keep the full bound)
       const uint32_t first = it > SW_STAGES ? it - SW_STAGES : 0;
       volatile int never = 0;
       for (uint32_t j = first; j < it; ++j)
-        mbar_wait(full0 + 8 * (j % SW_STAGES), (j / SW_STAGES) & 1, &never);
+        mbar_wait(full0 + 8 * (j % SW_STAGES), (j / SW_STAGES) & 1, &never, SW_TIMEOUT_CYCLES);
     }
     return;
   }
   // ---- consumers: the first stage of every tile carries its description
   while (true) {
     const uint32_t s = it % SW_STAGES;
-    if (!mbar_wait(full0 + 8 * s, (it / SW_STAGES) & 1, abort_flag)) {
+    if (!mbar_wait(full0 + 8 * s, (it / SW_STAGES) & 1, abort_flag, P.wait_cycles)) {
       if (lane == 0) {
         atomicExch(P.err, LX_ERR_TIMEOUT);
         *abort_flag = 1;
@@ -679,6 +689,8 @@ static lx_status run_stream(lx_layer* L, int g, std::initializer_list<const Stre
   if (P.n_ops == 0) return LX_OK;
   P.ctr = L->ws.sctr + g;
   P.err = L->ws.err;
+  P.wait_cycles = wait_limit(L);
+  P.unmet_wait = L->unmet_wait;
   // the z-side launch follows the SwiGLU kernel, whose output only its token
   // rows read
   P.early_weights = g == 2 ? 1 : 0;

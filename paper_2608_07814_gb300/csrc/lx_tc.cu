@@ -76,14 +76,15 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
-// bounded wait; false on timeout or when the CTA aborts
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag) {
+// bounded wait; false after `limit` SM clock cycles or when the CTA aborts
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+                                          unsigned long long limit = TC_TIMEOUT_CYCLES) {
   if (mbar_try_wait(bar, parity)) return true;
   const unsigned long long t0 = clock64();
   while (true) {
     if (mbar_try_wait(bar, parity)) return true;
     if (abort_flag && *abort_flag) return false;
-    if (clock64() - t0 > TC_TIMEOUT_CYCLES) return false;
+    if (clock64() - t0 > limit) return false;
   }
 }
 
@@ -305,7 +306,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
         const uint32_t s = it % TC_STAGES;
         int good = 1;
         if (lane == 0) {
-          good = mbar_wait(empty0 + 8 * s, ((it / TC_STAGES) & 1) ^ 1, abort_flag) ? 1 : 0;
+          good = mbar_wait(empty0 + 8 * s, ((it / TC_STAGES) & 1) ^ 1, abort_flag,
+                           P.wait_cycles) ? 1 : 0;
           if (good) {
             if (kb == 0) slot[s] = t;
             mbar_expect_tx(full0 + 8 * s, nbox * 8192 + (P.gather ? 0 : TC_A_BYTES));
@@ -375,7 +377,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
       const uint32_t s = it % TC_STAGES;
       int good = 1;
       if (lane == 0) {
-        good = mbar_wait(empty0 + 8 * s, ((it / TC_STAGES) & 1) ^ 1, abort_flag) ? 1 : 0;
+        good = mbar_wait(empty0 + 8 * s, ((it / TC_STAGES) & 1) ^ 1, abort_flag, P.wait_cycles)
+                   ? 1 : 0;
         if (good) {
           slot[s].BN = -1;
           mbar_arrive(full0 + 8 * s);
@@ -399,13 +402,23 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
     if (lane == 0) {
       uint32_t it = 0, tiles = 0;
       bool ok = true;
+      // An injected unmet wait: the drain barrier gets no arrival before the
+      // abort path, so this bounded wait runs out and the CTA takes that path.
+      if (P.unmet_wait == LX_WAIT_TC_MMA && !mbar_wait(drain, 0, abort_flag, P.wait_cycles))
+        ok = false;
       while (ok) {
         const uint32_t s = it % TC_STAGES;
-        if (!mbar_wait(full0 + 8 * s, (it / TC_STAGES) & 1, abort_flag)) { ok = false; break; }
+        if (!mbar_wait(full0 + 8 * s, (it / TC_STAGES) & 1, abort_flag, P.wait_cycles)) {
+          ok = false;
+          break;
+        }
         const TcTile t = slot[s];
         const uint32_t b = tiles & 1;
         // this accumulator must have been drained by the epilogue (two tiles ago)
-        if (!mbar_wait(tempty0 + 8 * b, ((tiles >> 1) & 1) ^ 1, abort_flag)) { ok = false; break; }
+        if (!mbar_wait(tempty0 + 8 * b, ((tiles >> 1) & 1) ^ 1, abort_flag, P.wait_cycles)) {
+          ok = false;
+          break;
+        }
         eslot[b] = t;  // tile info for the epilogue, released by this arrival
         mbar_arrive(tfull0 + 8 * b);
         if (t.BN < 0) {  // sentinel: the second arrival completes the phase
@@ -419,7 +432,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
         const int nkb = (t.K + TC_BK - 1) / TC_BK;
         for (int kb = 0; kb < nkb; ++kb, ++it) {
           const uint32_t s2 = it % TC_STAGES;
-          if (!mbar_wait(full0 + 8 * s2, (it / TC_STAGES) & 1, abort_flag)) { ok = false; break; }
+          if (!mbar_wait(full0 + 8 * s2, (it / TC_STAGES) & 1, abort_flag, P.wait_cycles)) {
+            ok = false;
+            break;
+          }
           tc_fence_after();
           const uint32_t a_s = smem_base + s2 * TC_STAGE_BYTES, b_s = a_s + TC_A_BYTES;
 #pragma unroll
@@ -447,7 +463,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
     uint32_t tiles = 0;
     while (true) {
       const uint32_t b = tiles & 1;
-      if (!mbar_wait(tfull0 + 8 * b, (tiles >> 1) & 1, abort_flag)) {
+      if (!mbar_wait(tfull0 + 8 * b, (tiles >> 1) & 1, abort_flag, P.wait_cycles)) {
         if (lane == 0) {
           atomicExch(P.err, LX_ERR_TIMEOUT);
           *abort_flag = 1;
@@ -584,6 +600,8 @@ static TcLaunch tc_op(lx_layer* L, int op, const __nv_bfloat16* X, long ldx, con
   P.out_f32 = out_f32 ? 1 : 0;
   P.ctr = w.sctr + N_STREAM_GROUPS + counter;
   P.err = w.err;
+  P.wait_cycles = wait_limit(L);
+  P.unmet_wait = L->unmet_wait;
   P.rows_cap = w.rows_cap;
   return P;
 }

@@ -30,8 +30,10 @@ EXPORTS = [
     "lx_moe_forward", "lx_get_buckets", "lx_layer_info", "lx_set_path", "lx_set_profiling",
     "lx_read_profile", "lx_last_error", "lx_bucket_noalloc", "lx_coact_accumulate",
     "lx_coact_npmi", "lx_align_cost", "lx_lap_solve", "lx_lap_solve_batch", "lx_permute_neurons",
-    "lx_compress_workspace", "lx_compress_factor",
+    "lx_compress_workspace", "lx_compress_factor", "lx_set_wait_limit", "lx_inject_unmet_wait",
+    "lx_clear_device_error",
 ]
+LX_WAIT_NONE, LX_WAIT_STREAM_DEP, LX_WAIT_TC_MMA = 0, 1, 2
 LX_NOALLOC_SCRATCH_BYTES = 16 << 20
 
 
@@ -86,6 +88,9 @@ def lib() -> ctypes.CDLL:
             "lx_layer_info": [vp, ctypes.POINTER(LayerInfo)],
             "lx_set_path": [vp, i32],
             "lx_set_profiling": [vp, i32],
+            "lx_set_wait_limit": [vp, ctypes.c_uint64],
+            "lx_inject_unmet_wait": [vp, i32],
+            "lx_clear_device_error": [vp],
             "lx_read_profile": [vp, ctypes.POINTER(KernelTime), i32, ctypes.POINTER(i32)],
             "lx_bucket_noalloc": [vp, vp, i32, i32, vp, vp, vp, vp, vp, vp],
             "lx_coact_accumulate": [vp, i32, i32, i32, vp, vp, vp],
@@ -203,6 +208,17 @@ class Layer:
 
     def reserve(self, max_tokens: int, k: int) -> None:
         _check(lib().lx_reserve(self.handle, max_tokens, k))
+
+    def set_wait_limit(self, cycles: int) -> None:
+        """Bound (SM clock cycles) of the kernels' device-side waits; 0 = default."""
+        _check(lib().lx_set_wait_limit(self.handle, int(cycles)))
+
+    def inject_unmet_wait(self, site: int) -> None:
+        """Test hook: make the wait at `site` (LX_WAIT_*) run out."""
+        _check(lib().lx_inject_unmet_wait(self.handle, int(site)))
+
+    def clear_device_error(self) -> None:
+        _check(lib().lx_clear_device_error(self.handle))
 
     def set_path(self, path: int) -> None:
         _check(lib().lx_set_path(self.handle, path))

@@ -67,10 +67,15 @@ CORR_SLOTS = ("Ug", "Vg", "Uu", "Vu", "Ud", "Vd")
 def bf16_bits(a: np.ndarray) -> np.ndarray:
     """Round float32 values to bfloat16 (round-to-nearest-even); return uint16 bits."""
     a = np.ascontiguousarray(a, dtype=np.float32)
-    u = a.view(np.uint32).astype(np.uint64)
-    lsb = (u >> 16) & 1
-    r = ((u + 0x7FFF + lsb) >> 16).astype(np.uint16)
-    return r
+    u = a.view(np.uint32)
+    # in uint32 (no overflow for any finite or infinite value): t = (u + 0x7FFF
+    # + lsb) >> 16, lsb the lowest kept bit, in place to keep it to a few passes
+    t = u >> 16
+    t &= 1
+    t += u
+    t += np.uint32(0x7FFF)
+    t >>= 16
+    return t.astype(np.uint16)
 
 
 def bf16_to_f32(b: np.ndarray) -> np.ndarray:
@@ -177,6 +182,13 @@ def _zipf_bias(rng, E: int, groups: Sequence[Sequence[int]], s: float, beta: flo
     return b.astype(np.float32)
 
 
+def _n_dead(n_dead: int, n_candidates: int) -> int:
+    """Dead experts of a skewed router: the calibrated count (25 of the 96
+    members of E = 128, Table 3), but at most a third of the candidates, so
+    that a small test layer keeps members the router can select."""
+    return min(n_dead, n_candidates // 3)
+
+
 def _factor_std(rank: int, factor_std) -> float:
     if factor_std is None:
         return 0.02 / np.sqrt(rank)            # "N(0, 0.02/sqrt(r))" read as std
@@ -243,7 +255,7 @@ def flat_layer(H: int, I: int, cluster_sizes: Sequence[int], rank, top_k: int,
         s, beta, rho, n_dead = skew
         Wr = _router(rng, E, H, groups, rho)
         members = [e for g in groups for e in g[1:]]
-        dead = rng.choice(members, size=min(n_dead, len(members)), replace=False) if n_dead else []
+        dead = rng.choice(members, size=_n_dead(n_dead, len(members)), replace=False) if n_dead else []
         bias = _zipf_bias(rng, E, groups, s, beta, dead)
     return CompressedLayer(
         d_model=H, d_ff=I, n_experts=E, dtype=dtype,
@@ -304,7 +316,7 @@ def tree_layer(H: int, I: int, n_roots: int, subs_per_root: int, leaves_per_sub:
         s, beta, rho, n_dead = skew
         Wr = _router(rng, E, H, sub_groups, rho * 0.5, outer=root_groups, rho_outer=rho * 0.45)
         leaves = [e for g in sub_groups for e in g[1:]]
-        dead = rng.choice(leaves, size=min(n_dead, len(leaves)), replace=False) if n_dead else []
+        dead = rng.choice(leaves, size=_n_dead(n_dead, len(leaves)), replace=False) if n_dead else []
         bias = _zipf_bias(rng, E, sub_groups, s, beta, dead)
     return CompressedLayer(
         d_model=H, d_ff=I, n_experts=E, dtype=dtype,
@@ -373,7 +385,7 @@ def binary_tree_layer(H: int, I: int, n_roots: int, levels: int, ranks: Sequence
         s, beta, rho, n_dead = skew
         Wr = _router(rng, E, H, pair_groups, rho * 0.5, outer=root_groups, rho_outer=rho * 0.45)
         cand = [e for g in pair_groups for e in g[1:]]
-        dead = rng.choice(cand, size=min(n_dead, len(cand)), replace=False) if n_dead else []
+        dead = rng.choice(cand, size=_n_dead(n_dead, len(cand)), replace=False) if n_dead else []
         bias = _zipf_bias(rng, E, pair_groups, s, beta, dead)
     return CompressedLayer(
         d_model=H, d_ff=I, n_experts=E, dtype=dtype,
@@ -415,7 +427,7 @@ def single_base_layer(H: int, I: int, E: int, rank, top_k: int, dtype: str = "bf
         s, beta, rho, n_dead = skew
         Wr = _router(rng, E, H, groups, rho)
         cand = [e for g in groups for e in g[1:]]
-        dead = rng.choice(cand, size=min(n_dead, len(cand)), replace=False) if n_dead else []
+        dead = rng.choice(cand, size=_n_dead(n_dead, len(cand)), replace=False) if n_dead else []
         bias = _zipf_bias(rng, E, groups, s, beta, dead)
     return CompressedLayer(
         d_model=H, d_ff=I, n_experts=E, dtype=dtype,

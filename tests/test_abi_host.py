@@ -152,3 +152,9 @@ def test_layer_desc_struct_matches_header():
     body = re.sub(r"/\*.*?\*/", "", body, flags=re.S)
     fields = re.findall(r"\b(\w+)\s*;", body)
     assert fields == [f for f, _ in lx.LayerDesc._fields_]
+
+
+def test_wait_hooks_reject_bad_arguments(L):
+    assert L.lx_set_wait_limit(None, 1000) == lx.LX_ERR_ARG
+    assert L.lx_inject_unmet_wait(None, lx.LX_WAIT_STREAM_DEP) == lx.LX_ERR_ARG
+    assert L.lx_clear_device_error(None) == lx.LX_ERR_ARG

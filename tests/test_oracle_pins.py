@@ -475,3 +475,16 @@ def test_planted_mistakes_fail_a_pin(monkeypatch, target, mutant):
     oracle.__dict__["_orig_correction"] = oracle._correction
     monkeypatch.setattr(oracle, target, mutant)
     assert not _pins_pass()
+
+
+def test_forward_from_reconstructed_experts_is_the_same_forward():
+    """moe_forward with experts reconstructed beforehand (the CPU baseline's
+    timing split) gives the identical result: the same weights, the same loop."""
+    src = synth.tiny_layer(seed=4)
+    x = synth.tokens(src, 40, seed=4)
+    ids, _, _ = oracle.route(src, x)
+    y0 = oracle.moe_forward(src, x)
+    part = oracle.reconstruct(src, ids[:, 0])          # some experts only: the rest on demand
+    assert np.array_equal(oracle.moe_forward(src, x, experts=part), y0)
+    full = oracle.reconstruct(src, np.arange(src.n_experts))
+    assert np.array_equal(oracle.moe_forward(src, x, experts=full), y0)

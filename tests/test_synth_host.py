@@ -49,3 +49,20 @@ def test_generators_are_seeded():
     b = synth.binary_tree_layer(64, 32, 1, 2, [8, 8], 2, "bf16", seed=3, signed=True)
     assert all(np.array_equal(x, y) for wa, wb in zip(a.node_w, b.node_w) for x, y in zip(wa, wb))
     assert np.array_equal(a.router_w, b.router_w)
+
+
+def test_small_skewed_layers_route_through_corrections():
+    """The Zipf router's dead experts (25 of 96 members at E = 128) are capped
+    at a third of the members, so that a small layer made with the same skew
+    still selects members: parity on it then exercises the corrections."""
+    import oracle
+    for src in (synth.flat_layer(512, 384, [4] * 8, 64, 8, "bf16", seed=13,
+                                 factor_std="visible", skew=synth.QWEN_SKEW),
+                synth.flat_layer(256, 192, [4, 4, 1, 3], 64, 4, "bf16", seed=1,
+                                 skew=synth.QWEN_SKEW)):
+        ids, _, _ = oracle.route(src, synth.tokens(src, 200, seed=5))
+        via = np.mean([len(src.path(int(e))) > 1 for e in ids.ravel()])
+        assert via > 0.3, via
+    # the full-size layers keep their calibrated dead counts (96 and 224 members)
+    assert synth._n_dead(25, 96) == 25 and synth._n_dead(50, 224) == 50
+    assert synth._n_dead(25, 24) == 8
