@@ -454,11 +454,11 @@ __device__ __forceinline__ void add_cols(Cols<CPL>& a, const Cols<CPL>& b) {
 }
 
 template <typename TH, typename TZ, int D, bool SPLIT, int CPL>
-__global__ void __launch_bounds__(WT_WARPS * 32, 2)
+__global__ void __launch_bounds__(WT_WARPS * 32, (sizeof(TH) == 2 && CPL >= 4 && D <= 2) ? 3 : 2)
 k_swiglu_warp(const float* __restrict__ topk_w, const int* __restrict__ node_row, int T, int k,
               const TH* __restrict__ h, int I, TZ* __restrict__ z, int cols_per_item,
               const SplitParts hs) {
-  extern __shared__ float zsm[];  // bf16 path: [warp][k * D rows][32 lanes * CPL]
+  extern __shared__ float zsm[];  // bf16 path: [warp][k slots][32 lanes * CPL] activations
   __shared__ WarpRows wrs[WT_WARPS];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   WarpRows& wr = wrs[warp];
@@ -488,85 +488,88 @@ k_swiglu_warp(const float* __restrict__ topk_w, const int* __restrict__ node_row
     for (int c = c_begin + CPL * lane; c < c_end; c += 32 * CPL) {
       Cols<CPL> act[WT_SLOTS];
       if constexpr (sizeof(TH) == 2) {
-        // bf16 rows: every load of this column block first (invalid entries
-        // read row 0 and are masked), so that they are all in flight at once
-        RawB<CPL> rg[WT_SLOTS][D], ru[WT_SLOTS][D];
-        bool val[WT_SLOTS][D], anc[WT_SLOTS][D];
+        // bf16 rows, in batches of SG slots: every path-row load of a batch
+        // first (rows past a path's end are not read), so that they are in
+        // flight at once; each slot's act then goes to this lane's slice of
+        // the warp's shared block
+        float* as = zsm + (size_t)warp * k * 32 * CPL;
         constexpr int NS = SPLIT ? LX_STREAM_MAX_SPLIT : 1;
-        Cols<CPL> sg[WT_SLOTS][NS], su[WT_SLOTS][NS];  // the anchor row's split-K partials
+        constexpr int SG = (CPL >= 4 && D >= 2) ? 4 : WT_SLOTS;  // bounds the live registers
 #pragma unroll
-        for (int sl = 0; sl < WT_SLOTS; ++sl) {
-          int ra = 0;
+        for (int s0 = 0; s0 < WT_SLOTS; s0 += SG) {
+          if (s0 >= k) break;
+          RawB<CPL> rg[SG][D], ru[SG][D];
+          bool val[SG][D], anc[SG][D];
+          Cols<CPL> sg[SG][NS], su[SG][NS];  // the anchor row's split-K partials
 #pragma unroll
-          for (int l = 0; l < D; ++l) {
-            const int r = sl < k ? wr.rows[sl * D + l] : -1;
-            const int rn = (sl < k && l + 1 < D) ? wr.rows[sl * D + l + 1] : -1;
-            val[sl][l] = r >= 0;
-            anc[sl][l] = SPLIT && r >= 0 && rn < 0;  // the path's anchor row
-            if (anc[sl][l]) ra = r;
-            const __nv_bfloat16* hp = reinterpret_cast<const __nv_bfloat16*>(h) +
-                                      (size_t)(r >= 0 ? r : 0) * 2 * I + c;
-            rg[sl][l] = ld_raw<CPL>(hp);
-            ru[sl][l] = ld_raw<CPL>(hp + I);
-          }
-          if constexpr (SPLIT) {
-#pragma unroll
-            for (int sp = 0; sp < NS; ++sp) {
-              const float* hp2 =
-                  hs.part + (long)(sp < hs.splits ? sp : 0) * hs.stride + (size_t)ra * 2 * I + c;
-              sg[sl][sp] = ld_cols<CPL>(hp2);
-              su[sl][sp] = ld_cols<CPL>(hp2 + I);
-            }
-          }
-        }
-#pragma unroll
-        for (int sl = 0; sl < WT_SLOTS; ++sl) {
-          Cols<CPL> pg, pu;
-#pragma unroll
-          for (int i = 0; i < CPL; ++i) pg.v[i] = pu.v[i] = 0.f;
-#pragma unroll
-          for (int l = 0; l < D; ++l) {  // path order: the expert's node up to its anchor
-            if (anc[sl][l]) {
-              // anchor row: its split-K partials (not h), in split order
-#pragma unroll
-              for (int sp = 0; sp < NS; ++sp) {
-                if (sp < hs.splits) {
-                  add_cols(pg, sg[sl][sp]);
-                  add_cols(pu, su[sl][sp]);
-                }
-              }
-            } else {
-              add_raw(pg, rg[sl][l], val[sl][l]);
-              add_raw(pu, ru[sl][l], val[sl][l]);
-            }
-          }
-          const float g = sl < k ? wr.g[sl] : 0.f;
-#pragma unroll
-          for (int i = 0; i < CPL; ++i) act[sl].v[i] = g * silu_fast(pg.v[i]) * pu.v[i];
-        }
-        // z: every slot's act into the accumulators of the distinct rows on its
-        // path, slots in ascending order; then each distinct row out once
-        float* zacc = zsm + (size_t)warp * kD * 32 * CPL;
-        for (int d = 0; d < nd; ++d)
-#pragma unroll
-          for (int i = 0; i < CPL; ++i) zacc[(d * 32 + lane) * CPL + i] = 0.f;
-#pragma unroll
-        for (int sl = 0; sl < WT_SLOTS; ++sl) {
-          if (sl < k) {
+          for (int j = 0; j < SG; ++j) {
+            const int sl = s0 + j;
+            int ra = 0;
 #pragma unroll
             for (int l = 0; l < D; ++l) {
-              const int d = wr.lrow[sl * D + l];
-              if (d >= 0) {
+              const int r = sl < k ? wr.rows[sl * D + l] : -1;
+              const int rn = (sl < k && l + 1 < D) ? wr.rows[sl * D + l + 1] : -1;
+              val[j][l] = r >= 0;
+              anc[j][l] = SPLIT && r >= 0 && rn < 0;  // the path's anchor row
+              if (anc[j][l]) ra = r;
+              if (r >= 0 && !anc[j][l]) {
+                const __nv_bfloat16* hp =
+                    reinterpret_cast<const __nv_bfloat16*>(h) + (size_t)r * 2 * I + c;
+                rg[j][l] = ld_raw<CPL>(hp);
+                ru[j][l] = ld_raw<CPL>(hp + I);
+              }
+            }
+            if constexpr (SPLIT) {
 #pragma unroll
-                for (int i = 0; i < CPL; ++i) zacc[(d * 32 + lane) * CPL + i] += act[sl].v[i];
+              for (int sp = 0; sp < NS; ++sp) {
+                const float* hp2 = hs.part + (long)(sp < hs.splits ? sp : 0) * hs.stride +
+                                   (size_t)ra * 2 * I + c;
+                sg[j][sp] = ld_cols<CPL>(hp2);
+                su[j][sp] = ld_cols<CPL>(hp2 + I);
               }
             }
           }
+#pragma unroll
+          for (int j = 0; j < SG; ++j) {
+            const int sl = s0 + j;
+            Cols<CPL> pg, pu;
+#pragma unroll
+            for (int i = 0; i < CPL; ++i) pg.v[i] = pu.v[i] = 0.f;
+#pragma unroll
+            for (int l = 0; l < D; ++l) {  // path order: the expert's node up to its anchor
+              if (anc[j][l]) {
+                // anchor row: its split-K partials (not h), in split order
+#pragma unroll
+                for (int sp = 0; sp < NS; ++sp) {
+                  if (sp < hs.splits) {
+                    add_cols(pg, sg[j][sp]);
+                    add_cols(pu, su[j][sp]);
+                  }
+                }
+              } else {
+                add_raw(pg, rg[j][l], val[j][l]);
+                add_raw(pu, ru[j][l], val[j][l]);
+              }
+            }
+            if (sl < k) {
+              const float g = wr.g[sl];
+#pragma unroll
+              for (int i = 0; i < CPL; ++i)
+                as[(sl * 32 + lane) * CPL + i] = g * silu_fast(pg.v[i]) * pu.v[i];
+            }
+          }
         }
+        // z: every distinct row's z is the sum of the acts of the slots whose
+        // path holds it (the row's slot mask), slots ascending
         for (int d = 0; d < nd; ++d) {
           Cols<CPL> zc;
 #pragma unroll
-          for (int i = 0; i < CPL; ++i) zc.v[i] = zacc[(d * 32 + lane) * CPL + i];
+          for (int i = 0; i < CPL; ++i) zc.v[i] = 0.f;
+          for (unsigned m = wr.dmask[d]; m; m &= m - 1) {
+            const int sl = __ffs(m) - 1;
+#pragma unroll
+            for (int i = 0; i < CPL; ++i) zc.v[i] += as[(sl * 32 + lane) * CPL + i];
+          }
           st_cols<TZ, CPL>(z + (size_t)wr.drow[d] * I + c, zc);
         }
         continue;
@@ -731,7 +734,7 @@ static void launch_swiglu_c(lx_layer* L, int T, int k, const TH* h, TZ* z, cudaS
   Workspace& w = L->ws;
   const int cols = warp_item_cols(L, T, L->I, 32 * CPL);
   const int grid = warp_grid(L, T, L->I, cols);
-  const size_t zs = sizeof(TH) == 2 ? (size_t)WT_WARPS * k * D * 32 * CPL * 4 : 0;
+  const size_t zs = sizeof(TH) == 2 ? (size_t)WT_WARPS * k * 32 * CPL * 4 : 0;
   if (zs > 0) {  // the accumulators plus the static rows may pass the 48 KB default
     static bool done_s[64] = {}, done_n[64] = {};
     if constexpr (CPL == 1) {

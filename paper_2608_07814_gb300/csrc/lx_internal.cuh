@@ -234,10 +234,7 @@ struct TcLaunch {
   const int* node_off;
   const int* rank;
   const CUtensorMap* wmaps;  // [n_nodes] weight tensor maps of the op
-  const __nv_bfloat16* X;    // gathered A rows (with gather), else unused
-  long ldx;
-  const int* gather;         // row -> X row, or null: A from xmap (rows in node-row order)
-  const CUtensorMap* xmap;   // TMA map of the A buffer when gather is null
+  const CUtensorMap* xmap;   // TMA map of the A buffer (rows in node-row order)
   int xcol;                  // column offset of A inside xmap
   void* out;
   long ldo;

@@ -18,8 +18,10 @@
 // Large bf16 batches (k_router_tiled): persistent CTAs walk tiles of 8
 // tokens.  A thread holds the lane partials of 8 tokens x 8 experts for its
 // lane's chunks (64 accumulators), so every widened weight value serves 8
-// tokens and every widened token value 8 experts; the weight chunks (read
-// through L2) are software-pipelined one chunk ahead.  The 32 lane partials are
+// tokens and every widened token value 8 experts; two tokens' partials of one
+// expert advance by one packed fp32x2 FMA (each half rounded once, as fmaf),
+// which halves the FMA instructions of this issue-bound loop; the weight
+// chunks (read through L2) are software-pipelined one chunk ahead.  The 32 lane partials are
 // then combined by a transpose-reduce whose pairs are those of the canonical
 // order (lane l with lane l ^ 16, then ^ 8, ^ 4, ^ 2, ^ 1; IEEE addition is
 // commutative, so each sum is bit-identical), leaving lane l with the logits
@@ -168,6 +170,23 @@ constexpr int RTT_THREADS = 256;   // 8 warps, each on 8-expert groups
 
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+__device__ __forceinline__ uint32_t word_of(const uint4& u, int i) {
+  return i == 0 ? u.x : i == 1 ? u.y : i == 2 ? u.z : u.w;
+}
+
+// (d0, d1) = (a0 * b + d0, a1 * b + d1): two fused multiply-adds, each
+// rounded once (the same result as two fmaf), issued as one packed fp32x2
+// instruction
+__device__ __forceinline__ void fma2_rn(float& d0, float& d1, float a0, float a1, float b) {
+  asm("{\n\t.reg .b64 ra, rb, rc;\n\t"
+      "mov.b64 ra, {%2, %3};\n\t"
+      "mov.b64 rb, {%4, %4};\n\t"
+      "mov.b64 rc, {%0, %1};\n\t"
+      "fma.rn.f32x2 rc, ra, rb, rc;\n\t"
+      "mov.b64 {%0, %1}, rc;\n\t}"
+      : "+f"(d0), "+f"(d1)
+      : "f"(a0), "f"(a1), "f"(b));
+}
 
 // x tile rows [t0, t0 + nt) into shared memory (16-byte cp.async), zeros after
 __device__ __forceinline__ void rtt_load_tile(const __nv_bfloat16* x, int t0, int nt, int H,
@@ -219,11 +238,14 @@ k_router_tiled(const __nv_bfloat16* __restrict__ x, const __nv_bfloat16* __restr
       rtt_load_tile(x, n0, min(RTT_TOK, Ttok - n0), H, buf ? xs0 : xs1);
     }
     for (int g = warp; g < ngroups; g += RTT_THREADS / 32) {
-      float acc[64];  // [token tt][expert ee] partials of this lane
+      // [expert ee][token tt] partials of this lane: a token pair (tt, tt + 1)
+      // of one expert is an adjacent pair, updated by one packed FMA
+      float acc[64];
 #pragma unroll
       for (int a = 0; a < 64; ++a) acc[a] = 0.f;
       // weight chunks are software-pipelined one chunk ahead (raw bf16 in
-      // registers); token words come from shared memory per element pair
+      // registers); each token's chunk comes from shared memory as one
+      // 16-byte load (lanes 16 bytes apart: conflict-free)
       uint4 wr[8];
       const int q_first = lane;
 #pragma unroll
@@ -245,27 +267,25 @@ k_router_tiled(const __nv_bfloat16* __restrict__ x, const __nv_bfloat16* __restr
                        ? __ldg(reinterpret_cast<const uint4*>(W + (size_t)e * H) + qn)
                        : make_uint4(0, 0, 0, 0);
         }
-        const uint32_t* xw = reinterpret_cast<const uint32_t*>(xs) + 4 * q;  // chunk q, token 0
+        uint4 xr[8];
 #pragma unroll
-        for (int wd = 0; wd < 4; ++wd) {
-          uint32_t xt[8];
+        for (int tt = 0; tt < 8; ++tt)
+          xr[tt] = *reinterpret_cast<const uint4*>(xs + (size_t)tt * H + 8 * q);
 #pragma unroll
-          for (int tt = 0; tt < 8; ++tt) xt[tt] = xw[(size_t)tt * (H / 2) + wd];
+        for (int el = 0; el < 8; ++el) {  // element 8 q + el of the chunk, ascending
+          float xv[8], wv[8];
 #pragma unroll
-          for (int hf = 0; hf < 2; ++hf) {  // element 2 wd + hf of the chunk, ascending
-            float xv[8], wv[8];
-#pragma unroll
-            for (int i = 0; i < 8; ++i) {
-              const uint32_t ww = wd == 0 ? wr[i].x : wd == 1 ? wr[i].y : wd == 2 ? wr[i].z : wr[i].w;
-              xv[i] = hf ? bf16_hi(xt[i]) : bf16_lo(xt[i]);
-              wv[i] = hf ? bf16_hi(ww) : bf16_lo(ww);
-            }
-#pragma unroll
-            for (int tt = 0; tt < 8; ++tt)
-#pragma unroll
-              for (int ee = 0; ee < 8; ++ee)
-                acc[tt * 8 + ee] = __fmaf_rn(xv[tt], wv[ee], acc[tt * 8 + ee]);
+          for (int i = 0; i < 8; ++i) {
+            const uint32_t xw = word_of(xr[i], el >> 1), ww = word_of(wr[i], el >> 1);
+            xv[i] = (el & 1) ? bf16_hi(xw) : bf16_lo(xw);
+            wv[i] = (el & 1) ? bf16_hi(ww) : bf16_lo(ww);
           }
+#pragma unroll
+          for (int ee = 0; ee < 8; ++ee)
+#pragma unroll
+            for (int tp = 0; tp < 4; ++tp)
+              fma2_rn(acc[ee * 8 + 2 * tp], acc[ee * 8 + 2 * tp + 1], xv[2 * tp], xv[2 * tp + 1],
+                      wv[ee]);
         }
 #pragma unroll
         for (int ee = 0; ee < 8; ++ee) wr[ee] = wn[ee];
@@ -282,11 +302,11 @@ k_router_tiled(const __nv_bfloat16* __restrict__ x, const __nv_bfloat16* __restr
           acc[a] = __fadd_rn(keep, __shfl_xor_sync(0xffffffffu, send, o));
         }
       }
-      // lane l now holds entries 2l, 2l + 1: token l / 4, experts 2 (l % 4) + {0, 1}
-      const int tt = lane >> 2;
+      // lane l now holds entries 2l, 2l + 1: expert l / 4, tokens 2 (l % 4) + {0, 1}
+      const int e = 8 * g + (lane >> 2);
 #pragma unroll
       for (int h = 0; h < 2; ++h) {
-        const int e = 8 * g + 2 * (lane & 3) + h;
+        const int tt = 2 * (lane & 3) + h;
         if (e < E) {
           const float v = bias ? __fadd_rn(acc[h], bias[e]) : acc[h];
           ls[tt * E + e] = v;

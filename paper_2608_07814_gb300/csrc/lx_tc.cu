@@ -6,14 +6,13 @@
 // amortised forward (Sec. 5.1), each evaluated once per (token, node).
 //
 // One persistent CTA per SM, 8 warps:
-//   warp 0      producer: claims tiles from the launch's counter (one ahead),
-//               loads the weight boxes (64 rows x 64 K, 128B swizzle, tiled
-//               layout) with TMA, and the 128 token rows either with one TMA
-//               box (rows already contiguous in node-row order: P, z, Q) or
-//               with 16-byte cp.async gathers (x rows by token id, eight lanes
-//               per 128-byte row so one instruction touches four rows);
-//               gathered rows are made visible to the tensor core's async
-//               proxy with fence.proxy.async before the stage is marked full;
+//   warp 2      scheduler: claims tiles from the launch's counter and
+//               decodes them (plan-prefix search, bucket lookups) into a small
+//               shared-memory queue ahead of the producer;
+//   warp 0      producer: takes decoded tiles from the queue and loads the
+//               weight boxes (64 rows x 64 K, 128B swizzle, tiled layout) and
+//               the 128 token rows (one box: rows are contiguous in node-row
+//               order, x rows having been gathered once) with TMA;
 //   warp 1      allocates 512 TMEM columns (two 256-column accumulators, so
 //               the epilogue of one tile overlaps the MMAs of the next); lane 0
 //               issues tcgen05.mma (kind::f16, bf16 x bf16 -> fp32, M=128,
@@ -48,6 +47,7 @@ constexpr int TC_TMEM_COLS = 2 * TC_ACC_COLS;    // double-buffered
 constexpr int TC_EPI_LD = 36;                    // staging row stride (floats)
 constexpr int TC_EPI_BYTES = 32 * TC_EPI_LD * 4; // per epilogue warp
 constexpr unsigned long long TC_TIMEOUT_CYCLES = 4000000000ull;  // ~2 s
+constexpr int TC_QN = 1;  // decoded tiles queued ahead of the producer (one, as a claim one tile ahead)
 static_assert(TC_STAGE_BYTES % 1024 == 0, "stages keep the 1024-byte swizzle alignment");
 static_assert(TC_STAGES <= 8 && TC_STAGES >= 2, "in-flight stage ring packs 4-bit stage ids");
 
@@ -103,21 +103,6 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
       " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
       "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(bar)
       : "memory");
-}
-__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst),
-               "l"(reinterpret_cast<uint64_t>(src))
-               : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() {
-  asm volatile("cp.async.commit_group;" ::: "memory");
-}
-template <int N>
-__device__ __forceinline__ void cp_async_wait() {
-  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
-}
-__device__ __forceinline__ void fence_proxy_async() {
-  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
 // ---- tcgen05 ---------------------------------------------------------------
@@ -222,16 +207,6 @@ __device__ __forceinline__ void tc_decode_warp(const TcLaunch& P, int tile, TcTi
   t.M = min(TC_BM, b1 - t.tok0);
 }
 
-// gathered token of row 4 i + r8 of a tile, or -1 past the bucket
-__device__ __forceinline__ void tc_load_trow(const TcLaunch& P, const TcTile& t, int r8,
-                                             int (&tr)[TC_BM / 4]) {
-#pragma unroll
-  for (int i = 0; i < TC_BM / 4; ++i) {
-    const int m = 4 * i + r8;
-    tr[i] = m < t.M ? __ldg(P.gather + t.tok0 + m) : -1;
-  }
-}
-
 __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant__ TcLaunch P) {
   pdl_wait();
   extern __shared__ uint8_t smem_raw[];
@@ -246,6 +221,9 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
   uint32_t* tmem_base_s = reinterpret_cast<uint32_t*>(bars + 2 * TC_STAGES + 6);
   TcTile* slot = reinterpret_cast<TcTile*>(bars + 2 * TC_STAGES + 7);     // [TC_STAGES]
   TcTile* eslot = slot + TC_STAGES;                                         // [2] epilogue hand-off
+  TcTile* qslot = eslot + 2;                                                // [TC_QN] decoded tiles
+  uint64_t* qbars = reinterpret_cast<uint64_t*>(qslot + TC_QN);             // qfull[QN], qempty[QN]
+  const uint32_t qfull0 = smem_u32(qbars), qempty0 = qfull0 + 8 * TC_QN;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t smem_base = smem_u32(smem);
   uint32_t prod_it = 0;  // stages the producer issued
@@ -260,6 +238,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
       mbar_init(tempty0 + 8 * b, 4);  // one arrival per epilogue warp
     }
     mbar_init(drain, 1);
+    for (int q = 0; q < TC_QN; ++q) {
+      mbar_init(qfull0 + 8 * q, 1);   // the scheduler's arrival (tile written)
+      mbar_init(qempty0 + 8 * q, 1);  // the producer's arrival (tile read)
+    }
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -277,28 +259,24 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
-    const int total = P.tile_off[P.n_items];
-    const int r8 = lane >> 3, u = lane & 7;  // gather: row within a group of 4, 16-byte chunk
-    int cur = lane == 0 ? atomicAdd(P.ctr, 1) : 0;
-    cur = __shfl_sync(0xffffffffu, cur, 0);
-    TcTile t;
-    int trow[TC_BM / 4];  // token of row 4 i + r8 of the current tile, or -1
-    if (cur < total) {
-      tc_decode_warp(P, cur, t);
-      if (P.gather) tc_load_trow(P, t, r8, trow);
-    }
-    int claim = lane == 0 ? atomicAdd(P.ctr, 1) : 0;  // the next tile, claimed one ahead
-    uint32_t it = 0;
+    // Tiles come decoded from the scheduler warp's queue, so that the TMA
+    // issue never waits on the plan lookups.
+    uint32_t it = 0, qi = 0;
     bool ok = true;
-    // Gathered stages still in flight (cp.async groups not yet waited for), oldest
-    // first, four bits per stage index: up to TC_STAGES - 1 stages of token rows
-    // stay in flight before the oldest is published to the MMA issuer.
-    uint32_t pq = 0;
-    int np = 0;
-    while (cur < total && ok) {
-      TcTile tn;
-      int trow_n[TC_BM / 4];
-      int nxt = total;
+    while (ok) {
+      const uint32_t q = qi % TC_QN;
+      int got = 1;
+      if (lane == 0) got = mbar_wait(qfull0 + 8 * q, (qi / TC_QN) & 1, abort_flag, P.wait_cycles);
+      if (!__shfl_sync(0xffffffffu, got, 0)) {
+        ok = false;
+        break;
+      }
+      __syncwarp();  // lane 0's acquire orders the scheduler's write before every lane's read
+      const TcTile t = qslot[q];
+      __syncwarp();
+      if (lane == 0) mbar_arrive(qempty0 + 8 * q);
+      ++qi;
+      if (t.BN < 0) break;  // no tile left
       const int nkb = (t.K + TC_BK - 1) / TC_BK;
       const int rt0 = (t.grp * t.Ng + t.row0) / 64;  // first 64-row weight tile
       const int nbox = (t.BN + 63) / 64;
@@ -310,7 +288,12 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
                            P.wait_cycles) ? 1 : 0;
           if (good) {
             if (kb == 0) slot[s] = t;
-            mbar_expect_tx(full0 + 8 * s, nbox * 8192 + (P.gather ? 0 : TC_A_BYTES));
+            mbar_expect_tx(full0 + 8 * s, nbox * 8192 + TC_A_BYTES);
+            const uint32_t a_s = smem_base + s * TC_STAGE_BYTES, b_s = a_s + TC_A_BYTES;
+            for (int b = 0; b < nbox; ++b)
+              tma_load_4d(b_s + b * 8192, P.wmaps + t.node, 0, 0, kb, rt0 + b, full0 + 8 * s);
+            tma_load_2d(a_s, P.xmap, (int)(t.grp * t.K) + kb * TC_BK + P.xcol, t.tok0,
+                        full0 + 8 * s);
           }
         }
         good = __shfl_sync(0xffffffffu, good, 0);
@@ -318,59 +301,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
           ok = false;
           break;
         }
-        const uint32_t a_s = smem_base + s * TC_STAGE_BYTES, b_s = a_s + TC_A_BYTES;
-        if (lane == 0) {
-          for (int b = 0; b < nbox; ++b)
-            tma_load_4d(b_s + b * 8192, P.wmaps + t.node, 0, 0, kb, rt0 + b, full0 + 8 * s);
-          if (!P.gather)
-            tma_load_2d(a_s, P.xmap, (int)(t.grp * t.K) + kb * TC_BK + P.xcol, t.tok0,
-                        full0 + 8 * s);
-        }
-        if (P.gather) {
-          // row m (128 bytes of K) in the 128-byte swizzle: chunk u goes to u ^ (m & 7);
-          // eight lanes cover one row, one instruction four rows
-          const __nv_bfloat16* xk = P.X + kb * TC_BK + 8 * u;
-#pragma unroll
-          for (int i = 0; i < TC_BM / 4; ++i) {
-            const int m = 4 * i + r8;
-            if (trow[i] >= 0)
-              cp_async16(a_s + m * 128 + ((u ^ (m & 7)) << 4), xk + (long)trow[i] * P.ldx);
-          }
-          cp_async_commit();
-          pq |= s << (4 * np);
-          if (++np == TC_STAGES - 1) {  // publish the oldest gathered stage
-            cp_async_wait<TC_STAGES - 2>();
-            fence_proxy_async();
-            mbar_arrive(full0 + 8 * (pq & 15u));
-            pq >>= 4;
-            --np;
-          }
-        } else {
-          mbar_arrive(full0 + 8 * s);
-        }
-        if (kb == 0) {
-          // the next tile: decoded (and its token rows looked up) while this
-          // one streams
-          nxt = __shfl_sync(0xffffffffu, claim, 0);
-          if (nxt < total) {
-            tc_decode_warp(P, nxt, tn);
-            if (P.gather) tc_load_trow(P, tn, r8, trow_n);
-          }
-        }
+        mbar_arrive(full0 + 8 * s);
       }
-      if (!ok) break;
-      cur = nxt;
-      if (cur < total) {
-        t = tn;
-#pragma unroll
-        for (int i = 0; i < TC_BM / 4; ++i) trow[i] = trow_n[i];
-        claim = lane == 0 ? atomicAdd(P.ctr, 1) : 0;
-      }
-    }
-    if (np > 0) {  // publish what is still in flight
-      cp_async_wait<0>();
-      fence_proxy_async();
-      for (; np > 0; --np, pq >>= 4) mbar_arrive(full0 + 8 * (pq & 15u));
     }
     if (ok) {
       // sentinel stage
@@ -397,6 +329,42 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
       *abort_flag = 1;
     }
     prod_it = it;
+  } else if (warp == 2) {
+    // ------------------------------------------------------------ scheduler
+    // Claims tiles from the launch's counter and decodes them (the plan-prefix
+    // search and the bucket lookups: dependent global loads) into a queue of
+    // TC_QN tiles ahead of the producer; a sentinel (BN < 0) ends the queue.
+    const int total = P.tile_off[P.n_items];
+    uint32_t qi = 0;
+    bool ok = true;
+    while (true) {
+      int cur = lane == 0 ? atomicAdd(P.ctr, 1) : 0;
+      cur = __shfl_sync(0xffffffffu, cur, 0);
+      TcTile t;
+      if (cur < total) tc_decode_warp(P, cur, t);
+      else t.BN = -1;
+      const uint32_t q = qi % TC_QN;
+      int good = 1;
+      if (lane == 0) {
+        good = mbar_wait(qempty0 + 8 * q, ((qi / TC_QN) & 1) ^ 1, abort_flag, P.wait_cycles)
+                   ? 1 : 0;
+        if (good) {
+          qslot[q] = t;
+          mbar_arrive(qfull0 + 8 * q);
+        }
+      }
+      good = __shfl_sync(0xffffffffu, good, 0);
+      if (!good) {
+        ok = false;
+        break;
+      }
+      ++qi;
+      if (cur >= total) break;
+    }
+    if (!ok && lane == 0) {
+      atomicExch(P.err, LX_ERR_TIMEOUT);
+      *abort_flag = 1;
+    }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
@@ -565,7 +533,7 @@ int tc_tile_cols() { return TC_BN; }
 
 static int tc_smem_bytes() {
   return TC_STAGES * TC_STAGE_BYTES + 4 * TC_EPI_BYTES + 8 * (2 * TC_STAGES + 7) +
-         3 * TC_STAGES * (int)sizeof(TcTile) + 1024;
+         (TC_STAGES + 2 + TC_QN) * (int)sizeof(TcTile) + 16 * TC_QN + 1024;
 }
 
 lx_status launch_tc(lx_layer* L, const TcLaunch& P, cudaStream_t s, const char* name) {
@@ -578,9 +546,8 @@ lx_status launch_tc(lx_layer* L, const TcLaunch& P, cudaStream_t s, const char* 
   return LX_OK;
 }
 
-static TcLaunch tc_op(lx_layer* L, int op, const __nv_bfloat16* X, long ldx, const int* gather,
-                      const CUtensorMap* xmap, int xcol, void* out, long ldo, bool out_f32,
-                      int counter) {
+static TcLaunch tc_op(lx_layer* L, int op, const CUtensorMap* xmap, int xcol, void* out,
+                      long ldo, bool out_f32, int counter) {
   Workspace& w = L->ws;
   TcLaunch P;
   P.shape = op_shape(L, op);
@@ -590,9 +557,6 @@ static TcLaunch tc_op(lx_layer* L, int op, const __nv_bfloat16* X, long ldx, con
   P.node_off = w.key_off;
   P.rank = L->d_rank;
   P.wmaps = L->d_tmaps + (size_t)op * L->N;
-  P.X = X;
-  P.ldx = ldx;
-  P.gather = gather;
   P.xmap = xmap;
   P.xcol = xcol;
   P.out = out;
@@ -618,10 +582,23 @@ k_gather_rows(const __nv_bfloat16* __restrict__ x, int H, const int* __restrict_
   const int lane = threadIdx.x & 31;
   const long warps = (long)gridDim.x * (blockDim.x >> 5);
   const int vec = H / 8;
-  for (long r = (long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); r < R; r += warps) {
-    const uint4* src = reinterpret_cast<const uint4*>(x + (size_t)node_tok[r] * H);
+  constexpr int U = 8;  // 16-byte loads of a row in flight per lane before any store
+  long r = (long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  int tok = r < R ? node_tok[r] : 0;
+  for (; r < R; r += warps) {
+    const uint4* src = reinterpret_cast<const uint4*>(x + (size_t)tok * H);
     uint4* dst = reinterpret_cast<uint4*>(xg + (size_t)r * H);
-    for (int i = lane; i < vec; i += 32) dst[i] = __ldg(src + i);
+    const long rn = r + warps;
+    tok = rn < R ? node_tok[rn] : 0;  // the next row's token, looked up early
+    for (int i0 = lane; i0 < vec; i0 += 32 * U) {
+      uint4 v[U];
+#pragma unroll
+      for (int u = 0; u < U; ++u)
+        if (i0 + 32 * u < vec) v[u] = __ldg(src + i0 + 32 * u);
+#pragma unroll
+      for (int u = 0; u < U; ++u)
+        if (i0 + 32 * u < vec) dst[i0 + 32 * u] = v[u];
+    }
   }
 }
 
@@ -643,18 +620,18 @@ lx_status launch_tc_experts(lx_layer* L, const void* x, int T, int k, void* y, c
              w.key_off + L->N, w.rows_cap, w.xg);
     LX_CUDA(cudaGetLastError());
   }
-  LX_TRY(run(tc_op(L, OP_UP_ANCHOR, nullptr, 0, nullptr, w.gmap, 0, w.hb, 2 * I, false, 0),
+  LX_TRY(run(tc_op(L, OP_UP_ANCHOR, w.gmap, 0, w.hb, 2 * I, false, 0),
              "tc_up_anchor"));
-  LX_TRY(run(tc_op(L, OP_UP_V, nullptr, 0, nullptr, w.gmap, 0, w.Pb, 2 * rmax, false, 1),
+  LX_TRY(run(tc_op(L, OP_UP_V, w.gmap, 0, w.Pb, 2 * rmax, false, 1),
              "tc_up_V"));
-  LX_TRY(run(tc_op(L, OP_UP_U, nullptr, 0, nullptr, w.xmaps + 0, 0, w.hb, 2 * I, false, 2),
+  LX_TRY(run(tc_op(L, OP_UP_U, w.xmaps + 0, 0, w.hb, 2 * I, false, 2),
              "tc_up_U"));
   LX_TRY(launch_swiglu(L, T, k, true, s));
-  LX_TRY(run(tc_op(L, OP_DN_ANCHOR, nullptr, 0, nullptr, w.xmaps + 1, 0, w.yb, H, false, 3),
+  LX_TRY(run(tc_op(L, OP_DN_ANCHOR, w.xmaps + 1, 0, w.yb, H, false, 3),
              "tc_dn_anchor"));
-  LX_TRY(run(tc_op(L, OP_DN_V, nullptr, 0, nullptr, w.xmaps + 1, 0, w.Qb, rmax, false, 4),
+  LX_TRY(run(tc_op(L, OP_DN_V, w.xmaps + 1, 0, w.Qb, rmax, false, 4),
              "tc_dn_V"));
-  LX_TRY(run(tc_op(L, OP_DN_U, nullptr, 0, nullptr, w.xmaps + 2, 0, w.yb, H, false, 5),
+  LX_TRY(run(tc_op(L, OP_DN_U, w.xmaps + 2, 0, w.yb, H, false, 5),
              "tc_dn_U"));
   LX_TRY(launch_combine(L, T, k, y, true, s));
   return LX_OK;
