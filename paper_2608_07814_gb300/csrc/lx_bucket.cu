@@ -414,7 +414,7 @@ static PlanArgs make_plans(const lx_layer* L, int n_plans, int first = 0) {
     pa.shape[p] = op_shape(L, op);
     pa.items[p] = pa.shape[p].on_anchors ? L->d_anchors : L->d_corrs;
     pa.n_items[p] = pa.shape[p].on_anchors ? L->n_anchor : L->n_corr;
-    pa.bm[p] = slot < PLAN_TC ? G_BM : tc_tile_tokens();
+    pa.bm[p] = slot < PLAN_TC ? G_BM : tc_tile_rows(op);
     pa.bn[p] = slot < PLAN_TC ? G_BN : tc_tile_cols();
   }
   return pa;

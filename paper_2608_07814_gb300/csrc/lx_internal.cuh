@@ -244,6 +244,7 @@ struct TcLaunch {
   int* err;
   unsigned long long wait_cycles;  // bound of every wait (SM clock cycles)
   int unmet_wait;            // lx_wait_site whose wait is made to run out (test hook), 0 = none
+  int bm;                    // tile rows: 128 or 256 (tc_tile_rows of the op)
 };
 
 // ---------------------------------------------------------------------------
@@ -432,8 +433,9 @@ lx_status launch_combine(lx_layer* L, int T, int k, void* y, bool bf16, cudaStre
                          SplitParts ys = SplitParts());
 lx_status launch_fast_experts(lx_layer* L, const void* x, int T, int k, void* y, cudaStream_t s);
 lx_status launch_tc_experts(lx_layer* L, const void* x, int T, int k, void* y, cudaStream_t s);
-int tc_tile_tokens();
+int tc_tile_tokens();  // rows of the TMA boxes of the tensor-core A operands
 int tc_tile_cols();
+int tc_tile_rows(int op);  // token rows of a tensor-core tile of op (its tile plan)
 lx_status launch_tc(lx_layer* L, const TcLaunch& P, cudaStream_t s, const char* name);
 lx_status launch_stream(lx_layer* L, const StreamLaunch& P, cudaStream_t s, const char* name);
 // plans = false: skip the generic GEMMs' tile plans (not read by the

@@ -37,21 +37,32 @@ namespace {
 
 using namespace tcg;
 
-constexpr int TC_BM = 128;          // tokens per tile (UMMA M)
 constexpr int TC_BN = 256;          // max output columns per tile (UMMA N)
 constexpr int TC_BK = 64;           // K per stage (one 128-byte swizzle row)
-constexpr int TC_STAGES = 4;
-constexpr int TC_A_BYTES = TC_BM * TC_BK * 2;   // 16 KiB
 constexpr int TC_B_BYTES = TC_BN * TC_BK * 2;   // 32 KiB
-constexpr int TC_STAGE_BYTES = TC_A_BYTES + TC_B_BYTES;
 constexpr int TC_THREADS = 256;
 constexpr int TC_ACC_COLS = 256;                 // one accumulator
 constexpr int TC_TMEM_COLS = 2 * TC_ACC_COLS;    // double-buffered
 constexpr int TC_EPI_LD = 36;                    // staging row stride (floats)
 constexpr int TC_EPI_BYTES = 32 * TC_EPI_LD * 4; // per epilogue warp
 constexpr int TC_QN = 1;  // decoded tiles queued ahead of the producer (one, as a claim one tile ahead)
-static_assert(TC_STAGE_BYTES % 1024 == 0, "stages keep the 1024-byte swizzle alignment");
-static_assert(TC_STAGES <= 8 && TC_STAGES >= 2, "in-flight stage ring packs 4-bit stage ids");
+
+// Tile rows BM (tokens): 128 (one M = 128 MMA per K step, two TMEM
+// accumulators so that a tile's epilogue overlaps the next tile's MMAs) or 256
+// (two M = 128 MMAs per K step share each weight box: 1.5x the tensor work per
+// byte in flight, which lifts the long-K products whose stage ring cannot
+// cover the load latency; one accumulator of 2 x 256 columns, so the epilogue
+// does not overlap the next tile).
+template <int BM>
+struct TcCfg {
+  static constexpr int NH = BM / 128;                    // 128-row halves of a tile
+  static constexpr int A_BYTES = BM * TC_BK * 2;
+  static constexpr int STAGE_BYTES = A_BYTES + TC_B_BYTES;
+  static constexpr int STAGES = NH == 1 ? 4 : 3;
+  static constexpr int NBUF = NH == 1 ? 2 : 1;           // accumulators of NH x 256 columns
+  static_assert(STAGE_BYTES % 1024 == 0, "stages keep the 1024-byte swizzle alignment");
+  static_assert(NBUF * NH * TC_ACC_COLS <= TC_TMEM_COLS, "accumulators fit the TMEM allocation");
+};
 
 struct TcTile {
   int node, grp, row0, tok0, M, Ng, K, BN;  // BN < 0: sentinel
@@ -62,6 +73,7 @@ struct TcTile {
 // prefix and ballots count the items whose first tile is <= `tile` (the
 // prefix is non-decreasing and starts at 0), instead of a chain of dependent
 // loads of a binary search.
+template <int BM>
 __device__ __forceinline__ void tc_decode_warp(const TcLaunch& P, int tile, TcTile& t) {
   const int lane = threadIdx.x & 31;
   const int* to = P.tile_off;
@@ -90,11 +102,15 @@ __device__ __forceinline__ void tc_decode_warp(const TcLaunch& P, int tile, TcTi
   t.row0 = (rem % ncol) * TC_BN;
   t.BN = min(TC_BN, t.Ng - t.row0);
   t.node = n;
-  t.tok0 = b0 + tb * TC_BM;
-  t.M = min(TC_BM, b1 - t.tok0);
+  t.tok0 = b0 + tb * BM;
+  t.M = min(BM, b1 - t.tok0);
 }
 
+template <int BM>
 __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant__ TcLaunch P) {
+  using C = TcCfg<BM>;
+  constexpr int TC_STAGES = C::STAGES, TC_STAGE_BYTES = C::STAGE_BYTES, TC_A_BYTES = C::A_BYTES;
+  constexpr int NH = C::NH, NBUF = C::NBUF;
   pdl_wait();
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -175,12 +191,16 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
                            P.wait_cycles) ? 1 : 0;
           if (good) {
             if (kb == 0) slot[s] = t;
-            mbar_expect_tx(full0 + 8 * s, nbox * 8192 + TC_A_BYTES);
+            // a 256-row tile whose rows end within its first half loads one half
+            const int nh = (NH == 2 && t.M > 128) ? 2 : 1;
+            mbar_expect_tx(full0 + 8 * s, nbox * 8192 + nh * 128 * TC_BK * 2);
             const uint32_t a_s = smem_base + s * TC_STAGE_BYTES, b_s = a_s + TC_A_BYTES;
             for (int b = 0; b < nbox; ++b)
               tma_load_4d(b_s + b * 8192, P.wmaps + t.node, 0, 0, kb, rt0 + b, full0 + 8 * s);
-            tma_load_2d(a_s, P.xmap, (int)(t.grp * t.K) + kb * TC_BK + P.xcol, t.tok0,
-                        full0 + 8 * s);
+            for (int h = 0; h < nh; ++h)
+              tma_load_2d(a_s + h * 128 * TC_BK * 2, P.xmap,
+                          (int)(t.grp * t.K) + kb * TC_BK + P.xcol, t.tok0 + 128 * h,
+                          full0 + 8 * s);
           }
         }
         good = __shfl_sync(0xffffffffu, good, 0);
@@ -228,7 +248,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
       int cur = lane == 0 ? atomicAdd(P.ctr, 1) : 0;
       cur = __shfl_sync(0xffffffffu, cur, 0);
       TcTile t;
-      if (cur < total) tc_decode_warp(P, cur, t);
+      if (cur < total) tc_decode_warp<BM>(P, cur, t);
       else t.BN = -1;
       const uint32_t q = qi % TC_QN;
       int good = 1;
@@ -268,9 +288,9 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
           break;
         }
         const TcTile t = slot[s];
-        const uint32_t b = tiles & 1;
-        // this accumulator must have been drained by the epilogue (two tiles ago)
-        if (!mbar_wait(tempty0 + 8 * b, ((tiles >> 1) & 1) ^ 1, abort_flag, P.wait_cycles)) {
+        const uint32_t b = tiles % NBUF, u = tiles / NBUF;
+        // this accumulator must have been drained by the epilogue (NBUF tiles ago)
+        if (!mbar_wait(tempty0 + 8 * b, (u & 1) ^ 1, abort_flag, P.wait_cycles)) {
           ok = false;
           break;
         }
@@ -282,8 +302,9 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
           break;
         }
         tc_fence_after();
-        const uint32_t d = tmem + b * TC_ACC_COLS;
-        const uint32_t idesc = instr_desc(TC_BM, t.BN);
+        const uint32_t d = tmem + b * NH * TC_ACC_COLS;
+        const uint32_t idesc = instr_desc(128, t.BN);
+        const int nh = (NH == 2 && t.M > 128) ? 2 : 1;
         const int nkb = (t.K + TC_BK - 1) / TC_BK;
         for (int kb = 0; kb < nkb; ++kb, ++it) {
           const uint32_t s2 = it % TC_STAGES;
@@ -295,8 +316,9 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
           const uint32_t a_s = smem_base + s2 * TC_STAGE_BYTES, b_s = a_s + TC_A_BYTES;
 #pragma unroll
           for (int k = 0; k < TC_BK / 16; ++k)
-            tc_mma(d, smem_desc(a_s + 32 * k), smem_desc(b_s + 32 * k), idesc,
-                   (kb | k) != 0 ? 1u : 0u);
+            for (int h = 0; h < nh; ++h)  // the 128-row halves share the weight box
+              tc_mma(d + h * TC_ACC_COLS, smem_desc(a_s + h * 128 * TC_BK * 2 + 32 * k),
+                     smem_desc(b_s + 32 * k), idesc, (kb | k) != 0 ? 1u : 0u);
           tc_commit(empty0 + 8 * s2);  // frees the stage once these MMAs are done
         }
         if (!ok) break;
@@ -317,8 +339,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
     float* stg = epi + ew * 32 * TC_EPI_LD;
     uint32_t tiles = 0;
     while (true) {
-      const uint32_t b = tiles & 1;
-      if (!mbar_wait(tfull0 + 8 * b, (tiles >> 1) & 1, abort_flag, P.wait_cycles)) {
+      const uint32_t b = tiles % NBUF, u = tiles / NBUF;
+      if (!mbar_wait(tfull0 + 8 * b, u & 1, abort_flag, P.wait_cycles)) {
         if (lane == 0) {
           atomicExch(P.err, LX_ERR_TIMEOUT);
           *abort_flag = 1;
@@ -331,10 +353,12 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
       const bool tile_ok = t.tok0 >= 0 && (long)t.grp * t.Ng + t.row0 + t.BN <= P.ldo;
       const long col0 = (long)t.grp * t.Ng + t.row0;
       const int cq = lane & 7;
+      for (int h = 0; h < NH && 128 * h < t.M; ++h) {
+      const uint32_t acc = tmem + (b * NH + h) * TC_ACC_COLS;
       if (P.out_f32) {
         for (int c0 = 0; c0 < t.BN; c0 += 32) {
           float v[32];
-          tc_ld32(tmem + b * TC_ACC_COLS + ((uint32_t)(32 * ew) << 16) + (uint32_t)c0, v);
+          tc_ld32(acc + ((uint32_t)(32 * ew) << 16) + (uint32_t)c0, v);
           // lane = accumulator row: stage the 32 x 32 block row-major
           float4* srow = reinterpret_cast<float4*>(stg + lane * TC_EPI_LD);
 #pragma unroll
@@ -345,7 +369,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
 #pragma unroll
           for (int j = 0; j < 8; ++j) {
             const int rr = 4 * j + (lane >> 3);
-            const int m = 32 * ew + rr;
+            const int m = 128 * h + 32 * ew + rr;
             const long grow = (long)t.tok0 + m;
             if (tile_ok && m < t.M && grow < P.rows_cap) {
               const float4 f = *reinterpret_cast<const float4*>(stg + rr * TC_EPI_LD + 4 * cq);
@@ -360,15 +384,20 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
         // segment is again 128 bytes
         for (int c0 = 0; c0 < t.BN; c0 += 64) {
           uint32_t pk[32];
-#pragma unroll
-          for (int h = 0; h < 2; ++h) {
-            float v[32];
-            tc_ld32(tmem + b * TC_ACC_COLS + ((uint32_t)(32 * ew) << 16) + (uint32_t)(c0 + 32 * h),
-                    v);
+          {
+            // both 32-column loads of the pass in flight, one wait
+            uint32_t r0[32], r1[32];
+            tc_ld32_async(acc + ((uint32_t)(32 * ew) << 16) + (uint32_t)c0, r0);
+            tc_ld32_async(acc + ((uint32_t)(32 * ew) << 16) + (uint32_t)(c0 + 32), r1);
+            tc_wait_ld();
 #pragma unroll
             for (int e = 0; e < 16; ++e) {
-              __nv_bfloat162 b2 = __floats2bfloat162_rn(v[2 * e], v[2 * e + 1]);
-              pk[16 * h + e] = *reinterpret_cast<uint32_t*>(&b2);
+              __nv_bfloat162 b0 = __floats2bfloat162_rn(__uint_as_float(r0[2 * e]),
+                                                        __uint_as_float(r0[2 * e + 1]));
+              __nv_bfloat162 b1 = __floats2bfloat162_rn(__uint_as_float(r1[2 * e]),
+                                                        __uint_as_float(r1[2 * e + 1]));
+              pk[e] = *reinterpret_cast<uint32_t*>(&b0);
+              pk[16 + e] = *reinterpret_cast<uint32_t*>(&b1);
             }
           }
           uint4* srow = reinterpret_cast<uint4*>(stg + lane * TC_EPI_LD);
@@ -379,7 +408,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
 #pragma unroll
           for (int j = 0; j < 8; ++j) {
             const int rr = 4 * j + (lane >> 3);
-            const int m = 32 * ew + rr;
+            const int m = 128 * h + 32 * ew + rr;
             const long grow = (long)t.tok0 + m;
             if (tile_ok && m < t.M && grow < P.rows_cap) {
               const uint4 u4 = *reinterpret_cast<const uint4*>(stg + rr * TC_EPI_LD + 4 * cq);
@@ -389,6 +418,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
           }
           __syncwarp();
         }
+      }
       }
       tc_fence_before();
       __syncwarp();
@@ -415,22 +445,35 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
 
 }  // namespace
 
-int tc_tile_tokens() { return TC_BM; }
+int tc_tile_tokens() { return 128; }
 int tc_tile_cols() { return TC_BN; }
+// The anchor gate/up product (K = d_model, anchor buckets of hundreds of
+// rows) takes 256-row tiles; the others 128 (measured at the Qwen3-shaped
+// prefill of 8192: tc_up_anchor 156 -> 146 us with 256 rows, while x V, whose
+// member buckets are a few hundred rows, loses more to half-empty tiles and a
+// single wave than it gains).
+int tc_tile_rows(int op) { return op == OP_UP_ANCHOR ? 256 : 128; }
 
+template <int BM>
 static int tc_smem_bytes() {
-  return TC_STAGES * TC_STAGE_BYTES + 4 * TC_EPI_BYTES + 8 * (2 * TC_STAGES + 7) +
-         (TC_STAGES + 2 + TC_QN) * (int)sizeof(TcTile) + 16 * TC_QN + 1024;
+  using C = TcCfg<BM>;
+  return C::STAGES * C::STAGE_BYTES + 4 * TC_EPI_BYTES + 8 * (2 * C::STAGES + 7) +
+         (C::STAGES + 2 + TC_QN) * (int)sizeof(TcTile) + 16 * TC_QN + 1024;
+}
+
+template <int BM>
+static lx_status launch_tc_bm(lx_layer* L, const TcLaunch& P, cudaStream_t s, const char* name) {
+  const int smem = tc_smem_bytes<BM>();
+  static bool done[64] = {};
+  LX_CUDA(smem_cap_once((const void*)k_tc_gemm<BM>, smem, L->device, done));
+  ProfScope ps(L, s, name);
+  launch_k(L, k_tc_gemm<BM>, L->num_sms, TC_THREADS, smem, s, P);
+  LX_CUDA(cudaGetLastError());
+  return LX_OK;
 }
 
 lx_status launch_tc(lx_layer* L, const TcLaunch& P, cudaStream_t s, const char* name) {
-  const int smem = tc_smem_bytes();
-  static bool done[64] = {};
-  LX_CUDA(smem_cap_once((const void*)k_tc_gemm, smem, L->device, done));
-  ProfScope ps(L, s, name);
-  launch_k(L, k_tc_gemm, L->num_sms, TC_THREADS, smem, s, P);
-  LX_CUDA(cudaGetLastError());
-  return LX_OK;
+  return P.bm == 256 ? launch_tc_bm<256>(L, P, s, name) : launch_tc_bm<128>(L, P, s, name);
 }
 
 static TcLaunch tc_op(lx_layer* L, int op, const CUtensorMap* xmap, int xcol, void* out,
@@ -438,6 +481,7 @@ static TcLaunch tc_op(lx_layer* L, int op, const CUtensorMap* xmap, int xcol, vo
   Workspace& w = L->ws;
   TcLaunch P;
   P.shape = op_shape(L, op);
+  P.bm = tc_tile_rows(op);
   P.items = P.shape.on_anchors ? L->d_anchors : L->d_corrs;
   P.n_items = P.shape.on_anchors ? L->n_anchor : L->n_corr;
   P.tile_off = w.tile_off + (PLAN_TC + op) * (op_max_items(L) + 1);
