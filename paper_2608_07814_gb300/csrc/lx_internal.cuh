@@ -245,6 +245,7 @@ struct TcLaunch {
   unsigned long long wait_cycles;  // bound of every wait (SM clock cycles)
   int unmet_wait;            // lx_wait_site whose wait is made to run out (test hook), 0 = none
   int bm;                    // tile rows: 128 or 256 (tc_tile_rows of the op)
+  int epi;                   // epilogue warps: 4 or 8
 };
 
 // ---------------------------------------------------------------------------

@@ -40,7 +40,6 @@ using namespace tcg;
 constexpr int TC_BN = 256;          // max output columns per tile (UMMA N)
 constexpr int TC_BK = 64;           // K per stage (one 128-byte swizzle row)
 constexpr int TC_B_BYTES = TC_BN * TC_BK * 2;   // 32 KiB
-constexpr int TC_THREADS = 256;
 constexpr int TC_ACC_COLS = 256;                 // one accumulator
 constexpr int TC_TMEM_COLS = 2 * TC_ACC_COLS;    // double-buffered
 constexpr int TC_EPI_LD = 36;                    // staging row stride (floats)
@@ -53,13 +52,18 @@ constexpr int TC_QN = 1;  // decoded tiles queued ahead of the producer (one, as
 // byte in flight, which lifts the long-K products whose stage ring cannot
 // cover the load latency; one accumulator of 2 x 256 columns, so the epilogue
 // does not overlap the next tile).
-template <int BM>
+// EPI: epilogue warps, 4 or 8 (two per TMEM lane quadrant, splitting the
+// column passes; for the short-K factor products, whose tiles are bound by
+// writing their output, with a 3-stage ring to make room for the staging).
+template <int BM, int EPI>
 struct TcCfg {
   static constexpr int NH = BM / 128;                    // 128-row halves of a tile
   static constexpr int A_BYTES = BM * TC_BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + TC_B_BYTES;
-  static constexpr int STAGES = NH == 1 ? 4 : 3;
+  static constexpr int STAGES = (NH == 1 && EPI == 4) ? 4 : 3;
   static constexpr int NBUF = NH == 1 ? 2 : 1;           // accumulators of NH x 256 columns
+  static constexpr int THREADS = 32 * (4 + EPI);
+  static_assert(EPI == 4 || EPI == 8, "four or eight epilogue warps");
   static_assert(STAGE_BYTES % 1024 == 0, "stages keep the 1024-byte swizzle alignment");
   static_assert(NBUF * NH * TC_ACC_COLS <= TC_TMEM_COLS, "accumulators fit the TMEM allocation");
 };
@@ -106,17 +110,18 @@ __device__ __forceinline__ void tc_decode_warp(const TcLaunch& P, int tile, TcTi
   t.M = min(BM, b1 - t.tok0);
 }
 
-template <int BM>
-__global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant__ TcLaunch P) {
-  using C = TcCfg<BM>;
+template <int BM, int EPI>
+__global__ void __launch_bounds__(TcCfg<BM, EPI>::THREADS, 1)
+k_tc_gemm(const __grid_constant__ TcLaunch P) {
+  using C = TcCfg<BM, EPI>;
   constexpr int TC_STAGES = C::STAGES, TC_STAGE_BYTES = C::STAGE_BYTES, TC_A_BYTES = C::A_BYTES;
   constexpr int NH = C::NH, NBUF = C::NBUF;
   pdl_wait();
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  float* epi = reinterpret_cast<float*>(smem + TC_STAGES * TC_STAGE_BYTES);  // [4][32][EPI_LD]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + TC_STAGES * TC_STAGE_BYTES + 4 * TC_EPI_BYTES);
+  float* epi = reinterpret_cast<float*>(smem + TC_STAGES * TC_STAGE_BYTES);  // [EPI][32][EPI_LD]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + TC_STAGES * TC_STAGE_BYTES + EPI * TC_EPI_BYTES);
   // full[S], empty[S], tmem_full[2], tmem_empty[2], drain
   const uint32_t full0 = smem_u32(bars), empty0 = full0 + 8 * TC_STAGES;
   const uint32_t tfull0 = empty0 + 8 * TC_STAGES, tempty0 = tfull0 + 16, drain = tempty0 + 16;
@@ -138,7 +143,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(tfull0 + 8 * b, 2);   // MMA thread's arrival (tile info written) + tcgen05.commit
-      mbar_init(tempty0 + 8 * b, 4);  // one arrival per epilogue warp
+      mbar_init(tempty0 + 8 * b, EPI);  // one arrival per epilogue warp
     }
     mbar_init(drain, 1);
     for (int q = 0; q < TC_QN; ++q) {
@@ -335,8 +340,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
     __syncwarp();
   } else if (warp >= 4) {
     // ------------------------------------------------------------ epilogue
-    const int ew = warp - 4;  // TMEM lanes 32 ew .. 32 ew + 31
-    float* stg = epi + ew * 32 * TC_EPI_LD;
+    const int ew = warp & 3;        // TMEM lanes 32 ew .. 32 ew + 31
+    const int eh = (warp - 4) >> 2; // with 8 warps: which column passes (alternate)
+    constexpr int ESTEP = EPI / 4;  // passes are dealt out to ESTEP warps per quadrant
+    float* stg = epi + (warp - 4) * 32 * TC_EPI_LD;
     uint32_t tiles = 0;
     while (true) {
       const uint32_t b = tiles % NBUF, u = tiles / NBUF;
@@ -356,7 +363,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
       for (int h = 0; h < NH && 128 * h < t.M; ++h) {
       const uint32_t acc = tmem + (b * NH + h) * TC_ACC_COLS;
       if (P.out_f32) {
-        for (int c0 = 0; c0 < t.BN; c0 += 32) {
+        for (int c0 = 32 * eh; c0 < t.BN; c0 += 32 * ESTEP) {
           float v[32];
           tc_ld32(acc + ((uint32_t)(32 * ew) << 16) + (uint32_t)c0, v);
           // lane = accumulator row: stage the 32 x 32 block row-major
@@ -382,7 +389,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) k_tc_gemm(const __grid_constant
       } else {
         // bf16: 64 columns per pass, converted before staging, so that a row
         // segment is again 128 bytes
-        for (int c0 = 0; c0 < t.BN; c0 += 64) {
+        for (int c0 = 64 * eh; c0 < t.BN; c0 += 64 * ESTEP) {
           uint32_t pk[32];
           {
             // both 32-column loads of the pass in flight, one wait
@@ -454,26 +461,28 @@ int tc_tile_cols() { return TC_BN; }
 // single wave than it gains).
 int tc_tile_rows(int op) { return op == OP_UP_ANCHOR ? 256 : 128; }
 
-template <int BM>
+template <int BM, int EPI>
 static int tc_smem_bytes() {
-  using C = TcCfg<BM>;
-  return C::STAGES * C::STAGE_BYTES + 4 * TC_EPI_BYTES + 8 * (2 * C::STAGES + 7) +
+  using C = TcCfg<BM, EPI>;
+  return C::STAGES * C::STAGE_BYTES + EPI * TC_EPI_BYTES + 8 * (2 * C::STAGES + 7) +
          (C::STAGES + 2 + TC_QN) * (int)sizeof(TcTile) + 16 * TC_QN + 1024;
 }
 
-template <int BM>
-static lx_status launch_tc_bm(lx_layer* L, const TcLaunch& P, cudaStream_t s, const char* name) {
-  const int smem = tc_smem_bytes<BM>();
+template <int BM, int EPI>
+static lx_status launch_tc_cfg(lx_layer* L, const TcLaunch& P, cudaStream_t s, const char* name) {
+  const int smem = tc_smem_bytes<BM, EPI>();
   static bool done[64] = {};
-  LX_CUDA(smem_cap_once((const void*)k_tc_gemm<BM>, smem, L->device, done));
+  LX_CUDA(smem_cap_once((const void*)k_tc_gemm<BM, EPI>, smem, L->device, done));
   ProfScope ps(L, s, name);
-  launch_k(L, k_tc_gemm<BM>, L->num_sms, TC_THREADS, smem, s, P);
+  launch_k(L, k_tc_gemm<BM, EPI>, L->num_sms, TcCfg<BM, EPI>::THREADS, smem, s, P);
   LX_CUDA(cudaGetLastError());
   return LX_OK;
 }
 
 lx_status launch_tc(lx_layer* L, const TcLaunch& P, cudaStream_t s, const char* name) {
-  return P.bm == 256 ? launch_tc_bm<256>(L, P, s, name) : launch_tc_bm<128>(L, P, s, name);
+  if (P.bm == 256) return launch_tc_cfg<256, 4>(L, P, s, name);
+  if (P.epi == 8) return launch_tc_cfg<128, 8>(L, P, s, name);
+  return launch_tc_cfg<128, 4>(L, P, s, name);
 }
 
 static TcLaunch tc_op(lx_layer* L, int op, const CUtensorMap* xmap, int xcol, void* out,
@@ -482,6 +491,9 @@ static TcLaunch tc_op(lx_layer* L, int op, const CUtensorMap* xmap, int xcol, vo
   TcLaunch P;
   P.shape = op_shape(L, op);
   P.bm = tc_tile_rows(op);
+  // short-K products (the U factors, K = rank; the down side, K = d_ff): tiles
+  // bound by writing their output take eight epilogue warps
+  P.epi = (op == OP_UP_U || op == OP_DN_U || op == OP_DN_ANCHOR || op == OP_DN_V) ? 8 : 4;
   P.items = P.shape.on_anchors ? L->d_anchors : L->d_corrs;
   P.n_items = P.shape.on_anchors ? L->n_anchor : L->n_corr;
   P.tile_off = w.tile_off + (PLAN_TC + op) * (op_max_items(L) + 1);
