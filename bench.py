@@ -214,6 +214,9 @@ def kernel_flops(name, st, src):
         "tc_up_anchor": 2 * Ra * 2 * I * H,
         "tc_up_V": 2 * rr * 2 * H,
         "tc_up_U": 2 * rr * 2 * I,
+        # the fused correction + SwiGLU kernel of flat layers: the members' P U^T
+        # products (the work tc_up_U does on the unfused path)
+        "ct_swiglu": 2 * rr * 2 * I,
         "tc_dn_anchor": 2 * Ra * H * I,
         "tc_dn_V": 2 * rr * I,
         "tc_dn_U": 2 * rr * H,

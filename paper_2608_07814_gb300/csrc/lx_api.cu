@@ -162,6 +162,12 @@ static lx_status ensure_workspace(lx_layer* L, int T, int k, cudaStream_t s) {
       {(void**)&w.hsplit, sizeof(float) * LX_STREAM_MAX_SPLIT * Rsplit * 2 * L->I},
       {(void**)&w.ysplit, sizeof(float) * LX_STREAM_MAX_SPLIT * Rsplit * L->H},
       {(void**)&w.err, 256},
+      // fused correction + SwiGLU tables (flat layers on the tensor-core path)
+      {(void**)&w.al_g, L->ct ? sizeof(float) * Rmax * ct_gstride(L) : 0},
+      {(void**)&w.al_row, L->ct ? sizeof(int) * Rmax * ct_rstride(L) : 0},
+      {(void**)&w.rho2al, L->ct ? sizeof(int) * Rmax : 0},
+      {(void**)&w.Pal, L->ct ? (size_t)2 * Rmax * L->ct_nch * 2 * rmax : 0},
+      {(void**)&w.pamap, L->ct ? 2 * sizeof(CUtensorMap) : 0},
   };
   size_t total = 0;
   for (auto& it : items) total += align_up(it.bytes, 256);
@@ -213,6 +219,16 @@ static lx_status ensure_workspace(lx_layer* L, int T, int k, cudaStream_t s) {
       e = cudaMemcpyAsync(w.gmap, maps + 6, sizeof(CUtensorMap), cudaMemcpyHostToDevice, s);
     if (e == cudaSuccess) e = cudaStreamSynchronize(s);
     if (e != cudaSuccess) return cuda_fail(e, "copy activation maps");
+  }
+  if (L->ct) {
+    CUtensorMap pm[2];
+    std::memset(pm, 0, sizeof(pm));
+    if (!encode_rows_map(&pm[0], w.Pal, Rmax, (long)L->ct_nch * 2 * rmax, tc_tile_tokens()) ||
+        !encode_rows_map(&pm[1], w.hb, Rmax, 2L * L->I, tc_tile_tokens()))
+      return fail(LX_ERR_CUDA, "cuTensorMapEncodeTiled(Pal, h) failed");
+    e = cudaMemcpyAsync(w.pamap, pm, 2 * sizeof(CUtensorMap), cudaMemcpyHostToDevice, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return cuda_fail(e, "copy Pal map");
   }
   L->last_T = L->last_k = 0;
   return LX_OK;
@@ -532,7 +548,33 @@ extern "C" lx_status lx_load_compressed_layer(const lx_layer_desc* d, const void
   const size_t o_anc = tadd(4 * std::max(1, L->n_anchor)), o_cor = tadd(4 * std::max(1, L->n_corr));
   const size_t o_p0 = tadd(sizeof(void*) * nptr), o_p1 = tadd(sizeof(void*) * nptr);
   const size_t o_p2 = tadd(sizeof(void*) * nptr), o_p3 = tadd(sizeof(void*) * nptr);
+  // children of every anchor (fused correction + SwiGLU of flat layers): a
+  // layer qualifies when every correction node is a direct child of an anchor
+  // and no anchor has more than CT_MAX_CH children
+  std::vector<int> child((size_t)L->N * CT_MAX_CH, -1), child_col(L->N, 0), nchild(L->N, 0);
+  bool flat = L->max_depth <= 2 && L->n_corr > 0;
+  for (int n = 0; n < L->N && flat; ++n) {
+    const int p = L->parent[n];
+    if (p < 0) continue;
+    if (L->parent[p] >= 0 || nchild[p] >= CT_MAX_CH) {
+      flat = false;
+      break;
+    }
+    child[(size_t)p * CT_MAX_CH + nchild[p]] = n;
+    child_col[n] = nchild[p] * 2 * std::max(1, L->max_rank);
+    ++nchild[p];
+  }
+  L->ct_nch = 0;
+  for (int n = 0; n < L->N; ++n) L->ct_nch = std::max(L->ct_nch, nchild[n]);
+  {
+    // LX_FUSED_SWIGLU=0 keeps the unfused tensor-core path (for A/B timing)
+    const char* env = std::getenv("LX_FUSED_SWIGLU");
+    L->ct = flat && L->tiled && !(env && env[0] == '0');
+  }
+  const size_t o_child = tadd(4 * child.size()), o_ccol = tadd(4 * (size_t)L->N);
   std::vector<char> tb(toff, 0);
+  std::memcpy(tb.data() + o_child, child.data(), 4 * child.size());
+  std::memcpy(tb.data() + o_ccol, child_col.data(), 4 * (size_t)L->N);
   std::memcpy(tb.data() + o_rank, L->rank.data(), 4 * L->N);
   std::memcpy(tb.data() + o_paths, paths.data(), 4 * paths.size());
   std::memcpy(tb.data() + o_plen, plen.data(), 4 * L->E);
@@ -554,11 +596,14 @@ extern "C" lx_status lx_load_compressed_layer(const lx_layer_desc* d, const void
   L->d_w_upU = (const void**)(tbase + o_p1);
   L->d_w_dn = (const void**)(tbase + o_p2);
   L->d_w_dnU = (const void**)(tbase + o_p3);
+  L->d_child = (int*)(tbase + o_child);
+  L->d_child_col = (int*)(tbase + o_ccol);
   ce = cudaMemcpyAsync(L->tables, tb.data(), toff, cudaMemcpyHostToDevice, s);
   if (ce == cudaSuccess) ce = cudaStreamSynchronize(s);
   if (ce != cudaSuccess) return cleanup(cuda_fail(ce, "copy tables"));
   const lx_status st = encode_tensor_maps(L, s);
   if (st != LX_OK) return cleanup(st);
+  L->ct = L->ct && L->stream_ok;
   *out = L;
   return LX_OK;
 }

@@ -416,6 +416,15 @@ static PlanArgs make_plans(const lx_layer* L, int n_plans, int first = 0) {
     pa.n_items[p] = pa.shape[p].on_anchors ? L->n_anchor : L->n_corr;
     pa.bm[p] = slot < PLAN_TC ? G_BM : tc_tile_rows(op);
     pa.bn[p] = slot < PLAN_TC ? G_BN : tc_tile_cols();
+    if (L->ct && slot == PLAN_TC + OP_UP_U) {
+      // the fused correction + SwiGLU kernel takes this slot: tiles of 128
+      // cluster rows x CT_CW d_ff columns over the anchors
+      pa.shape[p] = OpShape{L->I, 0, 0, 0, 1, 1};
+      pa.items[p] = L->d_anchors;
+      pa.n_items[p] = L->n_anchor;
+      pa.bm[p] = 128;
+      pa.bn[p] = CT_CW;
+    }
   }
   return pa;
 }

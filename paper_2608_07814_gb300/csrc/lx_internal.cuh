@@ -246,7 +246,15 @@ struct TcLaunch {
   int unmet_wait;            // lx_wait_site whose wait is made to run out (test hook), 0 = none
   int bm;                    // tile rows: 128 or 256 (tc_tile_rows of the op)
   int epi;                   // epilogue warps: 4 or 8
+  // optional output remap (bf16 outputs): row r of the tile plan is stored at
+  // row row_map[r], columns shifted by node_col[node] (null: identity)
+  const int* row_map;
+  const int* node_col;
 };
+
+// Fused correction + SwiGLU of flat layers (every correction node a direct
+// child of an anchor): children per anchor at most CT_MAX_CH.
+constexpr int CT_MAX_CH = 7;
 
 // ---------------------------------------------------------------------------
 // device workspace of one forward
@@ -300,6 +308,16 @@ struct Workspace {
   float* ysplit = nullptr;
   long split_rows = 0;
   int* err = nullptr;           // device error word
+  // fused correction + SwiGLU (flat layers): per anchor row a, the gates
+  // al_g[a][0] (the dominant's, 0 if not selected) and al_g[a][1 + j] (child
+  // slot j's), the child rows al_row[a][j] (-1: not selected), the anchor row
+  // of every child row (rho2al), and the children's x V products aligned to
+  // the anchor rows: Pal[a][j * 2 rmax + (0..2r)]
+  float* al_g = nullptr;
+  int* al_row = nullptr;
+  int* rho2al = nullptr;
+  __nv_bfloat16* Pal = nullptr;
+  CUtensorMap* pamap = nullptr;  // [2] TMA maps of Pal and of hb (128-row boxes)
 };
 
 struct ProfRec {
@@ -341,6 +359,11 @@ struct lx_layer {
   bool pdl = true;                  // programmatic dependent launch between kernels
   unsigned long long wait_cycles = 0;  // bound of the kernels' device-side waits (0: default)
   int unmet_wait = 0;               // lx_wait_site made to run out (test hook), 0 = none
+  // fused correction + SwiGLU on the tensor-core path (flat layers)
+  bool ct = false;
+  int ct_nch = 0;                   // most children of an anchor (table stride)
+  int* d_child = nullptr;           // [N][CT_MAX_CH] an anchor's children in node order, -1 padded
+  int* d_child_col = nullptr;       // [N] column of a child's slot in Pal (j * 2 rmax), 0 for anchors
   std::vector<lx::ProfRec> prof;
   std::vector<cudaEvent_t> event_pool;
 };
@@ -438,6 +461,14 @@ int tc_tile_tokens();  // rows of the TMA boxes of the tensor-core A operands
 int tc_tile_cols();
 int tc_tile_rows(int op);  // token rows of a tensor-core tile of op (its tile plan)
 lx_status launch_tc(lx_layer* L, const TcLaunch& P, cudaStream_t s, const char* name);
+// fused correction + SwiGLU (flat layers): the per-anchor-row gate / row
+// tables, then the fused kernel over (anchor, 128-row block, 64 d_ff columns)
+lx_status launch_ct_meta(lx_layer* L, int T, int k, cudaStream_t s);
+lx_status launch_ct_swiglu(lx_layer* L, cudaStream_t s);
+constexpr int CT_CW = 64;  // d_ff columns of a fused tile
+// row strides (4-byte words, 16-byte rows) of the per-anchor-row tables
+inline int ct_gstride(const lx_layer* L) { return (1 + L->ct_nch + 3) / 4 * 4; }
+inline int ct_rstride(const lx_layer* L) { return (L->ct_nch + 3) / 4 * 4; }
 lx_status launch_stream(lx_layer* L, const StreamLaunch& P, cudaStream_t s, const char* name);
 // plans = false: skip the generic GEMMs' tile plans (not read by the
 // streaming kernels or by lx_get_buckets)

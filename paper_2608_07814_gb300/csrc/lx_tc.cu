@@ -357,11 +357,15 @@ k_tc_gemm(const __grid_constant__ TcLaunch P) {
       tc_fence_after();
       const TcTile t = eslot[b];
       if (t.BN < 0) break;
-      const bool tile_ok = t.tok0 >= 0 && (long)t.grp * t.Ng + t.row0 + t.BN <= P.ldo;
-      const long col0 = (long)t.grp * t.Ng + t.row0;
+      const long col0 = (long)t.grp * t.Ng + t.row0 + (P.node_col ? P.node_col[t.node] : 0);
+      const bool tile_ok = t.tok0 >= 0 && col0 + t.BN <= P.ldo;
       const int cq = lane & 7;
       for (int h = 0; h < NH && 128 * h < t.M; ++h) {
       const uint32_t acc = tmem + (b * NH + h) * TC_ACC_COLS;
+      // output rows of this warp's 32 tile rows (remapped when row_map is set)
+      long orow_l = (long)t.tok0 + 128 * h + 32 * ew + lane;
+      if (P.row_map)
+        orow_l = (32 * ew + lane + 128 * h < t.M && orow_l < P.rows_cap) ? P.row_map[orow_l] : -1;
       if (P.out_f32) {
         for (int c0 = 32 * eh; c0 < t.BN; c0 += 32 * ESTEP) {
           float v[32];
@@ -416,8 +420,8 @@ k_tc_gemm(const __grid_constant__ TcLaunch P) {
           for (int j = 0; j < 8; ++j) {
             const int rr = 4 * j + (lane >> 3);
             const int m = 128 * h + 32 * ew + rr;
-            const long grow = (long)t.tok0 + m;
-            if (tile_ok && m < t.M && grow < P.rows_cap) {
+            const long grow = __shfl_sync(0xffffffffu, orow_l, rr);
+            if (tile_ok && m < t.M && grow >= 0 && grow < P.rows_cap) {
               const uint4 u4 = *reinterpret_cast<const uint4*>(stg + rr * TC_EPI_LD + 4 * cq);
               *reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(P.out) + (size_t)grow * P.ldo +
                                         col0 + c0 + 8 * cq) = u4;
@@ -510,6 +514,8 @@ static TcLaunch tc_op(lx_layer* L, int op, const CUtensorMap* xmap, int xcol, vo
   P.wait_cycles = wait_limit(L);
   P.unmet_wait = L->unmet_wait;
   P.rows_cap = w.rows_cap;
+  P.row_map = nullptr;
+  P.node_col = nullptr;
   return P;
 }
 
@@ -565,11 +571,22 @@ lx_status launch_tc_experts(lx_layer* L, const void* x, int T, int k, void* y, c
   }
   LX_TRY(run(tc_op(L, OP_UP_ANCHOR, w.gmap, 0, w.hb, 2 * I, false, 0),
              "tc_up_anchor"));
-  LX_TRY(run(tc_op(L, OP_UP_V, w.gmap, 0, w.Pb, 2 * rmax, false, 1),
-             "tc_up_V"));
-  LX_TRY(run(tc_op(L, OP_UP_U, w.xmaps + 0, 0, w.hb, 2 * I, false, 2),
-             "tc_up_U"));
-  LX_TRY(launch_swiglu(L, T, k, true, s));
+  if (L->ct) {
+    // flat layers: the members' x V rows land aligned to their cluster's rows,
+    // and one fused kernel adds the corrections and applies the SwiGLU
+    LX_TRY(launch_ct_meta(L, T, k, s));
+    TcLaunch pv = tc_op(L, OP_UP_V, w.gmap, 0, w.Pal, (long)L->ct_nch * 2 * rmax, false, 1);
+    pv.row_map = w.rho2al;
+    pv.node_col = L->d_child_col;
+    LX_TRY(run(pv, "tc_up_V"));
+    LX_TRY(launch_ct_swiglu(L, s));
+  } else {
+    LX_TRY(run(tc_op(L, OP_UP_V, w.gmap, 0, w.Pb, 2 * rmax, false, 1),
+               "tc_up_V"));
+    LX_TRY(run(tc_op(L, OP_UP_U, w.xmaps + 0, 0, w.hb, 2 * I, false, 2),
+               "tc_up_U"));
+    LX_TRY(launch_swiglu(L, T, k, true, s));
+  }
   LX_TRY(run(tc_op(L, OP_DN_ANCHOR, w.xmaps + 1, 0, w.yb, H, false, 3),
              "tc_dn_anchor"));
   LX_TRY(run(tc_op(L, OP_DN_V, w.xmaps + 1, 0, w.Qb, rmax, false, 4),
