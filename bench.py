@@ -218,6 +218,8 @@ def kernel_flops(name, st, src):
         # products (the work tc_up_U does on the unfused path)
         "ct_swiglu": 2 * rr * 2 * I,
         "tc_dn_anchor": 2 * Ra * H * I,
+        # flat layers: the members' Q Ud^T join the anchor's down tile along K
+        "tc_dn_anchor_U": 2 * Ra * H * I + 2 * rr * H,
         "tc_dn_V": 2 * rr * I,
         "tc_dn_U": 2 * rr * H,
     }

@@ -167,7 +167,8 @@ static lx_status ensure_workspace(lx_layer* L, int T, int k, cudaStream_t s) {
       {(void**)&w.al_row, L->ct ? sizeof(int) * Rmax * ct_rstride(L) : 0},
       {(void**)&w.rho2al, L->ct ? sizeof(int) * Rmax : 0},
       {(void**)&w.Pal, L->ct ? (size_t)2 * Rmax * L->ct_nch * 2 * rmax : 0},
-      {(void**)&w.pamap, L->ct ? 2 * sizeof(CUtensorMap) : 0},
+      {(void**)&w.Qal, L->ct ? (size_t)2 * Rmax * L->ct_nch * rmax : 0},
+      {(void**)&w.pamap, L->ct ? 3 * sizeof(CUtensorMap) : 0},
   };
   size_t total = 0;
   for (auto& it : items) total += align_up(it.bytes, 256);
@@ -221,12 +222,13 @@ static lx_status ensure_workspace(lx_layer* L, int T, int k, cudaStream_t s) {
     if (e != cudaSuccess) return cuda_fail(e, "copy activation maps");
   }
   if (L->ct) {
-    CUtensorMap pm[2];
+    CUtensorMap pm[3];
     std::memset(pm, 0, sizeof(pm));
     if (!encode_rows_map(&pm[0], w.Pal, Rmax, (long)L->ct_nch * 2 * rmax, tc_tile_tokens()) ||
-        !encode_rows_map(&pm[1], w.hb, Rmax, 2L * L->I, tc_tile_tokens()))
-      return fail(LX_ERR_CUDA, "cuTensorMapEncodeTiled(Pal, h) failed");
-    e = cudaMemcpyAsync(w.pamap, pm, 2 * sizeof(CUtensorMap), cudaMemcpyHostToDevice, s);
+        !encode_rows_map(&pm[1], w.hb, Rmax, 2L * L->I, tc_tile_tokens()) ||
+        !encode_rows_map(&pm[2], w.Qal, Rmax, (long)L->ct_nch * rmax, tc_tile_tokens()))
+      return fail(LX_ERR_CUDA, "cuTensorMapEncodeTiled(Pal, h, Qal) failed");
+    e = cudaMemcpyAsync(w.pamap, pm, 3 * sizeof(CUtensorMap), cudaMemcpyHostToDevice, s);
     if (e == cudaSuccess) e = cudaStreamSynchronize(s);
     if (e != cudaSuccess) return cuda_fail(e, "copy Pal map");
   }
@@ -551,7 +553,8 @@ extern "C" lx_status lx_load_compressed_layer(const lx_layer_desc* d, const void
   // children of every anchor (fused correction + SwiGLU of flat layers): a
   // layer qualifies when every correction node is a direct child of an anchor
   // and no anchor has more than CT_MAX_CH children
-  std::vector<int> child((size_t)L->N * CT_MAX_CH, -1), child_col(L->N, 0), nchild(L->N, 0);
+  std::vector<int> child((size_t)L->N * CT_MAX_CH, -1), child_col(L->N, 0), child_qcol(L->N, 0);
+  std::vector<int> nchild(L->N, 0);
   bool flat = L->max_depth <= 2 && L->n_corr > 0;
   for (int n = 0; n < L->N && flat; ++n) {
     const int p = L->parent[n];
@@ -562,6 +565,7 @@ extern "C" lx_status lx_load_compressed_layer(const lx_layer_desc* d, const void
     }
     child[(size_t)p * CT_MAX_CH + nchild[p]] = n;
     child_col[n] = nchild[p] * 2 * std::max(1, L->max_rank);
+    child_qcol[n] = nchild[p] * std::max(1, L->max_rank);
     ++nchild[p];
   }
   L->ct_nch = 0;
@@ -572,9 +576,11 @@ extern "C" lx_status lx_load_compressed_layer(const lx_layer_desc* d, const void
     L->ct = flat && L->tiled && !(env && env[0] == '0');
   }
   const size_t o_child = tadd(4 * child.size()), o_ccol = tadd(4 * (size_t)L->N);
+  const size_t o_cqcol = tadd(4 * (size_t)L->N);
   std::vector<char> tb(toff, 0);
   std::memcpy(tb.data() + o_child, child.data(), 4 * child.size());
   std::memcpy(tb.data() + o_ccol, child_col.data(), 4 * (size_t)L->N);
+  std::memcpy(tb.data() + o_cqcol, child_qcol.data(), 4 * (size_t)L->N);
   std::memcpy(tb.data() + o_rank, L->rank.data(), 4 * L->N);
   std::memcpy(tb.data() + o_paths, paths.data(), 4 * paths.size());
   std::memcpy(tb.data() + o_plen, plen.data(), 4 * L->E);
@@ -598,6 +604,7 @@ extern "C" lx_status lx_load_compressed_layer(const lx_layer_desc* d, const void
   L->d_w_dnU = (const void**)(tbase + o_p3);
   L->d_child = (int*)(tbase + o_child);
   L->d_child_col = (int*)(tbase + o_ccol);
+  L->d_child_qcol = (int*)(tbase + o_cqcol);
   ce = cudaMemcpyAsync(L->tables, tb.data(), toff, cudaMemcpyHostToDevice, s);
   if (ce == cudaSuccess) ce = cudaStreamSynchronize(s);
   if (ce != cudaSuccess) return cleanup(cuda_fail(ce, "copy tables"));

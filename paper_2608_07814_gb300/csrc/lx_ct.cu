@@ -81,6 +81,8 @@ struct CtLaunch {
   const CUtensorMap* hmap;   // anchor pre-activations h [R][2I], 128-row boxes
   int pslot;               // columns of a child's slot in Pal (2 rmax)
   __nv_bfloat16* z;        // [R][I]
+  __nv_bfloat16* qal;      // [R][qld]: child slot j at columns j * qslot (zeroed here
+  int qld, qslot;          //  where the row did not select the child)
   const float* al_g;       // [R][gstride]: dominant's gate, then the children's
   const int* al_row;       // [R][rstride]: the children's rows
   int gstride, rstride;    // multiples of 4 (16-byte rows), at most CT_TAB_STRIDE
@@ -517,6 +519,16 @@ __global__ void __launch_bounds__(CT_THREADS, 1) k_ct_swiglu(const __grid_consta
       __syncwarp();
       if (lane == 0) mbar_arrive(hempty0 + 8 * hb);
       ++nt;
+      // the down side sums every child slot of a cluster row: the slots of
+      // children this row did not select are zeroed (once, by the first chunk)
+      if (t.q == 0 && cs == 0 && valid) {
+#pragma unroll
+        for (int jj = 0; jj < CT_MAX_CH; ++jj) {
+          if (jj >= t.nch || rm[jj] >= 0) continue;
+          uint4* q = reinterpret_cast<uint4*>(P.qal + (size_t)a * P.qld + (size_t)jj * P.qslot);
+          for (int i = 0; i < t.rk[jj] / 8; ++i) q[i] = make_uint4(0u, 0u, 0u, 0u);
+        }
+      }
       // z starts with the dominant's own gated SwiGLU (if the token selected it)
       F2 zr[CT_EC / 2];
       if (__any_sync(0xffffffffu, gd != 0.f)) {
@@ -703,6 +715,9 @@ lx_status launch_ct_swiglu(lx_layer* L, cudaStream_t s) {
   P.hmap = w.pamap + 1;
   P.pslot = 2 * std::max(1, L->max_rank);
   P.z = w.zb;
+  P.qal = w.Qal;
+  P.qslot = std::max(1, L->max_rank);
+  P.qld = L->ct_nch * P.qslot;
   P.al_g = w.al_g;
   P.al_row = w.al_row;
   P.gstride = ct_gstride(L);

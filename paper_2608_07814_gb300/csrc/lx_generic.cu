@@ -628,7 +628,8 @@ k_swiglu_warp(const float* __restrict__ topk_w, const int* __restrict__ node_row
 template <typename TP, typename TY, int CPL, bool SPLIT>
 __global__ void __launch_bounds__(WT_WARPS * 32, 2)
 k_combine_warp(const int* __restrict__ node_row, int k, int D, const TP* __restrict__ ypart,
-               int H, TY* __restrict__ y, int T, int cols_per_item, const SplitParts ys) {
+               int H, TY* __restrict__ y, int T, int cols_per_item, const SplitParts ys,
+               int anchors_only) {
   __shared__ WarpRows wrs[WT_WARPS];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   WarpRows& wr = wrs[warp];
@@ -647,6 +648,56 @@ k_combine_warp(const int* __restrict__ node_row, int k, int D, const TP* __restr
     const int c_end = min(H, c_begin + cols_per_item);
     warp_token_rows(first ? v_pre : (lane < kD ? node_row[(size_t)t * kD + lane] : -1), kD, D, wr);
     const int nd = wr.nd;
+    if constexpr (!SPLIT && CPL == 8 && sizeof(TP) == 2) {
+      if (anchors_only) {
+        // only the anchor rows (their down tiles already hold the members'
+        // corrections), ascending; four column passes' 16-byte loads of a
+        // batch of four rows in flight at once, each column summed in row order
+        for (int c0 = c_begin + CPL * lane; c0 < c_end; c0 += 4 * 32 * CPL) {
+          Cols<CPL> acc[4];
+#pragma unroll
+          for (int u = 0; u < 4; ++u)
+#pragma unroll
+            for (int i = 0; i < CPL; ++i) acc[u].v[i] = 0.f;
+          for (unsigned am = wr.anchor_rows; am;) {
+            int rq[4];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              rq[q] = -1;
+              if (am) {
+                rq[q] = wr.drow[__ffs(am) - 1];
+                am &= am - 1u;
+              }
+            }
+            uint4 v[4][4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+#pragma unroll
+              for (int q = 0; q < 4; ++q)
+                if (rq[q] >= 0 && c0 + u * 32 * CPL < c_end)
+                  v[u][q] = __ldg(reinterpret_cast<const uint4*>(ypart + (size_t)rq[q] * H + c0 +
+                                                                 u * 32 * CPL));
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+#pragma unroll
+              for (int q = 0; q < 4; ++q)
+                if (rq[q] >= 0 && c0 + u * 32 * CPL < c_end) {
+                  const uint32_t w4[4] = {v[u][q].x, v[u][q].y, v[u][q].z, v[u][q].w};
+#pragma unroll
+                  for (int i = 0; i < 4; ++i) {
+                    acc[u].v[2 * i] += __uint_as_float(w4[i] << 16);
+                    acc[u].v[2 * i + 1] += __uint_as_float(w4[i] & 0xFFFF0000u);
+                  }
+                }
+          }
+#pragma unroll
+          for (int u = 0; u < 4; ++u)
+            if (c0 + u * 32 * CPL < c_end) st_cols<TY, CPL>(y + (size_t)t * H + c0 + u * 32 * CPL, acc[u]);
+        }
+        __syncwarp();
+        continue;
+      }
+    }
     for (int c = c_begin + CPL * lane; c < c_end; c += 32 * CPL) {
       Cols<CPL> acc;
 #pragma unroll
@@ -782,13 +833,13 @@ static void launch_swiglu_warp(lx_layer* L, int T, int k, const TH* h, TZ* z, cu
 // every batch size)
 template <typename TP, typename TY>
 static void launch_combine_warp(lx_layer* L, int T, int k, const TP* ypart, TY* y, cudaStream_t s,
-                                const SplitParts& ys) {
+                                const SplitParts& ys, bool anchors_only = false) {
   Workspace& w = L->ws;
   if (ys.splits > 1) {
     const int cols = warp_item_cols(L, T, L->H, 128);
     const int grid = warp_grid(L, T, L->H, cols);
     launch_k(L, k_combine_warp<TP, TY, 4, true>, grid, WT_WARPS * 32, 0, s, w.node_row, k,
-             L->max_depth, ypart, L->H, y, T, cols, ys);
+             L->max_depth, ypart, L->H, y, T, cols, ys, 0);
     return;
   }
   // eight columns per lane (16-byte bf16 loads): half the per-element address
@@ -796,7 +847,7 @@ static void launch_combine_warp(lx_layer* L, int T, int k, const TP* ypart, TY* 
   const int cols = warp_item_cols(L, T, L->H, 256);
   const int grid = warp_grid(L, T, L->H, cols);
   launch_k(L, k_combine_warp<TP, TY, 8, false>, grid, WT_WARPS * 32, 0, s, w.node_row, k,
-           L->max_depth, ypart, L->H, y, T, cols, ys);
+           L->max_depth, ypart, L->H, y, T, cols, ys, anchors_only ? 1 : 0);
 }
 
 lx_status launch_swiglu(lx_layer* L, int T, int k, bool bf16, cudaStream_t s, SplitParts hs) {
@@ -823,12 +874,14 @@ lx_status launch_swiglu(lx_layer* L, int T, int k, bool bf16, cudaStream_t s, Sp
 }
 
 lx_status launch_combine(lx_layer* L, int T, int k, void* y, bool bf16, cudaStream_t s,
-                         SplitParts ys) {
+                         SplitParts ys, bool anchors_only) {
   Workspace& w = L->ws;
   ProfScope ps(L, s, "combine");
+  if (anchors_only && !(bf16 && ys.splits <= 1 && warp_kernels_fit(L, k)))
+    return fail(LX_ERR_STATE, "anchor-row combine needs the bf16 warp form");
   if (warp_kernels_fit(L, k)) {
     if (bf16)
-      launch_combine_warp(L, T, k, L->ws.yb, static_cast<__nv_bfloat16*>(y), s, ys);
+      launch_combine_warp(L, T, k, L->ws.yb, static_cast<__nv_bfloat16*>(y), s, ys, anchors_only);
     else if (L->dtype == LX_BF16)
       launch_combine_warp(L, T, k, L->ws.ypart, static_cast<__nv_bfloat16*>(y), s, ys);
     else

@@ -250,6 +250,14 @@ struct TcLaunch {
   // row row_map[r], columns shifted by node_col[node] (null: identity)
   const int* row_map;
   const int* node_col;
+  // optional K concatenation (anchor down tiles of flat layers): after its own
+  // K, an anchor tile runs over each child c of kc_child[node] (CT_MAX_CH per
+  // node, -1 padded) for rank(c) more: A from kc_xmap at columns j * kc_slot
+  // (the child's slot j), B from kc_wmaps[c]
+  const int* kc_child;
+  const CUtensorMap* kc_wmaps;
+  const CUtensorMap* kc_xmap;
+  int kc_slot;
 };
 
 // Fused correction + SwiGLU of flat layers (every correction node a direct
@@ -317,7 +325,8 @@ struct Workspace {
   int* al_row = nullptr;
   int* rho2al = nullptr;
   __nv_bfloat16* Pal = nullptr;
-  CUtensorMap* pamap = nullptr;  // [2] TMA maps of Pal and of hb (128-row boxes)
+  __nv_bfloat16* Qal = nullptr;  // [R][nch * rmax] the children's z Vd rows, aligned likewise
+  CUtensorMap* pamap = nullptr;  // [3] TMA maps of Pal, hb and Qal (128-row boxes)
 };
 
 struct ProfRec {
@@ -364,6 +373,7 @@ struct lx_layer {
   int ct_nch = 0;                   // most children of an anchor (table stride)
   int* d_child = nullptr;           // [N][CT_MAX_CH] an anchor's children in node order, -1 padded
   int* d_child_col = nullptr;       // [N] column of a child's slot in Pal (j * 2 rmax), 0 for anchors
+  int* d_child_qcol = nullptr;      // [N] column of a child's slot in Qal (j * rmax)
   std::vector<lx::ProfRec> prof;
   std::vector<cudaEvent_t> event_pool;
 };
@@ -453,8 +463,10 @@ bool warp_kernels_fit(const lx_layer* L, int k);
 // all bf16); false: the generic form (fp32 h, z, ypart)
 lx_status launch_swiglu(lx_layer* L, int T, int k, bool bf16, cudaStream_t s,
                         SplitParts hs = SplitParts());
+// anchors_only: sum only the anchor rows of each token (their down tiles
+// already hold the members' corrections)
 lx_status launch_combine(lx_layer* L, int T, int k, void* y, bool bf16, cudaStream_t s,
-                         SplitParts ys = SplitParts());
+                         SplitParts ys = SplitParts(), bool anchors_only = false);
 lx_status launch_fast_experts(lx_layer* L, const void* x, int T, int k, void* y, cudaStream_t s);
 lx_status launch_tc_experts(lx_layer* L, const void* x, int T, int k, void* y, cudaStream_t s);
 int tc_tile_tokens();  // rows of the TMA boxes of the tensor-core A operands

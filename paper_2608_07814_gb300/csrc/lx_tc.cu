@@ -99,6 +99,14 @@ __device__ __forceinline__ void tc_decode_warp(const TcLaunch& P, int tile, TcTi
   const int b0 = __ldg(P.node_off + n), b1 = __ldg(P.node_off + n + 1);
   t.Ng = P.shape.n_const + P.shape.n_rank * r;
   t.K = P.shape.k_const + P.shape.k_rank * r;
+  if (P.kc_child) {
+    // K concatenation: the anchor's children's rank-r products follow its own K
+    const int c = lane < CT_MAX_CH ? __ldg(P.kc_child + (size_t)n * CT_MAX_CH + lane) : -1;
+    int rc = c >= 0 ? __ldg(P.rank + c) : 0;
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) rc += __shfl_xor_sync(0xffffffffu, rc, o);
+    t.K += rc;
+  }
   const int ncol = (t.Ng + TC_BN - 1) / TC_BN;
   const int per_tb = ncol * P.shape.groups;
   const int tb = local / per_tb, rem = local % per_tb;
@@ -188,6 +196,9 @@ k_tc_gemm(const __grid_constant__ TcLaunch P) {
       const int nkb = (t.K + TC_BK - 1) / TC_BK;
       const int rt0 = (t.grp * t.Ng + t.row0) / 64;  // first 64-row weight tile
       const int nbox = (t.BN + 63) / 64;
+      // K concatenation: k-blocks from kb_own on read child cj's k-block ckb
+      const int kb_own = P.kc_child ? P.shape.k_const / TC_BK : nkb;
+      int cj = 0, ckb = 0, cnode = -1, cnkb = 0;
       for (int kb = 0; kb < nkb; ++kb, ++it) {
         const uint32_t s = it % TC_STAGES;
         int good = 1;
@@ -200,12 +211,29 @@ k_tc_gemm(const __grid_constant__ TcLaunch P) {
             const int nh = (NH == 2 && t.M > 128) ? 2 : 1;
             mbar_expect_tx(full0 + 8 * s, nbox * 8192 + nh * 128 * TC_BK * 2);
             const uint32_t a_s = smem_base + s * TC_STAGE_BYTES, b_s = a_s + TC_A_BYTES;
-            for (int b = 0; b < nbox; ++b)
-              tma_load_4d(b_s + b * 8192, P.wmaps + t.node, 0, 0, kb, rt0 + b, full0 + 8 * s);
-            for (int h = 0; h < nh; ++h)
-              tma_load_2d(a_s + h * 128 * TC_BK * 2, P.xmap,
-                          (int)(t.grp * t.K) + kb * TC_BK + P.xcol, t.tok0 + 128 * h,
-                          full0 + 8 * s);
+            if (kb < kb_own) {
+              for (int b = 0; b < nbox; ++b)
+                tma_load_4d(b_s + b * 8192, P.wmaps + t.node, 0, 0, kb, rt0 + b, full0 + 8 * s);
+              for (int h = 0; h < nh; ++h)
+                tma_load_2d(a_s + h * 128 * TC_BK * 2, P.xmap,
+                            (int)(t.grp * t.K) + kb * TC_BK + P.xcol, t.tok0 + 128 * h,
+                            full0 + 8 * s);
+            } else {
+              if (cnode < 0) {
+                cnode = __ldg(P.kc_child + (size_t)t.node * CT_MAX_CH + cj);
+                cnkb = __ldg(P.rank + cnode) / TC_BK;
+              }
+              for (int b = 0; b < nbox; ++b)
+                tma_load_4d(b_s + b * 8192, P.kc_wmaps + cnode, 0, 0, ckb, rt0 + b, full0 + 8 * s);
+              for (int h = 0; h < nh; ++h)
+                tma_load_2d(a_s + h * 128 * TC_BK * 2, P.kc_xmap, cj * P.kc_slot + ckb * TC_BK,
+                            t.tok0 + 128 * h, full0 + 8 * s);
+              if (++ckb == cnkb) {
+                ckb = 0;
+                ++cj;
+                cnode = -1;
+              }
+            }
           }
         }
         good = __shfl_sync(0xffffffffu, good, 0);
@@ -516,6 +544,10 @@ static TcLaunch tc_op(lx_layer* L, int op, const CUtensorMap* xmap, int xcol, vo
   P.rows_cap = w.rows_cap;
   P.row_map = nullptr;
   P.node_col = nullptr;
+  P.kc_child = nullptr;
+  P.kc_wmaps = nullptr;
+  P.kc_xmap = nullptr;
+  P.kc_slot = 0;
   return P;
 }
 
@@ -580,6 +612,20 @@ lx_status launch_tc_experts(lx_layer* L, const void* x, int T, int k, void* y, c
     pv.node_col = L->d_child_col;
     LX_TRY(run(pv, "tc_up_V"));
     LX_TRY(launch_ct_swiglu(L, s));
+    // the members' down corrections join their anchor's down tile along K:
+    // [z | Q_1 | Q_2 | ...] . [Wd | Ud_1 | Ud_2 | ...]^T, Q stored aligned to
+    // the cluster's rows (zero where a member is not selected)
+    TcLaunch qv = tc_op(L, OP_DN_V, w.xmaps + 1, 0, w.Qal, (long)L->ct_nch * rmax, false, 4);
+    qv.row_map = w.rho2al;
+    qv.node_col = L->d_child_qcol;
+    LX_TRY(run(qv, "tc_dn_V"));
+    TcLaunch dn = tc_op(L, OP_DN_ANCHOR, w.xmaps + 1, 0, w.yb, H, false, 3);
+    dn.kc_child = L->d_child;
+    dn.kc_wmaps = L->d_tmaps + (size_t)OP_DN_U * L->N;
+    dn.kc_xmap = w.pamap + 2;
+    dn.kc_slot = (int)rmax;
+    LX_TRY(run(dn, "tc_dn_anchor_U"));
+    return launch_combine(L, T, k, y, true, s, SplitParts(), /*anchors_only=*/true);
   } else {
     LX_TRY(run(tc_op(L, OP_UP_V, w.gmap, 0, w.Pb, 2 * rmax, false, 1),
                "tc_up_V"));
