@@ -486,12 +486,12 @@ k_tc_gemm(const __grid_constant__ TcLaunch P) {
 
 int tc_tile_tokens() { return 128; }
 int tc_tile_cols() { return TC_BN; }
-// The anchor gate/up product (K = d_model, anchor buckets of hundreds of
-// rows) takes 256-row tiles; the others 128 (measured at the Qwen3-shaped
-// prefill of 8192: tc_up_anchor 156 -> 146 us with 256 rows, while x V, whose
-// member buckets are a few hundred rows, loses more to half-empty tiles and a
-// single wave than it gains).
-int tc_tile_rows(int op) { return op == OP_UP_ANCHOR ? 256 : 128; }
+// The anchor products (anchor buckets of hundreds of rows) take 256-row
+// tiles; the others 128 (measured at the Qwen3-shaped prefill of 8192:
+// tc_up_anchor 156 -> 146 us and the down tile with the members' corrections
+// 142 -> 128 us with 256 rows, while x V, whose member buckets are a few
+// hundred rows, loses more to half-empty tiles and a single wave than it gains).
+int tc_tile_rows(int op) { return (op == OP_UP_ANCHOR || op == OP_DN_ANCHOR) ? 256 : 128; }
 
 template <int BM, int EPI>
 static int tc_smem_bytes() {
