@@ -93,6 +93,20 @@ static PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
   return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
 }
 
+bool encode_bf16_2d(CUtensorMap* m, const void* base, long inner, long outer, int box_inner,
+                    int box_outer) {
+  auto encode = get_encode();
+  if (!encode) return false;
+  const cuuint64_t dims[2] = {(cuuint64_t)inner, (cuuint64_t)outer};
+  const cuuint64_t strides[1] = {(cuuint64_t)inner * 2};
+  const cuuint32_t box[2] = {(cuuint32_t)box_inner, (cuuint32_t)box_outer};
+  const cuuint32_t estr[2] = {1, 1};
+  return encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
+                box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) ==
+         CUDA_SUCCESS;
+}
+
 // TMA map of a bf16 activation buffer [rows][ld] read as box_rows x 64-column
 // boxes with the 128-byte swizzle (an A operand whose rows are already in
 // node-row order)

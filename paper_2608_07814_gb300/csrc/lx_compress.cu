@@ -26,6 +26,7 @@
 // float64 rate is a small fraction of its fp32 rate on this GPU.
 #include <algorithm>
 #include <cmath>
+#include <type_traits>
 
 #include "lx_internal.cuh"
 
@@ -463,6 +464,7 @@ size_t al256(size_t v) { return (v + 255) / 256 * 256; }
 struct CompressWs {
   float *y0, *y1, *z0, *z1, *T, *Wu, *Wv, *L1, *L2, *Xg, *Mt, *Wt, *MWn, *Wn, *Mg, *Wg;
   double *G, *sig64;
+  char* tc;  // the tensor-core residual products' scratch (bf16 weights)
   size_t bytes;
 };
 
@@ -495,6 +497,7 @@ CompressWs carve(char* base, long rows, long cols, long l, long r) {
   w.Wg = (float*)take(4 * Lp * Lp);
   w.G = (double*)take(8 * l * l);
   w.sig64 = (double*)take(8 * l);
+  w.tc = take(res_tc_workspace(rows, cols, l));
   w.bytes = off;
   return w;
 }
@@ -511,8 +514,23 @@ template <typename TW>
 lx_status run_compress(int rows, int cols, const TW* Wd, const TW* Wm, const float* omega, int l,
                        int r, int q, float* U, float* V, float* sigma, const CompressWs& w,
                        int dev, cudaStream_t s) {
+  int num_sms = 0;
+  LX_CUDA(cudaDeviceGetAttribute(&num_sms, cudaDevAttrMultiProcessorCount, dev));
+  // bf16 weights: the residual products R X and R^T X on the tensor cores
+  constexpr bool bf16_w = std::is_same<TW, __nv_bfloat16>::value;
+  const bool res_tc = bf16_w && res_tc_fits(rows, cols, l);
+  lx_status tc_status = LX_OK;
   auto gemm = [&](int mode, const float* X, const float* B, float* C, int M, int N, int K) {
     const dim3 grid((N + CG_TILE - 1) / CG_TILE, (M + CG_TILE - 1) / CG_TILE);
+    if constexpr (bf16_w) {
+      if (res_tc && (mode == A_RES || mode == A_RES_T)) {
+        const lx_status st = res_gemm_tc(mode == A_RES_T, reinterpret_cast<const __nv_bfloat16*>(Wm),
+                                         reinterpret_cast<const __nv_bfloat16*>(Wd), rows, cols, B, N,
+                                         C, w.tc, num_sms, dev, s);
+        if (st != LX_OK) tc_status = st;
+        return;
+      }
+    }
     if (mode == A_RES)
       k_cgemm<TW, A_RES><<<grid, CG_THREADS, 0, s>>>(Wm, Wd, nullptr, cols, B, C, M, N, K);
     else if (mode == A_RES_T)
@@ -564,7 +582,7 @@ lx_status run_compress(int rows, int cols, const TW* Wd, const TW* Wm, const flo
   gemm(A_F32, w.z0, w.Wv, V, cols, r, l);   // V_r S^(1/2)
   k_sign<<<r, 256, 0, s>>>(U, V, rows, cols, r);
   LX_CUDA(cudaGetLastError());
-  return LX_OK;
+  return tc_status;
 }
 }  // namespace
 }  // namespace lx

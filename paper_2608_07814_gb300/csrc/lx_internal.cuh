@@ -473,6 +473,19 @@ int tc_tile_tokens();  // rows of the TMA boxes of the tensor-core A operands
 int tc_tile_cols();
 int tc_tile_rows(int op);  // token rows of a tensor-core tile of op (its tile plan)
 lx_status launch_tc(lx_layer* L, const TcLaunch& P, cudaStream_t s, const char* name);
+// 2-D TMA map of a row-major bf16 matrix [outer][inner] read as box_inner x
+// box_outer boxes with the 128-byte swizzle
+bool encode_bf16_2d(CUtensorMap* m, const void* base, long inner, long outer, int box_inner,
+                    int box_outer);
+// the residual products of the member compression on the tensor cores
+// (bf16 weights): C [M][N] = R X (transposed = false: M = rows, K = cols) or
+// R^T X (M = cols, K = rows), R = Wm - Wd [rows][cols], X fp32 [K][N]
+constexpr int RES_TC_MAX_SPLITS = 32;
+size_t res_tc_workspace(long rows, long cols, long l);
+bool res_tc_fits(long rows, long cols, long l);
+lx_status res_gemm_tc(bool transposed, const __nv_bfloat16* Wm, const __nv_bfloat16* Wd,
+                      long rows, long cols, const float* X, long N, float* C, char* ws,
+                      int num_sms, int dev, cudaStream_t s);
 // fused correction + SwiGLU (flat layers): the per-anchor-row gate / row
 // tables, then the fused kernel over (anchor, 128-row block, 64 d_ff columns)
 lx_status launch_ct_meta(lx_layer* L, int T, int k, cudaStream_t s);
