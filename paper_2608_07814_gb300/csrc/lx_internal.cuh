@@ -258,6 +258,11 @@ struct TcLaunch {
   const CUtensorMap* kc_wmaps;
   const CUtensorMap* kc_xmap;
   int kc_slot;
+  // optional gathered A rows (in place of xmap): row r of the plan reads row
+  // gather[r] of xsrc [.][ldx] (bf16), copied into shared memory by a warp
+  const int* gather;
+  const __nv_bfloat16* xsrc;
+  long ldx;
 };
 
 // Fused correction + SwiGLU of flat layers (every correction node a direct

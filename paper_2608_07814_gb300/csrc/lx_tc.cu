@@ -118,7 +118,18 @@ __device__ __forceinline__ void tc_decode_warp(const TcLaunch& P, int tile, TcTi
   t.M = min(BM, b1 - t.tok0);
 }
 
-template <int BM, int EPI>
+// cp.async 16-byte copy global -> shared, completion tracked by cp.async groups
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+
+// GATHER: warp 3 fills the A stages with the tile's token rows, gathered from
+// x by row -> token (16-byte cp.async, eight lanes per 128-byte row segment,
+// stored in the 128-byte-swizzled K-major layout the MMA reads); a stage is
+// published once its copies have landed (cp.async.wait_group) and been made
+// visible to the tensor core's async proxy (fence.proxy.async), so no copy of
+// the token rows in node-row order is written to memory first.
+template <int BM, int EPI, bool GATHER>
 __global__ void __launch_bounds__(TcCfg<BM, EPI>::THREADS, 1)
 k_tc_gemm(const __grid_constant__ TcLaunch P) {
   using C = TcCfg<BM, EPI>;
@@ -156,7 +167,7 @@ k_tc_gemm(const __grid_constant__ TcLaunch P) {
     mbar_init(drain, 1);
     for (int q = 0; q < TC_QN; ++q) {
       mbar_init(qfull0 + 8 * q, 1);   // the scheduler's arrival (tile written)
-      mbar_init(qempty0 + 8 * q, 1);  // the producer's arrival (tile read)
+      mbar_init(qempty0 + 8 * q, GATHER ? 2 : 1);  // the producer's (and gather warp's) arrival
     }
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -208,7 +219,7 @@ k_tc_gemm(const __grid_constant__ TcLaunch P) {
           if (good) {
             if (kb == 0) slot[s] = t;
             // a 256-row tile whose rows end within its first half loads one half
-            const int nh = (NH == 2 && t.M > 128) ? 2 : 1;
+            const int nh = GATHER ? 0 : ((NH == 2 && t.M > 128) ? 2 : 1);
             mbar_expect_tx(full0 + 8 * s, nbox * 8192 + nh * 128 * TC_BK * 2);
             const uint32_t a_s = smem_base + s * TC_STAGE_BYTES, b_s = a_s + TC_A_BYTES;
             if (kb < kb_own) {
@@ -241,7 +252,7 @@ k_tc_gemm(const __grid_constant__ TcLaunch P) {
           ok = false;
           break;
         }
-        mbar_arrive(full0 + 8 * s);
+        if (!GATHER) mbar_arrive(full0 + 8 * s);  // else the gather warp's 32 lanes arrive
       }
     }
     if (ok) {
@@ -258,7 +269,7 @@ k_tc_gemm(const __grid_constant__ TcLaunch P) {
       }
       good = __shfl_sync(0xffffffffu, good, 0);
       if (good) {
-        mbar_arrive(full0 + 8 * s);
+        if (!GATHER) mbar_arrive(full0 + 8 * s);
         ++it;
       } else {
         ok = false;
@@ -269,6 +280,91 @@ k_tc_gemm(const __grid_constant__ TcLaunch P) {
       *abort_flag = 1;
     }
     prod_it = it;
+  } else if (GATHER && warp == 3) {
+    // ------------------------------------------------------------ gather
+    // Same tiles and stages as the producer: per stage, rows m = 4 i + r8 of
+    // the tile (lanes 8 r8 .. 8 r8 + 7), 16-byte unit u of the stage's 64-wide
+    // K slice; up to TC_STAGES - 1 stages in flight before the oldest is
+    // published (32 arrivals on its full barrier).
+    const int r8 = lane >> 3, u = lane & 7;
+    uint32_t it = 0, qi = 0, pq = 0;
+    int np = 0;
+    bool ok = true;
+    auto publish_oldest = [&]() {
+      asm volatile("cp.async.wait_group %0;" ::"n"(TC_STAGES - 2) : "memory");
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      mbar_arrive(full0 + 8 * (pq & 0xffu));
+      pq >>= 8;
+      --np;
+    };
+    while (ok) {
+      const uint32_t q = qi % TC_QN;
+      int got = 1;
+      if (lane == 0) got = mbar_wait(qfull0 + 8 * q, (qi / TC_QN) & 1, abort_flag, P.wait_cycles);
+      if (!__shfl_sync(0xffffffffu, got, 0)) {
+        ok = false;
+        break;
+      }
+      __syncwarp();
+      const TcTile t = qslot[q];
+      __syncwarp();
+      if (lane == 0) mbar_arrive(qempty0 + 8 * q);
+      ++qi;
+      if (t.BN < 0) break;
+      int trow[BM / 4];  // token of row 4 i + r8, or -1 past the bucket
+#pragma unroll
+      for (int i = 0; i < BM / 4; ++i) {
+        const int m = 4 * i + r8;
+        trow[i] = (m < t.M && (long)t.tok0 + m < P.rows_cap) ? __ldg(P.gather + t.tok0 + m) : -1;
+      }
+      const int nkb = (t.K + TC_BK - 1) / TC_BK;
+      for (int kb = 0; kb < nkb; ++kb, ++it) {
+        const uint32_t s = it % TC_STAGES;
+        int good = 1;
+        if (lane == 0)
+          good = mbar_wait(empty0 + 8 * s, ((it / TC_STAGES) & 1) ^ 1, abort_flag, P.wait_cycles)
+                     ? 1 : 0;
+        good = __shfl_sync(0xffffffffu, good, 0);
+        if (!good) {
+          ok = false;
+          break;
+        }
+        const uint32_t a_s = smem_base + s * TC_STAGE_BYTES;
+        const __nv_bfloat16* xk = P.xsrc + (size_t)(t.grp * t.K + kb * TC_BK) + 8 * u;
+#pragma unroll
+        for (int i = 0; i < BM / 4; ++i) {
+          const int m = 4 * i + r8;
+          if (trow[i] >= 0)
+            cp_async16(a_s + m * 128 + ((u ^ (m & 7)) << 4), xk + (size_t)trow[i] * P.ldx);
+        }
+        asm volatile("cp.async.commit_group;" ::: "memory");
+        pq |= s << (8 * np);
+        ++np;
+        if (np == TC_STAGES - 1) publish_oldest();
+      }
+    }
+    // the stages still in flight, oldest first, then the sentinel stage
+    asm volatile("cp.async.wait_group 0;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    while (np > 0) {
+      mbar_arrive(full0 + 8 * (pq & 0xffu));
+      pq >>= 8;
+      --np;
+    }
+    if (ok) {
+      const uint32_t s = it % TC_STAGES;
+      int good = 1;
+      if (lane == 0)
+        good = mbar_wait(empty0 + 8 * s, ((it / TC_STAGES) & 1) ^ 1, abort_flag, P.wait_cycles)
+                   ? 1 : 0;
+      good = __shfl_sync(0xffffffffu, good, 0);
+      if (good) mbar_arrive(full0 + 8 * s);
+      else ok = false;
+    }
+    if (!ok && lane == 0) {
+      atomicExch(P.err, LX_ERR_TIMEOUT);
+      *abort_flag = 1;
+    }
   } else if (warp == 2) {
     // ------------------------------------------------------------ scheduler
     // Claims tiles from the launch's counter and decodes them (the plan-prefix
@@ -494,27 +590,35 @@ int tc_tile_cols() { return TC_BN; }
 int tc_tile_rows(int op) { return (op == OP_UP_ANCHOR || op == OP_DN_ANCHOR) ? 256 : 128; }
 
 template <int BM, int EPI>
-static int tc_smem_bytes() {
+static int tc_smem_bytes_() {
   using C = TcCfg<BM, EPI>;
   return C::STAGES * C::STAGE_BYTES + EPI * TC_EPI_BYTES + 8 * (2 * C::STAGES + 7) +
          (C::STAGES + 2 + TC_QN) * (int)sizeof(TcTile) + 16 * TC_QN + 1024;
 }
-
 template <int BM, int EPI>
+static int tc_smem_bytes() { return tc_smem_bytes_<BM, EPI>(); }
+
+template <int BM, int EPI, bool GATHER>
 static lx_status launch_tc_cfg(lx_layer* L, const TcLaunch& P, cudaStream_t s, const char* name) {
   const int smem = tc_smem_bytes<BM, EPI>();
   static bool done[64] = {};
-  LX_CUDA(smem_cap_once((const void*)k_tc_gemm<BM, EPI>, smem, L->device, done));
+  LX_CUDA(smem_cap_once((const void*)k_tc_gemm<BM, EPI, GATHER>, smem, L->device, done));
   ProfScope ps(L, s, name);
-  launch_k(L, k_tc_gemm<BM, EPI>, L->num_sms, TcCfg<BM, EPI>::THREADS, smem, s, P);
+  launch_k(L, k_tc_gemm<BM, EPI, GATHER>, L->num_sms, TcCfg<BM, EPI>::THREADS, smem, s, P);
   LX_CUDA(cudaGetLastError());
   return LX_OK;
 }
 
 lx_status launch_tc(lx_layer* L, const TcLaunch& P, cudaStream_t s, const char* name) {
-  if (P.bm == 256) return launch_tc_cfg<256, 4>(L, P, s, name);
-  if (P.epi == 8) return launch_tc_cfg<128, 8>(L, P, s, name);
-  return launch_tc_cfg<128, 4>(L, P, s, name);
+  const bool g = P.gather != nullptr;
+  if (g && P.kc_child) return fail(LX_ERR_STATE, "gathered A rows with a K concatenation");
+  if (P.bm == 256)
+    return g ? launch_tc_cfg<256, 4, true>(L, P, s, name) : launch_tc_cfg<256, 4, false>(L, P, s, name);
+  if (P.epi == 8) {
+    if (g) return fail(LX_ERR_STATE, "gathered A rows need four epilogue warps");
+    return launch_tc_cfg<128, 8, false>(L, P, s, name);
+  }
+  return g ? launch_tc_cfg<128, 4, true>(L, P, s, name) : launch_tc_cfg<128, 4, false>(L, P, s, name);
 }
 
 static TcLaunch tc_op(lx_layer* L, int op, const CUtensorMap* xmap, int xcol, void* out,
@@ -548,15 +652,20 @@ static TcLaunch tc_op(lx_layer* L, int op, const CUtensorMap* xmap, int xcol, vo
   P.kc_wmaps = nullptr;
   P.kc_xmap = nullptr;
   P.kc_slot = 0;
+  P.gather = nullptr;
+  P.xsrc = nullptr;
+  P.ldx = 0;
   return P;
 }
 
 namespace {
 
-// xg[r] = x[node_tok[r]] for the rows r < R of this forward (R = the node
-// rows, key_off[N]): one warp per row, 16-byte loads and stores.
+// xg[r] = x[node_tok[r]] for the anchor rows r < R of this forward (R = the
+// node rows, key_off[N]; rows of correction nodes are skipped: their products
+// gather their rows themselves): one warp per row, 16-byte loads and stores.
 __global__ void __launch_bounds__(256)
 k_gather_rows(const __nv_bfloat16* __restrict__ x, int H, const int* __restrict__ node_tok,
+              const int* __restrict__ row_node, const int* __restrict__ rank,
               const int* __restrict__ rows_total, long rows_cap, __nv_bfloat16* __restrict__ xg) {
   pdl_wait();
   const long R = min((long)*rows_total, rows_cap);
@@ -566,11 +675,15 @@ k_gather_rows(const __nv_bfloat16* __restrict__ x, int H, const int* __restrict_
   constexpr int U = 8;  // 16-byte loads of a row in flight per lane before any store
   long r = (long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   int tok = r < R ? node_tok[r] : 0;
+  bool anc = r < R && __ldg(rank + row_node[r]) == 0;
   for (; r < R; r += warps) {
     const uint4* src = reinterpret_cast<const uint4*>(x + (size_t)tok * H);
     uint4* dst = reinterpret_cast<uint4*>(xg + (size_t)r * H);
     const long rn = r + warps;
+    const bool this_anc = anc;
     tok = rn < R ? node_tok[rn] : 0;  // the next row's token, looked up early
+    anc = rn < R && __ldg(rank + row_node[rn]) == 0;
+    if (!this_anc) continue;
     for (int i0 = lane; i0 < vec; i0 += 32 * U) {
       uint4 v[U];
 #pragma unroll
@@ -594,20 +707,28 @@ lx_status launch_tc_experts(lx_layer* L, const void* x, int T, int k, void* y, c
     if (P.n_items == 0) return LX_OK;
     return launch_tc(L, P, s, name);
   };
-  // token rows in node-row order once, so that every A tile below is a TMA box
+  // the anchor rows in node-row order once, so that the anchor product's A
+  // tiles are TMA boxes (its 256-row stages are too few to hide gathers); the
+  // correction products read their rows straight from x (gathered by the
+  // GEMM's gather warp)
   {
     ProfScope ps(L, s, "gather_rows");
-    launch_k(L, k_gather_rows, L->num_sms * 8, 256, 0, s, xb, (int)H, w.node_tok,
-             w.key_off + L->N, w.rows_cap, w.xg);
+    launch_k(L, k_gather_rows, L->num_sms * 8, 256, 0, s, xb, (int)H, w.node_tok, w.row_node,
+             L->d_rank, w.key_off + L->N, w.rows_cap, w.xg);
     LX_CUDA(cudaGetLastError());
   }
-  LX_TRY(run(tc_op(L, OP_UP_ANCHOR, w.gmap, 0, w.hb, 2 * I, false, 0),
-             "tc_up_anchor"));
+  auto gathered = [&](TcLaunch P) {
+    P.gather = w.node_tok;
+    P.xsrc = xb;
+    P.ldx = H;
+    return P;
+  };
+  LX_TRY(run(tc_op(L, OP_UP_ANCHOR, w.gmap, 0, w.hb, 2 * I, false, 0), "tc_up_anchor"));
   if (L->ct) {
     // flat layers: the members' x V rows land aligned to their cluster's rows,
     // and one fused kernel adds the corrections and applies the SwiGLU
     LX_TRY(launch_ct_meta(L, T, k, s));
-    TcLaunch pv = tc_op(L, OP_UP_V, w.gmap, 0, w.Pal, (long)L->ct_nch * 2 * rmax, false, 1);
+    TcLaunch pv = gathered(tc_op(L, OP_UP_V, w.gmap, 0, w.Pal, (long)L->ct_nch * 2 * rmax, false, 1));
     pv.row_map = w.rho2al;
     pv.node_col = L->d_child_col;
     LX_TRY(run(pv, "tc_up_V"));
@@ -627,7 +748,7 @@ lx_status launch_tc_experts(lx_layer* L, const void* x, int T, int k, void* y, c
     LX_TRY(run(dn, "tc_dn_anchor_U"));
     return launch_combine(L, T, k, y, true, s, SplitParts(), /*anchors_only=*/true);
   } else {
-    LX_TRY(run(tc_op(L, OP_UP_V, w.gmap, 0, w.Pb, 2 * rmax, false, 1),
+    LX_TRY(run(gathered(tc_op(L, OP_UP_V, w.gmap, 0, w.Pb, 2 * rmax, false, 1)),
                "tc_up_V"));
     LX_TRY(run(tc_op(L, OP_UP_U, w.xmaps + 0, 0, w.hb, 2 * I, false, 2),
                "tc_up_U"));
