@@ -234,6 +234,100 @@ __global__ void k_node_row(const int* __restrict__ topk_id, int T, int k, int E,
   }
 }
 
+// The fused path's per-cluster-row tables (flat layers on the tensor-core
+// path; al_g == nullptr: none): see k_assign_rows.
+struct CtMeta {
+  const float* topk_w;
+  float* al_g;
+  int* al_row;
+  int* rho2al;
+  const int* child_col;
+  int nch, gstride, rstride, pslot;
+};
+
+// The rows of every assignment, one warp per token (lane s = top-k slot s):
+// its position in its expert's bucket (perm), the rows of the nodes on its
+// path (node_row; the (token, node) pairs shared by several slots write the
+// same node_tok / row_node values), and, for flat layers on the fused
+// tensor-core path, the per-cluster-row tables: for each anchor row a of the
+// token, al_g[a] = {dominant's gate, gates of child slots 0, 1, ...} (0 where
+// not selected; slots whose experts share a node add up, in slot order) and
+// al_row[a] = the child rows (-1 where not selected), written by the first
+// slot of that anchor row; rho2al maps every child row to its anchor row.
+__global__ void __launch_bounds__(256)
+k_assign_rows(const int* __restrict__ topk_id, int T, int k, int N, int E, int D, long Tp,
+              const int* __restrict__ paths, const int* __restrict__ path_len,
+              const int* __restrict__ key_off, const int* __restrict__ rank_in,
+              int* __restrict__ node_tok, int* __restrict__ row_node, int* __restrict__ perm,
+              int* __restrict__ node_row, const CtMeta cm) {
+  pdl_wait();
+  const int lane = threadIdx.x & 31;
+  const int t = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (t >= T) return;
+  const size_t a = (size_t)t * k + lane;
+  int e = -1, len = 0;
+  if (lane < k) {
+    e = topk_id[a];
+    if (e >= 0 && e < E) {
+      len = path_len[e];
+      perm[key_off[N + 1 + e] + rank_in[(size_t)(N + e) * Tp + t]] = (int)a;
+    } else {
+      e = -1;
+    }
+  }
+  int r0 = -1, r1 = -1, n0 = -1;
+#pragma unroll
+  for (int l = 0; l < LX_MAX_DEPTH; ++l) {
+    if (l >= D) break;
+    int row = -1;
+    if (l < len) {
+      const int n = paths[e * LX_MAX_DEPTH + l];
+      row = key_off[n] + rank_in[(size_t)n * Tp + t];
+      node_tok[row] = t;
+      row_node[row] = n;
+      if (l == 0) n0 = n;
+    }
+    if (lane < k) node_row[a * D + l] = row;
+    if (l == 0) r0 = row;
+    if (l == 1) r1 = row;
+  }
+  if (!cm.al_g) return;
+  // flat layers: a path is [anchor] (the dominant) or [member, anchor]
+  const bool member = len >= 2;
+  const int an = lane < k && e >= 0 ? (member ? r1 : r0) : -1;
+  const int j = member ? cm.child_col[n0] / cm.pslot : -1;
+  const float g = an >= 0 ? cm.topk_w[a] : 0.f;
+  if (member) cm.rho2al[r0] = an;
+  const unsigned same = __match_any_sync(0xffffffffu, an);
+  const bool leader = an >= 0 && lane == __ffs(same) - 1;
+  float rg[1 + CT_MAX_CH];
+  int rr[CT_MAX_CH];
+#pragma unroll
+  for (int i = 0; i <= CT_MAX_CH; ++i) rg[i] = 0.f;
+#pragma unroll
+  for (int i = 0; i < CT_MAX_CH; ++i) rr[i] = -1;
+  for (int sl = 0; sl < k; ++sl) {
+    const int as = __shfl_sync(0xffffffffu, an, sl), js = __shfl_sync(0xffffffffu, j, sl);
+    const int rs = __shfl_sync(0xffffffffu, r0, sl);
+    const float gs = __shfl_sync(0xffffffffu, g, sl);
+    if (as == an && as >= 0) {
+#pragma unroll
+      for (int i = 0; i <= CT_MAX_CH; ++i)
+        if (i == js + 1) rg[i] += gs;
+#pragma unroll
+      for (int i = 0; i < CT_MAX_CH; ++i)
+        if (i == js) rr[i] = rs;
+    }
+  }
+  if (leader) {
+#pragma unroll
+    for (int i = 0; i <= CT_MAX_CH; ++i)
+      if (i <= cm.nch) cm.al_g[(size_t)an * cm.gstride + i] = rg[i];
+#pragma unroll
+    for (int i = 0; i < CT_MAX_CH; ++i)
+      if (i < cm.nch) cm.al_row[(size_t)an * cm.rstride + i] = rr[i];
+  }
+}
 
 // ---------------------------------------------------------------------------
 // Small batches (decode): top-k and the whole bucketing in one CTA, with the
@@ -414,7 +508,7 @@ static PlanArgs make_plans(const lx_layer* L, int n_plans, int first = 0) {
     pa.shape[p] = op_shape(L, op);
     pa.items[p] = pa.shape[p].on_anchors ? L->d_anchors : L->d_corrs;
     pa.n_items[p] = pa.shape[p].on_anchors ? L->n_anchor : L->n_corr;
-    pa.bm[p] = slot < PLAN_TC ? G_BM : tc_tile_rows(op);
+    pa.bm[p] = slot < PLAN_TC ? G_BM : tc_tile_rows(L, op);
     pa.bn[p] = slot < PLAN_TC ? G_BN : tc_tile_cols();
     if (L->ct && slot == PLAN_TC + OP_UP_U) {
       // the fused correction + SwiGLU kernel takes this slot: tiles of 128
@@ -490,17 +584,24 @@ lx_status launch_bucket(lx_layer* L, const int* topk_id, int T, int k, cudaStrea
     LX_CUDA(cudaGetLastError());
   }
   {
-    ProfScope ps(L, s, "bucket_scatter");
-    const dim3 grid((T + 255) / 256, keys);
-    launch_k(L, k_scatter, grid, 256, 0, s, w.marks, w.rank_in, w.key_off, topk_id, T, k, L->N, Tp,
-                                   w.node_tok, w.row_node, w.perm);
-    LX_CUDA(cudaGetLastError());
-  }
-  {
-    ProfScope ps(L, s, "bucket_node_row");
-    const long A = (long)T * k;
-    launch_k(L, k_node_row, (unsigned)((A + 255) / 256), 256, 0, s, topk_id, T, k, L->E,
-             L->max_depth, Tp, L->d_paths, L->d_path_len, w.key_off, w.rank_in, w.node_row);
+    // the fused tensor-core path of flat layers also takes its per-cluster-row
+    // tables from this pass
+    CtMeta cm{};
+    if (L->ct && plan_first == PLAN_TC) {
+      cm.topk_w = w.topk_w;
+      cm.al_g = w.al_g;
+      cm.al_row = w.al_row;
+      cm.rho2al = w.rho2al;
+      cm.child_col = L->d_child_col;
+      cm.nch = L->ct_nch;
+      cm.gstride = ct_gstride(L);
+      cm.rstride = ct_rstride(L);
+      cm.pslot = 2 * std::max(1, L->max_rank);
+    }
+    ProfScope ps(L, s, "bucket_rows");
+    launch_k(L, k_assign_rows, (unsigned)((T + 7) / 8), 256, 0, s, topk_id, T, k, L->N, L->E,
+             L->max_depth, Tp, L->d_paths, L->d_path_len, w.key_off, w.rank_in, w.node_tok,
+             w.row_node, w.perm, w.node_row, cm);
     LX_CUDA(cudaGetLastError());
   }
   return LX_OK;

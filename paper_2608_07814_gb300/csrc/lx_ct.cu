@@ -621,85 +621,7 @@ __global__ void __launch_bounds__(CT_THREADS, 1) k_ct_swiglu(const __grid_consta
   }
 }
 
-// Per-cluster-row tables of the fused kernel, one warp per token (lane s =
-// top-k slot s): for each anchor row a of the token, al_g[a] = {dominant's
-// gate, gate of child slot 0, 1, ...} (0 where not selected) and al_row[a] =
-// the child rows (-1 where not selected); rho2al maps every child row to its
-// anchor row.  The first slot of each anchor row writes its record; gates of
-// slots whose experts share a node add up in slot order.
-__global__ void __launch_bounds__(256)
-k_ct_meta(const int* __restrict__ topk_id, const float* __restrict__ topk_w,
-          const int* __restrict__ node_row, const int* __restrict__ paths,
-          const int* __restrict__ child_col, int T, int k, int D, int nch, int gstride,
-          int rstride, int pslot, float* __restrict__ al_g, int* __restrict__ al_row,
-          int* __restrict__ rho2al) {
-  pdl_wait();
-  const int lane = threadIdx.x & 31;
-  const int t = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-  if (t >= T) return;
-  const size_t base = (size_t)t * k;
-  int a = -1, j = -1, r = -1;
-  float g = 0.f;
-  if (lane < k) {
-    const int e = topk_id[base + lane];
-    g = topk_w[base + lane];
-    const int n0 = paths[(size_t)e * LX_MAX_DEPTH];
-    const bool member = paths[(size_t)e * LX_MAX_DEPTH + 1] >= 0;
-    const int r0 = node_row[(base + lane) * D];
-    if (member) {
-      a = node_row[(base + lane) * D + 1];
-      r = r0;
-      j = child_col[n0] / pslot;
-      rho2al[r] = a;
-    } else {
-      a = r0;
-    }
-  }
-  // leader of an anchor row: its first slot
-  const unsigned same = __match_any_sync(0xffffffffu, a);
-  const bool leader = a >= 0 && lane == __ffs(same) - 1;
-  float rg[1 + CT_MAX_CH];
-  int rr[CT_MAX_CH];
-#pragma unroll
-  for (int i = 0; i <= CT_MAX_CH; ++i) rg[i] = 0.f;
-#pragma unroll
-  for (int i = 0; i < CT_MAX_CH; ++i) rr[i] = -1;
-  for (int s = 0; s < k; ++s) {
-    const int as = __shfl_sync(0xffffffffu, a, s), js = __shfl_sync(0xffffffffu, j, s);
-    const int rs = __shfl_sync(0xffffffffu, r, s);
-    const float gs = __shfl_sync(0xffffffffu, g, s);
-    if (as == a) {
-#pragma unroll
-      for (int i = 0; i <= CT_MAX_CH; ++i)
-        if (i == js + 1) rg[i] += gs;
-#pragma unroll
-      for (int i = 0; i < CT_MAX_CH; ++i)
-        if (i == js) rr[i] = rs;
-    }
-  }
-  if (leader) {
-#pragma unroll
-    for (int i = 0; i <= CT_MAX_CH; ++i)
-      if (i <= nch) al_g[(size_t)a * gstride + i] = rg[i];
-#pragma unroll
-    for (int i = 0; i < CT_MAX_CH; ++i)
-      if (i < nch) al_row[(size_t)a * rstride + i] = rr[i];
-  }
-}
-
 }  // namespace
-
-lx_status launch_ct_meta(lx_layer* L, int T, int k, cudaStream_t s) {
-  Workspace& w = L->ws;
-  const int pslot = 2 * std::max(1, L->max_rank);
-  ProfScope ps(L, s, "ct_meta");
-  launch_k(L, k_ct_meta, (T + 7) / 8, 256, 0, s, (const int*)w.topk_id,
-           (const float*)w.topk_w, (const int*)w.node_row, (const int*)L->d_paths,
-           (const int*)L->d_child_col, T, k, L->max_depth, L->ct_nch, ct_gstride(L),
-           ct_rstride(L), pslot, w.al_g, w.al_row, w.rho2al);
-  LX_CUDA(cudaGetLastError());
-  return LX_OK;
-}
 
 lx_status launch_ct_swiglu(lx_layer* L, cudaStream_t s) {
   Workspace& w = L->ws;

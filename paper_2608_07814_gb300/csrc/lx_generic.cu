@@ -625,11 +625,10 @@ k_swiglu_warp(const float* __restrict__ topk_w, const int* __restrict__ node_row
 
 // y[t] = sum of ypart over t's distinct rows in ascending row order (an
 // anchor row split into K ranges contributes its partials in split order)
-template <typename TP, typename TY, int CPL, bool SPLIT>
+template <typename TP, typename TY, int CPL, bool SPLIT, bool ANCHORS = false>
 __global__ void __launch_bounds__(WT_WARPS * 32, 2)
 k_combine_warp(const int* __restrict__ node_row, int k, int D, const TP* __restrict__ ypart,
-               int H, TY* __restrict__ y, int T, int cols_per_item, const SplitParts ys,
-               int anchors_only) {
+               int H, TY* __restrict__ y, int T, int cols_per_item, const SplitParts ys) {
   __shared__ WarpRows wrs[WT_WARPS];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   WarpRows& wr = wrs[warp];
@@ -648,8 +647,8 @@ k_combine_warp(const int* __restrict__ node_row, int k, int D, const TP* __restr
     const int c_end = min(H, c_begin + cols_per_item);
     warp_token_rows(first ? v_pre : (lane < kD ? node_row[(size_t)t * kD + lane] : -1), kD, D, wr);
     const int nd = wr.nd;
-    if constexpr (!SPLIT && CPL == 8 && sizeof(TP) == 2) {
-      if (anchors_only) {
+    if constexpr (ANCHORS && !SPLIT && CPL == 8 && sizeof(TP) == 2) {
+      {
         // only the anchor rows (their down tiles already hold the members'
         // corrections), ascending; four column passes' 16-byte loads of a
         // batch of four rows in flight at once, each column summed in row order
@@ -839,15 +838,20 @@ static void launch_combine_warp(lx_layer* L, int T, int k, const TP* ypart, TY* 
     const int cols = warp_item_cols(L, T, L->H, 128);
     const int grid = warp_grid(L, T, L->H, cols);
     launch_k(L, k_combine_warp<TP, TY, 4, true>, grid, WT_WARPS * 32, 0, s, w.node_row, k,
-             L->max_depth, ypart, L->H, y, T, cols, ys, 0);
+             L->max_depth, ypart, L->H, y, T, cols, ys);
     return;
   }
   // eight columns per lane (16-byte bf16 loads): half the per-element address
   // and loop instructions of four (measured faster at decode and prefill)
   const int cols = warp_item_cols(L, T, L->H, 256);
   const int grid = warp_grid(L, T, L->H, cols);
+  if (anchors_only && sizeof(TP) == 2) {
+    launch_k(L, k_combine_warp<TP, TY, 8, false, true>, grid, WT_WARPS * 32, 0, s, w.node_row, k,
+             L->max_depth, ypart, L->H, y, T, cols, ys);
+    return;
+  }
   launch_k(L, k_combine_warp<TP, TY, 8, false>, grid, WT_WARPS * 32, 0, s, w.node_row, k,
-           L->max_depth, ypart, L->H, y, T, cols, ys, anchors_only ? 1 : 0);
+           L->max_depth, ypart, L->H, y, T, cols, ys);
 }
 
 lx_status launch_swiglu(lx_layer* L, int T, int k, bool bf16, cudaStream_t s, SplitParts hs) {

@@ -476,7 +476,7 @@ lx_status launch_fast_experts(lx_layer* L, const void* x, int T, int k, void* y,
 lx_status launch_tc_experts(lx_layer* L, const void* x, int T, int k, void* y, cudaStream_t s);
 int tc_tile_tokens();  // rows of the TMA boxes of the tensor-core A operands
 int tc_tile_cols();
-int tc_tile_rows(int op);  // token rows of a tensor-core tile of op (its tile plan)
+int tc_tile_rows(const lx_layer* L, int op);  // token rows of a tensor-core tile of op (its tile plan)
 lx_status launch_tc(lx_layer* L, const TcLaunch& P, cudaStream_t s, const char* name);
 // 2-D TMA map of a row-major bf16 matrix [outer][inner] read as box_inner x
 // box_outer boxes with the 128-byte swizzle
@@ -491,9 +491,9 @@ bool res_tc_fits(long rows, long cols, long l);
 lx_status res_gemm_tc(bool transposed, const __nv_bfloat16* Wm, const __nv_bfloat16* Wd,
                       long rows, long cols, const float* X, long N, float* C, char* ws,
                       int num_sms, int dev, cudaStream_t s);
-// fused correction + SwiGLU (flat layers): the per-anchor-row gate / row
-// tables, then the fused kernel over (anchor, 128-row block, 64 d_ff columns)
-lx_status launch_ct_meta(lx_layer* L, int T, int k, cudaStream_t s);
+// fused correction + SwiGLU (flat layers): the kernel over (anchor, 128-row
+// block, 64 d_ff columns); its per-cluster-row gate / child-row tables are
+// written by the bucketing (k_assign_rows)
 lx_status launch_ct_swiglu(lx_layer* L, cudaStream_t s);
 constexpr int CT_CW = 64;  // d_ff columns of a fused tile
 // row strides (4-byte words, 16-byte rows) of the per-anchor-row tables

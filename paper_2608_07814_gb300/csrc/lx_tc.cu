@@ -582,12 +582,16 @@ k_tc_gemm(const __grid_constant__ TcLaunch P) {
 
 int tc_tile_tokens() { return 128; }
 int tc_tile_cols() { return TC_BN; }
-// The anchor products (anchor buckets of hundreds of rows) take 256-row
-// tiles; the others 128 (measured at the Qwen3-shaped prefill of 8192:
-// tc_up_anchor 156 -> 146 us and the down tile with the members' corrections
-// 142 -> 128 us with 256 rows, while x V, whose member buckets are a few
-// hundred rows, loses more to half-empty tiles and a single wave than it gains).
-int tc_tile_rows(int op) { return (op == OP_UP_ANCHOR || op == OP_DN_ANCHOR) ? 256 : 128; }
+// The anchor gate/up product (anchor buckets of hundreds of rows) and, on
+// flat layers, the anchor down tile with the members' corrections along K take
+// 256-row tiles; the others 128 (measured at the Qwen3-shaped prefill of 8192:
+// tc_up_anchor 156 -> 146 us and the down tile with the corrections 142 -> 128
+// us with 256 rows; the tree layer's plain down tile is faster at 128 rows,
+// 34 vs 39 us, and x V, whose member buckets are a few hundred rows, loses more
+// to half-empty tiles and a single wave than it gains).
+int tc_tile_rows(const lx_layer* L, int op) {
+  return (op == OP_UP_ANCHOR || (op == OP_DN_ANCHOR && L->ct)) ? 256 : 128;
+}
 
 template <int BM, int EPI>
 static int tc_smem_bytes_() {
@@ -626,7 +630,7 @@ static TcLaunch tc_op(lx_layer* L, int op, const CUtensorMap* xmap, int xcol, vo
   Workspace& w = L->ws;
   TcLaunch P;
   P.shape = op_shape(L, op);
-  P.bm = tc_tile_rows(op);
+  P.bm = tc_tile_rows(L, op);
   // short-K products (the U factors, K = rank; the down side, K = d_ff): tiles
   // bound by writing their output take eight epilogue warps
   P.epi = (op == OP_UP_U || op == OP_DN_U || op == OP_DN_ANCHOR || op == OP_DN_V) ? 8 : 4;
@@ -727,7 +731,7 @@ lx_status launch_tc_experts(lx_layer* L, const void* x, int T, int k, void* y, c
   if (L->ct) {
     // flat layers: the members' x V rows land aligned to their cluster's rows,
     // and one fused kernel adds the corrections and applies the SwiGLU
-    LX_TRY(launch_ct_meta(L, T, k, s));
+    // (the per-cluster-row gate / child-row tables come from the bucketing)
     TcLaunch pv = gathered(tc_op(L, OP_UP_V, w.gmap, 0, w.Pal, (long)L->ct_nch * 2 * rmax, false, 1));
     pv.row_map = w.rho2al;
     pv.node_col = L->d_child_col;
