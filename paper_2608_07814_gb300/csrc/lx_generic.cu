@@ -645,7 +645,16 @@ k_combine_warp(const int* __restrict__ node_row, int k, int D, const TP* __restr
     const int t = (int)(it / per_tok);
     const int c_begin = (int)(it % per_tok) * cols_per_item;
     const int c_end = min(H, c_begin + cols_per_item);
-    warp_token_rows(first ? v_pre : (lane < kD ? node_row[(size_t)t * kD + lane] : -1), kD, D, wr);
+    int v_cur;
+    if constexpr (ANCHORS) {
+      // the next item's node rows are requested now, ahead of their use
+      v_cur = v_pre;
+      const long itn = it + (long)gridDim.x * WT_WARPS;
+      v_pre = (itn < items && lane < kD) ? node_row[(size_t)(itn / per_tok) * kD + lane] : -1;
+    } else {
+      v_cur = first ? v_pre : (lane < kD ? node_row[(size_t)t * kD + lane] : -1);
+    }
+    warp_token_rows(v_cur, kD, D, wr);
     const int nd = wr.nd;
     if constexpr (ANCHORS && !SPLIT && CPL == 8 && sizeof(TP) == 2) {
       {

@@ -63,6 +63,11 @@ struct TcCfg {
   static constexpr int STAGES = (NH == 1 && EPI == 4) ? 4 : 3;
   static constexpr int NBUF = NH == 1 ? 2 : 1;           // accumulators of NH x 256 columns
   static constexpr int THREADS = 32 * (4 + EPI);
+  // 256-row tiles with eight epilogue warps stage 32 bf16 columns per pass
+  // (80-byte rows), so that the staging fits beside the three 64 KiB stages
+  static constexpr bool HALF = BM == 256 && EPI == 8;
+  static constexpr int EPI_LD = HALF ? 20 : TC_EPI_LD;  // staging row stride (4-byte words)
+  static constexpr int EPI_BYTES = 32 * EPI_LD * 4;
   static_assert(EPI == 4 || EPI == 8, "four or eight epilogue warps");
   static_assert(STAGE_BYTES % 1024 == 0, "stages keep the 1024-byte swizzle alignment");
   static_assert(NBUF * NH * TC_ACC_COLS <= TC_TMEM_COLS, "accumulators fit the TMEM allocation");
@@ -140,7 +145,7 @@ k_tc_gemm(const __grid_constant__ TcLaunch P) {
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   float* epi = reinterpret_cast<float*>(smem + TC_STAGES * TC_STAGE_BYTES);  // [EPI][32][EPI_LD]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + TC_STAGES * TC_STAGE_BYTES + EPI * TC_EPI_BYTES);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + TC_STAGES * TC_STAGE_BYTES + EPI * C::EPI_BYTES);
   // full[S], empty[S], tmem_full[2], tmem_empty[2], drain
   const uint32_t full0 = smem_u32(bars), empty0 = full0 + 8 * TC_STAGES;
   const uint32_t tfull0 = empty0 + 8 * TC_STAGES, tempty0 = tfull0 + 16, drain = tempty0 + 16;
@@ -207,11 +212,23 @@ k_tc_gemm(const __grid_constant__ TcLaunch P) {
       const int nkb = (t.K + TC_BK - 1) / TC_BK;
       const int rt0 = (t.grp * t.Ng + t.row0) / 64;  // first 64-row weight tile
       const int nbox = (t.BN + 63) / 64;
-      // K concatenation: k-blocks from kb_own on read child cj's k-block ckb
+      // K concatenation: k-blocks from kb_own on read child cj's k-block ckb;
+      // the tile's children and their K blocks are looked up once, lane j
+      // holding child j (their loads overlap the tile's first stages)
       const int kb_own = P.kc_child ? P.shape.k_const / TC_BK : nkb;
-      int cj = 0, ckb = 0, cnode = -1, cnkb = 0;
+      int my_child = -1, my_nkb = 0;
+      if (P.kc_child && lane < CT_MAX_CH) {
+        my_child = __ldg(P.kc_child + (size_t)t.node * CT_MAX_CH + lane);
+        my_nkb = my_child >= 0 ? __ldg(P.rank + my_child) / TC_BK : 0;
+      }
+      int cj = 0, ckb = 0;
       for (int kb = 0; kb < nkb; ++kb, ++it) {
         const uint32_t s = it % TC_STAGES;
+        int cnode = -1, cnkb = 0;
+        if (kb >= kb_own) {  // warp-uniform: every lane takes child cj's entry
+          cnode = __shfl_sync(0xffffffffu, my_child, cj);
+          cnkb = __shfl_sync(0xffffffffu, my_nkb, cj);
+        }
         int good = 1;
         if (lane == 0) {
           good = mbar_wait(empty0 + 8 * s, ((it / TC_STAGES) & 1) ^ 1, abort_flag,
@@ -230,22 +247,17 @@ k_tc_gemm(const __grid_constant__ TcLaunch P) {
                             (int)(t.grp * t.K) + kb * TC_BK + P.xcol, t.tok0 + 128 * h,
                             full0 + 8 * s);
             } else {
-              if (cnode < 0) {
-                cnode = __ldg(P.kc_child + (size_t)t.node * CT_MAX_CH + cj);
-                cnkb = __ldg(P.rank + cnode) / TC_BK;
-              }
               for (int b = 0; b < nbox; ++b)
                 tma_load_4d(b_s + b * 8192, P.kc_wmaps + cnode, 0, 0, ckb, rt0 + b, full0 + 8 * s);
               for (int h = 0; h < nh; ++h)
                 tma_load_2d(a_s + h * 128 * TC_BK * 2, P.kc_xmap, cj * P.kc_slot + ckb * TC_BK,
                             t.tok0 + 128 * h, full0 + 8 * s);
-              if (++ckb == cnkb) {
-                ckb = 0;
-                ++cj;
-                cnode = -1;
-              }
             }
           }
+        }
+        if (kb >= kb_own && ++ckb == cnkb) {  // every lane walks the children alike
+          ckb = 0;
+          ++cj;
         }
         good = __shfl_sync(0xffffffffu, good, 0);
         if (!good) {
@@ -467,7 +479,7 @@ k_tc_gemm(const __grid_constant__ TcLaunch P) {
     const int ew = warp & 3;        // TMEM lanes 32 ew .. 32 ew + 31
     const int eh = (warp - 4) >> 2; // with 8 warps: which column passes (alternate)
     constexpr int ESTEP = EPI / 4;  // passes are dealt out to ESTEP warps per quadrant
-    float* stg = epi + (warp - 4) * 32 * TC_EPI_LD;
+    float* stg = epi + (warp - 4) * 32 * C::EPI_LD;
     uint32_t tiles = 0;
     while (true) {
       const uint32_t b = tiles % NBUF, u = tiles / NBUF;
@@ -490,7 +502,40 @@ k_tc_gemm(const __grid_constant__ TcLaunch P) {
       long orow_l = (long)t.tok0 + 128 * h + 32 * ew + lane;
       if (P.row_map)
         orow_l = (32 * ew + lane + 128 * h < t.M && orow_l < P.rows_cap) ? P.row_map[orow_l] : -1;
-      if (P.out_f32) {
+      if constexpr (C::HALF) {
+        // bf16, 32 columns per pass: one TMEM load, rows staged 64 bytes wide,
+        // stored as 64-byte row segments (four lanes per row, eight rows a pass)
+        for (int c0 = 32 * eh; c0 < t.BN; c0 += 32 * ESTEP) {
+          uint32_t r0[32];
+          tc_ld32_async(acc + ((uint32_t)(32 * ew) << 16) + (uint32_t)c0, r0);
+          tc_wait_ld();
+          uint32_t pk[16];
+#pragma unroll
+          for (int e = 0; e < 16; ++e) {
+            __nv_bfloat162 b0 = __floats2bfloat162_rn(__uint_as_float(r0[2 * e]),
+                                                      __uint_as_float(r0[2 * e + 1]));
+            pk[e] = *reinterpret_cast<uint32_t*>(&b0);
+          }
+          uint4* srow = reinterpret_cast<uint4*>(stg + lane * C::EPI_LD);
+#pragma unroll
+          for (int q = 0; q < 4; ++q)
+            srow[q] = make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
+          __syncwarp();
+          const int c4 = lane & 3;
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            const int rr = 8 * j + (lane >> 2);
+            const int m = 128 * h + 32 * ew + rr;
+            const long grow = __shfl_sync(0xffffffffu, orow_l, rr);
+            if (tile_ok && m < t.M && grow >= 0 && grow < P.rows_cap) {
+              const uint4 u4 = *reinterpret_cast<const uint4*>(stg + rr * C::EPI_LD + 4 * c4);
+              *reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(P.out) + (size_t)grow * P.ldo +
+                                        col0 + c0 + 8 * c4) = u4;
+            }
+          }
+          __syncwarp();
+        }
+      } else if (P.out_f32) {
         for (int c0 = 32 * eh; c0 < t.BN; c0 += 32 * ESTEP) {
           float v[32];
           tc_ld32(acc + ((uint32_t)(32 * ew) << 16) + (uint32_t)c0, v);
@@ -596,7 +641,7 @@ int tc_tile_rows(const lx_layer* L, int op) {
 template <int BM, int EPI>
 static int tc_smem_bytes_() {
   using C = TcCfg<BM, EPI>;
-  return C::STAGES * C::STAGE_BYTES + EPI * TC_EPI_BYTES + 8 * (2 * C::STAGES + 7) +
+  return C::STAGES * C::STAGE_BYTES + EPI * C::EPI_BYTES + 8 * (2 * C::STAGES + 7) +
          (C::STAGES + 2 + TC_QN) * (int)sizeof(TcTile) + 16 * TC_QN + 1024;
 }
 template <int BM, int EPI>
@@ -616,8 +661,12 @@ static lx_status launch_tc_cfg(lx_layer* L, const TcLaunch& P, cudaStream_t s, c
 lx_status launch_tc(lx_layer* L, const TcLaunch& P, cudaStream_t s, const char* name) {
   const bool g = P.gather != nullptr;
   if (g && P.kc_child) return fail(LX_ERR_STATE, "gathered A rows with a K concatenation");
-  if (P.bm == 256)
-    return g ? launch_tc_cfg<256, 4, true>(L, P, s, name) : launch_tc_cfg<256, 4, false>(L, P, s, name);
+  if (P.bm == 256) {
+    // eight epilogue warps: the single accumulator of a 256-row tile is
+    // drained while the tensor core waits, so the drain is split eight ways
+    if (g || P.out_f32) return fail(LX_ERR_STATE, "256-row tiles take TMA rows and bf16 output");
+    return launch_tc_cfg<256, 8, false>(L, P, s, name);
+  }
   if (P.epi == 8) {
     if (g) return fail(LX_ERR_STATE, "gathered A rows need four epilogue warps");
     return launch_tc_cfg<128, 8, false>(L, P, s, name);
