@@ -490,22 +490,19 @@ __global__ void __launch_bounds__(CT_THREADS, 1) k_ct_swiglu(const __grid_consta
         failed = true;
         break;
       }
-      uint32_t hg[CT_EC / 2], hu[CT_EC / 2];
+      // row m of each 128-byte-swizzled box: 16-byte unit u sits at u ^ (m % 8);
+      // the anchor values are read from the staged boxes where they are used
+      // (the registers go to a member's whole set of accumulator loads), and
+      // the buffer is released once the tile is done
+      const uint8_t* gbox = hbuf + hb * CT_H_BYTES + m * 128;
+      const uint8_t* ubox = gbox + CT_H_BYTES / 2;
+      auto h_unit = [&](const uint8_t* box, int i) {  // this warp's 16-byte unit i (8 columns)
+        return *reinterpret_cast<const uint4*>(box + 16 * (((CT_EC / 8) * cs + i) ^ (m & 7)));
+      };
       float gd = 0.f;
       float gm[CT_MAX_CH];
       int rm[CT_MAX_CH];
       {
-        // row m of each 128-byte-swizzled box: 16-byte unit u sits at u ^ (m % 8)
-        const uint8_t* gbox = hbuf + hb * CT_H_BYTES + m * 128;
-        const uint8_t* ubox = gbox + CT_H_BYTES / 2;
-#pragma unroll
-        for (int i = 0; i < CT_EC / 8; ++i) {
-          const int u = (CT_EC / 8) * cs + i;
-          const uint4 vg = *reinterpret_cast<const uint4*>(gbox + 16 * (u ^ (m & 7)));
-          const uint4 vu = *reinterpret_cast<const uint4*>(ubox + 16 * (u ^ (m & 7)));
-          hg[4 * i] = vg.x; hg[4 * i + 1] = vg.y; hg[4 * i + 2] = vg.z; hg[4 * i + 3] = vg.w;
-          hu[4 * i] = vu.x; hu[4 * i + 1] = vu.y; hu[4 * i + 2] = vu.z; hu[4 * i + 3] = vu.w;
-        }
         const float* tg = reinterpret_cast<const float*>(tbuf + hb * 2 * CT_TAB_BYTES) + m * P.gstride;
         const int* tr = reinterpret_cast<const int*>(tbuf + hb * 2 * CT_TAB_BYTES + CT_TAB_BYTES) +
                         m * P.rstride;
@@ -516,9 +513,6 @@ __global__ void __launch_bounds__(CT_THREADS, 1) k_ct_swiglu(const __grid_consta
           rm[jj] = (valid && jj < t.nch) ? tr[jj] : -1;
         }
       }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(hempty0 + 8 * hb);
-      ++nt;
       // the down side sums every child slot of a cluster row: the slots of
       // children this row did not select are zeroed (once, by the first chunk)
       if (t.q == 0 && cs == 0 && valid) {
@@ -534,8 +528,12 @@ __global__ void __launch_bounds__(CT_THREADS, 1) k_ct_swiglu(const __grid_consta
       if (__any_sync(0xffffffffu, gd != 0.f)) {
         const F2 gd2{gd, gd};
 #pragma unroll
-        for (int i = 0; i < CT_EC / 2; ++i)
-          zr[i] = mul2(mul2(silu2(bf2(hg[i])), bf2(hu[i])), gd2);
+        for (int i = 0; i < CT_EC / 8; ++i) {
+          const uint4 vg = h_unit(gbox, i), vu = h_unit(ubox, i);
+          const uint32_t wg[4] = {vg.x, vg.y, vg.z, vg.w}, wu[4] = {vu.x, vu.y, vu.z, vu.w};
+#pragma unroll
+          for (int q = 0; q < 4; ++q) zr[4 * i + q] = mul2(mul2(silu2(bf2(wg[q])), bf2(wu[q])), gd2);
+        }
       } else {
 #pragma unroll
         for (int i = 0; i < CT_EC / 2; ++i) zr[i] = F2{0.f, 0.f};
@@ -561,26 +559,29 @@ __global__ void __launch_bounds__(CT_THREADS, 1) k_ct_swiglu(const __grid_consta
               tmem + ((uint32_t)(32 * ew) << 16) + b * CT_ACC_COLS + CT_EC * cs;
           const F2 gj2{gj, gj};
           uint4* dst = reinterpret_cast<uint4*>(P.z + (size_t)(use ? rj : 0) * I + c0);
+          // all of the member's accumulator columns of this warp in flight, one wait
+          uint32_t cg[CT_EC], cu[CT_EC];
 #pragma unroll
           for (int q16 = 0; q16 < CT_EC / 16; ++q16) {
-            uint32_t cg[16], cu[16];
-            tc_ld16_async(acc + 16 * q16, cg);
-            tc_ld16_async(acc + CT_CW + 16 * q16, cu);
-            tc_wait_ld();
-            uint32_t pk[8];
+            tc_ld16_async(acc + 16 * q16, *reinterpret_cast<uint32_t(*)[16]>(cg + 16 * q16));
+            tc_ld16_async(acc + CT_CW + 16 * q16, *reinterpret_cast<uint32_t(*)[16]>(cu + 16 * q16));
+          }
+          tc_wait_ld();
 #pragma unroll
-            for (int i = 0; i < 8; ++i) {
-              const int w = 8 * q16 + i;  // column pair 2 w, 2 w + 1 of this warp
-              const F2 gp = add2(bf2(hg[w]), F2{__uint_as_float(cg[2 * i]), __uint_as_float(cg[2 * i + 1])});
-              const F2 up = add2(bf2(hu[w]), F2{__uint_as_float(cu[2 * i]), __uint_as_float(cu[2 * i + 1])});
+          for (int i = 0; i < CT_EC / 8; ++i) {  // 16-byte unit i: column pairs 4 i .. 4 i + 3
+            const uint4 vg = h_unit(gbox, i), vu = h_unit(ubox, i);
+            const uint32_t wg[4] = {vg.x, vg.y, vg.z, vg.w}, wu[4] = {vu.x, vu.y, vu.z, vu.w};
+            uint32_t pk[4];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              const int w = 4 * i + q;  // column pair 2 w, 2 w + 1 of this warp
+              const F2 gp = add2(bf2(wg[q]), F2{__uint_as_float(cg[2 * w]), __uint_as_float(cg[2 * w + 1])});
+              const F2 up = add2(bf2(wu[q]), F2{__uint_as_float(cu[2 * w]), __uint_as_float(cu[2 * w + 1])});
               const F2 av = mul2(mul2(silu2(gp), up), gj2);
               if (use) zr[w] = add2(zr[w], av);
-              pk[i] = pack_bf2(av.x, av.y);
+              pk[q] = pack_bf2(av.x, av.y);
             }
-            if (use) {
-              dst[2 * q16] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-              dst[2 * q16 + 1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
-            }
+            if (use) dst[i] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
           }
         }
         tc_fence_before();
@@ -588,6 +589,9 @@ __global__ void __launch_bounds__(CT_THREADS, 1) k_ct_swiglu(const __grid_consta
         if (lane == 0) mbar_arrive(tempty0 + 8 * b);
         ++mc;
       }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(hempty0 + 8 * hb);  // this tile's staged rows are done
+      ++nt;
       if (failed) break;
       if (valid) {
         uint4* dst = reinterpret_cast<uint4*>(P.z + a * I + c0);
