@@ -212,6 +212,8 @@ def kernel_flops(name, st, src):
     Ra, rr = st["R_anchor"], st["corr_r_rows"]
     table = {
         "tc_up_anchor": 2 * Ra * 2 * I * H,
+        # screened routing: the approximate logits of every (token, expert)
+        "router_screen": 2 * st["T"] * src.n_experts * H,
         "tc_up_V": 2 * rr * 2 * H,
         "tc_up_U": 2 * rr * 2 * I,
         # the fused correction + SwiGLU kernel of flat layers: the members' P U^T

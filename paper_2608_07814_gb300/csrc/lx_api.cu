@@ -3,6 +3,7 @@
 #include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <cmath>
 #include <cstdlib>
 #include <cstring>
 #include <string>
@@ -183,6 +184,8 @@ static lx_status ensure_workspace(lx_layer* L, int T, int k, cudaStream_t s) {
       {(void**)&w.Pal, L->ct ? (size_t)2 * Rmax * L->ct_nch * 2 * rmax : 0},
       {(void**)&w.Qal, L->ct ? (size_t)2 * Rmax * L->ct_nch * rmax : 0},
       {(void**)&w.pamap, L->ct ? 3 * sizeof(CUtensorMap) : 0},
+      {(void**)&w.rs_part, L->router_screen
+                               ? sizeof(float) * RS_MAX_SPLITS * (size_t)cT * router_epad(L) : 0},
   };
   size_t total = 0;
   for (auto& it : items) total += align_up(it.bytes, 256);
@@ -271,7 +274,7 @@ static lx_status bucket_ids(lx_layer* L, const int* ids, int T, int k, cudaStrea
 static lx_status route_and_bucket(lx_layer* L, const void* x, int T, int k, int* ids, float* w,
                                   float* logits_user, cudaStream_t s, int plan_first) {
   float* logits = logits_user ? logits_user : L->ws.logits;
-  LX_TRY(launch_router(L, x, T, k, logits, ids, w, s));
+  LX_TRY(launch_router(L, x, T, k, logits, ids, w, s, logits_user != nullptr));
   return bucket_ids(L, ids, T, k, s, plan_first);
 }
 
@@ -625,6 +628,33 @@ extern "C" lx_status lx_load_compressed_layer(const lx_layer_desc* d, const void
   const lx_status st = encode_tensor_maps(L, s);
   if (st != LX_OK) return cleanup(st);
   L->ct = L->ct && L->stream_ok;
+  {
+    // screened routing: bf16 router rows of a multiple of 64, at most 256
+    // experts (one N tile); the bound of its candidate test needs the largest
+    // row norm of the router matrix
+    const char* env = std::getenv("LX_ROUTER_SCREEN");
+    L->router_screen = L->dtype == LX_BF16 && L->H % 64 == 0 && L->E <= 256 &&
+                       !(env && env[0] == '0');
+    if (L->router_screen) {
+      const uint16_t* rw = static_cast<const uint16_t*>(router_w);
+      double wmax = 0.0;
+      for (int e = 0; e < L->E; ++e) {
+        double ss = 0.0;
+        for (long h = 0; h < H; ++h) {
+          const uint32_t bits = (uint32_t)rw[(size_t)e * H + h] << 16;
+          float f;
+          std::memcpy(&f, &bits, 4);
+          ss += (double)f * f;
+        }
+        wmax = std::max(wmax, std::sqrt(ss));
+      }
+      L->router_wmax = (float)(wmax * (1.0 + 1e-6));
+      std::memset(&L->router_map, 0, sizeof(L->router_map));
+      if (!std::isfinite(L->router_wmax) ||
+          !encode_bf16_2d(&L->router_map, L->router_w, H, L->E, 64, router_epad(L)))
+        L->router_screen = false;
+    }
+  }
   *out = L;
   return LX_OK;
 }

@@ -44,6 +44,7 @@ struct ResLaunch {
 };
 
 __global__ void __launch_bounds__(RM_THREADS, 1) k_res_mma(const __grid_constant__ ResLaunch P) {
+  pdl_wait();
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -277,6 +278,38 @@ lx_status res_gemm_tc(bool transposed, const __nv_bfloat16* Wm, const __nv_bfloa
   k_sum_parts<<<(unsigned)std::min<long>((total + 255) / 256, 4L * num_sms), 256, 0, s>>>(
       part, splits, (int)M, (int)N, (int)Npad, C);
   LX_CUDA(cudaGetLastError());
+  return LX_OK;
+}
+
+// A plain split-K product on the same kernel (one K segment): part[s][M][Npad]
+// = A[M][K-range s] . B[Npad][K-range s]^T, A and B given as 2-D bf16 maps of
+// 64 x 128 and 64 x Npad boxes (K a multiple of 64); returns the ranges used.
+lx_status tc_splitk_gemm(lx_layer* L, const CUtensorMap& a, const CUtensorMap& b, int M, int Npad,
+                         int K, float* part, int max_splits, int* splits_out, cudaStream_t s,
+                         const char* name) {
+  ResLaunch P;
+  std::memset(&P, 0, sizeof(P));
+  P.a_mem = a;
+  P.a_dom = a;
+  P.b = b;
+  const int mt = (M + RM_BM - 1) / RM_BM;
+  P.M = M;
+  P.Npad = Npad;
+  P.kb_seg = K / 64;
+  P.n_kb = P.kb_seg;  // one segment: every K block reads A from a_mem
+  int splits = std::max(1, std::min(max_splits, L->num_sms / mt));
+  splits = std::min(splits, std::max(1, P.n_kb / 4));
+  P.kb_split = (P.n_kb + splits - 1) / splits;
+  splits = (P.n_kb + P.kb_split - 1) / P.kb_split;
+  P.part = part;
+  P.wait_cycles = wait_limit(L);
+  const int b_bytes = Npad * 64 * 2;
+  const int smem = RM_STAGES * (RM_A_BYTES + ((b_bytes + 1023) & ~1023)) + 8 * (2 * RM_STAGES + 3) + 1024;
+  LX_CUDA(smem_cap_once((const void*)k_res_mma, 227 * 1024, L->device, g_rm_cap));
+  ProfScope ps(L, s, name);
+  launch_k(L, k_res_mma, dim3((unsigned)mt, (unsigned)splits), RM_THREADS, smem, s, P);
+  LX_CUDA(cudaGetLastError());
+  *splits_out = splits;
   return LX_OK;
 }
 

@@ -332,6 +332,8 @@ struct Workspace {
   __nv_bfloat16* Pal = nullptr;
   __nv_bfloat16* Qal = nullptr;  // [R][nch * rmax] the children's z Vd rows, aligned likewise
   CUtensorMap* pamap = nullptr;  // [3] TMA maps of Pal, hb and Qal (128-row boxes)
+  // screened routing: the tensor-core logit partials [splits][T][Epad]
+  float* rs_part = nullptr;
 };
 
 struct ProfRec {
@@ -373,6 +375,11 @@ struct lx_layer {
   bool pdl = true;                  // programmatic dependent launch between kernels
   unsigned long long wait_cycles = 0;  // bound of the kernels' device-side waits (0: default)
   int unmet_wait = 0;               // lx_wait_site made to run out (test hook), 0 = none
+  // screened routing (large bf16 batches): approximate logits on the tensor
+  // cores, exact canonical-order logits for the candidates only
+  bool router_screen = false;
+  float router_wmax = 0.f;          // max over experts of ||W_r[e]||_2
+  CUtensorMap router_map;           // W_r [E][H], 64 x Epad boxes
   // fused correction + SwiGLU on the tensor-core path (flat layers)
   bool ct = false;
   int ct_nch = 0;                   // most children of an anchor (table stride)
@@ -444,8 +451,12 @@ struct ProfScope {
 };
 
 // kernels / launchers (defined in the .cu files)
+// need_logits = false: the caller reads only the ids and gates, so large bf16
+// batches may take the screened path (logits of the candidates only)
 lx_status launch_router(lx_layer* L, const void* x, int T, int k, float* logits, int* topk_id,
-                        float* topk_w, cudaStream_t s);
+                        float* topk_w, cudaStream_t s, bool need_logits = true);
+constexpr int RS_MAX_SPLITS = 8;
+inline int router_epad(const lx_layer* L) { return (L->E + 15) / 16 * 16; }
 bool router_is_tiled(const lx_layer* L, int T);
 int router_tile_counters(int T);  // token tiles of the small-batch router
 // plan_first: tile plans for the generic GEMMs (0), the tensor-core GEMMs
@@ -491,6 +502,11 @@ bool res_tc_fits(long rows, long cols, long l);
 lx_status res_gemm_tc(bool transposed, const __nv_bfloat16* Wm, const __nv_bfloat16* Wd,
                       long rows, long cols, const float* X, long N, float* C, char* ws,
                       int num_sms, int dev, cudaStream_t s);
+// split-K tensor-core product part[s][M][Npad] = A . B^T over K range s (see
+// lx_compress_tc.cu); the number of ranges used is returned in splits_out
+lx_status tc_splitk_gemm(lx_layer* L, const CUtensorMap& a, const CUtensorMap& b, int M, int Npad,
+                         int K, float* part, int max_splits, int* splits_out, cudaStream_t s,
+                         const char* name);
 // fused correction + SwiGLU (flat layers): the kernel over (anchor, 128-row
 // block, 64 d_ff columns); its per-cluster-row gate / child-row tables are
 // written by the bucketing (k_assign_rows)

@@ -27,6 +27,8 @@
 // commutative, so each sum is bit-identical), leaving lane l with the logits
 // of entries 2l and 2l + 1 of the 8 x 8 block.
 #include <algorithm>
+#include <cmath>
+#include <cstring>
 
 #include "lx_internal.cuh"
 
@@ -329,6 +331,156 @@ k_router_tiled(const __nv_bfloat16* __restrict__ x, const __nv_bfloat16* __restr
   asm volatile("cp.async.wait_group 0;" ::: "memory");
 }
 
+// ---------------------------------------------------------------------------
+// Screened routing (large bf16 batches whose caller needs only the ids and
+// gates).  The tensor cores give approximate logits a_e (bf16 products, fp32
+// accumulation in the tensor core's order, K ranges added in order); their
+// distance to the canonical fp32 logits l_e is at most eps = RS_EPS_REL *
+// ||x_t|| * max_e ||W_r[e]|| (Cauchy-Schwarz bounds sum_h |x_h w_h| by the
+// norms; RS_EPS_REL is several times a per-MMA-step bound of 2^-20 of that sum
+// over H/16 steps, plus the canonical order's own 69 fp32 roundings).  If L is
+// the k-th largest a_e, every expert of the exact top-k has a_e >= L - 2 eps
+// (an expert with a_f > l_(k) + eps has l_f > l_(k), so at most k - 1 of them
+// exceed l_(k) + eps, i.e. L <= l_(k) + eps; and a_e >= l_e - eps >= l_(k) - eps).
+// So the canonical logits of the candidates {e : a_e >= L - 2 eps} decide the
+// top-k exactly as all E logits would: the same warp top-k runs on them (the
+// others are -inf) and gives the same ids, order and gates.  A token with more
+// than RS_MAX_CAND candidates, or a non-finite value, takes all E exact logits.
+// ---------------------------------------------------------------------------
+constexpr float RS_EPS_REL = 1e-3f;
+constexpr int RS_MAX_CAND = 32;
+constexpr int RS_WARPS = 8;
+constexpr int RS_U = 4;  // 16-byte weight chunks of a lane in flight per candidate
+
+template <int EPL>
+__global__ void __launch_bounds__(RS_WARPS * 32, 4)
+k_router_screen(const float* __restrict__ part, int splits, int Epad,
+                const __nv_bfloat16* __restrict__ x, const __nv_bfloat16* __restrict__ W,
+                const float* __restrict__ bias, int T, int E, int H, float wmax, int k,
+                int* __restrict__ topk_id, float* __restrict__ topk_w) {
+  extern __shared__ __align__(16) unsigned char smem[];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  __nv_bfloat16* xs = reinterpret_cast<__nv_bfloat16*>(smem) + (size_t)warp * H;
+  float* ls = reinterpret_cast<float*>(smem + (size_t)RS_WARPS * H * 2) + (size_t)warp * E;
+  pdl_wait();
+  const int t = blockIdx.x * RS_WARPS + warp;
+  if (t >= T) return;
+  // the token's row into shared memory, and ||x_t||^2
+  const uint4* xr = reinterpret_cast<const uint4*>(x + (size_t)t * H);
+  uint4* xw = reinterpret_cast<uint4*>(xs);
+  float ss = 0.f;
+  for (int i = lane; i < H / 8; i += 32) {
+    const uint4 v = __ldg(xr + i);
+    xw[i] = v;
+    const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const float a = __uint_as_float(w4[q] << 16), b = __uint_as_float(w4[q] & 0xFFFF0000u);
+      ss = fmaf(a, a, ss);
+      ss = fmaf(b, b, ss);
+    }
+  }
+#pragma unroll
+  for (int o = 16; o >= 1; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+  // the approximate logits (K ranges in order, then the bias)
+  float ap[EPL];
+  bool finite = ss == ss && ss <= 3.0e38f;
+#pragma unroll
+  for (int i = 0; i < EPL; ++i) {
+    const int e = lane + 32 * i;
+    float v = 0.f;
+    if (e < E) {
+      for (int sp = 0; sp < splits; ++sp) v += part[((size_t)sp * T + t) * Epad + e];
+      if (bias) v += bias[e];
+      finite = finite && (v - v == 0.f);
+      ls[e] = v;
+    }
+    ap[i] = v;
+  }
+  finite = __all_sync(0xffffffffu, finite);
+  __syncwarp();
+  unsigned cand[EPL];
+  int ncand = E;
+  if (finite) {
+    // the k-th largest approximate logit
+    int sid;
+    float sw;
+    warp_topk(ls, E, k, sid, sw);
+    const float Lk = ls[__shfl_sync(0xffffffffu, sid, k - 1)];
+    // both terms of the bound, with a margin for the fp32 norm itself
+    const float eps = RS_EPS_REL * sqrtf(ss) * 1.001f * wmax;
+    ncand = 0;
+#pragma unroll
+    for (int i = 0; i < EPL; ++i) {
+      const int e = lane + 32 * i;
+      cand[i] = __ballot_sync(0xffffffffu, e < E && ap[i] >= Lk - 2.f * eps);
+      ncand += __popc(cand[i]);
+    }
+  }
+  if (!finite || ncand > RS_MAX_CAND) {
+#pragma unroll
+    for (int i = 0; i < EPL; ++i) cand[i] = (lane + 32 * i) < E ? 0xffffffffu : 0u;
+#pragma unroll
+    for (int i = 0; i < EPL; ++i) cand[i] = __ballot_sync(0xffffffffu, lane + 32 * i < E);
+  }
+  __syncwarp();
+  // non-candidates can never be selected
+#pragma unroll
+  for (int i = 0; i < EPL; ++i) {
+    const int e = lane + 32 * i;
+    if (e < E && !((cand[i] >> lane) & 1u)) ls[e] = -INFINITY;
+  }
+  __syncwarp();
+  // canonical fp32 logits of the candidates: lane j accumulates the 8-element
+  // chunks q = j, j + 32, ... of the dot product with fused multiply-adds in
+  // ascending order; the lane partials are added at offsets 16, 8, 4, 2, 1
+  // (lane j, j < off, adds lane j + off's); the bias last
+  const int nchunk = H / 8;
+  auto lane_partial = [&](int e) {
+    const uint4* wr = reinterpret_cast<const uint4*>(W + (size_t)e * H);
+    float acc = 0.f;
+    for (int q0 = lane; q0 < nchunk; q0 += 32 * RS_U) {
+      uint4 wv[RS_U];
+#pragma unroll
+      for (int u = 0; u < RS_U; ++u)
+        wv[u] = q0 + 32 * u < nchunk ? __ldg(wr + q0 + 32 * u) : make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+      for (int u = 0; u < RS_U; ++u) {
+        if (q0 + 32 * u >= nchunk) break;
+        const uint4 xv = xw[q0 + 32 * u];
+        const uint32_t ww[4] = {wv[u].x, wv[u].y, wv[u].z, wv[u].w};
+        const uint32_t xx[4] = {xv.x, xv.y, xv.z, xv.w};
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          acc = __fmaf_rn(__uint_as_float(xx[c] << 16), __uint_as_float(ww[c] << 16), acc);
+          acc = __fmaf_rn(__uint_as_float(xx[c] & 0xFFFF0000u),
+                          __uint_as_float(ww[c] & 0xFFFF0000u), acc);
+        }
+      }
+    }
+    return acc;
+  };
+#pragma unroll
+  for (int i = 0; i < EPL; ++i) {
+    for (unsigned m = cand[i]; m; m &= m - 1) {
+      const int e = 32 * i + __ffs(m) - 1;
+      float acc = lane_partial(e);
+#pragma unroll
+      for (int off = 16; off >= 1; off >>= 1)
+        acc = __fadd_rn(acc, __shfl_down_sync(0xffffffffu, acc, off));
+      if (lane == 0) ls[e] = bias ? __fadd_rn(acc, bias[e]) : acc;
+    }
+  }
+  __syncwarp();
+  int id;
+  float w;
+  warp_topk(ls, E, k, id, w);
+  if (lane < k) {
+    topk_id[(size_t)t * k + lane] = id;
+    topk_w[(size_t)t * k + lane] = w;
+  }
+}
+
 }  // namespace
 
 bool router_is_tiled(const lx_layer* L, int T) {
@@ -338,10 +490,41 @@ bool router_is_tiled(const lx_layer* L, int T) {
 }
 
 lx_status launch_router(lx_layer* L, const void* x, int T, int k, float* logits, int* topk_id,
-                        float* topk_w, cudaStream_t s) {
+                        float* topk_w, cudaStream_t s, bool need_logits) {
   if (reinterpret_cast<uintptr_t>(x) % 16)
     return fail(LX_ERR_ARG, "x must be 16-byte aligned");
   const int tiles = (T + RT_TOK - 1) / RT_TOK;
+  if (!need_logits && L->router_screen && router_is_tiled(L, T)) {
+    // screened: approximate logits on the tensor cores, then the candidates'
+    // canonical logits and the top-k (the logits buffer is not written)
+    CUtensorMap xm;
+    std::memset(&xm, 0, sizeof(xm));
+    if (!encode_bf16_2d(&xm, x, L->H, T, 64, 128))
+      return fail(LX_ERR_CUDA, "cuTensorMapEncodeTiled(x) failed");
+    const int Epad = router_epad(L);
+    int splits = 1;
+    LX_TRY(tc_splitk_gemm(L, xm, L->router_map, T, Epad, L->H, L->ws.rs_part, RS_MAX_SPLITS,
+                          &splits, s, "router_screen"));
+    const size_t smem = (size_t)RS_WARPS * ((size_t)L->H * 2 + (size_t)L->E * 4);
+    if (smem > 200 * 1024) return fail(LX_ERR_SHAPE, "router screening rows exceed shared memory");
+    const unsigned grid = (unsigned)((T + RS_WARPS - 1) / RS_WARPS);
+    ProfScope ps(L, s, "router_select");
+    if (L->E <= 128) {
+      static bool done4[64] = {};
+      LX_CUDA(smem_cap_once((const void*)k_router_screen<4>, 200 * 1024, L->device, done4));
+      launch_k(L, k_router_screen<4>, grid, RS_WARPS * 32, smem, s, (const float*)L->ws.rs_part,
+               splits, Epad, (const __nv_bfloat16*)x, (const __nv_bfloat16*)L->router_w,
+               (const float*)L->router_bias, T, L->E, L->H, L->router_wmax, k, topk_id, topk_w);
+    } else {
+      static bool done8[64] = {};
+      LX_CUDA(smem_cap_once((const void*)k_router_screen<8>, 200 * 1024, L->device, done8));
+      launch_k(L, k_router_screen<8>, grid, RS_WARPS * 32, smem, s, (const float*)L->ws.rs_part,
+               splits, Epad, (const __nv_bfloat16*)x, (const __nv_bfloat16*)L->router_w,
+               (const float*)L->router_bias, T, L->E, L->H, L->router_wmax, k, topk_id, topk_w);
+    }
+    LX_CUDA(cudaGetLastError());
+    return LX_OK;
+  }
   if (router_is_tiled(L, T)) {
     // large batch: persistent register-tiled kernel
     const size_t smem2 = 2 * (size_t)RTT_TOK * L->H * 2 + (size_t)RTT_TOK * L->E * 4;
