@@ -128,6 +128,12 @@ LX_API lx_status lx_reserve(lx_layer* layer, int32_t max_tokens, int32_t k);
  *   x:       device [T][H] (layer dtype)
  *   topk_id: device [T][k] int32 out;  topk_w: device [T][k] fp32 out
  *   logits:  device [T][E] fp32 out, or NULL
+ * With logits == NULL, large bf16 batches (at least 8 tokens per SM; H a
+ * multiple of 64, E <= 256) may take the screened form: approximate logits on
+ * the tensor cores, and the canonical logits only of the experts whose
+ * approximate logit is within twice a proven error bound of the k-th largest
+ * (a set that contains the exact top-k); topk_id and topk_w are then identical
+ * to the full router's, bit for bit.  lx_moe_forward routes this way.
  * Also leaves the routing in the layer for lx_bucket / lx_get_buckets.
  * Errors: LX_ERR_ARG (k < 1, k > min(E, LX_MAX_K), T < 0, null pointers).
  */
