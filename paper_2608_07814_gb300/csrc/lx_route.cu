@@ -29,6 +29,7 @@
 #include <algorithm>
 #include <cmath>
 #include <cstring>
+#include <type_traits>
 
 #include "lx_internal.cuh"
 
@@ -47,6 +48,21 @@ __device__ __forceinline__ void widen8(const uint4& u, float (&v)[8]) {
     v[2 * i] = __uint_as_float(w[i] << 16);
     v[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
   }
+}
+
+// acc += lo(x) lo(w), then acc += hi(x) hi(w) for the two bf16 halves of the
+// packed words x and w: the mixed-precision fma (bf16 operands, fp32 addend and
+// result) rounds each product-sum once, exactly as fmaf on the widened
+// operands (widening bf16 to fp32 is exact), without the widening operations
+__device__ __forceinline__ float fma_bf16_pair(float acc, uint32_t x, uint32_t w) {
+  asm("{\n\t.reg .b16 xl, xh, wl, wh;\n\t"
+      "mov.b32 {xl, xh}, %1;\n\t"
+      "mov.b32 {wl, wh}, %2;\n\t"
+      "fma.rn.f32.bf16 %0, xl, wl, %0;\n\t"
+      "fma.rn.f32.bf16 %0, xh, wh, %0;\n\t}"
+      : "+f"(acc)
+      : "r"(x), "r"(w));
+  return acc;
 }
 
 // 8 consecutive elements as fp32 (bf16: one 16-byte load; fp32: two)
@@ -78,13 +94,21 @@ k_router_logits(const T* __restrict__ x, const T* __restrict__ W, const float* _
   const int e_end = min(E, e_begin + experts_per_cta);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
   const int nchunk = H / 8;
-  // weight chunks q0 + 32u (u < RT_PREF) of expert e: independent 16-byte loads
-  float wv[RT_PREF][8];
+  // weight chunks q0 + 32u (u < RT_PREF) of expert e: independent 16-byte
+  // loads (bf16: kept packed, multiplied by the mixed-precision fma)
+  constexpr bool kBF = std::is_same<T, __nv_bfloat16>::value;
+  float wv[kBF ? 1 : RT_PREF][8];
+  uint4 wr[kBF ? RT_PREF : 1];
   auto load_w = [&](int e, int q0) {
 #pragma unroll
     for (int u = 0; u < RT_PREF; ++u) {
       const int q = q0 + 32 * u;
-      if (q < nchunk) load8(W + (size_t)e * H + 8 * q, wv[u]);
+      if (q < nchunk) {
+        if constexpr (kBF)
+          wr[u] = *reinterpret_cast<const uint4*>(W + (size_t)e * H + 8 * q);
+        else
+          load8(W + (size_t)e * H + 8 * q, wv[u]);
+      }
     }
   };
   // The router matrix is a layer constant: the first expert's weights are
@@ -118,10 +142,18 @@ k_router_logits(const T* __restrict__ x, const T* __restrict__ W, const float* _
 #pragma unroll
         for (int tt = 0; tt < RT_TOK; ++tt) {
           if (tt < nt) {
-            float xv[8];
-            load8(xs + (size_t)tt * H + 8 * q, xv);
+            if constexpr (kBF) {
+              const uint4 xr = *reinterpret_cast<const uint4*>(xs + (size_t)tt * H + 8 * q);
+              acc[tt] = fma_bf16_pair(acc[tt], xr.x, wr[u].x);
+              acc[tt] = fma_bf16_pair(acc[tt], xr.y, wr[u].y);
+              acc[tt] = fma_bf16_pair(acc[tt], xr.z, wr[u].z);
+              acc[tt] = fma_bf16_pair(acc[tt], xr.w, wr[u].w);
+            } else {
+              float xv[8];
+              load8(xs + (size_t)tt * H + 8 * q, xv);
 #pragma unroll
-            for (int i = 0; i < 8; ++i) acc[tt] = __fmaf_rn(xv[i], wv[u][i], acc[tt]);
+              for (int i = 0; i < 8; ++i) acc[tt] = __fmaf_rn(xv[i], wv[u][i], acc[tt]);
+            }
           }
         }
       }
@@ -350,10 +382,10 @@ k_router_tiled(const __nv_bfloat16* __restrict__ x, const __nv_bfloat16* __restr
 constexpr float RS_EPS_REL = 1e-3f;
 constexpr int RS_MAX_CAND = 32;
 constexpr int RS_WARPS = 8;
-constexpr int RS_U = 4;  // 16-byte weight chunks of a lane in flight per candidate
+constexpr int RS_U = 4;  // 16-byte weight chunks of a lane in flight per candidate (two candidates)
 
 template <int EPL>
-__global__ void __launch_bounds__(RS_WARPS * 32, 4)
+__global__ void __launch_bounds__(RS_WARPS * 32, 3)
 k_router_screen(const float* __restrict__ part, int splits, int Epad,
                 const __nv_bfloat16* __restrict__ x, const __nv_bfloat16* __restrict__ W,
                 const float* __restrict__ bias, int T, int E, int H, float wmax, int k,
@@ -435,40 +467,53 @@ k_router_screen(const float* __restrict__ part, int splits, int Epad,
   // chunks q = j, j + 32, ... of the dot product with fused multiply-adds in
   // ascending order; the lane partials are added at offsets 16, 8, 4, 2, 1
   // (lane j, j < off, adds lane j + off's); the bias last
+  // Two candidates at a time (two independent chains sharing the x loads).
   const int nchunk = H / 8;
-  auto lane_partial = [&](int e) {
-    const uint4* wr = reinterpret_cast<const uint4*>(W + (size_t)e * H);
-    float acc = 0.f;
-    for (int q0 = lane; q0 < nchunk; q0 += 32 * RS_U) {
-      uint4 wv[RS_U];
+  auto pop = [&]() {  // the next candidate (warp-uniform), -1 when none is left
+    int e = -1;
 #pragma unroll
-      for (int u = 0; u < RS_U; ++u)
-        wv[u] = q0 + 32 * u < nchunk ? __ldg(wr + q0 + 32 * u) : make_uint4(0u, 0u, 0u, 0u);
+    for (int i = 0; i < EPL; ++i)
+      if (e < 0 && cand[i]) {
+        e = 32 * i + __ffs(cand[i]) - 1;
+        cand[i] &= cand[i] - 1;
+      }
+    return e;
+  };
+  for (int e0 = pop(); e0 >= 0; e0 = pop()) {
+    const int e1 = pop();
+    const uint4* w0 = reinterpret_cast<const uint4*>(W + (size_t)e0 * H);
+    const uint4* w1 = reinterpret_cast<const uint4*>(W + (size_t)(e1 >= 0 ? e1 : e0) * H);
+    float acc0 = 0.f, acc1 = 0.f;
+    for (int q0 = lane; q0 < nchunk; q0 += 32 * RS_U) {
+      uint4 wv0[RS_U], wv1[RS_U];
+#pragma unroll
+      for (int u = 0; u < RS_U; ++u) {
+        const bool in = q0 + 32 * u < nchunk;
+        wv0[u] = in ? __ldg(w0 + q0 + 32 * u) : make_uint4(0u, 0u, 0u, 0u);
+        wv1[u] = in && e1 >= 0 ? __ldg(w1 + q0 + 32 * u) : make_uint4(0u, 0u, 0u, 0u);
+      }
 #pragma unroll
       for (int u = 0; u < RS_U; ++u) {
         if (q0 + 32 * u >= nchunk) break;
         const uint4 xv = xw[q0 + 32 * u];
-        const uint32_t ww[4] = {wv[u].x, wv[u].y, wv[u].z, wv[u].w};
-        const uint32_t xx[4] = {xv.x, xv.y, xv.z, xv.w};
-#pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          acc = __fmaf_rn(__uint_as_float(xx[c] << 16), __uint_as_float(ww[c] << 16), acc);
-          acc = __fmaf_rn(__uint_as_float(xx[c] & 0xFFFF0000u),
-                          __uint_as_float(ww[c] & 0xFFFF0000u), acc);
-        }
+        acc0 = fma_bf16_pair(acc0, xv.x, wv0[u].x);
+        acc1 = fma_bf16_pair(acc1, xv.x, wv1[u].x);
+        acc0 = fma_bf16_pair(acc0, xv.y, wv0[u].y);
+        acc1 = fma_bf16_pair(acc1, xv.y, wv1[u].y);
+        acc0 = fma_bf16_pair(acc0, xv.z, wv0[u].z);
+        acc1 = fma_bf16_pair(acc1, xv.z, wv1[u].z);
+        acc0 = fma_bf16_pair(acc0, xv.w, wv0[u].w);
+        acc1 = fma_bf16_pair(acc1, xv.w, wv1[u].w);
       }
     }
-    return acc;
-  };
 #pragma unroll
-  for (int i = 0; i < EPL; ++i) {
-    for (unsigned m = cand[i]; m; m &= m - 1) {
-      const int e = 32 * i + __ffs(m) - 1;
-      float acc = lane_partial(e);
-#pragma unroll
-      for (int off = 16; off >= 1; off >>= 1)
-        acc = __fadd_rn(acc, __shfl_down_sync(0xffffffffu, acc, off));
-      if (lane == 0) ls[e] = bias ? __fadd_rn(acc, bias[e]) : acc;
+    for (int off = 16; off >= 1; off >>= 1) {
+      acc0 = __fadd_rn(acc0, __shfl_down_sync(0xffffffffu, acc0, off));
+      acc1 = __fadd_rn(acc1, __shfl_down_sync(0xffffffffu, acc1, off));
+    }
+    if (lane == 0) {
+      ls[e0] = bias ? __fadd_rn(acc0, bias[e0]) : acc0;
+      if (e1 >= 0) ls[e1] = bias ? __fadd_rn(acc1, bias[e1]) : acc1;
     }
   }
   __syncwarp();
