@@ -108,6 +108,21 @@ bool encode_bf16_2d(CUtensorMap* m, const void* base, long inner, long outer, in
          CUDA_SUCCESS;
 }
 
+// TMA store map of a bf16 output buffer [rows][ld]: 32 x 32 boxes staged with
+// the 64-byte swizzle (the 256-row tensor-core epilogue)
+static bool encode_store_map(CUtensorMap* m, void* base, long rows, long ld) {
+  auto encode = get_encode();
+  if (!encode || (ld * 2) % 16 != 0) return false;
+  const cuuint64_t dims[2] = {(cuuint64_t)ld, (cuuint64_t)rows};
+  const cuuint64_t strides[1] = {(cuuint64_t)ld * 2};
+  const cuuint32_t box[2] = {32, 32};
+  const cuuint32_t estr[2] = {1, 1};
+  return encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, dims, strides, box, estr,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B,
+                CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) ==
+         CUDA_SUCCESS;
+}
+
 // TMA map of a bf16 activation buffer [rows][ld] read as box_rows x 64-column
 // boxes with the 128-byte swizzle (an A operand whose rows are already in
 // node-row order)
@@ -184,6 +199,7 @@ static lx_status ensure_workspace(lx_layer* L, int T, int k, cudaStream_t s) {
       {(void**)&w.Pal, L->ct ? (size_t)2 * Rmax * L->ct_nch * 2 * rmax : 0},
       {(void**)&w.Qal, L->ct ? (size_t)2 * Rmax * L->ct_nch * rmax : 0},
       {(void**)&w.pamap, L->ct ? 3 * sizeof(CUtensorMap) : 0},
+      {(void**)&w.omaps, 2 * sizeof(CUtensorMap)},
       {(void**)&w.rs_part, L->router_screen
                                ? sizeof(float) * RS_MAX_SPLITS * (size_t)cT * router_epad(L) : 0},
   };
@@ -248,6 +264,19 @@ static lx_status ensure_workspace(lx_layer* L, int T, int k, cudaStream_t s) {
     e = cudaMemcpyAsync(w.pamap, pm, 3 * sizeof(CUtensorMap), cudaMemcpyHostToDevice, s);
     if (e == cudaSuccess) e = cudaStreamSynchronize(s);
     if (e != cudaSuccess) return cuda_fail(e, "copy Pal map");
+  }
+  {
+    // TMA store maps of the anchor products' outputs (hb [R][2I], yb [R][H]);
+    // left null (row-by-row stores) where the row pitch is not 16-byte aligned
+    CUtensorMap om[2];
+    std::memset(om, 0, sizeof(om));
+    if (encode_store_map(&om[0], w.hb, Rmax, 2L * L->I) && encode_store_map(&om[1], w.yb, Rmax, L->H)) {
+      e = cudaMemcpyAsync(w.omaps, om, 2 * sizeof(CUtensorMap), cudaMemcpyHostToDevice, s);
+      if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+      if (e != cudaSuccess) return cuda_fail(e, "copy store maps");
+    } else {
+      w.omaps = nullptr;
+    }
   }
   L->last_T = L->last_k = 0;
   return LX_OK;

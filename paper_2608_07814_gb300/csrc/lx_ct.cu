@@ -16,12 +16,12 @@
 // separate pass.  z_c feeds the shared down product of the anchor and a_e the
 // member's down correction (by linearity of the down projection).
 //
-// One persistent CTA per SM, 8 warps:
+// One persistent CTA per SM, 12 warps (warp 3 has no role):
 //   warp 2      scheduler: claims tiles (anchor, 128-row block, 64-column
 //               chunk; chunks of a block are consecutive, so the block's P
 //               rows are re-read from L2) and decodes them into a queue;
-//   warp 0      producer: per member, per gate/up half, per 64-wide K block of
-//               the rank: one stage = the 128 P rows (one TMA box of the
+//   warp 0      producer: per member, per 64-wide K block of the rank, the
+//               gate then the up half: one stage = the 128 P rows (one TMA box of the
 //               cluster-aligned P buffer) and the 64 U rows of the chunk (one
 //               64 x 64 box of the member's tiled [Ug;Uu]);
 //   warp 1      allocates 512 TMEM columns (four member accumulators of
@@ -321,8 +321,8 @@ __global__ void __launch_bounds__(CT_THREADS, 1) k_ct_swiglu(const __grid_consta
           bool first = true;
           for (int j = 0; j < t.nch && good; ++j) {
             const int kbn = t.rk[j] / CT_BK;
-            for (int g = 0; g < 2 && good; ++g) {
-              for (int kb = 0; kb < kbn; ++kb) {
+            for (int kb = 0; kb < kbn && good; ++kb) {
+              for (int g = 0; g < 2; ++g) {
                 const uint32_t s = it % S;
                 good = mbar_wait(empty0 + 8 * s, ((it / S) & 1) ^ 1, abort_flag, P.wait_cycles);
                 if (!good) break;
@@ -431,22 +431,29 @@ __global__ void __launch_bounds__(CT_THREADS, 1) k_ct_swiglu(const __grid_consta
           tc_fence_after();
           const uint32_t d = tmem + b * CT_ACC_COLS;
           const int kbn = t.rk[j] / CT_BK;
-          for (int g = 0; g < 2 && ok; ++g) {
-            for (int kb = 0; kb < kbn; ++kb) {
-              s = it % S;
-              if (!mbar_wait(full0 + 8 * s, (it / S) & 1, abort_flag, P.wait_cycles)) {
-                ok = false;
-                break;
-              }
-              tc_fence_after();
-              const uint32_t a_s = smem_base + s * CT_STAGE_BYTES, b_s = a_s + CT_A_BYTES;
-#pragma unroll
-              for (int k = 0; k < CT_BK / 16; ++k)
-                tc_mma(d + g * CT_CW, smem_desc(a_s + 32 * k), smem_desc(b_s + 32 * k), idesc,
-                       (kb | k) != 0 ? 1u : 0u);
-              tc_commit(empty0 + 8 * s);  // frees the stage once these MMAs are done
-              ++it;
+          // per K block, the gate and the up stage: their MMAs alternate between
+          // the two accumulators, so that consecutive MMAs are independent (an
+          // N = 64 MMA is shorter than the latency of accumulating into the
+          // result of the previous one)
+          for (int kb = 0; kb < kbn && ok; ++kb) {
+            const uint32_t s0 = it % S, s1 = (it + 1) % S;
+            if (!mbar_wait(full0 + 8 * s0, (it / S) & 1, abort_flag, P.wait_cycles) ||
+                !mbar_wait(full0 + 8 * s1, ((it + 1) / S) & 1, abort_flag, P.wait_cycles)) {
+              ok = false;
+              break;
             }
+            tc_fence_after();
+            const uint32_t a0 = smem_base + s0 * CT_STAGE_BYTES, b0 = a0 + CT_A_BYTES;
+            const uint32_t a1 = smem_base + s1 * CT_STAGE_BYTES, b1 = a1 + CT_A_BYTES;
+#pragma unroll
+            for (int k = 0; k < CT_BK / 16; ++k) {
+              const uint32_t acc = (kb | k) != 0 ? 1u : 0u;
+              tc_mma(d, smem_desc(a0 + 32 * k), smem_desc(b0 + 32 * k), idesc, acc);
+              tc_mma(d + CT_CW, smem_desc(a1 + 32 * k), smem_desc(b1 + 32 * k), idesc, acc);
+            }
+            tc_commit(empty0 + 8 * s0);  // free the stages once these MMAs are done
+            tc_commit(empty0 + 8 * s1);
+            it += 2;
           }
           if (!ok) break;
           tc_commit(tfull0 + 8 * b);  // the member's accumulator is ready

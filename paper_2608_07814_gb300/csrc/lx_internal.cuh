@@ -263,6 +263,9 @@ struct TcLaunch {
   const int* gather;
   const __nv_bfloat16* xsrc;
   long ldx;
+  // optional TMA map of out (bf16, 32 x 32 boxes, 64-byte swizzle): 256-row
+  // tiles store whole 32-row blocks with TMA (row_map null)
+  const CUtensorMap* omap;
 };
 
 // Fused correction + SwiGLU of flat layers (every correction node a direct
@@ -332,6 +335,7 @@ struct Workspace {
   __nv_bfloat16* Pal = nullptr;
   __nv_bfloat16* Qal = nullptr;  // [R][nch * rmax] the children's z Vd rows, aligned likewise
   CUtensorMap* pamap = nullptr;  // [3] TMA maps of Pal, hb and Qal (128-row boxes)
+  CUtensorMap* omaps = nullptr;  // [2] TMA store maps of hb and yb (null: not encodable)
   // screened routing: the tensor-core logit partials [splits][T][Epad]
   float* rs_part = nullptr;
 };

@@ -63,11 +63,13 @@ struct TcCfg {
   static constexpr int STAGES = (NH == 1 && EPI == 4) ? 4 : 3;
   static constexpr int NBUF = NH == 1 ? 2 : 1;           // accumulators of NH x 256 columns
   static constexpr int THREADS = 32 * (4 + EPI);
-  // 256-row tiles with eight epilogue warps stage 32 bf16 columns per pass
-  // (80-byte rows), so that the staging fits beside the three 64 KiB stages
+  // 256-row tiles with eight epilogue warps stage 32 bf16 columns per pass:
+  // two 2 KiB buffers per warp for TMA stores of 32 x 32 blocks (64-byte rows,
+  // 64-byte swizzle), or 80-byte rows for the row-by-row stores
   static constexpr bool HALF = BM == 256 && EPI == 8;
   static constexpr int EPI_LD = HALF ? 20 : TC_EPI_LD;  // staging row stride (4-byte words)
-  static constexpr int EPI_BYTES = 32 * EPI_LD * 4;
+  static constexpr int EPI_BYTES = HALF ? 4096 : 32 * EPI_LD * 4;
+  static_assert(!HALF || 32 * EPI_LD * 4 <= EPI_BYTES, "row-by-row staging fits the buffers");
   static_assert(EPI == 4 || EPI == 8, "four or eight epilogue warps");
   static_assert(STAGE_BYTES % 1024 == 0, "stages keep the 1024-byte swizzle alignment");
   static_assert(NBUF * NH * TC_ACC_COLS <= TC_TMEM_COLS, "accumulators fit the TMEM allocation");
@@ -479,7 +481,8 @@ k_tc_gemm(const __grid_constant__ TcLaunch P) {
     const int ew = warp & 3;        // TMEM lanes 32 ew .. 32 ew + 31
     const int eh = (warp - 4) >> 2; // with 8 warps: which column passes (alternate)
     constexpr int ESTEP = EPI / 4;  // passes are dealt out to ESTEP warps per quadrant
-    float* stg = epi + (warp - 4) * 32 * C::EPI_LD;
+    float* stg = epi + (warp - 4) * (C::EPI_BYTES / 4);  // 1024-byte aligned
+    uint32_t nstore = 0;  // TMA stores issued by this warp (lane 0), alternating buffers
     uint32_t tiles = 0;
     while (true) {
       const uint32_t b = tiles % NBUF, u = tiles / NBUF;
@@ -496,18 +499,32 @@ k_tc_gemm(const __grid_constant__ TcLaunch P) {
       const long col0 = (long)t.grp * t.Ng + t.row0 + (P.node_col ? P.node_col[t.node] : 0);
       const bool tile_ok = t.tok0 >= 0 && col0 + t.BN <= P.ldo;
       const int cq = lane & 7;
-      for (int h = 0; h < NH && 128 * h < t.M; ++h) {
-      const uint32_t acc = tmem + (b * NH + h) * TC_ACC_COLS;
-      // output rows of this warp's 32 tile rows (remapped when row_map is set)
-      long orow_l = (long)t.tok0 + 128 * h + 32 * ew + lane;
-      if (P.row_map)
-        orow_l = (32 * ew + lane + 128 * h < t.M && orow_l < P.rows_cap) ? P.row_map[orow_l] : -1;
       if constexpr (C::HALF) {
         // bf16, 32 columns per pass: one TMEM load, rows staged 64 bytes wide,
-        // stored as 64-byte row segments (four lanes per row, eight rows a pass)
-        for (int c0 = 32 * eh; c0 < t.BN; c0 += 32 * ESTEP) {
-          uint32_t r0[32];
-          tc_ld32_async(acc + ((uint32_t)(32 * ew) << 16) + (uint32_t)c0, r0);
+        // stored as 64-byte row segments (four lanes per row, eight rows a
+        // pass).  The passes of both 128-row halves form one sequence, and the
+        // next pass's TMEM load is issued before this pass's stores, so that
+        // its latency is spent storing.
+        const int nhh = t.M > 128 ? 2 : 1;
+        const int pph = t.BN > 32 * eh ? (t.BN - 32 * eh + 32 * ESTEP - 1) / (32 * ESTEP) : 0;
+        const int npass = nhh * pph;
+        auto pass_taddr = [&](int p) {
+          const int h = p / pph, c0 = 32 * eh + (p - h * pph) * 32 * ESTEP;
+          return tmem + (b * NH + h) * TC_ACC_COLS + ((uint32_t)(32 * ew) << 16) + (uint32_t)c0;
+        };
+        uint32_t r0[32];
+        if (npass > 0) tc_ld32_async(pass_taddr(0), r0);
+        long orow_l = 0;
+        int hcur = -1;
+        for (int p = 0; p < npass; ++p) {
+          const int h = p / pph, c0 = 32 * eh + (p - h * pph) * 32 * ESTEP;
+          if (h != hcur) {
+            // output rows of this warp's 32 tile rows (remapped when row_map is set)
+            hcur = h;
+            orow_l = (long)t.tok0 + 128 * h + 32 * ew + lane;
+            if (P.row_map)
+              orow_l = (32 * ew + lane + 128 * h < t.M && orow_l < P.rows_cap) ? P.row_map[orow_l] : -1;
+          }
           tc_wait_ld();
           uint32_t pk[16];
 #pragma unroll
@@ -516,6 +533,32 @@ k_tc_gemm(const __grid_constant__ TcLaunch P) {
                                                       __uint_as_float(r0[2 * e + 1]));
             pk[e] = *reinterpret_cast<uint32_t*>(&b0);
           }
+          if (p + 1 < npass) tc_ld32_async(pass_taddr(p + 1), r0);
+          // a whole 32-row block inside the tile's rows and the buffer, at a
+          // 16-byte-aligned column: one TMA store from the staged block
+          const long grow0 = (long)t.tok0 + 128 * h + 32 * ew;
+          const int xcol = (int)(col0 + c0);
+          if (P.omap && !P.row_map && tile_ok && 128 * h + 32 * ew + 32 <= t.M &&
+              c0 + 32 <= t.BN && grow0 + 32 <= P.rows_cap && (xcol & 7) == 0) {
+            uint8_t* tb = reinterpret_cast<uint8_t*>(stg) + (nstore & 1) * 2048;
+            if (lane == 0) bulk_wait_read<1>();  // the store that used this buffer has read it
+            __syncwarp();
+            // row `lane`, 16-byte chunk q at q ^ ((row / 2) % 4): the 64-byte swizzle
+            uint4* trow = reinterpret_cast<uint4*>(tb + lane * 64);
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
+              trow[q ^ ((lane >> 1) & 3)] = make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            __syncwarp();
+            if (lane == 0) {
+              tma_store_2d(P.omap, xcol, (int)grow0, smem_u32(tb));
+              bulk_commit();
+            }
+            ++nstore;
+            continue;
+          }
+          if (lane == 0) bulk_wait_read<0>();  // the staging is shared with the TMA stores
+          __syncwarp();
           uint4* srow = reinterpret_cast<uint4*>(stg + lane * C::EPI_LD);
 #pragma unroll
           for (int q = 0; q < 4; ++q)
@@ -535,7 +578,14 @@ k_tc_gemm(const __grid_constant__ TcLaunch P) {
           }
           __syncwarp();
         }
-      } else if (P.out_f32) {
+      } else {
+      for (int h = 0; h < NH && 128 * h < t.M; ++h) {
+      const uint32_t acc = tmem + (b * NH + h) * TC_ACC_COLS;
+      // output rows of this warp's 32 tile rows (remapped when row_map is set)
+      long orow_l = (long)t.tok0 + 128 * h + 32 * ew + lane;
+      if (P.row_map)
+        orow_l = (32 * ew + lane + 128 * h < t.M && orow_l < P.rows_cap) ? P.row_map[orow_l] : -1;
+      if (P.out_f32) {
         for (int c0 = 32 * eh; c0 < t.BN; c0 += 32 * ESTEP) {
           float v[32];
           tc_ld32(acc + ((uint32_t)(32 * ew) << 16) + (uint32_t)c0, v);
@@ -600,11 +650,15 @@ k_tc_gemm(const __grid_constant__ TcLaunch P) {
         }
       }
       }
+      }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(tempty0 + 8 * b);
       ++tiles;
     }
+    // the TMA stores complete before the CTA exits
+    if (lane == 0) bulk_wait_all();
+    __syncwarp();
   }
   // all roles meet before the TMEM is released
   tc_fence_before();
@@ -708,6 +762,7 @@ static TcLaunch tc_op(lx_layer* L, int op, const CUtensorMap* xmap, int xcol, vo
   P.gather = nullptr;
   P.xsrc = nullptr;
   P.ldx = 0;
+  P.omap = nullptr;
   return P;
 }
 
@@ -776,7 +831,11 @@ lx_status launch_tc_experts(lx_layer* L, const void* x, int T, int k, void* y, c
     P.ldx = H;
     return P;
   };
-  LX_TRY(run(tc_op(L, OP_UP_ANCHOR, w.gmap, 0, w.hb, 2 * I, false, 0), "tc_up_anchor"));
+  {
+    TcLaunch ua = tc_op(L, OP_UP_ANCHOR, w.gmap, 0, w.hb, 2 * I, false, 0);
+    ua.omap = w.omaps;  // hb (null when not encodable)
+    LX_TRY(run(ua, "tc_up_anchor"));
+  }
   if (L->ct) {
     // flat layers: the members' x V rows land aligned to their cluster's rows,
     // and one fused kernel adds the corrections and applies the SwiGLU
@@ -798,6 +857,7 @@ lx_status launch_tc_experts(lx_layer* L, const void* x, int T, int k, void* y, c
     dn.kc_wmaps = L->d_tmaps + (size_t)OP_DN_U * L->N;
     dn.kc_xmap = w.pamap + 2;
     dn.kc_slot = (int)rmax;
+    dn.omap = w.omaps ? w.omaps + 1 : nullptr;  // yb
     LX_TRY(run(dn, "tc_dn_anchor_U"));
     return launch_combine(L, T, k, y, true, s, SplitParts(), /*anchors_only=*/true);
   } else {

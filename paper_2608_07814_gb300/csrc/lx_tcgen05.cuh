@@ -62,6 +62,27 @@ static __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorM
       : "memory");
 }
 
+// TMA tile store shared -> global, tracked by the issuing thread's bulk async-groups
+static __device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, int c0, int c1,
+                                             uint32_t src) {
+  asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(c0), "r"(c1), "r"(src)
+               : "memory");
+}
+static __device__ __forceinline__ void bulk_commit() {
+  asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+}
+// at most N of this thread's bulk groups still reading shared memory
+template <int N>
+static __device__ __forceinline__ void bulk_wait_read() {
+  asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
+}
+// every bulk group of this thread complete (its writes performed)
+static __device__ __forceinline__ void bulk_wait_all() {
+  asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+}
+
 // ---- tcgen05 ---------------------------------------------------------------
 // Shared-memory matrix descriptor of a K-major tile whose rows are 128 bytes
 // (64 bf16) with the 128-byte swizzle, rows packed (8-row atoms 1024 bytes
