@@ -44,7 +44,8 @@ constexpr int TC_ACC_COLS = 256;                 // one accumulator
 constexpr int TC_TMEM_COLS = 2 * TC_ACC_COLS;    // double-buffered
 constexpr int TC_EPI_LD = 36;                    // staging row stride (floats)
 constexpr int TC_EPI_BYTES = 32 * TC_EPI_LD * 4; // per epilogue warp
-constexpr int TC_QN = 1;  // decoded tiles queued ahead of the producer (one, as a claim one tile ahead)
+constexpr int TC_QN = 1;
+constexpr int TC_GATHER_WARPS = 2;  // warps gathering the A rows of a gathered product  // decoded tiles queued ahead of the producer (one, as a claim one tile ahead)
 
 // Tile rows BM (tokens): 128 (one M = 128 MMA per K step, two TMEM
 // accumulators so that a tile's epilogue overlaps the next tile's MMAs) or 256
@@ -130,14 +131,15 @@ __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
 }
 
-// GATHER: warp 3 fills the A stages with the tile's token rows, gathered from
+// GATHER: warps 3 and 4 + EPI (TC_GATHER_WARPS, each half of the rows) fill
+// the A stages with the tile's token rows, gathered from
 // x by row -> token (16-byte cp.async, eight lanes per 128-byte row segment,
 // stored in the 128-byte-swizzled K-major layout the MMA reads); a stage is
 // published once its copies have landed (cp.async.wait_group) and been made
 // visible to the tensor core's async proxy (fence.proxy.async), so no copy of
 // the token rows in node-row order is written to memory first.
 template <int BM, int EPI, bool GATHER>
-__global__ void __launch_bounds__(TcCfg<BM, EPI>::THREADS, 1)
+__global__ void __launch_bounds__(TcCfg<BM, EPI>::THREADS + (GATHER ? 32 * (TC_GATHER_WARPS - 1) : 0), 1)
 k_tc_gemm(const __grid_constant__ TcLaunch P) {
   using C = TcCfg<BM, EPI>;
   constexpr int TC_STAGES = C::STAGES, TC_STAGE_BYTES = C::STAGE_BYTES, TC_A_BYTES = C::A_BYTES;
@@ -164,7 +166,9 @@ k_tc_gemm(const __grid_constant__ TcLaunch P) {
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < TC_STAGES; ++s) {
-      mbar_init(full0 + 8 * s, 1 + 32);  // producer arrival + one per producer lane
+      // the producer's arrival (with the bytes) + one per lane of the producer
+      // (or of every gather warp)
+      mbar_init(full0 + 8 * s, 1 + 32 * (GATHER ? TC_GATHER_WARPS : 1));
       mbar_init(empty0 + 8 * s, 1);      // tcgen05.commit
     }
     for (int b = 0; b < 2; ++b) {
@@ -174,7 +178,7 @@ k_tc_gemm(const __grid_constant__ TcLaunch P) {
     mbar_init(drain, 1);
     for (int q = 0; q < TC_QN; ++q) {
       mbar_init(qfull0 + 8 * q, 1);   // the scheduler's arrival (tile written)
-      mbar_init(qempty0 + 8 * q, GATHER ? 2 : 1);  // the producer's (and gather warp's) arrival
+      mbar_init(qempty0 + 8 * q, GATHER ? 1 + TC_GATHER_WARPS : 1);  // producer (+ gather warps)
     }
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -294,12 +298,15 @@ k_tc_gemm(const __grid_constant__ TcLaunch P) {
       *abort_flag = 1;
     }
     prod_it = it;
-  } else if (GATHER && warp == 3) {
+  } else if (GATHER && (warp == 3 || warp >= 4 + EPI)) {
     // ------------------------------------------------------------ gather
-    // Same tiles and stages as the producer: per stage, rows m = 4 i + r8 of
-    // the tile (lanes 8 r8 .. 8 r8 + 7), 16-byte unit u of the stage's 64-wide
-    // K slice; up to TC_STAGES - 1 stages in flight before the oldest is
-    // published (32 arrivals on its full barrier).
+    // Same tiles and stages as the producer: gather warp gw takes rows
+    // m = 4 i + r8 of the tile for i in its half (lanes 8 r8 .. 8 r8 + 7),
+    // 16-byte unit u of the stage's 64-wide K slice; up to TC_STAGES - 1
+    // stages in flight before the oldest is published (32 arrivals per warp
+    // on its full barrier).
+    constexpr int GR = BM / 4 / TC_GATHER_WARPS;  // row groups of a gather warp
+    const int gw = warp == 3 ? 0 : warp - (4 + EPI) + 1;
     const int r8 = lane >> 3, u = lane & 7;
     uint32_t it = 0, qi = 0, pq = 0;
     int np = 0;
@@ -325,11 +332,14 @@ k_tc_gemm(const __grid_constant__ TcLaunch P) {
       if (lane == 0) mbar_arrive(qempty0 + 8 * q);
       ++qi;
       if (t.BN < 0) break;
-      int trow[BM / 4];  // token of row 4 i + r8, or -1 past the bucket
+      // this lane's source row addresses (16-byte unit u of the row's first
+      // K slice), or null past the bucket
+      const __nv_bfloat16* src[GR];
 #pragma unroll
-      for (int i = 0; i < BM / 4; ++i) {
-        const int m = 4 * i + r8;
-        trow[i] = (m < t.M && (long)t.tok0 + m < P.rows_cap) ? __ldg(P.gather + t.tok0 + m) : -1;
+      for (int i = 0; i < GR; ++i) {
+        const int m = 4 * (gw * GR + i) + r8;
+        const int tr = (m < t.M && (long)t.tok0 + m < P.rows_cap) ? __ldg(P.gather + t.tok0 + m) : -1;
+        src[i] = tr >= 0 ? P.xsrc + (size_t)tr * P.ldx + (size_t)(t.grp * t.K) + 8 * u : nullptr;
       }
       const int nkb = (t.K + TC_BK - 1) / TC_BK;
       for (int kb = 0; kb < nkb; ++kb, ++it) {
@@ -344,12 +354,10 @@ k_tc_gemm(const __grid_constant__ TcLaunch P) {
           break;
         }
         const uint32_t a_s = smem_base + s * TC_STAGE_BYTES;
-        const __nv_bfloat16* xk = P.xsrc + (size_t)(t.grp * t.K + kb * TC_BK) + 8 * u;
 #pragma unroll
-        for (int i = 0; i < BM / 4; ++i) {
-          const int m = 4 * i + r8;
-          if (trow[i] >= 0)
-            cp_async16(a_s + m * 128 + ((u ^ (m & 7)) << 4), xk + (size_t)trow[i] * P.ldx);
+        for (int i = 0; i < GR; ++i) {
+          const int m = 4 * (gw * GR + i) + r8;
+          if (src[i]) cp_async16(a_s + m * 128 + ((u ^ (m & 7)) << 4), src[i] + kb * TC_BK);
         }
         asm volatile("cp.async.commit_group;" ::: "memory");
         pq |= s << (8 * np);
@@ -476,7 +484,7 @@ k_tc_gemm(const __grid_constant__ TcLaunch P) {
       }
     }
     __syncwarp();
-  } else if (warp >= 4) {
+  } else if (warp >= 4 && warp < 4 + EPI) {
     // ------------------------------------------------------------ epilogue
     const int ew = warp & 3;        // TMEM lanes 32 ew .. 32 ew + 31
     const int eh = (warp - 4) >> 2; // with 8 warps: which column passes (alternate)
@@ -707,7 +715,8 @@ static lx_status launch_tc_cfg(lx_layer* L, const TcLaunch& P, cudaStream_t s, c
   static bool done[64] = {};
   LX_CUDA(smem_cap_once((const void*)k_tc_gemm<BM, EPI, GATHER>, smem, L->device, done));
   ProfScope ps(L, s, name);
-  launch_k(L, k_tc_gemm<BM, EPI, GATHER>, L->num_sms, TcCfg<BM, EPI>::THREADS, smem, s, P);
+  launch_k(L, k_tc_gemm<BM, EPI, GATHER>, L->num_sms,
+           TcCfg<BM, EPI>::THREADS + (GATHER ? 32 * (TC_GATHER_WARPS - 1) : 0), smem, s, P);
   LX_CUDA(cudaGetLastError());
   return LX_OK;
 }
