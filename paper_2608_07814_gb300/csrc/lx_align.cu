@@ -10,14 +10,21 @@
 // three K segments (gate rows, up rows: K-major; down columns: MN-major) staged
 // through shared memory in 32-deep chunks; the tile's row norms are summed
 // from the same staged chunks, so every operand byte is read once per tile.
-// k_align_cost_mma: the same tile for bf16 experts on the tensor cores
-// (mma.sync, bf16 inputs, fp32 accumulation).
+// Tensor-core form (bf16 experts, d_model a multiple of 256): both experts'
+// neuron vectors are packed K-major, cat[i] = (gate[i, :], up[i, :], down[:, i])
+// (the down columns transposed through shared memory, the gate/up rows
+// copies; k_align_pack, which also takes ||cat[i]||^2), one tcgen05 split-K GEMM forms the
+// dot products (bf16 operands, fp32 accumulation; 256-column chunks of the
+// member's neurons in one launch), and k_align_finish adds the K ranges in
+// order and forms C.  k_align_cost_mma: the 64 x 64 tile form (mma.sync) for
+// the other bf16 shapes.
 // k_permute_rows / k_permute_cols: gathers (bit-exact copies).
 // lx_lap_solve / lx_lap_solve_batch: the exact assignment on the host (Jonker
 // and Volgenant: column reduction, augmenting row reduction, then shortest
 // augmenting paths with dual potentials); the batch form spreads independent
 // problems over host threads.
 #include <algorithm>
+#include <cstring>
 #include <atomic>
 #include <limits>
 #include <thread>
@@ -297,6 +304,129 @@ k_align_cost_mma(const __nv_bfloat16* __restrict__ dg, const __nv_bfloat16* __re
     }
 }
 
+// Packs one expert (blockIdx.z: 0 dominant, 1 member) for the tensor-core
+// cost: cat[i] = (gate[i, :], up[i, :], down[:, i]) as K-major bf16 rows of
+// 3H, and the squared norms of the pieces.  A CTA owns 32 neurons (warp w
+// rows 4 w .. 4 w + 3) and one 256-wide range hb of d_model: the gate and up
+// pieces are copied in 16-byte units, the down columns pass through shared
+// memory in 64 (h) x 32 (i) blocks; each lane sums its squares in a fixed
+// order (gate, up, then the down blocks), the 32 lane partials of a row are
+// added by a shuffle tree into npart[hb][i] (the ranges are added in order
+// by k_align_finish).  H is a multiple of 256.
+constexpr int AP_HB = 256;
+struct AlignPackArgs {
+  const __nv_bfloat16* g[2];
+  const __nv_bfloat16* u[2];
+  const __nv_bfloat16* d[2];
+  __nv_bfloat16* cat[2];
+  float* npart[2];  // [H / AP_HB][I]
+};
+__global__ void __launch_bounds__(256) k_align_pack(const AlignPackArgs A, int H, int I) {
+  __shared__ __align__(16) __nv_bfloat16 blk[64][34];
+  const int x = blockIdx.z, i0 = blockIdx.x * 32, hb = blockIdx.y;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const long K = 3L * H;
+  const __nv_bfloat16* g = A.g[x];
+  const __nv_bfloat16* u = A.u[x];
+  const __nv_bfloat16* d = A.d[x];
+  __nv_bfloat16* cat = A.cat[x];
+  float part[4] = {0.f, 0.f, 0.f, 0.f};
+  auto sq8 = [](const uint4& v, float acc) {
+    const __nv_bfloat162* h2 = reinterpret_cast<const __nv_bfloat162*>(&v);
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const float2 f = __bfloat1622float2(h2[e]);
+      acc = fmaf(f.x, f.x, acc);
+      acc = fmaf(f.y, f.y, acc);
+    }
+    return acc;
+  };
+  const int nq = H / 8, q = hb * (AP_HB / 8) + lane;  // this lane's 16-byte unit
+#pragma unroll
+  for (int r = 0; r < 4; ++r) {
+    const int i = i0 + 4 * warp + r;
+    if (i >= I) continue;
+    const uint4 a = reinterpret_cast<const uint4*>(g + (size_t)i * H)[q];
+    const uint4 b = reinterpret_cast<const uint4*>(u + (size_t)i * H)[q];
+    uint4* dst = reinterpret_cast<uint4*>(cat + (size_t)i * K);
+    dst[q] = a;
+    dst[nq + q] = b;
+    part[r] = sq8(b, sq8(a, part[r]));
+  }
+  for (int h0 = hb * AP_HB; h0 < (hb + 1) * AP_HB; h0 += 64) {
+    __syncthreads();
+    // the 64 x 32 block d[h0 .. h0 + 63][i0 .. i0 + 31] in 4-byte pieces
+    for (int e = threadIdx.x; e < 64 * 16; e += 256) {
+      const int hh = e >> 4, ii = 2 * (e & 15);
+      uint32_t v = 0u;
+      if (i0 + ii < I) v = *reinterpret_cast<const uint32_t*>(d + (size_t)(h0 + hh) * I + i0 + ii);
+      *reinterpret_cast<uint32_t*>(&blk[hh][ii]) = v;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int r = 0; r < 4; ++r) {
+      const int il = 4 * warp + r, i = i0 + il;
+      if (i >= I) continue;
+      // lane l: elements h0 + 2 l, h0 + 2 l + 1 of row i's down segment
+      __nv_bfloat162 pr;
+      pr.x = blk[2 * lane][il];
+      pr.y = blk[2 * lane + 1][il];
+      *reinterpret_cast<__nv_bfloat162*>(cat + (size_t)i * K + 2L * H + h0 + 2 * lane) = pr;
+      const float fa = __bfloat162float(pr.x), fb = __bfloat162float(pr.y);
+      part[r] = fmaf(fb, fb, fmaf(fa, fa, part[r]));
+    }
+  }
+#pragma unroll
+  for (int r = 0; r < 4; ++r) {
+    float v = part[r];
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    const int i = i0 + 4 * warp + r;
+    if (lane == 0 && i < I) A.npart[x][(size_t)hb * I + i] = v;
+  }
+}
+
+// cost[i][j] = na[i] + nb[j] - 2 sum_s part[z][s][i][j - z Npad], z = j / Npad
+// (the K ranges in ascending order), na / nb the sums of the nhb norm
+// partials [nhb][I] in range order
+__global__ void k_align_finish(const float* __restrict__ part, int splits, int I, int Npad,
+                               const float* __restrict__ npa, const float* __restrict__ npb,
+                               int nhb, float* __restrict__ cost) {
+  // four consecutive columns per thread (I and Npad are multiples of 4)
+  const long total = (long)I * I / 4;
+  for (long e = (long)blockIdx.x * blockDim.x + threadIdx.x; e < total;
+       e += (long)gridDim.x * blockDim.x) {
+    const int i = (int)(4 * e / I), j = (int)(4 * e % I), z = j / Npad, jj = j % Npad;
+    const float4* p = reinterpret_cast<const float4*>(part + ((size_t)z * splits * I + i) * Npad + jj);
+    const size_t st = (size_t)I * Npad / 4;
+    float4 dot = make_float4(0.f, 0.f, 0.f, 0.f);
+    int sp = 0;
+    for (; sp + 4 <= splits; sp += 4) {  // four ranges' loads in flight, added in order
+      float4 v[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) v[u] = p[(sp + u) * st];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        dot.x += v[u].x; dot.y += v[u].y; dot.z += v[u].z; dot.w += v[u].w;
+      }
+    }
+    for (; sp < splits; ++sp) {
+      const float4 v = p[sp * st];
+      dot.x += v.x; dot.y += v.y; dot.z += v.z; dot.w += v.w;
+    }
+    float a = 0.f;
+    float4 b = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int r = 0; r < nhb; ++r) {
+      a += npa[(size_t)r * I + i];
+      const float4 v = *reinterpret_cast<const float4*>(npb + (size_t)r * I + j);
+      b.x += v.x; b.y += v.y; b.z += v.z; b.w += v.w;
+    }
+    *reinterpret_cast<float4*>(cost + (size_t)i * I + j) =
+        make_float4(a + b.x - 2.f * dot.x, a + b.y - 2.f * dot.y, a + b.z - 2.f * dot.z,
+                    a + b.w - 2.f * dot.w);
+  }
+}
+
 // dst row i = src row perm[i] of a [rows][cols] matrix (16-byte pieces; a row
 // whose perm entry is outside [0, rows) is written as zeros)
 __global__ void k_permute_rows(const uint4* __restrict__ src, uint4* __restrict__ dst,
@@ -332,6 +462,72 @@ lx_status check_expert_args(int32_t dtype, int32_t H, int32_t I) {
 }  // namespace
 }  // namespace lx
 
+namespace lx {
+namespace {
+
+// The tensor-core form of the cost (bf16, H % 256 == 0): scratch from the
+// stream-ordered allocator (packed operands, norms, split-K partials), freed on
+// the stream after the last kernel.
+lx_status align_cost_tc(int H, int I, const void* dg, const void* du, const void* dd,
+                        const void* mg, const void* mu, const void* md, float* cost,
+                        cudaStream_t s) {
+  using B = __nv_bfloat16;
+  int dev = 0, sms = 0;
+  LX_CUDA(cudaGetDevice(&dev));
+  LX_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+  const long K = 3L * H;
+  const int nz = (I + 255) / 256;
+  const int Npad = ((I + nz - 1) / nz + 15) / 16 * 16;  // chunk width (<= 256)
+  auto al = [](size_t v) { return (v + 255) / 256 * 256; };
+  const int nhb = H / AP_HB;
+  const size_t b_cat = al((size_t)I * K * 2), b_nrm = al((size_t)nhb * I * 4);
+  const size_t b_part = al((size_t)nz * RES_TC_MAX_SPLITS * I * Npad * 4);
+  char* ws = nullptr;
+  LX_CUDA(cudaMallocAsync((void**)&ws, 2 * b_cat + 2 * b_nrm + b_part, s));
+  B* A = reinterpret_cast<B*>(ws);
+  B* Bm = reinterpret_cast<B*>(ws + b_cat);
+  float* na = reinterpret_cast<float*>(ws + 2 * b_cat);
+  float* nb = reinterpret_cast<float*>(ws + 2 * b_cat + b_nrm);
+  float* part = reinterpret_cast<float*>(ws + 2 * b_cat + 2 * b_nrm);
+  lx_status st = LX_OK;
+  AlignPackArgs pa;
+  pa.g[0] = static_cast<const B*>(dg);
+  pa.u[0] = static_cast<const B*>(du);
+  pa.d[0] = static_cast<const B*>(dd);
+  pa.g[1] = static_cast<const B*>(mg);
+  pa.u[1] = static_cast<const B*>(mu);
+  pa.d[1] = static_cast<const B*>(md);
+  pa.cat[0] = A;
+  pa.cat[1] = Bm;
+  pa.npart[0] = na;
+  pa.npart[1] = nb;
+  k_align_pack<<<dim3((I + 31) / 32, nhb, 2), 256, 0, s>>>(pa, H, I);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) st = cuda_fail(e, "pack alignment operands");
+  CUtensorMap ma, mb;
+  std::memset(&ma, 0, sizeof(ma));
+  std::memset(&mb, 0, sizeof(mb));
+  if (st == LX_OK && (!encode_bf16_2d(&ma, A, K, I, 64, 128) || !encode_bf16_2d(&mb, Bm, K, I, 64, Npad)))
+    st = fail(LX_ERR_CUDA, "cuTensorMapEncodeTiled(alignment operands) failed");
+  int splits = 1;
+  if (st == LX_OK)
+    st = tc_splitk_gemm_chunks(ma, mb, I, Npad, nz, (int)K, part, RES_TC_MAX_SPLITS, &splits, sms,
+                               dev, s);
+  if (st == LX_OK) {
+    const long total = (long)I * I;
+    k_align_finish<<<(unsigned)std::min<long>((total / 4 + 255) / 256, 8L * sms), 256, 0, s>>>(
+        part, splits, I, Npad, na, nb, nhb, cost);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) st = cuda_fail(e, "alignment cost");
+  }
+  e = cudaFreeAsync(ws, s);
+  if (st == LX_OK && e != cudaSuccess) st = cuda_fail(e, "free alignment scratch");
+  return st;
+}
+
+}  // namespace
+}  // namespace lx
+
 extern "C" lx_status lx_align_cost(int32_t dtype, int32_t d_model, int32_t d_ff,
                                    const void* dom_gate, const void* dom_up, const void* dom_down,
                                    const void* mem_gate, const void* mem_up, const void* mem_down,
@@ -346,6 +542,8 @@ extern "C" lx_status lx_align_cost(int32_t dtype, int32_t d_model, int32_t d_ff,
   const int H = d_model, I = d_ff;
   const dim3 grid((I + AC_TILE - 1) / AC_TILE, (I + AC_TILE - 1) / AC_TILE);
   cudaStream_t s = (cudaStream_t)stream;
+  if (dtype == LX_BF16 && H % 256 == 0) return align_cost_tc(H, I, dom_gate, dom_up, dom_down,
+                                                            mem_gate, mem_up, mem_down, cost, s);
   if (dtype == LX_BF16) {
     using B = __nv_bfloat16;
     k_align_cost_mma<<<grid, AM_THREADS, 0, s>>>((const B*)dom_gate, (const B*)dom_up,

@@ -39,7 +39,7 @@ struct ResLaunch {
   CUtensorMap a_dom;  // [M][K] bf16 (W_dom or W_dom^T)
   CUtensorMap b;      // [Npad][6 Kp] bf16, 64 x Npad boxes
   int M, Npad, kb_seg, kb_split, n_kb;  // 64-wide K blocks: per segment, per CTA, in all
-  float* part;        // [splits][M][Npad]
+  float* part;        // [gridDim.z][splits][M][Npad]: blockIdx.z takes B rows z Npad ..
   unsigned long long wait_cycles;
 };
 
@@ -94,7 +94,7 @@ __global__ void __launch_bounds__(RM_THREADS, 1) k_res_mma(const __grid_constant
         mbar_expect_tx(full0 + 8 * s, RM_A_BYTES + b_bytes);
         const uint32_t a_s = smem_base + s * stage_bytes, b_s = a_s + RM_A_BYTES;
         tma_load_2d(a_s, seg < 3 ? &P.a_mem : &P.a_dom, kk * RM_BK, m0, full0 + 8 * s);
-        tma_load_2d(b_s, &P.b, kb * RM_BK, 0, full0 + 8 * s);
+        tma_load_2d(b_s, &P.b, kb * RM_BK, (int)blockIdx.z * P.Npad, full0 + 8 * s);
         issued = i + 1;
       }
     }
@@ -130,20 +130,34 @@ __global__ void __launch_bounds__(RM_THREADS, 1) k_res_mma(const __grid_constant
     ok = __shfl_sync(0xffffffffu, ok, 0);  // warp-uniform: the TMEM loads are warp-wide
     __syncwarp();
     tc_fence_after();
-    const int row = 32 * q + lane;
-    float* out = P.part + ((size_t)blockIdx.y * P.M + m0 + row) * P.Npad;
+    // 32-column blocks of the warp's 32 rows staged in shared memory (the
+    // stages are free: every MMA has completed), then stored as whole 128-byte
+    // row segments (eight lanes per row, four rows per store)
+    float* out = P.part + (((size_t)blockIdx.z * gridDim.y + blockIdx.y) * P.M + m0 + 32 * q) * P.Npad;
+    float* stg = reinterpret_cast<float*>(smem) + q * 32 * 33;
     if (ok) {
-      for (int c0 = 0; c0 < P.Npad; c0 += 16) {
-        uint32_t v[16];
-        tc_ld16_async(tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)c0, v);
+      for (int c0 = 0; c0 < P.Npad; c0 += 32) {
+        const int w = min(32, P.Npad - c0);  // 16 or 32 (Npad is a multiple of 16)
+        const uint32_t ta = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)c0;
+        uint32_t v[32];
+        tc_ld16_async(ta, *reinterpret_cast<uint32_t(*)[16]>(v));
+        if (w == 32) tc_ld16_async(ta + 16, *reinterpret_cast<uint32_t(*)[16]>(v + 16));
         tc_wait_ld();
-        if (m0 + row < P.M) {
-          float4* o = reinterpret_cast<float4*>(out + c0);
 #pragma unroll
-          for (int j = 0; j < 4; ++j)
-            o[j] = make_float4(__uint_as_float(v[4 * j]), __uint_as_float(v[4 * j + 1]),
-                               __uint_as_float(v[4 * j + 2]), __uint_as_float(v[4 * j + 3]));
+        for (int c = 0; c < 32; ++c)
+          if (c < w) stg[lane * 33 + c] = __uint_as_float(v[c]);
+        __syncwarp();
+        const int cq = lane & 7;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const int rr = 4 * j + (lane >> 3);
+          if (m0 + 32 * q + rr < P.M && 4 * cq < w) {
+            const float* sr = stg + rr * 33 + 4 * cq;
+            *reinterpret_cast<float4*>(out + (size_t)rr * P.Npad + c0 + 4 * cq) =
+                make_float4(sr[0], sr[1], sr[2], sr[3]);
+          }
         }
+        __syncwarp();
       }
     }
   }
@@ -308,6 +322,37 @@ lx_status tc_splitk_gemm(lx_layer* L, const CUtensorMap& a, const CUtensorMap& b
   LX_CUDA(smem_cap_once((const void*)k_res_mma, 227 * 1024, L->device, g_rm_cap));
   ProfScope ps(L, s, name);
   launch_k(L, k_res_mma, dim3((unsigned)mt, (unsigned)splits), RM_THREADS, smem, s, P);
+  LX_CUDA(cudaGetLastError());
+  *splits_out = splits;
+  return LX_OK;
+}
+
+// The same kernel over column chunks: part[z][s][M][Npad] = A[M][K-range s] .
+// B[rows z Npad ..][K-range s]^T for z < nz (one launch, grid (M tiles, ranges,
+// nz)); a plain launch (no layer), for the stateless entry points.
+lx_status tc_splitk_gemm_chunks(const CUtensorMap& a, const CUtensorMap& b, int M, int Npad,
+                                int nz, int K, float* part, int max_splits, int* splits_out,
+                                int num_sms, int dev, cudaStream_t s) {
+  ResLaunch P;
+  std::memset(&P, 0, sizeof(P));
+  P.a_mem = a;
+  P.a_dom = a;
+  P.b = b;
+  const int mt = (M + RM_BM - 1) / RM_BM;
+  P.M = M;
+  P.Npad = Npad;
+  P.kb_seg = K / 64;
+  P.n_kb = P.kb_seg;
+  int splits = std::max(1, std::min(max_splits, num_sms / std::max(1, mt * nz)));
+  splits = std::min(splits, std::max(1, P.n_kb / 4));
+  P.kb_split = (P.n_kb + splits - 1) / splits;
+  splits = (P.n_kb + P.kb_split - 1) / P.kb_split;
+  P.part = part;
+  P.wait_cycles = kDefaultWaitCycles;
+  const int b_bytes = Npad * 64 * 2;
+  const int smem = RM_STAGES * (RM_A_BYTES + ((b_bytes + 1023) & ~1023)) + 8 * (2 * RM_STAGES + 3) + 1024;
+  LX_CUDA(smem_cap_once((const void*)k_res_mma, 227 * 1024, dev, g_rm_cap));
+  k_res_mma<<<dim3((unsigned)mt, (unsigned)splits, (unsigned)nz), RM_THREADS, smem, s>>>(P);
   LX_CUDA(cudaGetLastError());
   *splits_out = splits;
   return LX_OK;

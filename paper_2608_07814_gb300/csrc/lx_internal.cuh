@@ -508,6 +508,9 @@ lx_status res_gemm_tc(bool transposed, const __nv_bfloat16* Wm, const __nv_bfloa
                       int num_sms, int dev, cudaStream_t s);
 // split-K tensor-core product part[s][M][Npad] = A . B^T over K range s (see
 // lx_compress_tc.cu); the number of ranges used is returned in splits_out
+lx_status tc_splitk_gemm_chunks(const CUtensorMap& a, const CUtensorMap& b, int M, int Npad,
+                                int nz, int K, float* part, int max_splits, int* splits_out,
+                                int num_sms, int dev, cudaStream_t s);
 lx_status tc_splitk_gemm(lx_layer* L, const CUtensorMap& a, const CUtensorMap& b, int M, int Npad,
                          int K, float* part, int max_splits, int* splits_out, cudaStream_t s,
                          const char* name);

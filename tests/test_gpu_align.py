@@ -47,9 +47,13 @@ def _f64(t, dtype):
     return tuple(synth.from_storage(w, dtype) for w in t)
 
 
+# bf16 with d_model a multiple of 256 takes the tensor-core form (ragged
+# 128-row tiles and column chunks below); the other bf16 shapes the 64 x 64
+# tile form
 CASES = [(2048, 768, "bf16", False), (2048, 768, "bf16", True), (40, 72, "f32", False),
          (40, 72, "bf16", True), (136, 200, "f32", True), (8, 8, "f32", False),
-         (264, 64, "bf16", False)]
+         (264, 64, "bf16", False), (128, 200, "bf16", False), (256, 200, "bf16", False),
+         (256, 136, "bf16", True), (256, 24, "bf16", True), (512, 328, "bf16", False)]
 
 
 @pytest.mark.parametrize("H,I,dtype,planted", CASES)
