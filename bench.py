@@ -705,6 +705,10 @@ def run_offline(args, rank, world, local_rank):
             for p in range(3):
                 lx.compress_factor(dd[p], md[p], od[p], r, q, workspace=ws)
         ms_seq = _event_ms(step, max(3, args.steps // 4), args.warmup)
+        # one member alone: its three projections concurrently on three streams
+        wss1 = [torch.empty(wsz, dtype=torch.uint8, device=dev) for _ in range(3)]
+        ms_one = _event_ms(lambda: lx.compress_member(dd, md, od, r, q, workspaces=wss1),
+                           max(3, args.steps // 4), args.warmup)
         # a layer's members are independent: n_conc members (3 projections
         # each) in flight on their own streams, each with its own workspace
         n_conc = 8
@@ -729,9 +733,15 @@ def run_offline(args, rank, world, local_rank):
                 e.record(st)
                 main.wait_event(e)
         ms = _event_ms(step_conc, args.steps, args.warmup, world) / n_conc
+        # launches of one projection: the R products (split, transposes, MMA,
+        # ordered sum), 2q single and 2 double CholeskyQR passes (Gram, Cholesky,
+        # basis product each), then trmm, Jacobi, Ritz, finish, two factor
+        # products and the sign rule
+        launches_per_projection = ((1 + q) * 3 + (1 + q) * 5 + 3 * (2 * q + 4) + 7)
         big = sum((2 + 2 * q) * 2.0 * a * b * l for a, b in shapes)        # the R-sized products
-        small = sum(2 * (1 + 2 * q) * 2 * (2.0 * a * l * l + a * l * l) + 2.0 * b * l * l
-                    + 2.0 * (a + b) * l * r for a, b in shapes)           # Grams, orthonormalisation
+        # CholeskyQR passes: q + 2 on each side (rows and cols), each a lower
+        # Gram (n l^2) and a basis product (2 n l^2); then the two factor products
+        small = sum(3.0 * l * l * (q + 2) * (a + b) + 2.0 * (a + b) * l * r for a, b in shapes)
         alu = fp32_alu_peak_tflops(peaks)
         ach = (big + small) / (ms * 1e-3) / 1e12
         t0 = time.time()
@@ -741,10 +751,11 @@ def run_offline(args, rank, world, local_rank):
             ocomp.randomized_factors(R, r, oms[p].astype(np.float64), q)
         cpu_s = time.time() - t0
         line["sequential_ms_per_member"] = round(ms_seq, 3)
+        line["one_member_ms"] = round(ms_one, 3)
         line.update({"metric": "members compressed/s (gate, up and down residuals, rank 128)",
                      "value": round(1e3 / ms * world, 3), "unit": "members/s",
                      "ms_per_step": round(ms, 4), "higher_is_better": True, "dtype": "f32",
-                     "gpu_launches": args.steps * n_conc * 3 * (7 + 6 * (1 + 2 * q) + 2 * q),
+                     "gpu_launches": args.steps * n_conc * 3 * launches_per_projection,
                      "roofline": {"kernel": "whole compression step", "bound": "alu",
                                   "achieved": round(ach, 2), "peak": round(alu, 1),
                                   "unit": "TFLOP/s", "frac": round(ach / alu, 4), "traffic": None,

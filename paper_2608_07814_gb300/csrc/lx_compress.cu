@@ -8,22 +8,24 @@
 //   k_cgemm     fp32 GEMM (CUDA-core FMA, 64 x 64 tiles, 32-deep K chunks in
 //               shared memory); its A operand is R (rows of W_mem - W_dom,
 //               formed on load), R^T (columns of the same), or an fp32 matrix.
-//   k_gram      G = X^T X in float64 (fp32 inputs, float64 products and sums).
-//   k_chol32    one CTA: Cholesky G + s I = L L^T (fp32 in shared memory; a
-//               small relative shift in the first of the two passes keeps
-//               rank-deficient bases factorable) and T = L^-T, so that X T has
-//               orthonormal columns (CholeskyQR, run twice per
-//               orthonormalisation).
+//   k_gram      G = X^T X to float64 accuracy (exact fp32 products, error-free
+//               two-sum accumulation on the fp32 pipes), stored in float64.
+//   k_chol32    one CTA: Cholesky G + s I = L L^T (fp32 in shared memory, one
+//               barrier per step; a small relative shift in the first of the
+//               two passes keeps rank-deficient bases factorable) and
+//               T = L^-T by forward elimination, so that X T has orthonormal
+//               columns (CholeskyQR, run twice per orthonormalisation).
 //   k_trmm      M = L1 L2, the triangular factor of R^T Q = Z2 M^T.
 //   k_onesided  one CTA: one-sided Jacobi SVD of M (fp32 rotations, shared
-//               memory), M W = U S.
+//               memory, every pair of a round at once), M W = U S.
 //   k_ritz      sigma_j = |M w_j| / |w_j| in float64 (Rayleigh quotients).
 //   k_finish    the r largest sigma and the fp32 matrices that turn the bases
 //               into the split factors.
 //   k_sign      each factor column's largest-magnitude entry of U made
 //               positive (U and V negated together).
-// Only the Gram sums and the Rayleigh quotients use float64: a single SM's
-// float64 rate is a small fraction of its fp32 rate on this GPU.
+// Only the Rayleigh quotients use float64 arithmetic, and the Gram sums reach
+// float64 accuracy by compensated fp32 arithmetic: this GPU's float64 rate is
+// a small fraction of its fp32 rate.
 #include <algorithm>
 #include <cmath>
 #include <type_traits>
@@ -136,102 +138,223 @@ k_cgemm(const TW* __restrict__ Wm, const TW* __restrict__ Wd, const float* __res
   }
 }
 
-// G [L][L] = X^T X for X [n][L] fp32 row-major; float64 products and sums in
-// ascending row order.  16 x 16 outputs per CTA; only the tiles on or below
-// the diagonal are computed (the Cholesky reads the lower triangle alone).
+// G [L][L] = X^T X for X [n][L] fp32 row-major, to float64 accuracy on the
+// fp32 pipes (this GPU's float64 rate is a small fraction of its fp32 rate).
+// Each product is formed exactly as the pair p + e (p = x y rounded,
+// e = fma(x, y, -p)); the sum is carried as an unevaluated pair hi + lo, hi
+// taking the products through Knuth's error-free two-sum and lo collecting the
+// two-sum and product errors (the compensated dot product "Dot2" of Ogita,
+// Rump and Oishi, 2005), so G = hi + lo is as accurate as a dot product in
+// twice the fp32 precision: within 2^-24 |G| + (n 2^-24)^2 sum |x y| of the
+// exact sum, far below the fp32 rounding the Cholesky applies to it.  Four
+// such pairs per thread take the rows of a chunk in turn (independent chains)
+// and are added pairwise at the end; each 64-row chunk is staged in shared
+// memory while the next one is already loading into registers.  16 x 16
+// outputs per CTA; only the tiles on or below the diagonal are computed (the
+// Cholesky reads the lower triangle alone).
 constexpr int GR_T = 16;
-constexpr int GR_KC = 32;
+constexpr int GR_KC = 64;
+constexpr int GR_CH = 4;
+static_assert(GR_KC * GR_T % (GR_T * GR_T) == 0, "whole staged values per thread");
+
+struct DF {
+  float hi, lo;
+};
+// hi + lo += p + e, by the two-sum of hi and p (every step rounded on its own:
+// the intrinsics are never contracted into fused operations)
+__device__ __forceinline__ void df_add(DF& d, float p, float e) {
+  const float s = __fadd_rn(d.hi, p);
+  const float v = __fsub_rn(s, d.hi);
+  const float err = __fadd_rn(__fsub_rn(d.hi, __fsub_rn(s, v)), __fsub_rn(p, v));
+  d.hi = s;
+  d.lo = __fadd_rn(d.lo, __fadd_rn(err, e));
+}
+
 __global__ void __launch_bounds__(GR_T * GR_T)
 k_gram(const float* __restrict__ X, int n, int L, double* __restrict__ G) {
-  __shared__ double Xi[GR_KC][GR_T], Xj[GR_KC][GR_T];
+  constexpr int PER = GR_KC * GR_T / (GR_T * GR_T);  // staged values per thread and side
+  __shared__ float Xi[GR_KC][GR_T], Xj[GR_KC][GR_T];
   if (blockIdx.x > blockIdx.y) return;  // strictly above the diagonal
   const int ti = threadIdx.x / GR_T, tj = threadIdx.x % GR_T;
   const int i0 = blockIdx.y * GR_T, j0 = blockIdx.x * GR_T;
-  double acc = 0.0;
-  for (int m0 = 0; m0 < n; m0 += GR_KC) {
-    for (int q = threadIdx.x; q < GR_KC * GR_T; q += GR_T * GR_T) {
+  DF acc[GR_CH];
+#pragma unroll
+  for (int c = 0; c < GR_CH; ++c) acc[c] = DF{0.f, 0.f};
+  // the next chunk's rows are loaded into registers while this one is summed
+  float ri[PER], rj[PER];
+  auto fetch = [&](int m0) {
+#pragma unroll
+    for (int e = 0; e < PER; ++e) {
+      const int q = threadIdx.x + e * GR_T * GR_T;
       const int mr = q / GR_T, c = q % GR_T;
       const bool okm = m0 + mr < n;
-      Xi[mr][c] = (okm && i0 + c < L) ? (double)X[(size_t)(m0 + mr) * L + i0 + c] : 0.0;
-      Xj[mr][c] = (okm && j0 + c < L) ? (double)X[(size_t)(m0 + mr) * L + j0 + c] : 0.0;
+      ri[e] = (okm && i0 + c < L) ? X[(size_t)(m0 + mr) * L + i0 + c] : 0.f;
+      rj[e] = (okm && j0 + c < L) ? X[(size_t)(m0 + mr) * L + j0 + c] : 0.f;
+    }
+  };
+  fetch(0);
+  for (int m0 = 0; m0 < n; m0 += GR_KC) {
+#pragma unroll
+    for (int e = 0; e < PER; ++e) {
+      const int q = threadIdx.x + e * GR_T * GR_T;
+      Xi[q / GR_T][q % GR_T] = ri[e];
+      Xj[q / GR_T][q % GR_T] = rj[e];
     }
     __syncthreads();
-#pragma unroll 8
-    for (int mr = 0; mr < GR_KC; ++mr) acc = fma(Xi[mr][ti], Xj[mr][tj], acc);
+    if (m0 + GR_KC < n) fetch(m0 + GR_KC);
+#pragma unroll
+    for (int mr = 0; mr < GR_KC; mr += GR_CH) {
+#pragma unroll
+      for (int c = 0; c < GR_CH; ++c) {
+        const float x = Xi[mr + c][ti], y = Xj[mr + c][tj];
+        const float p = __fmul_rn(x, y);
+        df_add(acc[c], p, __fmaf_rn(x, y, -p));
+      }
+    }
     __syncthreads();
   }
-  if (i0 + ti < L && j0 + tj < L) G[(size_t)(i0 + ti) * L + j0 + tj] = acc;
+  // (chain 0 + chain 1) + (chain 2 + chain 3), each pair added as hi + lo
+  DF s01 = acc[0], s23 = acc[2];
+  df_add(s01, acc[1].hi, acc[1].lo);
+  df_add(s23, acc[3].hi, acc[3].lo);
+  df_add(s01, s23.hi, s23.lo);
+  if (i0 + ti < L && j0 + tj < L)
+    G[(size_t)(i0 + ti) * L + j0 + tj] = (double)s01.hi + (double)s01.lo;
 }
 
 // One CTA (L <= 256).  Cholesky of G + s I in fp32 (G float64, rounded once;
 // s = shift_rel * max diag(G)) in a packed lower triangle in shared memory
-// (L (L + 1) / 2 floats), pivots floored at 1e-30; then X = L^-1 by forward
-// substitution (thread c owns column c; X packed like L, in shared memory
-// when x_in_smem, else in the global scratch Xg, so that a warp reads one
-// contiguous piece of a row per step) and T = X^T, so that Y T = Y L^-T has
+// (L (L + 1) / 2 floats, row i from i (i + 1) / 2), pivots floored at 1e-30.
+// Right-looking with the column scaling deferred: step j subtracts
+// (a_ij / l_jj) (a_cj / l_jj) from every trailing entry (j < c <= i) and
+// leaves column j itself unscaled, so that one barrier separates the steps
+// (warps take rows, lanes columns, each lane holding its entries of column j
+// in registers for all of its warp's rows); the columns are scaled once at the
+// end.
+// Then X = L^-1 by forward elimination of L X = I, again one barrier per step:
+// with Y the rows of X before their division by the diagonal, step p
+// subtracts (l_ip / l_pp) y_p from every row i > p (y_p is final by then),
+// and X = Y / diag(L) at the end.  X is packed like L, in shared memory when
+// x_in_smem, else in the global scratch Xg.  T = X^T, so that Y T = Y L^-T has
 // orthonormal columns when Y^T Y = G (CholeskyQR).  The factor itself is
 // written to Lout [L][L] (zero above the diagonal).  A zero Gram gives
 // Lout = T = 0.
 constexpr int CH_THREADS = 1024;
+constexpr int CH_REGS = 8;  // 32 CH_REGS >= 256 >= L
+__device__ __forceinline__ int tri_off(int i) { return i * (i + 1) / 2; }
+
 __global__ void __launch_bounds__(CH_THREADS)
 k_chol32(const double* __restrict__ G, int L, float shift_rel, float* __restrict__ Lout,
          float* __restrict__ Xg, int x_in_smem, float* __restrict__ T) {
   extern __shared__ float Ls[];
-  float* Xp = x_in_smem ? Ls + L * (L + 1) / 2 : Xg;  // packed lower X
+  float* Xp = x_in_smem ? Ls + tri_off(L) : Xg;  // packed lower X
   __shared__ double s_md;
-  __shared__ float s_diag[256];  // the factor's diagonal (Ls keeps the raw pivots)
+  __shared__ float s_diag[256];  // the factor's diagonal
+  __shared__ float s_rdiag[256];  // its reciprocals
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nw = CH_THREADS / 32;
-  if (tid == 0) {
+  if (warp == 0) {
     double md = 0.0;
-    for (int i = 0; i < L; ++i) md = fmax(md, G[(size_t)i * L + i]);
-    s_md = md;
+    for (int i = lane; i < L; i += 32) md = fmax(md, G[(size_t)i * L + i]);
+#pragma unroll
+    for (int o = 16; o; o >>= 1) md = fmax(md, __shfl_xor_sync(0xffffffffu, md, o));
+    if (lane == 0) s_md = md;
   }
   __syncthreads();
   const double md = s_md;
   if (!(md > 0.0)) {
-    for (int q = tid; q < L * L; q += CH_THREADS) {
-      Lout[q] = 0.f;
-      T[q] = 0.f;
-    }
+    for (int i = warp; i < L; i += nw)
+      for (int c = lane; c < L; c += 32) {
+        Lout[(size_t)i * L + c] = 0.f;
+        T[(size_t)i * L + c] = 0.f;
+      }
     return;
   }
   const float shift = (float)(shift_rel * md);
   for (int i = warp; i < L; i += nw)
     for (int j = lane; j <= i; j += 32)
-      Ls[i * (i + 1) / 2 + j] = (float)G[(size_t)i * L + j] + (i == j ? shift : 0.f);
+      Ls[tri_off(i) + j] = (float)G[(size_t)i * L + j] + (i == j ? shift : 0.f);
+  // l_jj = sqrt(max(pivot, 1e-30)) and its reciprocal are formed once, by the
+  // thread that finalises the pivot: here for j = 0, else in step j - 1
+  if (tid == 0) {
+    const float l00 = sqrtf(fmaxf((float)G[0] + shift, 1e-30f));
+    s_diag[0] = l00;
+    s_rdiag[0] = 1.f / l00;
+  }
   __syncthreads();
   for (int j = 0; j < L; ++j) {
-    // every thread takes the pivot from the raw entry, which nothing writes
-    // after the previous step's barrier; the factor's diagonal goes to s_diag
-    const float ljj = sqrtf(fmaxf(Ls[j * (j + 1) / 2 + j], 1e-30f));
-    if (tid == 0) s_diag[j] = ljj;
-    for (int i = j + 1 + tid; i < L; i += CH_THREADS) Ls[i * (i + 1) / 2 + j] /= ljj;
-    __syncthreads();
+    const float rl = s_rdiag[j];
+    // this lane's entries of the scaled column j (rows c = j + 1 + lane + 32 k),
+    // the same for every row the warp updates
+    float lc[CH_REGS];
+#pragma unroll
+    for (int k = 0; k < CH_REGS; ++k) {
+      if (j + 1 + 32 * k >= L) break;  // warp-uniform
+      const int c = j + 1 + lane + 32 * k;
+      lc[k] = c < L ? Ls[tri_off(c) + j] * rl : 0.f;
+    }
     for (int i = j + 1 + warp; i < L; i += nw) {
-      const float lij = Ls[i * (i + 1) / 2 + j];
-      for (int c = j + 1 + lane; c <= i; c += 32) Ls[i * (i + 1) / 2 + c] -= lij * Ls[c * (c + 1) / 2 + j];
+      float* Ai = Ls + tri_off(i);
+      const float lij = Ai[j] * rl;
+#pragma unroll
+      for (int k = 0; k < CH_REGS; ++k) {
+        const int c = j + 1 + lane + 32 * k;
+        if (j + 1 + 32 * k > i) break;  // warp-uniform
+        if (c <= i) {
+          const float v = fmaf(-lij, lc[k], Ai[c]);
+          Ai[c] = v;
+          if (c == i && i == j + 1) {  // the next pivot is final
+            const float d = sqrtf(fmaxf(v, 1e-30f));
+            s_diag[i] = d;
+            s_rdiag[i] = 1.f / d;
+          }
+        }
+      }
     }
     __syncthreads();
   }
-  for (int j = tid; j < L; j += CH_THREADS) Ls[j * (j + 1) / 2 + j] = s_diag[j];
-  __syncthreads();
-  for (int q = tid; q < L * L; q += CH_THREADS) {
-    const int i = q / L, c = q % L;
-    Lout[q] = c <= i ? Ls[i * (i + 1) / 2 + c] : 0.f;
-  }
-  if (tid < L) {
-    const int c = tid;
-    for (int i = c; i < L; ++i) {
-      const float* Li = Ls + i * (i + 1) / 2;
-      float acc = 0.f;
-      for (int k = c; k < i; ++k) acc = fmaf(Li[k], Xp[k * (k + 1) / 2 + c], acc);
-      Xp[i * (i + 1) / 2 + c] = i == c ? 1.f / Li[i] : -acc / Li[i];
+  // scale the columns; Y = I
+  for (int i = warp; i < L; i += nw) {
+    float* Ai = Ls + tri_off(i);
+    float* Yi = Xp + tri_off(i);
+    for (int j = lane; j <= i; j += 32) {
+      Ai[j] = j == i ? s_diag[i] : Ai[j] * s_rdiag[j];
+      Yi[j] = j == i ? 1.f : 0.f;
     }
   }
   __syncthreads();
-  for (int q = tid; q < L * L; q += CH_THREADS) {
-    const int k = q / L, n = q % L;  // T[k][n] = X[n][k], zero below the diagonal
-    T[q] = k <= n ? Xp[n * (n + 1) / 2 + k] : 0.f;
+  for (int p = 0; p + 1 < L; ++p) {
+    const float rp = s_rdiag[p];
+    const float* yp = Xp + tri_off(p);
+    float yv[CH_REGS];  // this lane's entries of y_p (columns lane + 32 k)
+#pragma unroll
+    for (int k = 0; k < CH_REGS; ++k) {
+      if (32 * k > p) break;  // warp-uniform
+      const int c = lane + 32 * k;
+      yv[k] = c <= p ? yp[c] : 0.f;
+    }
+    for (int i = p + 1 + warp; i < L; i += nw) {
+      const float f = Ls[tri_off(i) + p] * rp;
+      float* yi = Xp + tri_off(i);
+#pragma unroll
+      for (int k = 0; k < CH_REGS; ++k) {
+        const int c = lane + 32 * k;
+        if (32 * k > p) break;  // warp-uniform
+        if (c <= p) yi[c] = fmaf(-f, yv[k], yi[c]);
+      }
+    }
+    __syncthreads();
+  }
+  for (int i = warp; i < L; i += nw) {
+    float* Yi = Xp + tri_off(i);
+    for (int c = lane; c <= i; c += 32) Yi[c] = Yi[c] * s_rdiag[i];
+  }
+  __syncthreads();
+  for (int i = warp; i < L; i += nw) {
+    const float* Ai = Ls + tri_off(i);
+    for (int c = lane; c < L; c += 32) {
+      Lout[(size_t)i * L + c] = c <= i ? Ai[c] : 0.f;
+      T[(size_t)i * L + c] = c >= i ? Xp[tri_off(c) + i] : 0.f;  // T[k][n] = X[n][k]
+    }
   }
 }
 
@@ -249,84 +372,207 @@ __global__ void k_trmm(const float* __restrict__ L1, const float* __restrict__ L
 // One-sided Jacobi SVD of M (Hestenes), one CTA: the columns of M are
 // orthogonalised by plane rotations applied from the right, M W = U S, W
 // orthogonal.  Lp = L rounded up to even (a zero padding column never rotates);
-// each round pairs the columns by the circle method, a warp takes a pair:
-// alpha = |m_p|^2, beta = |m_q|^2, gamma = m_p . m_q (fp32), and unless
-// |gamma| <= 1e-6 sqrt(alpha beta) (a little above the rounding of an fp32 dot
-// product, so that sweeps terminate) rotates columns p, q of M and of W by the
-// angle that makes them orthogonal (zeta = (beta - alpha) / (2 gamma),
-// t = sign(zeta) / (|zeta| + sqrt(1 + zeta^2)), c = 1 / sqrt(1 + t^2), s = c t).  Sweeps end when one makes no rotation, or after OS_MAX_SWEEPS.
-// M and W are column-major, in shared memory when they fit, else in Mg / Wg.
+// each round pairs the columns by the circle method and a group of OS_GROUP = 8
+// lanes takes one pair, so the 128 groups of the CTA cover every pair of a
+// round (Lp / 2 <= 128) at once and a round costs one pair's latency and one
+// barrier.  For a pair: alpha = |m_p|^2, beta = |m_q|^2, gamma = m_p . m_q
+// (fp32, each lane a strided share, then a butterfly inside the group, which
+// leaves every lane of the group the same sums), and unless
+// |gamma| <= 1e-6 sqrt(alpha beta) (a little above the rounding of an fp32
+// dot product, so that sweeps terminate) columns p, q of M and of W are
+// rotated by the angle that makes them orthogonal (zeta = (beta - alpha) /
+// (2 gamma), t = sign(zeta) / (|zeta| + sqrt(1 + zeta^2)), c = 1 / sqrt(1 + t^2),
+// s = c t).  Sweeps end when one makes no rotation, or after OS_MAX_SWEEPS.
+// M [Lp][ldm] and W [Lp][ldw] are column-major with column strides of 8 mod 32
+// floats (the four groups of a warp take consecutive columns, which then fall
+// on distinct banks), in shared memory when they fit, else in Mg / Wg.
 // Output: Wt [L][L], Wt[j][k] = W[k][j].
 constexpr int OS_THREADS = 1024;
+constexpr int OS_GROUP = 8;
 constexpr int OS_MAX_SWEEPS = 30;
+static_assert(OS_THREADS / OS_GROUP >= 128, "one group per pair of a round (l <= 256)");
+
 __global__ void __launch_bounds__(OS_THREADS)
 k_onesided(const float* __restrict__ Mt, int L, float* __restrict__ Mg, float* __restrict__ Wg,
-           int in_smem, float* __restrict__ Wt) {
+           int in_smem, int ldm, int ldw, float* __restrict__ Wt) {
   extern __shared__ float osm[];
   __shared__ int s_rot;
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nw = OS_THREADS / 32;
+  const int tid = threadIdx.x, grp = tid / OS_GROUP, u = tid % OS_GROUP;
   const int Lp = L + (L & 1), half = Lp / 2;
-  float* M = in_smem ? osm : Mg;                       // [Lp][L]
-  float* W = in_smem ? osm + (size_t)Lp * L : Wg;      // [Lp][Lp]
-  for (int q = tid; q < Lp * L; q += OS_THREADS) M[q] = q < L * L ? Mt[q] : 0.f;
-  for (int q = tid; q < Lp * Lp; q += OS_THREADS) W[q] = (q / Lp == q % Lp) ? 1.f : 0.f;
-  __syncthreads();
+  float* M = in_smem ? osm : Mg;                       // [Lp][ldm]
+  float* W = in_smem ? osm + (size_t)Lp * ldm : Wg;    // [Lp][ldw]
+  for (int e = tid; e < Lp * ldm; e += OS_THREADS) {
+    const int c = e / ldm, i = e - c * ldm;
+    M[e] = (c < L && i < L) ? Mt[(size_t)c * L + i] : 0.f;
+  }
+  for (int e = tid; e < Lp * ldw; e += OS_THREADS) {
+    const int c = e / ldw, i = e - c * ldw;
+    W[e] = i == c ? 1.f : 0.f;
+  }
+  const bool active = grp < half;
   for (int sweep = 0; sweep < OS_MAX_SWEEPS; ++sweep) {
     if (tid == 0) s_rot = 0;
     __syncthreads();
+    bool rotated = false;
     for (int round = 0; round < Lp - 1; ++round) {
-      for (int P = warp; P < half; P += nw) {
-        int p, q;
-        if (P == 0) {
-          p = round;
-          q = Lp - 1;
-        } else {
-          p = round + P;
-          if (p >= Lp - 1) p -= Lp - 1;
-          q = round - P;
-          if (q < 0) q += Lp - 1;
-        }
-        float* mp = M + (size_t)p * L;
-        float* mq = M + (size_t)q * L;
-        float a = 0.f, b = 0.f, g = 0.f;
-        for (int i = lane; i < L; i += 32) {
+      int p = 0, q = 1;
+      if (grp == 0) {
+        p = round;
+        q = Lp - 1;
+      } else if (active) {
+        p = round + grp;
+        if (p >= Lp - 1) p -= Lp - 1;
+        q = round - grp;
+        if (q < 0) q += Lp - 1;
+      }
+      float* mp = M + (size_t)p * ldm;
+      float* mq = M + (size_t)q * ldm;
+      float a = 0.f, b = 0.f, g = 0.f;
+      if (active) {
+#pragma unroll 4
+        for (int i = u; i < L; i += OS_GROUP) {
           const float x = mp[i], y = mq[i];
           a = fmaf(x, x, a);
           b = fmaf(y, y, b);
           g = fmaf(x, y, g);
         }
-        for (int o = 16; o; o >>= 1) {
-          a += __shfl_xor_sync(0xffffffffu, a, o);
-          b += __shfl_xor_sync(0xffffffffu, b, o);
-          g += __shfl_xor_sync(0xffffffffu, g, o);
-        }
-        if (g == 0.f || fabsf(g) <= 1e-6f * sqrtf(a * b)) continue;  // warp-uniform
+      }
+      // (xor offsets below OS_GROUP stay inside the aligned group)
+#pragma unroll
+      for (int o = OS_GROUP / 2; o; o >>= 1) {
+        a += __shfl_xor_sync(0xffffffffu, a, o);
+        b += __shfl_xor_sync(0xffffffffu, b, o);
+        g += __shfl_xor_sync(0xffffffffu, g, o);
+      }
+      if (active && g != 0.f && fabsf(g) > 1e-6f * sqrtf(a * b)) {  // group-uniform
         // (an overflowing zeta gives t = 0: no rotation, never a NaN)
         const float z = (b - a) / (2.f * g);
         const float t = (z >= 0.f ? 1.f : -1.f) / (fabsf(z) + sqrtf(1.f + z * z));
-        const float c = 1.f / sqrtf(1.f + t * t), s = t * c;
-        float* wp = W + (size_t)p * Lp;
-        float* wq = W + (size_t)q * Lp;
-        for (int i = lane; i < Lp; i += 32) {  // Lp >= L: one loop for M and W
-          if (i < L) {
-            const float x = mp[i], y = mq[i];
-            mp[i] = c * x - s * y;
-            mq[i] = s * x + c * y;
-          }
-          const float x = wp[i], y = wq[i];
-          wp[i] = c * x - s * y;
-          wq[i] = s * x + c * y;
+        const float c = 1.f / sqrtf(1.f + t * t), sn = t * c;
+#pragma unroll 4
+        for (int i = u; i < L; i += OS_GROUP) {
+          const float x = mp[i], y = mq[i];
+          mp[i] = c * x - sn * y;
+          mq[i] = sn * x + c * y;
         }
-        if (lane == 0) s_rot = 1;
+        float* wp = W + (size_t)p * ldw;
+        float* wq = W + (size_t)q * ldw;
+#pragma unroll 4
+        for (int i = u; i < Lp; i += OS_GROUP) {
+          const float x = wp[i], y = wq[i];
+          wp[i] = c * x - sn * y;
+          wq[i] = sn * x + c * y;
+        }
+        rotated = true;
       }
       __syncthreads();
     }
-    if (s_rot == 0) break;  // read after the round's barrier; every thread sees the same value
+    if (rotated) s_rot = 1;
+    __syncthreads();
+    if (s_rot == 0) break;  // every thread reads the same value after the barrier
     __syncthreads();        // before thread 0 clears s_rot for the next sweep
   }
-  for (int q = tid; q < L * L; q += OS_THREADS) {
-    const int j = q / L, k = q % L;
-    Wt[q] = W[(size_t)j * Lp + k];
+  for (int e = tid; e < L * L; e += OS_THREADS) {
+    const int j = e / L, k = e - j * L;
+    Wt[e] = W[(size_t)j * ldw + k];
+  }
+}
+
+// The same Jacobi for L <= 16 NV with M and W in shared memory: each lane of
+// a group holds NV float2 pieces of each of its two columns (elements
+// 16 v + 2 u, + 1), loaded once for the dot products and kept in registers
+// for the rotation; W's columns stream through as float2 too.  Column strides
+// ldm, ldw >= 16 NV are multiples of 8 but not of 32, so the four groups of a
+// warp (consecutive columns) spread each 256-byte access over two wavefronts.
+// The padding rows beyond L (beyond Lp for W) are zero and stay zero.
+template <int NV>
+__global__ void __launch_bounds__(OS_THREADS)
+k_onesided_v(const float* __restrict__ Mt, int L, int ldm, int ldw, float* __restrict__ Wt) {
+  extern __shared__ __align__(16) float osm[];
+  __shared__ int s_rot;
+  const int tid = threadIdx.x, grp = tid / OS_GROUP, u = tid % OS_GROUP;
+  const int Lp = L + (L & 1), half = Lp / 2;
+  float* M = osm;                       // [Lp][ldm]
+  float* W = osm + (size_t)Lp * ldm;    // [Lp][ldw]
+  for (int e = tid; e < Lp * ldm; e += OS_THREADS) {
+    const int c = e / ldm, i = e - c * ldm;
+    M[e] = (c < L && i < L) ? Mt[(size_t)c * L + i] : 0.f;
+  }
+  for (int e = tid; e < Lp * ldw; e += OS_THREADS) {
+    const int c = e / ldw, i = e - c * ldw;
+    W[e] = i == c ? 1.f : 0.f;
+  }
+  const bool active = grp < half;
+  for (int sweep = 0; sweep < OS_MAX_SWEEPS; ++sweep) {
+    if (tid == 0) s_rot = 0;
+    __syncthreads();
+    bool rotated = false;
+    for (int round = 0; round < Lp - 1; ++round) {
+      int p = 0, q = 1;
+      if (grp == 0) {
+        p = round;
+        q = Lp - 1;
+      } else if (active) {
+        p = round + grp;
+        if (p >= Lp - 1) p -= Lp - 1;
+        q = round - grp;
+        if (q < 0) q += Lp - 1;
+      }
+      float2* mp = reinterpret_cast<float2*>(M + (size_t)p * ldm) + u;
+      float2* mq = reinterpret_cast<float2*>(M + (size_t)q * ldm) + u;
+      float2 xp[NV], xq[NV];
+      float a = 0.f, b = 0.f, g = 0.f;
+      if (active) {
+#pragma unroll
+        for (int v = 0; v < NV; ++v) {
+          xp[v] = mp[8 * v];
+          xq[v] = mq[8 * v];
+        }
+#pragma unroll
+        for (int v = 0; v < NV; ++v) {
+          a = fmaf(xp[v].x, xp[v].x, a);
+          a = fmaf(xp[v].y, xp[v].y, a);
+          b = fmaf(xq[v].x, xq[v].x, b);
+          b = fmaf(xq[v].y, xq[v].y, b);
+          g = fmaf(xp[v].x, xq[v].x, g);
+          g = fmaf(xp[v].y, xq[v].y, g);
+        }
+      }
+#pragma unroll
+      for (int o = OS_GROUP / 2; o; o >>= 1) {
+        a += __shfl_xor_sync(0xffffffffu, a, o);
+        b += __shfl_xor_sync(0xffffffffu, b, o);
+        g += __shfl_xor_sync(0xffffffffu, g, o);
+      }
+      if (active && g != 0.f && fabsf(g) > 1e-6f * sqrtf(a * b)) {  // group-uniform
+        const float z = (b - a) / (2.f * g);
+        const float t = (z >= 0.f ? 1.f : -1.f) / (fabsf(z) + sqrtf(1.f + z * z));
+        const float c = 1.f / sqrtf(1.f + t * t), sn = t * c;
+#pragma unroll
+        for (int v = 0; v < NV; ++v) {
+          mp[8 * v] = make_float2(c * xp[v].x - sn * xq[v].x, c * xp[v].y - sn * xq[v].y);
+          mq[8 * v] = make_float2(sn * xp[v].x + c * xq[v].x, sn * xp[v].y + c * xq[v].y);
+        }
+        float2* wp = reinterpret_cast<float2*>(W + (size_t)p * ldw) + u;
+        float2* wq = reinterpret_cast<float2*>(W + (size_t)q * ldw) + u;
+#pragma unroll
+        for (int v = 0; v < NV; ++v) {
+          const float2 x = wp[8 * v], y = wq[8 * v];
+          wp[8 * v] = make_float2(c * x.x - sn * y.x, c * x.y - sn * y.y);
+          wq[8 * v] = make_float2(sn * x.x + c * y.x, sn * x.y + c * y.y);
+        }
+        rotated = true;
+      }
+      __syncthreads();
+    }
+    if (rotated) s_rot = 1;
+    __syncthreads();
+    if (s_rot == 0) break;
+    __syncthreads();
+  }
+  for (int e = tid; e < L * L; e += OS_THREADS) {
+    const int j = e / L, k = e - j * L;
+    Wt[e] = W[(size_t)j * ldw + k];
   }
 }
 
@@ -450,6 +696,7 @@ __global__ void k_sign(float* __restrict__ U, float* __restrict__ V, int rows, i
 
 bool g_ch_cap[64] = {};
 bool g_os_cap[64] = {};
+bool g_osv_cap[16][64] = {};
 
 }  // namespace
 }  // namespace lx
@@ -460,6 +707,19 @@ constexpr int CP_MAX_L = 256;
 constexpr size_t CP_SMEM_CAP = 200 * 1024;
 
 size_t al256(size_t v) { return (v + 255) / 256 * 256; }
+
+// Column stride (floats) of the Jacobi's M and W for columns of n entries: a
+// multiple of 8 that is 8 mod 32 (n + 39 at most).
+long os_ld(long n) {
+  long ld = (n + 7) / 8 * 8;
+  ld += ((8 - ld % 32) + 32) % 32;
+  return ld;
+}
+// Column stride of the register form: a multiple of 8 that is not one of 32.
+long os_ld_v(long n) {
+  long ld = (n + 7) / 8 * 8;
+  return ld % 32 == 0 ? ld + 8 : ld;
+}
 
 struct CompressWs {
   float *y0, *y1, *z0, *z1, *T, *Wu, *Wv, *L1, *L2, *Xg, *Mt, *Wt, *MWn, *Wn, *Mg, *Wg;
@@ -493,8 +753,8 @@ CompressWs carve(char* base, long rows, long cols, long l, long r) {
   w.Wt = (float*)take(4 * l * l);
   w.MWn = (float*)take(4 * l * l);
   w.Wn = (float*)take(4 * l * l);
-  w.Mg = (float*)take(4 * Lp * l);
-  w.Wg = (float*)take(4 * Lp * Lp);
+  w.Mg = (float*)take(4 * Lp * os_ld(l));
+  w.Wg = (float*)take(4 * Lp * os_ld(Lp));
   w.G = (double*)take(8 * l * l);
   w.sig64 = (double*)take(8 * l);
   w.tc = take(res_tc_workspace(rows, cols, l));
@@ -546,40 +806,70 @@ lx_status run_compress(int rows, int cols, const TW* Wd, const TW* Wm, const flo
   const bool x_smem = 2 * tri <= CP_SMEM_CAP;  // L and X both in shared memory
   const size_t ch_smem = x_smem ? 2 * tri : tri;
   LX_CUDA(smem_cap_once((const void*)k_chol32, (int)CP_SMEM_CAP, dev, g_ch_cap));
-  // CholeskyQR twice (the first pass shifted by 1e-6 of the largest Gram
-  // diagonal, so rank-deficient bases stay factorable); X [n][l] ends
-  // orthonormal, tmp is scratch; the two factors stay in L1, L2.
-  auto orth2 = [&](float* X, float* tmp, int n) {
-    gram(X, n);
+  // CholeskyQR (the first pass shifted by 1e-6 of the largest Gram diagonal,
+  // so rank-deficient bases stay factorable).  orth2 runs it twice, X [n][l]
+  // ends orthonormal and its two factors stay in L1, L2; orth1 runs the
+  // shifted pass once, for the intermediate bases of the power iterations,
+  // whose span is all the next product uses (the final Q and Z take orth2).
+  // Both leave the result in *X and swap *X with the scratch *tmp.
+  auto orth1 = [&](float** X, float** tmp, int n) {
+    gram(*X, n);
     k_chol32<<<1, CH_THREADS, ch_smem, s>>>(w.G, l, 1e-6f, w.L1, w.Xg, x_smem ? 1 : 0, w.T);
-    gemm(A_F32, X, w.T, tmp, n, l, l);
-    gram(tmp, n);
-    k_chol32<<<1, CH_THREADS, ch_smem, s>>>(w.G, l, 0.f, w.L2, w.Xg, x_smem ? 1 : 0, w.T);
-    gemm(A_F32, tmp, w.T, X, n, l, l);
+    gemm(A_F32, *X, w.T, *tmp, n, l, l);
+    std::swap(*X, *tmp);
   };
-  gemm(A_RES, nullptr, omega, w.y0, rows, l, cols);  // Y = R Omega
-  orth2(w.y0, w.y1, rows);                            // Q
+  auto orth2 = [&](float** X, float** tmp, int n) {
+    gram(*X, n);
+    k_chol32<<<1, CH_THREADS, ch_smem, s>>>(w.G, l, 1e-6f, w.L1, w.Xg, x_smem ? 1 : 0, w.T);
+    gemm(A_F32, *X, w.T, *tmp, n, l, l);
+    gram(*tmp, n);
+    k_chol32<<<1, CH_THREADS, ch_smem, s>>>(w.G, l, 0.f, w.L2, w.Xg, x_smem ? 1 : 0, w.T);
+    gemm(A_F32, *tmp, w.T, *X, n, l, l);
+  };
+  float *yc = w.y0, *yt = w.y1, *zc = w.z0, *zt = w.z1;
+  gemm(A_RES, nullptr, omega, yc, rows, l, cols);  // Y = R Omega
+  if (q == 0) orth2(&yc, &yt, rows);              // Q
+  else orth1(&yc, &yt, rows);
   for (int it = 0; it < q; ++it) {
-    gemm(A_RES_T, nullptr, w.y0, w.z0, cols, l, rows);  // R^T Q
-    orth2(w.z0, w.z1, cols);
-    gemm(A_RES, nullptr, w.z0, w.y0, rows, l, cols);    // R Z
-    orth2(w.y0, w.y1, rows);
+    gemm(A_RES_T, nullptr, yc, zc, cols, l, rows);  // R^T Q
+    orth1(&zc, &zt, cols);
+    gemm(A_RES, nullptr, zc, yc, rows, l, cols);    // R Z
+    if (it + 1 == q) orth2(&yc, &yt, rows);
+    else orth1(&yc, &yt, rows);
   }
   // Z = R^T Q = Bs^T = Z2 (L1 L2)^T with Z2 orthonormal, so Bs = M Z2^T for
   // M = L1 L2, and the SVD of Bs follows from the small SVD of M.
-  gemm(A_RES_T, nullptr, w.y0, w.z0, cols, l, rows);
-  orth2(w.z0, w.z1, cols);
+  gemm(A_RES_T, nullptr, yc, zc, cols, l, rows);
+  orth2(&zc, &zt, cols);
   k_trmm<<<l, 256, 0, s>>>(w.L1, w.L2, l, w.Mt);
   const int Lp = l + (l & 1);
-  const size_t os_bytes = sizeof(float) * ((size_t)Lp * l + (size_t)Lp * Lp);
-  const bool os_smem = os_bytes <= CP_SMEM_CAP;
-  if (os_smem) LX_CUDA(smem_cap_once((const void*)k_onesided, (int)CP_SMEM_CAP, dev, g_os_cap));
-  k_onesided<<<1, OS_THREADS, os_smem ? os_bytes : 0, s>>>(w.Mt, l, w.Mg, w.Wg, os_smem ? 1 : 0,
-                                                          w.Wt);
+  // register form when the columns fit NV float2 pieces per lane (NV <= 9,
+  // l <= 144) and M, W fit shared memory; else the strided form
+  const int nv = Lp <= 32 ? 2 : Lp <= 48 ? 3 : Lp <= 80 ? 5 : Lp <= 144 ? 9 : 0;
+  const long ldv = nv ? os_ld_v(16 * nv) : 0;
+  const size_t osv_bytes = sizeof(float) * (size_t)Lp * 2 * ldv;
+  if (nv && osv_bytes <= CP_SMEM_CAP) {
+    auto launch_v = [&](auto kern) -> lx_status {
+      LX_CUDA(smem_cap_once((const void*)kern, (int)CP_SMEM_CAP, dev, g_osv_cap[nv]));
+      kern<<<1, OS_THREADS, osv_bytes, s>>>(w.Mt, l, (int)ldv, (int)ldv, w.Wt);
+      return LX_OK;
+    };
+    if (nv == 2) LX_TRY(launch_v(k_onesided_v<2>));
+    else if (nv == 3) LX_TRY(launch_v(k_onesided_v<3>));
+    else if (nv == 5) LX_TRY(launch_v(k_onesided_v<5>));
+    else LX_TRY(launch_v(k_onesided_v<9>));
+  } else {
+    const long ldm = os_ld(l), ldw = os_ld(Lp);
+    const size_t os_bytes = sizeof(float) * (size_t)Lp * (ldm + ldw);
+    const bool os_smem = os_bytes <= CP_SMEM_CAP;
+    if (os_smem) LX_CUDA(smem_cap_once((const void*)k_onesided, (int)CP_SMEM_CAP, dev, g_os_cap));
+    k_onesided<<<1, OS_THREADS, os_smem ? os_bytes : 0, s>>>(w.Mt, l, w.Mg, w.Wg, os_smem ? 1 : 0,
+                                                            (int)ldm, (int)ldw, w.Wt);
+  }
   k_ritz<<<l, 256, 0, s>>>(w.Mt, w.Wt, l, w.MWn, w.Wn, w.sig64);
   k_finish<<<1, 256, 0, s>>>(w.sig64, w.MWn, w.Wn, l, r, w.Wu, w.Wv, sigma);
-  gemm(A_F32, w.y0, w.Wu, U, rows, r, l);   // U_r S^(1/2)
-  gemm(A_F32, w.z0, w.Wv, V, cols, r, l);   // V_r S^(1/2)
+  gemm(A_F32, yc, w.Wu, U, rows, r, l);   // U_r S^(1/2)
+  gemm(A_F32, zc, w.Wv, V, cols, r, l);   // V_r S^(1/2)
   k_sign<<<r, 256, 0, s>>>(U, V, rows, cols, r);
   LX_CUDA(cudaGetLastError());
   return tc_status;

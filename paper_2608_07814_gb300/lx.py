@@ -387,3 +387,34 @@ def compress_factor(w_dom: torch.Tensor, w_mem: torch.Tensor, omega: torch.Tenso
                                     _ptr(omega), l, r, power_iters, _ptr(U), _ptr(V), _ptr(s),
                                     _ptr(workspace), workspace.numel(), _stream(stream)))
     return U, V, s
+
+
+_MEMBER_STREAMS: Dict[int, list] = {}
+
+
+def compress_member(w_doms, w_mems, omegas, r: int, power_iters: int = 2, workspaces=None,
+                    outs=None):
+    """The gate, up and down projections of one member, each through
+    lx_compress_factor on a stream of its own (the three are independent), the
+    calling stream waiting for all three.  Lists of three: dominant and member
+    matrices, fp32 Gaussian test matrices, optional workspaces and outputs.
+    Returns the three (U, V, s)."""
+    dev = w_doms[0].device
+    main = torch.cuda.current_stream(dev)
+    streams = _MEMBER_STREAMS.setdefault(dev.index or 0,
+                                         [torch.cuda.Stream(device=dev) for _ in range(3)])
+    start = torch.cuda.Event()
+    start.record(main)
+    res = []
+    for j in range(3):
+        st = streams[j]
+        st.wait_event(start)
+        ws = workspaces[j] if workspaces is not None else None
+        out = outs[j] if outs is not None else None
+        with torch.cuda.stream(st):
+            res.append(compress_factor(w_doms[j], w_mems[j], omegas[j], r, power_iters,
+                                       workspace=ws, stream=st, out=out))
+        done = torch.cuda.Event()
+        done.record(st)
+        main.wait_event(done)
+    return res

@@ -55,6 +55,7 @@ CASES = [  # rows, cols, dtype, r, l, power_iters, kind
     (64, 64, "f32", 8, 16, 1, "zero"),
     (136, 200, "bf16", 20, 21, 0, "flat"),
     (256, 192, "bf16", 192, 192, 1, "decay"),
+    (256, 320, "bf16", 200, 256, 1, "decay"),   # l = 256: 128 column pairs per round
 ]
 
 
