@@ -676,6 +676,19 @@ static void split_op(lx_layer* L, StreamOp& o, float* part, long stride, int blo
   (void)L;
 }
 
+// Whether the anchors' split-K pays at this batch: measured on GB300 (decode
+// forwards of the Qwen3-30B-A3B-shaped and the high-expert-count layers, T from
+// 1 to 256), it shortens the launches only while the batch's tokens times the
+// anchors' gate/up column tiles lie between about 1.5 and 3 times the
+// streaming grid -- the whole-K anchor tiles then make a last partial wave --
+// and costs time elsewhere (fewer, longer tiles already balance, or every tile
+// fits the first wave), through the partials' extra traffic.
+static bool split_pays(const lx_layer* L, int T) {
+  const long grid = (long)L->num_sms * SW_CTAS_PER_SM;
+  const long work = (long)T * ((2L * L->I + SW_ROWS - 1) / SW_ROWS);
+  return 2 * work >= 3 * grid && 10 * work <= 31 * grid;
+}
+
 // One streaming launch (launch group g) over up to three ops' tile grids, in
 // claim order.
 static lx_status run_stream(lx_layer* L, int g, std::initializer_list<const StreamOp*> ops,
@@ -706,7 +719,8 @@ lx_status launch_fast_experts(lx_layer* L, const void* x, int T, int k, void* y,
   const long H = L->H, I = L->I, rmax = L->max_rank;
   const __nv_bfloat16* xb = static_cast<const __nv_bfloat16*>(x);
   const bool split = w.hsplit && w.ysplit && warp_kernels_fit(L, k) &&
-                     (long)T * std::min<long>(L->N, (long)k * L->max_depth) <= w.split_rows;
+                     (long)T * std::min<long>(L->N, (long)k * L->max_depth) <= w.split_rows &&
+                     split_pays(L, T);
   int* dep_up = w.sctr + N_TILE_COUNTERS;
   int* dep_dn = dep_up + (size_t)L->N * STREAM_DEP_TB;
   // x-side: x V of every correction (whole-K tiles, claimed first), the shared

@@ -347,15 +347,34 @@ def test_qwen_decode_batches(T):
 
 
 @pytest.mark.parametrize("name", ["high_e", "tree", "binary", "single_base"])
-@pytest.mark.parametrize("T", [1, 64])
+@pytest.mark.parametrize("T", [1, 32, 64])
 def test_full_layers_decode(name, T):
-    """Decode batches of the other full-size layers (split-K anchor tiles with
-    three and four K ranges, depth-3 tree paths)."""
+    """Decode batches of the other full-size layers (depth-3 tree paths; split-K
+    anchor tiles where the streaming path splits them: the high-expert-count
+    layer at T = 32, gate/up in four K ranges and down in two, the d_ff = 768
+    layers at T = 64, gate/up in four)."""
     src, L = installed(name, FULL[name])
     x = synth.tokens(src, T, seed=40 + T)
     ids, _ = check_route(src, L, x, 8)
     check_buckets(src, L, ids)
     check_forward(src, L, x, 8)
+
+
+@pytest.mark.parametrize("name", ["stream_split_ragged", "stream_split_tree"])
+def test_stream_split_band(name):
+    """A batch inside the band where the streaming path splits the anchors'
+    products along K (tokens x gate/up column tiles between 1.5 and 3.1 times
+    the streaming grid of 5 CTAs per SM): three K ranges with a ragged last one,
+    and two on a tree layer."""
+    src, L = installed(name, SMALL[name])
+    grid = 5 * torch.cuda.get_device_properties(0).multi_processor_count
+    ct = (2 * src.d_ff + 63) // 64
+    T = -(-3 * grid // (2 * ct)) + 1
+    assert 10 * T * ct <= 31 * grid and T <= 256
+    x = synth.tokens(src, T, seed=60)
+    ids, _ = check_route(src, L, x, src.top_k)
+    check_buckets(src, L, ids)
+    check_forward(src, L, x, src.top_k)
 
 
 def test_qwen_decode_correction_visible():
@@ -366,7 +385,7 @@ def test_qwen_decode_correction_visible():
 
 
 @pytest.mark.parametrize("name", ["qwen_visible", "qwen_zero_dom", "high_e_visible"])
-@pytest.mark.parametrize("T", [1, 8, 64])
+@pytest.mark.parametrize("T", [1, 8, 32, 64])
 def test_full_size_correction_visible_decode(name, T):
     """Full-size layers whose corrections are visible under the bf16 bar (or
     the only term), every token of a decode batch."""
