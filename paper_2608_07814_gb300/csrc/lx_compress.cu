@@ -10,11 +10,11 @@
 //               formed on load), R^T (columns of the same), or an fp32 matrix.
 //   k_gram      G = X^T X to float64 accuracy (exact fp32 products, error-free
 //               two-sum accumulation on the fp32 pipes), stored in float64.
-//   k_chol32    one CTA: Cholesky G + s I = L L^T (fp32 in shared memory, one
-//               barrier per step; a small relative shift in the first of the
-//               two passes keeps rank-deficient bases factorable) and
-//               T = L^-T by forward elimination, so that X T has orthonormal
-//               columns (CholeskyQR, run twice per orthonormalisation).
+//   k_chol32    one CTA: Cholesky G + s I = L L^T (fp32 in shared memory,
+//               blocked by 16 columns; a small relative shift in the first
+//               pass keeps rank-deficient bases factorable) and T = L^-T,
+//               blocked the same way, so that X T has orthonormal columns
+//               (CholeskyQR).
 //   k_trmm      M = L1 L2, the triangular factor of R^T Q = Z2 M^T.
 //   k_onesided  one CTA: one-sided Jacobi SVD of M (fp32 rotations, shared
 //               memory, every pair of a round at once), M W = U S.
@@ -224,34 +224,43 @@ k_gram(const float* __restrict__ X, int n, int L, double* __restrict__ G) {
 
 // One CTA (L <= 256).  Cholesky of G + s I in fp32 (G float64, rounded once;
 // s = shift_rel * max diag(G)) in a packed lower triangle in shared memory
-// (L (L + 1) / 2 floats, row i from i (i + 1) / 2), pivots floored at 1e-30.
-// Right-looking with the column scaling deferred: step j subtracts
-// (a_ij / l_jj) (a_cj / l_jj) from every trailing entry (j < c <= i) and
-// leaves column j itself unscaled, so that one barrier separates the steps
-// (warps take rows, lanes columns, each lane holding its entries of column j
-// in registers for all of its warp's rows); the columns are scaled once at the
-// end.
-// Then X = L^-1 by forward elimination of L X = I, again one barrier per step:
-// with Y the rows of X before their division by the diagonal, step p
-// subtracts (l_ip / l_pp) y_p from every row i > p (y_p is final by then),
-// and X = Y / diag(L) at the end.  X is packed like L, in shared memory when
-// x_in_smem, else in the global scratch Xg.  T = X^T, so that Y T = Y L^-T has
-// orthonormal columns when Y^T Y = G (CholeskyQR).  The factor itself is
-// written to Lout [L][L] (zero above the diagonal).  A zero Gram gives
-// Lout = T = 0.
-constexpr int CH_THREADS = 1024;
-constexpr int CH_REGS = 8;  // 32 CH_REGS >= 256 >= L
+// (L (L + 1) / 2 floats, row i from i (i + 1) / 2), pivots floored at 1e-30,
+// blocked by 16 columns (right-looking): warp 0 factors the diagonal block in
+// place (lane i updates row i; warp barriers only), one thread per row below
+// solves its 16 panel entries against it (forward substitution), and the
+// trailing triangle takes the panel's rank-16 update in 4 x 4 register tiles
+// from a transposed copy of the panel.  Then X = L^-1, blocked the same way:
+// the diagonal blocks' inverses
+// (one warp each, lane m column m), and for block row i and every block
+// column k < i, X_ik = -X_ii (sum_{k <= m < i} L_im X_mk) in two tiled
+// products.  X is packed like L, in shared memory when x_in_smem, else in the
+// global scratch Xg.  T = X^T, so that Y T = Y L^-T has orthonormal columns
+// when Y^T Y = G (CholeskyQR).  The factor is written to Lout [L][L] (zero
+// above the diagonal).  A zero Gram gives Lout = T = 0.
+constexpr int CH_THREADS = 512;  // 16 warps: nb <= 16 diagonal blocks, 128 registers a thread
+constexpr int CH_B = 16;  // block width
 __device__ __forceinline__ int tri_off(int i) { return i * (i + 1) / 2; }
 
-__global__ void __launch_bounds__(CH_THREADS)
+// row-major 4 x 4 tile index blk of a lower block triangle -> (bi, bc), bc <= bi
+__device__ __forceinline__ void tri_tile(int blk, int& bi, int& bc) {
+  int b = (int)((sqrtf(8.f * (float)blk + 1.f) - 1.f) * 0.5f);
+  while (b * (b + 1) / 2 > blk) --b;
+  while ((b + 1) * (b + 2) / 2 <= blk) ++b;
+  bi = b;
+  bc = blk - b * (b + 1) / 2;
+}
+
+__global__ void __launch_bounds__(CH_THREADS, 1)
 k_chol32(const double* __restrict__ G, int L, float shift_rel, float* __restrict__ Lout,
          float* __restrict__ Xg, int x_in_smem, float* __restrict__ T) {
-  extern __shared__ float Ls[];
-  float* Xp = x_in_smem ? Ls + tri_off(L) : Xg;  // packed lower X
+  extern __shared__ __align__(16) float Ls[];
+  const int ldp = (L + 3) & ~3;                      // panel copy: [CH_B][ldp], also S below
+  float* Pt = Ls + ((tri_off(L) + 3) & ~3);
+  float* Xp = x_in_smem ? Pt + CH_B * ldp : Xg;      // packed lower X
   __shared__ double s_md;
-  __shared__ float s_diag[256];  // the factor's diagonal
-  __shared__ float s_rdiag[256];  // its reciprocals
+  __shared__ float s_rdiag[256];  // reciprocals of the factor's diagonal
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nw = CH_THREADS / 32;
+  const int nb = (L + CH_B - 1) / CH_B;
   if (warp == 0) {
     double md = 0.0;
     for (int i = lane; i < L; i += 32) md = fmax(md, G[(size_t)i * L + i]);
@@ -273,82 +282,160 @@ k_chol32(const double* __restrict__ G, int L, float shift_rel, float* __restrict
   for (int i = warp; i < L; i += nw)
     for (int j = lane; j <= i; j += 32)
       Ls[tri_off(i) + j] = (float)G[(size_t)i * L + j] + (i == j ? shift : 0.f);
-  // l_jj = sqrt(max(pivot, 1e-30)) and its reciprocal are formed once, by the
-  // thread that finalises the pivot: here for j = 0, else in step j - 1
-  if (tid == 0) {
-    const float l00 = sqrtf(fmaxf((float)G[0] + shift, 1e-30f));
-    s_diag[0] = l00;
-    s_rdiag[0] = 1.f / l00;
-  }
   __syncthreads();
-  for (int j = 0; j < L; ++j) {
-    const float rl = s_rdiag[j];
-    // this lane's entries of the scaled column j (rows c = j + 1 + lane + 32 k),
-    // the same for every row the warp updates
-    float lc[CH_REGS];
-#pragma unroll
-    for (int k = 0; k < CH_REGS; ++k) {
-      if (j + 1 + 32 * k >= L) break;  // warp-uniform
-      const int c = j + 1 + lane + 32 * k;
-      lc[k] = c < L ? Ls[tri_off(c) + j] * rl : 0.f;
+  // ---- factorization
+  for (int kb = 0; kb < nb; ++kb) {
+    const int j0 = kb * CH_B, bw = min(CH_B, L - j0), j1 = j0 + bw, nt = L - j1;
+    if (warp == 0) {
+      // lane i: row j0 + i of the diagonal block, in place in the packed triangle
+      float* Ar = Ls + tri_off(j0 + min(lane, bw - 1)) + j0;
+      for (int j = 0; j < bw; ++j) {
+        const float d = sqrtf(fmaxf(Ls[tri_off(j0 + j) + j0 + j], 1e-30f));
+        const float rd = 1.f / d;
+        __syncwarp();
+        if (lane == j) Ar[j] = d;
+        else if (lane > j && lane < bw) Ar[j] *= rd;  // l_ij
+        __syncwarp();
+        if (lane > j && lane < bw) {
+          const float lij = Ar[j];
+          for (int c = j + 1; c <= lane; ++c) Ar[c] = fmaf(-lij, Ls[tri_off(j0 + c) + j0 + j], Ar[c]);
+        }
+        if (lane == 0) s_rdiag[j0 + j] = rd;
+        __syncwarp();
+      }
     }
-    for (int i = j + 1 + warp; i < L; i += nw) {
-      float* Ai = Ls + tri_off(i);
-      const float lij = Ai[j] * rl;
+    __syncthreads();
+    if (nt > 0) {
+      // panel: row i solves x L_kk^T = a_i[j0 : j1]
+      for (int i = j1 + tid; i < L; i += CH_THREADS) {
+        float x[CH_B];
+        float* Ai = Ls + tri_off(i) + j0;
 #pragma unroll
-      for (int k = 0; k < CH_REGS; ++k) {
-        const int c = j + 1 + lane + 32 * k;
-        if (j + 1 + 32 * k > i) break;  // warp-uniform
-        if (c <= i) {
-          const float v = fmaf(-lij, lc[k], Ai[c]);
-          Ai[c] = v;
-          if (c == i && i == j + 1) {  // the next pivot is final
-            const float d = sqrtf(fmaxf(v, 1e-30f));
-            s_diag[i] = d;
-            s_rdiag[i] = 1.f / d;
+        for (int c = 0; c < CH_B; ++c) x[c] = c < bw ? Ai[c] : 0.f;
+#pragma unroll
+        for (int c = 0; c < CH_B; ++c) {
+          if (c < bw) {
+            x[c] *= s_rdiag[j0 + c];
+#pragma unroll
+            for (int c2 = c + 1; c2 < CH_B; ++c2)
+              if (c2 < bw) x[c2] = fmaf(-x[c], Ls[tri_off(j0 + c2) + j0 + c], x[c2]);
+          }
+        }
+#pragma unroll
+        for (int c = 0; c < CH_B; ++c)
+          if (c < bw) {
+            Ai[c] = x[c];
+            Pt[c * ldp + (i - j1)] = x[c];
+          }
+      }
+      __syncthreads();
+      // trailing triangle: A_ic -= sum_m P_im P_cm, 4 x 4 tiles
+      const int n4 = (nt + 3) / 4;
+      for (int blk = tid; blk < n4 * (n4 + 1) / 2; blk += CH_THREADS) {
+        int bi, bc;
+        tri_tile(blk, bi, bc);
+        float acc[4][4] = {};
+        for (int m = 0; m < bw; ++m) {
+          const float4 a = *reinterpret_cast<const float4*>(Pt + m * ldp + 4 * bi);
+          const float4 b = *reinterpret_cast<const float4*>(Pt + m * ldp + 4 * bc);
+          const float av[4] = {a.x, a.y, a.z, a.w}, bv[4] = {b.x, b.y, b.z, b.w};
+#pragma unroll
+          for (int u = 0; u < 4; ++u)
+#pragma unroll
+            for (int v = 0; v < 4; ++v) acc[u][v] = fmaf(av[u], bv[v], acc[u][v]);
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int i = j1 + 4 * bi + u;
+#pragma unroll
+          for (int v = 0; v < 4; ++v) {
+            const int c = j1 + 4 * bc + v;
+            if (i < L && c <= i) Ls[tri_off(i) + c] -= acc[u][v];
           }
         }
       }
+      __syncthreads();
     }
-    __syncthreads();
   }
-  // scale the columns; Y = I
-  for (int i = warp; i < L; i += nw) {
-    float* Ai = Ls + tri_off(i);
-    float* Yi = Xp + tri_off(i);
-    for (int j = lane; j <= i; j += 32) {
-      Ai[j] = j == i ? s_diag[i] : Ai[j] * s_rdiag[j];
-      Yi[j] = j == i ? 1.f : 0.f;
+  // ---- X = L^-1: the diagonal blocks, one warp each (lane m: column m)
+  if (warp < nb) {
+    const int j0 = warp * CH_B, bw = min(CH_B, L - j0);
+    float x[CH_B];
+#pragma unroll
+    for (int i = 0; i < CH_B; ++i) x[i] = i == lane ? 1.f : 0.f;
+#pragma unroll
+    for (int p = 0; p < CH_B; ++p) {
+      if (p < bw) {
+        x[p] *= s_rdiag[j0 + p];
+#pragma unroll
+        for (int i = p + 1; i < CH_B; ++i)
+          if (i < bw) x[i] = fmaf(-Ls[tri_off(j0 + i) + j0 + p], x[p], x[i]);
+      }
+    }
+    if (lane < bw) {
+#pragma unroll
+      for (int i = 0; i < CH_B; ++i)
+        if (i >= lane && i < bw) Xp[tri_off(j0 + i) + j0 + lane] = x[i];
     }
   }
   __syncthreads();
-  for (int p = 0; p + 1 < L; ++p) {
-    const float rp = s_rdiag[p];
-    const float* yp = Xp + tri_off(p);
-    float yv[CH_REGS];  // this lane's entries of y_p (columns lane + 32 k)
+  // block row ib: S_k = sum_{k <= m < ib} L_{ib,m} X_{m,k} (into the panel
+  // buffer), then X_{ib,k} = -X_{ib,ib} S_k, for every k < ib
+  float* S = Pt;  // [k][CH_B rows][CH_B columns]
+  for (int ib = 1; ib < nb; ++ib) {
+    const int i0 = ib * CH_B, bwi = min(CH_B, L - i0), r4 = (bwi + 3) / 4;
+    const int ntile = ib * r4 * (CH_B / 4);
+    for (int tt = tid; tt < ntile; tt += CH_THREADS) {
+      const int kb = tt / (r4 * (CH_B / 4)), rem = tt - kb * r4 * (CH_B / 4);
+      const int rt = rem / (CH_B / 4), ct = rem - rt * (CH_B / 4);
+      const int col0 = kb * CH_B + 4 * ct;
+      float acc[4][4] = {};
+      for (int q = kb * CH_B; q < i0; ++q) {
+        float a[4], b[4];
 #pragma unroll
-    for (int k = 0; k < CH_REGS; ++k) {
-      if (32 * k > p) break;  // warp-uniform
-      const int c = lane + 32 * k;
-      yv[k] = c <= p ? yp[c] : 0.f;
+        for (int u = 0; u < 4; ++u) {
+          const int i = i0 + 4 * rt + u;
+          a[u] = i < L ? Ls[tri_off(i) + q] : 0.f;
+          b[u] = q >= col0 + u ? Xp[tri_off(q) + col0 + u] : 0.f;
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+#pragma unroll
+          for (int v = 0; v < 4; ++v) acc[u][v] = fmaf(a[u], b[v], acc[u][v]);
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+#pragma unroll
+        for (int v = 0; v < 4; ++v) S[(kb * CH_B + 4 * rt + u) * CH_B + 4 * ct + v] = acc[u][v];
     }
-    for (int i = p + 1 + warp; i < L; i += nw) {
-      const float f = Ls[tri_off(i) + p] * rp;
-      float* yi = Xp + tri_off(i);
+    __syncthreads();
+    for (int tt = tid; tt < ntile; tt += CH_THREADS) {
+      const int kb = tt / (r4 * (CH_B / 4)), rem = tt - kb * r4 * (CH_B / 4);
+      const int rt = rem / (CH_B / 4), ct = rem - rt * (CH_B / 4);
+      float acc[4][4] = {};
+      for (int p = 0; p < min(bwi, 4 * rt + 4); ++p) {
+        float a[4], b[4];
 #pragma unroll
-      for (int k = 0; k < CH_REGS; ++k) {
-        const int c = lane + 32 * k;
-        if (32 * k > p) break;  // warp-uniform
-        if (c <= p) yi[c] = fmaf(-f, yv[k], yi[c]);
+        for (int u = 0; u < 4; ++u) {
+          const int r = 4 * rt + u;
+          a[u] = (r < bwi && p <= r) ? Xp[tri_off(i0 + r) + i0 + p] : 0.f;
+          b[u] = S[(kb * CH_B + p) * CH_B + 4 * ct + u];
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+#pragma unroll
+          for (int v = 0; v < 4; ++v) acc[u][v] = fmaf(a[u], b[v], acc[u][v]);
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int r = 4 * rt + u;
+        if (r < bwi)
+#pragma unroll
+          for (int v = 0; v < 4; ++v) Xp[tri_off(i0 + r) + kb * CH_B + 4 * ct + v] = -acc[u][v];
       }
     }
     __syncthreads();
   }
-  for (int i = warp; i < L; i += nw) {
-    float* Yi = Xp + tri_off(i);
-    for (int c = lane; c <= i; c += 32) Yi[c] = Yi[c] * s_rdiag[i];
-  }
-  __syncthreads();
   for (int i = warp; i < L; i += nw) {
     const float* Ai = Ls + tri_off(i);
     for (int c = lane; c < L; c += 32) {
@@ -802,9 +889,12 @@ lx_status run_compress(int rows, int cols, const TW* Wd, const TW* Wm, const flo
     const dim3 grid((l + GR_T - 1) / GR_T, (l + GR_T - 1) / GR_T);
     k_gram<<<grid, GR_T * GR_T, 0, s>>>(X, n, l, w.G);
   };
+  // packed L (rounded to 16 bytes), the panel copy, and packed X
+  // when it fits too
   const size_t tri = sizeof(float) * (size_t)l * (l + 1) / 2;
-  const bool x_smem = 2 * tri <= CP_SMEM_CAP;  // L and X both in shared memory
-  const size_t ch_smem = x_smem ? 2 * tri : tri;
+  const size_t ch_base = (tri + 15) / 16 * 16 + sizeof(float) * CH_B * (size_t)((l + 3) & ~3);
+  const bool x_smem = ch_base + tri <= CP_SMEM_CAP;
+  const size_t ch_smem = x_smem ? ch_base + tri : ch_base;
   LX_CUDA(smem_cap_once((const void*)k_chol32, (int)CP_SMEM_CAP, dev, g_ch_cap));
   // CholeskyQR (the first pass shifted by 1e-6 of the largest Gram diagonal,
   // so rank-deficient bases stay factorable).  orth2 runs it twice, X [n][l]
