@@ -261,6 +261,24 @@ k_chol32(const double* __restrict__ G, int L, float shift_rel, float* __restrict
   __shared__ float s_rdiag[256];  // reciprocals of the factor's diagonal
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nw = CH_THREADS / 32;
   const int nb = (L + CH_B - 1) / CH_B;
+  // the lower triangle of G rounded to fp32, every load of a batch in flight
+  // (packed element e -> row i, column e - i (i + 1) / 2), while warp 0 also
+  // takes the largest diagonal entry
+  const int ntri = tri_off(L);
+  for (int e0 = tid; e0 < ntri; e0 += 4 * CH_THREADS) {
+    double g[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int e = e0 + u * CH_THREADS;
+      int i = (int)((sqrtf(8.f * (float)e + 1.f) - 1.f) * 0.5f);
+      while (tri_off(i) > e) --i;
+      while (tri_off(i + 1) <= e) ++i;
+      g[u] = e < ntri ? G[(size_t)i * L + (e - tri_off(i))] : 0.0;
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u)
+      if (e0 + u * CH_THREADS < ntri) Ls[e0 + u * CH_THREADS] = (float)g[u];
+  }
   if (warp == 0) {
     double md = 0.0;
     for (int i = lane; i < L; i += 32) md = fmax(md, G[(size_t)i * L + i]);
@@ -279,9 +297,7 @@ k_chol32(const double* __restrict__ G, int L, float shift_rel, float* __restrict
     return;
   }
   const float shift = (float)(shift_rel * md);
-  for (int i = warp; i < L; i += nw)
-    for (int j = lane; j <= i; j += 32)
-      Ls[tri_off(i) + j] = (float)G[(size_t)i * L + j] + (i == j ? shift : 0.f);
+  for (int i = tid; i < L; i += CH_THREADS) Ls[tri_off(i) + i] += shift;  // (float) g_ii + shift
   __syncthreads();
   // ---- factorization
   for (int kb = 0; kb < nb; ++kb) {
