@@ -105,3 +105,24 @@ def test_workspace_query_and_rejects():
                                 p(w), p(small), 256, None) == lx.LX_ERR_ARG    # workspace
     assert L.lx_compress_factor(lx.LX_F32, 64, 64, p(w), p(w), p(om), 16, 8, 99, p(w), p(w),
                                 p(w), p(small), 256, None) == lx.LX_ERR_ARG    # power_iters
+
+
+def test_member_projections_concurrent_same_bits():
+    """lx.compress_member runs a member's gate, up and down projections on three
+    streams; each projection's kernels are the same, so its factors equal, bit
+    for bit, those of the projections run one after another."""
+    rng = np.random.default_rng(99)
+    shapes = [(384, 512), (384, 512), (512, 384)]
+    r, l, q = 48, 56, 2
+    doms, mems, oms = [], [], []
+    for rows, cols in shapes:
+        Wd, Wm = _residual_pair(rows, cols, "flat", "bf16", rng)
+        doms.append(lx.host_to_torch(Wd, "bf16").cuda())
+        mems.append(lx.host_to_torch(Wm, "bf16").cuda())
+        oms.append(torch.from_numpy(rng.standard_normal((cols, l)).astype(np.float32)).cuda())
+    seq = [lx.compress_factor(doms[j], mems[j], oms[j], r, q) for j in range(3)]
+    conc = lx.compress_member(doms, mems, oms, r, q)
+    torch.cuda.synchronize()
+    for a, b in zip(seq, conc):
+        for x, y in zip(a, b):
+            assert torch.equal(x, y)
