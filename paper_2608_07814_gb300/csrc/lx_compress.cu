@@ -4,10 +4,12 @@
 // matrix given by the caller) and the symmetric split of Eq. factors,
 // U = U_r S_r^(1/2) [rows][r], V = V_r S_r^(1/2) [cols][r].
 //
-// Kernels:
+// Kernels (the products with R of bf16 weights run on the tensor cores, in
+// lx_compress_tc.cu):
 //   k_cgemm     fp32 GEMM (CUDA-core FMA, 64 x 64 tiles, 32-deep K chunks in
 //               shared memory); its A operand is R (rows of W_mem - W_dom,
-//               formed on load), R^T (columns of the same), or an fp32 matrix.
+//               formed on load; fp32 weights), R^T (columns of the same), or an
+//               fp32 matrix (the bases times the small factors).
 //   k_gram      G = X^T X to float64 accuracy (exact fp32 products, error-free
 //               two-sum accumulation on the fp32 pipes), stored in float64.
 //   k_chol32    one CTA: Cholesky G + s I = L L^T (fp32 in shared memory,
@@ -16,8 +18,11 @@
 //               blocked the same way, so that X T has orthonormal columns
 //               (CholeskyQR).
 //   k_trmm      M = L1 L2, the triangular factor of R^T Q = Z2 M^T.
-//   k_onesided  one CTA: one-sided Jacobi SVD of M (fp32 rotations, shared
-//               memory, every pair of a round at once), M W = U S.
+//   k_onesided_v, k_onesided
+//               one CTA: one-sided Jacobi SVD of M (fp32 rotations in shared
+//               memory, one 8-lane group per column pair so that every pair
+//               of a round runs at once), M W = U S; the _v form keeps the
+//               pair's columns in registers (l <= 144).
 //   k_ritz      sigma_j = |M w_j| / |w_j| in float64 (Rayleigh quotients).
 //   k_finish    the r largest sigma and the fp32 matrices that turn the bases
 //               into the split factors.
