@@ -401,8 +401,10 @@ def compress_member(w_doms, w_mems, omegas, r: int, power_iters: int = 2, worksp
     Returns the three (U, V, s)."""
     dev = w_doms[0].device
     main = torch.cuda.current_stream(dev)
-    streams = _MEMBER_STREAMS.setdefault(dev.index or 0,
-                                         [torch.cuda.Stream(device=dev) for _ in range(3)])
+    key = dev.index if dev.index is not None else torch.cuda.current_device()
+    if key not in _MEMBER_STREAMS:
+        _MEMBER_STREAMS[key] = [torch.cuda.Stream(device=dev) for _ in range(3)]
+    streams = _MEMBER_STREAMS[key]
     start = torch.cuda.Event()
     start.record(main)
     res = []
