@@ -419,4 +419,7 @@ def compress_member(w_doms, w_mems, omegas, r: int, power_iters: int = 2, worksp
         done = torch.cuda.Event()
         done.record(st)
         main.wait_event(done)
+        if out is None:
+            for t in res[-1]:  # allocated on the side stream, used on the caller's
+                t.record_stream(main)
     return res
